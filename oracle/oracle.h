@@ -1,0 +1,97 @@
+/*
+ * CPU oracle for barrier-free semaphore thresholds -- TEST INFRASTRUCTURE.
+ *
+ * Only the test suite, the smoke check and the benchmark's CPU-baseline leg
+ * may call this code.  It shares nothing with the GPU library: its own types,
+ * its own walk of the loop tree, its own arithmetic.
+ *
+ * Pair layout: dependency-major in batch dependency order; inside dependency
+ * d, one entry per dynamic instance of the consumer, in the order the
+ * consumer's loop iterates (its global iteration index g = 0, 1, ...).  No
+ * padding.
+ *
+ * Instance layout (issue/retire outputs): instruction-major in batch
+ * instruction order; instruction x has one entry per global iteration of its
+ * loop.
+ */
+#ifndef SYNC_ORACLE_H
+#define SYNC_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct {
+  int32_t n_programs;
+  const int32_t *prog_loop_ptr, *prog_instr_ptr, *prog_dep_ptr, *prog_n_engines;
+  const int32_t *loop_parent, *loop_pos;
+  const int32_t *instr_loop, *instr_pos, *instr_engine, *instr_latency;
+  const int32_t *dep_prod, *dep_cons, *dep_k;
+  const int64_t *trip_ptr;
+  const int32_t *trips;
+} orc_batch;
+
+enum { ORC_OK = 0, ORC_ERR_ARG = 1, ORC_ERR_MALFORMED = 2, ORC_ERR_NOT_ALLOCATABLE = 3,
+       ORC_ERR_OVERFLOW = 4, ORC_ERR_OOM = 6 };
+
+/* threshold modes: the producer-completion count c (Eq. 3) or the per-loop
+ * semaphore value T = N*c - (N-K), 0 when c = 0 (Eq. 5) */
+enum { ORC_COUNT = 0, ORC_PERLOOP = 1 };
+
+/* allocatable cases of Sec. 5.2 */
+enum { ORC_CASE_PS = 0, ORC_CASE_NEST_FWD = 1, ORC_CASE_NEST_BWD = 2, ORC_CASE_NONE = 3 };
+
+/* simulator variants and per-program status codes */
+enum { ORC_BARRIER_FREE = 0, ORC_BARRIER = 1 };
+enum { ORC_SIM_OK = 0, ORC_SIM_OVERFLOW = 4, ORC_SIM_DEADLOCK = 7 };
+
+typedef struct {
+  int32_t ii;                 /* issue interval of a datapath instruction      */
+  int32_t c_branch;           /* loop branch at each iteration start          */
+  int32_t c_regop;            /* one register operation                        */
+  int32_t c_wait_ops_count;   /* wait-value ops per dependency, count mode     */
+  int32_t c_wait_ops_perloop; /* wait-value ops per dependency, per-loop mode  */
+  int32_t c_barrier;          /* all-engine barrier handshake + reset          */
+} orc_sim_params;
+
+/* Sizes: pairs and instances in the layouts above. */
+int orc_sizes(const orc_batch *b, int64_t *n_pairs, int64_t *n_instances);
+
+/* Per dependency: innermost common loop S, producer parent loop P (program-
+ * local ids), allocatable case (ORC_CASE_*), N and K of the per-loop
+ * allocation.  Any output pointer may be NULL. */
+int orc_classify(const orc_batch *b, int32_t *S, int32_t *P, int32_t *kase, int32_t *N,
+                 int32_t *K);
+
+/* Eq. (1) by definition: for each consumer instance, the number of producer
+ * instances whose iteration vector restricted to the common loops is
+ * lexicographically <= the target t = v - delta (0 on underflow). */
+int orc_thresholds_bruteforce(const orc_batch *b, int mode, int32_t *out);
+/* The same definition evaluated by counting producer instances per iteration
+ * of the innermost common loop and prefix-summing. */
+int orc_thresholds(const orc_batch *b, int mode, int32_t *out);
+/* The paper's registers replayed literally per engine (Fig. 7/8): r-hat := 0
+ * at each loop statement, r++ and r-hat++ at each iteration start, and the
+ * masked wait value of Eq. (2)/(3)/(5) before each consumer.  Entries of
+ * non-allocatable dependencies are set to -1. */
+int orc_register_replay(const orc_batch *b, int mode, int32_t *out);
+
+/* Minimality check of a threshold array against Eq. (1): counts[0] = pairs
+ * whose threshold is below the minimum (unsafe), counts[1] = above it
+ * (over-synchronised); first_bad = first such pair index or -1. */
+int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[2],
+              int64_t *first_bad);
+
+/* Event-stepped semaphore machine (timing model stated in oracle.c).  `thr`
+ * is a threshold array in `mode`'s encoding; the machine waits on the
+ * per-producer semaphore (count) or the per-(loop, engine) semaphore
+ * (per-loop) until its value reaches the threshold.  issue/retire may be NULL. */
+int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim_params *prm,
+                 int variant, int32_t *makespan, uint64_t *checksum, int32_t *status,
+                 int32_t *issue, int32_t *retire);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,416 @@
+"""Pins of the CPU oracle to facts fixed outside it.
+
+Each test ties an oracle function to something other than the oracle itself:
+values the paper prints for a worked example (tests/golden), closed forms on
+single loops and nests, the paper's per-loop identity Eq. (4), exhaustive
+brute force, the paper's register mechanism (Thm. 1 consequence), a second
+statement of the timing model (tests/timing_model.py), and invariants of the
+timing model.  None of these needs a GPU.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from tests import golden_io
+from tests import timing_model
+
+COUNT, PERLOOP = oracle.COUNT, oracle.PERLOOP
+
+
+def pair_slices(batch):
+    """Per dependency, the slice of the pair layout it owns."""
+    cls = oracle.classify(batch)
+    out, off = [], 0
+    for d in range(batch.n_deps):
+        p = int(np.searchsorted(batch.prog_dep_ptr, d, side="right") - 1)
+        x = int(batch.dep_cons[d]) + int(batch.prog_instr_ptr[p])
+        l = int(batch.instr_loop[x]) + int(batch.prog_loop_ptr[p])
+        n = loop_totals(batch)[l]
+        out.append(slice(off, off + n))
+        off += n
+    return out
+
+
+def loop_totals(batch):
+    tot = np.zeros(batch.n_loops, dtype=np.int64)
+    for p in range(batch.n_programs):
+        l0, l1 = batch.prog_loop_ptr[p], batch.prog_loop_ptr[p + 1]
+        for l in range(l0, l1):
+            seg = batch.trips[batch.trip_ptr[l]:batch.trip_ptr[l + 1]]
+            tot[l] = int(seg.sum())
+    return tot
+
+
+# ------------------------------------------------------------ golden values
+
+@pytest.mark.parametrize("name", golden_io.all_names())
+def test_golden_worked_examples(name):
+    batch, expects = golden_io.load(name)
+    sl = pair_slices(batch)
+    for mode_name, d, want in expects:
+        mode = COUNT if mode_name == "count" else PERLOOP
+        for fn in (oracle.thresholds, oracle.thresholds_bruteforce, oracle.register_replay):
+            got = fn(batch, mode)[sl[d]]
+            assert got.tolist() == want, (name, fn.__name__, mode_name)
+
+
+def test_motivating_example_timeline():
+    """Sec. 2: with the barrier-free allocation, the third issue of I2 waits for
+    the first completion of I3 and nothing else waits; the pre- and post-loop
+    work of engine 0 runs back to back (Fig. 1b)."""
+    batch, _ = golden_io.load("motivating_example.txt")
+    thr = oracle.thresholds(batch, COUNT)
+    zero = oracle.sim_params(ii=1, c_branch=0, c_regop=0, c_wait_ops_count=0,
+                             c_wait_ops_perloop=0, c_barrier=0)
+    r = oracle.simulate(batch, thr, COUNT, oracle.BARRIER_FREE, zero, timeline=True)
+    assert r.status[0] == 0
+    # instance layout: I0, I1 (1 each), I2 (3), I3 (3), I4, I5
+    iss, ret = r.issue, r.retire
+    i2 = slice(2, 5)
+    i3 = slice(5, 8)
+    assert iss[i2][2] >= ret[i3][0]
+    assert iss[i2][2] == max(ret[i3][0], iss[i2][1] + 1)
+    # engine 0 (I0, I5) never waits: I5 issues one cycle after I0
+    assert iss[9] == iss[0] + 1
+
+
+# ------------------------------------------------------------ closed forms
+
+@pytest.mark.parametrize("trip,k", [(1, 0), (5, 0), (7, 1), (7, 2), (9, 5), (3, 4)])
+def test_closed_form_single_loop(trip, k):
+    """One loop under the top-level loop, producer and consumer directly in it:
+    the g-th consumer instance (1-based) waits for max(0, g - k) completions."""
+    b = workloads.ProgramBuilder(2)
+    L = b.loop(0, 0, [trip])
+    p = b.instr(L, 0, 0)
+    c = b.instr(L, 1, 1)
+    b.dep(p, c, k)
+    batch = b.batch()
+    want = [max(0, g - k) for g in range(1, trip + 1)]
+    assert oracle.thresholds(batch, COUNT).tolist() == want
+    assert oracle.thresholds_bruteforce(batch, COUNT).tolist() == want
+
+
+@pytest.mark.parametrize("outer,m", [(1, 1), (4, 3), (6, 1), (5, 7)])
+def test_closed_form_nested_forward(outer, m):
+    """Producer in an inner loop of constant trip m, consumer after it in the
+    outer loop (forward, offset 0): the wait in outer iteration g is m*g."""
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [outer])
+    B = b.loop(A, 0, [m] * outer)
+    p = b.instr(B, 0, 0)
+    c = b.instr(A, 1, 1)
+    b.dep(p, c, 0)
+    batch = b.batch()
+    want = [m * g for g in range(1, outer + 1)]
+    assert oracle.thresholds(batch, COUNT).tolist() == want
+    assert oracle.register_replay(batch, COUNT).tolist() == want
+
+
+def test_closed_form_top_level_offsets():
+    """Carried at the top-level loop (runs once): offset 0 counts every
+    earlier producer instance, any positive offset underflows."""
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [5])
+    p = b.instr(A, 0, 0)
+    c0 = b.instr(0, 1, 1)
+    c1 = b.instr(0, 2, 1)
+    b.dep(p, c0, 0)
+    b.dep(p, c1, 1)
+    batch = b.batch()
+    assert oracle.thresholds(batch, COUNT).tolist() == [5, 0]
+    assert oracle.thresholds_bruteforce(batch, COUNT).tolist() == [5, 0]
+
+
+@pytest.mark.parametrize("N", range(1, 9))
+def test_per_loop_identity_eq4(N):
+    """Eq. (4): after the K-th of N same-engine instructions of a loop body
+    retires in iteration r, the shared semaphore holds N*r - (N - K).  Checked
+    for every K and r: the per-loop threshold equals that value, and in the
+    oracle's semaphore machine the consumer issues exactly when that producer
+    instance retires (it neither waits for more nor for less)."""
+    R = 4
+    for K in range(1, N + 1):
+        b = workloads.ProgramBuilder(2)
+        A = b.loop(0, 0, [R])
+        xs = [b.instr(A, i, 0, latency=3 + 5 * i) for i in range(N)]
+        c = b.instr(A, N, 1)
+        b.dep(xs[K - 1], c, 0)
+        batch = b.batch()
+        thr = oracle.thresholds(batch, PERLOOP)
+        assert thr.tolist() == [N * r - (N - K) for r in range(1, R + 1)]
+        zero = oracle.sim_params(c_branch=0, c_regop=0, c_wait_ops_count=0,
+                                 c_wait_ops_perloop=0)
+        res = oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER_FREE, zero, timeline=True)
+        # instance layout: N producers x R, then the consumer x R
+        prod_ret = res.retire[(K - 1) * R:K * R]
+        cons_iss = res.issue[N * R:(N + 1) * R]
+        want, t = [], 0
+        for r in range(R):
+            want.append(max(t, int(prod_ret[r])))
+            t = want[-1] + 1
+        assert cons_iss.tolist() == want
+
+
+def test_per_loop_decoding_is_exact():
+    """T = 0 exactly when c = 0; otherwise T + N - K is a multiple of N and
+    (T + N - K) / N = c (the per-loop value decodes back to the count)."""
+    for seed in range(20):
+        batch = workloads.random_trees(seed, 10)
+        cls = oracle.classify(batch)
+        tc = oracle.thresholds(batch, COUNT)
+        tp = oracle.thresholds(batch, PERLOOP)
+        for d, sl in enumerate(pair_slices(batch)):
+            N, K = int(cls.N[d]), int(cls.K[d])
+            c, T = tc[sl].astype(np.int64), tp[sl].astype(np.int64)
+            assert ((T == 0) == (c == 0)).all()
+            nz = c > 0
+            assert ((T[nz] + N - K) % N == 0).all()
+            assert ((T[nz] + N - K) // N == c[nz]).all()
+
+
+# ---------------------------------------------- definitions agree (Thm. 1)
+
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def test_bruteforce_counting_and_registers_agree(mode):
+    """Eq. (1) by pairwise lexicographic comparison, Eq. (1) by counting, and
+    the paper's registers (Eq. 2, 3, 5) replayed per engine give the same
+    value on every pair of 1500 random allocatable programs."""
+    for seed in range(150):
+        batch = workloads.random_trees(seed, 10)
+        a = oracle.thresholds_bruteforce(batch, mode)
+        b = oracle.thresholds(batch, mode)
+        r = oracle.register_replay(batch, mode)
+        assert (a == b).all(), seed
+        assert (a == r).all(), seed
+
+
+def test_registers_differ_outside_allocatable_subset():
+    """Offsets outside the allocatable cases are classified as such, and the
+    register formula is then not the minimum (so the restriction matters)."""
+    seen_diff = 0
+    for seed in range(60):
+        batch = workloads.random_trees(seed, 10, workloads.tree_params(any_k=1, k_max=3))
+        cls = oracle.classify(batch)
+        a = oracle.thresholds_bruteforce(batch, COUNT)
+        r = oracle.register_replay(batch, COUNT)
+        for d, sl in enumerate(pair_slices(batch)):
+            if cls.kase[d] == oracle.CASE_NONE:
+                assert (r[sl] == -1).all()
+                continue
+            assert (a[sl] == r[sl]).all()
+        # a non-allocatable nested offset evaluated with the nested formula
+        seen_diff += int((cls.kase == oracle.CASE_NONE).sum())
+    assert seen_diff > 0
+
+
+def test_classification_cases():
+    """Sec. 5.2 cases on hand-built programs."""
+    def one(prod_where, cons_where, k, same_engine=False):
+        b = workloads.ProgramBuilder(2)
+        A = b.loop(0, 0, [3])
+        B = b.loop(A, 5, [2, 2, 2])
+        loops = {"A": A, "B": B}
+        p = b.instr(loops[prod_where[0]], prod_where[1], 0)
+        c = b.instr(loops[cons_where[0]], cons_where[1], 0 if same_engine else 1)
+        b.dep(p, c, k)
+        return int(oracle.classify(b.batch()).kase[0])
+    C = oracle
+    # producer nested in B, consumer after B in A: forward, offset 0 only
+    assert one(("B", 0), ("A", 9), 0) == C.CASE_NEST_FWD
+    assert one(("B", 0), ("A", 9), 1) == C.CASE_NONE
+    # consumer before B: backward, offset 1 only
+    assert one(("B", 0), ("A", 1), 1) == C.CASE_NEST_BWD
+    assert one(("B", 0), ("A", 1), 0) == C.CASE_NONE
+    assert one(("B", 0), ("A", 1), 2) == C.CASE_NONE
+    # producer in S: any offset; backward offset 0 only across engines
+    assert one(("A", 9), ("A", 1), 0) == C.CASE_PS
+    assert one(("A", 9), ("A", 1), 0, same_engine=True) == C.CASE_NONE
+    assert one(("A", 9), ("A", 1), 1, same_engine=True) == C.CASE_PS
+    assert one(("A", 1), ("B", 0), 0, same_engine=True) == C.CASE_PS
+    assert one(("A", 9), ("B", 0), 0, same_engine=True) == C.CASE_NONE
+
+
+# ---------------------------------------------------------------- checker
+
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def test_checker_counts_planted_errors(mode):
+    batch = workloads.generate("depth2", n_programs=8)
+    thr = oracle.thresholds(batch, mode)
+    assert oracle.check(batch, thr, mode) == (0, 0, -1)
+    rng = np.random.default_rng(7)
+    idx = np.sort(rng.choice(thr.size, size=40, replace=False))
+    bad = thr.copy()
+    up, down = idx[::2], idx[1::2]
+    bad[up] += 1
+    bad[down] -= 1
+    unsafe, over, first = oracle.check(batch, bad, mode)
+    assert (unsafe, over, first) == (down.size, up.size, int(idx[0]))
+
+
+# ------------------------------------------------------------ timing model
+
+ZERO = dict(c_branch=0, c_regop=0, c_wait_ops_count=0, c_wait_ops_perloop=0)
+
+
+@pytest.mark.parametrize("T,lat,cbar", [(1, 1, 32), (5, 3, 32), (16, 7, 5), (9, 1, 0)])
+def test_timing_closed_form_one_engine(T, lat, cbar):
+    """One engine, one loop of T iterations, one instruction, no control cost:
+    barrier-free makespan = T - 1 + lat (pipelined issue every cycle);
+    barrier scheme = T*(lat + c_barrier) + c_barrier (entry barrier plus a
+    drained barrier after every iteration)."""
+    b = workloads.ProgramBuilder(1)
+    L = b.loop(0, 0, [T])
+    b.instr(L, 0, 0, latency=lat)
+    batch = b.batch()
+    thr = np.zeros(0, dtype=np.int32)
+    prm = oracle.sim_params(c_barrier=cbar, **ZERO)
+    bf = oracle.simulate(batch, thr, COUNT, oracle.BARRIER_FREE, prm)
+    bb = oracle.simulate(batch, thr, COUNT, oracle.BARRIER, prm)
+    assert bf.makespan[0] == T - 1 + lat
+    assert bb.makespan[0] == T * (lat + cbar) + cbar
+
+
+def test_timing_straight_line_fig3():
+    """Fig. 3: I2 waits for I1 (s0 >= 2).  Engine 0 issues I0 at 0, I1 at 1;
+    I1 retires at max(1 + lat1, retire of I0); I2 issues then."""
+    batch, _ = golden_io.load("fig3_straight_line.txt")
+    batch.instr_latency[:] = [4, 2, 3, 1]
+    thr = oracle.thresholds(batch, PERLOOP)
+    prm = oracle.sim_params(**ZERO)
+    r = oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER_FREE, prm, timeline=True)
+    assert r.issue.tolist() == [0, 1, 4, 5]      # I1 retires at max(3, 4) = 4
+    assert r.retire.tolist() == [4, 4, 7, 7]
+    assert r.makespan[0] == 7
+
+
+def _random_batches(n=40, **kw):
+    for seed in range(n):
+        yield seed, workloads.random_trees(seed, 1, workloads.tree_params(**kw))
+
+
+@pytest.mark.parametrize("variant", [oracle.BARRIER_FREE, oracle.BARRIER])
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def test_timing_matches_recursive_statement(mode, variant):
+    """The event-stepped semaphore machine (waits on semaphore values, per
+    mode) and the recursive max-plus statement (waits on the c-th producer
+    retirement) give identical makespans, checksums and timelines."""
+    prm = oracle.sim_params(ii=2, c_branch=3, c_regop=1, c_barrier=7)
+    cwait = prm.c_wait_ops_count if mode == COUNT else prm.c_wait_ops_perloop
+    n = 0
+    for seed, batch in _random_batches(60):
+        thr = oracle.thresholds(batch, mode)
+        thr_c = oracle.thresholds(batch, COUNT)
+        r = oracle.simulate(batch, thr, mode, variant, prm, timeline=True)
+        assert r.status[0] == 0
+        ms, chk, tl = timing_model.simulate(batch, thr_c, prm, variant == oracle.BARRIER, cwait)
+        assert r.makespan[0] == ms, seed
+        assert int(r.checksum[0]) == chk, seed
+        off = 0
+        tot = loop_totals(batch)
+        for x in range(batch.n_instrs):
+            for g in range(int(tot[batch.instr_loop[x]])):
+                assert (r.issue[off + g], r.retire[off + g]) == tl[(x, g)]
+            off += int(tot[batch.instr_loop[x]])
+        n += 1
+    assert n == 60
+
+
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def test_timing_safety_and_exactness(mode):
+    """Safety: no consumer instance issues before the producer instance its
+    threshold names has retired.  Exactness: with zero wait-op cost it issues at
+    max(cursor, those retirements), so it never waits longer than required."""
+    prm = oracle.sim_params(**ZERO)
+    for seed, batch in _random_batches(40, body_hi=5, loops_hi=5):
+        thr_c = oracle.thresholds(batch, COUNT)
+        thr = oracle.thresholds(batch, mode)
+        r = oracle.simulate(batch, thr, mode, oracle.BARRIER_FREE, prm, timeline=True)
+        tot = loop_totals(batch)
+        inst_off = np.concatenate([[0], np.cumsum([tot[l] for l in batch.instr_loop])])
+        for d, sl in enumerate(pair_slices(batch)):
+            p, c = int(batch.dep_prod[d]), int(batch.dep_cons[d])
+            for g, cnt in enumerate(thr_c[sl]):
+                if cnt > 0:
+                    assert r.issue[inst_off[c] + g] >= r.retire[inst_off[p] + cnt - 1], seed
+
+
+def test_timing_barrier_free_never_slower_at_zero_cost():
+    """With zero control and wait-op costs the barrier scheme only adds
+    constraints to a monotone max-plus system: barrier-free <= barrier; on
+    straight-line programs (no loops) the two coincide."""
+    prm = oracle.sim_params(**ZERO)
+    for seed, batch in _random_batches(80):
+        thr = oracle.thresholds(batch, PERLOOP)
+        bf = oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER_FREE, prm)
+        bb = oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER, prm)
+        assert bf.makespan[0] <= bb.makespan[0], seed
+    for seed, batch in _random_batches(30, loops_lo=0, loops_hi=0, body_lo=1, body_hi=9):
+        thr = oracle.thresholds(batch, PERLOOP)
+        bf = oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER_FREE, prm)
+        bb = oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER, prm)
+        assert bf.makespan[0] == bb.makespan[0], seed
+
+
+def test_timing_deadlocks():
+    """A same-iteration cycle across two engines never issues (status 7 under
+    both schemes, Sec. 7.5); a backward offset-0 dependency across a nested
+    loop runs barrier-free but cannot pass the barrier in front of that loop."""
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [3])
+    x = b.instr(A, 0, 0)
+    y = b.instr(A, 1, 1)
+    b.dep(y, x, 0)
+    b.dep(x, y, 0)
+    batch = b.batch()
+    thr = oracle.thresholds(batch, PERLOOP)
+    for v in (oracle.BARRIER_FREE, oracle.BARRIER):
+        r = oracle.simulate(batch, thr, PERLOOP, v)
+        assert (r.status[0], r.makespan[0], int(r.checksum[0])) == (7, -1, 0)
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [3])
+    c = b.instr(A, 0, 1)
+    b.loop(A, 1, [2, 2, 2])
+    p = b.instr(A, 2, 0)
+    b.dep(p, c, 0)
+    batch = b.batch()
+    assert int(oracle.classify(batch).kase[0]) == oracle.CASE_PS
+    thr = oracle.thresholds(batch, PERLOOP)
+    assert oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER_FREE).status[0] == 0
+    assert oracle.simulate(batch, thr, PERLOOP, oracle.BARRIER).status[0] == 7
+
+
+def test_timing_overflow_status():
+    """The static time bound above INT32_MAX gives status 4."""
+    b = workloads.ProgramBuilder(1)
+    L = b.loop(0, 0, [3])
+    b.instr(L, 0, 0, latency=2 ** 30)
+    batch = b.batch()
+    thr = np.zeros(0, dtype=np.int32)
+    r = oracle.simulate(batch, thr, COUNT, oracle.BARRIER_FREE)
+    assert (r.status[0], r.makespan[0]) == (4, -1)
+    b = workloads.ProgramBuilder(1)
+    L = b.loop(0, 0, [1])
+    b.instr(L, 0, 0, latency=2 ** 30)
+    r = oracle.simulate(b.batch(), thr, COUNT, oracle.BARRIER_FREE)
+    # statement (c_regop) + iteration start (c_branch + 2*c_regop) before issue
+    assert r.status[0] == 0 and r.makespan[0] == 2 ** 30 + 4
+
+
+def test_generated_configs_are_allocatable_and_deadlock_free():
+    for name, n in (("small", None), ("depth2", 6), ("gemm", None), ("attention", 1),
+                    ("chain", 64), ("syncbound", 64)):
+        batch = workloads.generate(name, n_programs=n)
+        assert (oracle.classify(batch).kase != oracle.CASE_NONE).all(), name
+        thr = oracle.thresholds(batch, PERLOOP)
+        for v in (oracle.BARRIER_FREE, oracle.BARRIER):
+            assert (oracle.simulate(batch, thr, PERLOOP, v).status == 0).all(), name
+
+
+def test_program_ranges_are_independent():
+    full = workloads.generate("chain", n_programs=40)
+    part = workloads.generate("chain", n_programs=10, first_program=17)
+    sub = workloads.concat([full], programs=[(0, p) for p in range(17, 27)])
+    for k, v in sub.arrays().items():
+        assert np.array_equal(v, getattr(part, k)), k
