@@ -1,0 +1,409 @@
+#!/usr/bin/env python
+"""Benchmark of the barrier-free semaphore engine on one GB300 (or N, sharded).
+
+A step is one pass of the whole hot path over one batch: threshold kernel,
+minimality checker, barrier-free schedule simulation and barrier schedule
+simulation.  The metric is dynamic consumer instances -- (dependency,
+consumer instance) pairs -- per second, summed over all ranks.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 the script runs under torchrun, one rank per GPU; every rank
+processes its own programs (program ids rank*P .. rank*P+P-1, weak scaling)
+and no data crosses ranks.  Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "dynamic consumer instances/sec (threshold+check+sim), bit-exact; % HBM roofline"
+UNIT = "pairs/s"
+WORKLOADS = {
+    # name -> description for config.workload
+    "chain": "65536 random chain programs: 2-5 engines, up to 3 loops below the top level, "
+             "trips U[0,32] redrawn per parent iteration, 1-32 instructions per body, "
+             "dependency density 0.3",
+}
+KERNELS = ("thresholds", "check", "sim_barrier_free", "sim_barrier")
+CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--config", default="chain")
+    ap.add_argument("--programs", type=int, default=None, help="programs per rank")
+    ap.add_argument("--mode", choices=("perloop", "count"), default="perloop")
+    ap.add_argument("--cpu-sample", type=int, default=8192,
+                    help="programs of the workload the CPU oracle baseline runs")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d.get("sm_max_mhz", 2070.0)), "measured"
+    except Exception:
+        return 6800.0, 2070.0, "fallback"
+
+
+# --------------------------------------------------------------- clocks
+
+class ClockSampler:
+    def __init__(self, index: int):
+        self.proc = None
+        self.path = None
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={index}", f"--query-gpu={CLOCK_QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------- GPU side
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("k_thresholds.cu", "k_simulate.cu", "enc.h"):
+        with open(os.path.join(ROOT, "paper_2608_13757_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel sources."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            d = json.load(f)
+        e = d.get(workload, {}).get(kernel)
+        if e and e.get("source_hash") == kernel_hash():
+            return e["dram_bytes_per_launch"]
+    except Exception:
+        pass
+    return None
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import paper_2608_13757_gb300 as sg
+    import workloads
+
+    torch.cuda.set_device(local_rank)
+    mode = sg.THR_PERLOOP if args.mode == "perloop" else sg.THR_COUNT
+    P = args.programs or workloads.CONFIGS[args.config][1]
+    batch = workloads.generate(args.config, n_programs=P, first_program=rank * P)
+    t0 = time.perf_counter()
+    h = sg.sync_load_programs(batch, device=local_rank)
+    load_s = time.perf_counter() - t0
+    sz = h.sizes
+    dev = torch.device("cuda", local_rank)
+    thr = torch.empty(max(sz.n_pairs_padded, 4), dtype=torch.int32, device=dev)
+    counts = torch.empty(2, dtype=torch.int64, device=dev)
+    first_bad = torch.empty(1, dtype=torch.int64, device=dev)
+    prm = sg.SimParams()
+    mk = lambda: sg.SimOutputs(torch.empty(max(P, 1), dtype=torch.int32, device=dev),
+                               torch.empty(max(P, 1), dtype=torch.int64, device=dev),
+                               torch.empty(max(P, 1), dtype=torch.int32, device=dev))
+    bf, bb = mk(), mk()
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev: ev[0].record(stream)
+        sg.sync_eval_thresholds(h, mode, out=thr)
+        if ev: ev[1].record(stream)
+        sg.sync_check_minimal(h, mode, thr, counts, first_bad)
+        if ev: ev[2].record(stream)
+        sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE, out=bf)
+        if ev: ev[3].record(stream)
+        sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER, out=bb)
+        if ev: ev[4].record(stream)
+
+    for _ in range(max(args.warmup, 0)):
+        step()
+    torch.cuda.synchronize()
+    # correctness of the timed configuration: minimal thresholds, no deadlock
+    ok = counts.cpu().tolist() == [0, 0] and first_bad.item() == -1 and \
+        int(bf.status[:P].max().item()) == 0 and int(bb.status[:P].max().item()) == 0
+    dist_barrier(world)
+    clocks = ClockSampler(local_rank)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    start.record(stream)
+    for k in range(args.steps):
+        step(evs[k])
+    end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    dist_barrier(world)
+    total_ms = start.elapsed_time(end)
+    per_kernel = {name: 0.0 for name in KERNELS}
+    for e in evs:
+        for i, name in enumerate(KERNELS):
+            per_kernel[name] += e[i].elapsed_time(e[i + 1])
+    per_kernel = {k: v / args.steps for k, v in per_kernel.items()}
+    out = dict(ms=total_ms / args.steps, per_kernel=per_kernel, sizes=sz, clocks=clk, ok=ok,
+               load_s=load_s, P=P)
+    if not args.no_e2e:
+        out["e2e"] = run_e2e(args, sg, batch, mode, prm, dev, P)
+    h.close()
+    return out
+
+
+def run_e2e(args, sg, batch, mode, prm, dev, P):
+    """The same step through the public API from host arrays: load (host to
+    device copies), the four kernels, and the results read back to the host."""
+    import torch
+    steps = max(1, min(args.steps, 3))
+    times, h2d, d2h = [], 0, 0
+    for i in range(steps + 1):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        h = sg.sync_load_programs(batch, device=dev.index)
+        thr = sg.sync_eval_thresholds(h, mode)
+        counts, fb = sg.sync_check_minimal(h, mode, thr)
+        r1 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE)
+        r2 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER)
+        host = [t.cpu() for t in (counts, fb, r1.makespan, r1.checksum, r1.status,
+                                  r2.makespan, r2.checksum, r2.status)]
+        torch.cuda.synchronize()
+        t1 = time.perf_counter()
+        if i > 0:
+            times.append(t1 - t0)
+        h2d = h.sizes.h2d_bytes
+        d2h = sum(x.numel() * x.element_size() for x in host)
+        h.close()
+        del thr
+    return {"s": statistics.median(times), "h2d": int(h2d), "d2h": int(d2h)}
+
+
+def dist_barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------- CPU side
+
+def oracle_run(config, first, count, mode_name):
+    """The oracle on programs first..first+count-1: thresholds, check and both
+    simulations.  Returns (pairs, seconds of oracle work)."""
+    import oracle
+    import workloads
+    mode = oracle.PERLOOP if mode_name == "perloop" else oracle.COUNT
+    b = workloads.generate(config, n_programs=count, first_program=first)
+    t0 = time.perf_counter()
+    thr = oracle.thresholds(b, mode)
+    oracle.check(b, thr, mode)
+    oracle.simulate(b, thr, mode, oracle.BARRIER_FREE)
+    oracle.simulate(b, thr, mode, oracle.BARRIER)
+    return int(thr.size), time.perf_counter() - t0
+
+
+def cpu_baseline(config, sample, mode_name):
+    """Oracle on a bounded sample of the workload, spread over the host cores
+    (ctypes releases the GIL inside the oracle)."""
+    from concurrent.futures import ThreadPoolExecutor
+    import oracle
+    import workloads
+    oracle.build()
+    workloads.build()
+    cores = len(os.sched_getaffinity(0))
+    n_chunks = max(1, min(sample, cores * 4))
+    bounds = [(sample * i // n_chunks, sample * (i + 1) // n_chunks) for i in range(n_chunks)]
+    mode = oracle.PERLOOP if mode_name == "perloop" else oracle.COUNT
+    batches = [workloads.generate(config, n_programs=b - a, first_program=a) for a, b in bounds if b > a]
+
+    def work(b):
+        thr = oracle.thresholds(b, mode)
+        oracle.check(b, thr, mode)
+        oracle.simulate(b, thr, mode, oracle.BARRIER_FREE)
+        oracle.simulate(b, thr, mode, oracle.BARRIER)
+        return int(thr.size)
+
+    t0 = time.perf_counter()
+    with ThreadPoolExecutor(max_workers=cores) as ex:
+        pairs = sum(ex.map(work, batches))
+    dt = time.perf_counter() - t0
+    return {"value": pairs / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"programs 0..{sample - 1} of the {config} workload ({pairs} pairs), "
+                      f"thresholds + check + barrier-free and barrier simulation, {dt:.2f} s wall"}
+
+
+def run_reference(args, rank, world):
+    """The oracle as the reference arm: each step is the bounded sample."""
+    if rank != 0:
+        return
+    import oracle
+    import workloads
+    oracle.build()
+    workloads.build()
+    for _ in range(max(args.warmup, 0)):
+        cb = cpu_baseline(args.config, min(args.cpu_sample, 1024), args.mode)
+    vals = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        cb = cpu_baseline(args.config, args.cpu_sample, args.mode)
+        vals.append(cb["value"])
+    wall = time.perf_counter() - t0
+    v = statistics.median(vals)
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * wall / max(args.steps, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+            "data": "synthetic",
+            "config": {"workload": WORKLOADS.get(args.config, args.config),
+                       "sample_programs": args.cpu_sample, "threshold_mode": args.mode},
+            "cpu_baseline": {**cb, "value": v},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------- main
+
+def roofline(res, hbm_peak, peak_kind, sm_mhz, workload):
+    sz, pk = res["sizes"], res["per_kernel"]
+    # algorithmic bytes per launch: thresholds written / read once (padded
+    # array) plus the loop-structure arrays and tables, each once
+    alg = {"thresholds": 4 * sz.n_pairs_padded + sz.struct_bytes,
+           "check": 4 * sz.n_pairs_padded + sz.struct_bytes}
+    kernels = {}
+    for name in ("thresholds", "check"):
+        t = pk[name] / 1e3
+        ach = alg[name] / t / 1e9 if t > 0 else 0.0
+        kernels[name] = {"bound": "hbm", "ms": pk[name], "achieved": ach, "peak": hbm_peak,
+                         "unit": "GB/s", "frac": ach / hbm_peak, "alg_bytes": alg[name],
+                         "traffic": traffic_for(name, workload)}
+    # simulator: integer ops of the max-plus recurrence (per instance: wait
+    # cost, one max per dependency, issue, retire max, cursor, checksum terms)
+    # against the SM integer lanes: 152 SMs x 128 lanes x clock
+    lanes_peak = 152 * 128 * (sm_mhz or 2070.0) * 1e6 / 1e12
+    for name in ("sim_barrier_free", "sim_barrier"):
+        ops = 12 * sz.n_instances + 2 * sz.n_pairs
+        t = pk[name] / 1e3
+        ach = ops / t / 1e12 if t > 0 else 0.0
+        kernels[name] = {"bound": "alu", "ms": pk[name], "achieved": ach, "peak": lanes_peak,
+                         "unit": "Tops/s", "frac": ach / lanes_peak, "alg_ops": ops,
+                         "traffic": traffic_for(name, workload)}
+    dom = max(pk, key=pk.get)
+    d = dict(kernels[dom])
+    d["kernel"] = dom
+    d["peak_source"] = peak_kind if d["bound"] == "hbm" else "derived: 152 SMs x 128 int32 lanes x SM clock"
+    return d, kernels
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    import paper_2608_13757_gb300.build as b
+    b.build()
+    res = run_gpu(args, rank, world, local_rank)
+    ms = res["ms"]
+    pairs = res["sizes"].n_pairs
+    e2e_s = res["e2e"]["s"] if "e2e" in res else None
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([ms, e2e_s or 0.0, float(pairs)], dtype=torch.float64, device="cuda")
+        mx = t.clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        sm = t.clone()
+        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+        ms, e2e_s, total_pairs = mx[0].item(), mx[1].item() or None, sm[2].item()
+    else:
+        total_pairs = float(pairs)
+    if rank != 0:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
+    hbm_peak, sm_max, peak_kind = peaks()
+    clk = res["clocks"] or {}
+    roof, kernels = roofline(res, hbm_peak, peak_kind, clk.get("sm_mhz"), args.config)
+    line = {
+        "metric": METRIC, "value": total_pairs / (ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": {"workload": WORKLOADS.get(args.config, args.config), "programs_per_gpu": res["P"],
+                   "pairs_per_gpu": int(pairs), "instances_per_gpu": int(res["sizes"].n_instances),
+                   "threshold_mode": args.mode, "l2": "inputs larger than L2 (thresholds "
+                   f"{4 * res['sizes'].n_pairs_padded / 1e9:.2f} GB per pass)",
+                   "parallelism": f"programs sharded over {world} GPU(s)"},
+        "roofline": roof,
+        "kernels": kernels,
+        "gpu_launches": 4 * args.steps,
+        "results_minimal_and_deadlock_free": res["ok"],
+        "load_s": res["load_s"],
+        "clocks": clk or None,
+    }
+    if e2e_s:
+        line["e2e"] = {"value": total_pairs / e2e_s, "unit": UNIT,
+                       "h2d_bytes_per_step": res["e2e"]["h2d"], "d2h_bytes_per_step": res["e2e"]["d2h"]}
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.config, min(args.cpu_sample, res["P"]), args.mode)
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

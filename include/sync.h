@@ -1,0 +1,231 @@
+/*
+ * sync.h -- C ABI of the GB300 barrier-free semaphore engine.
+ *
+ * The engine evaluates, checks and simulates the semaphore thresholds of
+ * "A Barrier-Free Synchronization Algorithm for Multi-Engine AI Accelerators"
+ * (arxiv 2608.13757) over batches of structured multi-engine programs, on one
+ * GPU.  C99-compatible; no C++ types cross this boundary.
+ *
+ * Program model (Sec. 4.1): every construct is a loop (a conditional is a
+ * loop of trip 0 or 1; the program itself is a top-level loop that runs
+ * once).  Loops form a tree; a loop body is an ordered list of items --
+ * datapath instructions, each bound to one engine, and child loops -- ordered
+ * by a per-item position.  All engines walk this common tree with the same
+ * trip counts.  A dependency (producer p, consumer c, offset k) is carried at
+ * the innermost common loop S of p and c: consumer iteration v waits for the
+ * producer through target t = v - k on S (Sec. 5.1).
+ *
+ * Conventions shared by every call:
+ *  - Every call returns a sync_status; no C++ exception crosses the ABI.
+ *    On a non-OK status, sync_last_error() describes it (thread-local).
+ *  - Argument and structure errors are detected on the host before anything
+ *    is launched.  Kernels run asynchronously on the caller's CUDA stream
+ *    (`stream` is a cudaStream_t; NULL means the legacy default stream); a
+ *    launch failure returns SYNC_ERR_CUDA.
+ *  - "d_" arguments are caller-owned device buffers on the handle's device.
+ *    The handle owns the device-resident program encoding and its scratch.
+ *  - Results are integers and deterministic (sums and minima that do not
+ *    depend on execution order).
+ *
+ * Pair layout (thresholds): one segment per dependency, in batch dependency
+ * order; segment d starts at the offset reported by sync_pair_offsets and
+ * holds one int32 per dynamic instance of the consumer, in the order of the
+ * consumer loop's global iteration index g (0-based: iterations of a loop
+ * numbered in program order across all iterations of its ancestors), padded
+ * with zeros to a multiple of 4 entries.
+ *
+ * Instance layout (optional timelines): instruction-major in batch
+ * instruction order; instruction x owns one int32 per global iteration of its
+ * loop, starting at the sum of the instance counts of earlier instructions.
+ */
+#ifndef SYNC_H
+#define SYNC_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SYNC_OK = 0,
+  SYNC_ERR_ARG = 1,              /* NULL pointer, bad enum, size mismatch      */
+  SYNC_ERR_MALFORMED = 2,        /* the batch is not a valid program batch     */
+  SYNC_ERR_NOT_ALLOCATABLE = 3,  /* a dependency outside Sec. 5.2's cases      */
+  SYNC_ERR_OVERFLOW = 4,         /* a value stored as int32 would overflow     */
+  SYNC_ERR_CUDA = 5,             /* a CUDA runtime call or launch failed       */
+  SYNC_ERR_OOM = 6               /* host or device allocation failed           */
+} sync_status;
+
+/* Threshold encodings.  COUNT: the producer-completion count c of Eq. (3)
+ * (per-instruction semaphores).  PERLOOP: the value T = N*c - (N-K), or 0
+ * when c = 0, of the per-(loop, engine) semaphore of Eq. (5), where N is the
+ * number of instructions directly in the producer's loop body on the
+ * producer's engine and K the producer's 1-based rank among them. */
+typedef enum { SYNC_THR_COUNT = 0, SYNC_THR_PERLOOP = 1 } sync_thr_mode;
+
+/* Schedules simulated: barrier-free waits only, or the barrier-based scheme
+ * of Sec. 3.4 (an all-engine barrier at every loop statement and at the end
+ * of every iteration). */
+typedef enum { SYNC_SIM_BARRIER_FREE = 0, SYNC_SIM_BARRIER = 1 } sync_sim_variant;
+
+/* Per-program simulation status (d_status). */
+enum {
+  SYNC_PROG_OK = 0,
+  SYNC_PROG_OVERFLOW = 4,        /* static time bound exceeds INT32_MAX        */
+  SYNC_PROG_DEADLOCK = 7,        /* no engine can progress before the end      */
+  SYNC_PROG_ROUND_GUARD = 8      /* internal round limit hit (a defect)        */
+};
+
+/* Deepest supported nesting below the top-level loop. */
+#define SYNC_MAX_DEPTH 15
+
+/* A program batch in structure-of-arrays form.  Host pointers, borrowed for
+ * the duration of sync_load_programs only (the data is copied).  Ids inside
+ * a program are program-local (0-based).
+ *   prog_loop_ptr, prog_instr_ptr, prog_dep_ptr [n_programs+1]: CSR row
+ *     pointers into the loop / instruction / dependency arrays, starting at 0;
+ *   prog_n_engines [n_programs]: 1..32;
+ *   loop_parent, loop_pos [n_loops]: loop 0 of each program is the top-level
+ *     loop (parent -1); every other loop's parent has a smaller id; loop_pos
+ *     >= 0 is the loop's position among its parent's body items;
+ *   instr_loop, instr_pos, instr_engine, instr_latency [n_instrs]: enclosing
+ *     loop, position (>= 0, unique among the items of that loop body),
+ *     engine (0..n_engines-1), latency in cycles (>= 1);
+ *   dep_prod, dep_cons, dep_k [n_deps]: instruction ids and offset k >= 0;
+ *   trip_ptr [n_loops+1] (starting at 0) and trips [trip_ptr[n_loops]]: loop
+ *     l has one trip count (>= 0) per global iteration of its parent, in
+ *     trips[trip_ptr[l] .. trip_ptr[l+1]); the top-level loop has exactly one
+ *     entry, equal to 1. */
+typedef struct {
+  int32_t n_programs;
+  const int32_t *prog_loop_ptr, *prog_instr_ptr, *prog_dep_ptr;
+  const int32_t *prog_n_engines;
+  const int32_t *loop_parent, *loop_pos;
+  const int32_t *instr_loop, *instr_pos, *instr_engine, *instr_latency;
+  const int32_t *dep_prod, *dep_cons, *dep_k;
+  const int64_t *trip_ptr;
+  const int32_t *trips;
+} sync_batch_desc;
+
+typedef struct {
+  int64_t n_pairs;          /* (dependency, consumer instance) pairs          */
+  int64_t n_pairs_padded;   /* entries of a threshold array                   */
+  int64_t n_instances;      /* dynamic datapath instruction instances         */
+  int64_t n_loop_iters;     /* loop iterations, all loops of all programs     */
+  int32_t n_programs, n_loops, n_instrs, n_deps;
+  int64_t device_bytes;     /* device memory held by the handle               */
+  int64_t h2d_bytes;        /* bytes sync_load_programs copied host -> device */
+  int64_t struct_bytes;     /* encoding bytes the threshold and check kernels
+                               read besides the thresholds: parent indices and
+                               trip prefix sums of the loops on dependency
+                               paths (each array once), dependency tables     */
+} sync_sizes;
+
+/* Timing-model constants in cycles, all >= 0 (see sync_simulate). */
+typedef struct {
+  int32_t ii;                 /* issue interval of a datapath instruction     */
+  int32_t c_branch;           /* loop branch at each iteration start         */
+  int32_t c_regop;            /* one register operation                       */
+  int32_t c_wait_ops_count;   /* wait-value ops per dependency, COUNT (3, Table 1) */
+  int32_t c_wait_ops_perloop; /* wait-value ops per dependency, PERLOOP (5, Table 1) */
+  int32_t c_barrier;          /* all-engine barrier: handshake, reset, handshake */
+} sync_sim_params;
+
+typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
+
+/* Validates a batch, classifies every dependency into the allocatable cases
+ * of Sec. 5.2 (producer in S with any offset -- except offset 0 when the
+ * consumer precedes the producer in S's body on the same engine, which can
+ * never issue; producer nested below S and forward with offset 0; nested and
+ * backward with offset 1), computes N and K of the per-loop allocation
+ * (Sec. 5.5), and builds the device-resident encoding on `device`: loop
+ * table, per-loop trip prefix sums (rowptr) and expanded parent-iteration
+ * indices, dependency table, per-(loop, engine) instruction streams.
+ * Returns SYNC_ERR_MALFORMED for structural errors (listed with sync.h's
+ * batch description), SYNC_ERR_NOT_ALLOCATABLE for a dependency outside the
+ * cases above, SYNC_ERR_OVERFLOW when a loop's iteration total, a per-loop
+ * threshold N*total, a pair count or an instance count exceeds INT32_MAX
+ * (int64 totals are supported for pairs and instances across programs).
+ * On SYNC_OK, *out receives a handle to free with sync_free_programs.  The
+ * call synchronizes `stream` before returning. */
+sync_status sync_load_programs(const sync_batch_desc *desc, int device, void *stream,
+                               sync_programs **out);
+
+/* Sizes of a loaded batch (host struct). */
+sync_status sync_query(const sync_programs *h, sync_sizes *out);
+
+/* Host copies of the pair layout: offsets [n_deps + 1] int64 (segment starts;
+ * entry n_deps is n_pairs_padded) and, unless NULL, counts [n_deps] int32
+ * (consumer instances of each dependency, i.e. unpadded segment lengths). */
+sync_status sync_pair_offsets(const sync_programs *h, int64_t *offsets, int32_t *counts);
+
+/* Threshold kernel: for every pair (dependency d, consumer instance g) the
+ * wait value of Sec. 5.3, Eq. (2), with the trip register r-hat_S (position
+ * of the consumer's S-iteration in its trip, 1-based), the monotone registers
+ * (iteration counts including the current one, Sec. 5.1) and expr of
+ * Sec. 5.2 (r_S - k for a producer in S, r_P for a nested producer, r_P
+ * counted through the current / previous S-iteration when forward /
+ * backward), in `mode`'s encoding (Eq. 3 or Eq. 5).
+ * d_thr: [n_pairs_padded] int32, caller-owned device memory, fully written
+ * (padding entries 0). */
+sync_status sync_eval_thresholds(const sync_programs *h, sync_thr_mode mode, int32_t *d_thr,
+                                 void *stream);
+
+/* Minimality checker: recomputes the dependency-satisfaction condition of
+ * Eq. (1) for every pair (the target t = v - k on S, underflow when its
+ * S-component is <= 0, otherwise the producer instances lexicographically
+ * <= t) and compares the value stored in d_thr (read in `mode`'s encoding)
+ * with the required minimum: below it is unsafe (the consumer could issue
+ * before its producer, Sec. 4), above it over-synchronises.
+ * d_counts: [2] uint64 device -- unsafe, over-synchronised pair counts;
+ * d_first_bad: [1] int64 device -- smallest offending index into d_thr, or
+ * -1.  Both are overwritten (no accumulation across calls); padding entries
+ * of d_thr are ignored. */
+sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const int32_t *d_thr,
+                               unsigned long long *d_counts, long long *d_first_bad,
+                               void *stream);
+
+/* Schedule simulator.  Runs every program under a timing model of the
+ * paper's execution model: per-engine in-order issue and in-order
+ * retirement, waits `semaphore >= threshold` at issue, increments at
+ * retirement (Sec. 3.2-3.3, Appendix A.5), counters starting at 0
+ * (Appendix A.6).  Semaphores are per producer instruction (COUNT) or per
+ * (loop, engine) (PERLOOP); d_thr holds the thresholds in that encoding
+ * (normally the output of sync_eval_thresholds).  Costs in cycles, per
+ * engine cursor t:
+ *   loop statement: barrier-free t += c_regop (r-hat := 0); barrier: barrier
+ *   iteration start: barrier-free t += c_branch + 2*c_regop; barrier: t += c_branch
+ *   iteration end: barrier only: barrier
+ *   datapath x: barrier-free t += |D(x)| * c_wait_ops(mode);
+ *     issue = max(t, times at which the waited semaphores reached their
+ *     thresholds); retire = max(issue + latency, previous retire on the
+ *     engine); t = issue + ii
+ *   barrier: release = max over engines of max(t, last retire) + c_barrier;
+ *     every engine continues at release
+ *   the top-level loop costs nothing; makespan = max over engines of
+ *   max(t, last retire).
+ * Outputs per program (device, [n_programs]): d_makespan (int32, -1 unless
+ * status OK), d_checksum (uint64: sum over instances of
+ * issue*0x9E3779B97F4A7C15 ^ retire*0xC2B2AE3D27D4EB4F ^
+ * (n*0x165667B19E3779F9 + engine), n the 1-based ordinal in the engine's
+ * stream; 0 unless OK), d_status (SYNC_PROG_*).  d_issue / d_retire:
+ * [n_instances] int32 in instance layout, both NULL or both set (entries of
+ * programs whose status is not OK are unspecified).  The handle's history
+ * scratch is shared: calls on one handle must not overlap on the GPU. */
+sync_status sync_simulate(const sync_programs *h, sync_thr_mode mode, const int32_t *d_thr,
+                          const sync_sim_params *params, sync_sim_variant variant,
+                          int32_t *d_makespan, unsigned long long *d_checksum, int32_t *d_status,
+                          int32_t *d_issue, int32_t *d_retire, void *stream);
+
+/* Releases a handle (NULL is ignored).  Waits for the device to finish work
+ * that may still use the handle's memory. */
+void sync_free_programs(sync_programs *h);
+
+/* Message for the last non-OK status returned on this thread ("" if none). */
+const char *sync_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SYNC_H */

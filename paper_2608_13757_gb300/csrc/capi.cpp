@@ -1,0 +1,620 @@
+// C ABI of the engine: host loader (validation, dependency classification,
+// device encoding) and the launch wrappers.  Declarations and contracts are
+// in include/sync.h.
+#include <algorithm>
+#include <cstring>
+#include <memory>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "enc.h"
+
+using namespace syncgb;
+
+namespace {
+
+thread_local std::string g_err;
+
+struct Failure {
+  sync_status status;
+  std::string msg;
+};
+
+[[noreturn]] void raise(sync_status s, std::string msg) { throw Failure{s, std::move(msg)}; }
+
+void cuda_check(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return;
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    raise(SYNC_ERR_OOM, std::string(what) + ": " + cudaGetErrorString(e));
+  }
+  raise(SYNC_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+sync_status report(const Failure& f) {
+  g_err = f.msg;
+  return f.status;
+}
+
+constexpr int64_t kI32Max = 2147483647;
+
+int64_t pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
+
+}  // namespace
+
+struct sync_programs {
+  int device = 0;
+  int num_sms = 0;
+  sync_sizes sz{};
+  std::vector<int64_t> seg_host;
+  std::vector<int32_t> count_host;
+  std::vector<void*> blocks;
+  // threshold / checker encoding
+  LoopInfo* loop = nullptr;
+  int32_t* rowptr = nullptr;
+  int32_t* pidx = nullptr;
+  DepInfo* dep = nullptr;
+  int64_t* seg = nullptr;
+  int32_t* tile_first = nullptr;
+  int64_t* path = nullptr;
+  int64_t n_chunks = 0;
+  // simulator encoding
+  ProgInfo* prog = nullptr;
+  int32_t* order = nullptr;
+  int32_t* op_ptr = nullptr;
+  int32_t* ops = nullptr;
+  InstrSim* instr = nullptr;
+  ConsDep* cdep = nullptr;
+  int32_t* hist = nullptr;          // scratch: retire time of each semaphore increment
+  int32_t nsem_max[2] = {0, 0};
+  int32_t ne_max = 1;
+  int32_t depth_max = 0;
+
+  ~sync_programs() {
+    if (blocks.empty()) return;
+    int prev = 0;
+    cudaGetDevice(&prev);
+    cudaSetDevice(device);
+    cudaDeviceSynchronize();
+    for (void* p : blocks) cudaFree(p);
+    cudaSetDevice(prev);
+  }
+
+  template <class T>
+  T* upload(const std::vector<T>& v, cudaStream_t s, const char* what) {
+    const size_t bytes = std::max<size_t>(v.size(), 1) * sizeof(T);
+    void* p = nullptr;
+    cuda_check(cudaMalloc(&p, bytes), what);
+    blocks.push_back(p);
+    sz.device_bytes += (int64_t)bytes;
+    if (!v.empty()) cuda_check(cudaMemcpyAsync(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice, s), what);
+    sz.h2d_bytes += (int64_t)(v.size() * sizeof(T));
+    return static_cast<T*>(p);
+  }
+  template <class T>
+  T* alloc(int64_t n, const char* what) {
+    const size_t bytes = (size_t)std::max<int64_t>(n, 1) * sizeof(T);
+    void* p = nullptr;
+    cuda_check(cudaMalloc(&p, bytes), what);
+    blocks.push_back(p);
+    sz.device_bytes += (int64_t)bytes;
+    return static_cast<T*>(p);
+  }
+};
+
+namespace {
+
+struct Batch {
+  const sync_batch_desc& d;
+  int32_t P;
+  int64_t NL, NX, ND, NT;
+};
+
+void check_csr(const int32_t* ptr, int32_t P, const char* name) {
+  if (ptr[0] != 0) raise(SYNC_ERR_MALFORMED, std::string(name) + "[0] must be 0");
+  for (int32_t p = 0; p < P; ++p)
+    if (ptr[p + 1] < ptr[p]) raise(SYNC_ERR_MALFORMED, std::string(name) + " is not nondecreasing");
+}
+
+// Per-program scratch of the loader (reused across programs).
+struct ProgScratch {
+  std::vector<int32_t> depth, body_ptr, body, rank, nloop_eng;
+  std::vector<int64_t> total, keys;
+};
+
+std::string where(int32_t p, const char* what, int64_t i) {
+  return "program " + std::to_string(p) + ", " + what + " " + std::to_string(i);
+}
+
+}  // namespace
+
+static void build(const sync_batch_desc& d, int device, cudaStream_t stream, sync_programs& h) {
+  // ---------------------------------------------------------- shape checks
+  if (d.n_programs < 0) raise(SYNC_ERR_ARG, "n_programs < 0");
+  const int32_t P = d.n_programs;
+  if (!d.prog_loop_ptr || !d.prog_instr_ptr || !d.prog_dep_ptr || (P > 0 && !d.prog_n_engines))
+    raise(SYNC_ERR_ARG, "program CSR arrays must not be NULL");
+  check_csr(d.prog_loop_ptr, P, "prog_loop_ptr");
+  check_csr(d.prog_instr_ptr, P, "prog_instr_ptr");
+  check_csr(d.prog_dep_ptr, P, "prog_dep_ptr");
+  const int64_t NL = d.prog_loop_ptr[P], NX = d.prog_instr_ptr[P], ND = d.prog_dep_ptr[P];
+  if (NL > 0 && (!d.loop_parent || !d.loop_pos || !d.trip_ptr))
+    raise(SYNC_ERR_ARG, "loop arrays must not be NULL");
+  if (NX > 0 && (!d.instr_loop || !d.instr_pos || !d.instr_engine || !d.instr_latency))
+    raise(SYNC_ERR_ARG, "instruction arrays must not be NULL");
+  if (ND > 0 && (!d.dep_prod || !d.dep_cons || !d.dep_k))
+    raise(SYNC_ERR_ARG, "dependency arrays must not be NULL");
+  if (NL > 0) {
+    if (d.trip_ptr[0] != 0) raise(SYNC_ERR_MALFORMED, "trip_ptr[0] must be 0");
+    for (int64_t l = 0; l < NL; ++l)
+      if (d.trip_ptr[l + 1] < d.trip_ptr[l]) raise(SYNC_ERR_MALFORMED, "trip_ptr is not nondecreasing");
+    if (d.trip_ptr[NL] > 0 && !d.trips) raise(SYNC_ERR_ARG, "trips must not be NULL");
+  }
+
+  // ------------------------------------ per-program validation and tables
+  std::vector<LoopInfo> loop(NL);
+  std::vector<int32_t> rowptr_host;
+  std::vector<DepInfo> dep(ND);
+  std::vector<int64_t> path;
+  std::vector<ProgInfo> prog(P);
+  std::vector<int32_t> op_ptr, ops;
+  std::vector<InstrSim> instr(NX);
+  std::vector<ConsDep> cdep(ND);
+  std::vector<int64_t> seg(ND + 1, 0);
+  // per dependency, for the simulator's semaphore numbering
+  std::vector<int32_t> dep_N(ND), dep_K(ND);
+  std::vector<int64_t> hist_len(2, 0);
+  std::vector<uint8_t> reads_pidx(NL, 0), reads_rowptr(NL, 0);
+  int64_t n_pairs = 0, n_pairs_padded = 0, n_inst = 0, n_iters = 0, rowptr_len = 0;
+  ProgScratch S;
+
+  for (int32_t p = 0; p < P; ++p) {
+    const int32_t l0 = d.prog_loop_ptr[p], x0 = d.prog_instr_ptr[p], d0 = d.prog_dep_ptr[p];
+    const int32_t nl = d.prog_loop_ptr[p + 1] - l0, nx = d.prog_instr_ptr[p + 1] - x0,
+                  nd = d.prog_dep_ptr[p + 1] - d0;
+    const int32_t ne = d.prog_n_engines[p];
+    if (nl < 1) raise(SYNC_ERR_MALFORMED, where(p, "has no top-level loop", 0));
+    if (ne < 1 || ne > 32) raise(SYNC_ERR_MALFORMED, where(p, "n_engines", ne));
+    const int32_t* par = d.loop_parent + l0;
+    const int32_t* lpos = d.loop_pos + l0;
+    S.depth.assign(nl, 0);
+    S.total.assign(nl, 0);
+    if (par[0] != -1) raise(SYNC_ERR_MALFORMED, where(p, "loop 0 must have parent -1, loop", 0));
+    int32_t depth_max = 0;
+    for (int32_t l = 1; l < nl; ++l) {
+      if (par[l] < 0 || par[l] >= l) raise(SYNC_ERR_MALFORMED, where(p, "parent must precede the loop, loop", l));
+      if (lpos[l] < 0) raise(SYNC_ERR_MALFORMED, where(p, "negative position, loop", l));
+      S.depth[l] = S.depth[par[l]] + 1;
+      if (S.depth[l] > SYNC_MAX_DEPTH) raise(SYNC_ERR_MALFORMED, where(p, "nesting deeper than SYNC_MAX_DEPTH, loop", l));
+      depth_max = std::max(depth_max, S.depth[l]);
+    }
+    // trips and iteration totals
+    for (int32_t l = 0; l < nl; ++l) {
+      const int64_t gl = l0 + l;
+      const int64_t t0 = d.trip_ptr[gl], t1 = d.trip_ptr[gl + 1];
+      const int64_t want = l == 0 ? 1 : S.total[par[l]];
+      if (t1 - t0 != want) raise(SYNC_ERR_MALFORMED, where(p, "trip count array length != parent's iterations, loop", l));
+      int64_t tot = 0;
+      for (int64_t j = t0; j < t1; ++j) {
+        const int32_t t = d.trips[j];
+        if (t < 0) raise(SYNC_ERR_MALFORMED, where(p, "negative trip count, loop", l));
+        tot += t;
+      }
+      if (l == 0 && tot != 1) raise(SYNC_ERR_MALFORMED, where(p, "top-level loop must run once, loop", 0));
+      if (tot > kI32Max) raise(SYNC_ERR_OVERFLOW, where(p, "iterations exceed INT32_MAX, loop", l));
+      S.total[l] = tot;
+      LoopInfo& L = loop[gl];
+      L.parent = l == 0 ? -1 : l0 + par[l];
+      L.total = (int32_t)tot;
+      L.n_parent = (int32_t)want;
+      L.depth = S.depth[l];
+      L.rowptr_off = rowptr_len;
+      L.pidx_off = n_iters;
+      rowptr_len += want + 1;
+      n_iters += tot;
+    }
+    // instructions
+    for (int32_t x = 0; x < nx; ++x) {
+      const int64_t gx = x0 + x;
+      if (d.instr_loop[gx] < 0 || d.instr_loop[gx] >= nl) raise(SYNC_ERR_MALFORMED, where(p, "loop out of range, instruction", x));
+      if (d.instr_pos[gx] < 0) raise(SYNC_ERR_MALFORMED, where(p, "negative position, instruction", x));
+      if (d.instr_engine[gx] < 0 || d.instr_engine[gx] >= ne) raise(SYNC_ERR_MALFORMED, where(p, "engine out of range, instruction", x));
+      if (d.instr_latency[gx] < 1) raise(SYNC_ERR_MALFORMED, where(p, "latency < 1, instruction", x));
+    }
+    // bodies sorted by position; positions unique within a body
+    S.body_ptr.assign(nl + 1, 0);
+    for (int32_t x = 0; x < nx; ++x) S.body_ptr[d.instr_loop[x0 + x] + 1]++;
+    for (int32_t l = 1; l < nl; ++l) S.body_ptr[par[l] + 1]++;
+    for (int32_t l = 0; l < nl; ++l) S.body_ptr[l + 1] += S.body_ptr[l];
+    S.keys.resize(S.body_ptr[nl]);
+    {
+      std::vector<int32_t> fill(S.body_ptr.begin(), S.body_ptr.end() - 1);
+      for (int32_t x = 0; x < nx; ++x)
+        S.keys[fill[d.instr_loop[x0 + x]]++] = ((int64_t)d.instr_pos[x0 + x] << 32) | (uint32_t)x;
+      for (int32_t l = 1; l < nl; ++l)
+        S.keys[fill[par[l]]++] = ((int64_t)lpos[l] << 32) | (uint32_t)(-(l + 1));
+    }
+    S.body.resize(S.keys.size());
+    for (int32_t l = 0; l < nl; ++l) {
+      auto b = S.keys.begin() + S.body_ptr[l], e = S.keys.begin() + S.body_ptr[l + 1];
+      std::sort(b, e);
+      for (auto it = b; it != e; ++it) {
+        if (it != b && (*it >> 32) == (*(it - 1) >> 32))
+          raise(SYNC_ERR_MALFORMED, where(p, "two items share a position in the body of loop", l));
+        S.body[it - S.keys.begin()] = (int32_t)(uint32_t)(*it & 0xffffffffu);
+      }
+    }
+    // N (instructions directly in a loop body on one engine) and K (rank)
+    S.rank.assign(nx, 0);
+    S.nloop_eng.assign((size_t)nl * ne, 0);
+    for (int32_t l = 0; l < nl; ++l)
+      for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i) {
+        const int32_t it = S.body[i];
+        if (it >= 0) S.rank[it] = ++S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + it]];
+      }
+    // per-program aggregates and instruction table
+    ProgInfo& pi = prog[p];
+    std::memset(&pi, 0, sizeof pi);
+    pi.loop_base = l0;
+    pi.ne = ne;
+    pi.le_base = (int32_t)op_ptr.size();
+    pi.depth = depth_max;
+    __int128 agg = 0;
+    for (int32_t x = 0; x < nx; ++x) {
+      const int64_t tot = S.total[d.instr_loop[x0 + x]];
+      agg += (__int128)tot * d.instr_latency[x0 + x];
+      InstrSim& X = instr[x0 + x];
+      std::memset(&X, 0, sizeof X);
+      X.lat = d.instr_latency[x0 + x];
+      X.inst_off = n_inst;
+      X.own_sem[0] = X.own_sem[1] = -1;
+      n_inst += tot;
+      pi.n_inst += tot;
+    }
+    pi.agg_lat = agg > (__int128)INT64_MAX ? INT64_MAX : (int64_t)agg;
+    for (int32_t l = 1; l < nl; ++l) { pi.n_stmt += S.total[par[l]]; pi.n_iter += S.total[l]; }
+    // per-(loop, engine) instruction streams: own instructions and child loops
+    for (int32_t l = 0; l < nl; ++l)
+      for (int32_t e = 0; e < ne; ++e) {
+        op_ptr.push_back((int32_t)ops.size());
+        for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i) {
+          const int32_t it = S.body[i];
+          if (it < 0) ops.push_back(-(l0 + (-it - 1)) - 1);
+          else if (d.instr_engine[x0 + it] == e) ops.push_back(x0 + it);
+        }
+      }
+    // dependencies: innermost common loop S, cases of Sec. 5.2, N and K
+    std::vector<int32_t> by_cons(nd);
+    for (int32_t k = 0; k < nd; ++k) by_cons[k] = k;
+    for (int32_t k = 0; k < nd; ++k) {
+      const int64_t gd = d0 + k;
+      const int32_t px = d.dep_prod[gd], cx = d.dep_cons[gd], off = d.dep_k[gd];
+      if (px < 0 || px >= nx || cx < 0 || cx >= nx) raise(SYNC_ERR_MALFORMED, where(p, "instruction out of range, dependency", k));
+      if (off < 0) raise(SYNC_ERR_MALFORMED, where(p, "negative offset, dependency", k));
+      const int32_t Pl = d.instr_loop[x0 + px], Cl = d.instr_loop[x0 + cx];
+      // climb to the innermost common loop; remember the child of it on each side
+      int32_t a = Pl, b = Cl, ca = -1, cb = -1;
+      while (S.depth[a] > S.depth[b]) { ca = a; a = par[a]; }
+      while (S.depth[b] > S.depth[a]) { cb = b; b = par[b]; }
+      while (a != b) { ca = a; a = par[a]; cb = b; b = par[b]; }
+      const int32_t Sl = a;
+      const int32_t ppos = ca < 0 ? d.instr_pos[x0 + px] : lpos[ca];
+      const int32_t cpos = cb < 0 ? d.instr_pos[x0 + cx] : lpos[cb];
+      const bool forward = cpos > ppos;
+      const bool same_engine = d.instr_engine[x0 + px] == d.instr_engine[x0 + cx];
+      int32_t kase;
+      if (ca < 0) {
+        // producer directly in S: any offset; offset 0 with the consumer not
+        // after the producer on the same engine can never issue (in-order)
+        if (off == 0 && !forward && same_engine)
+          raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "offset 0 to a later producer on the same engine, dependency", k));
+        kase = CASE_PS;
+      } else if (forward) {
+        if (off != 0) raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested forward producer needs offset 0, dependency", k));
+        kase = CASE_NEST_FWD;
+      } else {
+        if (off != 1) raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested backward producer needs offset 1, dependency", k));
+        kase = CASE_NEST_BWD;
+      }
+      const int32_t N = S.nloop_eng[(size_t)Pl * ne + d.instr_engine[x0 + px]];
+      const int32_t K = S.rank[px];
+      if ((int64_t)N * S.total[Pl] > kI32Max)
+        raise(SYNC_ERR_OVERFLOW, where(p, "per-loop semaphore value N*iterations exceeds INT32_MAX, dependency", k));
+      DepInfo& D = dep[gd];
+      std::memset(&D, 0, sizeof D);
+      D.total = (int32_t)S.total[Cl];
+      D.up = S.depth[Cl] - S.depth[Sl];
+      D.clen = S.depth[Pl] - S.depth[Sl];
+      D.kase = kase;
+      D.k = off; D.N = N; D.K = K;
+      D.path = (int64_t)path.size();
+      for (int32_t l = Cl; l != Sl; l = par[l]) { path.push_back(loop[l0 + l].pidx_off); reads_pidx[l0 + l] = 1; }
+      reads_pidx[l0 + Sl] = 1;
+      reads_rowptr[l0 + Sl] = 1;
+      for (int32_t l = Pl; l != Sl; l = par[l]) reads_rowptr[l0 + l] = 1;
+      path.push_back(loop[l0 + Sl].pidx_off);
+      path.push_back(loop[l0 + Sl].rowptr_off);
+      {
+        const size_t at = path.size();
+        for (int32_t l = Pl; l != Sl; l = par[l]) path.push_back(loop[l0 + l].rowptr_off);
+        std::reverse(path.begin() + at, path.end());
+      }
+      D.seg_off = n_pairs_padded;
+      seg[gd] = n_pairs_padded;
+      n_pairs += S.total[Cl];
+      n_pairs_padded += pad4(S.total[Cl]);
+      pi.n_pairs += S.total[Cl];
+      dep_N[gd] = N;
+      dep_K[gd] = K;
+    }
+    // semaphores that some dependency waits on, per mode, with their history
+    // slots: mode 0 = one per producer instruction (one increment per
+    // iteration); mode 1 = one per (loop, engine) (N increments per iteration)
+    std::vector<int32_t> sem_of(std::max(nx, nl * ne), -1);
+    for (int m = 0; m < 2; ++m) {
+      std::fill(sem_of.begin(), sem_of.end(), -1);
+      std::vector<int64_t> sem_hist;
+      for (int32_t k = 0; k < nd; ++k) {
+        const int64_t gd = d0 + k;
+        const int32_t px = d.dep_prod[gd];
+        const int32_t Pl = d.instr_loop[x0 + px];
+        const int32_t key = m == 0 ? px : Pl * ne + d.instr_engine[x0 + px];
+        if (sem_of[key] < 0) {
+          sem_of[key] = (int32_t)sem_hist.size();
+          sem_hist.push_back(hist_len[m]);
+          hist_len[m] += (m == 0 ? 1 : dep_N[gd]) * S.total[Pl];
+        }
+      }
+      pi.nsem[m] = (int32_t)sem_hist.size();
+      for (int32_t x = 0; x < nx; ++x) {
+        const int32_t l = d.instr_loop[x0 + x];
+        const int32_t key = m == 0 ? x : l * ne + d.instr_engine[x0 + x];
+        const int32_t s = sem_of[key];
+        InstrSim& X = instr[x0 + x];
+        X.own_sem[m] = s;
+        if (s < 0) continue;
+        X.hstride[m] = m == 0 ? 1 : S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]];
+        X.hbase[m] = sem_hist[s] + (m == 0 ? 0 : S.rank[x] - 1);
+      }
+      for (int32_t k = 0; k < nd; ++k) {
+        const int64_t gd = d0 + k;
+        const int32_t px = d.dep_prod[gd];
+        const int32_t key = m == 0 ? px : d.instr_loop[x0 + px] * ne + d.instr_engine[x0 + px];
+        cdep[gd].tsem[m] = sem_of[key];
+        cdep[gd].thist[m] = sem_hist[sem_of[key]];
+      }
+    }
+    // consumer-grouped dependency list (stable by dependency id)
+    std::stable_sort(by_cons.begin(), by_cons.end(), [&](int32_t u, int32_t v) {
+      return d.dep_cons[d0 + u] < d.dep_cons[d0 + v];
+    });
+    {
+      std::vector<ConsDep> grouped(nd);
+      for (int32_t i = 0; i < nd; ++i) {
+        grouped[i] = cdep[d0 + by_cons[i]];
+        grouped[i].seg_off = seg[d0 + by_cons[i]];
+      }
+      for (int32_t i = 0; i < nd; ++i) cdep[d0 + i] = grouped[i];
+      for (int32_t x = 0; x < nx; ++x) instr[x0 + x].dep_begin = d0;
+      for (int32_t i = nd - 1; i >= 0; --i) instr[x0 + d.dep_cons[d0 + by_cons[i]]].dep_begin = d0 + i;
+      for (int32_t i = 0; i < nd; ++i) instr[x0 + d.dep_cons[d0 + by_cons[i]]].ndeps++;
+    }
+    h.nsem_max[0] = std::max(h.nsem_max[0], pi.nsem[0]);
+    h.nsem_max[1] = std::max(h.nsem_max[1], pi.nsem[1]);
+    h.ne_max = std::max(h.ne_max, ne);
+    h.depth_max = std::max(h.depth_max, depth_max);
+  }
+  if ((int64_t)ops.size() > kI32Max) raise(SYNC_ERR_OVERFLOW, "instruction streams exceed INT32_MAX entries");
+  op_ptr.push_back((int32_t)ops.size());
+  seg[ND] = n_pairs_padded;
+
+  // trip prefix sums (rowptr) per loop: [0, t0, t0+t1, ...]
+  rowptr_host.resize(rowptr_len);
+  for (int64_t l = 0; l < NL; ++l) {
+    int32_t* rp = rowptr_host.data() + loop[l].rowptr_off;
+    const int64_t t0 = d.trip_ptr[l];
+    rp[0] = 0;
+    for (int32_t j = 0; j < loop[l].n_parent; ++j) rp[j + 1] = rp[j] + d.trips[t0 + j];
+  }
+  // tile tables
+  const int64_t n_tiles = (n_pairs_padded + kTilePairs - 1) / kTilePairs;
+  std::vector<int32_t> tile_first(n_tiles + 1, ND > 0 ? (int32_t)(ND - 1) : 0);
+  {
+    int64_t di = 0;
+    for (int64_t t = 0; t < n_tiles; ++t) {
+      const int64_t q = t * kTilePairs;
+      while (di + 1 < ND && seg[di + 1] <= q) ++di;
+      tile_first[t] = (int32_t)di;
+    }
+  }
+  const int64_t n_itiles = (n_iters + kTilePairs - 1) / kTilePairs;
+  std::vector<int32_t> tile_loop(n_itiles + 1, NL > 0 ? (int32_t)(NL - 1) : 0);
+  {
+    int64_t li = 0;
+    for (int64_t t = 0; t < n_itiles; ++t) {
+      const int64_t q = t * kTilePairs;
+      while (li + 1 < NL && loop[li + 1].pidx_off <= q) ++li;
+      tile_loop[t] = (int32_t)li;
+    }
+  }
+  // programs in descending order of simulated work
+  std::vector<int32_t> order(P);
+  for (int32_t p = 0; p < P; ++p) order[p] = p;
+  std::stable_sort(order.begin(), order.end(), [&](int32_t u, int32_t v) {
+    auto w = [&](int32_t q) { return prog[q].n_inst + prog[q].n_pairs + (prog[q].n_stmt + prog[q].n_iter) * prog[q].ne; };
+    return w(u) > w(v);
+  });
+
+  h.sz.n_pairs = n_pairs;
+  h.sz.n_pairs_padded = n_pairs_padded;
+  h.sz.n_instances = n_inst;
+  h.sz.n_loop_iters = n_iters;
+  h.sz.n_programs = P;
+  h.sz.n_loops = (int32_t)NL;
+  h.sz.n_instrs = (int32_t)NX;
+  h.sz.n_deps = (int32_t)ND;
+  {
+    int64_t sb = (int64_t)ND * (int64_t)sizeof(DepInfo) + 8 * (ND + 1) + 8 * (int64_t)path.size() +
+                 4 * (int64_t)tile_first.size();
+    for (int64_t l = 0; l < NL; ++l) {
+      if (reads_pidx[l]) sb += 4 * (int64_t)loop[l].total;
+      if (reads_rowptr[l]) sb += 4 * ((int64_t)loop[l].n_parent + 1);
+    }
+    h.sz.struct_bytes = sb;
+  }
+  h.seg_host = seg;
+  h.count_host.resize(ND);
+  for (int64_t i = 0; i < ND; ++i) h.count_host[i] = dep[i].total;
+  h.n_chunks = n_pairs_padded / kChunk;
+
+  // ---------------------------------------------------------------- device
+  cuda_check(cudaSetDevice(device), "cudaSetDevice");
+  h.device = device;
+  cuda_check(cudaDeviceGetAttribute(&h.num_sms, cudaDevAttrMultiProcessorCount, device), "device attributes");
+  h.loop = h.upload(loop, stream, "loop table");
+  h.rowptr = h.upload(rowptr_host, stream, "rowptr");
+  h.pidx = h.alloc<int32_t>(n_iters, "parent indices");
+  h.dep = h.upload(dep, stream, "dependency table");
+  h.seg = h.upload(seg, stream, "segment offsets");
+  h.tile_first = h.upload(tile_first, stream, "tile table");
+  h.path = h.upload(path, stream, "path pool");
+  int32_t* d_tile_loop = h.upload(tile_loop, stream, "loop tile table");
+  h.prog = h.upload(prog, stream, "program table");
+  h.order = h.upload(order, stream, "program order");
+  h.op_ptr = h.upload(op_ptr, stream, "stream offsets");
+  h.ops = h.upload(ops, stream, "streams");
+  h.instr = h.upload(instr, stream, "instruction table");
+  h.cdep = h.upload(cdep, stream, "consumer dependency table");
+  h.hist = h.alloc<int32_t>(std::max(hist_len[0], hist_len[1]), "semaphore history");
+  cuda_check(launch_expand(h.loop, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
+  cuda_check(cudaStreamSynchronize(stream), "load");
+}
+
+extern "C" {
+
+sync_status sync_load_programs(const sync_batch_desc* desc, int device, void* stream,
+                               sync_programs** out) {
+  try {
+    if (!desc || !out) raise(SYNC_ERR_ARG, "desc and out must not be NULL");
+    *out = nullptr;
+    std::unique_ptr<sync_programs> h(new sync_programs());
+    build(*desc, device, static_cast<cudaStream_t>(stream), *h);
+    *out = h.release();
+    g_err.clear();
+    return SYNC_OK;
+  } catch (const Failure& f) {
+    return report(f);
+  } catch (const std::bad_alloc&) {
+    return report(Failure{SYNC_ERR_OOM, "host allocation failed"});
+  } catch (...) {
+    return report(Failure{SYNC_ERR_ARG, "unexpected error"});
+  }
+}
+
+sync_status sync_query(const sync_programs* h, sync_sizes* out) {
+  if (!h || !out) return report(Failure{SYNC_ERR_ARG, "handle and out must not be NULL"});
+  *out = h->sz;
+  return SYNC_OK;
+}
+
+sync_status sync_pair_offsets(const sync_programs* h, int64_t* offsets, int32_t* counts) {
+  if (!h || !offsets) return report(Failure{SYNC_ERR_ARG, "handle and offsets must not be NULL"});
+  std::memcpy(offsets, h->seg_host.data(), h->seg_host.size() * sizeof(int64_t));
+  if (counts) std::memcpy(counts, h->count_host.data(), h->count_host.size() * sizeof(int32_t));
+  return SYNC_OK;
+}
+
+static ThrArgs thr_args(const sync_programs* h, sync_thr_mode mode) {
+  ThrArgs a;
+  a.dep = h->dep; a.seg = h->seg; a.tile_first = h->tile_first; a.path = h->path;
+  a.rowptr = h->rowptr; a.pidx = h->pidx; a.n_chunks = h->n_chunks; a.mode = mode;
+  return a;
+}
+
+static void check_mode(sync_thr_mode mode) {
+  if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP) raise(SYNC_ERR_ARG, "unknown threshold mode");
+}
+
+sync_status sync_eval_thresholds(const sync_programs* h, sync_thr_mode mode, int32_t* d_thr,
+                                 void* stream) {
+  try {
+    if (!h) raise(SYNC_ERR_ARG, "handle must not be NULL");
+    check_mode(mode);
+    if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
+    if (reinterpret_cast<uintptr_t>(d_thr) % 16) raise(SYNC_ERR_ARG, "d_thr must be 16-byte aligned");
+    cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
+    cuda_check(launch_thresholds(thr_args(h, mode), d_thr, h->num_sms, static_cast<cudaStream_t>(stream)),
+               "threshold kernel");
+    return SYNC_OK;
+  } catch (const Failure& f) {
+    return report(f);
+  }
+}
+
+sync_status sync_check_minimal(const sync_programs* h, sync_thr_mode mode, const int32_t* d_thr,
+                               unsigned long long* d_counts, long long* d_first_bad, void* stream) {
+  try {
+    if (!h || !d_counts || !d_first_bad) raise(SYNC_ERR_ARG, "handle and outputs must not be NULL");
+    check_mode(mode);
+    if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
+    if (reinterpret_cast<uintptr_t>(d_thr) % 16) raise(SYNC_ERR_ARG, "d_thr must be 16-byte aligned");
+    cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
+    CheckArgs a;
+    a.t = thr_args(h, mode);
+    a.thr = d_thr;
+    a.counts = d_counts;
+    a.first_bad = reinterpret_cast<unsigned long long*>(d_first_bad);
+    cuda_check(launch_check(a, h->num_sms, static_cast<cudaStream_t>(stream)), "checker kernel");
+    return SYNC_OK;
+  } catch (const Failure& f) {
+    return report(f);
+  }
+}
+
+sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int32_t* d_thr,
+                          const sync_sim_params* params, sync_sim_variant variant,
+                          int32_t* d_makespan, unsigned long long* d_checksum, int32_t* d_status,
+                          int32_t* d_issue, int32_t* d_retire, void* stream) {
+  try {
+    if (!h || !params) raise(SYNC_ERR_ARG, "handle and params must not be NULL");
+    check_mode(mode);
+    if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER) raise(SYNC_ERR_ARG, "unknown variant");
+    if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
+      raise(SYNC_ERR_ARG, "per-program outputs must not be NULL");
+    if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
+    if ((d_issue == nullptr) != (d_retire == nullptr)) raise(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");
+    const sync_sim_params& q = *params;
+    if (q.ii < 0 || q.c_branch < 0 || q.c_regop < 0 || q.c_wait_ops_count < 0 ||
+        q.c_wait_ops_perloop < 0 || q.c_barrier < 0)
+      raise(SYNC_ERR_ARG, "timing constants must be >= 0");
+    cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
+    SimArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.prog = h->prog; a.order = h->order; a.loop = h->loop; a.rowptr = h->rowptr;
+    a.op_ptr = h->op_ptr; a.ops = h->ops; a.instr = h->instr; a.cdep = h->cdep;
+    a.thr = d_thr; a.hist = h->hist;
+    a.makespan = d_makespan; a.checksum = d_checksum; a.status = d_status;
+    a.issue = d_issue; a.retire = d_retire;
+    a.prm = q;
+    a.n_programs = h->sz.n_programs;
+    a.mode = mode;
+    a.sem_ints = (h->nsem_max[mode] + 3) & ~3;
+    a.frame_depth = std::max(1, h->depth_max);
+    a.ne_max = h->ne_max;
+    const size_t per_warp = simulate_smem_per_warp(a.sem_ints, a.frame_depth, a.ne_max);
+    if (per_warp * 4 > 200 * 1024)
+      raise(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
+    cuda_check(launch_simulate(a, variant == SYNC_SIM_BARRIER, h->num_sms, static_cast<cudaStream_t>(stream)),
+               "simulator kernel");
+    return SYNC_OK;
+  } catch (const Failure& f) {
+    return report(f);
+  }
+}
+
+void sync_free_programs(sync_programs* h) { delete h; }
+
+const char* sync_last_error(void) { return g_err.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,265 @@
+"""GPU path vs the CPU oracle, through the C ABI.  All results are integers and
+must match bit for bit: thresholds in both encodings, checker counts and first
+offending index, simulated makespans, checksums, statuses and timelines."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from tests import golden_io
+
+pytestmark = pytest.mark.gpu
+
+COUNT, PERLOOP = oracle.COUNT, oracle.PERLOOP
+MODES = (COUNT, PERLOOP)
+VARIANTS = (oracle.BARRIER_FREE, oracle.BARRIER)
+
+
+@pytest.fixture(scope="module")
+def sg():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2608_13757_gb300 as m
+    return m
+
+
+def gpu_thresholds(sg, h, mode):
+    thr = sg.sync_eval_thresholds(h, mode)
+    host = thr.cpu().numpy()
+    n = h.sizes.n_pairs_padded
+    pad = np.ones(n, dtype=bool)
+    idx = h.unpadded_index()
+    pad[idx] = False
+    assert (host[:n][pad] == 0).all(), "padding entries must be 0"
+    return thr, host[idx]
+
+
+def sim_params(oracle_prm):
+    import paper_2608_13757_gb300 as m
+    return m.SimParams(*[getattr(oracle_prm, f) for f, _ in oracle_prm._fields_])
+
+
+def compare_all(sg, batch, params=None, timeline=False, modes=MODES):
+    prm = params if params is not None else oracle.sim_params()
+    h = sg.sync_load_programs(batch)
+    npairs, ninst = oracle.sizes(batch)
+    assert h.sizes.n_pairs == npairs and h.sizes.n_instances == ninst
+    for mode in modes:
+        thr, got = gpu_thresholds(sg, h, mode)
+        want = oracle.thresholds(batch, mode)
+        assert np.array_equal(got, want), f"thresholds differ (mode {mode})"
+        counts, fb = sg.sync_check_minimal(h, mode, thr)
+        assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
+        for v in VARIANTS:
+            res = sg.sync_simulate(h, mode, thr, sim_params(prm), v, timeline=timeline)
+            ref = oracle.simulate(batch, want, mode, v, prm, timeline=timeline)
+            P = batch.n_programs
+            st = res.status.cpu().numpy()[:P]
+            assert np.array_equal(st, ref.status), (mode, v)
+            assert np.array_equal(res.makespan.cpu().numpy()[:P], ref.makespan), (mode, v)
+            ck = res.checksum.cpu().numpy()[:P].view(np.uint64)
+            assert np.array_equal(ck, ref.checksum), (mode, v)
+            if timeline:
+                ok = np.repeat(ref.status == 0, _instances_per_program(batch))
+                assert np.array_equal(res.issue.cpu().numpy()[:ninst][ok], ref.issue[ok])
+                assert np.array_equal(res.retire.cpu().numpy()[:ninst][ok], ref.retire[ok])
+    return h
+
+
+def _instances_per_program(batch):
+    out = []
+    for p in range(batch.n_programs):
+        out.append(oracle.sizes(batch.program(p))[1])
+    return np.array(out, dtype=np.int64)
+
+
+# ------------------------------------------------------------------ configs
+
+@pytest.mark.parametrize("name,n", [("small", None), ("depth2", 48), ("gemm", None),
+                                    ("attention", 2), ("chain", 400), ("syncbound", 400)])
+def test_configs_bit_exact(sg, name, n):
+    batch = workloads.generate(name, n_programs=n)
+    compare_all(sg, batch, timeline=name in ("small", "depth2"))
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_trees_bit_exact(sg, seed):
+    batch = workloads.random_trees(1000 + seed, 150, workloads.tree_params(
+        engines_hi=6, loops_hi=6, body_hi=6, trip_hi=4, max_depth=4))
+    compare_all(sg, batch, timeline=True,
+                params=oracle.sim_params(ii=2, c_branch=3, c_regop=2, c_barrier=9))
+
+
+def test_golden_fixtures_on_gpu(sg):
+    for name in golden_io.all_names():
+        batch, expects = golden_io.load(name)
+        h = sg.sync_load_programs(batch)
+        for mode_name, d, want in expects:
+            mode = COUNT if mode_name == "count" else PERLOOP
+            _, got = gpu_thresholds(sg, h, mode)
+            off = np.concatenate([[0], np.cumsum(h.pair_counts)])
+            assert got[off[d]:off[d + 1]].tolist() == want, name
+
+
+# ------------------------------------------------------------------ checker
+
+@pytest.mark.parametrize("mode", MODES)
+def test_checker_planted_errors(sg, mode):
+    import torch
+    batch = workloads.generate("depth2", n_programs=24)
+    h = sg.sync_load_programs(batch)
+    thr, good = gpu_thresholds(sg, h, mode)
+    idx = h.unpadded_index()
+    rng = np.random.default_rng(11)
+    pick = np.sort(rng.choice(idx.size, size=101, replace=False))
+    bad = good.copy()
+    bad[pick[::2]] += 1
+    bad[pick[1::2]] -= 1
+    dev = thr.clone()
+    dev[torch.from_numpy(idx[pick]).to(dev.device)] = torch.from_numpy(bad[pick]).to(dev.device)
+    counts, fb = sg.sync_check_minimal(h, mode, dev)
+    unsafe, over, first = oracle.check(batch, bad, mode)
+    assert counts.cpu().tolist() == [unsafe, over]
+    assert fb.item() == int(idx[first])
+    # calls overwrite, they do not accumulate
+    counts, fb = sg.sync_check_minimal(h, mode, thr)
+    assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
+
+
+def test_checker_detects_swapped_encoding(sg):
+    """Count-mode values read as per-loop values are below the minimum wherever
+    N > 1 and c > 0."""
+    batch = workloads.generate("gemm")
+    h = sg.sync_load_programs(batch)
+    thr_c, good_c = gpu_thresholds(sg, h, COUNT)
+    counts, _ = sg.sync_check_minimal(h, PERLOOP, thr_c)
+    unsafe, over, _ = oracle.check(batch, good_c, PERLOOP)
+    assert counts.cpu().tolist() == [unsafe, over] and unsafe > 0
+
+
+# --------------------------------------------------------------- edge cases
+
+def test_empty_batch(sg):
+    b = workloads.generate("chain", n_programs=0)
+    h = sg.sync_load_programs(b)
+    assert h.sizes.n_pairs_padded == 0
+    thr = sg.sync_eval_thresholds(h, PERLOOP)
+    counts, fb = sg.sync_check_minimal(h, PERLOOP, thr)
+    assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
+    sg.sync_simulate(h, PERLOOP, thr)
+
+
+def test_edge_programs(sg):
+    """Zero-trip consumer loops (empty segments), conditionals, programs with no
+    dependencies, 32 engines, nesting 15 deep, a deadlock under both schemes,
+    a deadlock under the barrier scheme only, and a time-bound overflow."""
+    progs = []
+    b = workloads.ProgramBuilder(3)          # empty segment in the middle
+    A = b.loop(0, 0, [4])
+    B = b.loop(A, 1, [0, 0, 0, 0])
+    x = b.instr(A, 0, 0)
+    y = b.instr(B, 0, 1)
+    z = b.instr(A, 2, 2)
+    b.dep(x, y, 0); b.dep(y, z, 0); b.dep(x, z, 1)
+    progs.append(b.batch())
+    b = workloads.ProgramBuilder(1)          # no dependencies
+    b.instr(0, 0, 0, latency=5)
+    progs.append(b.batch())
+    b = workloads.ProgramBuilder(32)         # 32 engines, a ring of waits
+    A = b.loop(0, 0, [5])
+    xs = [b.instr(A, i, i, latency=1 + i % 7) for i in range(32)]
+    for i in range(1, 32):
+        b.dep(xs[i - 1], xs[i], 0)
+    b.dep(xs[31], xs[0], 1)
+    progs.append(b.batch())
+    b = workloads.ProgramBuilder(2)          # nesting 15 deep, trips 1..2
+    par, tot, inner = 0, 1, []
+    for lvl in range(15):
+        t = 2 if lvl >= 13 else 1
+        par = b.loop(par, 1, [t] * tot)
+        tot *= t
+        inner.append(par)
+    p = b.instr(inner[2], 0, 0)
+    c = b.instr(inner[14], 0, 1)
+    b.dep(p, c, 0)
+    progs.append(b.batch())
+    b = workloads.ProgramBuilder(2)          # same-iteration cycle: deadlock
+    A = b.loop(0, 0, [3])
+    u = b.instr(A, 0, 0); v = b.instr(A, 1, 1)
+    b.dep(v, u, 0); b.dep(u, v, 0)
+    progs.append(b.batch())
+    b = workloads.ProgramBuilder(2)          # backward offset 0 across a loop
+    A = b.loop(0, 0, [3])
+    c = b.instr(A, 0, 1)
+    b.loop(A, 1, [2, 2, 2])
+    p = b.instr(A, 2, 0)
+    b.dep(p, c, 0)
+    progs.append(b.batch())
+    b = workloads.ProgramBuilder(1)          # time bound above INT32_MAX
+    L = b.loop(0, 0, [3])
+    b.instr(L, 0, 0, latency=2 ** 30)
+    progs.append(b.batch())
+    batch = workloads.concat(progs)
+    compare_all(sg, batch, timeline=True)
+    ref = oracle.simulate(batch, oracle.thresholds(batch, PERLOOP), PERLOOP, oracle.BARRIER)
+    assert 7 in ref.status.tolist() and 4 in ref.status.tolist()
+
+
+def test_zero_costs_and_large_costs(sg):
+    batch = workloads.random_trees(77, 120)
+    compare_all(sg, batch, params=oracle.sim_params(ii=0, c_branch=0, c_regop=0,
+                                                    c_wait_ops_count=0, c_wait_ops_perloop=0,
+                                                    c_barrier=0))
+    compare_all(sg, batch, params=oracle.sim_params(ii=7, c_branch=100, c_regop=50,
+                                                    c_wait_ops_count=9, c_wait_ops_perloop=13,
+                                                    c_barrier=1000))
+
+
+def test_repeated_calls_are_identical(sg):
+    batch = workloads.generate("chain", n_programs=300)
+    h = sg.sync_load_programs(batch)
+    thr = sg.sync_eval_thresholds(h, PERLOOP)
+    a = sg.sync_simulate(h, PERLOOP, thr)
+    b = sg.sync_simulate(h, PERLOOP, thr, variant=sg.SIM_BARRIER)
+    c = sg.sync_simulate(h, PERLOOP, thr)
+    assert np.array_equal(a.makespan.cpu().numpy(), c.makespan.cpu().numpy())
+    assert np.array_equal(a.checksum.cpu().numpy(), c.checksum.cpu().numpy())
+    assert not np.array_equal(a.makespan.cpu().numpy(), b.makespan.cpu().numpy())
+
+
+# ------------------------------------------------- full sizes, sampled checks
+
+@pytest.mark.parametrize("name", ["chain", "depth2", "attention", "syncbound"])
+def test_full_size_sampled(sg, name):
+    """The full configuration in one launch; a sample of its programs is
+    recomputed by the oracle program by program."""
+    batch = workloads.generate(name)
+    P = batch.n_programs
+    h = sg.sync_load_programs(batch)
+    rng = np.random.default_rng(5)
+    sample = np.unique(np.concatenate([[0, P - 1], rng.choice(P, size=min(P, 12), replace=False)]))
+    for mode in MODES:
+        thr = sg.sync_eval_thresholds(h, mode)
+        host = thr.cpu().numpy()
+        counts, fb = sg.sync_check_minimal(h, mode, thr)
+        assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
+        sims = {v: sg.sync_simulate(h, mode, thr, variant=v) for v in VARIANTS}
+        for p in sample.tolist():
+            one = workloads.generate(name, n_programs=1, first_program=p)
+            want = oracle.thresholds(one, mode)
+            d0, d1 = int(batch.prog_dep_ptr[p]), int(batch.prog_dep_ptr[p + 1])
+            got = np.concatenate([host[h.pair_offsets[d]:h.pair_offsets[d] + h.pair_counts[d]]
+                                  for d in range(d0, d1)] or [np.zeros(0, np.int32)])
+            assert np.array_equal(got, want), (name, mode, p)
+            for v in VARIANTS:
+                ref = oracle.simulate(one, want, mode, v)
+                assert sims[v].status[p].item() == ref.status[0]
+                assert sims[v].makespan[p].item() == ref.makespan[0], (name, mode, v, p)
+                assert np.uint64(sims[v].checksum[p].item() & (2 ** 64 - 1)) == ref.checksum[0]
+
+
+def test_full_size_gemm_timeline(sg):
+    """The single 1.25M-instance GEMM program, complete timeline."""
+    batch = workloads.generate("gemm")
+    compare_all(sg, batch, timeline=True, modes=(PERLOOP,))
