@@ -2,8 +2,8 @@
 
 A thin ctypes layer over ``include/sync.h``: it marshals arguments and owns
 torch tensors for outputs; every step of the path runs in the library's CUDA
-kernels.  Importing this module loads ``_lib/libsyncgb.so`` and fails loudly
-if it is missing -- there is no CPU fallback.
+kernels.  The first call loads ``_lib/libsyncgb.so`` and fails loudly if it
+is missing -- there is no CPU fallback.
 
     import paper_2608_13757_gb300 as sg
     h = sg.sync_load_programs(batch)                  # workloads.Batch or dict
@@ -90,12 +90,20 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     return lib
 
 
-_lib = load_library()
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library (loaded on first use; raises if it was not built)."""
+    global _lib
+    if _lib is None:
+        _lib = load_library()
+    return _lib
 
 
 def _check(status: int):
     if status != OK:
-        raise SyncError(status, _lib.sync_last_error().decode())
+        raise SyncError(status, lib().sync_last_error().decode())
 
 
 def _stream(stream):
@@ -132,11 +140,11 @@ class Programs:
         self._h = handle
         self.device = device
         s = Sizes()
-        _check(_lib.sync_query(self._h, ctypes.byref(s)))
+        _check(lib().sync_query(self._h, ctypes.byref(s)))
         self.sizes = s
         off = np.zeros(s.n_deps + 1, dtype=np.int64)
         cnt = np.zeros(max(s.n_deps, 1), dtype=np.int32)
-        _check(_lib.sync_pair_offsets(self._h, off.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+        _check(lib().sync_pair_offsets(self._h, off.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
                                       cnt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))))
         self.pair_offsets = off
         self.pair_counts = cnt[:s.n_deps]
@@ -157,7 +165,7 @@ class Programs:
 
     def close(self):
         if self._h:
-            _lib.sync_free_programs(self._h)
+            lib().sync_free_programs(self._h)
             self._h = None
 
     def __del__(self):
@@ -172,7 +180,7 @@ def sync_load_programs(batch, device: int = 0, stream=None) -> Programs:
     desc, keep = batch_desc(batch)
     h = ctypes.c_void_p()
     with torch.cuda.device(device):
-        _check(_lib.sync_load_programs(ctypes.byref(desc), int(device), _stream(stream),
+        _check(lib().sync_load_programs(ctypes.byref(desc), int(device), _stream(stream),
                                        ctypes.byref(h)))
     del keep
     return Programs(h, device)
@@ -183,7 +191,7 @@ def sync_eval_thresholds(h: Programs, mode: int = THR_PERLOOP, out=None, stream=
     n = h.sizes.n_pairs_padded
     if out is None:
         out = torch.empty(max(n, 4), dtype=torch.int32, device=f"cuda:{h.device}")
-    _check(_lib.sync_eval_thresholds(h.handle, int(mode), _ptr(out), _stream(stream)))
+    _check(lib().sync_eval_thresholds(h.handle, int(mode), _ptr(out), _stream(stream)))
     return out
 
 
@@ -195,7 +203,7 @@ def sync_check_minimal(h: Programs, mode, thr, counts=None, first_bad=None, stre
         counts = torch.empty(2, dtype=torch.int64, device=dev)
     if first_bad is None:
         first_bad = torch.empty(1, dtype=torch.int64, device=dev)
-    _check(_lib.sync_check_minimal(h.handle, int(mode), _ptr(thr), _ptr(counts), _ptr(first_bad),
+    _check(lib().sync_check_minimal(h.handle, int(mode), _ptr(thr), _ptr(counts), _ptr(first_bad),
                                    _stream(stream)))
     return counts, first_bad
 
@@ -224,7 +232,7 @@ def sync_simulate(h: Programs, mode, thr, params: SimParams | None = None,
             out.issue = torch.full((n,), -1, dtype=torch.int32, device=dev)
             out.retire = torch.full((n,), -1, dtype=torch.int32, device=dev)
     prm = params if params is not None else SimParams()
-    _check(_lib.sync_simulate(h.handle, int(mode), _ptr(thr), ctypes.byref(prm), int(variant),
+    _check(lib().sync_simulate(h.handle, int(mode), _ptr(thr), ctypes.byref(prm), int(variant),
                               _ptr(out.makespan), _ptr(out.checksum), _ptr(out.status),
                               _ptr(out.issue), _ptr(out.retire), _stream(stream)))
     return out

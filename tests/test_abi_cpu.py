@@ -37,19 +37,18 @@ def test_exports_every_declared_symbol(sg):
 
 
 def test_no_gpu_dependency_at_import(sg):
-    assert sg._lib.sync_last_error() is not None
+    assert sg.lib().sync_last_error() is not None
 
 
 def _status(sg, batch):
     desc, keep = sg.batch_desc(batch)
     h = ctypes.c_void_p()
-    st = sg._lib.sync_load_programs(ctypes.byref(desc), 0, None, ctypes.byref(h))
+    st = sg.lib().sync_load_programs(ctypes.byref(desc), 0, None, ctypes.byref(h))
     if st == sg.OK:
-        sg._lib.sync_free_programs(h)
-    return st, sg._lib.sync_last_error().decode()
+        sg.lib().sync_free_programs(h)
+    return st, sg.lib().sync_last_error().decode()
 
 
-VALIDATED = None  # set per environment: OK with a GPU, ERR_CUDA without one
 
 
 def _validated(sg):
@@ -62,16 +61,16 @@ def test_valid_batch_passes_validation(sg):
 
 
 def test_null_arguments(sg):
-    assert sg._lib.sync_load_programs(None, 0, None, None) == sg.ERR_ARG
+    assert sg.lib().sync_load_programs(None, 0, None, None) == sg.ERR_ARG
     s = sg.Sizes()
-    assert sg._lib.sync_query(None, ctypes.byref(s)) == sg.ERR_ARG
-    assert sg._lib.sync_eval_thresholds(None, 0, None, None) == sg.ERR_ARG
-    assert sg._lib.sync_check_minimal(None, 0, None, None, None, None) == sg.ERR_ARG
+    assert sg.lib().sync_query(None, ctypes.byref(s)) == sg.ERR_ARG
+    assert sg.lib().sync_eval_thresholds(None, 0, None, None) == sg.ERR_ARG
+    assert sg.lib().sync_check_minimal(None, 0, None, None, None, None) == sg.ERR_ARG
     prm = sg.SimParams()
-    assert sg._lib.sync_simulate(None, 0, None, ctypes.byref(prm), 0, None, None, None, None,
+    assert sg.lib().sync_simulate(None, 0, None, ctypes.byref(prm), 0, None, None, None, None,
                                  None, None) == sg.ERR_ARG
-    assert sg._lib.sync_last_error().decode() != ""
-    sg._lib.sync_free_programs(None)
+    assert sg.lib().sync_last_error().decode() != ""
+    sg.lib().sync_free_programs(None)
 
 
 def _base():
