@@ -206,10 +206,11 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  *   the top-level loop costs nothing; makespan = max over engines of
  *   max(t, last retire).
  * Outputs per program (device, [n_programs]): d_makespan (int32, -1 unless
- * status OK), d_checksum (uint64: sum over instances of
- * issue*0x9E3779B97F4A7C15 ^ retire*0xC2B2AE3D27D4EB4F ^
- * (n*0x165667B19E3779F9 + engine), n the 1-based ordinal in the engine's
- * stream; 0 unless OK), d_status (SYNC_PROG_*).  d_issue / d_retire:
+ * status OK), d_checksum (uint64, 0 unless OK: the sum mod 2^64 over
+ * datapath instances of (a << 32) | b in 32-bit arithmetic, a = (issue ^
+ * (n*0x9E3779B9 + e)) * 0x85EBCA6B, a ^= a >> 13, b = (retire ^
+ * (n*0xC2B2AE35 + e)) * 0x27D4EB2F, b ^= b >> 15, e the engine and n the
+ * instance's 1-based ordinal in engine e's stream), d_status (SYNC_PROG_*).  d_issue / d_retire:
  * [n_instances] int32 in instance layout, both NULL or both set (entries of
  * programs whose status is not OK are unspecified).  The handle's history
  * scratch is shared: calls on one handle must not overlap on the GPU. */

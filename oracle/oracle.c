@@ -63,10 +63,12 @@
  * (increments of one semaphore all come from one engine, in retire order).
  * Under the barrier scheme the waits stay in place; after a barrier they can
  * only be already satisfied or concern the current barrier interval.
- * Checksum: sum over datapath instances of
- *   issue*0x9E3779B97F4A7C15 ^ retire*0xC2B2AE3D27D4EB4F ^ (n*0x165667B19E3779F9 + e)
- * (mod 2^64, issue/retire as unsigned 32-bit, n = 1-based ordinal of the
- * instance in engine e's stream).  Status: 4 when the static time bound
+ * Checksum: the sum (mod 2^64) over datapath instances of
+ *   (a << 32) | b, with 32-bit arithmetic mod 2^32,
+ *   a = (issue ^ (n*0x9E3779B9 + e)) * 0x85EBCA6B, a ^= a >> 13,
+ *   b = (retire ^ (n*0xC2B2AE35 + e)) * 0x27D4EB2F, b ^= b >> 15,
+ * where e is the engine and n the instance's 1-based ordinal among engine
+ * e's datapath instances.  Status: 4 when the static time bound
  *   sum_x inst(x)*(lat(x)+ii+|D(x)|*c_wait) + E*(stmts*c_regop + iters*(c_branch+2*c_regop))
  * (barrier-free), or
  *   sum_x inst(x)*(lat(x)+ii) + E*iters*c_branch + (stmts+iters)*c_barrier
@@ -640,9 +642,11 @@ typedef struct {
 } sim_ctx;
 
 static uint64_t inst_term(int64_t issue, int64_t retire, int32_t e, int64_t n) {
-  return ((uint64_t)(uint32_t)issue * 0x9E3779B97F4A7C15ULL) ^
-         ((uint64_t)(uint32_t)retire * 0xC2B2AE3D27D4EB4FULL) ^
-         ((uint64_t)n * 0x165667B19E3779F9ULL + (uint64_t)e);
+  uint32_t a = ((uint32_t)issue ^ ((uint32_t)n * 0x9E3779B9u + (uint32_t)e)) * 0x85EBCA6Bu;
+  a ^= a >> 13;
+  uint32_t b = ((uint32_t)retire ^ ((uint32_t)n * 0xC2B2AE35u + (uint32_t)e)) * 0x27D4EB2Fu;
+  b ^= b >> 15;
+  return ((uint64_t)a << 32) | b;
 }
 
 static int64_t max64(int64_t a, int64_t b) { return a > b ? a : b; }

@@ -63,10 +63,17 @@ struct sync_programs {
   ProgInfo* prog = nullptr;
   int32_t* order = nullptr;
   int32_t* op_ptr = nullptr;
-  int32_t* ops = nullptr;
-  InstrSim* instr = nullptr;
-  ConsDep* cdep = nullptr;
+  int2* rowinfo = nullptr;
+  int4* ops = nullptr;
+  int32_t* opstop = nullptr;
+  int4* opsem = nullptr;            // [2][n_ops]
+  int64_t* dseg = nullptr;
+  int32_t* dsem = nullptr;          // [2][n_deps]
+  int64_t* semhb = nullptr;
+  int64_t* inst_off = nullptr;
+  int64_t n_ops = 0;
   int32_t* hist = nullptr;          // scratch: retire time of each semaphore increment
+  int32_t* next_slot = nullptr;     // scratch: simulator's program-slot counter
   int32_t nsem_max[2] = {0, 0};
   int32_t ne_max = 1;
   int32_t depth_max = 0;
@@ -119,7 +126,8 @@ void check_csr(const int32_t* ptr, int32_t P, const char* name) {
 
 // Per-program scratch of the loader (reused across programs).
 struct ProgScratch {
-  std::vector<int32_t> depth, body_ptr, body, rank, nloop_eng;
+  std::vector<int32_t> depth, body_ptr, body, rank, nloop_eng, x_ndeps, x_dep_begin;
+  std::vector<int32_t> x_own[2], x_hstride[2], x_koff[2];
   std::vector<int64_t> total, keys;
 };
 
@@ -158,9 +166,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<DepInfo> dep(ND);
   std::vector<int64_t> path;
   std::vector<ProgInfo> prog(P);
-  std::vector<int32_t> op_ptr, ops;
-  std::vector<InstrSim> instr(NX);
-  std::vector<ConsDep> cdep(ND);
+  std::vector<int32_t> op_ptr, opstop;
+  std::vector<int2> rowinfo;
+  std::vector<int4> ops, opsem[2];
+  std::vector<int64_t> inst_off(NX), dseg(ND), semhb;
+  std::vector<int32_t> dsem[2] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
   std::vector<int64_t> seg(ND + 1, 0);
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
@@ -253,37 +263,24 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         const int32_t it = S.body[i];
         if (it >= 0) S.rank[it] = ++S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + it]];
       }
-    // per-program aggregates and instruction table
+    // per-program aggregates
     ProgInfo& pi = prog[p];
     std::memset(&pi, 0, sizeof pi);
-    pi.loop_base = l0;
     pi.ne = ne;
     pi.le_base = (int32_t)op_ptr.size();
-    pi.depth = depth_max;
     __int128 agg = 0;
     for (int32_t x = 0; x < nx; ++x) {
       const int64_t tot = S.total[d.instr_loop[x0 + x]];
       agg += (__int128)tot * d.instr_latency[x0 + x];
-      InstrSim& X = instr[x0 + x];
-      std::memset(&X, 0, sizeof X);
-      X.lat = d.instr_latency[x0 + x];
-      X.inst_off = n_inst;
-      X.own_sem[0] = X.own_sem[1] = -1;
+      inst_off[x0 + x] = n_inst;
       n_inst += tot;
       pi.n_inst += tot;
     }
     pi.agg_lat = agg > (__int128)INT64_MAX ? INT64_MAX : (int64_t)agg;
     for (int32_t l = 1; l < nl; ++l) { pi.n_stmt += S.total[par[l]]; pi.n_iter += S.total[l]; }
-    // per-(loop, engine) instruction streams: own instructions and child loops
-    for (int32_t l = 0; l < nl; ++l)
-      for (int32_t e = 0; e < ne; ++e) {
-        op_ptr.push_back((int32_t)ops.size());
-        for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i) {
-          const int32_t it = S.body[i];
-          if (it < 0) ops.push_back(-(l0 + (-it - 1)) - 1);
-          else if (d.instr_engine[x0 + it] == e) ops.push_back(x0 + it);
-        }
-      }
+    S.x_ndeps.assign(nx, 0);
+    S.x_dep_begin.assign(nx, d0);
+    for (int m = 0; m < 2; ++m) { S.x_own[m].assign(nx, -1); S.x_hstride[m].assign(nx, 0); S.x_koff[m].assign(nx, 0); }
     // dependencies: innermost common loop S, cases of Sec. 5.2, N and K
     std::vector<int32_t> by_cons(nd);
     for (int32_t k = 0; k < nd; ++k) by_cons[k] = k;
@@ -367,45 +364,74 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         }
       }
       pi.nsem[m] = (int32_t)sem_hist.size();
+      pi.semhb_off[m] = (int32_t)semhb.size();
+      semhb.insert(semhb.end(), sem_hist.begin(), sem_hist.end());
       for (int32_t x = 0; x < nx; ++x) {
         const int32_t l = d.instr_loop[x0 + x];
         const int32_t key = m == 0 ? x : l * ne + d.instr_engine[x0 + x];
         const int32_t s = sem_of[key];
-        InstrSim& X = instr[x0 + x];
-        X.own_sem[m] = s;
+        S.x_own[m][x] = s;
         if (s < 0) continue;
-        X.hstride[m] = m == 0 ? 1 : S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]];
-        X.hbase[m] = sem_hist[s] + (m == 0 ? 0 : S.rank[x] - 1);
+        S.x_hstride[m][x] = m == 0 ? 1 : S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]];
+        S.x_koff[m][x] = m == 0 ? 1 : S.rank[x];
       }
-      for (int32_t k = 0; k < nd; ++k) {
-        const int64_t gd = d0 + k;
+      // dependencies grouped by consumer (stable by dependency id)
+      if (m == 0)
+        std::stable_sort(by_cons.begin(), by_cons.end(), [&](int32_t u, int32_t v) {
+          return d.dep_cons[d0 + u] < d.dep_cons[d0 + v];
+        });
+      for (int32_t i = 0; i < nd; ++i) {
+        const int64_t gd = d0 + by_cons[i];
         const int32_t px = d.dep_prod[gd];
         const int32_t key = m == 0 ? px : d.instr_loop[x0 + px] * ne + d.instr_engine[x0 + px];
-        cdep[gd].tsem[m] = sem_of[key];
-        cdep[gd].thist[m] = sem_hist[sem_of[key]];
+        dsem[m][d0 + i] = sem_of[key];
+        if (m == 0) dseg[d0 + i] = seg[gd];
       }
     }
-    // consumer-grouped dependency list (stable by dependency id)
-    std::stable_sort(by_cons.begin(), by_cons.end(), [&](int32_t u, int32_t v) {
-      return d.dep_cons[d0 + u] < d.dep_cons[d0 + v];
-    });
-    {
-      std::vector<ConsDep> grouped(nd);
-      for (int32_t i = 0; i < nd; ++i) {
-        grouped[i] = cdep[d0 + by_cons[i]];
-        grouped[i].seg_off = seg[d0 + by_cons[i]];
+    for (int32_t i = nd - 1; i >= 0; --i) S.x_dep_begin[d.dep_cons[d0 + by_cons[i]]] = d0 + i;
+    for (int32_t i = 0; i < nd; ++i) S.x_ndeps[d.dep_cons[d0 + by_cons[i]]]++;
+    // per-(loop, engine) op records: own instructions and child loops in body
+    // order, then an END record
+    for (int32_t l = 0; l < nl; ++l)
+      for (int32_t e = 0; e < ne; ++e) {
+        const int32_t first = (int32_t)ops.size();
+        op_ptr.push_back(first);
+        bool has_loop = false;
+        for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i) {
+          const int32_t it = S.body[i];
+          if (it < 0) {
+            const int32_t m = -it - 1;
+            const int64_t rp = loop[l0 + m].rowptr_off;
+            ops.push_back(make_int4(OP_LOOP, pi.le_base + m * ne, (int32_t)(uint32_t)(rp & 0xffffffffu),
+                                    (int32_t)(rp >> 32)));
+            opsem[0].push_back(make_int4(-1, 0, 0, 0));
+            opsem[1].push_back(make_int4(-1, 0, 0, 0));
+            has_loop = true;
+          } else if (d.instr_engine[x0 + it] == e) {
+            ops.push_back(make_int4(x0 + it, d.instr_latency[x0 + it], S.x_ndeps[it], S.x_dep_begin[it]));
+            for (int m = 0; m < 2; ++m)
+              opsem[m].push_back(make_int4(S.x_own[m][it], S.x_hstride[m][it], S.x_koff[m][it], 0));
+          }
+        }
+        const int32_t end_idx = (int32_t)ops.size();
+        ops.push_back(make_int4(OP_END, 0, 0, 0));
+        opsem[0].push_back(make_int4(-1, 0, 0, 0));
+        opsem[1].push_back(make_int4(-1, 0, 0, 0));
+        rowinfo.push_back(make_int2(end_idx, has_loop ? 1 : 0));
+        // next LOOP or END record at or after each record of the row
+        opstop.resize(ops.size());
+        int32_t next = end_idx;
+        for (int32_t r = end_idx; r >= first; --r) {
+          if (ops[r].x < 0) next = r;
+          opstop[r] = next;
+        }
       }
-      for (int32_t i = 0; i < nd; ++i) cdep[d0 + i] = grouped[i];
-      for (int32_t x = 0; x < nx; ++x) instr[x0 + x].dep_begin = d0;
-      for (int32_t i = nd - 1; i >= 0; --i) instr[x0 + d.dep_cons[d0 + by_cons[i]]].dep_begin = d0 + i;
-      for (int32_t i = 0; i < nd; ++i) instr[x0 + d.dep_cons[d0 + by_cons[i]]].ndeps++;
-    }
     h.nsem_max[0] = std::max(h.nsem_max[0], pi.nsem[0]);
     h.nsem_max[1] = std::max(h.nsem_max[1], pi.nsem[1]);
     h.ne_max = std::max(h.ne_max, ne);
     h.depth_max = std::max(h.depth_max, depth_max);
+    if ((int64_t)ops.size() > kI32Max) raise(SYNC_ERR_OVERFLOW, "op records exceed INT32_MAX entries");
   }
-  if ((int64_t)ops.size() > kI32Max) raise(SYNC_ERR_OVERFLOW, "instruction streams exceed INT32_MAX entries");
   op_ptr.push_back((int32_t)ops.size());
   seg[ND] = n_pairs_padded;
 
@@ -482,11 +508,24 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   int32_t* d_tile_loop = h.upload(tile_loop, stream, "loop tile table");
   h.prog = h.upload(prog, stream, "program table");
   h.order = h.upload(order, stream, "program order");
-  h.op_ptr = h.upload(op_ptr, stream, "stream offsets");
-  h.ops = h.upload(ops, stream, "streams");
-  h.instr = h.upload(instr, stream, "instruction table");
-  h.cdep = h.upload(cdep, stream, "consumer dependency table");
+  h.op_ptr = h.upload(op_ptr, stream, "op record offsets");
+  h.rowinfo = h.upload(rowinfo, stream, "row info");
+  h.ops = h.upload(ops, stream, "op records");
+  h.opstop = h.upload(opstop, stream, "op stops");
+  {
+    std::vector<int4> both(opsem[0]);
+    both.insert(both.end(), opsem[1].begin(), opsem[1].end());
+    h.opsem = h.upload(both, stream, "op semaphore records");
+    std::vector<int32_t> dboth(dsem[0]);
+    dboth.insert(dboth.end(), dsem[1].begin(), dsem[1].end());
+    h.dsem = h.upload(dboth, stream, "dependency semaphores");
+  }
+  h.n_ops = (int64_t)ops.size();
+  h.dseg = h.upload(dseg, stream, "dependency segments");
+  h.semhb = h.upload(semhb, stream, "semaphore history bases");
+  h.inst_off = h.upload(inst_off, stream, "instance offsets");
   h.hist = h.alloc<int32_t>(std::max(hist_len[0], hist_len[1]), "semaphore history");
+  h.next_slot = h.alloc<int32_t>(1, "program-slot counter");
   cuda_check(launch_expand(h.loop, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
   cuda_check(cudaStreamSynchronize(stream), "load");
 }
@@ -591,19 +630,22 @@ sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int3
     cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
     SimArgs a;
     std::memset(&a, 0, sizeof a);
-    a.prog = h->prog; a.order = h->order; a.loop = h->loop; a.rowptr = h->rowptr;
-    a.op_ptr = h->op_ptr; a.ops = h->ops; a.instr = h->instr; a.cdep = h->cdep;
-    a.thr = d_thr; a.hist = h->hist;
+    a.prog = h->prog; a.order = h->order; a.rowptr = h->rowptr;
+    a.op_ptr = h->op_ptr; a.rowinfo = h->rowinfo; a.ops = h->ops; a.opstop = h->opstop;
+    a.opsem = h->opsem + (size_t)mode * h->n_ops;
+    a.dseg = h->dseg; a.dsem = h->dsem + (size_t)mode * h->sz.n_deps;
+    a.semhb = h->semhb;
+    a.inst_off = h->inst_off;
+    a.thr = d_thr; a.hist = h->hist; a.next_slot = h->next_slot;
     a.makespan = d_makespan; a.checksum = d_checksum; a.status = d_status;
     a.issue = d_issue; a.retire = d_retire;
     a.prm = q;
     a.n_programs = h->sz.n_programs;
     a.mode = mode;
-    a.sem_ints = (h->nsem_max[mode] + 3) & ~3;
+    a.sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
     a.frame_depth = std::max(1, h->depth_max);
-    a.ne_max = h->ne_max;
-    const size_t per_warp = simulate_smem_per_warp(a.sem_ints, a.frame_depth, a.ne_max);
-    if (per_warp * 4 > 200 * 1024)
+    a.warps = h->ne_max;
+    if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024)
       raise(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
     cuda_check(launch_simulate(a, variant == SYNC_SIM_BARRIER, h->num_sms, static_cast<cudaStream_t>(stream)),
                "simulator kernel");

@@ -55,33 +55,34 @@ struct alignas(16) ProgInfo {
   int64_t n_pairs;    // (dependency, consumer instance) pairs
   int64_t n_stmt;     // loop statements reached (sum over non-top loops of total(parent))
   int64_t n_iter;     // loop iterations (sum over non-top loops of total)
-  int32_t loop_base;  // global id of the program's top-level loop
   int32_t ne;
-  int32_t le_base;    // index of (top-level loop, engine 0) in op_ptr
+  int32_t le_base;    // row of (top-level loop, engine 0); row of (program-local
+                      // loop l, engine e) = le_base + l*ne + e
   int32_t nsem[2];    // waited semaphores, per threshold mode
-  int32_t depth;      // deepest nesting level
+  int32_t semhb_off[2];  // first entry of the program's history bases, per mode
 };
 
-// Per instruction, for the simulator.  Semaphore fields per threshold mode
-// (0 = per instruction, 1 = per (loop, engine)); own_sem -1 when nothing
-// waits on that semaphore (no history kept).
-struct alignas(16) InstrSim {
-  int64_t hbase[2];   // history slot of this instruction's increment in g = 0
-  int64_t inst_off;   // instance-layout offset
-  int32_t own_sem[2];
-  int32_t hstride[2]; // history slots between consecutive iterations
-  int32_t lat;
-  int32_t ndeps;      // dependencies consumed
-  int32_t dep_begin;  // first entry in the consumer-grouped dependency list
-  int32_t pad_;
-};
-
-// Per (consumer, dependency), grouped by consumer.
-struct alignas(16) ConsDep {
-  int64_t seg_off;    // pair-layout offset of the dependency's segment
-  int64_t thist[2];   // history base of the waited semaphore
-  int32_t tsem[2];    // local id of the waited semaphore
-};
+// Simulator op records, one list ("row") per (loop, engine): the engine's own
+// instructions and every child loop of the loop's body, in body order, then
+// an END record.  16 bytes each:
+//   datapath  {x >= 0 (global instruction), latency, dependencies consumed,
+//              first entry in the consumer-grouped dependency list}
+//   loop      {OP_LOOP, row of (child, engine 0), rowptr offset lo, hi}
+//   end       {OP_END, 0, 0, 0}
+// Per record: opstop = index of the first LOOP or END record at or after it
+// in its row.  Per row: op_ptr = first record, rowinfo = {END record index,
+// 1 if the row holds a LOOP record}.
+// Per-mode semaphore records parallel to the op records (mode 0 = one
+// semaphore per producer instruction, mode 1 = one per (loop, engine)):
+//   {semaphore (program-local, -1 if nothing waits on it), increments per
+//    iteration (1 or N), koff (1 or K)}: the increment of iteration g brings
+//    the semaphore to stride*g + koff and its retire time lives at history
+//    slot semhb[semaphore] + stride*g + koff - 1.
+// Consumer-grouped dependencies: segment offset (int64) and, per mode, the
+// waited semaphore (program-local).  semhb: per program and mode, the
+// history base of each waited semaphore.
+constexpr int32_t OP_LOOP = -1;
+constexpr int32_t OP_END = -2;
 
 struct ThrArgs {
   const DepInfo* dep;
@@ -103,15 +104,20 @@ struct CheckArgs {
 
 struct SimArgs {
   const ProgInfo* prog;
-  const int32_t* order;      // program slots in descending-work order
-  const LoopInfo* loop;
+  const int32_t* order;      // program ids in descending-work order
   const int32_t* rowptr;
-  const int32_t* op_ptr;
-  const int32_t* ops;        // x >= 0 own instruction, -(m+1) child loop m
-  const InstrSim* instr;
-  const ConsDep* cdep;
+  const int32_t* op_ptr;     // [rows] first record of each row
+  const int2* rowinfo;       // [rows]
+  const int4* ops;
+  const int32_t* opstop;
+  const int4* opsem;         // per-mode records, parallel to ops
+  const int64_t* dseg;
+  const int32_t* dsem;       // per-mode waited semaphore, parallel to dseg
+  const int64_t* semhb;
+  const int64_t* inst_off;   // per instruction, instance-layout offset
   const int32_t* thr;
-  int32_t* hist;
+  int32_t* hist;             // scratch: retire time of each semaphore increment
+  int32_t* next_slot;        // scratch: next program slot to fetch (zeroed per launch)
   int32_t* makespan;
   unsigned long long* checksum;
   int32_t* status;
@@ -120,9 +126,9 @@ struct SimArgs {
   sync_sim_params prm;
   int32_t n_programs;
   int32_t mode;
-  int32_t sem_ints;          // shared-memory ints for semaphore values per warp
-  int32_t frame_depth;       // frames per lane
-  int32_t ne_max;
+  int32_t warps;             // warps per CTA (largest engine count of the batch)
+  int32_t sem_cap;           // semaphore slots in shared memory
+  int32_t frame_depth;       // frames per warp
 };
 
 // Launchers (return the launch error, if any).
@@ -133,6 +139,6 @@ cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const 
 cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s);
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStream_t s);
-size_t simulate_smem_per_warp(int sem_ints, int frame_depth, int ne_max);
+size_t simulate_smem_bytes(int warps, int sem_cap, int frame_depth);
 
 }  // namespace syncgb

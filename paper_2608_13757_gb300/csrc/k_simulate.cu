@@ -1,35 +1,58 @@
-// Schedule simulator: one warp per program, lane e = engine e.
+// Schedule simulator: one CTA per program at a time, warp e = engine e.
 //
-// Every lane walks the common loop tree with its own cursor (a stack of
-// frames in shared memory) and its own time t, visiting its engine's
-// instructions and every loop's control points.  Lanes run independently in
-// bursts of up to kBurst events and meet once per round at a __syncwarp:
-//   - a datapath instruction waits on semaphores: the value of a semaphore
-//     (increments processed so far) lives in shared memory, written only by
-//     the owning engine's lane with a release store after the increment's
-//     retire time was written to the history array; a waiting lane reads the
-//     value with an acquire load and, once it reaches the threshold, takes
-//     the retire time of that increment (the time the semaphore reached it);
-//     otherwise it stops its burst and retries in the next round;
-//   - a barrier (barrier scheme) stops the lane; when the ballot shows every
-//     engine of the program at its barrier, the release time is the
-//     warp-reduced maximum arrival plus the barrier cost;
-//   - a round in which no lane moved is a deadlock (every lane saw the state
-//     published before the previous __syncwarp and still could not move).
-// Times are int32: a program whose static time bound exceeds INT32_MAX gets
-// status 4 without being simulated, so no time can overflow.
+// Each warp walks the common loop tree for its engine (current row of op
+// records, iteration range, a stack of frames in shared memory), but instead
+// of one event per step it takes up to 32 consecutive events of its stream at
+// once, one per lane:
+//   - inside a loop body with no child loop (barrier-free), the events run on
+//     across iteration boundaries (the body's records repeat, the END record
+//     between two iterations is an iteration start);
+//   - otherwise they stop at the next child loop or END record, which the
+//     whole warp then handles as one control step (loop statement, next
+//     iteration, loop exit, barrier).
+// The engine's cursor obeys t' = max(t + A, B) for every event -- A the cost
+// of the event (wait ops, issue interval, iteration start), B the time its
+// waits become satisfied plus the issue interval (or -inf) -- and these
+// max-plus affine maps compose associatively, so a 5-step warp scan gives
+// every lane the cursor before its event; issue = max(cursor + wait ops,
+// ready), and retire (in-order retirement) is a max-scan of issue + latency.
+//
+// Waits: a semaphore's value (its increments processed so far) and the
+// history base of its retire times live in shared memory; only the owning
+// engine's warp writes them -- the retire times to the history array first,
+// then, after __syncwarp, one release store of the semaphore's new value per
+// semaphore touched by the chunk.  A lane whose wait is not yet satisfied
+// cuts the chunk before itself; a warp whose first event is blocked polls
+// that semaphore a bounded number of times, then ends its round.
+// Barriers (barrier scheme) are met in shared memory: each engine stores its
+// arrival time and counts itself in; the last one computes the release (the
+// maximum arrival plus the barrier cost) and advances a generation counter,
+// which the others poll a bounded number of times before ending their round.
+// Warps meet once per round at a CTA barrier; a round in which no warp moved
+// is a deadlock.
+//
+// CTAs are persistent and fetch program ids from a counter in descending-work
+// order.  Times are int32: a program whose static time bound exceeds
+// INT32_MAX gets status 4 without being simulated, so no time can overflow.
 #include "enc.h"
 
 namespace syncgb {
 namespace {
 
-constexpr int kWarps = 4;       // warps per CTA
-constexpr int kBurst = 16;      // events per lane between two warp meetings
+constexpr int kChunks = 16;                 // chunks per warp per round
+constexpr int kSpin = 64;                   // polls of a semaphore or barrier per round
+// A program still running after this many SM clock cycles (about 2 s) stops at
+// the next round boundary with status 8, so a launch always ends.
+constexpr long long kWatchdogCycles = 4000000000ll;
+constexpr unsigned kFull = 0xffffffffu;
+// "-infinity" of the max-plus maps t' = max(t + A, B): cursors are >= 0 and
+// costs A >= 0, so a composed term -1 + (later costs) never exceeds the
+// t + (all costs) term and -1 acts exactly as -infinity in int32.
+constexpr int32_t kNeg = -1;
 
 enum : int { ST_RUN = 0, ST_BAR = 1, ST_DONE = 2 };
-enum : int { R_MOVED = 0, R_BLOCKED = 1, R_BARRIER = 2, R_DONE = 3 };
 
-struct Frame { int32_t loop, ptr, g, g_end; };
+struct Frame { int32_t row, ptr, g, g_end; };
 
 __device__ __forceinline__ int32_t ld_acquire(const int32_t* p) {
   int32_t v;
@@ -41,6 +64,11 @@ __device__ __forceinline__ void st_release(int32_t* p, int32_t v) {
   asm volatile("st.release.cta.shared.b32 [%0], %1;"
                :: "r"((unsigned)__cvta_generic_to_shared(p)), "r"(v) : "memory");
 }
+__device__ __forceinline__ unsigned lanemask_le() {
+  unsigned m;
+  asm("mov.u32 %0, %%lanemask_le;" : "=r"(m));
+  return m;
+}
 
 __device__ __forceinline__ unsigned long long sat_add(unsigned long long a, unsigned long long b) {
   const unsigned long long r = a + b;
@@ -49,216 +77,407 @@ __device__ __forceinline__ unsigned long long sat_add(unsigned long long a, unsi
 __device__ __forceinline__ unsigned long long sat_mul(unsigned long long a, unsigned long long b) {
   return __umul64hi(a, b) ? ~0ull : a * b;
 }
-
-__device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t retire, int32_t e,
-                                                        long long n) {
-  return ((unsigned long long)(uint32_t)issue * 0x9E3779B97F4A7C15ull) ^
-         ((unsigned long long)(uint32_t)retire * 0xC2B2AE3D27D4EB4Full) ^
-         ((unsigned long long)n * 0x165667B19E3779F9ull + (unsigned long long)e);
+__device__ __forceinline__ int64_t lohi(int32_t lo, int32_t hi) {
+  return (int64_t)(((uint64_t)(uint32_t)hi << 32) | (uint32_t)lo);
 }
 
-// Lane-private state of one engine.
-struct Lane {
-  int32_t cur, ptr, pend, g, g_end, sp;
-  int32_t t, lastret, arrival;
-  long long n;
-  unsigned long long chk;
+// Per-instance checksum term (see include/sync.h).
+__device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t retire, uint32_t e,
+                                                        uint32_t n) {
+  uint32_t x = ((uint32_t)issue ^ (n * 0x9E3779B9u + e)) * 0x85EBCA6Bu;
+  x ^= x >> 13;
+  uint32_t y = ((uint32_t)retire ^ (n * 0xC2B2AE35u + e)) * 0x27D4EB2Fu;
+  y ^= y >> 15;
+  return ((unsigned long long)x << 32) | y;
+}
+
+// Static time bound of a program under the given costs (saturating).
+template <bool BB>
+__device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, const sync_sim_params& q,
+                                                         int32_t cwait) {
+  typedef unsigned long long u64;
+  u64 b = sat_add((u64)pi.agg_lat, sat_mul((u64)q.ii, (u64)pi.n_inst));
+  if (BB) {
+    b = sat_add(b, sat_mul(sat_mul((u64)pi.ne, (u64)pi.n_iter), (u64)q.c_branch));
+    b = sat_add(b, sat_mul((u64)(pi.n_stmt + pi.n_iter), (u64)q.c_barrier));
+  } else {
+    b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
+    const u64 ctl = sat_add(sat_mul((u64)pi.n_stmt, (u64)q.c_regop),
+                            sat_mul((u64)pi.n_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop));
+    b = sat_add(b, sat_mul((u64)pi.ne, ctl));
+  }
+  return b;
+}
+
+struct Smem {
+  int64_t* semhb;          // [sem_cap]
+  int32_t* sem;            // [sem_cap]
+  int32_t* w_moved;        // [warps]
+  int32_t* w_state;
+  int32_t* w_arrival;      // barrier arrival times
+  int32_t* w_ms;
+  unsigned long long* w_chk;
+  int32_t* slot;           // [4]: program slot, barrier count, generation, release
+  Frame* frames;           // [warps][frame_depth]
+};
+
+// Engine state, identical in the 32 lanes of the engine's warp.
+struct Eng {
+  int32_t row, pbeg, rend, ptr, g, g_end, sp;
+  bool loops;              // the current row holds a child loop
+  int32_t t, lastret;
+  int32_t bar_gen;         // barrier generation this engine waits to see pass
+  uint32_t n;              // datapath instances issued so far
+  int state;
   bool bar_passed;
 };
 
-template <int MODE, bool BB, bool TL>
-__device__ __forceinline__ int step(const SimArgs& a, const ProgInfo& pi, Lane& L, Frame* stk,
-                                    int32_t* sem, int lane, int32_t iter_cost, int32_t cwait) {
-  if (L.ptr == L.pend) {                       // end of an iteration's body
-    if (L.sp == 0) return R_DONE;              // the top-level loop runs once
-    if (BB && !L.bar_passed) { L.arrival = max(L.t, L.lastret); return R_BARRIER; }
-    L.bar_passed = false;
-    if (++L.g < L.g_end) {                     // next iteration starts
-      L.t += iter_cost;
-      L.ptr = __ldg(a.op_ptr + pi.le_base + (L.cur - pi.loop_base) * pi.ne + lane);
-      return R_MOVED;
+// Arrive at the program's next barrier; the last engine to arrive releases it.
+// Returns true once the barrier has been released for this engine.
+template <bool BB>
+__device__ __forceinline__ bool barrier_arrive(const SimArgs& a, const Smem& S, Eng& E, int w, int lane,
+                                              int ne) {
+  E.bar_gen = ld_acquire(S.slot + 2);
+  int last = 0;
+  if (lane == 0) {
+    S.w_arrival[w] = max(E.t, E.lastret);
+    __threadfence_block();
+    last = atomicAdd(S.slot + 1, 1) == ne - 1;
+    if (last) {
+      __threadfence_block();
+      int32_t rel = 0;
+      for (int i = 0; i < ne; ++i) rel = max(rel, *(volatile int32_t*)(S.w_arrival + i));
+      S.slot[3] = rel + a.prm.c_barrier;
+      S.slot[1] = 0;
+      st_release(S.slot + 2, E.bar_gen + 1);
     }
-    const Frame f = stk[--L.sp];               // loop exit
-    L.cur = f.loop; L.ptr = f.ptr; L.g = f.g; L.g_end = f.g_end;
-    L.pend = __ldg(a.op_ptr + pi.le_base + (L.cur - pi.loop_base) * pi.ne + lane + 1);
-    return R_MOVED;
   }
-  const int32_t op = __ldg(a.ops + L.ptr);
-  if (op < 0) {                                // a loop statement
-    if (BB && !L.bar_passed) { L.arrival = max(L.t, L.lastret); return R_BARRIER; }
-    L.bar_passed = false;
-    if (!BB) L.t += a.prm.c_regop;
-    const int32_t m = -op - 1;
-    const int64_t rp = __ldg(&a.loop[m].rowptr_off) + L.g;
-    const int32_t lo = __ldg(a.rowptr + rp), hi = __ldg(a.rowptr + rp + 1);
-    ++L.ptr;
-    if (lo < hi) {
-      stk[L.sp++] = Frame{L.cur, L.ptr, L.g, L.g_end};
-      const int32_t row = pi.le_base + (m - pi.loop_base) * pi.ne + lane;
-      L.cur = m; L.g = lo; L.g_end = hi;
-      L.ptr = __ldg(a.op_ptr + row);
-      L.pend = __ldg(a.op_ptr + row + 1);
-      L.t += iter_cost;
-    }
-    return R_MOVED;
+  E.state = ST_BAR;
+  return __shfl_sync(kFull, last, 0) != 0;
+}
+
+// Has the barrier this engine waits at been released?  Polls at most kSpin times.
+__device__ __forceinline__ bool barrier_poll(const Smem& S, const Eng& E, int spins) {
+  for (int i = 0;; ++i) {
+    if (ld_acquire(S.slot + 2) != E.bar_gen) return true;
+    if (i >= spins) return false;
   }
-  // datapath instruction `op` in global iteration L.g of its loop
-  const InstrSim& X = a.instr[op];
-  const int32_t ndeps = __ldg(&X.ndeps);
-  const int32_t dep_begin = __ldg(&X.dep_begin);
-  const int32_t tw = L.t + (BB ? 0 : ndeps * cwait);
-  int32_t ready = 0;
-  for (int j = 0; j < ndeps; ++j) {
-    const ConsDep& C = a.cdep[dep_begin + j];
-    const int32_t T = __ldg(a.thr + __ldg(&C.seg_off) + L.g);
-    if (T <= 0) continue;
-    const int32_t s = __ldg(&C.tsem[MODE]);
-    if (ld_acquire(sem + s) < T) return R_BLOCKED;   // semaphore below threshold
-    ready = max(ready, a.hist[__ldg(&C.thist[MODE]) + (T - 1)]);
-  }
-  const int32_t issue = max(tw, ready);
-  const int32_t retire = max(issue + __ldg(&X.lat), L.lastret);
-  L.t = issue + a.prm.ii;
-  L.lastret = retire;
-  const int32_t s = __ldg(&X.own_sem[MODE]);
-  if (s >= 0) {                                // someone waits on this semaphore
-    a.hist[__ldg(&X.hbase[MODE]) + (int64_t)__ldg(&X.hstride[MODE]) * L.g] = retire;
-    st_release(sem + s, sem[s] + 1);
-  }
-  ++L.n;
-  L.chk += inst_term(issue, retire, lane, L.n);
-  if (TL) {
-    const int64_t o = __ldg(&X.inst_off) + L.g;
-    a.issue[o] = issue;
-    a.retire[o] = retire;
-  }
-  ++L.ptr;
-  return R_MOVED;
 }
 
 template <int MODE, bool BB, bool TL>
-__global__ void __launch_bounds__(kWarps * 32) k_simulate(const SimArgs a) {
-  extern __shared__ __align__(16) int32_t smem[];
-  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-  const int per_warp = a.sem_ints + a.ne_max * a.frame_depth * 4;
-  int32_t* sem = smem + wib * per_warp;
-  Frame* stk = reinterpret_cast<Frame*>(sem + a.sem_ints) + (lane < a.ne_max ? lane : 0) * a.frame_depth;
+__device__ __forceinline__ void set_row(const SimArgs& a, Eng& E, int32_t row) {
+  E.row = row;
+  E.pbeg = __ldg(a.op_ptr + row);
+  const int2 ri = __ldg(a.rowinfo + row);
+  E.rend = ri.x;
+  E.loops = ri.y != 0;
+}
+
+// One round of engine w: up to kChunks chunks or control steps.
+template <int MODE, bool BB, bool TL>
+__device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng& E, int w, int lane,
+                                           int ne, unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
-  const long long n_warps = (long long)gridDim.x * kWarps;
-
-  for (long long slot = (long long)blockIdx.x * kWarps + wib; slot < a.n_programs; slot += n_warps) {
-    const int p = __ldg(a.order + slot);
-    const ProgInfo pi = a.prog[p];
-    // static time bound (identical in every lane)
-    unsigned long long bound = (unsigned long long)pi.agg_lat;
-    bound = sat_add(bound, sat_mul((unsigned long long)a.prm.ii, (unsigned long long)pi.n_inst));
-    if (BB) {
-      bound = sat_add(bound, sat_mul(sat_mul((unsigned long long)pi.ne, (unsigned long long)pi.n_iter),
-                                     (unsigned long long)a.prm.c_branch));
-      bound = sat_add(bound, sat_mul((unsigned long long)(pi.n_stmt + pi.n_iter),
-                                     (unsigned long long)a.prm.c_barrier));
-    } else {
-      bound = sat_add(bound, sat_mul((unsigned long long)cwait, (unsigned long long)pi.n_pairs));
-      const unsigned long long ctl =
-          sat_add(sat_mul((unsigned long long)pi.n_stmt, (unsigned long long)a.prm.c_regop),
-                  sat_mul((unsigned long long)pi.n_iter,
-                          (unsigned long long)a.prm.c_branch + 2ull * (unsigned long long)a.prm.c_regop));
-      bound = sat_add(bound, sat_mul((unsigned long long)pi.ne, ctl));
+  const int32_t ii = a.prm.ii;
+  Frame* frames = S.frames + w * a.frame_depth;
+  bool moved = false;
+  int spins = kSpin;
+  if (BB && E.state == ST_BAR) {                     // waiting at a barrier
+    if (!barrier_poll(S, E, spins)) return false;
+    E.t = *(volatile int32_t*)(S.slot + 3);
+    E.state = ST_RUN;
+    E.bar_passed = true;
+    moved = true;
+  }
+  for (int c = 0; c < kChunks; ++c) {
+    const int4 r0 = __ldg(a.ops + E.ptr);
+    if (BB && (r0.x == OP_LOOP || (r0.x == OP_END && E.sp != 0)) && !E.bar_passed) {
+      // an all-engine barrier before the loop statement / after the iteration
+      moved = true;
+      if (!barrier_arrive<BB>(a, S, E, w, lane, ne) && !barrier_poll(S, E, spins)) return true;
+      E.t = *(volatile int32_t*)(S.slot + 3);
+      E.state = ST_RUN;
+      E.bar_passed = true;
     }
-    if (bound > 2147483647ull) {
-      if (lane == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
+    if (r0.x == OP_LOOP) {                           // a loop statement
+      E.bar_passed = false;
+      if (!BB) E.t += a.prm.c_regop;
+      const int64_t rp = lohi(r0.z, r0.w) + E.g;
+      const int32_t lo = __ldg(a.rowptr + rp), hi = __ldg(a.rowptr + rp + 1);
+      ++E.ptr;
+      if (lo < hi) {
+        __syncwarp();
+        if (lane == 0) frames[E.sp] = Frame{E.row, E.ptr, E.g, E.g_end};
+        ++E.sp;
+        set_row<MODE, BB, TL>(a, E, r0.y + w);
+        E.ptr = E.pbeg;
+        E.g = lo;
+        E.g_end = hi;
+        E.t += iter_cost;
+      }
+      moved = true;
       continue;
     }
-    for (int i = lane; i < pi.nsem[MODE]; i += 32) sem[i] = 0;
-    __syncwarp();
+    if (r0.x == OP_END) {                            // end of an iteration's body
+      if (E.sp == 0) { E.state = ST_DONE; return true; }   // the top-level loop runs once
+      E.bar_passed = false;
+      if (++E.g < E.g_end) {
+        E.t += iter_cost;
+        E.ptr = E.pbeg;
+      } else {
+        __syncwarp();
+        const Frame f = frames[--E.sp];
+        set_row<MODE, BB, TL>(a, E, f.row);
+        E.ptr = f.ptr; E.g = f.g; E.g_end = f.g_end;
+      }
+      moved = true;
+      continue;
+    }
+    // ---- a chunk of datapath events (and, run-on, iteration starts)
+    const bool periodic = !BB && !E.loops;
+    const int32_t period = E.rend - E.pbeg + 1;      // the body's records and its END
+    int32_t idx, gj;
+    bool valid, is_end;
+    if (periodic) {
+      const int32_t off = (E.ptr - E.pbeg) + lane;
+      const int32_t it = off / period;
+      idx = E.pbeg + (off - it * period);
+      gj = E.g + it;
+      is_end = idx == E.rend;
+      valid = gj < E.g_end && !(is_end && gj == E.g_end - 1);   // stop before the loop exit
+    } else {
+      const int32_t stop = __ldg(a.opstop + E.ptr);
+      idx = E.ptr + lane;
+      gj = E.g;
+      is_end = false;
+      valid = idx < stop;
+    }
+    const int32_t nev = __popc(__ballot_sync(kFull, valid));
+    const bool dp = valid && !is_end;
+    int4 rec = make_int4(0, 0, 0, 0), srec = make_int4(-1, 0, 0, 0);
+    if (dp) {
+      rec = __ldg(a.ops + idx);
+      srec = __ldg(a.opsem + idx);
+    }
+    // waits: every dependency's semaphore must have reached the threshold
+    int32_t ready = 0, bsem = 0, bthr = 0;
+    bool waited = false, blocked = false;
+    for (int j = 0; dp && j < rec.z; ++j) {
+      const int32_t T = __ldg(a.thr + __ldg(a.dseg + rec.w + j) + gj);
+      if (T <= 0) continue;
+      const int32_t s = __ldg(a.dsem + rec.w + j);
+      if (ld_acquire(S.sem + s) < T) { blocked = true; bsem = s; bthr = T; break; }
+      ready = max(ready, a.hist[S.semhb[s] + (T - 1)]);
+      waited = true;
+    }
+    const unsigned bm = __ballot_sync(kFull, blocked);
+    const int32_t cut = bm ? min(nev, __ffs(bm) - 1) : nev;
+    if (cut == 0) {                                  // blocked at the first event
+      const int32_t s = __shfl_sync(kFull, bsem, 0), T = __shfl_sync(kFull, bthr, 0);
+      for (;;) {                                     // poll the semaphore, bounded
+        if (spins <= 0) return moved;
+        --spins;
+        if (ld_acquire(S.sem + s) >= T) break;
+      }
+      --c;                                           // retry this chunk
+      continue;
+    }
+    const bool in = lane < cut;
+    // cursor maps t' = max(t + A, B), inclusive scan over the lanes
+    const int32_t wcost = BB ? 0 : rec.z * cwait;
+    int32_t A = 0, B = kNeg;
+    if (in) {
+      if (dp) { A = wcost + ii; B = waited ? ready + ii : kNeg; }
+      else A = iter_cost;
+    }
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t Ap = __shfl_up_sync(kFull, A, o), Bp = __shfl_up_sync(kFull, B, o);
+      if (lane >= o) { B = max(Bp + A, B); A = Ap + A; }
+    }
+    int32_t Ae = __shfl_up_sync(kFull, A, 1), Be = __shfl_up_sync(kFull, B, 1);
+    if (lane == 0) { Ae = 0; Be = kNeg; }
+    const int32_t tb = max(E.t + Ae, Be);           // cursor before the event
+    int32_t issue = 0, v = INT_MIN;
+    if (in && dp) {
+      issue = max(tb + wcost, ready);
+      v = issue + rec.y;
+    }
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t vp = __shfl_up_sync(kFull, v, o);
+      if (lane >= o) v = max(v, vp);
+    }
+    const int32_t retire = max(E.lastret, v);       // in-order retirement
+    // publish this chunk's semaphore increments
+    const bool prod = in && dp && srec.x >= 0;
+    if (prod) a.hist[S.semhb[srec.x] + (int64_t)srec.y * gj + (srec.z - 1)] = retire;
+    __syncwarp();                                    // orders the warp's history writes
+    const unsigned pm = __ballot_sync(kFull, prod);
+    if (prod) {
+      const unsigned peers = __match_any_sync(pm, srec.x);
+      if (lane == 31 - __clz(peers)) st_release(S.sem + srec.x, srec.y * gj + srec.z);
+    }
+    const unsigned dm = __ballot_sync(kFull, in && dp);
+    if (in && dp) {
+      const uint32_t nj = E.n + __popc(dm & lanemask_le());
+      chk += inst_term(issue, retire, (uint32_t)w, nj);
+      if (TL) {
+        const int64_t o = __ldg(a.inst_off + rec.x) + gj;
+        a.issue[o] = issue;
+        a.retire[o] = retire;
+      }
+    }
+    E.n += __popc(dm);
+    // advance to the event after lane cut-1
+    E.t = __shfl_sync(kFull, max(E.t + A, B), cut - 1);
+    E.lastret = __shfl_sync(kFull, retire, cut - 1);
+    if (periodic) {
+      const int32_t off = (E.ptr - E.pbeg) + cut;
+      const int32_t it = off / period;
+      E.g += it;
+      E.ptr = E.pbeg + (off - it * period);
+    } else {
+      E.ptr += cut;
+    }
+    moved = true;
+  }
+  return moved;
+}
 
-    const bool active = lane < pi.ne;
-    Lane L;
-    L.cur = pi.loop_base; L.g = 0; L.g_end = 1; L.sp = 0;
-    L.ptr = active ? __ldg(a.op_ptr + pi.le_base + lane) : 0;
-    L.pend = active ? __ldg(a.op_ptr + pi.le_base + lane + 1) : 0;
-    L.t = 0; L.lastret = 0; L.arrival = 0; L.n = 0; L.chk = 0; L.bar_passed = false;
-    int state = active ? ST_RUN : ST_DONE;
-    // every round moves at least one event or releases a barrier, so events
-    // plus barriers bound the rounds; exceeding it would be a defect (status 8)
+template <int MODE, bool BB, bool TL>
+__global__ void k_simulate(const SimArgs a) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int W = a.warps;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  Smem S;
+  {
+    unsigned char* p = smem_raw;
+    S.semhb = reinterpret_cast<int64_t*>(p); p += 8 * a.sem_cap;
+    S.w_chk = reinterpret_cast<unsigned long long*>(p); p += 8 * W;
+    S.frames = reinterpret_cast<Frame*>(p); p += sizeof(Frame) * W * a.frame_depth;
+    S.sem = reinterpret_cast<int32_t*>(p); p += 4 * a.sem_cap;
+    S.w_moved = reinterpret_cast<int32_t*>(p); p += 4 * W;
+    S.w_state = reinterpret_cast<int32_t*>(p); p += 4 * W;
+    S.w_arrival = reinterpret_cast<int32_t*>(p); p += 4 * W;
+    S.w_ms = reinterpret_cast<int32_t*>(p); p += 4 * W;
+    S.slot = reinterpret_cast<int32_t*>(p);   // 4 ints
+  }
+  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+
+  for (;;) {
+    __syncthreads();
+    if (threadIdx.x == 0) *S.slot = atomicAdd(a.next_slot, 1);
+    __syncthreads();
+    const int slot = *S.slot;
+    if (slot >= a.n_programs) break;
+    const int p = __ldg(a.order + slot);
+    const ProgInfo pi = a.prog[p];
+    if (time_bound<BB>(pi, a.prm, cwait) > 2147483647ull) {
+      if (threadIdx.x == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
+      continue;
+    }
+    for (int i = threadIdx.x; i < pi.nsem[MODE]; i += blockDim.x) {
+      S.sem[i] = 0;
+      S.semhb[i] = __ldg(a.semhb + pi.semhb_off[MODE] + i);
+    }
+    if (threadIdx.x == 0) { S.slot[1] = 0; S.slot[2] = 0; S.slot[3] = 0; }
+    const bool live = w < pi.ne;
+    Eng E;
+    E.sp = 0; E.g = 0; E.g_end = 1;
+    E.t = 0; E.lastret = 0; E.bar_gen = 0; E.n = 0;
+    E.state = live ? ST_RUN : ST_DONE;
+    E.bar_passed = false;
+    E.row = 0; E.pbeg = 0; E.rend = 0; E.loops = false; E.ptr = 0;
+    if (live) {
+      set_row<MODE, BB, TL>(a, E, pi.le_base + w);
+      E.ptr = E.pbeg;
+    }
+    unsigned long long chk = 0;
+    // every round moves an event or releases a barrier
     const long long guard = pi.n_inst + 4ll * (pi.n_stmt + pi.n_iter) * (pi.ne + 1) + 64;
     long long rounds = 0;
-    int result = SYNC_PROG_OK;
-    for (;;) {
+    int verdict = -1;
+    const long long started = clock64();
+    __syncthreads();
+    while (verdict < 0) {
       bool moved = false;
-      if (state == ST_RUN) {
-        for (int b = 0; b < kBurst; ++b) {
-          const int r = step<MODE, BB, TL>(a, pi, L, stk, sem, lane, iter_cost, cwait);
-          if (r == R_MOVED) { moved = true; continue; }
-          if (r == R_BARRIER) { state = ST_BAR; moved = true; }
-          else if (r == R_DONE) { state = ST_DONE; moved = true; }
-          break;
-        }
+      if (E.state != ST_DONE) moved = run_engine<MODE, BB, TL>(a, S, E, w, lane, pi.ne, chk);
+      if (lane == 0) {
+        S.w_moved[w] = moved;
+        S.w_state[w] = E.state;
       }
-      __syncwarp();
-      const unsigned any_moved = __ballot_sync(0xffffffffu, moved);
-      const unsigned at_bar = __ballot_sync(0xffffffffu, state == ST_BAR);
-      const unsigned running = __ballot_sync(0xffffffffu, state == ST_RUN);
-      const unsigned lanes = pi.ne >= 32 ? 0xffffffffu : ((1u << pi.ne) - 1u);
-      if (++rounds > guard) { result = SYNC_PROG_ROUND_GUARD; break; }
-      if (BB && at_bar == lanes) {             // every engine drained: release
-        const int32_t rel = (int32_t)__reduce_max_sync(0xffffffffu, (unsigned)(state == ST_BAR ? L.arrival : 0)) +
-                            a.prm.c_barrier;
-        if (state == ST_BAR) { L.t = rel; state = ST_RUN; L.bar_passed = true; }
-        continue;
+      __syncthreads();
+      bool any_moved = false;
+      int n_live = 0;
+      for (int i = 0; i < pi.ne; ++i) {
+        any_moved |= S.w_moved[i] != 0;
+        n_live += S.w_state[i] != ST_DONE;
       }
-      if (running == 0 && at_bar == 0) break;  // all engines done
-      if (any_moved == 0) { result = SYNC_PROG_DEADLOCK; break; }
+      // a barrier released after its waiters stopped polling is progress too
+      const bool released = BB && S.slot[2] != E.bar_gen && E.state == ST_BAR;
+      const bool any_released = __syncthreads_or(released) != 0;
+      // the watchdog reads thread 0's clock so that every thread agrees
+      if (threadIdx.x == 0) S.w_ms[0] = clock64() - started > kWatchdogCycles;
+      __syncthreads();
+      if (++rounds > guard || S.w_ms[0]) verdict = SYNC_PROG_ROUND_GUARD;
+      else if (n_live == 0) verdict = SYNC_PROG_OK;
+      else if (!any_moved && !any_released) verdict = SYNC_PROG_DEADLOCK;
+      __syncthreads();
     }
-    int32_t ms = active ? max(L.t, L.lastret) : 0;
-    ms = (int32_t)__reduce_max_sync(0xffffffffu, (unsigned)ms);
-    unsigned long long chk = active ? L.chk : 0ull;
-    for (int o = 16; o > 0; o >>= 1) chk += __shfl_xor_sync(0xffffffffu, chk, o);
+    for (int o = 16; o > 0; o >>= 1) chk += __shfl_xor_sync(kFull, chk, o);
     if (lane == 0) {
-      const bool ok = result == SYNC_PROG_OK;
-      a.makespan[p] = ok ? ms : -1;
-      a.checksum[p] = ok ? chk : 0ull;
-      a.status[p] = result;
+      S.w_chk[w] = live ? chk : 0ull;
+      S.w_ms[w] = live ? max(E.t, E.lastret) : 0;
     }
-    __syncwarp();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned long long ck = 0;
+      int32_t ms = 0;
+      for (int i = 0; i < pi.ne; ++i) { ck += S.w_chk[i]; ms = max(ms, S.w_ms[i]); }
+      const bool ok = verdict == SYNC_PROG_OK;
+      a.makespan[p] = ok ? ms : -1;
+      a.checksum[p] = ok ? ck : 0ull;
+      a.status[p] = verdict;
+    }
   }
 }
 
 template <int MODE, bool BB>
-cudaError_t launch3(const SimArgs& a, int grid, size_t smem, cudaStream_t s) {
-  cudaError_t e;
-  if (a.issue) {
-    e = cudaFuncSetAttribute(k_simulate<MODE, BB, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+cudaError_t launch3(const SimArgs& a, size_t smem, int num_sms, cudaStream_t s) {
+  auto run = [&](auto kern) -> cudaError_t {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_simulate<MODE, BB, true><<<grid, kWarps * 32, smem, s>>>(a);
-  } else {
-    e = cudaFuncSetAttribute(k_simulate<MODE, BB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const int threads = 32 * a.warps;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
     if (e != cudaSuccess) return e;
-    k_simulate<MODE, BB, false><<<grid, kWarps * 32, smem, s>>>(a);
-  }
-  return cudaGetLastError();
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const long long cap = (long long)num_sms * per_sm;
+    const int grid = (int)(a.n_programs < cap ? a.n_programs : cap);
+    e = cudaMemsetAsync(a.next_slot, 0, sizeof(int32_t), s);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, threads, smem, s>>>(a);
+    return cudaGetLastError();
+  };
+  if (a.issue) return run(k_simulate<MODE, BB, true>);
+  return run(k_simulate<MODE, BB, false>);
 }
 
 }  // namespace
 
-size_t simulate_smem_per_warp(int sem_ints, int frame_depth, int ne_max) {
-  return (size_t)(sem_ints + ne_max * frame_depth * 4) * sizeof(int32_t);
+size_t simulate_smem_bytes(int warps, int sem_cap, int frame_depth) {
+  return (size_t)12 * sem_cap + (size_t)8 * warps + sizeof(Frame) * (size_t)warps * frame_depth +
+         (size_t)16 * warps + 16;
 }
 
 cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStream_t s) {
   if (a.n_programs == 0) return cudaSuccess;
-  const size_t smem = kWarps * simulate_smem_per_warp(a.sem_ints, a.frame_depth, a.ne_max);
-  const long long want = ((long long)a.n_programs + kWarps - 1) / kWarps;
-  // 16 resident CTAs (64 warps) per SM at most; programs beyond that are
-  // picked up grid-stride in descending-work order
-  const long long cap = (long long)num_sms * 16;
-  const int grid = (int)(want < cap ? want : cap);
+  const size_t smem = simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth);
   if (a.mode == SYNC_THR_PERLOOP)
-    return barrier ? launch3<SYNC_THR_PERLOOP, true>(a, grid, smem, s)
-                   : launch3<SYNC_THR_PERLOOP, false>(a, grid, smem, s);
-  return barrier ? launch3<SYNC_THR_COUNT, true>(a, grid, smem, s)
-                 : launch3<SYNC_THR_COUNT, false>(a, grid, smem, s);
+    return barrier ? launch3<SYNC_THR_PERLOOP, true>(a, smem, num_sms, s)
+                   : launch3<SYNC_THR_PERLOOP, false>(a, smem, num_sms, s);
+  return barrier ? launch3<SYNC_THR_COUNT, true>(a, smem, num_sms, s)
+                 : launch3<SYNC_THR_COUNT, false>(a, smem, num_sms, s);
 }
 
 }  // namespace syncgb

@@ -152,10 +152,12 @@ def simulate(batch, thr_count, params, barrier, cwait):
                 n += 1
                 _, _, iss, ret = state(e, i)
                 tl[(v[1], v[2])] = (iss, ret)
-                term = (((iss & 0xFFFFFFFF) * 0x9E3779B97F4A7C15) & MASK64) ^ \
-                       (((ret & 0xFFFFFFFF) * 0xC2B2AE3D27D4EB4F) & MASK64) ^ \
-                       ((n * 0x165667B19E3779F9 + e) & MASK64)
-                chk = (chk + term) & MASK64
+                M = 0xFFFFFFFF
+                a = (((iss & M) ^ ((n * 0x9E3779B9 + e) & M)) * 0x85EBCA6B) & M
+                a ^= a >> 13
+                b = (((ret & M) ^ ((n * 0xC2B2AE35 + e) & M)) * 0x27D4EB2F) & M
+                b ^= b >> 15
+                chk = (chk + ((a << 32) | b)) & MASK64
         return makespan, chk, tl
     finally:
         sys.setrecursionlimit(old)
