@@ -74,6 +74,15 @@ struct sync_programs {
   int64_t n_ops = 0;
   int32_t* hist = nullptr;          // scratch: retire time of each semaphore increment
   int32_t* next_slot = nullptr;     // scratch: simulator's program-slot counter
+  int32_t* fallback = nullptr;      // scratch: programs handed to the per-engine kernel
+  // program-order sweep
+  int32_t* plan_ptr = nullptr;
+  int4* plan = nullptr;
+  int4* chunk = nullptr;
+  int4* lrec = nullptr;
+  int4* lmeta = nullptr;
+  int4* lsem = nullptr;             // [2][n_lanes]
+  int64_t n_lanes = 0;
   int32_t nsem_max[2] = {0, 0};
   int32_t ne_max = 1;
   int32_t depth_max = 0;
@@ -131,6 +140,29 @@ struct ProgScratch {
   std::vector<int64_t> total, keys;
 };
 
+// Appends one sweep chunk: lanes `recs` (program-local instructions, already
+// engine-major) with their iteration copies.
+void add_chunk(const sync_batch_desc& d, int32_t x0, const ProgScratch& S, const std::vector<int32_t>& recs,
+               const std::vector<int32_t>& copies, int32_t ncopies, std::vector<int4>& chunks,
+               std::vector<int4>& lrec, std::vector<int4>& lmeta, std::vector<int4> (&lsem)[2]) {
+  const int32_t base = (int32_t)lrec.size();
+  const int32_t n = (int32_t)recs.size();
+  int32_t emask = 0;
+  for (int32_t i = 0; i < n; ++i) {
+    const int32_t x = recs[i];
+    const int32_t e = d.instr_engine[x0 + x];
+    emask |= 1 << e;
+    int32_t head = i;
+    while (head > 0 && d.instr_engine[x0 + recs[head - 1]] == e) --head;
+    const bool last = i + 1 == n || d.instr_engine[x0 + recs[i + 1]] != e;
+    const bool first_in_copy = copies[i] > 0 && (i == head || copies[i - 1] != copies[i]);
+    lrec.push_back(make_int4(x0 + x, d.instr_latency[x0 + x], S.x_ndeps[x], S.x_dep_begin[x]));
+    lmeta.push_back(make_int4(e, copies[i], head, (first_in_copy ? LANE_ITER_START : 0) | (last ? LANE_RUN_LAST : 0)));
+    for (int m = 0; m < 2; ++m) lsem[m].push_back(make_int4(S.x_own[m][x], S.x_hstride[m][x], S.x_koff[m][x], 0));
+  }
+  chunks.push_back(make_int4(base, n, ncopies, emask));
+}
+
 std::string where(int32_t p, const char* what, int64_t i) {
   return "program " + std::to_string(p) + ", " + what + " " + std::to_string(i);
 }
@@ -171,6 +203,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<int4> ops, opsem[2];
   std::vector<int64_t> inst_off(NX), dseg(ND), semhb;
   std::vector<int32_t> dsem[2] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
+  std::vector<int32_t> plan_ptr;
+  std::vector<int4> plan, chunks, lrec, lmeta, lsem[2];
   std::vector<int64_t> seg(ND + 1, 0);
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
@@ -267,6 +301,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     ProgInfo& pi = prog[p];
     std::memset(&pi, 0, sizeof pi);
     pi.ne = ne;
+    pi.loop_base = l0;
     pi.le_base = (int32_t)op_ptr.size();
     __int128 agg = 0;
     for (int32_t x = 0; x < nx; ++x) {
@@ -426,6 +461,48 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
           opstop[r] = next;
         }
       }
+    // program-order sweep plan: per loop, its body cut at child loops into
+    // straight-line segments, each segment in chunks of <= 32 engine-sorted lanes
+    for (int32_t l = 0; l < nl; ++l) {
+      plan_ptr.push_back((int32_t)plan.size());
+      std::vector<int32_t> seg;
+      int32_t nseg = 0, nloops = 0;
+      for (int32_t i = S.body_ptr[l]; i <= S.body_ptr[l + 1]; ++i) {
+        const bool at_end = i == S.body_ptr[l + 1];
+        const int32_t it = at_end ? -1 : S.body[i];
+        if (!at_end && it >= 0) { seg.push_back(it); continue; }
+        if (!seg.empty()) {
+          ++nseg;
+          const int32_t first_chunk = (int32_t)chunks.size();
+          for (size_t b = 0; b < seg.size(); b += 32) {
+            std::vector<int32_t> piece(seg.begin() + b, seg.begin() + std::min(seg.size(), b + 32));
+            std::stable_sort(piece.begin(), piece.end(), [&](int32_t u, int32_t v) {
+              return d.instr_engine[x0 + u] < d.instr_engine[x0 + v];
+            });
+            std::vector<int32_t> copy0(piece.size(), 0);
+            add_chunk(d, x0, S, piece, copy0, 1, chunks, lrec, lmeta, lsem);
+          }
+          plan.push_back(make_int4(ITEM_SEG, first_chunk, (int32_t)chunks.size() - first_chunk, -1));
+          seg.clear();
+        }
+        if (!at_end) {
+          ++nloops;
+          plan.push_back(make_int4(ITEM_LOOP, l0 + (-it - 1), 0, 0));
+        }
+      }
+      // a short body with no child loop: a template of several iterations
+      const int32_t L = S.body_ptr[l + 1] - S.body_ptr[l];
+      if (nloops == 0 && nseg == 1 && L >= 1 && L <= 16) {
+        const int32_t k = 32 / L;
+        std::vector<int32_t> recs, copies;
+        for (int32_t e = 0; e < ne; ++e)
+          for (int32_t c = 0; c < k; ++c)
+            for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i)
+              if (d.instr_engine[x0 + S.body[i]] == e) { recs.push_back(S.body[i]); copies.push_back(c); }
+        plan.back().w = (int32_t)chunks.size();
+        add_chunk(d, x0, S, recs, copies, k, chunks, lrec, lmeta, lsem);
+      }
+    }
     h.nsem_max[0] = std::max(h.nsem_max[0], pi.nsem[0]);
     h.nsem_max[1] = std::max(h.nsem_max[1], pi.nsem[1]);
     h.ne_max = std::max(h.ne_max, ne);
@@ -433,6 +510,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     if ((int64_t)ops.size() > kI32Max) raise(SYNC_ERR_OVERFLOW, "op records exceed INT32_MAX entries");
   }
   op_ptr.push_back((int32_t)ops.size());
+  plan_ptr.push_back((int32_t)plan.size());
   seg[ND] = n_pairs_padded;
 
   // trip prefix sums (rowptr) per loop: [0, t0, t0+t1, ...]
@@ -526,6 +604,18 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.inst_off = h.upload(inst_off, stream, "instance offsets");
   h.hist = h.alloc<int32_t>(std::max(hist_len[0], hist_len[1]), "semaphore history");
   h.next_slot = h.alloc<int32_t>(1, "program-slot counter");
+  h.fallback = h.alloc<int32_t>((int64_t)P + 1, "fallback list");
+  h.plan_ptr = h.upload(plan_ptr, stream, "sweep plan offsets");
+  h.plan = h.upload(plan, stream, "sweep plan");
+  h.chunk = h.upload(chunks, stream, "sweep chunks");
+  h.lrec = h.upload(lrec, stream, "sweep lanes");
+  h.lmeta = h.upload(lmeta, stream, "sweep lane meta");
+  {
+    std::vector<int4> both(lsem[0]);
+    both.insert(both.end(), lsem[1].begin(), lsem[1].end());
+    h.lsem = h.upload(both, stream, "sweep lane semaphores");
+  }
+  h.n_lanes = (int64_t)lrec.size();
   cuda_check(launch_expand(h.loop, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
   cuda_check(cudaStreamSynchronize(stream), "load");
 }
@@ -645,10 +735,25 @@ sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int3
     a.sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
     a.frame_depth = std::max(1, h->depth_max);
     a.warps = h->ne_max;
-    if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024)
+    if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024 ||
+        sweep_smem_bytes(a.sem_cap, a.frame_depth) > 200 * 1024)
       raise(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
-    cuda_check(launch_simulate(a, variant == SYNC_SIM_BARRIER, h->num_sms, static_cast<cudaStream_t>(stream)),
-               "simulator kernel");
+    SweepArgs w;
+    std::memset(&w, 0, sizeof w);
+    w.prog = h->prog; w.order = h->order; w.loop = h->loop; w.rowptr = h->rowptr;
+    w.plan_ptr = h->plan_ptr; w.plan = h->plan; w.chunk = h->chunk;
+    w.lrec = h->lrec; w.lmeta = h->lmeta; w.lsem = h->lsem + (size_t)mode * h->n_lanes;
+    w.dseg = h->dseg; w.dsem = a.dsem; w.semhb = h->semhb; w.inst_off = h->inst_off;
+    w.thr = d_thr; w.hist = h->hist; w.next_slot = h->next_slot; w.fallback = h->fallback;
+    w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
+    w.issue = d_issue; w.retire = d_retire;
+    w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
+    w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const bool barrier = variant == SYNC_SIM_BARRIER;
+    cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");
+    a.only = h->fallback;
+    cuda_check(launch_simulate(a, barrier, h->num_sms, st), "per-engine simulator kernel");
     return SYNC_OK;
   } catch (const Failure& f) {
     return report(f);

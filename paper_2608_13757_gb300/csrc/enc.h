@@ -60,7 +60,27 @@ struct alignas(16) ProgInfo {
                       // loop l, engine e) = le_base + l*ne + e
   int32_t nsem[2];    // waited semaphores, per threshold mode
   int32_t semhb_off[2];  // first entry of the program's history bases, per mode
+  int32_t loop_base;  // global id of the program's top-level loop
+  int32_t pad_[3];
 };
+
+// Program-order sweep tables.  Per loop, a plan: its body cut at child loops
+// into straight-line segments; items [plan_ptr[l], plan_ptr[l+1]):
+//   {ITEM_SEG, first chunk, chunks, multi-iteration chunk or -1}
+//   {ITEM_LOOP, child loop (global id), 0, 0}
+// A chunk holds up to 32 datapath records of one segment (all engines), in
+// lanes ordered engine-major (then iteration copy, then body position):
+//   chunk {first lane record, lanes, iteration copies, engine bitmask}
+// A multi-iteration chunk repeats a short innermost segment for `copies`
+// consecutive iterations (barrier-free sweep only).  Per lane:
+//   lrec {x (global instruction), latency, dependencies, first dependency}
+//   lmeta {engine, copy, first lane of the engine's run, flags}
+//     flags bit 0: first record of its engine in a copy >= 1 (an iteration
+//     start precedes it); bit 1: last lane of its engine's run
+//   lsem per mode {semaphore, stride, koff, 0} as the simulator's records.
+enum : int32_t { ITEM_SEG = 0, ITEM_LOOP = 1 };
+constexpr int32_t LANE_ITER_START = 1;
+constexpr int32_t LANE_RUN_LAST = 2;
 
 // Simulator op records, one list ("row") per (loop, engine): the engine's own
 // instructions and every child loop of the loop's body, in body order, then
@@ -129,6 +149,38 @@ struct SimArgs {
   int32_t warps;             // warps per CTA (largest engine count of the batch)
   int32_t sem_cap;           // semaphore slots in shared memory
   int32_t frame_depth;       // frames per warp
+  const int32_t* only;       // if set: [0] count, [1..] the program ids to simulate
+};
+
+struct SweepArgs {
+  const ProgInfo* prog;
+  const int32_t* order;
+  const LoopInfo* loop;
+  const int32_t* rowptr;
+  const int32_t* plan_ptr;   // [n_loops + 1]
+  const int4* plan;
+  const int4* chunk;
+  const int4* lrec;
+  const int4* lmeta;
+  const int4* lsem;          // per-mode records, parallel to lrec
+  const int64_t* dseg;
+  const int32_t* dsem;       // per-mode, parallel to dseg
+  const int64_t* semhb;
+  const int64_t* inst_off;
+  const int32_t* thr;
+  int32_t* hist;
+  int32_t* next_slot;        // scratch: program slot counter (zeroed per launch)
+  int32_t* fallback;         // scratch: [0] count, [1..] programs for the fallback kernel
+  int32_t* makespan;
+  unsigned long long* checksum;
+  int32_t* status;
+  int32_t* issue;
+  int32_t* retire;
+  sync_sim_params prm;
+  int32_t n_programs;
+  int32_t mode;
+  int32_t sem_cap;
+  int32_t frame_depth;
 };
 
 // Launchers (return the launch error, if any).
@@ -139,6 +191,11 @@ cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const 
 cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s);
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStream_t s);
+// The sweep simulates every program it can; programs whose waits reach
+// forward in program order are listed in a.fallback and then simulated by
+// the per-engine kernel (launch_simulate with SimArgs::only set).
+cudaError_t launch_sweep(const SweepArgs& a, bool barrier, int num_sms, cudaStream_t s);
+size_t sweep_smem_bytes(int sem_cap, int frame_depth);
 size_t simulate_smem_bytes(int warps, int sem_cap, int frame_depth);
 
 }  // namespace syncgb

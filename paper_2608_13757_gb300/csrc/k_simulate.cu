@@ -369,8 +369,9 @@ __global__ void k_simulate(const SimArgs a) {
     if (threadIdx.x == 0) *S.slot = atomicAdd(a.next_slot, 1);
     __syncthreads();
     const int slot = *S.slot;
-    if (slot >= a.n_programs) break;
-    const int p = __ldg(a.order + slot);
+    const int limit = a.only ? *(volatile const int32_t*)a.only : a.n_programs;
+    if (slot >= limit) break;
+    const int p = a.only ? a.only[1 + slot] : __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
     if (time_bound<BB>(pi, a.prm, cwait) > 2147483647ull) {
       if (threadIdx.x == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
