@@ -50,7 +50,7 @@ def parse():
     ap.add_argument("--config", default="chain")
     ap.add_argument("--programs", type=int, default=None, help="programs per rank")
     ap.add_argument("--mode", choices=("perloop", "count"), default="perloop")
-    ap.add_argument("--cpu-sample", type=int, default=8192,
+    ap.add_argument("--cpu-sample", type=int, default=32768,
                     help="programs of the workload the CPU oracle baseline runs")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -139,8 +139,8 @@ def run_gpu(args, rank, world, local_rank):
 
     torch.cuda.set_device(local_rank)
     mode = sg.THR_PERLOOP if args.mode == "perloop" else sg.THR_COUNT
-    P = args.programs or workloads.CONFIGS[args.config][1]
-    batch = workloads.generate(args.config, n_programs=P, first_program=rank * P)
+    first, P = shard(rank, args.programs or workloads.CONFIGS[args.config][1])
+    batch = workloads.generate(args.config, n_programs=P, first_program=first)
     t0 = time.perf_counter()
     h = sg.sync_load_programs(batch, device=local_rank)
     load_s = time.perf_counter() - t0
@@ -224,6 +224,24 @@ def run_e2e(args, sg, batch, mode, prm, dev, P):
         h.close()
         del thr
     return {"s": statistics.median(times), "h2d": int(h2d), "d2h": int(d2h)}
+
+
+def shard(rank: int, programs_per_rank: int):
+    """Program ids of a rank: rank*P .. rank*P+P-1 (weak scaling, no overlap)."""
+    return rank * programs_per_rank, programs_per_rank
+
+
+def reduce_over_ranks(ms: float, e2e_s, pairs: int, device):
+    """(max step time, max end-to-end time, total pairs) over the ranks of the
+    default process group; the only cross-rank traffic of a run."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms, e2e_s or 0.0, float(pairs)], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    sm = t.clone()
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return mx[0].item(), (mx[1].item() or None), sm[2].item()
 
 
 def dist_barrier(world):
@@ -360,14 +378,7 @@ def main():
     pairs = res["sizes"].n_pairs
     e2e_s = res["e2e"]["s"] if "e2e" in res else None
     if world > 1:
-        import torch
-        import torch.distributed as dist
-        t = torch.tensor([ms, e2e_s or 0.0, float(pairs)], dtype=torch.float64, device="cuda")
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = t.clone()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        ms, e2e_s, total_pairs = mx[0].item(), mx[1].item() or None, sm[2].item()
+        ms, e2e_s, total_pairs = reduce_over_ranks(ms, e2e_s, pairs, "cuda")
     else:
         total_pairs = float(pairs)
     if rank != 0:
@@ -389,7 +400,9 @@ def main():
                    "parallelism": f"programs sharded over {world} GPU(s)"},
         "roofline": roof,
         "kernels": kernels,
-        "gpu_launches": 4 * args.steps,
+        # per step: thresholds, check, and per schedule the sweep plus the
+        # per-engine kernel for programs it hands over
+        "gpu_launches": 6 * args.steps,
         "results_minimal_and_deadlock_free": res["ok"],
         "load_s": res["load_s"],
         "clocks": clk or None,
