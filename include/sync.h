@@ -219,6 +219,39 @@ sync_status sync_simulate(const sync_programs *h, sync_thr_mode mode, const int3
                           int32_t *d_makespan, unsigned long long *d_checksum, int32_t *d_status,
                           int32_t *d_issue, int32_t *d_retire, void *stream);
 
+/* Size of the device scratch used by sync_simulate_noalloc (see below). */
+#define SYNC_NOALLOC_SCRATCH_BYTES (64u << 20)
+
+/* sync_simulate without any device allocation during the call.
+ *
+ * The paper has no counterpart; this entry point exists for callers of this
+ * library that cannot call cudaMalloc or cudaFree around a simulation: for
+ * example a host thread that must not trigger the implicit device-wide
+ * synchronisation an allocation may cause, or a process whose device memory
+ * is fully reserved up front by its own allocator.  The handle must already
+ * be loaded; the outputs are caller-owned as for sync_simulate, and the
+ * results are identical to sync_simulate's.
+ *
+ * Instead of the handle's scratch, the call uses one scratch array of
+ * SYNC_NOALLOC_SCRATCH_BYTES that the library declares statically in device
+ * memory: every GPU that loads the library holds it until the process exits.
+ * It must hold the semaphore history of the batch (one int32 per increment
+ * of every waited semaphore), a program list and two counters; a batch that
+ * does not fit returns SYNC_ERR_ARG with the required size in
+ * sync_last_error(), before anything is launched.  The call zeroes the
+ * counters it needs on `stream`; the history is written before it is read.
+ *
+ * The first call on a device looks up the array's device address (with that
+ * device current); make that first call before any stream capture.  All
+ * calls share the one array and it keeps the last call's contents, so calls
+ * whose work overlaps on the GPU (other streams, other threads) race with
+ * each other: serialise them, e.g. on one stream. */
+sync_status sync_simulate_noalloc(const sync_programs *h, sync_thr_mode mode, const int32_t *d_thr,
+                                  const sync_sim_params *params, sync_sim_variant variant,
+                                  int32_t *d_makespan, unsigned long long *d_checksum,
+                                  int32_t *d_status, int32_t *d_issue, int32_t *d_retire,
+                                  void *stream);
+
 /* Releases a handle (NULL is ignored).  Waits for the device to finish work
  * that may still use the handle's memory. */
 void sync_free_programs(sync_programs *h);

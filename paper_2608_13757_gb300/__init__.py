@@ -29,7 +29,9 @@ PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD = 0, 4, 7, 8
 
 # every symbol include/sync.h declares
 EXPORTS = ("sync_load_programs", "sync_query", "sync_pair_offsets", "sync_eval_thresholds",
-           "sync_check_minimal", "sync_simulate", "sync_free_programs", "sync_last_error")
+           "sync_check_minimal", "sync_simulate", "sync_simulate_noalloc", "sync_free_programs",
+           "sync_last_error")
+NOALLOC_SCRATCH_BYTES = 64 << 20
 
 
 class SyncError(RuntimeError):
@@ -80,6 +82,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sync_check_minimal.argtypes = [vp, ctypes.c_int, vp, vp, vp, vp]
     lib.sync_simulate.argtypes = [vp, ctypes.c_int, vp, P(SimParams), ctypes.c_int, vp, vp, vp,
                                   vp, vp, vp]
+    lib.sync_simulate_noalloc.argtypes = lib.sync_simulate.argtypes
     lib.sync_free_programs.argtypes = [vp]
     lib.sync_free_programs.restype = None
     lib.sync_last_error.argtypes = []
@@ -235,6 +238,33 @@ def sync_simulate(h: Programs, mode, thr, params: SimParams | None = None,
     _check(lib().sync_simulate(h.handle, int(mode), _ptr(thr), ctypes.byref(prm), int(variant),
                               _ptr(out.makespan), _ptr(out.checksum), _ptr(out.status),
                               _ptr(out.issue), _ptr(out.retire), _stream(stream)))
+    return out
+
+
+def sync_simulate_noalloc(h: Programs, mode, thr, params: SimParams | None = None,
+                          variant: int = SIM_BARRIER_FREE, out: SimOutputs | None = None,
+                          timeline: bool = False, stream=None) -> SimOutputs:
+    """sync_simulate for callers that cannot allocate device memory around a
+    simulation: the call allocates nothing and uses the library's static
+    scratch (NOALLOC_SCRATCH_BYTES per GPU).  Pass preallocated outputs in
+    `out` to keep the whole call free of allocations; without `out` this
+    wrapper allocates the output tensors itself (the library call does not).
+    Calls share the scratch, so calls that overlap on the GPU race."""
+    import torch
+    dev = f"cuda:{h.device}"
+    P = h.sizes.n_programs
+    if out is None:
+        out = SimOutputs(torch.empty(max(P, 1), dtype=torch.int32, device=dev),
+                         torch.empty(max(P, 1), dtype=torch.int64, device=dev),
+                         torch.empty(max(P, 1), dtype=torch.int32, device=dev))
+        if timeline:
+            n = max(h.sizes.n_instances, 1)
+            out.issue = torch.full((n,), -1, dtype=torch.int32, device=dev)
+            out.retire = torch.full((n,), -1, dtype=torch.int32, device=dev)
+    prm = params if params is not None else SimParams()
+    _check(lib().sync_simulate_noalloc(h.handle, int(mode), _ptr(thr), ctypes.byref(prm), int(variant),
+                                       _ptr(out.makespan), _ptr(out.checksum), _ptr(out.status),
+                                       _ptr(out.issue), _ptr(out.retire), _stream(stream)))
     return out
 
 

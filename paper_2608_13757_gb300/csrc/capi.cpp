@@ -9,6 +9,7 @@
 #include <vector>
 
 #include "enc.h"
+#include "handle.h"
 
 using namespace syncgb;
 
@@ -37,87 +38,23 @@ sync_status report(const Failure& f) {
   return f.status;
 }
 
+}  // namespace
+
+namespace syncgb {
+sync_status set_error(sync_status status, const std::string& msg) {
+  g_err = msg;
+  return status;
+}
+void cuda_or_raise(cudaError_t e, const char* what) { cuda_check(e, what); }
+}  // namespace syncgb
+
+namespace {
+
 constexpr int64_t kI32Max = 2147483647;
 
 int64_t pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
 }  // namespace
-
-struct sync_programs {
-  int device = 0;
-  int num_sms = 0;
-  sync_sizes sz{};
-  std::vector<int64_t> seg_host;
-  std::vector<int32_t> count_host;
-  std::vector<void*> blocks;
-  // threshold / checker encoding
-  LoopInfo* loop = nullptr;
-  int32_t* rowptr = nullptr;
-  int32_t* pidx = nullptr;
-  DepInfo* dep = nullptr;
-  int64_t* seg = nullptr;
-  int32_t* tile_first = nullptr;
-  int64_t* path = nullptr;
-  int64_t n_chunks = 0;
-  // simulator encoding
-  ProgInfo* prog = nullptr;
-  int32_t* order = nullptr;
-  int32_t* op_ptr = nullptr;
-  int2* rowinfo = nullptr;
-  int4* ops = nullptr;
-  int32_t* opstop = nullptr;
-  int4* opsem = nullptr;            // [2][n_ops]
-  int64_t* dseg = nullptr;
-  int32_t* dsem = nullptr;          // [2][n_deps]
-  int64_t* semhb = nullptr;
-  int64_t* inst_off = nullptr;
-  int64_t n_ops = 0;
-  int32_t* hist = nullptr;          // scratch: retire time of each semaphore increment
-  int32_t* next_slot = nullptr;     // scratch: simulator's program-slot counter
-  int32_t* fallback = nullptr;      // scratch: programs handed to the per-engine kernel
-  // program-order sweep
-  int32_t* plan_ptr = nullptr;
-  int4* plan = nullptr;
-  int4* chunk = nullptr;
-  int4* lrec = nullptr;
-  int4* lmeta = nullptr;
-  int4* lsem = nullptr;             // [2][n_lanes]
-  int64_t n_lanes = 0;
-  int32_t nsem_max[2] = {0, 0};
-  int32_t ne_max = 1;
-  int32_t depth_max = 0;
-
-  ~sync_programs() {
-    if (blocks.empty()) return;
-    int prev = 0;
-    cudaGetDevice(&prev);
-    cudaSetDevice(device);
-    cudaDeviceSynchronize();
-    for (void* p : blocks) cudaFree(p);
-    cudaSetDevice(prev);
-  }
-
-  template <class T>
-  T* upload(const std::vector<T>& v, cudaStream_t s, const char* what) {
-    const size_t bytes = std::max<size_t>(v.size(), 1) * sizeof(T);
-    void* p = nullptr;
-    cuda_check(cudaMalloc(&p, bytes), what);
-    blocks.push_back(p);
-    sz.device_bytes += (int64_t)bytes;
-    if (!v.empty()) cuda_check(cudaMemcpyAsync(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice, s), what);
-    sz.h2d_bytes += (int64_t)(v.size() * sizeof(T));
-    return static_cast<T*>(p);
-  }
-  template <class T>
-  T* alloc(int64_t n, const char* what) {
-    const size_t bytes = (size_t)std::max<int64_t>(n, 1) * sizeof(T);
-    void* p = nullptr;
-    cuda_check(cudaMalloc(&p, bytes), what);
-    blocks.push_back(p);
-    sz.device_bytes += (int64_t)bytes;
-    return static_cast<T*>(p);
-  }
-};
 
 namespace {
 
@@ -603,6 +540,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.semhb = h.upload(semhb, stream, "semaphore history bases");
   h.inst_off = h.upload(inst_off, stream, "instance offsets");
   h.hist = h.alloc<int32_t>(std::max(hist_len[0], hist_len[1]), "semaphore history");
+  h.hist_len[0] = hist_len[0];
+  h.hist_len[1] = hist_len[1];
   h.next_slot = h.alloc<int32_t>(1, "program-slot counter");
   h.fallback = h.alloc<int32_t>((int64_t)P + 1, "fallback list");
   h.plan_ptr = h.upload(plan_ptr, stream, "sweep plan offsets");
