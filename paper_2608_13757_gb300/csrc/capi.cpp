@@ -304,6 +304,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       for (int32_t l = Pl; l != Sl; l = par[l]) reads_rowptr[l0 + l] = 1;
       path.push_back(loop[l0 + Sl].pidx_off);
       path.push_back(loop[l0 + Sl].rowptr_off);
+      D.s_pidx = loop[l0 + Sl].pidx_off;
+      D.s_rowptr = loop[l0 + Sl].rowptr_off;
       {
         const size_t at = path.size();
         for (int32_t l = Pl; l != Sl; l = par[l]) path.push_back(loop[l0 + l].rowptr_off);

@@ -41,6 +41,8 @@ struct alignas(16) LoopInfo {
 struct alignas(16) DepInfo {
   int64_t seg_off;    // pair-layout offset of this dependency's segment
   int64_t path;
+  int64_t s_pidx;     // S's pidx and rowptr offsets (= path entries up, up+1)
+  int64_t s_rowptr;
   int32_t total;      // consumer instances (= total of the consumer's loop)
   int32_t up;
   int32_t clen;

@@ -3,9 +3,18 @@
 // A pair is (dependency d, consumer instance g), g the global iteration index
 // of the consumer's loop.  Pairs are laid out dependency-major with every
 // segment padded to a multiple of 4, so each thread owns one int4 chunk that
-// never straddles two dependencies.  Both kernels are HBM-streaming: 4 bytes
-// per pair written (thresholds) or read (checker), plus the loop-structure
-// reads, which consecutive pairs of one dependency share through L1/L2.
+// never straddles two dependencies; consecutive threads own consecutive
+// chunks, so a warp's store or load is 512 contiguous bytes.  Both kernels
+// are HBM-streaming: 4 bytes per pair written (thresholds) or read
+// (checker), plus the loop-structure reads, which consecutive pairs of one
+// dependency share through L1/L2.
+//
+// Both results depend on g only through g_S, the enclosing iteration of the
+// dependency's common loop S, and the start of g_S's trip of S (Eq. 1, and
+// Sec. 5.1's registers r_S and r-hat_S).  A chunk's four consumer iterations
+// usually share g_S (consumer nested below S) or the trip (consumer directly
+// in S), so the chunk looks them up for its first and last iteration and
+// evaluates once per distinct g_S.
 #include "enc.h"
 
 namespace syncgb {
@@ -26,18 +35,22 @@ __device__ __forceinline__ int find_dep(const ThrArgs& a, int64_t q) {
   return lo;
 }
 
-// Global iteration of S that encloses the consumer's global iteration g:
-// follow the expanded parent indices up `up` levels.
-__device__ __forceinline__ int32_t up_to_S(const ThrArgs& a, const DepInfo& D, int32_t g) {
-  for (int i = 0; i < D.up; ++i) g = __ldg(a.pidx + __ldg(a.path + D.path + i) + g);
-  return g;
+// Global iterations of S enclosing the consumer's global iterations ga and
+// gb: both walked up the expanded parent indices together, `up` levels.
+__device__ __forceinline__ void up_to_S(const ThrArgs& a, const DepInfo& D, int32_t& ga, int32_t& gb) {
+  for (int i = 0; i < D.up; ++i) {
+    const int32_t* p = a.pidx + __ldg(a.path + D.path + i);
+    ga = __ldg(p + ga);
+    gb = __ldg(p + gb);
+  }
 }
 
-// Global index of the first iteration of S in the trip that holds gs.
-__device__ __forceinline__ int32_t trip_start(const ThrArgs& a, const DepInfo& D, int32_t gs) {
-  const int64_t pidx_S = __ldg(a.path + D.path + D.up);
-  const int64_t rowptr_S = __ldg(a.path + D.path + D.up + 1);
-  return __ldg(a.rowptr + rowptr_S + __ldg(a.pidx + pidx_S + gs));
+// First global iteration of S in the trip that holds gs, and (in `end`) the
+// first one after it.
+__device__ __forceinline__ int32_t trip_of(const ThrArgs& a, const DepInfo& D, int32_t gs, int32_t& end) {
+  const int32_t* rp = a.rowptr + D.s_rowptr + __ldg(a.pidx + D.s_pidx + gs);
+  end = __ldg(rp + 1);
+  return __ldg(rp);
 }
 
 // Iterations of P that start inside the first x iterations of S (x may equal
@@ -53,16 +66,14 @@ __device__ __forceinline__ int32_t encode(const DepInfo& D, int32_t c, int mode)
 }
 
 // The paper's register form (Sec. 5.1-5.3): r_S = gs + 1 and r-hat_S = gs -
-// trip_start + 1 are the monotone and trip registers of S at the consumer's
+// start + 1 are the monotone and trip registers of S at the consumer's
 // issue; mask = isGT(r-hat_S, k) (Eq. 2); expr = r_S - k when the producer
 // sits in S, otherwise r_P, the producer loop's monotone register, which
 // counts P's iterations through the current S-iteration (forward) or through
 // the previous one (backward, consumer ahead of P in S's body).
-__device__ __forceinline__ int32_t wait_value(const ThrArgs& a, const DepInfo& D, int32_t g,
-                                              int mode) {
-  const int32_t gs = up_to_S(a, D, g);
-  const int32_t rhat = gs - trip_start(a, D, gs) + 1;
-  if (rhat <= D.k) return 0;
+__device__ __forceinline__ int32_t wait_value(const ThrArgs& a, const DepInfo& D, int32_t gs,
+                                              int32_t start, int mode) {
+  if (gs - start + 1 <= D.k) return 0;
   int32_t expr;
   if (D.kase == CASE_PS) expr = gs + 1 - D.k;
   else expr = count_down(a, D, D.kase == CASE_NEST_FWD ? gs + 1 : gs);
@@ -74,29 +85,75 @@ __device__ __forceinline__ int32_t wait_value(const ThrArgs& a, const DepInfo& D
 // consumer's, all >= 1), no wait on underflow, else the producer instances
 // in every S-iteration up to and including the target (lexicographic order
 // of iteration vectors = global iteration order of S).
-__device__ __forceinline__ int32_t minimum(const ThrArgs& a, const DepInfo& D, int32_t g,
-                                           int mode) {
-  const int32_t gs = up_to_S(a, D, g);
-  const int32_t start = trip_start(a, D, gs);
+__device__ __forceinline__ int32_t minimum(const ThrArgs& a, const DepInfo& D, int32_t gs,
+                                           int32_t start, int mode) {
   const int32_t tS = gs - start + 1 - D.k;
   if (tS <= 0) return 0;
   const int32_t gt = start + tS - 1;
   return encode(D, count_down(a, D, gt + 1), mode);
 }
 
+// Values of the chunk's pairs g0 .. g0+3 (entries at or past `total` are
+// padding and get 0).
+template <bool CHECK>
+__device__ __forceinline__ int32_t eval_at(const ThrArgs& a, const DepInfo& D, int32_t gs, int32_t start,
+                                           int mode) {
+  return CHECK ? minimum(a, D, gs, start, mode) : wait_value(a, D, gs, start, mode);
+}
+
+template <bool CHECK>
+__device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D, int32_t g0, int mode) {
+  const int32_t n = D.total - g0 < kChunk ? D.total - g0 : kChunk;   // >= 1
+  int32_t v[kChunk] = {0, 0, 0, 0};
+  if (D.up == 0) {
+    // consumer directly in S: g_S = g; one trip lookup unless the chunk
+    // crosses into the next trip
+    int32_t end;
+    int32_t start = trip_of(a, D, g0, end);
+#pragma unroll
+    for (int i = 0; i < kChunk; ++i) {
+      if (i < n) {
+        const int32_t g = g0 + i;
+        if (g >= end) start = trip_of(a, D, g, end);
+        v[i] = eval_at<CHECK>(a, D, g, start, mode);
+      }
+    }
+  } else {
+    // consumer nested below S: one value per distinct g_S; the first and
+    // last iteration's g_S decide whether the chunk stays in one
+    int32_t gs = g0, gl = g0 + n - 1;
+    up_to_S(a, D, gs, gl);
+    int32_t end;
+    int32_t val = eval_at<CHECK>(a, D, gs, trip_of(a, D, gs, end), mode);
+    v[0] = val;
+    if (gl == gs) {
+#pragma unroll
+      for (int i = 1; i < kChunk; ++i) v[i] = i < n ? val : 0;
+    } else {
+#pragma unroll
+      for (int i = 1; i < kChunk; ++i) {
+        if (i < n) {
+          int32_t gi = g0 + i;
+          for (int l = 0; l < D.up; ++l) gi = __ldg(a.pidx + __ldg(a.path + D.path + l) + gi);
+          if (gi != gs) {
+            gs = gi;
+            val = eval_at<CHECK>(a, D, gs, trip_of(a, D, gs, end), mode);
+          }
+          v[i] = val;
+        }
+      }
+    }
+  }
+  return make_int4(v[0], v[1], v[2], v[3]);
+}
+
 template <int MODE>
-__global__ void __launch_bounds__(kThreads) k_thresholds(const ThrArgs a, int32_t* __restrict__ thr) {
+__global__ void __launch_bounds__(kThreads, 4) k_thresholds(const ThrArgs a, int32_t* __restrict__ thr) {
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.n_chunks; c += stride) {
     const int64_t q = c * kChunk;
     const DepInfo D = a.dep[find_dep(a, q)];
-    const int32_t g0 = (int32_t)(q - D.seg_off);
-    int4 v;
-    v.x = g0 + 0 < D.total ? wait_value(a, D, g0 + 0, MODE) : 0;
-    v.y = g0 + 1 < D.total ? wait_value(a, D, g0 + 1, MODE) : 0;
-    v.z = g0 + 2 < D.total ? wait_value(a, D, g0 + 2, MODE) : 0;
-    v.w = g0 + 3 < D.total ? wait_value(a, D, g0 + 3, MODE) : 0;
-    __stcs(reinterpret_cast<int4*>(thr + q), v);
+    __stcs(reinterpret_cast<int4*>(thr + q), chunk_values<false>(a, D, (int32_t)(q - D.seg_off), MODE));
   }
 }
 
@@ -109,18 +166,20 @@ __device__ __forceinline__ void tally(int32_t got, int32_t want, int64_t idx,
 }
 
 template <int MODE>
-__global__ void __launch_bounds__(kThreads) k_check(const CheckArgs a) {
+__global__ void __launch_bounds__(kThreads, 4) k_check(const CheckArgs a) {
   unsigned long long unsafe = 0, over = 0, first = ~0ull;
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.t.n_chunks; c += stride) {
     const int64_t q = c * kChunk;
+    const int4 v = __ldcs(reinterpret_cast<const int4*>(a.thr + q));
     const DepInfo D = a.t.dep[find_dep(a.t, q)];
     const int32_t g0 = (int32_t)(q - D.seg_off);
-    const int4 v = __ldcs(reinterpret_cast<const int4*>(a.thr + q));
-    if (g0 + 0 < D.total) tally(v.x, minimum(a.t, D, g0 + 0, MODE), q + 0, unsafe, over, first);
-    if (g0 + 1 < D.total) tally(v.y, minimum(a.t, D, g0 + 1, MODE), q + 1, unsafe, over, first);
-    if (g0 + 2 < D.total) tally(v.z, minimum(a.t, D, g0 + 2, MODE), q + 2, unsafe, over, first);
-    if (g0 + 3 < D.total) tally(v.w, minimum(a.t, D, g0 + 3, MODE), q + 3, unsafe, over, first);
+    const int4 m = chunk_values<true>(a.t, D, g0, MODE);
+    // padding entries are not pairs: the checker reads only the first n
+    tally(v.x, m.x, q + 0, unsafe, over, first);
+    if (g0 + 1 < D.total) tally(v.y, m.y, q + 1, unsafe, over, first);
+    if (g0 + 2 < D.total) tally(v.z, m.z, q + 2, unsafe, over, first);
+    if (g0 + 3 < D.total) tally(v.w, m.w, q + 3, unsafe, over, first);
   }
   for (int o = 16; o > 0; o >>= 1) {
     unsafe += __shfl_xor_sync(0xffffffffu, unsafe, o);
@@ -135,31 +194,46 @@ __global__ void __launch_bounds__(kThreads) k_check(const CheckArgs a) {
   }
 }
 
-int grid_for(int64_t n_chunks, int num_sms) {
-  // 8 resident 256-thread CTAs per SM; grid-stride beyond that.
+// Resident CTAs of `kern` on every SM, capped by the work; grid-stride
+// beyond that.
+template <class K>
+cudaError_t grid_for(K kern, int64_t n_chunks, int num_sms, int& grid) {
+  int per_sm = 0;
+  const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
+  if (e != cudaSuccess) return e;
+  if (per_sm < 1) per_sm = 1;
   const int64_t want = (n_chunks + kThreads - 1) / kThreads;
-  const int64_t cap = (int64_t)num_sms * 8;
-  return (int)(want < cap ? (want > 0 ? want : 1) : cap);
+  const int64_t cap = (int64_t)num_sms * per_sm;
+  grid = (int)(want < cap ? (want > 0 ? want : 1) : cap);
+  return cudaSuccess;
 }
 
 }  // namespace
 
 cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s) {
   if (a.n_chunks == 0) return cudaSuccess;
-  const int grid = grid_for(a.n_chunks, num_sms);
-  if (a.mode == SYNC_THR_PERLOOP) k_thresholds<SYNC_THR_PERLOOP><<<grid, kThreads, 0, s>>>(a, thr);
-  else k_thresholds<SYNC_THR_COUNT><<<grid, kThreads, 0, s>>>(a, thr);
-  return cudaGetLastError();
+  auto run = [&](auto kern) -> cudaError_t {
+    int grid = 0;
+    const cudaError_t e = grid_for(kern, a.n_chunks, num_sms, grid);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kThreads, 0, s>>>(a, thr);
+    return cudaGetLastError();
+  };
+  return a.mode == SYNC_THR_PERLOOP ? run(k_thresholds<SYNC_THR_PERLOOP>) : run(k_thresholds<SYNC_THR_COUNT>);
 }
 
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(a.counts, 0, 2 * sizeof(unsigned long long), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(a.first_bad, 0xff, sizeof(unsigned long long), s);
   if (e != cudaSuccess || a.t.n_chunks == 0) return e;
-  const int grid = grid_for(a.t.n_chunks, num_sms);
-  if (a.t.mode == SYNC_THR_PERLOOP) k_check<SYNC_THR_PERLOOP><<<grid, kThreads, 0, s>>>(a);
-  else k_check<SYNC_THR_COUNT><<<grid, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  auto run = [&](auto kern) -> cudaError_t {
+    int grid = 0;
+    const cudaError_t e2 = grid_for(kern, a.t.n_chunks, num_sms, grid);
+    if (e2 != cudaSuccess) return e2;
+    kern<<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+  };
+  return a.t.mode == SYNC_THR_PERLOOP ? run(k_check<SYNC_THR_PERLOOP>) : run(k_check<SYNC_THR_COUNT>);
 }
 
 }  // namespace syncgb
