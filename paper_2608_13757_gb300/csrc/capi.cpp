@@ -676,8 +676,8 @@ sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int3
     a.sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
     a.frame_depth = std::max(1, h->depth_max);
     a.warps = h->ne_max;
-    if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024 ||
-        sweep_smem_bytes(a.sem_cap, a.frame_depth) > 200 * 1024)
+    const int ring = sweep_ring_for(a.sem_cap, a.frame_depth, 200 * 1024);
+    if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024 || ring == 0)
       raise(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
     SweepArgs w;
     std::memset(&w, 0, sizeof w);
@@ -689,7 +689,7 @@ sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int3
     w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
     w.issue = d_issue; w.retire = d_retire;
     w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
-    w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth;
+    w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const bool barrier = variant == SYNC_SIM_BARRIER;
     cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");

@@ -183,6 +183,7 @@ struct SweepArgs {
   int32_t mode;
   int32_t sem_cap;
   int32_t frame_depth;
+  int32_t ring;              // latest increments kept per semaphore (power of two)
 };
 
 // Launchers (return the launch error, if any).
@@ -197,7 +198,10 @@ cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStr
 // forward in program order are listed in a.fallback and then simulated by
 // the per-engine kernel (launch_simulate with SimArgs::only set).
 cudaError_t launch_sweep(const SweepArgs& a, bool barrier, int num_sms, cudaStream_t s);
-size_t sweep_smem_bytes(int sem_cap, int frame_depth);
+size_t sweep_smem_bytes(int sem_cap, int frame_depth, int ring);
+// Largest ring (32, 16, ..., 1) whose sweep shared memory fits in `limit`
+// bytes, or 0 if none does.
+int sweep_ring_for(int sem_cap, int frame_depth, size_t limit);
 size_t simulate_smem_bytes(int warps, int sem_cap, int frame_depth);
 
 }  // namespace syncgb

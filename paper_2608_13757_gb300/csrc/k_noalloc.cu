@@ -77,8 +77,8 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
                                    " (use sync_simulate)");
   const int32_t sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
   const int32_t frame_depth = std::max(1, h->depth_max);
-  if (simulate_smem_bytes(h->ne_max, sem_cap, frame_depth) > 200 * 1024 ||
-      sweep_smem_bytes(sem_cap, frame_depth) > 200 * 1024)
+  const int ring = sweep_ring_for(sem_cap, frame_depth, 200 * 1024);
+  if (simulate_smem_bytes(h->ne_max, sem_cap, frame_depth) > 200 * 1024 || ring == 0)
     return set_error(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
   sync_status st = cuda_error(cudaSetDevice(h->device), "cudaSetDevice");
   if (st != SYNC_OK) return st;
@@ -99,7 +99,7 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
   w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
   w.issue = d_issue; w.retire = d_retire;
   w.prm = q; w.n_programs = h->sz.n_programs; w.mode = mode;
-  w.sem_cap = sem_cap; w.frame_depth = frame_depth;
+  w.sem_cap = sem_cap; w.frame_depth = frame_depth; w.ring = ring;
   st = cuda_error(launch_sweep(w, barrier, h->num_sms, s), "sweep simulator kernel");
   if (st != SYNC_OK) return st;
   SimArgs a;

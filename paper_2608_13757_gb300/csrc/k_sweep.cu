@@ -7,22 +7,27 @@
 // records (more chunks if longer), or -- barrier-free, for a short innermost
 // body -- as several consecutive iterations at once.  The chunk's lanes are
 // ordered engine-major, so each engine's events form a run of lanes:
-//   - an engine's cursor obeys t' = max(t + A, B) per event (A its costs,
-//     B the time its waits are satisfied plus the issue interval), maps that
-//     compose associatively, so a segmented 5-step warp scan gives every
-//     event the cursor before it; issue = max(cursor + wait ops, ready) and
-//     in-order retirement is a segmented max-scan of issue + latency;
+//   - an engine's cursor obeys t' = max(t + A, B) per event (A its costs
+//     and the issue interval, B the time its waits are satisfied plus the
+//     issue interval), maps that compose associatively, so a segmented
+//     5-step warp scan gives every event its cursor after issue, t' = issue
+//     + ii; in-order retirement is a segmented max-scan of issue + latency;
 //   - a wait on a semaphore whose threshold increment happened in an earlier
-//     chunk reads its retire time from the history array; an increment inside
-//     the chunk is the k-th lane of the semaphore's lanes (increments come in
-//     lane order), and these in-chunk waits are solved by repeating the scans
-//     until no time changes (a least fixed point of the max-plus system;
-//     times only grow, a cycle never settles and is a deadlock);
+//     chunk reads its retire time from a ring of the semaphore's latest
+//     increments (up to 32) in shared memory, or from the history array if older; an
+//     increment inside the chunk is the k-th lane of the semaphore's lanes
+//     (increments come in lane order), and these in-chunk waits are solved by
+//     repeating the scans until no producer retires after its consumer's
+//     issue (a least fixed point of the max-plus system; times only grow, a
+//     cycle never settles and is a deadlock);
 //   - a threshold beyond every increment up to this chunk points forward in
 //     program order: the program is handed to the per-engine kernel.
-// Barriers (barrier scheme) are a warp maximum of the engines' drained times.
-// Per-engine cursor, last retire and instance count live in shared memory,
-// read by the engine's lanes and written back by the last lane of its run.
+// A loop whose body is one chunk runs all its iterations in a tight loop
+// with the lanes' records in registers and the next iteration's thresholds
+// in flight.  Barriers (barrier scheme) are a warp maximum of the engines'
+// drained times.  Per-engine cursor, last retire and instance count live in
+// shared memory, read by the engine's lanes and written back by the last
+// lane of its run.
 #include "enc.h"
 
 namespace syncgb {
@@ -30,6 +35,8 @@ namespace {
 
 constexpr int kWarps = 8;                   // programs (warps) per CTA
 constexpr int kMaxIntra = 4;                // in-chunk waits per lane before falling back
+constexpr int kMaxDeps = 2;                 // dependencies per lane held in registers
+constexpr int kRingMax = 32;                // most recent increments kept per semaphore
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int32_t kNeg = -1;                // -infinity of the cursor maps (cursors, costs >= 0)
 constexpr int SIM_FALLBACK = 9;             // internal: handed to the per-engine kernel
@@ -37,8 +44,8 @@ constexpr int SIM_FALLBACK = 9;             // internal: handed to the per-engin
 struct Frame { int32_t loop, item, g, g_end; };
 
 // Shared memory of one warp (program), 16-byte aligned.
-__host__ __device__ __forceinline__ size_t warp_bytes(int sem_cap, int frame_depth) {
-  const size_t per = (size_t)20 * sem_cap + sizeof(Frame) * (size_t)frame_depth + 3 * 4 * 32;
+__host__ __device__ __forceinline__ size_t warp_bytes(int sem_cap, int frame_depth, int ring) {
+  const size_t per = (size_t)(20 + 4 * ring + 32) * sem_cap + sizeof(Frame) * (size_t)frame_depth + 3 * 4 * 32;
   return (per + 15) & ~(size_t)15;
 }
 
@@ -54,12 +61,6 @@ __device__ __forceinline__ unsigned lanemask_le() {
   asm("mov.u32 %0, %%lanemask_le;" : "=r"(m));
   return m;
 }
-// Lane of the k-th (1-based) set bit of m.
-__device__ __forceinline__ int kth_bit(unsigned m, int k) {
-  for (int i = 1; i < k; ++i) m &= m - 1;
-  return __ffs(m) - 1;
-}
-
 __device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t retire, uint32_t e,
                                                         uint32_t n) {
   uint32_t x = ((uint32_t)issue ^ (n * 0x9E3779B9u + e)) * 0x85EBCA6Bu;
@@ -94,60 +95,115 @@ struct WarpSmem {
   int64_t* semhb;      // [cap] history base
   uint32_t* grp;       // [cap] lanes of the current chunk that increment it
   int32_t* tag;        // [cap] chunk that wrote grp
+  int32_t* ring;       // [cap][ring] retire times of the latest increments
+  uint8_t* rank_lane;  // [cap][32] lane of the chunk's k-th increment (k from 0)
+  int32_t rmask;       // ring - 1
   Frame* frames;       // [depth]
 };
 
-// One chunk: `copies` iterations (g .. g+copies-1) of a segment's records.
-// Returns 0, SYNC_PROG_DEADLOCK or SIM_FALLBACK.
-template <int MODE, bool BB, bool TL>
-__device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, int32_t g,
-                                         int32_t copies, int32_t ctag, int lane,
-                                         unsigned long long& chk) {
-  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
-  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
-  const bool have = lane < ch.y;
-  int4 rec = make_int4(0, 0, 0, 0), meta = make_int4(0, 0, lane, 0), sr = make_int4(-1, 0, 0, 0);
-  if (have) {
-    rec = __ldg(a.lrec + ch.x + lane);
-    meta = __ldg(a.lmeta + ch.x + lane);
-    sr = __ldg(a.lsem + ch.x + lane);
-  }
-  const bool valid = have && meta.y < copies;
-  const int32_t e = meta.x, head = meta.z;
-  const int32_t gl = g + meta.y;
-  const int32_t t_in = S.t[e], lr_in = S.lr[e], n_in = S.nn[e];
+// One lane's record of a chunk, with its first kMaxDeps dependencies.
+struct LaneRec {
+  int4 rec;                      // {global instruction, latency, dependencies, first dependency}
+  int4 meta;                     // {engine, copy, first lane of the engine's run, flags}
+  int4 sr;                       // {semaphore it increments or -1, stride, koff, 0}
+  const int32_t* tp[kMaxDeps];   // threshold segment of dependency j
+  int32_t sm[kMaxDeps];          // semaphore dependency j waits on
+};
 
-  // semaphores incremented in this chunk: lanes in order of their increments
-  const bool prod = valid && sr.x >= 0;
+__device__ __forceinline__ void load_lane(const SweepArgs& a, const int4 ch, int lane, LaneRec& L) {
+  L.rec = make_int4(0, 0, 0, 0);
+  L.meta = make_int4(0, 0, lane, 0);
+  L.sr = make_int4(-1, 0, 0, 0);
+  if (lane < ch.y) {
+    L.rec = __ldg(a.lrec + ch.x + lane);
+    L.meta = __ldg(a.lmeta + ch.x + lane);
+    L.sr = __ldg(a.lsem + ch.x + lane);
+  }
+#pragma unroll
+  for (int j = 0; j < kMaxDeps; ++j) {
+    L.tp[j] = a.thr;
+    L.sm[j] = 0;
+    if (j < L.rec.z) {
+      L.tp[j] = a.thr + __ldg(a.dseg + L.rec.w + j);
+      L.sm[j] = __ldg(a.dsem + L.rec.w + j);
+    }
+  }
+}
+
+// Thresholds of the lane's first kMaxDeps dependencies at its iteration gl.
+__device__ __forceinline__ void load_thr(const LaneRec& L, bool valid, int32_t gl, int32_t (&T)[kMaxDeps]) {
+#pragma unroll
+  for (int j = 0; j < kMaxDeps; ++j) T[j] = (valid && j < L.rec.z) ? __ldg(L.tp[j] + gl) : 0;
+}
+
+// Lanes that increment each semaphore in this chunk (`copies` iterations
+// valid), published under tag ctag.
+__device__ __forceinline__ void set_groups(const WarpSmem& S, const LaneRec& L, int lane, bool have,
+                                           int32_t copies, int32_t ctag) {
+  const bool prod = have && L.meta.y < copies && L.sr.x >= 0;
   const unsigned pm = __ballot_sync(kFull, prod);
-  int32_t pub_own = 0;
   if (prod) {
-    const unsigned peers = __match_any_sync(pm, sr.x);
-    pub_own = S.semv[sr.x];
-    if (lane == __ffs(peers) - 1) { S.grp[sr.x] = peers; S.tag[sr.x] = ctag; }
+    const unsigned peers = __match_any_sync(pm, L.sr.x);
+    if (lane == __ffs(peers) - 1) { S.grp[L.sr.x] = peers; S.tag[L.sr.x] = ctag; }
+    unsigned lt;
+    asm("mov.u32 %0, %%lanemask_lt;" : "=r"(lt));
+    S.rank_lane[L.sr.x * 32 + __popc(peers & lt)] = (uint8_t)lane;
   }
   __syncwarp();
+}
 
-  // waits: earlier increments from the history, in-chunk ones by lane
+// One chunk: `copies` iterations (g .. g+copies-1) of a segment's records,
+// given the lane's record, its first thresholds T and the semaphore groups
+// of this chunk (set_groups with the same copies and ctag).  Returns 0,
+// SYNC_PROG_DEADLOCK or SIM_FALLBACK.
+template <int MODE, bool BB, bool TL>
+__device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, const LaneRec& L,
+                                         const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
+                                         int32_t ctag, int lane, unsigned long long& chk) {
+  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+  const int4 rec = L.rec, sr = L.sr;
+  const bool have = lane < ch.y;
+  const bool valid = have && L.meta.y < copies;
+  const int32_t e = L.meta.x, head = L.meta.z;
+  const int32_t gl = g + L.meta.y;
+  const int32_t t_in = S.t[e], lr_in = S.lr[e], n_in = S.nn[e];
+  const bool prod = valid && sr.x >= 0;
+  const int32_t pub_own = prod ? S.semv[sr.x] : 0;
+
+  // waits: increments before this chunk from the ring (or, if older, the
+  // history), increments inside it by lane
   int32_t known = kNeg;                        // satisfied before this chunk (kNeg: none)
   int intra[kMaxIntra];
   int n_intra = 0;
   bool fallback = false;
-  for (int j = 0; valid && j < rec.z; ++j) {
-    const int32_t T = __ldg(a.thr + __ldg(a.dseg + rec.w + j) + gl);
-    if (T <= 0) continue;
-    const int32_t s = __ldg(a.dsem + rec.w + j);
+  auto wait_on = [&](int32_t Tj, int32_t s) {
+    if (Tj <= 0 || fallback) return;
     const int32_t pub = S.semv[s];
-    if (T <= pub) { known = max(known, a.hist[S.semhb[s] + (T - 1)]); continue; }
+    if (Tj <= pub) {
+      const int32_t r = pub - Tj <= S.rmask ? S.ring[s * (S.rmask + 1) + ((Tj - 1) & S.rmask)]
+                                            : a.hist[S.semhb[s] + (Tj - 1)];
+      known = max(known, r);
+      return;
+    }
     const unsigned m = S.tag[s] == ctag ? S.grp[s] : 0u;
-    const int k = T - pub;
-    if (k > __popc(m) || n_intra == kMaxIntra) { fallback = true; break; }
-    intra[n_intra++] = kth_bit(m, k);
-  }
+    const int k = Tj - pub;
+    if (k > __popc(m) || n_intra == kMaxIntra) { fallback = true; return; }
+    const int src = S.rank_lane[s * 32 + k - 1];
+#pragma unroll
+    for (int i = 0; i < kMaxIntra; ++i)
+      if (i == n_intra) intra[i] = src;         // static indices: intra stays in registers
+    ++n_intra;
+  };
+#pragma unroll
+  for (int j = 0; j < kMaxDeps; ++j)
+    if (valid && j < rec.z) wait_on(T[j], L.sm[j]);
+  for (int j = kMaxDeps; valid && j < rec.z; ++j)
+    wait_on(__ldg(a.thr + __ldg(a.dseg + rec.w + j) + gl), __ldg(a.dsem + rec.w + j));
   if (__ballot_sync(kFull, fallback)) return SIM_FALLBACK;
 
   const int32_t wcost = BB ? 0 : rec.z * cwait;
-  const int32_t apre = (meta.w & LANE_ITER_START) ? iter_cost : 0;
+  const int32_t apre = (L.meta.w & LANE_ITER_START) ? iter_cost : 0;
   const int32_t A = valid ? apre + wcost + a.prm.ii : 0;
   int32_t r_intra = kNeg;                      // retire of in-chunk producers (lower bound)
   int32_t issue = 0, retire = 0, t_after = 0;
@@ -157,24 +213,26 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
   for (int pass = 0; pass < passes; ++pass) {
     const int32_t ready = max(known, r_intra);
     const int32_t B0 = (valid && ready >= 0) ? ready + a.prm.ii : kNeg;
-    // segmented inclusive scan of the cursor maps over the engine's run
+    // segmented inclusive scan of the cursor maps over the engine's run;
+    // t' = max(t + A, B) with B = ready + ii gives issue = t' - ii
     int32_t Ai = A, Bi = B0;
+#pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int32_t Ap = __shfl_up_sync(kFull, Ai, o), Bp = __shfl_up_sync(kFull, Bi, o);
       if (lane - o >= head) { Bi = max(Bp + Ai, Bi); Ai = Ap + Ai; }
     }
-    int32_t Ae = __shfl_up_sync(kFull, Ai, 1), Be = __shfl_up_sync(kFull, Bi, 1);
-    if (lane == head) { Ae = 0; Be = kNeg; }
-    const int32_t tb = max(t_in + Ae, Be);
     t_after = max(t_in + Ai, Bi);
-    issue = max(tb + apre + wcost, max(ready, 0));
+    issue = t_after - a.prm.ii;
     int32_t v = valid ? issue + rec.y : kNeg;
+#pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int32_t vp = __shfl_up_sync(kFull, v, o);
       if (lane - o >= head) v = max(v, vp);
     }
     retire = max(lr_in, v);
-    // new lower bound from the in-chunk producers' retire times
+    if (!any_intra) { settled = true; break; }
+    // new lower bound from the in-chunk producers' retire times; settled
+    // once it binds nowhere (no issue would move)
     int32_t nr = kNeg;
 #pragma unroll
     for (int i = 0; i < kMaxIntra; ++i) {
@@ -182,14 +240,16 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
       const int32_t rv = __shfl_sync(kFull, retire, src);
       if (i < n_intra) nr = max(nr, rv);
     }
-    if (!__ballot_sync(kFull, nr != r_intra)) { settled = true; break; }
+    if (!__ballot_sync(kFull, valid && nr > issue)) { settled = true; break; }
     r_intra = nr;
   }
   if (!settled) return SYNC_PROG_DEADLOCK;   // a cycle of waits inside the chunk
 
   // publish increments, instance counts, checksum terms, engine state
   if (prod) {
-    a.hist[S.semhb[sr.x] + (int64_t)sr.y * gl + (sr.z - 1)] = retire;
+    const int32_t n = sr.y * gl + sr.z;        // the increment this retirement makes
+    S.ring[sr.x * (S.rmask + 1) + ((n - 1) & S.rmask)] = retire;
+    a.hist[S.semhb[sr.x] + (n - 1)] = retire;
   }
   const unsigned vm = __ballot_sync(kFull, valid);
   const unsigned run_le = vm & lanemask_le() & ~((1u << head) - 1u);
@@ -203,26 +263,262 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
     }
   }
   __syncwarp();
-  if (prod && lane == 31 - __clz(__match_any_sync(pm, sr.x))) S.semv[sr.x] = pub_own + __popc(S.grp[sr.x]);
-  if (have && (meta.w & LANE_RUN_LAST)) {
+  if (prod) {
+    const unsigned grp = S.grp[sr.x];
+    if (lane == 31 - __clz(grp)) S.semv[sr.x] = pub_own + __popc(grp);
+  }
+  if (have && (L.meta.w & LANE_RUN_LAST)) {
     S.t[e] = t_after;
     S.lr[e] = retire;
     S.nn[e] = n_in + __popc(run_le);
   }
   __syncwarp();
   // engines without records here still pass the iteration starts between copies
-  if (copies > 1 && lane < 32 && !((ch.w >> lane) & 1)) S.t[lane] += (copies - 1) * iter_cost;
+  if (copies > 1 && !((ch.w >> lane) & 1)) S.t[lane] += (copies - 1) * iter_cost;
   __syncwarp();
   return 0;
 }
 
+// All engines: the drain-and-release barrier of the barrier scheme.
+__device__ __forceinline__ void barrier_all(const WarpSmem& S, int ne, int32_t c_barrier, int lane) {
+  int32_t arr = lane < ne ? max(S.t[lane], S.lr[lane]) : 0;
+  arr = (int32_t)__reduce_max_sync(kFull, (unsigned)arr);
+  __syncwarp();
+  if (lane < ne) S.t[lane] = arr + c_barrier;
+  __syncwarp();
+}
+
+// Iterations lo .. hi-1 of a loop whose body is one straight-line segment of
+// one chunk (or, barrier-free, one multi-iteration chunk) and whose lanes
+// wait on at most kMaxDeps semaphores each; the first iteration start has
+// been charged.  Everything the iterations pass on stays in registers: lane
+// e < ne holds engine e's cursor, last retire and instance count and hands
+// them to its engine's lanes by shuffle; every lane keeps its record, its
+// waited semaphores' increment counts and the next iteration's thresholds.
+// Returns 0, SYNC_PROG_DEADLOCK or SIM_FALLBACK (then the program is
+// abandoned, so nothing is written back).
 template <int MODE, bool BB, bool TL>
-__global__ void __launch_bounds__(kWarps * 32) k_sweep(const SweepArgs a) {
+__device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi,
+                                             const int4 ch, const LaneRec& L, int32_t lo, int32_t hi,
+                                             int32_t ctag, int lane, unsigned long long& chk) {
+  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+  const int32_t ii = a.prm.ii;
+  const int32_t copies = ch.z;
+  const bool have = lane < ch.y;
+  const int32_t e = L.meta.x, head = L.meta.z, copy = L.meta.y, lat = L.rec.y;
+  const int ndep = have ? L.rec.z : 0;
+  const unsigned run_from_head = ~((1u << head) - 1u);
+
+  // semaphore groups of the chunk and the increment counts so far
+  set_groups(S, L, lane, have, copies, ctag);
+  uint32_t wg0 = 0, wg1 = 0;
+  int32_t pub0 = 0, pub1 = 0;
+  const int32_t* ring0 = S.ring;
+  const int32_t* ring1 = S.ring;
+  int64_t hist0 = 0, hist1 = 0;                       // history offsets of increment 1 minus 1
+  if (ndep > 0) {
+    const int32_t s = L.sm[0];
+    wg0 = S.tag[s] == ctag ? S.grp[s] : 0u;
+    pub0 = S.semv[s];
+    ring0 = S.ring + s * (S.rmask + 1);
+    hist0 = S.semhb[s] - 1;
+  }
+  if (ndep > 1) {
+    const int32_t s = L.sm[kMaxDeps > 1 ? 1 : 0];
+    wg1 = S.tag[s] == ctag ? S.grp[s] : 0u;
+    pub1 = S.semv[s];
+    ring1 = S.ring + s * (S.rmask + 1);
+    hist1 = S.semhb[s] - 1;
+  }
+  const bool prod_lane = have && L.sr.x >= 0;
+  const uint32_t own_grp = prod_lane ? S.grp[L.sr.x] : 0u;
+  int32_t own_pub = prod_lane ? S.semv[L.sr.x] : 0;
+  int32_t* own_ring = S.ring + (prod_lane ? L.sr.x : 0) * (S.rmask + 1);
+  const int64_t own_hist = prod_lane ? S.semhb[L.sr.x] - 1 : 0;
+  const int32_t own_stride = L.sr.y, own_koff = L.sr.z;
+  int64_t tl_off = 0;
+  if (TL && have) tl_off = __ldg(a.inst_off + L.rec.x);
+
+  // state lanes: engine `lane`'s run in the chunk (if any)
+  const unsigned lastm = __ballot_sync(kFull, have && (L.meta.w & LANE_RUN_LAST));
+  const bool present = lane < pi.ne && ((ch.w >> lane) & 1);
+  int my_last = lane;
+  unsigned my_run = 0;
+  if (present) {
+    const int rank = __popc((unsigned)ch.w & ((1u << lane) - 1u));
+    my_last = (int)__fns(lastm, 0, rank + 1);
+    const int first = rank == 0 ? 0 : (int)__fns(lastm, 0, rank) + 1;
+    my_run = (my_last == 31 ? kFull : ((1u << (my_last + 1)) - 1u)) & ~((1u << first) - 1u);
+  }
+  int32_t ts = 0, lrs = 0, ns = 0;
+  if (lane < pi.ne) { ts = S.t[lane]; lrs = S.lr[lane]; ns = S.nn[lane]; }
+
+  const int32_t P = (BB ? 0 : L.rec.z * cwait) + ((L.meta.w & LANE_ITER_START) ? iter_cost : 0);
+  const int32_t A = P + ii;                           // cursor advance of a valid lane with no wait
+  int32_t T0n = 0, T1n = 0;
+  {
+    const bool vn = have && copy < hi - lo;
+    if (vn && ndep > 0) T0n = __ldg(L.tp[0] + lo + copy);
+    if (vn && ndep > 1) T1n = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + lo + copy);
+  }
+  for (int32_t g = lo; g < hi;) {
+    const int32_t v = min(copies, hi - g);
+    const int32_t T0 = T0n, T1 = T1n;
+    const int32_t gn = g + v;
+    const bool valid = have && copy < v;
+    if (gn < hi) {
+      const bool vn = have && copy < hi - gn;
+      if (vn && ndep > 0) T0n = __ldg(L.tp[0] + gn + copy);
+      if (vn && ndep > 1) T1n = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + gn + copy);
+    }
+    const unsigned vm = __ballot_sync(kFull, valid);
+    const int32_t gl = g + copy;
+    const int32_t t_in = __shfl_sync(kFull, ts, e), lr_in = __shfl_sync(kFull, lrs, e);
+    const int32_t n_in = __shfl_sync(kFull, ns, e);
+
+    // waits: earlier increments from the ring or history, in-chunk ones by lane
+    int32_t known = kNeg;
+    int src0 = -1, src1 = -1;
+    bool fallback = false;
+    if (valid && T0 > 0) {
+      if (T0 <= pub0) {
+        known = pub0 - T0 <= S.rmask ? ring0[(T0 - 1) & S.rmask] : a.hist[hist0 + T0];
+      } else {
+        const unsigned m = wg0 & vm;
+        const int k = T0 - pub0;
+        if (k > __popc(m)) fallback = true; else src0 = S.rank_lane[L.sm[0] * 32 + k - 1];
+      }
+    }
+    if (valid && T1 > 0) {
+      if (T1 <= pub1) {
+        known = max(known, pub1 - T1 <= S.rmask ? ring1[(T1 - 1) & S.rmask] : a.hist[hist1 + T1]);
+      } else {
+        const unsigned m = wg1 & vm;
+        const int k = T1 - pub1;
+        if (k > __popc(m)) fallback = true; else src1 = S.rank_lane[L.sm[kMaxDeps > 1 ? 1 : 0] * 32 + k - 1];
+      }
+    }
+    const unsigned intra = __ballot_sync(kFull, src0 >= 0 || src1 >= 0);
+    if (__ballot_sync(kFull, fallback)) return SIM_FALLBACK;
+
+    const int32_t Av = valid ? A : 0;
+    int32_t r_intra = kNeg;
+    int32_t issue = 0, retire = 0, t_after = 0;
+    const int passes = intra ? ch.y + 2 : 1;
+    bool settled = false;
+    for (int pass = 0; pass < passes; ++pass) {
+      const int32_t ready = max(known, r_intra);
+      // segmented scan of t' = max(t + A, B), B = ready + ii: issue = t' - ii
+      int32_t Ai = Av, Bi = (valid && ready >= 0) ? ready + ii : kNeg;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int32_t Ap = __shfl_up_sync(kFull, Ai, o), Bp = __shfl_up_sync(kFull, Bi, o);
+        if (lane - o >= head) { Bi = max(Bp + Ai, Bi); Ai += Ap; }
+      }
+      t_after = max(t_in + Ai, Bi);
+      issue = t_after - ii;
+      // in-order retirement: segmented max-scan of issue + latency
+      int32_t rv = valid ? issue + lat : kNeg;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int32_t vp = __shfl_up_sync(kFull, rv, o);
+        if (lane - o >= head) rv = max(rv, vp);
+      }
+      retire = max(lr_in, rv);
+      if (!intra) { settled = true; break; }
+      const int32_t p0 = __shfl_sync(kFull, retire, src0 < 0 ? lane : src0);
+      const int32_t p1 = __shfl_sync(kFull, retire, src1 < 0 ? lane : src1);
+      const int32_t nr = max(src0 < 0 ? kNeg : p0, src1 < 0 ? kNeg : p1);
+      if (!__ballot_sync(kFull, valid && nr > issue)) { settled = true; break; }   // binds nowhere
+      r_intra = nr;
+    }
+    if (!settled) return SYNC_PROG_DEADLOCK;
+
+    // publish
+    if (valid && prod_lane) {
+      const int32_t n = own_stride * gl + own_koff;
+      own_ring[(n - 1) & S.rmask] = retire;
+      a.hist[own_hist + n] = retire;
+    }
+    if (valid) {
+      const uint32_t nj = (uint32_t)n_in + __popc(vm & lanemask_le() & run_from_head);
+      chk += inst_term(issue, retire, (uint32_t)e, nj);
+      if (TL) {
+        a.issue[tl_off + gl] = issue;
+        a.retire[tl_off + gl] = retire;
+      }
+    }
+    pub0 += __popc(wg0 & vm);
+    pub1 += __popc(wg1 & vm);
+    own_pub += __popc(own_grp & vm);
+    const int32_t t_last = __shfl_sync(kFull, t_after, my_last), r_last = __shfl_sync(kFull, retire, my_last);
+    if (present) {
+      ts = t_last;
+      lrs = r_last;
+      ns += __popc(vm & my_run);
+    } else if (v > 1 && lane < pi.ne) {
+      ts += (v - 1) * iter_cost;                      // iteration starts between copies
+    }
+    __syncwarp();                                     // ring entries visible to the next iteration
+    g = gn;
+    if (BB) {
+      const int32_t arr = (int32_t)__reduce_max_sync(kFull, lane < pi.ne ? (unsigned)max(ts, lrs) : 0u);
+      if (lane < pi.ne) ts = arr + a.prm.c_barrier;
+    }
+    if (g < hi && lane < pi.ne) ts += iter_cost;
+  }
+  if (lane < pi.ne) { S.t[lane] = ts; S.lr[lane] = lrs; S.nn[lane] = ns; }
+  if (prod_lane && lane == 31 - __clz(own_grp)) S.semv[L.sr.x] = own_pub;
+  __syncwarp();
+  return 0;
+}
+
+// Iterations lo .. hi-1 of a loop whose body is one straight-line segment of
+// one chunk (or, barrier-free, one multi-iteration chunk); the first
+// iteration start has been charged.  The lane's record and thresholds stay
+// in registers; the next chunk's thresholds load while this one runs.
+template <int MODE, bool BB, bool TL>
+__device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi, const int4 ch,
+                                        int32_t lo, int32_t hi, int32_t ctag, int lane,
+                                        unsigned long long& chk) {
+  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+  const int32_t copies = ch.z;
+  const bool have = lane < ch.y;
+  LaneRec L;
+  load_lane(a, ch, lane, L);
+  if (!__ballot_sync(kFull, have && L.rec.z > kMaxDeps))
+    return run_loop_regs<MODE, BB, TL>(a, S, pi, ch, L, lo, hi, ctag, lane, chk);
+  set_groups(S, L, lane, have, min(copies, hi - lo), ctag);
+  int32_t Tn[kMaxDeps];
+  load_thr(L, have && L.meta.y < hi - lo, lo + L.meta.y, Tn);
+  for (int32_t g = lo; g < hi;) {
+    const int32_t v = min(copies, hi - g);
+    int32_t T[kMaxDeps];
+#pragma unroll
+    for (int j = 0; j < kMaxDeps; ++j) T[j] = Tn[j];
+    const int32_t gn = g + v;
+    if (gn < hi) load_thr(L, have && L.meta.y < hi - gn, gn + L.meta.y, Tn);
+    if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
+    const int verdict = run_chunk<MODE, BB, TL>(a, S, ch, L, T, g, v, ctag, lane, chk);
+    if (verdict) return verdict;
+    g = gn;
+    if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
+    if (g < hi) {
+      if (lane < pi.ne) S.t[lane] += iter_cost;
+      __syncwarp();
+    }
+  }
+  return 0;
+}
+
+template <int MODE, bool BB, bool TL>
+__global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   WarpSmem S;
   {
-    unsigned char* p = smem_raw + wib * warp_bytes(a.sem_cap, a.frame_depth);
+    unsigned char* p = smem_raw + wib * warp_bytes(a.sem_cap, a.frame_depth, a.ring);
     S.semhb = reinterpret_cast<int64_t*>(p); p += 8 * a.sem_cap;
     S.frames = reinterpret_cast<Frame*>(p); p += sizeof(Frame) * a.frame_depth;
     S.t = reinterpret_cast<int32_t*>(p); p += 4 * 32;
@@ -230,7 +526,10 @@ __global__ void __launch_bounds__(kWarps * 32) k_sweep(const SweepArgs a) {
     S.nn = reinterpret_cast<int32_t*>(p); p += 4 * 32;
     S.semv = reinterpret_cast<int32_t*>(p); p += 4 * a.sem_cap;
     S.grp = reinterpret_cast<uint32_t*>(p); p += 4 * a.sem_cap;
-    S.tag = reinterpret_cast<int32_t*>(p);
+    S.tag = reinterpret_cast<int32_t*>(p); p += 4 * a.sem_cap;
+    S.ring = reinterpret_cast<int32_t*>(p); p += 4 * (size_t)a.ring * a.sem_cap;
+    S.rank_lane = reinterpret_cast<uint8_t*>(p);
+    S.rmask = a.ring - 1;
   }
   const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
@@ -260,13 +559,7 @@ __global__ void __launch_bounds__(kWarps * 32) k_sweep(const SweepArgs a) {
     for (;;) {
       if (pbeg + item == pend) {                       // end of an iteration's body
         if (sp == 0) break;                            // the top-level loop runs once
-        if (BB) {                                      // all-engine barrier: drain, release
-          int32_t arr = lane < pi.ne ? max(S.t[lane], S.lr[lane]) : 0;
-          arr = (int32_t)__reduce_max_sync(kFull, (unsigned)arr);
-          __syncwarp();
-          if (lane < pi.ne) S.t[lane] = arr + a.prm.c_barrier;
-          __syncwarp();
-        }
+        if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
         if (++g < g_end) {
           if (lane < pi.ne) S.t[lane] += iter_cost;
           __syncwarp();
@@ -282,24 +575,34 @@ __global__ void __launch_bounds__(kWarps * 32) k_sweep(const SweepArgs a) {
       const int4 it = __ldg(a.plan + pbeg + item);
       if (it.x == ITEM_LOOP) {                         // a loop statement
         if (BB) {
-          int32_t arr = lane < pi.ne ? max(S.t[lane], S.lr[lane]) : 0;
-          arr = (int32_t)__reduce_max_sync(kFull, (unsigned)arr);
-          __syncwarp();
-          if (lane < pi.ne) S.t[lane] = arr + a.prm.c_barrier;
-        } else if (lane < pi.ne) {
-          S.t[lane] += a.prm.c_regop;
+          barrier_all(S, pi.ne, a.prm.c_barrier, lane);
+        } else {
+          if (lane < pi.ne) S.t[lane] += a.prm.c_regop;
         }
         const LoopInfo L = a.loop[it.y];
         const int32_t lo = __ldg(a.rowptr + L.rowptr_off + g), hi = __ldg(a.rowptr + L.rowptr_off + g + 1);
         ++item;
         if (lo < hi) {
+          const int32_t cb = __ldg(a.plan_ptr + it.y), ce = __ldg(a.plan_ptr + it.y + 1);
           __syncwarp();
+          if (lane < pi.ne) S.t[lane] += iter_cost;    // the first iteration starts
+          __syncwarp();
+          if (ce - cb == 1) {
+            const int4 body = __ldg(a.plan + cb);
+            const bool multi = !BB && body.w >= 0;
+            if (body.x == ITEM_SEG && (multi || body.z == 1)) {
+              // a loop around one chunk: all its iterations in registers
+              verdict = run_loop<MODE, BB, TL>(a, S, pi, __ldg(a.chunk + (multi ? body.w : body.y)), lo, hi,
+                                               ++ctag, lane, chk);
+              if (verdict) break;
+              continue;
+            }
+          }
           if (lane == 0) S.frames[sp] = Frame{loop, item, g, g_end};
           ++sp;
           loop = it.y; item = 0; g = lo; g_end = hi;
-          pbeg = __ldg(a.plan_ptr + loop);
-          pend = __ldg(a.plan_ptr + loop + 1);
-          if (lane < pi.ne) S.t[lane] += iter_cost;
+          pbeg = cb;
+          pend = ce;
         }
         __syncwarp();
         continue;
@@ -308,14 +611,26 @@ __global__ void __launch_bounds__(kWarps * 32) k_sweep(const SweepArgs a) {
       if (!BB && it.w >= 0) {                          // several iterations at once
         const int4 ch = __ldg(a.chunk + it.w);
         const int32_t v = min(ch.z, g_end - g);
-        verdict = run_chunk<MODE, BB, TL>(a, S, ch, g, v, ++ctag, lane, chk);
+        LaneRec Lr;
+        load_lane(a, ch, lane, Lr);
+        int32_t T[kMaxDeps];
+        load_thr(Lr, lane < ch.y && Lr.meta.y < v, g + Lr.meta.y, T);
+        set_groups(S, Lr, lane, lane < ch.y, v, ++ctag);
+        verdict = run_chunk<MODE, BB, TL>(a, S, ch, Lr, T, g, v, ctag, lane, chk);
         if (verdict) break;
         g += v - 1;
         item = pend - pbeg;                            // continue at the END of iteration g
         continue;
       }
-      for (int c = 0; c < it.z && !verdict; ++c)
-        verdict = run_chunk<MODE, BB, TL>(a, S, __ldg(a.chunk + it.y + c), g, 1, ++ctag, lane, chk);
+      for (int c = 0; c < it.z && !verdict; ++c) {
+        const int4 ch = __ldg(a.chunk + it.y + c);
+        LaneRec Lr;
+        load_lane(a, ch, lane, Lr);
+        int32_t T[kMaxDeps];
+        load_thr(Lr, lane < ch.y, g, T);
+        set_groups(S, Lr, lane, lane < ch.y, 1, ++ctag);
+        verdict = run_chunk<MODE, BB, TL>(a, S, ch, Lr, T, g, 1, ctag, lane, chk);
+      }
       if (verdict) break;
       ++item;
     }
@@ -365,13 +680,19 @@ cudaError_t launch3(const SweepArgs& a, size_t smem, int num_sms, cudaStream_t s
 
 }  // namespace
 
-size_t sweep_smem_bytes(int sem_cap, int frame_depth) {
-  return kWarps * warp_bytes(sem_cap, frame_depth);
+size_t sweep_smem_bytes(int sem_cap, int frame_depth, int ring) {
+  return kWarps * warp_bytes(sem_cap, frame_depth, ring);
+}
+
+int sweep_ring_for(int sem_cap, int frame_depth, size_t limit) {
+  for (int r = kRingMax; r >= 1; r >>= 1)
+    if (sweep_smem_bytes(sem_cap, frame_depth, r) <= limit) return r;
+  return 0;
 }
 
 cudaError_t launch_sweep(const SweepArgs& a, bool barrier, int num_sms, cudaStream_t s) {
   if (a.n_programs == 0) return cudaSuccess;
-  const size_t smem = sweep_smem_bytes(a.sem_cap, a.frame_depth);
+  const size_t smem = sweep_smem_bytes(a.sem_cap, a.frame_depth, a.ring);
   if (a.mode == SYNC_THR_PERLOOP)
     return barrier ? launch3<SYNC_THR_PERLOOP, true>(a, smem, num_sms, s)
                    : launch3<SYNC_THR_PERLOOP, false>(a, smem, num_sms, s);
