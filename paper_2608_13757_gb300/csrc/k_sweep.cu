@@ -378,12 +378,15 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     const int32_t n_in = __shfl_sync(kFull, ns, e);
 
     // waits: earlier increments from the ring or history, in-chunk ones by lane
+    // (barrier scheme: an increment before this iteration retired before the
+    // barrier that ended the last iteration or opened the loop, so that wait
+    // never binds)
     int32_t known = kNeg;
     int src0 = -1, src1 = -1;
     bool fallback = false;
     if (valid && T0 > 0) {
       if (T0 <= pub0) {
-        known = pub0 - T0 <= S.rmask ? ring0[(T0 - 1) & S.rmask] : a.hist[hist0 + T0];
+        if (!BB) known = pub0 - T0 <= S.rmask ? ring0[(T0 - 1) & S.rmask] : a.hist[hist0 + T0];
       } else {
         const unsigned m = wg0 & vm;
         const int k = T0 - pub0;
@@ -392,7 +395,7 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     }
     if (valid && T1 > 0) {
       if (T1 <= pub1) {
-        known = max(known, pub1 - T1 <= S.rmask ? ring1[(T1 - 1) & S.rmask] : a.hist[hist1 + T1]);
+        if (!BB) known = max(known, pub1 - T1 <= S.rmask ? ring1[(T1 - 1) & S.rmask] : a.hist[hist1 + T1]);
       } else {
         const unsigned m = wg1 & vm;
         const int k = T1 - pub1;
