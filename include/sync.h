@@ -117,9 +117,10 @@ typedef struct {
   int64_t device_bytes;     /* device memory held by the handle               */
   int64_t h2d_bytes;        /* bytes sync_load_programs copied host -> device */
   int64_t struct_bytes;     /* encoding bytes the threshold and check kernels
-                               read besides the thresholds: parent indices and
-                               trip prefix sums of the loops on dependency
-                               paths (each array once), dependency tables     */
+                               read besides the thresholds, each array once:
+                               per-iteration trip starts and ancestors derived
+                               at load time, trip prefix sums of nested
+                               producers' loops, dependency tables            */
 } sync_sizes;
 
 /* Timing-model constants in cycles, all >= 0 (see sync_simulate). */

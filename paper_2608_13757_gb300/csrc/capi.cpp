@@ -6,6 +6,7 @@
 #include <memory>
 #include <new>
 #include <string>
+#include <unordered_map>
 #include <vector>
 
 #include "enc.h"
@@ -75,6 +76,8 @@ struct ProgScratch {
   std::vector<int32_t> depth, body_ptr, body, rank, nloop_eng, x_ndeps, x_dep_begin;
   std::vector<int32_t> x_own[2], x_hstride[2], x_koff[2];
   std::vector<int64_t> total, keys;
+  std::vector<int64_t> tstart_of;                 // derived trip-start array per loop, -1 if none
+  std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
 };
 
 // Appends one sweep chunk: lanes `recs` (program-local instructions, already
@@ -146,7 +149,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
   std::vector<int64_t> hist_len(2, 0);
-  std::vector<uint8_t> reads_pidx(NL, 0), reads_rowptr(NL, 0);
+  std::vector<uint8_t> reads_rowptr(NL, 0);
+  std::vector<DeriveJob> jobs;
+  int64_t n_derived = 0;
   int64_t n_pairs = 0, n_pairs_padded = 0, n_inst = 0, n_iters = 0, rowptr_len = 0;
   ProgScratch S;
 
@@ -161,6 +166,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     const int32_t* lpos = d.loop_pos + l0;
     S.depth.assign(nl, 0);
     S.total.assign(nl, 0);
+    S.tstart_of.assign(nl, -1);
+    S.anc_of.clear();
     if (par[0] != -1) raise(SYNC_ERR_MALFORMED, where(p, "loop 0 must have parent -1, loop", 0));
     int32_t depth_max = 0;
     for (int32_t l = 1; l < nl; ++l) {
@@ -298,10 +305,32 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       D.kase = kase;
       D.k = off; D.N = N; D.K = K;
       D.path = (int64_t)path.size();
-      for (int32_t l = Cl; l != Sl; l = par[l]) { path.push_back(loop[l0 + l].pidx_off); reads_pidx[l0 + l] = 1; }
-      reads_pidx[l0 + Sl] = 1;
-      reads_rowptr[l0 + Sl] = 1;
+      for (int32_t l = Cl; l != Sl; l = par[l]) path.push_back(loop[l0 + l].pidx_off);
       for (int32_t l = Pl; l != Sl; l = par[l]) reads_rowptr[l0 + l] = 1;
+      // derived arrays: trip starts of S, and the S-ancestors of the consumer loop
+      if (S.tstart_of[Sl] < 0) {
+        S.tstart_of[Sl] = n_derived;
+        DeriveJob J{};
+        J.out = n_derived; J.a = loop[l0 + Sl].pidx_off; J.b = loop[l0 + Sl].rowptr_off;
+        J.n = (int32_t)S.total[Sl]; J.kind = DERIVE_TSTART;
+        jobs.push_back(J);
+        n_derived += pad4(S.total[Sl]);
+      }
+      D.tstart = S.tstart_of[Sl];
+      D.anc = -1;
+      if (D.up > 0) {
+        const int64_t key = (int64_t)Cl * nl + Sl;
+        auto f = S.anc_of.find(key);
+        if (f == S.anc_of.end()) {
+          DeriveJob J{};
+          J.out = n_derived; J.a = D.path; J.b = 0;
+          J.n = (int32_t)S.total[Cl]; J.kind = DERIVE_ANC; J.up = D.up;
+          jobs.push_back(J);
+          f = S.anc_of.emplace(key, n_derived).first;
+          n_derived += pad4(S.total[Cl]);
+        }
+        D.anc = f->second;
+      }
       path.push_back(loop[l0 + Sl].pidx_off);
       path.push_back(loop[l0 + Sl].rowptr_off);
       D.s_pidx = loop[l0 + Sl].pidx_off;
@@ -471,6 +500,16 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       tile_first[t] = (int32_t)di;
     }
   }
+  const int64_t n_jtiles = (n_derived + kTilePairs - 1) / kTilePairs;
+  std::vector<int32_t> tile_job(n_jtiles + 1, jobs.empty() ? 0 : (int32_t)(jobs.size() - 1));
+  {
+    int64_t ji = 0;
+    for (int64_t t = 0; t < n_jtiles; ++t) {
+      const int64_t q = t * kTilePairs;
+      while (ji + 1 < (int64_t)jobs.size() && jobs[ji + 1].out <= q) ++ji;
+      tile_job[t] = (int32_t)ji;
+    }
+  }
   const int64_t n_itiles = (n_iters + kTilePairs - 1) / kTilePairs;
   std::vector<int32_t> tile_loop(n_itiles + 1, NL > 0 ? (int32_t)(NL - 1) : 0);
   {
@@ -500,10 +539,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   {
     int64_t sb = (int64_t)ND * (int64_t)sizeof(DepInfo) + 8 * (ND + 1) + 8 * (int64_t)path.size() +
                  4 * (int64_t)tile_first.size();
-    for (int64_t l = 0; l < NL; ++l) {
-      if (reads_pidx[l]) sb += 4 * (int64_t)loop[l].total;
+    sb += 4 * n_derived;
+    for (int64_t l = 0; l < NL; ++l)
       if (reads_rowptr[l]) sb += 4 * ((int64_t)loop[l].n_parent + 1);
-    }
     h.sz.struct_bytes = sb;
   }
   h.seg_host = seg;
@@ -522,6 +560,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.seg = h.upload(seg, stream, "segment offsets");
   h.tile_first = h.upload(tile_first, stream, "tile table");
   h.path = h.upload(path, stream, "path pool");
+  h.derived = h.alloc<int32_t>(n_derived, "derived trip starts and ancestors");
+  DeriveJob* d_jobs = h.upload(jobs, stream, "derive jobs");
+  int32_t* d_tile_job = h.upload(tile_job, stream, "derive tile table");
   int32_t* d_tile_loop = h.upload(tile_loop, stream, "loop tile table");
   h.prog = h.upload(prog, stream, "program table");
   h.order = h.upload(order, stream, "program order");
@@ -558,6 +599,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   }
   h.n_lanes = (int64_t)lrec.size();
   cuda_check(launch_expand(h.loop, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
+  cuda_check(launch_derive(d_jobs, d_tile_job, h.rowptr, h.pidx, h.path, h.derived, n_derived, h.num_sms, stream),
+             "derive");
   cuda_check(cudaStreamSynchronize(stream), "load");
 }
 
@@ -597,7 +640,7 @@ sync_status sync_pair_offsets(const sync_programs* h, int64_t* offsets, int32_t*
 
 static ThrArgs thr_args(const sync_programs* h, sync_thr_mode mode) {
   ThrArgs a;
-  a.dep = h->dep; a.seg = h->seg; a.tile_first = h->tile_first; a.path = h->path;
+  a.dep = h->dep; a.derived = h->derived; a.seg = h->seg; a.tile_first = h->tile_first; a.path = h->path;
   a.rowptr = h->rowptr; a.pidx = h->pidx; a.n_chunks = h->n_chunks; a.mode = mode;
   return a;
 }

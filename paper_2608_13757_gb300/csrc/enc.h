@@ -43,6 +43,8 @@ struct alignas(16) DepInfo {
   int64_t path;
   int64_t s_pidx;     // S's pidx and rowptr offsets (= path entries up, up+1)
   int64_t s_rowptr;
+  int64_t tstart;     // derived pool: first iteration of the trip, per iteration of S
+  int64_t anc;        // derived pool: enclosing S-iteration per consumer iteration (up > 0)
   int32_t total;      // consumer instances (= total of the consumer's loop)
   int32_t up;
   int32_t clen;
@@ -106,8 +108,27 @@ constexpr int32_t LANE_RUN_LAST = 2;
 constexpr int32_t OP_LOOP = -1;
 constexpr int32_t OP_END = -2;
 
+// Derived per-iteration arrays of the threshold and check kernels, built at
+// load time from the trip prefix sums and parent indices (one job each):
+//   DERIVE_TSTART  out[gs] = rowptr_S[pidx_S[gs]]   (a = pidx offset of S,
+//                  b = rowptr offset of S)
+//   DERIVE_ANC     out[g]  = g walked `up` levels up the parent indices
+//                  (a = path pool offset of the pidx offsets, innermost first)
+// Every array starts at a multiple of 4 entries, so a 4-pair chunk reads its
+// four entries with one int4 load.
+enum : int32_t { DERIVE_TSTART = 0, DERIVE_ANC = 1 };
+struct alignas(16) DeriveJob {
+  int64_t out;
+  int64_t a, b;
+  int32_t n;
+  int32_t kind;
+  int32_t up;
+  int32_t pad_;
+};
+
 struct ThrArgs {
   const DepInfo* dep;
+  const int32_t* derived;
   const int64_t* seg;        // [n_deps + 1] segment offsets
   const int32_t* tile_first; // [n_tiles + 1]
   const int64_t* path;
@@ -191,6 +212,10 @@ struct SweepArgs {
 // with pidx_off[l] <= t*kTilePairs), with one extra entry n_loops-1.
 cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const int32_t* rowptr,
                           int32_t* pidx, int64_t n_iters, int num_sms, cudaStream_t s);
+// tile_job[t] = job whose output holds pool entry t*kTilePairs.
+cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
+                          const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,
+                          int num_sms, cudaStream_t s);
 cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s);
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStream_t s);

@@ -28,6 +28,7 @@ struct sync_programs {
   int64_t* seg = nullptr;
   int32_t* tile_first = nullptr;
   int64_t* path = nullptr;
+  int32_t* derived = nullptr;       // per-iteration trip starts and S-ancestors
   int64_t n_chunks = 0;
   // simulator encoding
   syncgb::ProgInfo* prog = nullptr;

@@ -1,4 +1,5 @@
-// Load-time expansion of the trip prefix sums into parent-iteration indices.
+// Load-time expansion of the trip prefix sums into parent-iteration indices,
+// and the derived per-iteration arrays of the threshold kernels.
 //
 // For every loop l and every global iteration g of l, pidx_l[g] is the
 // parent's global iteration j with rowptr_l[j] <= g < rowptr_l[j+1] (the CSR
@@ -34,7 +35,47 @@ k_expand(const LoopInfo* __restrict__ loop, const int32_t* __restrict__ tile_loo
   }
 }
 
+// One thread per derived entry; the job is found inside the range the
+// host's tile table gives.
+__global__ void __launch_bounds__(kThreads)
+k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_job,
+         const int32_t* __restrict__ rowptr, const int32_t* __restrict__ pidx,
+         const int64_t* __restrict__ path, int32_t* __restrict__ out, int64_t n) {
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < n; q += stride) {
+    const int64_t t = q / kTilePairs;
+    int lo = tile_job[t], hi = tile_job[t + 1];
+    while (lo < hi) {                 // largest job with out <= q
+      const int mid = (lo + hi + 1) >> 1;
+      if (jobs[mid].out <= q) lo = mid; else hi = mid - 1;
+    }
+    const DeriveJob J = jobs[lo];
+    const int32_t g = (int32_t)(q - J.out);
+    int32_t v = 0;                    // padding entries
+    if (g < J.n) {
+      if (J.kind == DERIVE_TSTART) {
+        v = rowptr[J.b + pidx[J.a + g]];
+      } else {
+        v = g;
+        for (int i = 0; i < J.up; ++i) v = pidx[path[J.a + i] + v];
+      }
+    }
+    out[q] = v;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
+                          const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,
+                          int num_sms, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  const int64_t want = (n + kThreads - 1) / kThreads;
+  const int64_t cap = (int64_t)num_sms * 8;
+  const int grid = (int)(want < cap ? want : cap);
+  k_derive<<<grid, kThreads, 0, s>>>(jobs, tile_job, rowptr, pidx, path, derived, n);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const int32_t* rowptr,
                           int32_t* pidx, int64_t n_iters, int num_sms, cudaStream_t s) {

@@ -6,15 +6,17 @@
 // never straddles two dependencies; consecutive threads own consecutive
 // chunks, so a warp's store or load is 512 contiguous bytes.  Both kernels
 // are HBM-streaming: 4 bytes per pair written (thresholds) or read
-// (checker), plus the loop-structure reads, which consecutive pairs of one
-// dependency share through L1/L2.
+// (checker), plus the derived per-iteration arrays, which consecutive pairs
+// of one dependency share through L1/L2.
 //
 // Both results depend on g only through g_S, the enclosing iteration of the
 // dependency's common loop S, and the start of g_S's trip of S (Eq. 1, and
-// Sec. 5.1's registers r_S and r-hat_S).  A chunk's four consumer iterations
-// usually share g_S (consumer nested below S) or the trip (consumer directly
-// in S), so the chunk looks them up for its first and last iteration and
-// evaluates once per distinct g_S.
+// Sec. 5.1's registers r_S and r-hat_S).  Both come from arrays derived at
+// load time (S-ancestor per consumer iteration, trip start per S-iteration),
+// so a chunk needs the dependency record, one int4 of ancestors or trip
+// starts, and a trip start per distinct g_S: a short chain of dependent
+// loads.  A chunk's four consumer iterations usually share g_S, evaluated
+// once.
 #include "enc.h"
 
 namespace syncgb {
@@ -33,24 +35,6 @@ __device__ __forceinline__ int find_dep(const ThrArgs& a, int64_t q) {
     if (__ldg(a.seg + mid) <= q) lo = mid; else hi = mid - 1;
   }
   return lo;
-}
-
-// Global iterations of S enclosing the consumer's global iterations ga and
-// gb: both walked up the expanded parent indices together, `up` levels.
-__device__ __forceinline__ void up_to_S(const ThrArgs& a, const DepInfo& D, int32_t& ga, int32_t& gb) {
-  for (int i = 0; i < D.up; ++i) {
-    const int32_t* p = a.pidx + __ldg(a.path + D.path + i);
-    ga = __ldg(p + ga);
-    gb = __ldg(p + gb);
-  }
-}
-
-// First global iteration of S in the trip that holds gs, and (in `end`) the
-// first one after it.
-__device__ __forceinline__ int32_t trip_of(const ThrArgs& a, const DepInfo& D, int32_t gs, int32_t& end) {
-  const int32_t* rp = a.rowptr + D.s_rowptr + __ldg(a.pidx + D.s_pidx + gs);
-  end = __ldg(rp + 1);
-  return __ldg(rp);
 }
 
 // Iterations of P that start inside the first x iterations of S (x may equal
@@ -93,54 +77,42 @@ __device__ __forceinline__ int32_t minimum(const ThrArgs& a, const DepInfo& D, i
   return encode(D, count_down(a, D, gt + 1), mode);
 }
 
-// Values of the chunk's pairs g0 .. g0+3 (entries at or past `total` are
-// padding and get 0).
 template <bool CHECK>
 __device__ __forceinline__ int32_t eval_at(const ThrArgs& a, const DepInfo& D, int32_t gs, int32_t start,
                                            int mode) {
   return CHECK ? minimum(a, D, gs, start, mode) : wait_value(a, D, gs, start, mode);
 }
 
+// Values of the chunk's pairs g0 .. g0+3 (entries at or past `total` are
+// padding and get 0).  g0 is a multiple of 4, and so is every derived
+// array's start, so the chunk's four trip starts (consumer in S) or
+// S-ancestors (consumer below S) come in one int4 load.
 template <bool CHECK>
 __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D, int32_t g0, int mode) {
   const int32_t n = D.total - g0 < kChunk ? D.total - g0 : kChunk;   // >= 1
   int32_t v[kChunk] = {0, 0, 0, 0};
   if (D.up == 0) {
-    // consumer directly in S: g_S = g; one trip lookup unless the chunk
-    // crosses into the next trip
-    int32_t end;
-    int32_t start = trip_of(a, D, g0, end);
+    // consumer directly in S: g_S = g
+    const int4 ts = __ldg(reinterpret_cast<const int4*>(a.derived + D.tstart + g0));
+    const int32_t st[kChunk] = {ts.x, ts.y, ts.z, ts.w};
 #pragma unroll
-    for (int i = 0; i < kChunk; ++i) {
-      if (i < n) {
-        const int32_t g = g0 + i;
-        if (g >= end) start = trip_of(a, D, g, end);
-        v[i] = eval_at<CHECK>(a, D, g, start, mode);
-      }
-    }
+    for (int i = 0; i < kChunk; ++i)
+      if (i < n) v[i] = eval_at<CHECK>(a, D, g0 + i, st[i], mode);
   } else {
-    // consumer nested below S: one value per distinct g_S; the first and
-    // last iteration's g_S decide whether the chunk stays in one
-    int32_t gs = g0, gl = g0 + n - 1;
-    up_to_S(a, D, gs, gl);
-    int32_t end;
-    int32_t val = eval_at<CHECK>(a, D, gs, trip_of(a, D, gs, end), mode);
+    // consumer nested below S: one value per distinct g_S (non-decreasing)
+    const int4 an = __ldg(reinterpret_cast<const int4*>(a.derived + D.anc + g0));
+    const int32_t gs[kChunk] = {an.x, an.y, an.z, an.w};
+    int32_t cur = gs[0];
+    int32_t val = eval_at<CHECK>(a, D, cur, __ldg(a.derived + D.tstart + cur), mode);
     v[0] = val;
-    if (gl == gs) {
 #pragma unroll
-      for (int i = 1; i < kChunk; ++i) v[i] = i < n ? val : 0;
-    } else {
-#pragma unroll
-      for (int i = 1; i < kChunk; ++i) {
-        if (i < n) {
-          int32_t gi = g0 + i;
-          for (int l = 0; l < D.up; ++l) gi = __ldg(a.pidx + __ldg(a.path + D.path + l) + gi);
-          if (gi != gs) {
-            gs = gi;
-            val = eval_at<CHECK>(a, D, gs, trip_of(a, D, gs, end), mode);
-          }
-          v[i] = val;
+    for (int i = 1; i < kChunk; ++i) {
+      if (i < n) {
+        if (gs[i] != cur) {
+          cur = gs[i];
+          val = eval_at<CHECK>(a, D, cur, __ldg(a.derived + D.tstart + cur), mode);
         }
+        v[i] = val;
       }
     }
   }
