@@ -120,7 +120,7 @@ __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D,
 }
 
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 4) k_thresholds(const ThrArgs a, int32_t* __restrict__ thr) {
+__global__ void __launch_bounds__(kThreads, 8) k_thresholds(const ThrArgs a, int32_t* __restrict__ thr) {
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.n_chunks; c += stride) {
     const int64_t q = c * kChunk;
@@ -138,7 +138,7 @@ __device__ __forceinline__ void tally(int32_t got, int32_t want, int64_t idx,
 }
 
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 4) k_check(const CheckArgs a) {
+__global__ void __launch_bounds__(kThreads, 6) k_check(const CheckArgs a) {
   unsigned long long unsafe = 0, over = 0, first = ~0ull;
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.t.n_chunks; c += stride) {
