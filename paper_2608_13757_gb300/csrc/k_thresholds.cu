@@ -129,9 +129,8 @@ __global__ void __launch_bounds__(kThreads, 8) k_thresholds(const ThrArgs a, int
   }
 }
 
-__device__ __forceinline__ void tally(int32_t got, int32_t want, int64_t idx,
-                                      unsigned long long& unsafe, unsigned long long& over,
-                                      unsigned long long& first) {
+__device__ __forceinline__ void tally(int32_t got, int32_t want, int64_t idx, uint32_t& unsafe,
+                                      uint32_t& over, unsigned long long& first) {
   if (got == want) return;
   if (got < want) ++unsafe; else ++over;
   if ((unsigned long long)idx < first) first = (unsigned long long)idx;
@@ -139,7 +138,9 @@ __device__ __forceinline__ void tally(int32_t got, int32_t want, int64_t idx,
 
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 6) k_check(const CheckArgs a) {
-  unsigned long long unsafe = 0, over = 0, first = ~0ull;
+  // a thread's counts fit 32 bits (it sees at most n_chunks / threads chunks)
+  uint32_t unsafe = 0, over = 0;
+  unsigned long long first = ~0ull;
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.t.n_chunks; c += stride) {
     const int64_t q = c * kChunk;
@@ -148,20 +149,25 @@ __global__ void __launch_bounds__(kThreads, 6) k_check(const CheckArgs a) {
     const int32_t g0 = (int32_t)(q - D.seg_off);
     const int4 m = chunk_values<true>(a.t, D, g0, MODE);
     // padding entries are not pairs: the checker reads only the first n
-    tally(v.x, m.x, q + 0, unsafe, over, first);
-    if (g0 + 1 < D.total) tally(v.y, m.y, q + 1, unsafe, over, first);
-    if (g0 + 2 < D.total) tally(v.z, m.z, q + 2, unsafe, over, first);
-    if (g0 + 3 < D.total) tally(v.w, m.w, q + 3, unsafe, over, first);
+    const int32_t n = D.total - g0;
+    const bool bad = v.x != m.x || (n > 1 && v.y != m.y) || (n > 2 && v.z != m.z) || (n > 3 && v.w != m.w);
+    if (bad) {
+      tally(v.x, m.x, q + 0, unsafe, over, first);
+      if (n > 1) tally(v.y, m.y, q + 1, unsafe, over, first);
+      if (n > 2) tally(v.z, m.z, q + 2, unsafe, over, first);
+      if (n > 3) tally(v.w, m.w, q + 3, unsafe, over, first);
+    }
   }
-  for (int o = 16; o > 0; o >>= 1) {
-    unsafe += __shfl_xor_sync(0xffffffffu, unsafe, o);
-    over += __shfl_xor_sync(0xffffffffu, over, o);
-    const unsigned long long f = __shfl_xor_sync(0xffffffffu, first, o);
+  unsigned long long u = unsafe, o = over;
+  for (int s = 16; s > 0; s >>= 1) {
+    u += __shfl_xor_sync(0xffffffffu, u, s);
+    o += __shfl_xor_sync(0xffffffffu, o, s);
+    const unsigned long long f = __shfl_xor_sync(0xffffffffu, first, s);
     first = f < first ? f : first;
   }
   if ((threadIdx.x & 31) == 0) {
-    if (unsafe) atomicAdd(a.counts + 0, unsafe);
-    if (over) atomicAdd(a.counts + 1, over);
+    if (u) atomicAdd(a.counts + 0, u);
+    if (o) atomicAdd(a.counts + 1, o);
     if (first != ~0ull) atomicMin(a.first_bad, first);
   }
 }

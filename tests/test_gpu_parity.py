@@ -20,6 +20,8 @@ def sg():
     import torch
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
+    from paper_2608_13757_gb300 import build
+    build.build()
     import paper_2608_13757_gb300 as m
     return m
 
