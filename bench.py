@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--config", default="chain")
     ap.add_argument("--programs", type=int, default=None, help="programs per rank")
+    ap.add_argument("--first-program", type=int, default=0,
+                    help="id of rank 0's first program (ranks follow contiguously)")
     ap.add_argument("--mode", choices=("perloop", "count"), default="perloop")
     ap.add_argument("--cpu-sample", type=int, default=32768,
                     help="programs of the workload the CPU oracle baseline runs")
@@ -140,6 +142,7 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     mode = sg.THR_PERLOOP if args.mode == "perloop" else sg.THR_COUNT
     first, P = shard(rank, args.programs or workloads.CONFIGS[args.config][1])
+    first += args.first_program
     batch = workloads.generate(args.config, n_programs=P, first_program=first)
     t0 = time.perf_counter()
     h = sg.sync_load_programs(batch, device=local_rank)
@@ -178,6 +181,9 @@ def run_gpu(args, rank, world, local_rank):
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
+    # keep the GPU busy (about 5 ms) while the host queues the timed steps, so
+    # host-side launch latency never shows up as GPU time between the events
+    torch.cuda._sleep(10_000_000)
     start.record(stream)
     for k in range(args.steps):
         step(evs[k])
