@@ -24,7 +24,7 @@ _LIB = os.path.join(_LIBDIR, "liboracle.so")
 _SRC = [os.path.join(_HERE, "oracle.c")]
 _HDR = [os.path.join(_HERE, "oracle.h")]
 
-COUNT, PERLOOP = 0, 1
+COUNT, PERLOOP, PERENGINE = 0, 1, 2
 BARRIER_FREE, BARRIER = 0, 1
 CASE_PS, CASE_NEST_FWD, CASE_NEST_BWD, CASE_NONE = 0, 1, 2, 3
 SIM_OK, SIM_OVERFLOW, SIM_DEADLOCK = 0, 4, 7

@@ -296,10 +296,53 @@ static int64_t perloop_value(int64_t c, int32_t N, int32_t K) {
   return v > INT32_MAX ? -1 : v;
 }
 
-static int store(int32_t *out, int64_t i, int mode, int64_t c, const dep_class *dc) {
-  int64_t v = mode == ORC_PERLOOP ? perloop_value(c, dc->N, dc->K) : c;
+/* Encodes a completion count c in `mode`; `ord` (per-engine mode only) lists
+ * the engine ordinal of each of the producer's instances in program order. */
+static int store(int32_t *out, int64_t i, int mode, int64_t c, const dep_class *dc,
+                 const int64_t *ord) {
+  int64_t v;
+  if (mode == ORC_PERLOOP) v = perloop_value(c, dc->N, dc->K);
+  else if (mode == ORC_PERENGINE) v = c > 0 ? ord[c - 1] : 0;
+  else v = c;
   if (v < 0 || v > INT32_MAX) return ORC_ERR_OVERFLOW;
   out[i] = (int32_t)v;
+  return ORC_OK;
+}
+
+/* ---------------------------------------------- per-engine stream ordinals */
+
+/* Walk the program in program order, counting each engine's datapath
+ * instances: ord[ioff[x] + g] is the 1-based position of instruction x's
+ * instance at global iteration g of its loop in the dynamic stream of x's
+ * engine (Sec. 6.1: a per-engine counter reaches it when that instance
+ * retires, retirement being in order on an engine). */
+typedef struct {
+  int64_t *ord, *ioff, *count;
+} ord_ctx;
+
+static void ord_visit(walker *w, int32_t x) {
+  ord_ctx *O = (ord_ctx *)w->ctx;
+  prog_t *P = w->P;
+  int32_t e = P->xe[x];
+  O->ord[O->ioff[x] + w->gl[P->depth[P->xl[x]]]] = ++O->count[e];
+}
+
+/* *ord_out / *ioff_out: malloc'd tables (caller frees) */
+static int engine_ordinals(prog_t *P, int64_t **ord_out, int64_t **ioff_out) {
+  ord_ctx O;
+  O.ioff = (int64_t *)malloc(((size_t)P->nx + 1) * sizeof(int64_t));
+  O.count = (int64_t *)calloc((size_t)P->ne, sizeof(int64_t));
+  if (!O.ioff || !O.count) { free(O.ioff); free(O.count); return ORC_ERR_OOM; }
+  int64_t n = 0;
+  for (int32_t x = 0; x < P->nx; ++x) { O.ioff[x] = n; n += P->total[P->xl[x]]; }
+  O.ioff[P->nx] = n;
+  O.ord = (int64_t *)malloc(((size_t)n + 1) * sizeof(int64_t));
+  if (!O.ord) { free(O.ioff); free(O.count); return ORC_ERR_OOM; }
+  int rc = walk(P, ord_visit, &O);
+  free(O.count);
+  if (rc) { free(O.ord); free(O.ioff); return rc; }
+  *ord_out = O.ord;
+  *ioff_out = O.ioff;
   return ORC_OK;
 }
 
@@ -371,7 +414,7 @@ static void bf_visit(walker *w, int32_t x) {
 }
 
 int orc_thresholds_bruteforce(const orc_batch *b, int mode, int32_t *out) {
-  if (!b || !out || (mode != ORC_COUNT && mode != ORC_PERLOOP)) return ORC_ERR_ARG;
+  if (!b || !out || (mode != ORC_COUNT && mode != ORC_PERLOOP && mode != ORC_PERENGINE)) return ORC_ERR_ARG;
   int64_t base = 0;
   for (int32_t p = 0; p < b->n_programs; ++p) {
     prog_t P;
@@ -380,6 +423,8 @@ int orc_thresholds_bruteforce(const orc_batch *b, int mode, int32_t *out) {
     inst_list L;
     memset(&L, 0, sizeof L);
     rc = walk(&P, bf_visit, &L);
+    int64_t *ord = NULL, *ioff = NULL;
+    if (rc == ORC_OK && mode == ORC_PERENGINE) rc = engine_ordinals(&P, &ord, &ioff);
     int64_t *t = (int64_t *)malloc(((size_t)P.maxdepth + 1) * sizeof(int64_t));
     for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) {
       dep_class dc = classify(&P, d);
@@ -401,10 +446,11 @@ int orc_thresholds_bruteforce(const orc_batch *b, int mode, int32_t *out) {
             if (cmp <= 0) ++c;
           }
         }
-        rc = store(out, base + L.g[i], mode, c, &dc);
+        rc = store(out, base + L.g[i], mode, c, &dc, ord ? ord + ioff[P.dp[d]] : NULL);
       }
       base += P.total[P.xl[P.dc[d]]];
     }
+    free(ord); free(ioff);
     free(t); free(L.x); free(L.g); free(L.voff); free(L.vec);
     prog_close(&P);
     if (rc) return rc;
@@ -457,6 +503,8 @@ static int prog_thresholds(prog_t *P, int mode, int32_t *out) {
     if (!C.cnt[d] || !C.pg[d] || !C.pv[d]) rc = ORC_ERR_OOM;
   }
   if (rc == ORC_OK) rc = walk(P, cnt_visit, &C);
+  int64_t *ord = NULL, *ioff = NULL;
+  if (rc == ORC_OK && mode == ORC_PERENGINE) rc = engine_ordinals(P, &ord, &ioff);
   int64_t base = 0;
   for (int32_t d = 0; d < nd && rc == ORC_OK; ++d) {
     int64_t nS = P->total[cls[d].S];
@@ -467,10 +515,11 @@ static int prog_thresholds(prog_t *P, int mode, int32_t *out) {
       /* t lies in the same trip of S as v when tS >= 1, so its global index is
        * the consumer's S-iteration minus k */
       int64_t c = tS <= 0 ? 0 : C.cnt[d][C.pg[d][j] - P->dk[d]];
-      rc = store(out, base + j, mode, c, &cls[d]);
+      rc = store(out, base + j, mode, c, &cls[d], ord ? ord + ioff[P->dp[d]] : NULL);
     }
     base += ncons;
   }
+  free(ord); free(ioff);
   for (int32_t d = 0; d < nd; ++d) {
     if (C.cnt) free(C.cnt[d]);
     if (C.pg) free(C.pg[d]);
@@ -481,7 +530,7 @@ static int prog_thresholds(prog_t *P, int mode, int32_t *out) {
 }
 
 int orc_thresholds(const orc_batch *b, int mode, int32_t *out) {
-  if (!b || !out || (mode != ORC_COUNT && mode != ORC_PERLOOP)) return ORC_ERR_ARG;
+  if (!b || !out || (mode != ORC_COUNT && mode != ORC_PERLOOP && mode != ORC_PERENGINE)) return ORC_ERR_ARG;
   int64_t base = 0;
   for (int32_t p = 0; p < b->n_programs; ++p) {
     prog_t P;
@@ -585,7 +634,8 @@ int orc_register_replay(const orc_batch *b, int mode, int32_t *out) {
 
 int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[2],
               int64_t *first_bad) {
-  if (!b || !thr || !counts || !first_bad || (mode != ORC_COUNT && mode != ORC_PERLOOP))
+  if (!b || !thr || !counts || !first_bad ||
+      (mode != ORC_COUNT && mode != ORC_PERLOOP && mode != ORC_PERENGINE))
     return ORC_ERR_ARG;
   counts[0] = counts[1] = 0;
   *first_bad = -1;

@@ -35,9 +35,12 @@ typedef struct {
 enum { ORC_OK = 0, ORC_ERR_ARG = 1, ORC_ERR_MALFORMED = 2, ORC_ERR_NOT_ALLOCATABLE = 3,
        ORC_ERR_OVERFLOW = 4, ORC_ERR_OOM = 6 };
 
-/* threshold modes: the producer-completion count c (Eq. 3) or the per-loop
- * semaphore value T = N*c - (N-K), 0 when c = 0 (Eq. 5) */
-enum { ORC_COUNT = 0, ORC_PERLOOP = 1 };
+/* threshold modes: the producer-completion count c (Eq. 3), the per-loop
+ * semaphore value T = N*c - (N-K), 0 when c = 0 (Eq. 5), or the per-engine
+ * semaphore value (Sec. 6.1): one counter per engine counts every retirement
+ * on that engine, so the wait is for the 1-based ordinal of the producer's
+ * c-th instance in its engine's dynamic instruction stream, 0 when c = 0 */
+enum { ORC_COUNT = 0, ORC_PERLOOP = 1, ORC_PERENGINE = 2 };
 
 /* allocatable cases of Sec. 5.2 */
 enum { ORC_CASE_PS = 0, ORC_CASE_NEST_FWD = 1, ORC_CASE_NEST_BWD = 2, ORC_CASE_NONE = 3 };
@@ -74,7 +77,8 @@ int orc_thresholds(const orc_batch *b, int mode, int32_t *out);
 /* The paper's registers replayed literally per engine (Fig. 7/8): r-hat := 0
  * at each loop statement, r++ and r-hat++ at each iteration start, and the
  * masked wait value of Eq. (2)/(3)/(5) before each consumer.  Entries of
- * non-allocatable dependencies are set to -1. */
+ * non-allocatable dependencies are set to -1.  Count and per-loop modes
+ * only. */
 int orc_register_replay(const orc_batch *b, int mode, int32_t *out);
 
 /* Minimality check of a threshold array against Eq. (1): counts[0] = pairs
@@ -86,7 +90,8 @@ int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[
 /* Event-stepped semaphore machine (timing model stated in oracle.c).  `thr`
  * is a threshold array in `mode`'s encoding; the machine waits on the
  * per-producer semaphore (count) or the per-(loop, engine) semaphore
- * (per-loop) until its value reaches the threshold.  issue/retire may be NULL. */
+ * (per-loop) until its value reaches the threshold.  issue/retire may be NULL.
+ * Count and per-loop modes only. */
 int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim_params *prm,
                  int variant, int32_t *makespan, uint64_t *checksum, int32_t *status,
                  int32_t *issue, int32_t *retire);

@@ -15,7 +15,7 @@ import workloads
 from tests import golden_io
 from tests import timing_model
 
-COUNT, PERLOOP = oracle.COUNT, oracle.PERLOOP
+COUNT, PERLOOP, PERENGINE = oracle.COUNT, oracle.PERLOOP, oracle.PERENGINE
 
 
 def pair_slices(batch):
@@ -232,9 +232,116 @@ def test_classification_cases():
     assert one(("A", 9), ("B", 0), 0, same_engine=True) == C.CASE_NONE
 
 
+# ------------------------------------------------- per-engine allocation
+
+def engine_streams(batch, p):
+    """Program p's dynamic instruction stream of every engine, in program
+    order, as lists of (program-local instruction, global iteration of its
+    loop): a direct walk of the loop tree with the actual trips."""
+    l0, l1 = int(batch.prog_loop_ptr[p]), int(batch.prog_loop_ptr[p + 1])
+    x0, x1 = int(batch.prog_instr_ptr[p]), int(batch.prog_instr_ptr[p + 1])
+    nl = l1 - l0
+    body = [[] for _ in range(nl)]
+    for x in range(x1 - x0):
+        body[int(batch.instr_loop[x0 + x])].append((int(batch.instr_pos[x0 + x]), "x", x))
+    for l in range(1, nl):
+        body[int(batch.loop_parent[l0 + l])].append((int(batch.loop_pos[l0 + l]), "l", l))
+    for b in body:
+        b.sort()
+    trips = [batch.trips[batch.trip_ptr[l0 + l]:batch.trip_ptr[l0 + l + 1]] for l in range(nl)]
+    nxt = [0] * nl
+    nxt[0] = 1
+    streams = {e: [] for e in range(int(batch.prog_n_engines[p]))}
+
+    def run(l, g):
+        for _, kind, i in body[l]:
+            if kind == "x":
+                streams[int(batch.instr_engine[x0 + i])].append((i, g))
+            else:
+                for _ in range(int(trips[i][g])):
+                    gm = nxt[i]
+                    nxt[i] += 1
+                    run(i, gm)
+    run(0, 0)
+    return streams
+
+
+def test_perengine_is_the_producer_ordinal_in_its_engine_stream():
+    """Sec. 6.1: one semaphore per engine counts all its retirements, so the
+    wait value is the 1-based position of the producer's c-th instance (c from
+    Eq. 1) in its engine's dynamic stream; checked against a direct walk."""
+    for seed in range(60):
+        batch = workloads.random_trees(seed, 6)
+        count = oracle.thresholds(batch, COUNT)
+        per_engine = oracle.thresholds(batch, PERENGINE)
+        assert np.array_equal(per_engine, oracle.thresholds_bruteforce(batch, PERENGINE))
+        sl = pair_slices(batch)
+        d = 0
+        for p in range(batch.n_programs):
+            streams = engine_streams(batch, p)
+            pos = {e: {inst: k + 1 for k, inst in enumerate(st)} for e, st in streams.items()}
+            x0 = int(batch.prog_instr_ptr[p])
+            for _ in range(int(batch.prog_dep_ptr[p + 1] - batch.prog_dep_ptr[p])):
+                px = int(batch.dep_prod[d])
+                e = int(batch.instr_engine[x0 + px])
+                want = [pos[e][(px, c - 1)] if c > 0 else 0 for c in count[sl[d]]]
+                assert per_engine[sl[d]].tolist() == want, (seed, d)
+                d += 1
+
+
+def test_perengine_reduces_to_perloop_when_alone_on_the_engine():
+    """When the producer's loop is the only place its engine has datapath
+    instructions and that loop sits directly under the top level, the engine
+    counter is the per-(loop, engine) counter: per-engine = per-loop (Eq. 5)."""
+    for trips in ([5], [3, 0, 4], [1, 7]):
+        b = workloads.ProgramBuilder(2)
+        A = b.loop(0, 1, trips[:1])
+        b.instr(0, 0, 1)                   # engine 1 only outside the loop
+        p0 = b.instr(A, 0, 0)
+        p1 = b.instr(A, 2, 0)
+        c0 = b.instr(A, 1, 1)
+        c1 = b.instr(A, 3, 1)
+        b.dep(p0, c0, 0)
+        b.dep(p1, c1, 1)
+        b.dep(p1, c0, 2)
+        batch = b.batch()
+        assert np.array_equal(oracle.thresholds(batch, PERENGINE), oracle.thresholds(batch, PERLOOP))
+
+
+def test_perengine_bounds():
+    """The c-th producer instance is at least the c-th instruction of its
+    engine, exactly so when the producer is its engine's only instruction;
+    0 exactly when c = 0."""
+    for seed in range(40):
+        batch = workloads.random_trees(seed, 6)
+        c = oracle.thresholds(batch, COUNT).astype(np.int64)
+        t = oracle.thresholds(batch, PERENGINE).astype(np.int64)
+        assert ((c == 0) == (t == 0)).all()
+        assert (t >= c).all()
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [6])
+    B = b.loop(A, 1, [2, 0, 3, 1, 1, 2])
+    p = b.instr(B, 0, 0)                   # engine 0's only instruction
+    x = b.instr(A, 2, 1)
+    b.dep(p, x, 0)
+    batch = b.batch()
+    assert np.array_equal(oracle.thresholds(batch, PERENGINE), oracle.thresholds(batch, COUNT))
+
+
+def test_perengine_nondecreasing_where_nonzero():
+    """For a fixed dependency the engine ordinal grows with c, so it is
+    nondecreasing over the pairs where it is nonzero (the c-xi invariant)."""
+    for seed in range(40):
+        batch = workloads.random_trees(seed, 6)
+        t = oracle.thresholds(batch, PERENGINE)
+        for s in pair_slices(batch):
+            nz = t[s][t[s] > 0]
+            assert (np.diff(nz) >= 0).all()
+
+
 # ---------------------------------------------------------------- checker
 
-@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP, PERENGINE])
 def test_checker_counts_planted_errors(mode):
     batch = workloads.generate("depth2", n_programs=8)
     thr = oracle.thresholds(batch, mode)
