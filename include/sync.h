@@ -61,8 +61,13 @@ typedef enum {
  * (per-instruction semaphores).  PERLOOP: the value T = N*c - (N-K), or 0
  * when c = 0, of the per-(loop, engine) semaphore of Eq. (5), where N is the
  * number of instructions directly in the producer's loop body on the
- * producer's engine and K the producer's 1-based rank among them. */
-typedef enum { SYNC_THR_COUNT = 0, SYNC_THR_PERLOOP = 1 } sync_thr_mode;
+ * producer's engine and K the producer's 1-based rank among them.
+ * PERENGINE: the per-engine allocation of Sec. 6.1 -- one semaphore per
+ * engine counts every retirement on it, so the value is the 1-based position
+ * of the producer's c-th instance in its engine's dynamic instruction stream
+ * (program order), or 0 when c = 0.  PERENGINE thresholds are evaluated and
+ * checked, not simulated. */
+typedef enum { SYNC_THR_COUNT = 0, SYNC_THR_PERLOOP = 1, SYNC_THR_PERENGINE = 2 } sync_thr_mode;
 
 /* Schedules simulated: barrier-free waits only, or the barrier-based scheme
  * of Sec. 3.4 (an all-engine barrier at every loop statement and at the end
@@ -167,9 +172,15 @@ sync_status sync_pair_offsets(const sync_programs *h, int64_t *offsets, int32_t 
  * (iteration counts including the current one, Sec. 5.1) and expr of
  * Sec. 5.2 (r_S - k for a producer in S, r_P for a nested producer, r_P
  * counted through the current / previous S-iteration when forward /
- * backward), in `mode`'s encoding (Eq. 3 or Eq. 5).
+ * backward), in `mode`'s encoding (Eq. 3, Eq. 5 or Sec. 6.1).
  * d_thr: [n_pairs_padded] int32, caller-owned device memory, fully written
- * (padding entries 0). */
+ * (padding entries 0).
+ * The first PERENGINE call (thresholds or check) on a handle derives the
+ * engine-stream positions of the waited producers' instances on the GPU: it
+ * allocates device memory held by the handle (sync_sizes.device_bytes grows)
+ * and synchronizes `stream`; later calls reuse them.  It returns
+ * SYNC_ERR_OVERFLOW if an engine of a program has more than INT32_MAX
+ * instances. */
 sync_status sync_eval_thresholds(const sync_programs *h, sync_thr_mode mode, int32_t *d_thr,
                                  void *stream);
 
@@ -187,7 +198,8 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
                                unsigned long long *d_counts, long long *d_first_bad,
                                void *stream);
 
-/* Schedule simulator.  Runs every program under a timing model of the
+/* Schedule simulator (COUNT and PERLOOP; PERENGINE returns SYNC_ERR_ARG).
+ * Runs every program under a timing model of the
  * paper's execution model: per-engine in-order issue and in-order
  * retirement, waits `semaphore >= threshold` at issue, increments at
  * retirement (Sec. 3.2-3.3, Appendix A.5), counters starting at 0

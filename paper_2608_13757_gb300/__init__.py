@@ -23,7 +23,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libsyncgb.so")
 
 OK, ERR_ARG, ERR_MALFORMED, ERR_NOT_ALLOCATABLE, ERR_OVERFLOW, ERR_CUDA, ERR_OOM = range(7)
-THR_COUNT, THR_PERLOOP = 0, 1
+THR_COUNT, THR_PERLOOP, THR_PERENGINE = 0, 1, 2
 SIM_BARRIER_FREE, SIM_BARRIER = 0, 1
 PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD = 0, 4, 7, 8
 

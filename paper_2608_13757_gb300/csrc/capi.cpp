@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cstring>
 #include <memory>
+#include <mutex>
 #include <new>
 #include <string>
 #include <unordered_map>
@@ -146,6 +147,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<int32_t> plan_ptr;
   std::vector<int4> plan, chunks, lrec, lmeta, lsem[2];
   std::vector<int64_t> seg(ND + 1, 0);
+  std::vector<int64_t> ord_off(NX, -1);   // per instruction: ordinal pool offset (waited producers)
+  int64_t n_ord = 0;
+  bool ord_overflow = false;
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
   std::vector<int64_t> hist_len(2, 0);
@@ -256,6 +260,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       pi.n_inst += tot;
     }
     pi.agg_lat = agg > (__int128)INT64_MAX ? INT64_MAX : (int64_t)agg;
+    {
+      std::vector<int64_t> per_engine(ne, 0);
+      for (int32_t x = 0; x < nx; ++x) per_engine[d.instr_engine[x0 + x]] += S.total[d.instr_loop[x0 + x]];
+      for (int64_t c : per_engine) if (c > kI32Max) ord_overflow = true;
+    }
     for (int32_t l = 1; l < nl; ++l) { pi.n_stmt += S.total[par[l]]; pi.n_iter += S.total[l]; }
     S.x_ndeps.assign(nx, 0);
     S.x_dep_begin.assign(nx, d0);
@@ -317,6 +326,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         n_derived += pad4(S.total[Sl]);
       }
       D.tstart = S.tstart_of[Sl];
+      if (ord_off[x0 + px] < 0) {
+        ord_off[x0 + px] = n_ord;
+        n_ord += S.total[Pl];
+      }
+      D.ordp = ord_off[x0 + px];
       D.anc = -1;
       if (D.up > 0) {
         const int64_t key = (int64_t)Cl * nl + Sl;
@@ -545,6 +559,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     h.sz.struct_bytes = sb;
   }
   h.seg_host = seg;
+  h.ord_off_host = std::move(ord_off);
+  h.n_ord = n_ord;
+  h.ord_overflow = ord_overflow;
   h.count_host.resize(ND);
   for (int64_t i = 0; i < ND; ++i) h.count_host[i] = dep[i].total;
   h.n_chunks = n_pairs_padded / kChunk;
@@ -640,23 +657,49 @@ sync_status sync_pair_offsets(const sync_programs* h, int64_t* offsets, int32_t*
 
 static ThrArgs thr_args(const sync_programs* h, sync_thr_mode mode) {
   ThrArgs a;
-  a.dep = h->dep; a.derived = h->derived; a.seg = h->seg; a.tile_first = h->tile_first; a.path = h->path;
-  a.rowptr = h->rowptr; a.pidx = h->pidx; a.n_chunks = h->n_chunks; a.mode = mode;
+  a.dep = h->dep; a.derived = h->derived; a.ord = h->ord; a.seg = h->seg; a.tile_first = h->tile_first;
+  a.path = h->path; a.rowptr = h->rowptr; a.pidx = h->pidx; a.n_chunks = h->n_chunks; a.mode = mode;
   return a;
 }
 
+// thresholds and check: all three encodings
+static void check_thr_mode(sync_thr_mode mode) {
+  if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP && mode != SYNC_THR_PERENGINE)
+    raise(SYNC_ERR_ARG, "unknown threshold mode");
+}
+
+// simulation: the two semaphore allocations the simulator models
 static void check_mode(sync_thr_mode mode) {
+  if (mode == SYNC_THR_PERENGINE) raise(SYNC_ERR_ARG, "per-engine thresholds are evaluated and checked, not simulated");
   if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP) raise(SYNC_ERR_ARG, "unknown threshold mode");
+}
+
+// Per-engine mode: derive the engine-stream positions of the waited
+// producers' instances on first use (kept by the handle).
+static void ensure_ordinals(const sync_programs* h, cudaStream_t s) {
+  std::lock_guard<std::mutex> lock(h->ord_mu);
+  if (h->ord_ready) return;
+  if (h->ord_overflow)
+    raise(SYNC_ERR_OVERFLOW, "an engine of a program has more than INT32_MAX instances: its stream positions do not fit int32");
+  sync_programs* m = const_cast<sync_programs*>(h);
+  int32_t* ord = m->alloc<int32_t>(h->n_ord, "engine-stream positions");
+  int64_t* off = m->upload(h->ord_off_host, s, "engine-stream position offsets");
+  cuda_check(launch_ordinals(h->prog, h->order, h->sz.n_programs, h->ne_max, h->op_ptr, h->ops, h->rowptr, off, ord,
+                             h->num_sms, s), "engine-stream positions");
+  cuda_check(cudaStreamSynchronize(s), "engine-stream positions");
+  h->ord = ord;
+  h->ord_ready = true;
 }
 
 sync_status sync_eval_thresholds(const sync_programs* h, sync_thr_mode mode, int32_t* d_thr,
                                  void* stream) {
   try {
     if (!h) raise(SYNC_ERR_ARG, "handle must not be NULL");
-    check_mode(mode);
+    check_thr_mode(mode);
     if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
     if (reinterpret_cast<uintptr_t>(d_thr) % 16) raise(SYNC_ERR_ARG, "d_thr must be 16-byte aligned");
     cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
+    if (mode == SYNC_THR_PERENGINE) ensure_ordinals(h, static_cast<cudaStream_t>(stream));
     cuda_check(launch_thresholds(thr_args(h, mode), d_thr, h->num_sms, static_cast<cudaStream_t>(stream)),
                "threshold kernel");
     return SYNC_OK;
@@ -669,10 +712,11 @@ sync_status sync_check_minimal(const sync_programs* h, sync_thr_mode mode, const
                                unsigned long long* d_counts, long long* d_first_bad, void* stream) {
   try {
     if (!h || !d_counts || !d_first_bad) raise(SYNC_ERR_ARG, "handle and outputs must not be NULL");
-    check_mode(mode);
+    check_thr_mode(mode);
     if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
     if (reinterpret_cast<uintptr_t>(d_thr) % 16) raise(SYNC_ERR_ARG, "d_thr must be 16-byte aligned");
     cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
+    if (mode == SYNC_THR_PERENGINE) ensure_ordinals(h, static_cast<cudaStream_t>(stream));
     CheckArgs a;
     a.t = thr_args(h, mode);
     a.thr = d_thr;

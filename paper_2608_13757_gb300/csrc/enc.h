@@ -45,6 +45,7 @@ struct alignas(16) DepInfo {
   int64_t s_rowptr;
   int64_t tstart;     // derived pool: first iteration of the trip, per iteration of S
   int64_t anc;        // derived pool: enclosing S-iteration per consumer iteration (up > 0)
+  int64_t ordp;       // ordinal pool: engine-stream position per producer instance
   int32_t total;      // consumer instances (= total of the consumer's loop)
   int32_t up;
   int32_t clen;
@@ -129,6 +130,7 @@ struct alignas(16) DeriveJob {
 struct ThrArgs {
   const DepInfo* dep;
   const int32_t* derived;
+  const int32_t* ord;        // per-engine mode: engine-stream positions (ordinal pool)
   const int64_t* seg;        // [n_deps + 1] segment offsets
   const int32_t* tile_first; // [n_tiles + 1]
   const int64_t* path;
@@ -216,6 +218,13 @@ cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const 
 cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
                           const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,
                           int num_sms, cudaStream_t s);
+// Per-engine allocation (Sec. 6.1): ord[ord_off[x] + g] = 1-based position of
+// instruction x's instance at global iteration g of its loop in its engine's
+// dynamic stream, for every x with ord_off[x] >= 0; one thread per (program,
+// engine) walks that engine's op rows in program order.
+cudaError_t launch_ordinals(const ProgInfo* prog, const int32_t* order, int32_t n_programs, int32_t ne_max,
+                            const int32_t* op_ptr, const int4* ops, const int32_t* rowptr,
+                            const int64_t* ord_off, int32_t* ord, int num_sms, cudaStream_t s);
 cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s);
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s);
 cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStream_t s);

@@ -1,6 +1,7 @@
 // The handle behind sync_programs (internal to the library).
 #pragma once
 
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -29,6 +30,14 @@ struct sync_programs {
   int32_t* tile_first = nullptr;
   int64_t* path = nullptr;
   int32_t* derived = nullptr;       // per-iteration trip starts and S-ancestors
+  // per-engine mode, derived on first use: engine-stream positions of the
+  // waited producers' instances
+  mutable std::mutex ord_mu;
+  mutable int32_t* ord = nullptr;
+  mutable bool ord_ready = false;
+  int64_t n_ord = 0;
+  bool ord_overflow = false;        // an engine of a program has > INT32_MAX instances
+  std::vector<int64_t> ord_off_host;  // per instruction: pool offset or -1
   int64_t n_chunks = 0;
   // simulator encoding
   syncgb::ProgInfo* prog = nullptr;
@@ -79,6 +88,11 @@ struct sync_programs {
     if (!v.empty()) syncgb::cuda_or_raise(cudaMemcpyAsync(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice, s), what);
     sz.h2d_bytes += (int64_t)(v.size() * sizeof(T));
     return static_cast<T*>(p);
+  }
+  // device memory the handle frees (mutable: lazily derived tables)
+  template <class T>
+  T* alloc_lazy(int64_t n, const char* what) const {
+    return const_cast<sync_programs*>(this)->alloc<T>(n, what);
   }
   template <class T>
   T* alloc(int64_t n, const char* what) {

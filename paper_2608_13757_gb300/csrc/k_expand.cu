@@ -1,5 +1,6 @@
 // Load-time expansion of the trip prefix sums into parent-iteration indices,
-// and the derived per-iteration arrays of the threshold kernels.
+// the derived per-iteration arrays of the threshold kernels, and (on first
+// per-engine use) the engine-stream positions of producer instances.
 //
 // For every loop l and every global iteration g of l, pidx_l[g] is the
 // parent's global iteration j with rowptr_l[j] <= g < rowptr_l[j+1] (the CSR
@@ -64,7 +65,68 @@ k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_jo
   }
 }
 
+// One thread per (program, engine), programs in descending-work order:
+// walk the engine's op rows (its own instructions and the child-loop
+// statements of each loop body, in body order) through every iteration,
+// counting the engine's instances.
+__global__ void __launch_bounds__(kThreads)
+k_ordinals(const ProgInfo* __restrict__ prog, const int32_t* __restrict__ order, int32_t n_programs,
+           int32_t ne_max, const int32_t* __restrict__ op_ptr, const int4* __restrict__ ops,
+           const int32_t* __restrict__ rowptr, const int64_t* __restrict__ ord_off,
+           int32_t* __restrict__ ord) {
+  struct Frame { int32_t row, pos, g, g_end; };
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  const int64_t n = (int64_t)n_programs * ne_max;
+  for (int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x; t < n; t += stride) {
+    const int32_t p = order[t / ne_max], e = (int32_t)(t % ne_max);
+    const ProgInfo pi = prog[p];
+    if (e >= pi.ne) continue;
+    Frame st[SYNC_MAX_DEPTH + 1];
+    int sp = 0;
+    int32_t row = pi.le_base + e, pos = op_ptr[row], g = 0, g_end = 1, count = 0;
+    for (;;) {
+      const int4 op = ops[pos];
+      if (op.x >= 0) {                              // a datapath instance of this engine
+        ++count;
+        const int64_t o = ord_off[op.x];
+        if (o >= 0) ord[o + g] = count;
+        ++pos;
+      } else if (op.x == OP_LOOP) {                 // a child loop statement
+        const int64_t rp = ((int64_t)(uint32_t)op.w << 32) | (uint32_t)op.z;
+        const int32_t lo = rowptr[rp + g], hi = rowptr[rp + g + 1];
+        ++pos;
+        if (lo < hi) {
+          st[sp++] = Frame{row, pos, g, g_end};
+          row = op.y + e;
+          pos = op_ptr[row];
+          g = lo;
+          g_end = hi;
+        }
+      } else if (++g < g_end) {                     // end of an iteration: the next one
+        pos = op_ptr[row];
+      } else if (sp > 0) {                          // end of the loop: back to the parent
+        const Frame f = st[--sp];
+        row = f.row; pos = f.pos; g = f.g; g_end = f.g_end;
+      } else {
+        break;                                      // the top-level loop runs once
+      }
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_ordinals(const ProgInfo* prog, const int32_t* order, int32_t n_programs, int32_t ne_max,
+                            const int32_t* op_ptr, const int4* ops, const int32_t* rowptr,
+                            const int64_t* ord_off, int32_t* ord, int num_sms, cudaStream_t s) {
+  const int64_t n = (int64_t)n_programs * ne_max;
+  if (n == 0) return cudaSuccess;
+  const int64_t want = (n + kThreads - 1) / kThreads;
+  const int64_t cap = (int64_t)num_sms * 8;
+  const int grid = (int)(want < cap ? want : cap);
+  k_ordinals<<<grid, kThreads, 0, s>>>(prog, order, n_programs, ne_max, op_ptr, ops, rowptr, ord_off, ord);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
                           const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,

@@ -56,6 +56,8 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
                                              void* stream) {
   using namespace syncgb;
   if (!h || !params) return set_error(SYNC_ERR_ARG, "handle and params must not be NULL");
+  if (mode == SYNC_THR_PERENGINE)
+    return set_error(SYNC_ERR_ARG, "per-engine thresholds are evaluated and checked, not simulated");
   if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP) return set_error(SYNC_ERR_ARG, "unknown threshold mode");
   if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER) return set_error(SYNC_ERR_ARG, "unknown variant");
   if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))

@@ -44,9 +44,13 @@ __device__ __forceinline__ int32_t count_down(const ThrArgs& a, const DepInfo& D
   return x;
 }
 
-__device__ __forceinline__ int32_t encode(const DepInfo& D, int32_t c, int mode) {
-  // Eq. (5): N*c - (N-K) for the per-(loop, engine) semaphore; 0 stays 0.
-  return (mode == SYNC_THR_PERLOOP && c != 0) ? D.N * c - (D.N - D.K) : c;
+__device__ __forceinline__ int32_t encode(const ThrArgs& a, const DepInfo& D, int32_t c, int mode) {
+  if (c == 0) return 0;
+  // Eq. (5): N*c - (N-K) for the per-(loop, engine) semaphore
+  if (mode == SYNC_THR_PERLOOP) return D.N * c - (D.N - D.K);
+  // Sec. 6.1: the c-th producer instance's position in its engine's stream
+  if (mode == SYNC_THR_PERENGINE) return __ldg(a.ord + D.ordp + (c - 1));
+  return c;
 }
 
 // The paper's register form (Sec. 5.1-5.3): r_S = gs + 1 and r-hat_S = gs -
@@ -61,7 +65,7 @@ __device__ __forceinline__ int32_t wait_value(const ThrArgs& a, const DepInfo& D
   int32_t expr;
   if (D.kase == CASE_PS) expr = gs + 1 - D.k;
   else expr = count_down(a, D, D.kase == CASE_NEST_FWD ? gs + 1 : gs);
-  return encode(D, expr, mode);
+  return encode(a, D, expr, mode);
 }
 
 // Eq. (1) directly, without the case split: the consumer's 1-based position
@@ -74,7 +78,7 @@ __device__ __forceinline__ int32_t minimum(const ThrArgs& a, const DepInfo& D, i
   const int32_t tS = gs - start + 1 - D.k;
   if (tS <= 0) return 0;
   const int32_t gt = start + tS - 1;
-  return encode(D, count_down(a, D, gt + 1), mode);
+  return encode(a, D, count_down(a, D, gt + 1), mode);
 }
 
 template <bool CHECK>
@@ -197,7 +201,9 @@ cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaS
     kern<<<grid, kThreads, 0, s>>>(a, thr);
     return cudaGetLastError();
   };
-  return a.mode == SYNC_THR_PERLOOP ? run(k_thresholds<SYNC_THR_PERLOOP>) : run(k_thresholds<SYNC_THR_COUNT>);
+  if (a.mode == SYNC_THR_PERLOOP) return run(k_thresholds<SYNC_THR_PERLOOP>);
+  if (a.mode == SYNC_THR_PERENGINE) return run(k_thresholds<SYNC_THR_PERENGINE>);
+  return run(k_thresholds<SYNC_THR_COUNT>);
 }
 
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s) {
@@ -211,7 +217,9 @@ cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s) {
     kern<<<grid, kThreads, 0, s>>>(a);
     return cudaGetLastError();
   };
-  return a.t.mode == SYNC_THR_PERLOOP ? run(k_check<SYNC_THR_PERLOOP>) : run(k_check<SYNC_THR_COUNT>);
+  if (a.t.mode == SYNC_THR_PERLOOP) return run(k_check<SYNC_THR_PERLOOP>);
+  if (a.t.mode == SYNC_THR_PERENGINE) return run(k_check<SYNC_THR_PERENGINE>);
+  return run(k_check<SYNC_THR_COUNT>);
 }
 
 }  // namespace syncgb

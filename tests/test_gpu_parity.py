@@ -129,6 +129,46 @@ def test_checker_planted_errors(sg, mode):
     assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
 
 
+# ------------------------------------------------- per-engine allocation
+
+@pytest.mark.parametrize("name,n", [("small", None), ("depth2", 48), ("gemm", None),
+                                    ("attention", 2), ("chain", 400), ("syncbound", 400)])
+def test_perengine_thresholds_bit_exact(sg, name, n):
+    """Sec. 6.1 thresholds (engine-stream position of the c-th producer
+    instance) equal the oracle's, and the checker finds them minimal."""
+    batch = workloads.generate(name, n_programs=n)
+    h = sg.sync_load_programs(batch)
+    thr, got = gpu_thresholds(sg, h, oracle.PERENGINE)
+    assert np.array_equal(got, oracle.thresholds(batch, oracle.PERENGINE))
+    counts, fb = sg.sync_check_minimal(h, sg.THR_PERENGINE, thr)
+    assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
+    # the derived positions are kept: a second call gives the same values
+    thr2, got2 = gpu_thresholds(sg, h, oracle.PERENGINE)
+    assert np.array_equal(got2, got)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_perengine_random_trees(sg, seed):
+    batch = workloads.random_trees(2000 + seed, 200, workloads.tree_params(
+        engines_hi=6, loops_hi=6, body_hi=6, trip_hi=4, max_depth=4))
+    h = sg.sync_load_programs(batch)
+    _, got = gpu_thresholds(sg, h, oracle.PERENGINE)
+    assert np.array_equal(got, oracle.thresholds(batch, oracle.PERENGINE))
+
+
+def test_perengine_checker_planted_errors(sg):
+    test_checker_planted_errors(sg, oracle.PERENGINE)
+
+
+def test_perengine_is_not_simulated(sg):
+    batch = workloads.generate("small")
+    h = sg.sync_load_programs(batch)
+    thr = sg.sync_eval_thresholds(h, sg.THR_PERENGINE)
+    with pytest.raises(sg.SyncError) as err:
+        sg.sync_simulate(h, sg.THR_PERENGINE, thr)
+    assert err.value.status == sg.ERR_ARG
+
+
 def test_checker_detects_swapped_encoding(sg):
     """Count-mode values read as per-loop values are below the minimum wherever
     N > 1 and c > 0."""
