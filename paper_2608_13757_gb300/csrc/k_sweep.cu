@@ -354,6 +354,10 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
   int32_t ts = 0, lrs = 0, ns = 0;
   if (lane < pi.ne) { ts = S.t[lane]; lrs = S.lr[lane]; ns = S.nn[lane]; }
 
+  // barrier scheme: relative schedule of the last fully computed iteration
+  bool rep = false;
+  int32_t rd_issue = 0, rd_retire = 0, rd_t = 0, rd_r = 0, rk0 = 0, rk1 = 0;
+
   const int32_t P = (BB ? 0 : L.rec.z * cwait) + ((L.meta.w & LANE_ITER_START) ? iter_cost : 0);
   const int32_t A = P + ii;                           // cursor advance of a valid lane with no wait
   int32_t T0n = 0, T1n = 0;
@@ -382,61 +386,85 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     // barrier that ended the last iteration or opened the loop, so that wait
     // never binds)
     int32_t known = kNeg;
-    int src0 = -1, src1 = -1;
+    int k0 = 0, k1 = 0;                               // in-chunk increment waited on (1-based), or 0
     bool fallback = false;
     if (valid && T0 > 0) {
       if (T0 <= pub0) {
         if (!BB) known = pub0 - T0 <= S.rmask ? ring0[(T0 - 1) & S.rmask] : a.hist[hist0 + T0];
       } else {
-        const unsigned m = wg0 & vm;
-        const int k = T0 - pub0;
-        if (k > __popc(m)) fallback = true; else src0 = S.rank_lane[L.sm[0] * 32 + k - 1];
+        k0 = T0 - pub0;
+        if (k0 > __popc(wg0 & vm)) fallback = true;
       }
     }
     if (valid && T1 > 0) {
       if (T1 <= pub1) {
         if (!BB) known = max(known, pub1 - T1 <= S.rmask ? ring1[(T1 - 1) & S.rmask] : a.hist[hist1 + T1]);
       } else {
-        const unsigned m = wg1 & vm;
-        const int k = T1 - pub1;
-        if (k > __popc(m)) fallback = true; else src1 = S.rank_lane[L.sm[kMaxDeps > 1 ? 1 : 0] * 32 + k - 1];
+        k1 = T1 - pub1;
+        if (k1 > __popc(wg1 & vm)) fallback = true;
       }
     }
-    const unsigned intra = __ballot_sync(kFull, src0 >= 0 || src1 >= 0);
     if (__ballot_sync(kFull, fallback)) return SIM_FALLBACK;
 
-    const int32_t Av = valid ? A : 0;
-    int32_t r_intra = kNeg;
-    int32_t issue = 0, retire = 0, t_after = 0;
-    const int passes = intra ? ch.y + 2 : 1;
-    bool settled = false;
-    for (int pass = 0; pass < passes; ++pass) {
-      const int32_t ready = max(known, r_intra);
-      // segmented scan of t' = max(t + A, B), B = ready + ii: issue = t' - ii
-      int32_t Ai = Av, Bi = (valid && ready >= 0) ? ready + ii : kNeg;
+    int32_t issue = 0, retire = 0, t_last = 0, r_last = 0;
+    // barrier scheme: every engine starts the iteration at the same cursor
+    // `base` with everything earlier retired, and only in-chunk waits can
+    // bind, so an iteration whose waits target the same in-chunk increments
+    // as the last fully computed one has that iteration's schedule shifted
+    // by the difference of the bases
+    const int32_t base = BB ? __shfl_sync(kFull, ts, 0) : 0;
+    if (BB && rep && !__ballot_sync(kFull, k0 != rk0 || k1 != rk1)) {
+      issue = base + rd_issue;
+      retire = base + rd_retire;
+      t_last = base + rd_t;
+      r_last = base + rd_r;
+    } else {
+      const int src0 = k0 > 0 ? S.rank_lane[L.sm[0] * 32 + k0 - 1] : -1;
+      const int src1 = k1 > 0 ? S.rank_lane[L.sm[kMaxDeps > 1 ? 1 : 0] * 32 + k1 - 1] : -1;
+      const unsigned intra = __ballot_sync(kFull, src0 >= 0 || src1 >= 0);
+      const int32_t Av = valid ? A : 0;
+      int32_t r_intra = kNeg, t_after = 0;
+      const int passes = intra ? ch.y + 2 : 1;
+      bool settled = false;
+      for (int pass = 0; pass < passes; ++pass) {
+        const int32_t ready = max(known, r_intra);
+        // segmented scan of t' = max(t + A, B), B = ready + ii: issue = t' - ii
+        int32_t Ai = Av, Bi = (valid && ready >= 0) ? ready + ii : kNeg;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int32_t Ap = __shfl_up_sync(kFull, Ai, o), Bp = __shfl_up_sync(kFull, Bi, o);
-        if (lane - o >= head) { Bi = max(Bp + Ai, Bi); Ai += Ap; }
-      }
-      t_after = max(t_in + Ai, Bi);
-      issue = t_after - ii;
-      // in-order retirement: segmented max-scan of issue + latency
-      int32_t rv = valid ? issue + lat : kNeg;
+        for (int o = 1; o < 32; o <<= 1) {
+          const int32_t Ap = __shfl_up_sync(kFull, Ai, o), Bp = __shfl_up_sync(kFull, Bi, o);
+          if (lane - o >= head) { Bi = max(Bp + Ai, Bi); Ai += Ap; }
+        }
+        t_after = max(t_in + Ai, Bi);
+        issue = t_after - ii;
+        // in-order retirement: segmented max-scan of issue + latency
+        int32_t rv = valid ? issue + lat : kNeg;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int32_t vp = __shfl_up_sync(kFull, rv, o);
-        if (lane - o >= head) rv = max(rv, vp);
+        for (int o = 1; o < 32; o <<= 1) {
+          const int32_t vp = __shfl_up_sync(kFull, rv, o);
+          if (lane - o >= head) rv = max(rv, vp);
+        }
+        retire = max(lr_in, rv);
+        if (!intra) { settled = true; break; }
+        const int32_t p0 = __shfl_sync(kFull, retire, src0 < 0 ? lane : src0);
+        const int32_t p1 = __shfl_sync(kFull, retire, src1 < 0 ? lane : src1);
+        const int32_t nr = max(src0 < 0 ? kNeg : p0, src1 < 0 ? kNeg : p1);
+        if (!__ballot_sync(kFull, valid && nr > issue)) { settled = true; break; }   // binds nowhere
+        r_intra = nr;
       }
-      retire = max(lr_in, rv);
-      if (!intra) { settled = true; break; }
-      const int32_t p0 = __shfl_sync(kFull, retire, src0 < 0 ? lane : src0);
-      const int32_t p1 = __shfl_sync(kFull, retire, src1 < 0 ? lane : src1);
-      const int32_t nr = max(src0 < 0 ? kNeg : p0, src1 < 0 ? kNeg : p1);
-      if (!__ballot_sync(kFull, valid && nr > issue)) { settled = true; break; }   // binds nowhere
-      r_intra = nr;
+      if (!settled) return SYNC_PROG_DEADLOCK;
+      t_last = __shfl_sync(kFull, t_after, my_last);
+      r_last = __shfl_sync(kFull, retire, my_last);
+      if (BB) {                                       // the reference for the next iterations
+        rd_issue = issue - base;
+        rd_retire = retire - base;
+        rd_t = t_last - base;
+        rd_r = r_last - base;
+        rk0 = k0;
+        rk1 = k1;
+        rep = true;
+      }
     }
-    if (!settled) return SYNC_PROG_DEADLOCK;
 
     // publish
     if (valid && prod_lane) {
@@ -455,7 +483,6 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     pub0 += __popc(wg0 & vm);
     pub1 += __popc(wg1 & vm);
     own_pub += __popc(own_grp & vm);
-    const int32_t t_last = __shfl_sync(kFull, t_after, my_last), r_last = __shfl_sync(kFull, retire, my_last);
     if (present) {
       ts = t_last;
       lrs = r_last;
