@@ -171,6 +171,17 @@ static void bb_emit(bbuild *B, pbuild *b, rng_t *tr) {
 
 /* 1 program, 2 engines (PE=0, DMA=1), one loop of trip 16, 6-instruction
  * body, 3 cross-engine deps, one of them loop-carried at distance 1. */
+/* An instruction with a drawn engine and then a drawn latency.  Each draw is
+ * its own statement: the order of evaluation of a call's arguments is
+ * unspecified in C, so two draws in one argument list would give different
+ * programs on different compilers or targets. */
+static int32_t pb_instr_drawn(pbuild *b, int32_t loop, int32_t pos, rng_t *r, int32_t e_lo, int32_t e_hi,
+                              int32_t lat_lo, int32_t lat_hi) {
+  const int32_t e = rng_uni(r, e_lo, e_hi);
+  const int32_t lat = rng_uni(r, lat_lo, lat_hi);
+  return pb_instr(b, loop, pos, e, lat);
+}
+
 static void gen_small(pbuild *b, rng_t *r) {
   enum { PE = 0, DMA = 1 };
   pb_init(b, 2);
@@ -193,10 +204,10 @@ static void gen_depth2(pbuild *b, rng_t *r) {
   pb_init(b, 4);
   int32_t A = pb_loop(b, 0, 0, TRIP_UNIFORM, 1, 64);
   int32_t a[16], bx[16];
-  for (int i = 0; i < 8; ++i) a[i] = pb_instr(b, A, i, rng_uni(r, 0, 3), rng_uni(r, 1, 256));
+  for (int i = 0; i < 8; ++i) a[i] = pb_instr_drawn(b, A, i, r, 0, 3, 1, 256);
   int32_t B = pb_loop(b, A, 8, TRIP_UNIFORM, 1, 64);
-  for (int i = 8; i < 16; ++i) a[i] = pb_instr(b, A, i + 1, rng_uni(r, 0, 3), rng_uni(r, 1, 256));
-  for (int i = 0; i < 16; ++i) bx[i] = pb_instr(b, B, i, rng_uni(r, 0, 3), rng_uni(r, 1, 256));
+  for (int i = 8; i < 16; ++i) a[i] = pb_instr_drawn(b, A, i + 1, r, 0, 3, 1, 256);
+  for (int i = 0; i < 16; ++i) bx[i] = pb_instr_drawn(b, B, i, r, 0, 3, 1, 256);
   /* B body: 6 same-iteration deps (producer earlier), 2 carried at 1..2 */
   for (int i = 0; i < 6; ++i) {
     int32_t c = rng_uni(r, 1, 15), p = rng_uni(r, 0, c - 1);
@@ -214,14 +225,21 @@ static void gen_depth2(pbuild *b, rng_t *r) {
       int32_t c = rng_uni(r, 1, 15), p = rng_uni(r, 0, c - 1);
       pb_dep(b, a[p], a[c], 0);
     } else {
-      pb_dep(b, bx[rng_uni(r, 0, 15)], a[rng_uni(r, 8, 15)], 0);
+      const int32_t pi = rng_uni(r, 0, 15);
+      const int32_t ci = rng_uni(r, 8, 15);
+      pb_dep(b, bx[pi], a[ci], 0);
     }
   }
   for (int i = 0; i < 2; ++i) {
     if (rng_uni(r, 0, 1)) {
-      pb_dep(b, a[rng_uni(r, 0, 15)], a[rng_uni(r, 0, 15)], rng_uni(r, 1, 2));
+      const int32_t pi = rng_uni(r, 0, 15);
+      const int32_t ci = rng_uni(r, 0, 15);
+      const int32_t k = rng_uni(r, 1, 2);
+      pb_dep(b, a[pi], a[ci], k);
     } else {
-      pb_dep(b, bx[rng_uni(r, 0, 15)], a[rng_uni(r, 0, 7)], 1);
+      const int32_t pi = rng_uni(r, 0, 15);
+      const int32_t ci = rng_uni(r, 0, 7);
+      pb_dep(b, bx[pi], a[ci], 1);
     }
   }
 }
@@ -328,7 +346,7 @@ static void gen_chain(pbuild *b, rng_t *r) {
     first[i + 1] = first[i] + nb[i];
     for (int j = 0; j < nb[i]; ++j) {
       int32_t pos = (i < d && j >= lev_child_pos[i]) ? j + 1 : j;
-      pb_instr(b, lev_loop[i], pos, rng_uni(r, 0, ne - 1), rng_uni(r, 1, 256));
+      (void)pb_instr_drawn(b, lev_loop[i], pos, r, 0, ne - 1, 1, 256);
     }
   }
   int32_t nx = first[d + 1];
@@ -442,7 +460,7 @@ static void gen_tree(pbuild *b, rng_t *r, const synth_tree_params *p) {
   for (int32_t l = 0; l < nloops; ++l)
     for (int32_t i = 0; i < nbody[l]; ++i) {
       int32_t pos = 3 * slots[l][used[l]++] + rng_uni(r, 0, 2);
-      pb_instr(b, l, pos, rng_uni(r, 0, ne - 1), rng_uni(r, p->lat_lo, p->lat_hi));
+      (void)pb_instr_drawn(b, l, pos, r, 0, ne - 1, p->lat_lo, p->lat_hi);
     }
   int32_t nx = (int32_t)b->xl.n;
   /* dependencies */
