@@ -314,27 +314,23 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
   set_groups(S, L, lane, have, copies, ctag);
   uint32_t wg0 = 0, wg1 = 0;
   int32_t pub0 = 0, pub1 = 0;
-  const int32_t* ring0 = S.ring;
-  const int32_t* ring1 = S.ring;
-  int64_t hist0 = 0, hist1 = 0;                       // history offsets of increment 1 minus 1
+  int32_t ring0 = 0, ring1 = 0;                       // ring rows of the waited semaphores
   if (ndep > 0) {
     const int32_t s = L.sm[0];
     wg0 = S.tag[s] == ctag ? S.grp[s] : 0u;
     pub0 = S.semv[s];
-    ring0 = S.ring + s * (S.rmask + 1);
-    hist0 = S.semhb[s] - 1;
+    ring0 = s * (S.rmask + 1);
   }
   if (ndep > 1) {
     const int32_t s = L.sm[kMaxDeps > 1 ? 1 : 0];
     wg1 = S.tag[s] == ctag ? S.grp[s] : 0u;
     pub1 = S.semv[s];
-    ring1 = S.ring + s * (S.rmask + 1);
-    hist1 = S.semhb[s] - 1;
+    ring1 = s * (S.rmask + 1);
   }
   const bool prod_lane = have && L.sr.x >= 0;
   const uint32_t own_grp = prod_lane ? S.grp[L.sr.x] : 0u;
   int32_t own_pub = prod_lane ? S.semv[L.sr.x] : 0;
-  int32_t* own_ring = S.ring + (prod_lane ? L.sr.x : 0) * (S.rmask + 1);
+  const int32_t own_ring = (prod_lane ? L.sr.x : 0) * (S.rmask + 1);
   const int64_t own_hist = prod_lane ? S.semhb[L.sr.x] - 1 : 0;
   const int32_t own_stride = L.sr.y, own_koff = L.sr.z;
   int64_t tl_off = 0;
@@ -390,7 +386,8 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     bool fallback = false;
     if (valid && T0 > 0) {
       if (T0 <= pub0) {
-        if (!BB) known = pub0 - T0 <= S.rmask ? ring0[(T0 - 1) & S.rmask] : a.hist[hist0 + T0];
+        if (!BB) known = pub0 - T0 <= S.rmask ? S.ring[ring0 + ((T0 - 1) & S.rmask)]
+                                              : a.hist[S.semhb[L.sm[0]] + (T0 - 1)];
       } else {
         k0 = T0 - pub0;
         if (k0 > __popc(wg0 & vm)) fallback = true;
@@ -398,7 +395,8 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     }
     if (valid && T1 > 0) {
       if (T1 <= pub1) {
-        if (!BB) known = max(known, pub1 - T1 <= S.rmask ? ring1[(T1 - 1) & S.rmask] : a.hist[hist1 + T1]);
+        if (!BB) known = max(known, pub1 - T1 <= S.rmask ? S.ring[ring1 + ((T1 - 1) & S.rmask)]
+                                                         : a.hist[S.semhb[L.sm[kMaxDeps > 1 ? 1 : 0]] + (T1 - 1)]);
       } else {
         k1 = T1 - pub1;
         if (k1 > __popc(wg1 & vm)) fallback = true;
@@ -469,7 +467,7 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     // publish
     if (valid && prod_lane) {
       const int32_t n = own_stride * gl + own_koff;
-      own_ring[(n - 1) & S.rmask] = retire;
+      S.ring[own_ring + ((n - 1) & S.rmask)] = retire;
       a.hist[own_hist + n] = retire;
     }
     if (valid) {
