@@ -65,14 +65,20 @@ typedef enum {
  * PERENGINE: the per-engine allocation of Sec. 6.1 -- one semaphore per
  * engine counts every retirement on it, so the value is the 1-based position
  * of the producer's c-th instance in its engine's dynamic instruction stream
- * (program order), or 0 when c = 0.  PERENGINE thresholds are evaluated and
- * checked, not simulated. */
+ * (program order), or 0 when c = 0. */
 typedef enum { SYNC_THR_COUNT = 0, SYNC_THR_PERLOOP = 1, SYNC_THR_PERENGINE = 2 } sync_thr_mode;
 
 /* Schedules simulated: barrier-free waits only, or the barrier-based scheme
  * of Sec. 3.4 (an all-engine barrier at every loop statement and at the end
  * of every iteration). */
-typedef enum { SYNC_SIM_BARRIER_FREE = 0, SYNC_SIM_BARRIER = 1 } sync_sim_variant;
+/* Simulation variants.  BARRIER_FREE: the thresholds as semaphore waits
+ * (Sec. 5).  BARRIER: all-engine barriers at loop statements and iteration
+ * ends (Sec. 3.4).  UNROLLED: the straight-line program the loops would
+ * unroll to (Sec. 3.3, the unrolled comparison of Sec. 7): per-engine
+ * semaphores with static waits, so no loop-control and no wait-value
+ * operations -- PERENGINE thresholds only.  Its code size is one
+ * instruction per instance (sync_sizes.n_instances). */
+typedef enum { SYNC_SIM_BARRIER_FREE = 0, SYNC_SIM_BARRIER = 1, SYNC_SIM_UNROLLED = 2 } sync_sim_variant;
 
 /* Per-program simulation status (d_status). */
 enum {
@@ -136,6 +142,10 @@ typedef struct {
   int32_t c_wait_ops_count;   /* wait-value ops per dependency, COUNT (3, Table 1) */
   int32_t c_wait_ops_perloop; /* wait-value ops per dependency, PERLOOP (5, Table 1) */
   int32_t c_barrier;          /* all-engine barrier: handshake, reset, handshake */
+  int32_t c_wait_ops_perengine_level; /* PERENGINE: extra ops per wait for every loop
+                                 strictly between the top level and the
+                                 producer's loop (3: the term N_l*(r_l - 1) of
+                                 Sec. 6.1's path sum, O(D) in Table 1) */
 } sync_sim_params;
 
 typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
@@ -198,19 +208,23 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
                                unsigned long long *d_counts, long long *d_first_bad,
                                void *stream);
 
-/* Schedule simulator (COUNT and PERLOOP; PERENGINE returns SYNC_ERR_ARG).
- * Runs every program under a timing model of the
+/* Schedule simulator.  Runs every program under a timing model of the
  * paper's execution model: per-engine in-order issue and in-order
  * retirement, waits `semaphore >= threshold` at issue, increments at
  * retirement (Sec. 3.2-3.3, Appendix A.5), counters starting at 0
- * (Appendix A.6).  Semaphores are per producer instruction (COUNT) or per
- * (loop, engine) (PERLOOP); d_thr holds the thresholds in that encoding
+ * (Appendix A.6).  Semaphores are per producer instruction (COUNT), per
+ * (loop, engine) (PERLOOP) or per engine (PERENGINE, incremented by every
+ * retirement on the engine); d_thr holds the thresholds in that encoding
  * (normally the output of sync_eval_thresholds).  Costs in cycles, per
  * engine cursor t:
  *   loop statement: barrier-free t += c_regop (r-hat := 0); barrier: barrier
  *   iteration start: barrier-free t += c_branch + 2*c_regop; barrier: t += c_branch
  *   iteration end: barrier only: barrier
- *   datapath x: barrier-free t += |D(x)| * c_wait_ops(mode);
+ *   datapath x: barrier-free t += sum over its dependencies of the wait
+ *     ops: c_wait_ops_count (COUNT), c_wait_ops_perloop (PERLOOP), or
+ *     c_wait_ops_perloop + c_wait_ops_perengine_level * (depth of the
+ *     producer's loop - 1, at least 0; the top level has depth 0)
+ *     (PERENGINE);
  *     issue = max(t, times at which the waited semaphores reached their
  *     thresholds); retire = max(issue + latency, previous retire on the
  *     engine); t = issue + ii
@@ -218,6 +232,9 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  *     every engine continues at release
  *   the top-level loop costs nothing; makespan = max over engines of
  *   max(t, last retire).
+ * UNROLLED: as barrier-free with c_branch, c_regop and every wait-op cost
+ * taken as 0 (ii and latencies unchanged); it requires PERENGINE and returns
+ * SYNC_ERR_ARG otherwise.
  * Outputs per program (device, [n_programs]): d_makespan (int32, -1 unless
  * status OK), d_checksum (uint64, 0 unless OK: the sum mod 2^64 over
  * datapath instances of (a << 32) | b in 32-bit arithmetic, a = (issue ^

@@ -25,7 +25,7 @@ _SRC = [os.path.join(_HERE, "oracle.c")]
 _HDR = [os.path.join(_HERE, "oracle.h")]
 
 COUNT, PERLOOP, PERENGINE = 0, 1, 2
-BARRIER_FREE, BARRIER = 0, 1
+BARRIER_FREE, BARRIER, UNROLLED = 0, 1, 2
 CASE_PS, CASE_NEST_FWD, CASE_NEST_BWD, CASE_NONE = 0, 1, 2, 3
 SIM_OK, SIM_OVERFLOW, SIM_DEADLOCK = 0, 4, 7
 
@@ -54,13 +54,16 @@ class _Batch(ctypes.Structure):
 
 class SimParams(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
-        "ii", "c_branch", "c_regop", "c_wait_ops_count", "c_wait_ops_perloop", "c_barrier")]
+        "ii", "c_branch", "c_regop", "c_wait_ops_count", "c_wait_ops_perloop", "c_barrier",
+        "c_wait_ops_perengine_level")]
 
 
 def sim_params(**kw) -> SimParams:
     """Timing-model constants; defaults ii=1, c_branch=1, c_regop=1, 3 / 5 wait
-    ops per dependency (count / per-loop, Table 1), c_barrier=32."""
-    d = dict(ii=1, c_branch=1, c_regop=1, c_wait_ops_count=3, c_wait_ops_perloop=5, c_barrier=32)
+    ops per dependency (count / per-loop, Table 1), c_barrier=32, and 3 more
+    ops per enclosing loop level for a per-engine wait (Sec. 6.1)."""
+    d = dict(ii=1, c_branch=1, c_regop=1, c_wait_ops_count=3, c_wait_ops_perloop=5, c_barrier=32,
+             c_wait_ops_perengine_level=3)
     d.update(kw)
     return SimParams(**d)
 

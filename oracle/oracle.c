@@ -51,7 +51,11 @@
  *                              (branch, r++, r-hat++); barrier: t += c_branch;
  *  - iteration end:            barrier scheme only: an all-engine barrier;
  *  - datapath instruction x with dependency set D(x):
- *      barrier-free: t += |D(x)| * c_wait (per-mode op count);
+ *      barrier-free: t += sum over D(x) of the wait-value ops (Table 1):
+ *        c_wait_ops_count (count), c_wait_ops_perloop (per-loop), or
+ *        c_wait_ops_perloop + c_wait_ops_perengine_level * max(0, depth(P)
+ *        - 1) (per-engine, Sec. 6.1: one N_l*(r_l - 1) term per loop
+ *        strictly between the top level and the producer's loop P);
  *      issue  = max(t, time each waited semaphore reached its threshold);
  *      retire = max(issue + latency, previous retire on this engine);
  *      t = issue + ii;
@@ -59,8 +63,12 @@
  *    max_e a_e + c_barrier (handshake, reset, handshake); every t_e = release;
  *  - the top-level loop has no statement, branch or barrier costs;
  *  - makespan = max over engines of max(t_e, last retire on e).
+ *  - unrolled variant (the straight-line program of Sec. 3.3 the loops would
+ *    unroll to): as barrier-free with no loop statement, iteration start or
+ *    wait-value costs; per-engine semaphores with static waits.
  * A semaphore's value reaches v at the retire time of its v-th increment
- * (increments of one semaphore all come from one engine, in retire order).
+ * (increments of one semaphore all come from one engine, in retire order;
+ * a per-engine semaphore is incremented by every retirement on its engine).
  * Under the barrier scheme the waits stay in place; after a barrier they can
  * only be already satisfied or concern the current barrier interval.
  * Checksum: the sum (mod 2^64) over datapath instances of
@@ -69,8 +77,8 @@
  *   b = (retire ^ (n*0xC2B2AE35 + e)) * 0x27D4EB2F, b ^= b >> 15,
  * where e is the engine and n the instance's 1-based ordinal among engine
  * e's datapath instances.  Status: 4 when the static time bound
- *   sum_x inst(x)*(lat(x)+ii+|D(x)|*c_wait) + E*(stmts*c_regop + iters*(c_branch+2*c_regop))
- * (barrier-free), or
+ *   sum_x inst(x)*(lat(x)+ii+wait ops(x)) + E*(stmts*c_regop + iters*(c_branch+2*c_regop))
+ * (barrier-free; unrolled: without the control and wait terms), or
  *   sum_x inst(x)*(lat(x)+ii) + E*iters*c_branch + (stmts+iters)*c_barrier
  * (barrier scheme) exceeds INT32_MAX; 7 when no engine can make progress
  * before the end; for both, makespan = -1 and checksum = 0.
@@ -681,7 +689,8 @@ typedef struct {
   prog_t *P;
   const orc_sim_params *prm;
   int mode, barrier;
-  int32_t cwait;
+  int64_t *wcost;              /* per instruction: wait-value ops before issue */
+  int64_t iter_cost, stmt_cost; /* per iteration start / loop statement */
   const int32_t *thr;          /* program's pairs */
   int64_t *pair_off;           /* per dep */
   int32_t *own_sem, *dep_sem;  /* semaphore incremented by x / waited by d */
@@ -715,7 +724,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
     }
     E->bar_passed = 0;
     if (++f->g < f->g_end) {                   /* next iteration starts */
-      E->t += X->barrier ? q->c_branch : q->c_branch + 2 * q->c_regop;
+      E->t += X->iter_cost;
       E->next[f->loop]++;
       f->item = 0;
     } else {
@@ -731,7 +740,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
       return S_BARRIER;
     }
     E->bar_passed = 0;
-    if (!X->barrier) E->t += q->c_regop;
+    if (!X->barrier) E->t += X->stmt_cost;
     int32_t m = -it - 1;
     int32_t trip = P->trips[P->tptr[m] + f->g];
     f->item++;
@@ -740,14 +749,13 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
       c->loop = m; c->item = 0;
       c->g = E->next[m]; c->g_end = c->g + trip;
       E->next[m]++;
-      E->t += X->barrier ? q->c_branch : q->c_branch + 2 * q->c_regop;
+      E->t += X->iter_cost;
     }
     return S_PROGRESS;
   }
   if (P->xe[it] != e) { f->item++; return S_PROGRESS; }
   /* datapath instruction `it` in iteration f->g of its loop */
-  int32_t nd = P->cons_ptr[it + 1] - P->cons_ptr[it];
-  int64_t tw = E->t + (X->barrier ? 0 : (int64_t)nd * X->cwait);
+  int64_t tw = E->t + (X->barrier ? 0 : X->wcost[it]);
   int64_t ready = 0;
   for (int32_t j = P->cons_ptr[it]; j < P->cons_ptr[it + 1]; ++j) {
     int32_t d = P->cons_dep[j];
@@ -779,32 +787,46 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
                        int32_t *issue, int32_t *retire) {
   int32_t nl = P->nl, nx = P->nx, nd = P->nd, ne = P->ne;
   int barrier = variant == ORC_BARRIER;
-  int32_t cwait = mode == ORC_COUNT ? q->c_wait_ops_count : q->c_wait_ops_perloop;
+  int unrolled = variant == ORC_UNROLLED;       /* straight-line: no control or wait-value ops */
+  /* wait-value ops of each dependency (Table 1; per-engine: O(D), Sec. 6.1) */
+  int64_t *wcost = (int64_t *)calloc((size_t)nx + 1, sizeof(int64_t));
+  if (!wcost) return ORC_ERR_OOM;
+  for (int32_t d = 0; d < nd && !unrolled; ++d) {
+    int64_t c = mode == ORC_COUNT ? q->c_wait_ops_count : q->c_wait_ops_perloop;
+    if (mode == ORC_PERENGINE) {
+      int32_t lev = P->depth[P->xl[P->dp[d]]] - 1;
+      c += (int64_t)q->c_wait_ops_perengine_level * (lev > 0 ? lev : 0);
+    }
+    wcost[P->dc[d]] += c;
+  }
+  int64_t iter_cost = unrolled ? 0 : barrier ? q->c_branch : q->c_branch + 2 * (int64_t)q->c_regop;
+  int64_t stmt_cost = unrolled ? 0 : q->c_regop;
   /* the static time bound */
   u128 bound = 0;
   int64_t stmts = 0, iters = 0;
   for (int32_t l = 1; l < nl; ++l) { stmts += P->total[P->par[l]]; iters += P->total[l]; }
   for (int32_t x = 0; x < nx; ++x) {
     int64_t per = (int64_t)P->xlat[x] + q->ii;
-    if (!barrier) per += (int64_t)(P->cons_ptr[x + 1] - P->cons_ptr[x]) * cwait;
+    if (!barrier) per += wcost[x];
     bound += (u128)P->total[P->xl[x]] * (u128)per;
   }
   if (barrier) {
     bound += (u128)ne * (u128)iters * (u128)q->c_branch;
     bound += (u128)(stmts + iters) * (u128)q->c_barrier;
   } else {
-    bound += (u128)ne * ((u128)stmts * (u128)q->c_regop +
-                         (u128)iters * (u128)(q->c_branch + 2 * (int64_t)q->c_regop));
+    bound += (u128)ne * ((u128)stmts * (u128)stmt_cost + (u128)iters * (u128)iter_cost);
   }
   if (bound > (u128)INT32_MAX) {
+    free(wcost);
     *makespan = -1; *checksum = 0; *status = ORC_SIM_OVERFLOW;
     return ORC_OK;
   }
   sim_ctx X;
   memset(&X, 0, sizeof X);
-  X.P = P; X.prm = q; X.mode = mode; X.barrier = barrier; X.cwait = cwait; X.thr = thr;
+  X.P = P; X.prm = q; X.mode = mode; X.barrier = barrier; X.wcost = wcost; X.thr = thr;
+  X.iter_cost = iter_cost; X.stmt_cost = stmt_cost;
   X.issue = issue; X.retire = retire;
-  int32_t nsem = mode == ORC_COUNT ? nx : nl * ne;
+  int32_t nsem = mode == ORC_COUNT ? nx : mode == ORC_PERLOOP ? nl * ne : ne;
   X.pair_off = (int64_t *)malloc(((size_t)nd + 1) * sizeof(int64_t));
   X.inst_off = (int64_t *)malloc(((size_t)nx + 1) * sizeof(int64_t));
   X.own_sem = (int32_t *)malloc(((size_t)nx + 1) * sizeof(int32_t));
@@ -821,12 +843,12 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     off = 0;
     for (int32_t x = 0; x < nx; ++x) {
       X.inst_off[x] = off; off += P->total[P->xl[x]];
-      X.own_sem[x] = mode == ORC_COUNT ? x : P->xl[x] * ne + P->xe[x];
+      X.own_sem[x] = mode == ORC_COUNT ? x : mode == ORC_PERLOOP ? P->xl[x] * ne + P->xe[x] : P->xe[x];
       incs[X.own_sem[x]] += P->total[P->xl[x]];
     }
     for (int32_t d = 0; d < nd; ++d) {
       int32_t p = P->dp[d];
-      X.dep_sem[d] = mode == ORC_COUNT ? p : P->xl[p] * ne + P->xe[p];
+      X.dep_sem[d] = mode == ORC_COUNT ? p : mode == ORC_PERLOOP ? P->xl[p] * ne + P->xe[p] : P->xe[p];
       int32_t s = X.dep_sem[d];
       if (!X.times[s]) {
         X.times[s] = (int64_t *)malloc(((size_t)incs[s] + 1) * sizeof(int64_t));
@@ -881,7 +903,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   for (int32_t e = 0; E && e < ne; ++e) { free(E[e].st); free(E[e].next); }
   for (int32_t s = 0; X.times && s < nsem; ++s) free(X.times[s]);
   free(E); free(incs); free(X.pair_off); free(X.inst_off); free(X.own_sem); free(X.dep_sem);
-  free(X.value); free(X.times);
+  free(X.value); free(X.times); free(wcost);
   return rc;
 }
 
@@ -889,8 +911,9 @@ int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim
                  int variant, int32_t *makespan, uint64_t *checksum, int32_t *status,
                  int32_t *issue, int32_t *retire) {
   if (!b || !thr || !prm || !makespan || !checksum || !status) return ORC_ERR_ARG;
-  if ((mode != ORC_COUNT && mode != ORC_PERLOOP) ||
-      (variant != ORC_BARRIER_FREE && variant != ORC_BARRIER) || (!issue) != (!retire))
+  if ((mode != ORC_COUNT && mode != ORC_PERLOOP && mode != ORC_PERENGINE) ||
+      (variant != ORC_BARRIER_FREE && variant != ORC_BARRIER && variant != ORC_UNROLLED) ||
+      (variant == ORC_UNROLLED && mode != ORC_PERENGINE) || (!issue) != (!retire))
     return ORC_ERR_ARG;
   int64_t pbase = 0, ibase = 0;
   for (int32_t p = 0; p < b->n_programs; ++p) {

@@ -45,8 +45,10 @@ enum { ORC_COUNT = 0, ORC_PERLOOP = 1, ORC_PERENGINE = 2 };
 /* allocatable cases of Sec. 5.2 */
 enum { ORC_CASE_PS = 0, ORC_CASE_NEST_FWD = 1, ORC_CASE_NEST_BWD = 2, ORC_CASE_NONE = 3 };
 
-/* simulator variants and per-program status codes */
-enum { ORC_BARRIER_FREE = 0, ORC_BARRIER = 1 };
+/* simulator variants (UNROLLED: the straight-line program, per-engine
+ * thresholds, no loop-control or wait-value operations) and per-program
+ * status codes */
+enum { ORC_BARRIER_FREE = 0, ORC_BARRIER = 1, ORC_UNROLLED = 2 };
 enum { ORC_SIM_OK = 0, ORC_SIM_OVERFLOW = 4, ORC_SIM_DEADLOCK = 7 };
 
 typedef struct {
@@ -56,6 +58,7 @@ typedef struct {
   int32_t c_wait_ops_count;   /* wait-value ops per dependency, count mode     */
   int32_t c_wait_ops_perloop; /* wait-value ops per dependency, per-loop mode  */
   int32_t c_barrier;          /* all-engine barrier handshake + reset          */
+  int32_t c_wait_ops_perengine_level; /* per-engine mode: per enclosing loop level */
 } orc_sim_params;
 
 /* Sizes: pairs and instances in the layouts above. */
@@ -89,9 +92,11 @@ int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[
 
 /* Event-stepped semaphore machine (timing model stated in oracle.c).  `thr`
  * is a threshold array in `mode`'s encoding; the machine waits on the
- * per-producer semaphore (count) or the per-(loop, engine) semaphore
- * (per-loop) until its value reaches the threshold.  issue/retire may be NULL.
- * Count and per-loop modes only. */
+ * per-producer semaphore (count), the per-(loop, engine) semaphore
+ * (per-loop) or the producer's engine semaphore, which every retirement on
+ * that engine increments (per-engine), until its value reaches the
+ * threshold.  The unrolled variant needs per-engine thresholds.
+ * issue/retire may be NULL. */
 int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim_params *prm,
                  int variant, int32_t *makespan, uint64_t *checksum, int32_t *status,
                  int32_t *issue, int32_t *retire);

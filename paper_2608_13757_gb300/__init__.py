@@ -24,7 +24,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libsyncgb.so")
 
 OK, ERR_ARG, ERR_MALFORMED, ERR_NOT_ALLOCATABLE, ERR_OVERFLOW, ERR_CUDA, ERR_OOM = range(7)
 THR_COUNT, THR_PERLOOP, THR_PERENGINE = 0, 1, 2
-SIM_BARRIER_FREE, SIM_BARRIER = 0, 1
+SIM_BARRIER_FREE, SIM_BARRIER, SIM_UNROLLED = 0, 1, 2
 PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD = 0, 4, 7, 8
 
 # every symbol include/sync.h declares
@@ -61,11 +61,13 @@ class Sizes(ctypes.Structure):
 class SimParams(ctypes.Structure):
     """Timing-model constants (cycles); defaults as in the library's docs."""
     _fields_ = [(n, ctypes.c_int32) for n in (
-        "ii", "c_branch", "c_regop", "c_wait_ops_count", "c_wait_ops_perloop", "c_barrier")]
+        "ii", "c_branch", "c_regop", "c_wait_ops_count", "c_wait_ops_perloop", "c_barrier",
+        "c_wait_ops_perengine_level")]
 
     def __init__(self, ii=1, c_branch=1, c_regop=1, c_wait_ops_count=3, c_wait_ops_perloop=5,
-                 c_barrier=32):
-        super().__init__(ii, c_branch, c_regop, c_wait_ops_count, c_wait_ops_perloop, c_barrier)
+                 c_barrier=32, c_wait_ops_perengine_level=3):
+        super().__init__(ii, c_branch, c_regop, c_wait_ops_count, c_wait_ops_perloop, c_barrier,
+                         c_wait_ops_perengine_level)
 
 
 def load_library(path: str = LIB_PATH) -> ctypes.CDLL:

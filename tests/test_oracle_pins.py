@@ -397,21 +397,45 @@ def _random_batches(n=40, **kw):
         yield seed, workloads.random_trees(seed, 1, workloads.tree_params(**kw))
 
 
-@pytest.mark.parametrize("variant", [oracle.BARRIER_FREE, oracle.BARRIER])
-@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def loop_depths(batch):
+    """Depth of every loop of a one-program batch (top level 0)."""
+    dep = [0] * batch.n_loops
+    for l in range(1, batch.n_loops):
+        dep[l] = dep[int(batch.loop_parent[l])] + 1
+    return dep
+
+
+def wait_ops(batch, mode, prm):
+    """Wait-value ops of each dependency (Table 1): 3 / 5 per wait, and for a
+    per-engine wait one more term per loop strictly between the top level and
+    the producer's loop (Sec. 6.1's path sum)."""
+    if mode == COUNT:
+        return prm.c_wait_ops_count
+    if mode == PERLOOP:
+        return prm.c_wait_ops_perloop
+    dep = loop_depths(batch)
+    lvl = [max(0, dep[int(batch.instr_loop[int(batch.dep_prod[d])])] - 1) for d in range(batch.n_deps)]
+    return lambda d: prm.c_wait_ops_perloop + prm.c_wait_ops_perengine_level * lvl[d]
+
+
+@pytest.mark.parametrize("mode,variant", [(COUNT, oracle.BARRIER_FREE), (COUNT, oracle.BARRIER),
+                                          (PERLOOP, oracle.BARRIER_FREE), (PERLOOP, oracle.BARRIER),
+                                          (PERENGINE, oracle.BARRIER_FREE), (PERENGINE, oracle.BARRIER),
+                                          (PERENGINE, oracle.UNROLLED)])
 def test_timing_matches_recursive_statement(mode, variant):
     """The event-stepped semaphore machine (waits on semaphore values, per
-    mode) and the recursive max-plus statement (waits on the c-th producer
-    retirement) give identical makespans, checksums and timelines."""
-    prm = oracle.sim_params(ii=2, c_branch=3, c_regop=1, c_barrier=7)
-    cwait = prm.c_wait_ops_count if mode == COUNT else prm.c_wait_ops_perloop
+    mode: per producer, per (loop, engine), or per engine counting every
+    retirement) and the recursive max-plus statement (waits on the c-th
+    producer retirement) give identical makespans, checksums and timelines."""
+    prm = oracle.sim_params(ii=2, c_branch=3, c_regop=1, c_barrier=7, c_wait_ops_perengine_level=2)
     n = 0
     for seed, batch in _random_batches(60):
         thr = oracle.thresholds(batch, mode)
         thr_c = oracle.thresholds(batch, COUNT)
         r = oracle.simulate(batch, thr, mode, variant, prm, timeline=True)
         assert r.status[0] == 0
-        ms, chk, tl = timing_model.simulate(batch, thr_c, prm, variant == oracle.BARRIER, cwait)
+        ms, chk, tl = timing_model.simulate(batch, thr_c, prm, variant == oracle.BARRIER,
+                                            wait_ops(batch, mode, prm), unrolled=variant == oracle.UNROLLED)
         assert r.makespan[0] == ms, seed
         assert int(r.checksum[0]) == chk, seed
         off = 0
@@ -422,6 +446,31 @@ def test_timing_matches_recursive_statement(mode, variant):
             off += int(tot[batch.instr_loop[x]])
         n += 1
     assert n == 60
+
+
+def test_unrolled_and_per_engine_cost_order():
+    """Same waits, costs only removed or added (max-plus monotonicity): the
+    unrolled program (no control, no wait ops) is never later than the
+    barrier-free per-loop schedule, which is never later than the per-engine
+    one (at least as many wait ops); with every cost zero all three agree."""
+    prm = oracle.sim_params()
+    zero = oracle.sim_params(c_branch=0, c_regop=0, c_wait_ops_count=0, c_wait_ops_perloop=0,
+                             c_wait_ops_perengine_level=0)
+    deeper = 0
+    for seed, batch in _random_batches(60):
+        t_pl = oracle.thresholds(batch, PERLOOP)
+        t_pe = oracle.thresholds(batch, PERENGINE)
+        un = oracle.simulate(batch, t_pe, PERENGINE, oracle.UNROLLED, prm).makespan[0]
+        pl = oracle.simulate(batch, t_pl, PERLOOP, oracle.BARRIER_FREE, prm).makespan[0]
+        pe = oracle.simulate(batch, t_pe, PERENGINE, oracle.BARRIER_FREE, prm).makespan[0]
+        assert 0 <= un <= pl <= pe, seed
+        z = [oracle.simulate(batch, t_pl, PERLOOP, oracle.BARRIER_FREE, zero).makespan[0],
+             oracle.simulate(batch, t_pe, PERENGINE, oracle.BARRIER_FREE, zero).makespan[0],
+             oracle.simulate(batch, t_pe, PERENGINE, oracle.UNROLLED, zero).makespan[0]]
+        assert z[0] == z[1] == z[2] == un, seed
+        dep = loop_depths(batch)
+        deeper += any(dep[int(batch.instr_loop[int(batch.dep_prod[d])])] >= 2 for d in range(batch.n_deps))
+    assert deeper > 10     # the per-level term is exercised
 
 
 @pytest.mark.parametrize("mode", [COUNT, PERLOOP])

@@ -11,9 +11,11 @@ Events per engine, in program order: a loop statement ("stmt"), an iteration
 start ("iter"), an iteration end ("end", barrier scheme only), and the
 engine's datapath instances.  Costs (barrier-free / barrier scheme):
 stmt c_regop / barrier; iter c_branch + 2*c_regop / c_branch; end - / barrier;
-datapath: t += |D| * c_wait (barrier-free only), issue = max(t, producer
-retirements), retire = max(issue + lat, previous retire), t = issue + ii.
-Barrier j: release = max over engines of max(t, last retire) + c_barrier.
+datapath: t += the wait ops of its dependencies (barrier-free only), issue =
+max(t, producer retirements), retire = max(issue + lat, previous retire),
+t = issue + ii.  Barrier j: release = max over engines of max(t, last
+retire) + c_barrier.  Unrolled (the straight-line program): as barrier-free
+without stmt, iter or wait-op costs.
 """
 import sys
 
@@ -59,8 +61,10 @@ def _events(batch, e, barrier):
     return ev
 
 
-def simulate(batch, thr_count, params, barrier, cwait):
-    """(makespan, checksum, {(x, g): (issue, retire)}) or raises Deadlock."""
+def simulate(batch, thr_count, params, barrier, cwait, unrolled=False):
+    """(makespan, checksum, {(x, g): (issue, retire)}) or raises Deadlock.
+    cwait: wait ops per dependency, an int or a function of the dependency."""
+    wait_ops = cwait if callable(cwait) else (lambda d: cwait)
     ne = int(batch.prog_n_engines[0])
     ev = [_events(batch, e, barrier) for e in range(ne)]
     where = {}
@@ -108,7 +112,7 @@ def simulate(batch, thr_count, params, barrier, cwait):
         if v[0] == "x":
             x, g = v[1], v[2]
             ds = deps_of.get(x, [])
-            tw = t + (0 if barrier else len(ds) * cwait)
+            tw = t + (0 if barrier or unrolled else sum(wait_ops(d) for d in ds))
             ready = 0
             for d in ds:
                 c = int(thr_count[pair_off[d] + g])
@@ -131,7 +135,9 @@ def simulate(batch, thr_count, params, barrier, cwait):
                 rel = max(rel, ft, flr)
             out = (rel + params.c_barrier, lr, None, None)
         elif v[0] == "stmt":
-            out = (t + params.c_regop, lr, None, None)
+            out = (t + (0 if unrolled else params.c_regop), lr, None, None)
+        elif unrolled:  # iteration start of the unrolled program: nothing
+            out = (t, lr, None, None)
         else:  # iteration start
             out = (t + params.c_branch + (0 if barrier else 2 * params.c_regop), lr, None, None)
         busy.discard(key)
