@@ -48,6 +48,20 @@ sync_status set_error(sync_status status, const std::string& msg) {
   return status;
 }
 void cuda_or_raise(cudaError_t e, const char* what) { cuda_check(e, what); }
+
+// Timing constants a variant runs with: the unrolled variant has no loop
+// control and static waits, so it costs neither.
+bool sim_params_for(const sync_sim_params& p, sync_sim_variant variant, sync_sim_params& q) {
+  if (p.ii < 0 || p.c_branch < 0 || p.c_regop < 0 || p.c_wait_ops_count < 0 || p.c_wait_ops_perloop < 0 ||
+      p.c_barrier < 0 || p.c_wait_ops_perengine_level < 0)
+    return false;
+  q = p;
+  if (variant == SYNC_SIM_UNROLLED) {
+    q.c_branch = q.c_regop = 0;
+    q.c_wait_ops_count = q.c_wait_ops_perloop = q.c_wait_ops_perengine_level = 0;
+  }
+  return true;
+}
 }  // namespace syncgb
 
 namespace {
@@ -75,7 +89,7 @@ void check_csr(const int32_t* ptr, int32_t P, const char* name) {
 // Per-program scratch of the loader (reused across programs).
 struct ProgScratch {
   std::vector<int32_t> depth, body_ptr, body, rank, nloop_eng, x_ndeps, x_dep_begin;
-  std::vector<int32_t> x_own[2], x_hstride[2], x_koff[2];
+  std::vector<int32_t> x_own[kModes], x_hstride[kModes], x_koff[kModes], x_levels;
   std::vector<int64_t> total, keys;
   std::vector<int64_t> tstart_of;                 // derived trip-start array per loop, -1 if none
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
@@ -85,7 +99,7 @@ struct ProgScratch {
 // engine-major) with their iteration copies.
 void add_chunk(const sync_batch_desc& d, int32_t x0, const ProgScratch& S, const std::vector<int32_t>& recs,
                const std::vector<int32_t>& copies, int32_t ncopies, std::vector<int4>& chunks,
-               std::vector<int4>& lrec, std::vector<int4>& lmeta, std::vector<int4> (&lsem)[2]) {
+               std::vector<int4>& lrec, std::vector<int4>& lmeta, std::vector<int4> (&lsem)[kModes]) {
   const int32_t base = (int32_t)lrec.size();
   const int32_t n = (int32_t)recs.size();
   int32_t emask = 0;
@@ -99,7 +113,8 @@ void add_chunk(const sync_batch_desc& d, int32_t x0, const ProgScratch& S, const
     const bool first_in_copy = copies[i] > 0 && (i == head || copies[i - 1] != copies[i]);
     lrec.push_back(make_int4(x0 + x, d.instr_latency[x0 + x], S.x_ndeps[x], S.x_dep_begin[x]));
     lmeta.push_back(make_int4(e, copies[i], head, (first_in_copy ? LANE_ITER_START : 0) | (last ? LANE_RUN_LAST : 0)));
-    for (int m = 0; m < 2; ++m) lsem[m].push_back(make_int4(S.x_own[m][x], S.x_hstride[m][x], S.x_koff[m][x], 0));
+    for (int m = 0; m < kModes; ++m)
+      lsem[m].push_back(make_int4(S.x_own[m][x], S.x_hstride[m][x], S.x_koff[m][x], m == 2 ? S.x_levels[x] : 0));
   }
   chunks.push_back(make_int4(base, n, ncopies, emask));
 }
@@ -141,18 +156,18 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<ProgInfo> prog(P);
   std::vector<int32_t> op_ptr, opstop;
   std::vector<int2> rowinfo;
-  std::vector<int4> ops, opsem[2];
+  std::vector<int4> ops, opsem[kModes];
   std::vector<int64_t> inst_off(NX), dseg(ND), semhb;
-  std::vector<int32_t> dsem[2] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
+  std::vector<int32_t> dsem[kModes] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
   std::vector<int32_t> plan_ptr;
-  std::vector<int4> plan, chunks, lrec, lmeta, lsem[2];
+  std::vector<int4> plan, chunks, lrec, lmeta, lsem[kModes];
   std::vector<int64_t> seg(ND + 1, 0);
   std::vector<int64_t> ord_off(NX, -1);   // per instruction: ordinal pool offset (waited producers)
   int64_t n_ord = 0;
   bool ord_overflow = false;
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
-  std::vector<int64_t> hist_len(2, 0);
+  std::vector<int64_t> hist_len(kModes, 0);
   std::vector<uint8_t> reads_rowptr(NL, 0);
   std::vector<DeriveJob> jobs;
   int64_t n_derived = 0;
@@ -268,7 +283,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     for (int32_t l = 1; l < nl; ++l) { pi.n_stmt += S.total[par[l]]; pi.n_iter += S.total[l]; }
     S.x_ndeps.assign(nx, 0);
     S.x_dep_begin.assign(nx, d0);
-    for (int m = 0; m < 2; ++m) { S.x_own[m].assign(nx, -1); S.x_hstride[m].assign(nx, 0); S.x_koff[m].assign(nx, 0); }
+    for (int m = 0; m < kModes; ++m) { S.x_own[m].assign(nx, -1); S.x_hstride[m].assign(nx, 0); S.x_koff[m].assign(nx, 0); }
+    S.x_levels.assign(nx, 0);
     // dependencies: innermost common loop S, cases of Sec. 5.2, N and K
     std::vector<int32_t> by_cons(nd);
     for (int32_t k = 0; k < nd; ++k) by_cons[k] = k;
@@ -364,20 +380,35 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     }
     // semaphores that some dependency waits on, per mode, with their history
     // slots: mode 0 = one per producer instruction (one increment per
-    // iteration); mode 1 = one per (loop, engine) (N increments per iteration)
+    // iteration); mode 1 = one per (loop, engine) (N increments per
+    // iteration); mode 2 = one per engine (one increment per instance of the
+    // engine, numbered by the instance's ordinal)
+    std::vector<int64_t> inst_eng(ne, 0);
+    for (int32_t x = 0; x < nx; ++x) inst_eng[d.instr_engine[x0 + x]] += S.total[d.instr_loop[x0 + x]];
+    auto sem_key = [&](int m, int32_t x) {
+      const int32_t e = d.instr_engine[x0 + x];
+      return m == 0 ? x : m == 1 ? d.instr_loop[x0 + x] * ne + e : e;
+    };
+    // per-engine waits: loops strictly between the top level and the producer's loop
+    auto levels = [&](int32_t px) { return std::max(0, S.depth[d.instr_loop[x0 + px]] - 1); };
+    for (int32_t k = 0; k < nd; ++k) {
+      const int64_t gd = d0 + k;
+      S.x_levels[d.dep_cons[gd]] += levels(d.dep_prod[gd]);
+      pi.pair_levels += (int64_t)levels(d.dep_prod[gd]) * S.total[d.instr_loop[x0 + d.dep_cons[gd]]];
+    }
     std::vector<int32_t> sem_of(std::max(nx, nl * ne), -1);
-    for (int m = 0; m < 2; ++m) {
+    for (int m = 0; m < kModes; ++m) {
       std::fill(sem_of.begin(), sem_of.end(), -1);
       std::vector<int64_t> sem_hist;
       for (int32_t k = 0; k < nd; ++k) {
         const int64_t gd = d0 + k;
         const int32_t px = d.dep_prod[gd];
         const int32_t Pl = d.instr_loop[x0 + px];
-        const int32_t key = m == 0 ? px : Pl * ne + d.instr_engine[x0 + px];
+        const int32_t key = sem_key(m, px);
         if (sem_of[key] < 0) {
           sem_of[key] = (int32_t)sem_hist.size();
           sem_hist.push_back(hist_len[m]);
-          hist_len[m] += (m == 0 ? 1 : dep_N[gd]) * S.total[Pl];
+          hist_len[m] += m == 0 ? S.total[Pl] : m == 1 ? dep_N[gd] * S.total[Pl] : inst_eng[d.instr_engine[x0 + px]];
         }
       }
       pi.nsem[m] = (int32_t)sem_hist.size();
@@ -385,12 +416,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       semhb.insert(semhb.end(), sem_hist.begin(), sem_hist.end());
       for (int32_t x = 0; x < nx; ++x) {
         const int32_t l = d.instr_loop[x0 + x];
-        const int32_t key = m == 0 ? x : l * ne + d.instr_engine[x0 + x];
-        const int32_t s = sem_of[key];
+        const int32_t s = sem_of[sem_key(m, x)];
         S.x_own[m][x] = s;
         if (s < 0) continue;
-        S.x_hstride[m][x] = m == 0 ? 1 : S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]];
-        S.x_koff[m][x] = m == 0 ? 1 : S.rank[x];
+        S.x_hstride[m][x] = m == 0 ? 1 : m == 1 ? S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]] : -1;
+        S.x_koff[m][x] = m == 0 ? 1 : m == 1 ? S.rank[x] : 0;
       }
       // dependencies grouped by consumer (stable by dependency id)
       if (m == 0)
@@ -399,9 +429,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         });
       for (int32_t i = 0; i < nd; ++i) {
         const int64_t gd = d0 + by_cons[i];
-        const int32_t px = d.dep_prod[gd];
-        const int32_t key = m == 0 ? px : d.instr_loop[x0 + px] * ne + d.instr_engine[x0 + px];
-        dsem[m][d0 + i] = sem_of[key];
+        dsem[m][d0 + i] = sem_of[sem_key(m, d.dep_prod[gd])];
         if (m == 0) dseg[d0 + i] = seg[gd];
       }
     }
@@ -421,19 +449,18 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
             const int64_t rp = loop[l0 + m].rowptr_off;
             ops.push_back(make_int4(OP_LOOP, pi.le_base + m * ne, (int32_t)(uint32_t)(rp & 0xffffffffu),
                                     (int32_t)(rp >> 32)));
-            opsem[0].push_back(make_int4(-1, 0, 0, 0));
-            opsem[1].push_back(make_int4(-1, 0, 0, 0));
+            for (int m = 0; m < kModes; ++m) opsem[m].push_back(make_int4(-1, 0, 0, 0));
             has_loop = true;
           } else if (d.instr_engine[x0 + it] == e) {
             ops.push_back(make_int4(x0 + it, d.instr_latency[x0 + it], S.x_ndeps[it], S.x_dep_begin[it]));
-            for (int m = 0; m < 2; ++m)
-              opsem[m].push_back(make_int4(S.x_own[m][it], S.x_hstride[m][it], S.x_koff[m][it], 0));
+            for (int m = 0; m < kModes; ++m)
+              opsem[m].push_back(make_int4(S.x_own[m][it], S.x_hstride[m][it], S.x_koff[m][it],
+                                           m == 2 ? S.x_levels[it] : 0));
           }
         }
         const int32_t end_idx = (int32_t)ops.size();
         ops.push_back(make_int4(OP_END, 0, 0, 0));
-        opsem[0].push_back(make_int4(-1, 0, 0, 0));
-        opsem[1].push_back(make_int4(-1, 0, 0, 0));
+        for (int m = 0; m < kModes; ++m) opsem[m].push_back(make_int4(-1, 0, 0, 0));
         rowinfo.push_back(make_int2(end_idx, has_loop ? 1 : 0));
         // next LOOP or END record at or after each record of the row
         opstop.resize(ops.size());
@@ -485,8 +512,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         add_chunk(d, x0, S, recs, copies, k, chunks, lrec, lmeta, lsem);
       }
     }
-    h.nsem_max[0] = std::max(h.nsem_max[0], pi.nsem[0]);
-    h.nsem_max[1] = std::max(h.nsem_max[1], pi.nsem[1]);
+    for (int m = 0; m < kModes; ++m) h.nsem_max[m] = std::max(h.nsem_max[m], pi.nsem[m]);
     h.ne_max = std::max(h.ne_max, ne);
     h.depth_max = std::max(h.depth_max, depth_max);
     if ((int64_t)ops.size() > kI32Max) raise(SYNC_ERR_OVERFLOW, "op records exceed INT32_MAX entries");
@@ -589,19 +615,18 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.opstop = h.upload(opstop, stream, "op stops");
   {
     std::vector<int4> both(opsem[0]);
-    both.insert(both.end(), opsem[1].begin(), opsem[1].end());
+    for (int m = 1; m < kModes; ++m) both.insert(both.end(), opsem[m].begin(), opsem[m].end());
     h.opsem = h.upload(both, stream, "op semaphore records");
     std::vector<int32_t> dboth(dsem[0]);
-    dboth.insert(dboth.end(), dsem[1].begin(), dsem[1].end());
+    for (int m = 1; m < kModes; ++m) dboth.insert(dboth.end(), dsem[m].begin(), dsem[m].end());
     h.dsem = h.upload(dboth, stream, "dependency semaphores");
   }
   h.n_ops = (int64_t)ops.size();
   h.dseg = h.upload(dseg, stream, "dependency segments");
   h.semhb = h.upload(semhb, stream, "semaphore history bases");
   h.inst_off = h.upload(inst_off, stream, "instance offsets");
-  h.hist = h.alloc<int32_t>(std::max(hist_len[0], hist_len[1]), "semaphore history");
-  h.hist_len[0] = hist_len[0];
-  h.hist_len[1] = hist_len[1];
+  h.hist = h.alloc<int32_t>(*std::max_element(hist_len.begin(), hist_len.end()), "semaphore history");
+  for (int m = 0; m < kModes; ++m) h.hist_len[m] = hist_len[m];
   h.next_slot = h.alloc<int32_t>(1, "program-slot counter");
   h.fallback = h.alloc<int32_t>((int64_t)P + 1, "fallback list");
   h.plan_ptr = h.upload(plan_ptr, stream, "sweep plan offsets");
@@ -611,7 +636,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.lmeta = h.upload(lmeta, stream, "sweep lane meta");
   {
     std::vector<int4> both(lsem[0]);
-    both.insert(both.end(), lsem[1].begin(), lsem[1].end());
+    for (int m = 1; m < kModes; ++m) both.insert(both.end(), lsem[m].begin(), lsem[m].end());
     h.lsem = h.upload(both, stream, "sweep lane semaphores");
   }
   h.n_lanes = (int64_t)lrec.size();
@@ -666,12 +691,6 @@ static ThrArgs thr_args(const sync_programs* h, sync_thr_mode mode) {
 static void check_thr_mode(sync_thr_mode mode) {
   if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP && mode != SYNC_THR_PERENGINE)
     raise(SYNC_ERR_ARG, "unknown threshold mode");
-}
-
-// simulation: the two semaphore allocations the simulator models
-static void check_mode(sync_thr_mode mode) {
-  if (mode == SYNC_THR_PERENGINE) raise(SYNC_ERR_ARG, "per-engine thresholds are evaluated and checked, not simulated");
-  if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP) raise(SYNC_ERR_ARG, "unknown threshold mode");
 }
 
 // Per-engine mode: derive the engine-stream positions of the waited
@@ -735,16 +754,17 @@ sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int3
                           int32_t* d_issue, int32_t* d_retire, void* stream) {
   try {
     if (!h || !params) raise(SYNC_ERR_ARG, "handle and params must not be NULL");
-    check_mode(mode);
-    if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER) raise(SYNC_ERR_ARG, "unknown variant");
+    check_thr_mode(mode);
+    if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER && variant != SYNC_SIM_UNROLLED)
+      raise(SYNC_ERR_ARG, "unknown variant");
+    if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
+      raise(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
     if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
       raise(SYNC_ERR_ARG, "per-program outputs must not be NULL");
     if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
     if ((d_issue == nullptr) != (d_retire == nullptr)) raise(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");
-    const sync_sim_params& q = *params;
-    if (q.ii < 0 || q.c_branch < 0 || q.c_regop < 0 || q.c_wait_ops_count < 0 ||
-        q.c_wait_ops_perloop < 0 || q.c_barrier < 0)
-      raise(SYNC_ERR_ARG, "timing constants must be >= 0");
+    sync_sim_params q;
+    if (!syncgb::sim_params_for(*params, variant, q)) raise(SYNC_ERR_ARG, "timing constants must be >= 0");
     cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
     SimArgs a;
     std::memset(&a, 0, sizeof a);

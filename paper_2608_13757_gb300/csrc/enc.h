@@ -54,19 +54,22 @@ struct alignas(16) DepInfo {
 };
 
 // Per program, for the simulator.
+constexpr int kModes = 3;   // threshold encodings: COUNT, PERLOOP, PERENGINE
+
 struct alignas(16) ProgInfo {
   int64_t agg_lat;    // sum over instructions of instances * latency (saturated)
   int64_t n_inst;     // datapath instances
   int64_t n_pairs;    // (dependency, consumer instance) pairs
   int64_t n_stmt;     // loop statements reached (sum over non-top loops of total(parent))
   int64_t n_iter;     // loop iterations (sum over non-top loops of total)
+  int64_t pair_levels;  // sum over pairs of the per-engine wait's extra levels
   int32_t ne;
   int32_t le_base;    // row of (top-level loop, engine 0); row of (program-local
                       // loop l, engine e) = le_base + l*ne + e
-  int32_t nsem[2];    // waited semaphores, per threshold mode
-  int32_t semhb_off[2];  // first entry of the program's history bases, per mode
+  int32_t nsem[kModes];    // waited semaphores, per threshold mode
+  int32_t semhb_off[kModes];  // first entry of the program's history bases, per mode
   int32_t loop_base;  // global id of the program's top-level loop
-  int32_t pad_[3];
+  int32_t pad_;
 };
 
 // Program-order sweep tables.  Per loop, a plan: its body cut at child loops
@@ -82,7 +85,7 @@ struct alignas(16) ProgInfo {
 //   lmeta {engine, copy, first lane of the engine's run, flags}
 //     flags bit 0: first record of its engine in a copy >= 1 (an iteration
 //     start precedes it); bit 1: last lane of its engine's run
-//   lsem per mode {semaphore, stride, koff, 0} as the simulator's records.
+//   lsem per mode {semaphore, stride, koff, levels} as the simulator's records.
 enum : int32_t { ITEM_SEG = 0, ITEM_LOOP = 1 };
 constexpr int32_t LANE_ITER_START = 1;
 constexpr int32_t LANE_RUN_LAST = 2;
@@ -98,11 +101,17 @@ constexpr int32_t LANE_RUN_LAST = 2;
 // in its row.  Per row: op_ptr = first record, rowinfo = {END record index,
 // 1 if the row holds a LOOP record}.
 // Per-mode semaphore records parallel to the op records (mode 0 = one
-// semaphore per producer instruction, mode 1 = one per (loop, engine)):
+// semaphore per producer instruction, mode 1 = one per (loop, engine),
+// mode 2 = one per engine):
 //   {semaphore (program-local, -1 if nothing waits on it), increments per
-//    iteration (1 or N), koff (1 or K)}: the increment of iteration g brings
-//    the semaphore to stride*g + koff and its retire time lives at history
-//    slot semhb[semaphore] + stride*g + koff - 1.
+//    iteration (1 or N), koff (1 or K), levels}: the increment of iteration g
+//    brings the semaphore to stride*g + koff and its retire time lives at
+//    history slot semhb[semaphore] + stride*g + koff - 1.  Per-engine
+//    semaphores have stride -1: every instance of the engine increments, and
+//    the increment is the instance's ordinal n in the engine's stream (slot
+//    n - 1).  levels (mode 2): sum over the record's dependencies of the
+//    loops strictly between the top level and the producer's loop, the
+//    extra terms of a per-engine wait.
 // Consumer-grouped dependencies: segment offset (int64) and, per mode, the
 // waited semaphore (program-local).  semhb: per program and mode, the
 // history base of each waited semaphore.

@@ -12,6 +12,10 @@ namespace syncgb {
 void cuda_or_raise(cudaError_t e, const char* what);
 // Sets the message sync_last_error() returns on this thread; returns status.
 sync_status set_error(sync_status status, const std::string& msg);
+// The timing constants the simulation kernels take: false if any is
+// negative; for the unrolled variant (the straight-line program) the
+// loop-control and wait-value costs are 0.
+bool sim_params_for(const sync_sim_params& p, sync_sim_variant variant, sync_sim_params& q);
 }  // namespace syncgb
 
 struct sync_programs {
@@ -46,9 +50,9 @@ struct sync_programs {
   int2* rowinfo = nullptr;
   int4* ops = nullptr;
   int32_t* opstop = nullptr;
-  int4* opsem = nullptr;            // [2][n_ops]
+  int4* opsem = nullptr;            // [kModes][n_ops]
   int64_t* dseg = nullptr;
-  int32_t* dsem = nullptr;          // [2][n_deps]
+  int32_t* dsem = nullptr;          // [kModes][n_deps]
   int64_t* semhb = nullptr;
   int64_t* inst_off = nullptr;
   int64_t n_ops = 0;
@@ -61,10 +65,10 @@ struct sync_programs {
   int4* chunk = nullptr;
   int4* lrec = nullptr;
   int4* lmeta = nullptr;
-  int4* lsem = nullptr;             // [2][n_lanes]
+  int4* lsem = nullptr;             // [kModes][n_lanes]
   int64_t n_lanes = 0;
-  int64_t hist_len[2] = {0, 0};     // history entries needed per threshold mode
-  int32_t nsem_max[2] = {0, 0};
+  int64_t hist_len[syncgb::kModes] = {0, 0, 0};  // history entries needed per threshold mode
+  int32_t nsem_max[syncgb::kModes] = {0, 0, 0};
   int32_t ne_max = 1;
   int32_t depth_max = 0;
 

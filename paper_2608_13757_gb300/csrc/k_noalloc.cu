@@ -56,19 +56,19 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
                                              void* stream) {
   using namespace syncgb;
   if (!h || !params) return set_error(SYNC_ERR_ARG, "handle and params must not be NULL");
-  if (mode == SYNC_THR_PERENGINE)
-    return set_error(SYNC_ERR_ARG, "per-engine thresholds are evaluated and checked, not simulated");
-  if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP) return set_error(SYNC_ERR_ARG, "unknown threshold mode");
-  if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER) return set_error(SYNC_ERR_ARG, "unknown variant");
+  if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP && mode != SYNC_THR_PERENGINE)
+    return set_error(SYNC_ERR_ARG, "unknown threshold mode");
+  if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER && variant != SYNC_SIM_UNROLLED)
+    return set_error(SYNC_ERR_ARG, "unknown variant");
+  if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
+    return set_error(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
   if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
     return set_error(SYNC_ERR_ARG, "per-program outputs must not be NULL");
   if (h->sz.n_pairs_padded > 0 && !d_thr) return set_error(SYNC_ERR_ARG, "d_thr must not be NULL");
   if ((d_issue == nullptr) != (d_retire == nullptr))
     return set_error(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");
-  const sync_sim_params& q = *params;
-  if (q.ii < 0 || q.c_branch < 0 || q.c_regop < 0 || q.c_wait_ops_count < 0 || q.c_wait_ops_perloop < 0 ||
-      q.c_barrier < 0)
-    return set_error(SYNC_ERR_ARG, "timing constants must be >= 0");
+  sync_sim_params q;
+  if (!sim_params_for(*params, variant, q)) return set_error(SYNC_ERR_ARG, "timing constants must be >= 0");
   if (h->device < 0 || h->device >= kMaxDevices) return set_error(SYNC_ERR_ARG, "device id out of range");
   // the scratch must hold two counters, the fallback list and the history
   const int64_t list_ints = ((2 + (int64_t)h->sz.n_programs) + 63) & ~int64_t(63);

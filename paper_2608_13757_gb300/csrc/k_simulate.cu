@@ -92,7 +92,7 @@ __device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t r
 }
 
 // Static time bound of a program under the given costs (saturating).
-template <bool BB>
+template <int MODE, bool BB>
 __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, const sync_sim_params& q,
                                                          int32_t cwait) {
   typedef unsigned long long u64;
@@ -102,6 +102,8 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul((u64)(pi.n_stmt + pi.n_iter), (u64)q.c_barrier));
   } else {
     b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
+    if (MODE == SYNC_THR_PERENGINE)
+      b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
     const u64 ctl = sat_add(sat_mul((u64)pi.n_stmt, (u64)q.c_regop),
                             sat_mul((u64)pi.n_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop));
     b = sat_add(b, sat_mul((u64)pi.ne, ctl));
@@ -177,7 +179,7 @@ __device__ __forceinline__ void set_row(const SimArgs& a, Eng& E, int32_t row) {
 template <int MODE, bool BB, bool TL>
 __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng& E, int w, int lane,
                                            int ne, unsigned long long& chk) {
-  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int32_t ii = a.prm.ii;
   Frame* frames = S.frames + w * a.frame_depth;
@@ -285,7 +287,8 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
     }
     const bool in = lane < cut;
     // cursor maps t' = max(t + A, B), inclusive scan over the lanes
-    const int32_t wcost = BB ? 0 : rec.z * cwait;
+    const int32_t wcost =
+        BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * srec.w : 0);
     int32_t A = 0, B = kNeg;
     if (in) {
       if (dp) { A = wcost + ii; B = waited ? ready + ii : kNeg; }
@@ -308,18 +311,20 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
       if (lane >= o) v = max(v, vp);
     }
     const int32_t retire = max(E.lastret, v);       // in-order retirement
-    // publish this chunk's semaphore increments
+    // publish this chunk's semaphore increments: per-engine semaphores count
+    // the engine's instances, the others a fixed number per iteration
+    const unsigned dm = __ballot_sync(kFull, in && dp);
+    const uint32_t nj = E.n + __popc(dm & lanemask_le());   // the instance's position in the engine's stream
     const bool prod = in && dp && srec.x >= 0;
-    if (prod) a.hist[S.semhb[srec.x] + (int64_t)srec.y * gj + (srec.z - 1)] = retire;
+    const int32_t ninc = srec.y < 0 ? (int32_t)nj : srec.y * gj + srec.z;
+    if (prod) a.hist[S.semhb[srec.x] + (ninc - 1)] = retire;
     __syncwarp();                                    // orders the warp's history writes
     const unsigned pm = __ballot_sync(kFull, prod);
     if (prod) {
       const unsigned peers = __match_any_sync(pm, srec.x);
-      if (lane == 31 - __clz(peers)) st_release(S.sem + srec.x, srec.y * gj + srec.z);
+      if (lane == 31 - __clz(peers)) st_release(S.sem + srec.x, ninc);
     }
-    const unsigned dm = __ballot_sync(kFull, in && dp);
     if (in && dp) {
-      const uint32_t nj = E.n + __popc(dm & lanemask_le());
       chk += inst_term(issue, retire, (uint32_t)w, nj);
       if (TL) {
         const int64_t o = __ldg(a.inst_off + rec.x) + gj;
@@ -362,7 +367,7 @@ __global__ void k_simulate(const SimArgs a) {
     S.w_ms = reinterpret_cast<int32_t*>(p); p += 4 * W;
     S.slot = reinterpret_cast<int32_t*>(p);   // 4 ints
   }
-  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
 
   for (;;) {
     __syncthreads();
@@ -373,7 +378,7 @@ __global__ void k_simulate(const SimArgs a) {
     if (slot >= limit) break;
     const int p = a.only ? a.only[1 + slot] : __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
-    if (time_bound<BB>(pi, a.prm, cwait) > 2147483647ull) {
+    if (time_bound<MODE, BB>(pi, a.prm, cwait) > 2147483647ull) {
       if (threadIdx.x == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
       continue;
     }
@@ -477,6 +482,9 @@ cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStr
   if (a.mode == SYNC_THR_PERLOOP)
     return barrier ? launch3<SYNC_THR_PERLOOP, true>(a, smem, num_sms, s)
                    : launch3<SYNC_THR_PERLOOP, false>(a, smem, num_sms, s);
+  if (a.mode == SYNC_THR_PERENGINE)
+    return barrier ? launch3<SYNC_THR_PERENGINE, true>(a, smem, num_sms, s)
+                   : launch3<SYNC_THR_PERENGINE, false>(a, smem, num_sms, s);
   return barrier ? launch3<SYNC_THR_COUNT, true>(a, smem, num_sms, s)
                  : launch3<SYNC_THR_COUNT, false>(a, smem, num_sms, s);
 }

@@ -70,7 +70,7 @@ __device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t r
   return ((unsigned long long)x << 32) | y;
 }
 
-template <bool BB>
+template <int MODE, bool BB>
 __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, const sync_sim_params& q,
                                                          int32_t cwait) {
   typedef unsigned long long u64;
@@ -80,6 +80,8 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul((u64)(pi.n_stmt + pi.n_iter), (u64)q.c_barrier));
   } else {
     b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
+    if (MODE == SYNC_THR_PERENGINE)
+      b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
     const u64 ctl = sat_add(sat_mul((u64)pi.n_stmt, (u64)q.c_regop),
                             sat_mul((u64)pi.n_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop));
     b = sat_add(b, sat_mul((u64)pi.ne, ctl));
@@ -160,7 +162,7 @@ template <int MODE, bool BB, bool TL>
 __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, const LaneRec& L,
                                          const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
                                          int32_t ctag, int lane, unsigned long long& chk) {
-  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int4 rec = L.rec, sr = L.sr;
   const bool have = lane < ch.y;
@@ -202,7 +204,7 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
     wait_on(__ldg(a.thr + __ldg(a.dseg + rec.w + j) + gl), __ldg(a.dsem + rec.w + j));
   if (__ballot_sync(kFull, fallback)) return SIM_FALLBACK;
 
-  const int32_t wcost = BB ? 0 : rec.z * cwait;
+  const int32_t wcost = BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * sr.w : 0);
   const int32_t apre = (L.meta.w & LANE_ITER_START) ? iter_cost : 0;
   const int32_t A = valid ? apre + wcost + a.prm.ii : 0;
   int32_t r_intra = kNeg;                      // retire of in-chunk producers (lower bound)
@@ -246,15 +248,17 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
   if (!settled) return SYNC_PROG_DEADLOCK;   // a cycle of waits inside the chunk
 
   // publish increments, instance counts, checksum terms, engine state
+  const unsigned vm = __ballot_sync(kFull, valid);
+  const unsigned run_le = vm & lanemask_le() & ~((1u << head) - 1u);
+  const uint32_t nj = (uint32_t)n_in + __popc(run_le);   // the instance's position in its engine's stream
   if (prod) {
-    const int32_t n = sr.y * gl + sr.z;        // the increment this retirement makes
+    // the increment this retirement makes: per-engine semaphores count the
+    // engine's instances, the others a fixed number per iteration
+    const int32_t n = sr.y < 0 ? (int32_t)nj : sr.y * gl + sr.z;
     S.ring[sr.x * (S.rmask + 1) + ((n - 1) & S.rmask)] = retire;
     a.hist[S.semhb[sr.x] + (n - 1)] = retire;
   }
-  const unsigned vm = __ballot_sync(kFull, valid);
-  const unsigned run_le = vm & lanemask_le() & ~((1u << head) - 1u);
   if (valid) {
-    const uint32_t nj = (uint32_t)n_in + __popc(run_le);
     chk += inst_term(issue, retire, (uint32_t)e, nj);
     if (TL) {
       const int64_t o = __ldg(a.inst_off + rec.x) + gl;
@@ -301,7 +305,7 @@ template <int MODE, bool BB, bool TL>
 __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi,
                                              const int4 ch, const LaneRec& L, int32_t lo, int32_t hi,
                                              int32_t ctag, int lane, unsigned long long& chk) {
-  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int32_t ii = a.prm.ii;
   const int32_t copies = ch.z;
@@ -354,7 +358,8 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
   bool rep = false;
   int32_t rd_issue = 0, rd_retire = 0, rd_t = 0, rd_r = 0, rk0 = 0, rk1 = 0;
 
-  const int32_t P = (BB ? 0 : L.rec.z * cwait) + ((L.meta.w & LANE_ITER_START) ? iter_cost : 0);
+  const int32_t wcost = L.rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * L.sr.w : 0);
+  const int32_t P = (BB ? 0 : wcost) + ((L.meta.w & LANE_ITER_START) ? iter_cost : 0);
   const int32_t A = P + ii;                           // cursor advance of a valid lane with no wait
   int32_t T0n = 0, T1n = 0;
   {
@@ -465,13 +470,13 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     }
 
     // publish
+    const uint32_t nj = (uint32_t)n_in + __popc(vm & lanemask_le() & run_from_head);
     if (valid && prod_lane) {
-      const int32_t n = own_stride * gl + own_koff;
+      const int32_t n = own_stride < 0 ? (int32_t)nj : own_stride * gl + own_koff;
       S.ring[own_ring + ((n - 1) & S.rmask)] = retire;
       a.hist[own_hist + n] = retire;
     }
     if (valid) {
-      const uint32_t nj = (uint32_t)n_in + __popc(vm & lanemask_le() & run_from_head);
       chk += inst_term(issue, retire, (uint32_t)e, nj);
       if (TL) {
         a.issue[tl_off + gl] = issue;
@@ -559,7 +564,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     S.rank_lane = reinterpret_cast<uint8_t*>(p);
     S.rmask = a.ring - 1;
   }
-  const int32_t cwait = MODE == SYNC_THR_PERLOOP ? a.prm.c_wait_ops_perloop : a.prm.c_wait_ops_count;
+  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
 
   for (;;) {
@@ -569,7 +574,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     if (slot >= a.n_programs) break;
     const int p = __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
-    if (time_bound<BB>(pi, a.prm, cwait) > 2147483647ull) {
+    if (time_bound<MODE, BB>(pi, a.prm, cwait) > 2147483647ull) {
       if (lane == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
       continue;
     }
@@ -724,6 +729,9 @@ cudaError_t launch_sweep(const SweepArgs& a, bool barrier, int num_sms, cudaStre
   if (a.mode == SYNC_THR_PERLOOP)
     return barrier ? launch3<SYNC_THR_PERLOOP, true>(a, smem, num_sms, s)
                    : launch3<SYNC_THR_PERLOOP, false>(a, smem, num_sms, s);
+  if (a.mode == SYNC_THR_PERENGINE)
+    return barrier ? launch3<SYNC_THR_PERENGINE, true>(a, smem, num_sms, s)
+                   : launch3<SYNC_THR_PERENGINE, false>(a, smem, num_sms, s);
   return barrier ? launch3<SYNC_THR_COUNT, true>(a, smem, num_sms, s)
                  : launch3<SYNC_THR_COUNT, false>(a, smem, num_sms, s);
 }

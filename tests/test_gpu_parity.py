@@ -10,9 +10,15 @@ from tests import golden_io
 
 pytestmark = pytest.mark.gpu
 
-COUNT, PERLOOP = oracle.COUNT, oracle.PERLOOP
+COUNT, PERLOOP, PERENGINE = oracle.COUNT, oracle.PERLOOP, oracle.PERENGINE
 MODES = (COUNT, PERLOOP)
+ALL_MODES = (COUNT, PERLOOP, PERENGINE)
 VARIANTS = (oracle.BARRIER_FREE, oracle.BARRIER)
+
+
+def variants_for(mode):
+    """The unrolled variant runs on per-engine semaphores only."""
+    return VARIANTS + ((oracle.UNROLLED,) if mode == PERENGINE else ())
 
 
 @pytest.fixture(scope="module")
@@ -53,7 +59,7 @@ def compare_all(sg, batch, params=None, timeline=False, modes=MODES):
         assert np.array_equal(got, want), f"thresholds differ (mode {mode})"
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
-        for v in VARIANTS:
+        for v in variants_for(mode):
             res = sg.sync_simulate(h, mode, thr, sim_params(prm), v, timeline=timeline)
             ref = oracle.simulate(batch, want, mode, v, prm, timeline=timeline)
             P = batch.n_programs
@@ -160,13 +166,33 @@ def test_perengine_checker_planted_errors(sg):
     test_checker_planted_errors(sg, oracle.PERENGINE)
 
 
-def test_perengine_is_not_simulated(sg):
+@pytest.mark.parametrize("name,n", [("small", None), ("depth2", 48), ("gemm", None),
+                                    ("attention", 2), ("chain", 400), ("syncbound", 400)])
+def test_perengine_simulation_bit_exact(sg, name, n):
+    """Per-engine semaphores (Sec. 6.1) under the barrier-free, barrier and
+    unrolled schemes: makespans, checksums, statuses (and timelines on the
+    small cases) equal the oracle's."""
+    batch = workloads.generate(name, n_programs=n)
+    compare_all(sg, batch, timeline=name in ("small", "depth2"), modes=(PERENGINE,))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_perengine_simulation_random_trees(sg, seed):
+    batch = workloads.random_trees(3000 + seed, 150, workloads.tree_params(
+        engines_hi=6, loops_hi=6, body_hi=6, trip_hi=4, max_depth=4))
+    compare_all(sg, batch, timeline=True, modes=(PERENGINE,),
+                params=oracle.sim_params(ii=2, c_branch=3, c_regop=2, c_barrier=9,
+                                         c_wait_ops_perengine_level=5))
+
+
+def test_unrolled_requires_perengine(sg):
     batch = workloads.generate("small")
     h = sg.sync_load_programs(batch)
-    thr = sg.sync_eval_thresholds(h, sg.THR_PERENGINE)
-    with pytest.raises(sg.SyncError) as err:
-        sg.sync_simulate(h, sg.THR_PERENGINE, thr)
-    assert err.value.status == sg.ERR_ARG
+    for mode in MODES:
+        thr = sg.sync_eval_thresholds(h, mode)
+        with pytest.raises(sg.SyncError) as err:
+            sg.sync_simulate(h, mode, thr, variant=sg.SIM_UNROLLED)
+        assert err.value.status == sg.ERR_ARG
 
 
 def test_checker_detects_swapped_encoding(sg):
@@ -243,19 +269,21 @@ def test_edge_programs(sg):
     b.instr(L, 0, 0, latency=2 ** 30)
     progs.append(b.batch())
     batch = workloads.concat(progs)
-    compare_all(sg, batch, timeline=True)
+    compare_all(sg, batch, timeline=True, modes=ALL_MODES)
     ref = oracle.simulate(batch, oracle.thresholds(batch, PERLOOP), PERLOOP, oracle.BARRIER)
     assert 7 in ref.status.tolist() and 4 in ref.status.tolist()
 
 
 def test_zero_costs_and_large_costs(sg):
     batch = workloads.random_trees(77, 120)
-    compare_all(sg, batch, params=oracle.sim_params(ii=0, c_branch=0, c_regop=0,
-                                                    c_wait_ops_count=0, c_wait_ops_perloop=0,
-                                                    c_barrier=0))
-    compare_all(sg, batch, params=oracle.sim_params(ii=7, c_branch=100, c_regop=50,
-                                                    c_wait_ops_count=9, c_wait_ops_perloop=13,
-                                                    c_barrier=1000))
+    compare_all(sg, batch, modes=ALL_MODES,
+                params=oracle.sim_params(ii=0, c_branch=0, c_regop=0, c_wait_ops_count=0,
+                                         c_wait_ops_perloop=0, c_barrier=0,
+                                         c_wait_ops_perengine_level=0))
+    compare_all(sg, batch, modes=ALL_MODES,
+                params=oracle.sim_params(ii=7, c_branch=100, c_regop=50, c_wait_ops_count=9,
+                                         c_wait_ops_perloop=13, c_barrier=1000,
+                                         c_wait_ops_perengine_level=21))
 
 
 def test_repeated_calls_are_identical(sg):
@@ -281,12 +309,12 @@ def test_full_size_sampled(sg, name):
     h = sg.sync_load_programs(batch)
     rng = np.random.default_rng(5)
     sample = np.unique(np.concatenate([[0, P - 1], rng.choice(P, size=min(P, 12), replace=False)]))
-    for mode in MODES:
+    for mode in ALL_MODES:
         thr = sg.sync_eval_thresholds(h, mode)
         host = thr.cpu().numpy()
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
-        sims = {v: sg.sync_simulate(h, mode, thr, variant=v) for v in VARIANTS}
+        sims = {v: sg.sync_simulate(h, mode, thr, variant=v) for v in variants_for(mode)}
         for p in sample.tolist():
             one = workloads.generate(name, n_programs=1, first_program=p)
             want = oracle.thresholds(one, mode)
@@ -294,7 +322,7 @@ def test_full_size_sampled(sg, name):
             got = np.concatenate([host[h.pair_offsets[d]:h.pair_offsets[d] + h.pair_counts[d]]
                                   for d in range(d0, d1)] or [np.zeros(0, np.int32)])
             assert np.array_equal(got, want), (name, mode, p)
-            for v in VARIANTS:
+            for v in variants_for(mode):
                 ref = oracle.simulate(one, want, mode, v)
                 assert sims[v].status[p].item() == ref.status[0]
                 assert sims[v].makespan[p].item() == ref.makespan[0], (name, mode, v, p)

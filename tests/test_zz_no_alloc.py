@@ -72,9 +72,10 @@ def test_noalloc_matches_simulate_on_consecutive_calls(sg):
     h = sg.sync_load_programs(batch)
     P = h.sizes.n_programs
     inst = _instances_per_program(batch)
-    for mode in (sg.THR_COUNT, sg.THR_PERLOOP):
+    for mode in (sg.THR_COUNT, sg.THR_PERLOOP, sg.THR_PERENGINE):
         thr = sg.sync_eval_thresholds(h, mode)
-        for variant in (sg.SIM_BARRIER_FREE, sg.SIM_BARRIER):
+        unrolled = (sg.SIM_UNROLLED,) if mode == sg.THR_PERENGINE else ()
+        for variant in (sg.SIM_BARRIER_FREE, sg.SIM_BARRIER) + unrolled:
             ref = sg.sync_simulate(h, mode, thr, variant=variant, timeline=True)
             torch.cuda.synchronize()
             ok = ref.status.cpu().numpy() == sg.PROG_OK
