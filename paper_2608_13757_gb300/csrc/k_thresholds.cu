@@ -14,9 +14,9 @@
 // Sec. 5.1's registers r_S and r-hat_S).  Both come from arrays derived at
 // load time (S-ancestor per consumer iteration, trip start per S-iteration),
 // so a chunk needs the dependency record, one int4 of ancestors or trip
-// starts, and a trip start per distinct g_S: a short chain of dependent
-// loads.  A chunk's four consumer iterations usually share g_S, evaluated
-// once.
+// starts, and a trip start per distinct g_S (loaded in parallel): a short
+// chain of dependent loads.  A nested producer's count (rare) is evaluated
+// once per distinct g_S.
 #include "enc.h"
 
 namespace syncgb {
@@ -90,89 +90,124 @@ __device__ __forceinline__ int32_t eval_at(const ThrArgs& a, const DepInfo& D, i
 // Values of the chunk's pairs g0 .. g0+3 (entries at or past `total` are
 // padding and get 0).  g0 is a multiple of 4, and so is every derived
 // array's start, so the chunk's four trip starts (consumer in S) or
-// S-ancestors (consumer below S) come in one int4 load.
+// S-ancestors (consumer below S) come in one int4 load; below S, the trip
+// start of each distinct S-iteration is loaded once (the ancestors are
+// non-decreasing), all in parallel.
 template <bool CHECK>
 __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D, int32_t g0, int mode) {
   const int32_t n = D.total - g0 < kChunk ? D.total - g0 : kChunk;   // >= 1
-  int32_t v[kChunk] = {0, 0, 0, 0};
+  const int32_t* ts = a.derived + D.tstart;
+  int32_t gs[kChunk], st[kChunk];
   if (D.up == 0) {
     // consumer directly in S: g_S = g
-    const int4 ts = __ldg(reinterpret_cast<const int4*>(a.derived + D.tstart + g0));
-    const int32_t st[kChunk] = {ts.x, ts.y, ts.z, ts.w};
-#pragma unroll
-    for (int i = 0; i < kChunk; ++i)
-      if (i < n) v[i] = eval_at<CHECK>(a, D, g0 + i, st[i], mode);
+    const int4 x = __ldg(reinterpret_cast<const int4*>(ts + g0));
+    gs[0] = g0; gs[1] = g0 + 1; gs[2] = g0 + 2; gs[3] = g0 + 3;
+    st[0] = x.x; st[1] = x.y; st[2] = x.z; st[3] = x.w;
   } else {
-    // consumer nested below S: one value per distinct g_S (non-decreasing)
-    const int4 an = __ldg(reinterpret_cast<const int4*>(a.derived + D.anc + g0));
-    const int32_t gs[kChunk] = {an.x, an.y, an.z, an.w};
-    int32_t cur = gs[0];
-    int32_t val = eval_at<CHECK>(a, D, cur, __ldg(a.derived + D.tstart + cur), mode);
+    const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.anc + g0));
+    gs[0] = x.x; gs[1] = x.y; gs[2] = x.z; gs[3] = x.w;
+    st[0] = __ldg(ts + gs[0]);
+    st[3] = n > 3 && gs[3] != gs[0] ? __ldg(ts + gs[3]) : st[0];
+    st[1] = n > 1 && gs[1] != gs[0] ? (gs[1] == gs[3] ? st[3] : __ldg(ts + gs[1])) : st[0];
+    st[2] = n > 2 && gs[2] != gs[0] ? (gs[2] == gs[3] ? st[3] : __ldg(ts + gs[2])) : st[0];
+  }
+  int32_t v[kChunk];
+  if (D.clen == 0) {
+    // producer directly in S: the count through the target is its position
+#pragma unroll
+    for (int i = 0; i < kChunk; ++i) {
+      if (CHECK) {
+        const int32_t tS = gs[i] - st[i] + 1 - D.k;      // target's position in its trip
+        v[i] = i < n && tS > 0 ? encode(a, D, st[i] + tS, mode) : 0;
+      } else {
+        v[i] = i < n && gs[i] - st[i] + 1 > D.k ? encode(a, D, gs[i] + 1 - D.k, mode) : 0;
+      }
+    }
+  } else {
+    // nested producer: one evaluation per distinct g_S
+    int32_t val = eval_at<CHECK>(a, D, gs[0], st[0], mode);
     v[0] = val;
 #pragma unroll
     for (int i = 1; i < kChunk; ++i) {
-      if (i < n) {
-        if (gs[i] != cur) {
-          cur = gs[i];
-          val = eval_at<CHECK>(a, D, cur, __ldg(a.derived + D.tstart + cur), mode);
-        }
-        v[i] = val;
-      }
+      if (i < n && gs[i] != gs[i - 1]) val = eval_at<CHECK>(a, D, gs[i], st[i], mode);
+      v[i] = i < n ? val : 0;
     }
   }
   return make_int4(v[0], v[1], v[2], v[3]);
 }
 
+// Prefetch hints (no register is held and nothing waits for them).
+__device__ __forceinline__ void prefetch_l1(const void* p) { asm volatile("prefetch.global.L1 [%0];" :: "l"(p)); }
+__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" :: "l"(p)); }
+
+// The chunk's chain of dependent loads is latency-bound; the tile-table
+// entry of the thread's next chunk is brought into L1 while this one runs,
+// which takes the first link out of the next chain.
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 8) k_thresholds(const ThrArgs a, int32_t* __restrict__ thr) {
   const int64_t stride = (int64_t)gridDim.x * kThreads;
   for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.n_chunks; c += stride) {
     const int64_t q = c * kChunk;
+    if (c + stride < a.n_chunks) prefetch_l1(a.tile_first + (q + stride * kChunk) / kTilePairs);
     const DepInfo D = a.dep[find_dep(a, q)];
     __stcs(reinterpret_cast<int4*>(thr + q), chunk_values<false>(a, D, (int32_t)(q - D.seg_off), MODE));
   }
 }
 
-__device__ __forceinline__ void tally(int32_t got, int32_t want, int64_t idx, uint32_t& unsafe,
-                                      uint32_t& over, unsigned long long& first) {
-  if (got == want) return;
-  if (got < want) ++unsafe; else ++over;
-  if ((unsigned long long)idx < first) first = (unsigned long long)idx;
-}
-
-template <int MODE>
-__global__ void __launch_bounds__(kThreads, 6) k_check(const CheckArgs a) {
-  // a thread's counts fit 32 bits (it sees at most n_chunks / threads chunks)
-  uint32_t unsafe = 0, over = 0;
+// A warp's chunks with a mismatch: tally them warp-wide (unsafe: below the
+// minimum, over-synchronised: above it) and record the first offending pair.
+__device__ __forceinline__ void report(const CheckArgs& a, const int4 v, const int4 m, int32_t n, int64_t q,
+                                       bool bad) {
+  const int32_t got[kChunk] = {v.x, v.y, v.z, v.w}, want[kChunk] = {m.x, m.y, m.z, m.w};
+  unsigned u = 0, o = 0;
   unsigned long long first = ~0ull;
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.t.n_chunks; c += stride) {
-    const int64_t q = c * kChunk;
-    const int4 v = __ldcs(reinterpret_cast<const int4*>(a.thr + q));
-    const DepInfo D = a.t.dep[find_dep(a.t, q)];
-    const int32_t g0 = (int32_t)(q - D.seg_off);
-    const int4 m = chunk_values<true>(a.t, D, g0, MODE);
-    // padding entries are not pairs: the checker reads only the first n
-    const int32_t n = D.total - g0;
-    const bool bad = v.x != m.x || (n > 1 && v.y != m.y) || (n > 2 && v.z != m.z) || (n > 3 && v.w != m.w);
-    if (bad) {
-      tally(v.x, m.x, q + 0, unsafe, over, first);
-      if (n > 1) tally(v.y, m.y, q + 1, unsafe, over, first);
-      if (n > 2) tally(v.z, m.z, q + 2, unsafe, over, first);
-      if (n > 3) tally(v.w, m.w, q + 3, unsafe, over, first);
+  if (bad) {
+#pragma unroll
+    for (int i = kChunk - 1; i >= 0; --i) {
+      if (i < n && got[i] != want[i]) {
+        if (got[i] < want[i]) ++u; else ++o;
+        first = (unsigned long long)(q + i);
+      }
     }
   }
-  unsigned long long u = unsafe, o = over;
+  u = __reduce_add_sync(0xffffffffu, u);
+  o = __reduce_add_sync(0xffffffffu, o);
   for (int s = 16; s > 0; s >>= 1) {
-    u += __shfl_xor_sync(0xffffffffu, u, s);
-    o += __shfl_xor_sync(0xffffffffu, o, s);
     const unsigned long long f = __shfl_xor_sync(0xffffffffu, first, s);
     first = f < first ? f : first;
   }
   if ((threadIdx.x & 31) == 0) {
-    if (u) atomicAdd(a.counts + 0, u);
-    if (o) atomicAdd(a.counts + 1, o);
-    if (first != ~0ull) atomicMin(a.first_bad, first);
+    if (u) atomicAdd(a.counts + 0, (unsigned long long)u);
+    if (o) atomicAdd(a.counts + 1, (unsigned long long)o);
+    atomicMin(a.first_bad, first);
+  }
+}
+
+// Warps step through the chunks together (every lane runs every iteration,
+// lanes past the end idle), so a mismatch can be tallied warp-wide where it
+// occurs and nothing is carried in registers.  The stored thresholds are
+// prefetched into L2 when the chunk starts and read after its minimum is
+// known, so no register holds them across the chain of lookups.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 8) k_check(const CheckArgs a) {
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  const int64_t end = (a.t.n_chunks + 31) & ~int64_t(31);
+  for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < end; c += stride) {
+    const int64_t q = c * kChunk;
+    bool bad = false;
+    int4 v = make_int4(0, 0, 0, 0), m = v;
+    int32_t n = 0;
+    if (c < a.t.n_chunks) {
+      prefetch_l2(a.thr + q);
+      const DepInfo D = a.t.dep[find_dep(a.t, q)];
+      const int32_t g0 = (int32_t)(q - D.seg_off);
+      m = chunk_values<true>(a.t, D, g0, MODE);
+      v = __ldcs(reinterpret_cast<const int4*>(a.thr + q));
+      // padding entries are not pairs: the checker reads only the first n
+      n = D.total - g0;
+      bad = v.x != m.x || (n > 1 && v.y != m.y) || (n > 2 && v.z != m.z) || (n > 3 && v.w != m.w);
+    }
+    if (__ballot_sync(0xffffffffu, bad)) report(a, v, m, n, q, bad);
   }
 }
 
