@@ -347,7 +347,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         n_ord += S.total[Pl];
       }
       D.ordp = ord_off[x0 + px];
-      D.anc = -1;
+      D.src = D.tstart;
       if (D.up > 0) {
         const int64_t key = (int64_t)Cl * nl + Sl;
         auto f = S.anc_of.find(key);
@@ -359,12 +359,10 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
           f = S.anc_of.emplace(key, n_derived).first;
           n_derived += pad4(S.total[Cl]);
         }
-        D.anc = f->second;
+        D.src = f->second;
       }
       path.push_back(loop[l0 + Sl].pidx_off);
       path.push_back(loop[l0 + Sl].rowptr_off);
-      D.s_pidx = loop[l0 + Sl].pidx_off;
-      D.s_rowptr = loop[l0 + Sl].rowptr_off;
       {
         const size_t at = path.size();
         for (int32_t l = Pl; l != Sl; l = par[l]) path.push_back(loop[l0 + l].rowptr_off);

@@ -39,20 +39,20 @@ struct alignas(16) LoopInfo {
 //   [up+2, up+2+clen)  rowptr offsets of the loops from S's child down to P
 //                      (nested cases; clen = 0 when P = S).
 struct alignas(16) DepInfo {
+  // read for every chunk: the first 48 bytes (three 16-byte loads)
   int64_t seg_off;    // pair-layout offset of this dependency's segment
-  int64_t path;
-  int64_t s_pidx;     // S's pidx and rowptr offsets (= path entries up, up+1)
-  int64_t s_rowptr;
+  int64_t src;        // derived pool, per consumer iteration: its trip start of S
+                      // (consumer directly in S) or its enclosing S-iteration (below S)
   int64_t tstart;     // derived pool: first iteration of the trip, per iteration of S
-  int64_t anc;        // derived pool: enclosing S-iteration per consumer iteration (up > 0)
-  int64_t ordp;       // ordinal pool: engine-stream position per producer instance
   int32_t total;      // consumer instances (= total of the consumer's loop)
-  int32_t up;
-  int32_t clen;
-  int32_t kase;
-  int32_t k, N, K, pad_;
+  int32_t k, N, K;
+  int32_t up;         // consumer depth below S
+  int32_t clen;       // producer depth below S
+  // read for nested producers and per-engine values only
+  int64_t path;
+  int64_t ordp;       // ordinal pool: engine-stream position per producer instance
+  int32_t kase, pad_;
 };
-
 // Per program, for the simulator.
 constexpr int kModes = 3;   // threshold encodings: COUNT, PERLOOP, PERENGINE
 

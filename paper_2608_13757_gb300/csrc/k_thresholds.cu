@@ -17,6 +17,8 @@
 // starts, and a trip start per distinct g_S (loaded in parallel): a short
 // chain of dependent loads.  A nested producer's count (rare) is evaluated
 // once per distinct g_S.
+#include <cstdlib>
+
 #include "enc.h"
 
 namespace syncgb {
@@ -27,8 +29,9 @@ constexpr int kThreads = 256;
 // Dependency owning pair q: the largest d with seg[d] <= q, searched inside
 // the range the tile table gives for q's tile (empty segments share their
 // offset with the next dependency, which then wins).
-__device__ __forceinline__ int find_dep(const ThrArgs& a, int64_t q) {
-  const int64_t t = q / kTilePairs;
+template <typename I>
+__device__ __forceinline__ int find_dep(const ThrArgs& a, I q) {
+  const I t = q / kTilePairs;
   int lo = __ldg(a.tile_first + t), hi = __ldg(a.tile_first + t + 1);
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -97,14 +100,13 @@ template <bool CHECK>
 __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D, int32_t g0, int mode) {
   const int32_t n = D.total - g0 < kChunk ? D.total - g0 : kChunk;   // >= 1
   const int32_t* ts = a.derived + D.tstart;
+  const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.src + g0));
   int32_t gs[kChunk], st[kChunk];
   if (D.up == 0) {
     // consumer directly in S: g_S = g
-    const int4 x = __ldg(reinterpret_cast<const int4*>(ts + g0));
     gs[0] = g0; gs[1] = g0 + 1; gs[2] = g0 + 2; gs[3] = g0 + 3;
     st[0] = x.x; st[1] = x.y; st[2] = x.z; st[3] = x.w;
   } else {
-    const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.anc + g0));
     gs[0] = x.x; gs[1] = x.y; gs[2] = x.z; gs[3] = x.w;
     st[0] = __ldg(ts + gs[0]);
     st[3] = n > 3 && gs[3] != gs[0] ? __ldg(ts + gs[3]) : st[0];
@@ -140,15 +142,19 @@ __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D,
 __device__ __forceinline__ void prefetch_l1(const void* p) { asm volatile("prefetch.global.L1 [%0];" :: "l"(p)); }
 __device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" :: "l"(p)); }
 
+// I is the chunk-index type: 32-bit while every pair index of the launch
+// (plus one grid stride) fits, which saves the 64-bit address arithmetic
+// of the loop; 64-bit otherwise.
+//
 // The chunk's chain of dependent loads is latency-bound; the tile-table
 // entry of the thread's next chunk is brought into L1 while this one runs,
 // which takes the first link out of the next chain.
-template <int MODE>
+template <int MODE, typename I>
 __global__ void __launch_bounds__(kThreads, 8) k_thresholds(const ThrArgs a, int32_t* __restrict__ thr) {
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < a.n_chunks; c += stride) {
-    const int64_t q = c * kChunk;
-    if (c + stride < a.n_chunks) prefetch_l1(a.tile_first + (q + stride * kChunk) / kTilePairs);
+  const I stride = (I)gridDim.x * kThreads, n_chunks = (I)a.n_chunks;
+  for (I c = (I)blockIdx.x * kThreads + threadIdx.x; c < n_chunks; c += stride) {
+    const I q = c * kChunk;
+    if (c + stride < n_chunks) prefetch_l1(a.tile_first + (q + stride * kChunk) / kTilePairs);
     const DepInfo D = a.dep[find_dep(a, q)];
     __stcs(reinterpret_cast<int4*>(thr + q), chunk_values<false>(a, D, (int32_t)(q - D.seg_off), MODE));
   }
@@ -188,16 +194,16 @@ __device__ __forceinline__ void report(const CheckArgs& a, const int4 v, const i
 // occurs and nothing is carried in registers.  The stored thresholds are
 // prefetched into L2 when the chunk starts and read after its minimum is
 // known, so no register holds them across the chain of lookups.
-template <int MODE>
+template <int MODE, typename I>
 __global__ void __launch_bounds__(kThreads, 8) k_check(const CheckArgs a) {
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  const int64_t end = (a.t.n_chunks + 31) & ~int64_t(31);
-  for (int64_t c = (int64_t)blockIdx.x * kThreads + threadIdx.x; c < end; c += stride) {
-    const int64_t q = c * kChunk;
+  const I stride = (I)gridDim.x * kThreads, n_chunks = (I)a.t.n_chunks;
+  const I end = (n_chunks + 31) & ~I(31);
+  for (I c = (I)blockIdx.x * kThreads + threadIdx.x; c < end; c += stride) {
+    const I q = c * kChunk;
     bool bad = false;
     int4 v = make_int4(0, 0, 0, 0), m = v;
     int32_t n = 0;
-    if (c < a.t.n_chunks) {
+    if (c < n_chunks) {
       prefetch_l2(a.thr + q);
       const DepInfo D = a.t.dep[find_dep(a.t, q)];
       const int32_t g0 = (int32_t)(q - D.seg_off);
@@ -225,36 +231,52 @@ cudaError_t grid_for(K kern, int64_t n_chunks, int num_sms, int& grid) {
   return cudaSuccess;
 }
 
+
+// 64-bit chunk indices when 32 bits could overflow (or when the
+// SYNCGB_WIDE_INDEX environment variable is set to 1, which tests use to
+// run the 64-bit kernels on small batches).
+bool wide_index(int64_t n_chunks, int grid) {
+  const char* f = std::getenv("SYNCGB_WIDE_INDEX");
+  if (f && f[0] == '1') return true;
+  return (n_chunks + (int64_t)grid * kThreads) * kChunk > (int64_t)INT32_MAX;
+}
+
+template <int MODE>
+cudaError_t launch_thr_mode(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s) {
+  int grid = 0;
+  cudaError_t e = grid_for(k_thresholds<MODE, int64_t>, a.n_chunks, num_sms, grid);
+  if (e != cudaSuccess) return e;
+  if (wide_index(a.n_chunks, grid)) k_thresholds<MODE, int64_t><<<grid, kThreads, 0, s>>>(a, thr);
+  else k_thresholds<MODE, int32_t><<<grid, kThreads, 0, s>>>(a, thr);
+  return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_check_mode(const CheckArgs& a, int num_sms, cudaStream_t s) {
+  int grid = 0;
+  cudaError_t e = grid_for(k_check<MODE, int64_t>, a.t.n_chunks, num_sms, grid);
+  if (e != cudaSuccess) return e;
+  if (wide_index(a.t.n_chunks, grid)) k_check<MODE, int64_t><<<grid, kThreads, 0, s>>>(a);
+  else k_check<MODE, int32_t><<<grid, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_thresholds(const ThrArgs& a, int32_t* thr, int num_sms, cudaStream_t s) {
   if (a.n_chunks == 0) return cudaSuccess;
-  auto run = [&](auto kern) -> cudaError_t {
-    int grid = 0;
-    const cudaError_t e = grid_for(kern, a.n_chunks, num_sms, grid);
-    if (e != cudaSuccess) return e;
-    kern<<<grid, kThreads, 0, s>>>(a, thr);
-    return cudaGetLastError();
-  };
-  if (a.mode == SYNC_THR_PERLOOP) return run(k_thresholds<SYNC_THR_PERLOOP>);
-  if (a.mode == SYNC_THR_PERENGINE) return run(k_thresholds<SYNC_THR_PERENGINE>);
-  return run(k_thresholds<SYNC_THR_COUNT>);
+  if (a.mode == SYNC_THR_PERLOOP) return launch_thr_mode<SYNC_THR_PERLOOP>(a, thr, num_sms, s);
+  if (a.mode == SYNC_THR_PERENGINE) return launch_thr_mode<SYNC_THR_PERENGINE>(a, thr, num_sms, s);
+  return launch_thr_mode<SYNC_THR_COUNT>(a, thr, num_sms, s);
 }
 
 cudaError_t launch_check(const CheckArgs& a, int num_sms, cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(a.counts, 0, 2 * sizeof(unsigned long long), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(a.first_bad, 0xff, sizeof(unsigned long long), s);
   if (e != cudaSuccess || a.t.n_chunks == 0) return e;
-  auto run = [&](auto kern) -> cudaError_t {
-    int grid = 0;
-    const cudaError_t e2 = grid_for(kern, a.t.n_chunks, num_sms, grid);
-    if (e2 != cudaSuccess) return e2;
-    kern<<<grid, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
-  };
-  if (a.t.mode == SYNC_THR_PERLOOP) return run(k_check<SYNC_THR_PERLOOP>);
-  if (a.t.mode == SYNC_THR_PERENGINE) return run(k_check<SYNC_THR_PERENGINE>);
-  return run(k_check<SYNC_THR_COUNT>);
+  if (a.t.mode == SYNC_THR_PERLOOP) return launch_check_mode<SYNC_THR_PERLOOP>(a, num_sms, s);
+  if (a.t.mode == SYNC_THR_PERENGINE) return launch_check_mode<SYNC_THR_PERENGINE>(a, num_sms, s);
+  return launch_check_mode<SYNC_THR_COUNT>(a, num_sms, s);
 }
 
 }  // namespace syncgb

@@ -195,6 +195,24 @@ def test_unrolled_requires_perengine(sg):
         assert err.value.status == sg.ERR_ARG
 
 
+@pytest.mark.parametrize("mode", ALL_MODES)
+def test_wide_index_kernels(sg, mode, monkeypatch):
+    """The 64-bit-index threshold and check kernels (taken for batches past
+    2^31 pair indices) give the same values and verdicts; the switch forces
+    them on a small batch."""
+    batch = workloads.random_trees(4000 + mode, 120, workloads.tree_params(
+        engines_hi=5, loops_hi=5, body_hi=6, trip_hi=6, max_depth=4))
+    h = sg.sync_load_programs(batch)
+    _, narrow = gpu_thresholds(sg, h, mode)
+    monkeypatch.setenv("SYNCGB_WIDE_INDEX", "1")
+    thr, wide = gpu_thresholds(sg, h, mode)
+    assert np.array_equal(wide, narrow)
+    assert np.array_equal(wide, oracle.thresholds(batch, mode))
+    counts, fb = sg.sync_check_minimal(h, mode, thr)
+    assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
+    test_checker_planted_errors(sg, mode)
+
+
 def test_checker_detects_swapped_encoding(sg):
     """Count-mode values read as per-loop values are below the minimum wherever
     N > 1 and c > 0."""
