@@ -52,6 +52,10 @@ def parse():
     ap.add_argument("--first-program", type=int, default=0,
                     help="id of rank 0's first program (ranks follow contiguously)")
     ap.add_argument("--mode", choices=("perloop", "count"), default="perloop")
+    ap.add_argument("--pipeline", choices=("arrays", "fused"), default="arrays",
+                    help="arrays: threshold kernel, checker, two simulations over the stored thresholds; "
+                         "fused: the two simulations compute (and, barrier-free, check) every wait value "
+                         "themselves")
     ap.add_argument("--cpu-sample", type=int, default=32768,
                     help="programs of the workload the CPU oracle baseline runs")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -159,15 +163,22 @@ def run_gpu(args, rank, world, local_rank):
     bf, bb = mk(), mk()
     stream = torch.cuda.current_stream()
 
+    fused = args.pipeline == "fused"
+
     def step(ev=None):
         if ev: ev[0].record(stream)
-        sg.sync_eval_thresholds(h, mode, out=thr)
+        if not fused: sg.sync_eval_thresholds(h, mode, out=thr)
         if ev: ev[1].record(stream)
-        sg.sync_check_minimal(h, mode, thr, counts, first_bad)
+        if not fused: sg.sync_check_minimal(h, mode, thr, counts, first_bad)
         if ev: ev[2].record(stream)
-        sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE, out=bf)
+        if fused:
+            sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER_FREE, out=bf, check=True, counts=counts,
+                                   first_bad=first_bad)
+        else:
+            sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE, out=bf)
         if ev: ev[3].record(stream)
-        sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER, out=bb)
+        if fused: sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER, out=bb)
+        else: sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER, out=bb)
         if ev: ev[4].record(stream)
 
     for _ in range(max(args.warmup, 0)):
@@ -197,6 +208,8 @@ def run_gpu(args, rank, world, local_rank):
         for i, name in enumerate(KERNELS):
             per_kernel[name] += e[i].elapsed_time(e[i + 1])
     per_kernel = {k: v / args.steps for k, v in per_kernel.items()}
+    if fused:                             # no threshold kernel or checker launched
+        per_kernel["thresholds"] = per_kernel["check"] = 0.0
     out = dict(ms=total_ms / args.steps, per_kernel=per_kernel, sizes=sz, clocks=clk, ok=ok,
                load_s=load_s, P=P)
     if not args.no_e2e:
@@ -215,10 +228,15 @@ def run_e2e(args, sg, batch, mode, prm, dev, P):
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         h = sg.sync_load_programs(batch, device=dev.index)
-        thr = sg.sync_eval_thresholds(h, mode)
-        counts, fb = sg.sync_check_minimal(h, mode, thr)
-        r1 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE)
-        r2 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER)
+        if args.pipeline == "fused":
+            thr = None
+            r1, counts, fb = sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER_FREE, check=True)
+            r2 = sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER)
+        else:
+            thr = sg.sync_eval_thresholds(h, mode)
+            counts, fb = sg.sync_check_minimal(h, mode, thr)
+            r1 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE)
+            r2 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER)
         host = [t.cpu() for t in (counts, fb, r1.makespan, r1.checksum, r1.status,
                                   r2.makespan, r2.checksum, r2.status)]
         torch.cuda.synchronize()
@@ -341,6 +359,8 @@ def roofline(res, hbm_peak, peak_kind, sm_mhz, workload):
            "check": 4 * sz.n_pairs_padded + sz.struct_bytes}
     kernels = {}
     for name in ("thresholds", "check"):
+        if pk[name] <= 0:
+            continue                      # fused pipeline: no threshold array
         t = pk[name] / 1e3
         ach = alg[name] / t / 1e9 if t > 0 else 0.0
         kernels[name] = {"bound": "hbm", "ms": pk[name], "achieved": ach, "peak": hbm_peak,
@@ -401,14 +421,15 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
         "config": {"workload": WORKLOADS.get(args.config, args.config), "programs_per_gpu": res["P"],
                    "pairs_per_gpu": int(pairs), "instances_per_gpu": int(res["sizes"].n_instances),
-                   "threshold_mode": args.mode, "l2": "inputs larger than L2 (thresholds "
+                   "threshold_mode": args.mode, "pipeline": args.pipeline,
+                   "l2": "inputs larger than L2 (thresholds "
                    f"{4 * res['sizes'].n_pairs_padded / 1e9:.2f} GB per pass)",
                    "parallelism": f"programs sharded over {world} GPU(s)"},
         "roofline": roof,
         "kernels": kernels,
         # per step: thresholds, check, and per schedule the sweep plus the
         # per-engine kernel for programs it hands over
-        "gpu_launches": 6 * args.steps,
+        "gpu_launches": (4 if args.pipeline == "fused" else 6) * args.steps,
         "results_minimal_and_deadlock_free": res["ok"],
         "load_s": res["load_s"],
         "clocks": clk or None,

@@ -249,6 +249,23 @@ sync_status sync_simulate(const sync_programs *h, sync_thr_mode mode, const int3
                           int32_t *d_makespan, unsigned long long *d_checksum, int32_t *d_status,
                           int32_t *d_issue, int32_t *d_retire, void *stream);
 
+/* Fused threshold -> check -> simulate: sync_simulate without a threshold
+ * array.  Every wait value is computed where the simulators reach the
+ * consumer, from the loop state of the walk (the register form of Sec. 5.1:
+ * the masked r_S - k or r_P, encoded as the mode says), so the 4 bytes per
+ * pair are neither written nor read.  Outputs, statuses and argument rules
+ * as sync_simulate (identical results).  d_counts ([2] uint64 device) and
+ * d_first_bad ([1] int64 device), both NULL or both set: each wait value is
+ * also recomputed by Eq. (1) as sync_check_minimal does, and mismatches are
+ * counted (unsafe, over-synchronised) with the smallest offending pair index
+ * (in sync_eval_thresholds' layout), or -1; only programs whose status is
+ * OK contribute.  Both are overwritten.  PERENGINE derives the engine-stream
+ * positions on first use, as sync_eval_thresholds does. */
+sync_status sync_simulate_fused(const sync_programs *h, sync_thr_mode mode, const sync_sim_params *params,
+                                sync_sim_variant variant, int32_t *d_makespan, unsigned long long *d_checksum,
+                                int32_t *d_status, int32_t *d_issue, int32_t *d_retire,
+                                unsigned long long *d_counts, long long *d_first_bad, void *stream);
+
 /* Size of the device scratch used by sync_simulate_noalloc (see below). */
 #define SYNC_NOALLOC_SCRATCH_BYTES (64u << 20)
 

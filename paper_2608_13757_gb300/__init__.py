@@ -29,8 +29,8 @@ PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD = 0, 4, 7, 8
 
 # every symbol include/sync.h declares
 EXPORTS = ("sync_load_programs", "sync_query", "sync_pair_offsets", "sync_eval_thresholds",
-           "sync_check_minimal", "sync_simulate", "sync_simulate_noalloc", "sync_free_programs",
-           "sync_last_error")
+           "sync_check_minimal", "sync_simulate", "sync_simulate_fused", "sync_simulate_noalloc",
+           "sync_free_programs", "sync_last_error")
 NOALLOC_SCRATCH_BYTES = 64 << 20
 
 
@@ -85,6 +85,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sync_simulate.argtypes = [vp, ctypes.c_int, vp, P(SimParams), ctypes.c_int, vp, vp, vp,
                                   vp, vp, vp]
     lib.sync_simulate_noalloc.argtypes = lib.sync_simulate.argtypes
+    lib.sync_simulate_fused.argtypes = [vp, ctypes.c_int, P(SimParams), ctypes.c_int, vp, vp, vp, vp, vp,
+                                        vp, vp, vp]
     lib.sync_free_programs.argtypes = [vp]
     lib.sync_free_programs.restype = None
     lib.sync_last_error.argtypes = []
@@ -241,6 +243,38 @@ def sync_simulate(h: Programs, mode, thr, params: SimParams | None = None,
                               _ptr(out.makespan), _ptr(out.checksum), _ptr(out.status),
                               _ptr(out.issue), _ptr(out.retire), _stream(stream)))
     return out
+
+
+def sync_simulate_fused(h: Programs, mode, params: SimParams | None = None,
+                        variant: int = SIM_BARRIER_FREE, timeline: bool = False, check: bool = False,
+                        out: SimOutputs | None = None, counts=None, first_bad=None, stream=None):
+    """Simulation with every wait value computed inside the simulators (no
+    threshold array).  Returns the SimOutputs, and with check=True also
+    (counts [2], first_bad [1]) as sync_check_minimal does, for the programs
+    whose status is OK."""
+    import torch
+    dev = f"cuda:{h.device}"
+    P = h.sizes.n_programs
+    if out is None:
+        out = SimOutputs(torch.empty(max(P, 1), dtype=torch.int32, device=dev),
+                         torch.empty(max(P, 1), dtype=torch.int64, device=dev),
+                         torch.empty(max(P, 1), dtype=torch.int32, device=dev))
+        if timeline:
+            n = max(h.sizes.n_instances, 1)
+            out.issue = torch.full((n,), -1, dtype=torch.int32, device=dev)
+            out.retire = torch.full((n,), -1, dtype=torch.int32, device=dev)
+    if check:
+        if counts is None:
+            counts = torch.empty(2, dtype=torch.int64, device=dev)
+        if first_bad is None:
+            first_bad = torch.empty(1, dtype=torch.int64, device=dev)
+    prm = params if params is not None else SimParams()
+    _check(lib().sync_simulate_fused(h.handle, int(mode), ctypes.byref(prm), int(variant),
+                                    _ptr(out.makespan), _ptr(out.checksum), _ptr(out.status),
+                                    _ptr(out.issue), _ptr(out.retire),
+                                    _ptr(counts) if check else None, _ptr(first_bad) if check else None,
+                                    _stream(stream)))
+    return (out, counts, first_bad) if check else out
 
 
 def sync_simulate_noalloc(h: Programs, mode, thr, params: SimParams | None = None,

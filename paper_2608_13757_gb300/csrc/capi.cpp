@@ -158,6 +158,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<int2> rowinfo;
   std::vector<int4> ops, opsem[kModes];
   std::vector<int64_t> inst_off(NX), dseg(ND), semhb;
+  std::vector<int32_t> ddep(ND);
   std::vector<int32_t> dsem[kModes] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
   std::vector<int32_t> plan_ptr;
   std::vector<int4> plan, chunks, lrec, lmeta, lsem[kModes];
@@ -428,7 +429,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       for (int32_t i = 0; i < nd; ++i) {
         const int64_t gd = d0 + by_cons[i];
         dsem[m][d0 + i] = sem_of[sem_key(m, d.dep_prod[gd])];
-        if (m == 0) dseg[d0 + i] = seg[gd];
+        if (m == 0) { dseg[d0 + i] = seg[gd]; ddep[d0 + i] = (int32_t)gd; }
       }
     }
     for (int32_t i = nd - 1; i >= 0; --i) S.x_dep_begin[d.dep_cons[d0 + by_cons[i]]] = d0 + i;
@@ -621,6 +622,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   }
   h.n_ops = (int64_t)ops.size();
   h.dseg = h.upload(dseg, stream, "dependency segments");
+  h.ddep = h.upload(ddep, stream, "consumer-grouped dependency ids");
   h.semhb = h.upload(semhb, stream, "semaphore history bases");
   h.inst_off = h.upload(inst_off, stream, "instance offsets");
   h.hist = h.alloc<int32_t>(*std::max_element(hist_len.begin(), hist_len.end()), "semaphore history");
@@ -746,60 +748,97 @@ sync_status sync_check_minimal(const sync_programs* h, sync_thr_mode mode, const
   }
 }
 
+// Both simulation entry points: thresholds from d_thr, or (fused) from the
+// simulators' loop state, optionally checked.
+static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, const int32_t* d_thr,
+                     const sync_sim_params* params,
+                     sync_sim_variant variant, int32_t* d_makespan, unsigned long long* d_checksum,
+                     int32_t* d_status, int32_t* d_issue, int32_t* d_retire, unsigned long long* d_counts,
+                     long long* d_first_bad, void* stream) {
+  if (!h || !params) raise(SYNC_ERR_ARG, "handle and params must not be NULL");
+  check_thr_mode(mode);
+  if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER && variant != SYNC_SIM_UNROLLED)
+    raise(SYNC_ERR_ARG, "unknown variant");
+  if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
+    raise(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
+  if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
+    raise(SYNC_ERR_ARG, "per-program outputs must not be NULL");
+  if ((d_issue == nullptr) != (d_retire == nullptr)) raise(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");
+  if ((d_counts == nullptr) != (d_first_bad == nullptr))
+    raise(SYNC_ERR_ARG, "d_counts and d_first_bad: both or neither");
+  sync_sim_params q;
+  if (!syncgb::sim_params_for(*params, variant, q)) raise(SYNC_ERR_ARG, "timing constants must be >= 0");
+  cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (fused && mode == SYNC_THR_PERENGINE) ensure_ordinals(h, st);
+  if (d_counts) {
+    cuda_check(cudaMemsetAsync(d_counts, 0, 2 * sizeof(unsigned long long), st), "cudaMemsetAsync");
+    cuda_check(cudaMemsetAsync(d_first_bad, 0xff, sizeof(long long), st), "cudaMemsetAsync");
+  }
+  SimArgs a;
+  std::memset(&a, 0, sizeof a);
+  a.prog = h->prog; a.order = h->order; a.rowptr = h->rowptr;
+  a.op_ptr = h->op_ptr; a.rowinfo = h->rowinfo; a.ops = h->ops; a.opstop = h->opstop;
+  a.opsem = h->opsem + (size_t)mode * h->n_ops;
+  a.dseg = h->dseg; a.dsem = h->dsem + (size_t)mode * h->sz.n_deps;
+  a.semhb = h->semhb;
+  a.inst_off = h->inst_off;
+  a.thr = d_thr; a.hist = h->hist; a.next_slot = h->next_slot;
+  a.makespan = d_makespan; a.checksum = d_checksum; a.status = d_status;
+  a.issue = d_issue; a.retire = d_retire;
+  a.prm = q;
+  a.n_programs = h->sz.n_programs;
+  a.mode = mode;
+  a.sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
+  a.frame_depth = std::max(1, h->depth_max);
+  a.warps = h->ne_max;
+  if (fused) {
+    a.dep = h->dep; a.ddep = h->ddep; a.path = h->path; a.ord = h->ord;
+    a.chk_counts = d_counts; a.chk_first = reinterpret_cast<unsigned long long*>(d_first_bad);
+  }
+  const int ring = sweep_ring_for(a.sem_cap, a.frame_depth, 200 * 1024);
+  if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024 || ring == 0)
+    raise(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
+  SweepArgs w;
+  std::memset(&w, 0, sizeof w);
+  w.prog = h->prog; w.order = h->order; w.loop = h->loop; w.rowptr = h->rowptr;
+  w.plan_ptr = h->plan_ptr; w.plan = h->plan; w.chunk = h->chunk;
+  w.lrec = h->lrec; w.lmeta = h->lmeta; w.lsem = h->lsem + (size_t)mode * h->n_lanes;
+  w.dseg = h->dseg; w.dsem = a.dsem; w.semhb = h->semhb; w.inst_off = h->inst_off;
+  w.thr = d_thr; w.hist = h->hist; w.next_slot = h->next_slot; w.fallback = h->fallback;
+  w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
+  w.issue = d_issue; w.retire = d_retire;
+  w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
+  w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring;
+  w.dep = a.dep; w.ddep = a.ddep; w.path = a.path; w.ord = a.ord;
+  w.chk_counts = a.chk_counts; w.chk_first = a.chk_first;
+  const bool barrier = variant == SYNC_SIM_BARRIER;
+  cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");
+  a.only = h->fallback;
+  cuda_check(launch_simulate(a, barrier, h->num_sms, st), "per-engine simulator kernel");
+}
+
 sync_status sync_simulate(const sync_programs* h, sync_thr_mode mode, const int32_t* d_thr,
                           const sync_sim_params* params, sync_sim_variant variant,
                           int32_t* d_makespan, unsigned long long* d_checksum, int32_t* d_status,
                           int32_t* d_issue, int32_t* d_retire, void* stream) {
   try {
-    if (!h || !params) raise(SYNC_ERR_ARG, "handle and params must not be NULL");
-    check_thr_mode(mode);
-    if (variant != SYNC_SIM_BARRIER_FREE && variant != SYNC_SIM_BARRIER && variant != SYNC_SIM_UNROLLED)
-      raise(SYNC_ERR_ARG, "unknown variant");
-    if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
-      raise(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
-    if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
-      raise(SYNC_ERR_ARG, "per-program outputs must not be NULL");
-    if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
-    if ((d_issue == nullptr) != (d_retire == nullptr)) raise(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");
-    sync_sim_params q;
-    if (!syncgb::sim_params_for(*params, variant, q)) raise(SYNC_ERR_ARG, "timing constants must be >= 0");
-    cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
-    SimArgs a;
-    std::memset(&a, 0, sizeof a);
-    a.prog = h->prog; a.order = h->order; a.rowptr = h->rowptr;
-    a.op_ptr = h->op_ptr; a.rowinfo = h->rowinfo; a.ops = h->ops; a.opstop = h->opstop;
-    a.opsem = h->opsem + (size_t)mode * h->n_ops;
-    a.dseg = h->dseg; a.dsem = h->dsem + (size_t)mode * h->sz.n_deps;
-    a.semhb = h->semhb;
-    a.inst_off = h->inst_off;
-    a.thr = d_thr; a.hist = h->hist; a.next_slot = h->next_slot;
-    a.makespan = d_makespan; a.checksum = d_checksum; a.status = d_status;
-    a.issue = d_issue; a.retire = d_retire;
-    a.prm = q;
-    a.n_programs = h->sz.n_programs;
-    a.mode = mode;
-    a.sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
-    a.frame_depth = std::max(1, h->depth_max);
-    a.warps = h->ne_max;
-    const int ring = sweep_ring_for(a.sem_cap, a.frame_depth, 200 * 1024);
-    if (simulate_smem_bytes(a.warps, a.sem_cap, a.frame_depth) > 200 * 1024 || ring == 0)
-      raise(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
-    SweepArgs w;
-    std::memset(&w, 0, sizeof w);
-    w.prog = h->prog; w.order = h->order; w.loop = h->loop; w.rowptr = h->rowptr;
-    w.plan_ptr = h->plan_ptr; w.plan = h->plan; w.chunk = h->chunk;
-    w.lrec = h->lrec; w.lmeta = h->lmeta; w.lsem = h->lsem + (size_t)mode * h->n_lanes;
-    w.dseg = h->dseg; w.dsem = a.dsem; w.semhb = h->semhb; w.inst_off = h->inst_off;
-    w.thr = d_thr; w.hist = h->hist; w.next_slot = h->next_slot; w.fallback = h->fallback;
-    w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
-    w.issue = d_issue; w.retire = d_retire;
-    w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
-    w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const bool barrier = variant == SYNC_SIM_BARRIER;
-    cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");
-    a.only = h->fallback;
-    cuda_check(launch_simulate(a, barrier, h->num_sms, st), "per-engine simulator kernel");
+    if (h && h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
+    simulate(h, mode, false, d_thr, params, variant, d_makespan, d_checksum, d_status, d_issue, d_retire, nullptr,
+             nullptr, stream);
+    return SYNC_OK;
+  } catch (const Failure& f) {
+    return report(f);
+  }
+}
+
+sync_status sync_simulate_fused(const sync_programs* h, sync_thr_mode mode, const sync_sim_params* params,
+                                sync_sim_variant variant, int32_t* d_makespan, unsigned long long* d_checksum,
+                                int32_t* d_status, int32_t* d_issue, int32_t* d_retire,
+                                unsigned long long* d_counts, long long* d_first_bad, void* stream) {
+  try {
+    simulate(h, mode, true, nullptr, params, variant, d_makespan, d_checksum, d_status, d_issue, d_retire, d_counts,
+             d_first_bad, stream);
     return SYNC_OK;
   } catch (const Failure& f) {
     return report(f);

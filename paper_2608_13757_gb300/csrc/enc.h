@@ -184,6 +184,14 @@ struct SimArgs {
   int32_t sem_cap;           // semaphore slots in shared memory
   int32_t frame_depth;       // frames per warp
   const int32_t* only;       // if set: [0] count, [1..] the program ids to simulate
+  // fused simulation (thresholds from the walk's loop state, no threshold
+  // array): dep is set (NULL otherwise) and thr is unused
+  const DepInfo* dep;
+  const int32_t* ddep;       // per consumer-grouped dependency: its dependency id
+  const int64_t* path;
+  const int32_t* ord;        // per-engine mode: engine-stream positions
+  unsigned long long* chk_counts;  // optional: [2] unsafe / over-synchronised wait values
+  unsigned long long* chk_first;   // optional: [1] smallest offending pair index
 };
 
 struct SweepArgs {
@@ -216,6 +224,14 @@ struct SweepArgs {
   int32_t sem_cap;
   int32_t frame_depth;
   int32_t ring;              // latest increments kept per semaphore (power of two)
+  // fused simulation (thresholds from the walk's loop state, no threshold
+  // array): dep is set (NULL otherwise) and thr is unused
+  const DepInfo* dep;
+  const int32_t* ddep;       // per consumer-grouped dependency: its dependency id
+  const int64_t* path;
+  const int32_t* ord;        // per-engine mode: engine-stream positions
+  unsigned long long* chk_counts;  // optional: [2] unsafe / over-synchronised wait values
+  unsigned long long* chk_first;   // optional: [1] smallest offending pair index
 };
 
 // Launchers (return the launch error, if any).

@@ -34,7 +34,7 @@
 // CTAs are persistent and fetch program ids from a counter in descending-work
 // order.  Times are int32: a program whose static time bound exceeds
 // INT32_MAX gets status 4 without being simulated, so no time can overflow.
-#include "enc.h"
+#include "waitval.cuh"
 
 namespace syncgb {
 namespace {
@@ -52,7 +52,7 @@ constexpr int32_t kNeg = -1;
 
 enum : int { ST_RUN = 0, ST_BAR = 1, ST_DONE = 2 };
 
-struct Frame { int32_t row, ptr, g, g_end; };
+struct Frame { int32_t row, ptr, g, g_end, lo; };   // lo: start of the trip of iteration g
 
 __device__ __forceinline__ int32_t ld_acquire(const int32_t* p) {
   int32_t v;
@@ -121,11 +121,13 @@ struct Smem {
   unsigned long long* w_chk;
   int32_t* slot;           // [4]: program slot, barrier count, generation, release
   Frame* frames;           // [warps][frame_depth]
+  unsigned long long* tally;  // [3] fused check: unsafe, over-synchronised, first offending pair
 };
 
 // Engine state, identical in the 32 lanes of the engine's warp.
 struct Eng {
   int32_t row, pbeg, rend, ptr, g, g_end, sp;
+  int32_t lo;              // start of the current trip
   bool loops;              // the current row holds a child loop
   int32_t t, lastret;
   int32_t bar_gen;         // barrier generation this engine waits to see pass
@@ -175,8 +177,36 @@ __device__ __forceinline__ void set_row(const SimArgs& a, Eng& E, int32_t row) {
   E.loops = ri.y != 0;
 }
 
+// Fused simulation: the wait value of consumer-grouped dependency r for the
+// engine's instance at global iteration gj of its current loop, from the
+// engine's loop state (the register form of Sec. 5.1, r_S and r-hat_S read
+// off the level of S); with the optional check, the Eq. (1) minimum beside
+// it, mismatches counted in nu / no and the smallest offending pair in first.
+template <int MODE>
+__device__ __forceinline__ int32_t fused_value(const SimArgs& a, const Frame* frames, const Eng& E, int r,
+                                               int32_t gj, unsigned& nu, unsigned& no,
+                                               unsigned long long& first) {
+  const DepInfo& D = a.dep[__ldg(a.ddep + r)];
+  int32_t gs = gj, st = E.lo;
+  if (D.up > 0) {
+    const Frame f = frames[E.sp - D.up];
+    gs = f.g;
+    st = f.lo;
+  }
+  const int32_t T = wait_value(a, D, gs, st, MODE);
+  if (a.chk_counts) {
+    const int32_t m = minimum(a, D, gs, st, MODE);
+    if (T != m) {
+      if (T < m) ++nu; else ++no;
+      const unsigned long long q = (unsigned long long)(__ldg(a.dseg + r) + gj);
+      first = q < first ? q : first;
+    }
+  }
+  return T;
+}
+
 // One round of engine w: up to kChunks chunks or control steps.
-template <int MODE, bool BB, bool TL>
+template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng& E, int w, int lane,
                                            int ne, unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
@@ -210,12 +240,13 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
       ++E.ptr;
       if (lo < hi) {
         __syncwarp();
-        if (lane == 0) frames[E.sp] = Frame{E.row, E.ptr, E.g, E.g_end};
+        if (lane == 0) frames[E.sp] = Frame{E.row, E.ptr, E.g, E.g_end, E.lo};
         ++E.sp;
         set_row<MODE, BB, TL>(a, E, r0.y + w);
         E.ptr = E.pbeg;
         E.g = lo;
         E.g_end = hi;
+        E.lo = lo;
         E.t += iter_cost;
       }
       moved = true;
@@ -231,7 +262,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
         __syncwarp();
         const Frame f = frames[--E.sp];
         set_row<MODE, BB, TL>(a, E, f.row);
-        E.ptr = f.ptr; E.g = f.g; E.g_end = f.g_end;
+        E.ptr = f.ptr; E.g = f.g; E.g_end = f.g_end; E.lo = f.lo;
       }
       moved = true;
       continue;
@@ -265,8 +296,11 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
     // waits: every dependency's semaphore must have reached the threshold
     int32_t ready = 0, bsem = 0, bthr = 0;
     bool waited = false, blocked = false;
+    unsigned nu = 0, no = 0;                         // fused check, this lane's dependencies
+    unsigned long long first = ~0ull;
     for (int j = 0; dp && j < rec.z; ++j) {
-      const int32_t T = __ldg(a.thr + __ldg(a.dseg + rec.w + j) + gj);
+      const int32_t T = FUSED ? fused_value<MODE>(a, frames, E, rec.w + j, gj, nu, no, first)
+                              : __ldg(a.thr + __ldg(a.dseg + rec.w + j) + gj);
       if (T <= 0) continue;
       const int32_t s = __ldg(a.dsem + rec.w + j);
       if (ld_acquire(S.sem + s) < T) { blocked = true; bsem = s; bthr = T; break; }
@@ -286,6 +320,11 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
       continue;
     }
     const bool in = lane < cut;
+    if (FUSED && in && (nu | no)) {                  // consumed events only (a cut one is re-evaluated)
+      if (nu) atomicAdd(S.tally + 0, (unsigned long long)nu);
+      if (no) atomicAdd(S.tally + 1, (unsigned long long)no);
+      atomicMin(S.tally + 2, first);
+    }
     // cursor maps t' = max(t + A, B), inclusive scan over the lanes
     const int32_t wcost =
         BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * srec.w : 0);
@@ -349,8 +388,9 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
   return moved;
 }
 
-template <int MODE, bool BB, bool TL>
-__global__ void k_simulate(const SimArgs a) {
+// Up to 32 engines: 1024 threads, so at most 64 registers a thread.
+template <int MODE, bool BB, bool TL, bool FUSED>
+__global__ void __launch_bounds__(1024) k_simulate(const SimArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int W = a.warps;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -358,6 +398,7 @@ __global__ void k_simulate(const SimArgs a) {
   {
     unsigned char* p = smem_raw;
     S.semhb = reinterpret_cast<int64_t*>(p); p += 8 * a.sem_cap;
+    S.tally = reinterpret_cast<unsigned long long*>(p); p += 3 * 8;
     S.w_chk = reinterpret_cast<unsigned long long*>(p); p += 8 * W;
     S.frames = reinterpret_cast<Frame*>(p); p += sizeof(Frame) * W * a.frame_depth;
     S.sem = reinterpret_cast<int32_t*>(p); p += 4 * a.sem_cap;
@@ -386,10 +427,14 @@ __global__ void k_simulate(const SimArgs a) {
       S.sem[i] = 0;
       S.semhb[i] = __ldg(a.semhb + pi.semhb_off[MODE] + i);
     }
-    if (threadIdx.x == 0) { S.slot[1] = 0; S.slot[2] = 0; S.slot[3] = 0; }
+    if (threadIdx.x == 0) {
+      S.slot[1] = 0; S.slot[2] = 0; S.slot[3] = 0;
+      S.tally[0] = S.tally[1] = 0;
+      S.tally[2] = ~0ull;
+    }
     const bool live = w < pi.ne;
     Eng E;
-    E.sp = 0; E.g = 0; E.g_end = 1;
+    E.sp = 0; E.g = 0; E.g_end = 1; E.lo = 0;
     E.t = 0; E.lastret = 0; E.bar_gen = 0; E.n = 0;
     E.state = live ? ST_RUN : ST_DONE;
     E.bar_passed = false;
@@ -407,7 +452,7 @@ __global__ void k_simulate(const SimArgs a) {
     __syncthreads();
     while (verdict < 0) {
       bool moved = false;
-      if (E.state != ST_DONE) moved = run_engine<MODE, BB, TL>(a, S, E, w, lane, pi.ne, chk);
+      if (E.state != ST_DONE) moved = run_engine<MODE, BB, TL, FUSED>(a, S, E, w, lane, pi.ne, chk);
       if (lane == 0) {
         S.w_moved[w] = moved;
         S.w_state[w] = E.state;
@@ -444,6 +489,12 @@ __global__ void k_simulate(const SimArgs a) {
       a.makespan[p] = ok ? ms : -1;
       a.checksum[p] = ok ? ck : 0ull;
       a.status[p] = verdict;
+      // fused check: the pairs of programs that ran to the end
+      if (FUSED && ok && a.chk_counts) {
+        if (S.tally[0]) atomicAdd(a.chk_counts + 0, S.tally[0]);
+        if (S.tally[1]) atomicAdd(a.chk_counts + 1, S.tally[1]);
+        if (S.tally[2] != ~0ull) atomicMin(a.chk_first, S.tally[2]);
+      }
     }
   }
 }
@@ -465,14 +516,14 @@ cudaError_t launch3(const SimArgs& a, size_t smem, int num_sms, cudaStream_t s) 
     kern<<<grid, threads, smem, s>>>(a);
     return cudaGetLastError();
   };
-  if (a.issue) return run(k_simulate<MODE, BB, true>);
-  return run(k_simulate<MODE, BB, false>);
+  if (a.dep) return a.issue ? run(k_simulate<MODE, BB, true, true>) : run(k_simulate<MODE, BB, false, true>);
+  return a.issue ? run(k_simulate<MODE, BB, true, false>) : run(k_simulate<MODE, BB, false, false>);
 }
 
 }  // namespace
 
 size_t simulate_smem_bytes(int warps, int sem_cap, int frame_depth) {
-  return (size_t)12 * sem_cap + (size_t)8 * warps + sizeof(Frame) * (size_t)warps * frame_depth +
+  return (size_t)12 * sem_cap + 3 * 8 + (size_t)8 * warps + sizeof(Frame) * (size_t)warps * frame_depth +
          (size_t)16 * warps + 16;
 }
 

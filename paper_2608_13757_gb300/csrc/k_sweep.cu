@@ -28,7 +28,7 @@
 // drained times.  Per-engine cursor, last retire and instance count live in
 // shared memory, read by the engine's lanes and written back by the last
 // lane of its run.
-#include "enc.h"
+#include "waitval.cuh"
 
 namespace syncgb {
 namespace {
@@ -45,7 +45,8 @@ struct Frame { int32_t loop, item, g, g_end; };
 
 // Shared memory of one warp (program), 16-byte aligned.
 __host__ __device__ __forceinline__ size_t warp_bytes(int sem_cap, int frame_depth, int ring) {
-  const size_t per = (size_t)(20 + 4 * ring + 32) * sem_cap + sizeof(Frame) * (size_t)frame_depth + 3 * 4 * 32;
+  const size_t per = (size_t)(20 + 4 * ring + 32) * sem_cap + sizeof(Frame) * (size_t)frame_depth +
+                     8 * (size_t)(frame_depth + 1) + 3 * 8 + 8 + 3 * 4 * 32;
   return (per + 15) & ~(size_t)15;
 }
 
@@ -101,7 +102,36 @@ struct WarpSmem {
   uint8_t* rank_lane;  // [cap][32] lane of the chunk's k-th increment (k from 0)
   int32_t rmask;       // ring - 1
   Frame* frames;       // [depth]
+  int2* lvl;           // [depth + 1] per level of the walk: {current iteration, start of its trip}
+  unsigned long long* tally;  // [3] fused check: unsafe, over-synchronised, first offending pair
 };
+
+// Fused simulation: the wait value of consumer-grouped dependency r for the
+// consumer instance at global iteration gl of the loop at walk level lc
+// (whose trip started at lo_c), from the walk's loop state -- the register
+// form of Sec. 5.1 with r_S, r-hat_S read off the level of S.  With the
+// optional check, the Eq. (1) minimum is evaluated beside it and a mismatch
+// is tallied for the program.
+template <int MODE>
+__device__ __forceinline__ int32_t fused_wait(const SweepArgs& a, const WarpSmem& S, int r, int32_t gl, int lc,
+                                              int32_t lo_c) {
+  const DepInfo& D = a.dep[__ldg(a.ddep + r)];
+  int32_t gs = gl, st = lo_c;
+  if (D.up > 0) {
+    const int2 v = S.lvl[lc - D.up];
+    gs = v.x;
+    st = v.y;
+  }
+  const int32_t T = wait_value(a, D, gs, st, MODE);
+  if (a.chk_counts) {
+    const int32_t m = minimum(a, D, gs, st, MODE);
+    if (T != m) {
+      atomicAdd(S.tally + (T < m ? 0 : 1), 1ull);
+      atomicMin(S.tally + 2, (unsigned long long)(__ldg(a.dseg + r) + gl));
+    }
+  }
+  return T;
+}
 
 // One lane's record of a chunk, with its first kMaxDeps dependencies.
 struct LaneRec {
@@ -132,10 +162,17 @@ __device__ __forceinline__ void load_lane(const SweepArgs& a, const int4 ch, int
   }
 }
 
-// Thresholds of the lane's first kMaxDeps dependencies at its iteration gl.
-__device__ __forceinline__ void load_thr(const LaneRec& L, bool valid, int32_t gl, int32_t (&T)[kMaxDeps]) {
+// Thresholds of the lane's first kMaxDeps dependencies at its iteration gl
+// of the loop at walk level lc (trip start lo_c): read from the threshold
+// array, or (fused) from the walk's loop state.
+template <int MODE, bool FUSED>
+__device__ __forceinline__ void load_thr(const SweepArgs& a, const WarpSmem& S, const LaneRec& L, bool valid,
+                                         int32_t gl, int lc, int32_t lo_c, int32_t (&T)[kMaxDeps]) {
 #pragma unroll
-  for (int j = 0; j < kMaxDeps; ++j) T[j] = (valid && j < L.rec.z) ? __ldg(L.tp[j] + gl) : 0;
+  for (int j = 0; j < kMaxDeps; ++j) {
+    if (FUSED) T[j] = (valid && j < L.rec.z) ? fused_wait<MODE>(a, S, L.rec.w + j, gl, lc, lo_c) : 0;
+    else T[j] = (valid && j < L.rec.z) ? __ldg(L.tp[j] + gl) : 0;
+  }
 }
 
 // Lanes that increment each semaphore in this chunk (`copies` iterations
@@ -158,10 +195,11 @@ __device__ __forceinline__ void set_groups(const WarpSmem& S, const LaneRec& L, 
 // given the lane's record, its first thresholds T and the semaphore groups
 // of this chunk (set_groups with the same copies and ctag).  Returns 0,
 // SYNC_PROG_DEADLOCK or SIM_FALLBACK.
-template <int MODE, bool BB, bool TL>
+template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, const LaneRec& L,
                                          const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
-                                         int32_t ctag, int lane, unsigned long long& chk) {
+                                         int32_t ctag, int lane, int lc, int32_t lo_c,
+                                         unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int4 rec = L.rec, sr = L.sr;
@@ -201,7 +239,8 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
   for (int j = 0; j < kMaxDeps; ++j)
     if (valid && j < rec.z) wait_on(T[j], L.sm[j]);
   for (int j = kMaxDeps; valid && j < rec.z; ++j)
-    wait_on(__ldg(a.thr + __ldg(a.dseg + rec.w + j) + gl), __ldg(a.dsem + rec.w + j));
+    wait_on(FUSED ? fused_wait<MODE>(a, S, rec.w + j, gl, lc, lo_c) : __ldg(a.thr + __ldg(a.dseg + rec.w + j) + gl),
+            __ldg(a.dsem + rec.w + j));
   if (__ballot_sync(kFull, fallback)) return SIM_FALLBACK;
 
   const int32_t wcost = BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * sr.w : 0);
@@ -292,6 +331,56 @@ __device__ __forceinline__ void barrier_all(const WarpSmem& S, int ne, int32_t c
   __syncwarp();
 }
 
+// Fused simulation inside a register-resident loop (levels: the loop is at
+// walk level lc, its trip is [lo, hi)).  Per waited dependency, either a
+// value fixed for the whole loop (S encloses the loop: fk = -1, value in fc),
+// or -- S being the loop itself, so the producer sits in it -- fk = k and the
+// per-loop encoding's N and N-K in fc, fn; per-engine values (fk = -2) are
+// evaluated in full for every iteration.
+template <int MODE>
+__device__ __forceinline__ void fused_setup(const SweepArgs& a, const WarpSmem& S, int r, int32_t lo, int32_t hi,
+                                            int32_t copy, int32_t copies, int lc, int32_t& fk, int32_t& fc,
+                                            int32_t& fn) {
+  const DepInfo& D = a.dep[__ldg(a.ddep + r)];
+  if (D.up == 0) {
+    fk = MODE == SYNC_THR_PERENGINE ? -2 : D.k;
+    fc = D.N;
+    fn = D.N - D.K;
+    return;
+  }
+  fk = -1;
+  const int2 v = S.lvl[lc - D.up];
+  fc = wait_value(a, D, v.x, v.y, MODE);
+  if (a.chk_counts) {
+    const int32_t m = minimum(a, D, v.x, v.y, MODE);
+    if (fc != m) {                 // the same mismatch at each of the lane's iterations
+      atomicAdd(S.tally + (fc < m ? 0 : 1), (unsigned long long)((hi - lo - copy + copies - 1) / copies));
+      atomicMin(S.tally + 2, (unsigned long long)(__ldg(a.dseg + r) + lo + copy));
+    }
+  }
+}
+
+template <int MODE>
+__device__ __forceinline__ int32_t fused_iter(const SweepArgs& a, const WarpSmem& S, int r, int32_t fk, int32_t fc,
+                                              int32_t fn, int32_t gl, int32_t lo, int lc) {
+  if (fk == -1) return fc;
+  if (fk == -2) return fused_wait<MODE>(a, S, r, gl, lc, lo);
+  // Eq. (2) with S = this loop: r-hat_S = gl - lo + 1, expr = r_S - k
+  const int32_t c = gl - lo + 1 > fk ? gl + 1 - fk : 0;
+  const int32_t T = c == 0 ? 0 : MODE == SYNC_THR_PERLOOP ? fc * c - fn : c;
+  if (a.chk_counts) {
+    // Eq. (1): target position tS in this trip, producers through it
+    const int32_t tS = gl - lo + 1 - fk;
+    const int32_t cm = tS > 0 ? lo + tS : 0;
+    const int32_t m = cm == 0 ? 0 : MODE == SYNC_THR_PERLOOP ? fc * cm - fn : cm;
+    if (T != m) {
+      atomicAdd(S.tally + (T < m ? 0 : 1), 1ull);
+      atomicMin(S.tally + 2, (unsigned long long)(__ldg(a.dseg + r) + gl));
+    }
+  }
+  return T;
+}
+
 // Iterations lo .. hi-1 of a loop whose body is one straight-line segment of
 // one chunk (or, barrier-free, one multi-iteration chunk) and whose lanes
 // wait on at most kMaxDeps semaphores each; the first iteration start has
@@ -301,10 +390,10 @@ __device__ __forceinline__ void barrier_all(const WarpSmem& S, int ne, int32_t c
 // waited semaphores' increment counts and the next iteration's thresholds.
 // Returns 0, SYNC_PROG_DEADLOCK or SIM_FALLBACK (then the program is
 // abandoned, so nothing is written back).
-template <int MODE, bool BB, bool TL>
+template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi,
                                              const int4 ch, const LaneRec& L, int32_t lo, int32_t hi,
-                                             int32_t ctag, int lane, unsigned long long& chk) {
+                                             int32_t ctag, int lane, int lc, unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int32_t ii = a.prm.ii;
@@ -362,17 +451,29 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
   const int32_t P = (BB ? 0 : wcost) + ((L.meta.w & LANE_ITER_START) ? iter_cost : 0);
   const int32_t A = P + ii;                           // cursor advance of a valid lane with no wait
   int32_t T0n = 0, T1n = 0;
-  {
+  int32_t fk0 = -1, fc0 = 0, fn0 = 0, fk1 = -1, fc1 = 0, fn1 = 0;   // fused: see fused_setup
+  if (FUSED) {
+    const bool vn = have && copy < hi - lo;
+    if (vn && ndep > 0) fused_setup<MODE>(a, S, L.rec.w, lo, hi, copy, copies, lc, fk0, fc0, fn0);
+    if (vn && ndep > 1) fused_setup<MODE>(a, S, L.rec.w + 1, lo, hi, copy, copies, lc, fk1, fc1, fn1);
+  } else {
     const bool vn = have && copy < hi - lo;
     if (vn && ndep > 0) T0n = __ldg(L.tp[0] + lo + copy);
     if (vn && ndep > 1) T1n = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + lo + copy);
   }
   for (int32_t g = lo; g < hi;) {
     const int32_t v = min(copies, hi - g);
-    const int32_t T0 = T0n, T1 = T1n;
+    int32_t T0, T1;
+    if (FUSED) {
+      T0 = have && copy < v && ndep > 0 ? fused_iter<MODE>(a, S, L.rec.w, fk0, fc0, fn0, g + copy, lo, lc) : 0;
+      T1 = have && copy < v && ndep > 1 ? fused_iter<MODE>(a, S, L.rec.w + 1, fk1, fc1, fn1, g + copy, lo, lc) : 0;
+    } else {
+      T0 = T0n;
+      T1 = T1n;
+    }
     const int32_t gn = g + v;
     const bool valid = have && copy < v;
-    if (gn < hi) {
+    if (!FUSED && gn < hi) {
       const bool vn = have && copy < hi - gn;
       if (vn && ndep > 0) T0n = __ldg(L.tp[0] + gn + copy);
       if (vn && ndep > 1) T1n = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + gn + copy);
@@ -511,9 +612,9 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
 // one chunk (or, barrier-free, one multi-iteration chunk); the first
 // iteration start has been charged.  The lane's record and thresholds stay
 // in registers; the next chunk's thresholds load while this one runs.
-template <int MODE, bool BB, bool TL>
+template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi, const int4 ch,
-                                        int32_t lo, int32_t hi, int32_t ctag, int lane,
+                                        int32_t lo, int32_t hi, int32_t ctag, int lane, int lc,
                                         unsigned long long& chk) {
   const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int32_t copies = ch.z;
@@ -521,19 +622,19 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
   LaneRec L;
   load_lane(a, ch, lane, L);
   if (!__ballot_sync(kFull, have && L.rec.z > kMaxDeps))
-    return run_loop_regs<MODE, BB, TL>(a, S, pi, ch, L, lo, hi, ctag, lane, chk);
+    return run_loop_regs<MODE, BB, TL, FUSED>(a, S, pi, ch, L, lo, hi, ctag, lane, lc, chk);
   set_groups(S, L, lane, have, min(copies, hi - lo), ctag);
   int32_t Tn[kMaxDeps];
-  load_thr(L, have && L.meta.y < hi - lo, lo + L.meta.y, Tn);
+  load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - lo, lo + L.meta.y, lc, lo, Tn);
   for (int32_t g = lo; g < hi;) {
     const int32_t v = min(copies, hi - g);
     int32_t T[kMaxDeps];
 #pragma unroll
     for (int j = 0; j < kMaxDeps; ++j) T[j] = Tn[j];
     const int32_t gn = g + v;
-    if (gn < hi) load_thr(L, have && L.meta.y < hi - gn, gn + L.meta.y, Tn);
+    if (gn < hi) load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - gn, gn + L.meta.y, lc, lo, Tn);
     if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
-    const int verdict = run_chunk<MODE, BB, TL>(a, S, ch, L, T, g, v, ctag, lane, chk);
+    const int verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, chk);
     if (verdict) return verdict;
     g = gn;
     if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
@@ -545,14 +646,20 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
   return 0;
 }
 
-template <int MODE, bool BB, bool TL>
+template <int MODE, bool BB, bool TL, bool FUSED>
 __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   WarpSmem S;
   {
     unsigned char* p = smem_raw + wib * warp_bytes(a.sem_cap, a.frame_depth, a.ring);
+    // the walk-level table and check tallies go first in the barrier sweep and
+    // last in the barrier-free one (a measured code-generation preference)
     S.semhb = reinterpret_cast<int64_t*>(p); p += 8 * a.sem_cap;
+    if (BB) {
+      S.tally = reinterpret_cast<unsigned long long*>(p); p += 3 * 8;
+      S.lvl = reinterpret_cast<int2*>(p); p += 8 * (a.frame_depth + 1);
+    }
     S.frames = reinterpret_cast<Frame*>(p); p += sizeof(Frame) * a.frame_depth;
     S.t = reinterpret_cast<int32_t*>(p); p += 4 * 32;
     S.lr = reinterpret_cast<int32_t*>(p); p += 4 * 32;
@@ -561,7 +668,12 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     S.grp = reinterpret_cast<uint32_t*>(p); p += 4 * a.sem_cap;
     S.tag = reinterpret_cast<int32_t*>(p); p += 4 * a.sem_cap;
     S.ring = reinterpret_cast<int32_t*>(p); p += 4 * (size_t)a.ring * a.sem_cap;
-    S.rank_lane = reinterpret_cast<uint8_t*>(p);
+    S.rank_lane = reinterpret_cast<uint8_t*>(p); p += 32 * (size_t)a.sem_cap;
+    if (!BB) {
+      p = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 7) & ~uintptr_t(7));
+      S.tally = reinterpret_cast<unsigned long long*>(p); p += 3 * 8;
+      S.lvl = reinterpret_cast<int2*>(p);
+    }
     S.rmask = a.ring - 1;
   }
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
@@ -584,6 +696,11 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       S.tag[i] = -1;
     }
     S.t[lane] = 0; S.lr[lane] = 0; S.nn[lane] = 0;
+    if (FUSED && lane == 0) {
+      S.lvl[0] = make_int2(0, 0);                      // the top-level loop: iteration 0 of a trip at 0
+      S.tally[0] = S.tally[1] = 0;
+      S.tally[2] = ~0ull;
+    }
     __syncwarp();
     unsigned long long chk = 0;
     int32_t loop = pi.loop_base, item = 0, g = 0, g_end = 1, sp = 0, ctag = 0;
@@ -595,6 +712,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
         if (++g < g_end) {
           if (lane < pi.ne) S.t[lane] += iter_cost;
+          if (FUSED && lane == 0) S.lvl[sp].x = g;
           __syncwarp();
           item = 0;
         } else {
@@ -625,14 +743,15 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
             const bool multi = !BB && body.w >= 0;
             if (body.x == ITEM_SEG && (multi || body.z == 1)) {
               // a loop around one chunk: all its iterations in registers
-              verdict = run_loop<MODE, BB, TL>(a, S, pi, __ldg(a.chunk + (multi ? body.w : body.y)), lo, hi,
-                                               ++ctag, lane, chk);
+              verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + (multi ? body.w : body.y)), lo,
+                                                      hi, ++ctag, lane, sp + 1, chk);
               if (verdict) break;
               continue;
             }
           }
           if (lane == 0) S.frames[sp] = Frame{loop, item, g, g_end};
           ++sp;
+          if (FUSED && lane == 0) S.lvl[sp] = make_int2(lo, lo);
           loop = it.y; item = 0; g = lo; g_end = hi;
           pbeg = cb;
           pend = ce;
@@ -647,9 +766,10 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         LaneRec Lr;
         load_lane(a, ch, lane, Lr);
         int32_t T[kMaxDeps];
-        load_thr(Lr, lane < ch.y && Lr.meta.y < v, g + Lr.meta.y, T);
+        const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
+        load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y && Lr.meta.y < v, g + Lr.meta.y, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, v, ++ctag);
-        verdict = run_chunk<MODE, BB, TL>(a, S, ch, Lr, T, g, v, ctag, lane, chk);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, chk);
         if (verdict) break;
         g += v - 1;
         item = pend - pbeg;                            // continue at the END of iteration g
@@ -660,9 +780,10 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         LaneRec Lr;
         load_lane(a, ch, lane, Lr);
         int32_t T[kMaxDeps];
-        load_thr(Lr, lane < ch.y, g, T);
+        const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
+        load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y, g, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, 1, ++ctag);
-        verdict = run_chunk<MODE, BB, TL>(a, S, ch, Lr, T, g, 1, ctag, lane, chk);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, chk);
       }
       if (verdict) break;
       ++item;
@@ -684,6 +805,12 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       a.makespan[p] = ok ? ms : -1;
       a.checksum[p] = ok ? chk : 0ull;
       a.status[p] = verdict;
+      // fused check: the pairs of programs that ran to the end
+      if (FUSED && ok && a.chk_counts) {
+        if (S.tally[0]) atomicAdd(a.chk_counts + 0, S.tally[0]);
+        if (S.tally[1]) atomicAdd(a.chk_counts + 1, S.tally[1]);
+        if (S.tally[2] != ~0ull) atomicMin(a.chk_first, S.tally[2]);
+      }
     }
     __syncwarp();
   }
@@ -707,8 +834,8 @@ cudaError_t launch3(const SweepArgs& a, size_t smem, int num_sms, cudaStream_t s
     kern<<<grid, kWarps * 32, smem, s>>>(a);
     return cudaGetLastError();
   };
-  if (a.issue) return run(k_sweep<MODE, BB, true>);
-  return run(k_sweep<MODE, BB, false>);
+  if (a.dep) return a.issue ? run(k_sweep<MODE, BB, true, true>) : run(k_sweep<MODE, BB, false, true>);
+  return a.issue ? run(k_sweep<MODE, BB, true, false>) : run(k_sweep<MODE, BB, false, false>);
 }
 
 }  // namespace

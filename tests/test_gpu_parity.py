@@ -60,18 +60,22 @@ def compare_all(sg, batch, params=None, timeline=False, modes=MODES):
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
         for v in variants_for(mode):
-            res = sg.sync_simulate(h, mode, thr, sim_params(prm), v, timeline=timeline)
             ref = oracle.simulate(batch, want, mode, v, prm, timeline=timeline)
-            P = batch.n_programs
-            st = res.status.cpu().numpy()[:P]
-            assert np.array_equal(st, ref.status), (mode, v)
-            assert np.array_equal(res.makespan.cpu().numpy()[:P], ref.makespan), (mode, v)
-            ck = res.checksum.cpu().numpy()[:P].view(np.uint64)
-            assert np.array_equal(ck, ref.checksum), (mode, v)
-            if timeline:
-                ok = np.repeat(ref.status == 0, _instances_per_program(batch))
-                assert np.array_equal(res.issue.cpu().numpy()[:ninst][ok], ref.issue[ok])
-                assert np.array_equal(res.retire.cpu().numpy()[:ninst][ok], ref.retire[ok])
+            res = sg.sync_simulate(h, mode, thr, sim_params(prm), v, timeline=timeline)
+            fused, fcounts, ffirst = sg.sync_simulate_fused(h, mode, sim_params(prm), v, timeline=timeline,
+                                                            check=True)
+            assert fcounts.cpu().tolist() == [0, 0] and ffirst.item() == -1, (mode, v)
+            for name, r in (("array", res), ("fused", fused)):
+                P = batch.n_programs
+                st = r.status.cpu().numpy()[:P]
+                assert np.array_equal(st, ref.status), (name, mode, v)
+                assert np.array_equal(r.makespan.cpu().numpy()[:P], ref.makespan), (name, mode, v)
+                ck = r.checksum.cpu().numpy()[:P].view(np.uint64)
+                assert np.array_equal(ck, ref.checksum), (name, mode, v)
+                if timeline:
+                    ok = np.repeat(ref.status == 0, _instances_per_program(batch))
+                    assert np.array_equal(r.issue.cpu().numpy()[:ninst][ok], ref.issue[ok]), (name, mode, v)
+                    assert np.array_equal(r.retire.cpu().numpy()[:ninst][ok], ref.retire[ok]), (name, mode, v)
     return h
 
 
@@ -322,6 +326,7 @@ def test_repeated_calls_are_identical(sg):
 def test_full_size_sampled(sg, name):
     """The full configuration in one launch; a sample of its programs is
     recomputed by the oracle program by program."""
+    import torch
     batch = workloads.generate(name)
     P = batch.n_programs
     h = sg.sync_load_programs(batch)
@@ -333,6 +338,11 @@ def test_full_size_sampled(sg, name):
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
         sims = {v: sg.sync_simulate(h, mode, thr, variant=v) for v in variants_for(mode)}
+        for v in variants_for(mode):      # fused: identical results on every program
+            f, fc, ff = sg.sync_simulate_fused(h, mode, variant=v, check=True)
+            assert fc.cpu().tolist() == [0, 0] and ff.item() == -1, (name, mode, v)
+            for k in ("status", "makespan", "checksum"):
+                assert torch.equal(getattr(f, k), getattr(sims[v], k)), (name, mode, v, k)
         for p in sample.tolist():
             one = workloads.generate(name, n_programs=1, first_program=p)
             want = oracle.thresholds(one, mode)
