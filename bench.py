@@ -118,7 +118,7 @@ class ClockSampler:
 
 def kernel_hash() -> str:
     h = hashlib.sha256()
-    for f in ("k_thresholds.cu", "k_simulate.cu", "k_sweep.cu", "enc.h"):
+    for f in ("k_thresholds.cu", "k_simulate.cu", "k_sweep.cu", "enc.h", "waitval.cuh"):
         with open(os.path.join(ROOT, "paper_2608_13757_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
