@@ -49,7 +49,8 @@ class _Batch(ctypes.Structure):
             "prog_loop_ptr", "prog_instr_ptr", "prog_dep_ptr", "prog_n_engines",
             "loop_parent", "loop_pos", "instr_loop", "instr_pos", "instr_engine",
             "instr_latency", "dep_prod", "dep_cons", "dep_k")
-    ] + [("trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("trips", ctypes.POINTER(ctypes.c_int32))]
+    ] + [("trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("trips", ctypes.POINTER(ctypes.c_int32)),
+         ("eng_trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("eng_trips", ctypes.POINTER(ctypes.c_int32))]
 
 
 class SimParams(ctypes.Structure):
@@ -105,8 +106,10 @@ class _View:
         cb = _Batch()
         cb.n_programs = int(batch.n_programs)
         for name, _ in _Batch._fields_[1:]:
-            a = getattr(batch, name)
-            dt = np.int64 if name == "trip_ptr" else np.int32
+            a = getattr(batch, name, None)
+            if a is None:                 # shared trips: the per-engine rows stay NULL
+                continue
+            dt = np.int64 if name in ("trip_ptr", "eng_trip_ptr") else np.int32
             a = np.ascontiguousarray(a, dtype=dt)
             self.keep[name] = a
             setattr(cb, name, _ptr(a, ctypes.c_int64 if dt == np.int64 else ctypes.c_int32))

@@ -95,17 +95,23 @@ typedef unsigned __int128 u128;
 typedef struct {
   int32_t ne, nl, nx, nd;
   const int32_t *par, *lpos, *xl, *xp, *xe, *xlat, *dp, *dc, *dk;
-  const int64_t *tptr;
+  const int64_t *tptr;               /* per loop: first trip of the current view */
   const int32_t *trips;
   int32_t maxdepth;
   int32_t *depth;
-  int64_t *total;
+  int64_t *total;                    /* per loop: iterations in the current view */
+  /* per-engine trips: rows (loop, engine) of this program, their totals,
+   * and the engine whose trips the view (tptr, trips, total) shows */
+  int div, view;
+  const int64_t *etptr;
+  int64_t *etot, *vtptr;
   int32_t *body_ptr, *body;          /* items by position: x >= 0, or -(loop+1) */
   int32_t *prod_ptr, *prod_dep;      /* dependencies grouped by producer */
   int32_t *cons_ptr, *cons_dep;      /* dependencies grouped by consumer */
 } prog_t;
 
 static void prog_close(prog_t *P) {
+  free(P->etot); free(P->vtptr);
   free(P->depth); free(P->total); free(P->body_ptr); free(P->body);
   free(P->prod_ptr); free(P->prod_dep); free(P->cons_ptr); free(P->cons_dep);
   memset(P, 0, sizeof *P);
@@ -129,6 +135,35 @@ static int group(int32_t n, int32_t m, const int32_t *key, int32_t **ptr, int32_
   free(fill);
   return ORC_OK;
 }
+
+/* Per-engine trips: show engine e's trips and totals through tptr, trips
+ * and total (no-op for shared trips). */
+static void prog_view(prog_t *P, int32_t e) {
+  if (!P->div || P->view == e) return;
+  for (int32_t l = 0; l < P->nl; ++l) {
+    P->vtptr[l] = P->etptr[(int64_t)l * P->ne + e];
+    P->total[l] = P->etot[(int64_t)l * P->ne + e];
+  }
+  P->view = e;
+}
+
+/* iterations of loop l on engine e */
+static int64_t tot_on(const prog_t *P, int32_t l, int32_t e) {
+  return P->div ? P->etot[(int64_t)l * P->ne + e] : P->total[l];
+}
+
+/* trip of loop m on engine e during global iteration g of its parent there */
+static int32_t trip_on(const prog_t *P, int32_t m, int32_t e, int64_t g) {
+  return P->div ? P->trips[P->etptr[(int64_t)m * P->ne + e] + g] : P->trips[P->tptr[m] + g];
+}
+
+/* pairs of dependency d: its consumer's instances */
+static int64_t cons_total(const prog_t *P, int32_t d) {
+  return tot_on(P, P->xl[P->dc[d]], P->xe[P->dc[d]]);
+}
+
+/* instances of instruction x */
+static int64_t inst_total(const prog_t *P, int32_t x) { return tot_on(P, P->xl[x], P->xe[x]); }
 
 static int prog_open(const orc_batch *b, int32_t p, prog_t *P) {
   memset(P, 0, sizeof *P);
@@ -155,18 +190,50 @@ static int prog_open(const orc_batch *b, int32_t p, prog_t *P) {
     if (P->depth[l] > P->maxdepth) P->maxdepth = P->depth[l];
   }
   /* trips: one per iteration of the parent; the top-level loop runs once */
-  for (int32_t l = 0; l < nl; ++l) {
-    int64_t n = P->tptr[l + 1] - P->tptr[l];
-    int64_t want = l == 0 ? 1 : P->total[P->par[l]];
-    if (n != want) return ORC_ERR_MALFORMED;
-    int64_t s = 0;
-    for (int64_t j = 0; j < n; ++j) {
-      int32_t t = P->trips[P->tptr[l] + j];
-      if (t < 0) return ORC_ERR_MALFORMED;
-      s += t;
+  if (b->eng_trip_ptr) {
+    /* per-engine rows: (loop l, engine e) is row rb + l*ne + e */
+    int64_t rb = 0;
+    for (int32_t q = 0; q < p; ++q)
+      rb += (int64_t)(b->prog_loop_ptr[q + 1] - b->prog_loop_ptr[q]) * b->prog_n_engines[q];
+    int32_t ne = P->ne;
+    P->div = 1;
+    P->etptr = b->eng_trip_ptr + rb;
+    P->etot = (int64_t *)calloc((size_t)nl * ne, sizeof(int64_t));
+    P->vtptr = (int64_t *)calloc((size_t)nl, sizeof(int64_t));
+    if (!P->etot || !P->vtptr || !b->eng_trips) return P->etot && P->vtptr ? ORC_ERR_ARG : ORC_ERR_OOM;
+    for (int32_t l = 0; l < nl; ++l)
+      for (int32_t e = 0; e < ne; ++e) {
+        const int64_t *r = P->etptr + (int64_t)l * ne + e;
+        int64_t n = r[1] - r[0];
+        int64_t want = l == 0 ? 1 : P->etot[(int64_t)P->par[l] * ne + e];
+        if (n != want) return ORC_ERR_MALFORMED;
+        int64_t s = 0;
+        for (int64_t j = 0; j < n; ++j) {
+          int32_t t = b->eng_trips[r[0] + j];
+          if (t < 0) return ORC_ERR_MALFORMED;
+          s += t;
+        }
+        if (l == 0 && s != 1) return ORC_ERR_MALFORMED;
+        P->etot[(int64_t)l * ne + e] = s;
+      }
+    P->trips = b->eng_trips;
+    P->tptr = P->vtptr;
+    P->view = -1;
+    prog_view(P, 0);
+  } else {
+    for (int32_t l = 0; l < nl; ++l) {
+      int64_t n = P->tptr[l + 1] - P->tptr[l];
+      int64_t want = l == 0 ? 1 : P->total[P->par[l]];
+      if (n != want) return ORC_ERR_MALFORMED;
+      int64_t s = 0;
+      for (int64_t j = 0; j < n; ++j) {
+        int32_t t = P->trips[P->tptr[l] + j];
+        if (t < 0) return ORC_ERR_MALFORMED;
+        s += t;
+      }
+      if (l == 0 && s != 1) return ORC_ERR_MALFORMED;
+      P->total[l] = s;
     }
-    if (l == 0 && s != 1) return ORC_ERR_MALFORMED;
-    P->total[l] = s;
   }
   for (int32_t x = 0; x < nx; ++x) {
     if (P->xl[x] < 0 || P->xl[x] >= nl || P->xp[x] < 0) return ORC_ERR_MALFORMED;
@@ -363,8 +430,8 @@ int orc_sizes(const orc_batch *b, int64_t *n_pairs, int64_t *n_instances) {
     prog_t P;
     int rc = prog_open(b, p, &P);
     if (rc) { prog_close(&P); return rc; }
-    for (int32_t d = 0; d < P.nd; ++d) np += P.total[P.xl[P.dc[d]]];
-    for (int32_t x = 0; x < P.nx; ++x) ni += P.total[P.xl[x]];
+    for (int32_t d = 0; d < P.nd; ++d) np += cons_total(&P, d);
+    for (int32_t x = 0; x < P.nx; ++x) ni += inst_total(&P, x);
     prog_close(&P);
   }
   if (n_pairs) *n_pairs = np;
@@ -421,45 +488,83 @@ static void bf_visit(walker *w, int32_t x) {
   L->n++;
 }
 
+/* Eq. (1) by definition for every dependency of the program, in the pair
+ * layout of the current view */
+static int prog_bruteforce(prog_t *P, int mode, int32_t *out) {
+  inst_list L;
+  memset(&L, 0, sizeof L);
+  int rc = walk(P, bf_visit, &L);
+  int64_t *ord = NULL, *ioff = NULL;
+  if (rc == ORC_OK && mode == ORC_PERENGINE) rc = engine_ordinals(P, &ord, &ioff);
+  int64_t *t = (int64_t *)malloc(((size_t)P->maxdepth + 1) * sizeof(int64_t));
+  if (!t && rc == ORC_OK) rc = ORC_ERR_OOM;
+  int64_t base = 0;
+  for (int32_t d = 0; d < P->nd && rc == ORC_OK; ++d) {
+    dep_class dc = classify(P, d);
+    int32_t dS = P->depth[dc.S];
+    for (int64_t i = 0; i < L.n && rc == ORC_OK; ++i) {
+      if (L.x[i] != P->dc[d]) continue;
+      /* target t = v restricted to the common loops, minus k on S */
+      for (int32_t j = 0; j <= dS; ++j) t[j] = L.vec[L.voff[i] + j];
+      t[dS] -= P->dk[d];
+      int64_t c = 0;
+      if (t[dS] > 0) {
+        for (int64_t q = 0; q < L.n; ++q) {
+          if (L.x[q] != P->dp[d]) continue;
+          int cmp = 0;
+          for (int32_t j = 0; j <= dS && cmp == 0; ++j) {
+            int64_t a = L.vec[L.voff[q] + j];
+            cmp = a < t[j] ? -1 : a > t[j];
+          }
+          if (cmp <= 0) ++c;
+        }
+      }
+      rc = store(out, base + L.g[i], mode, c, &dc, ord ? ord + ioff[P->dp[d]] : NULL);
+    }
+    base += P->total[P->xl[P->dc[d]]];
+  }
+  free(ord); free(ioff);
+  free(t); free(L.x); free(L.g); free(L.voff); free(L.vec);
+  return rc;
+}
+
+/* Per-engine trips: every dependency is evaluated in its consumer engine's
+ * view (the loop-entry counts of Eq. (1) are the consumer engine's); f
+ * computes all dependencies of one view, and each keeps the segment of the
+ * view of its consumer's engine. */
+static int per_consumer_view(prog_t *P, int mode, int32_t *out,
+                             int (*f)(prog_t *, int, int32_t *)) {
+  if (!P->div) return f(P, mode, out);
+  if (mode == ORC_PERENGINE) return ORC_ERR_ARG;
+  int rc = ORC_OK;
+  for (int32_t e = 0; e < P->ne && rc == ORC_OK; ++e) {
+    prog_view(P, e);
+    int64_t nv = 0;
+    for (int32_t d = 0; d < P->nd; ++d) nv += P->total[P->xl[P->dc[d]]];
+    int32_t *tmp = (int32_t *)malloc(((size_t)nv + 1) * sizeof(int32_t));
+    if (!tmp) return ORC_ERR_OOM;
+    rc = f(P, mode, tmp);
+    int64_t src = 0, dst = 0;
+    for (int32_t d = 0; d < P->nd && rc == ORC_OK; ++d) {
+      int64_t n = P->total[P->xl[P->dc[d]]];
+      if (P->xe[P->dc[d]] == e) memcpy(out + dst, tmp + src, (size_t)n * sizeof(int32_t));
+      src += n;
+      dst += cons_total(P, d);
+    }
+    free(tmp);
+  }
+  prog_view(P, 0);
+  return rc;
+}
+
 int orc_thresholds_bruteforce(const orc_batch *b, int mode, int32_t *out) {
   if (!b || !out || (mode != ORC_COUNT && mode != ORC_PERLOOP && mode != ORC_PERENGINE)) return ORC_ERR_ARG;
   int64_t base = 0;
   for (int32_t p = 0; p < b->n_programs; ++p) {
     prog_t P;
     int rc = prog_open(b, p, &P);
-    if (rc) { prog_close(&P); return rc; }
-    inst_list L;
-    memset(&L, 0, sizeof L);
-    rc = walk(&P, bf_visit, &L);
-    int64_t *ord = NULL, *ioff = NULL;
-    if (rc == ORC_OK && mode == ORC_PERENGINE) rc = engine_ordinals(&P, &ord, &ioff);
-    int64_t *t = (int64_t *)malloc(((size_t)P.maxdepth + 1) * sizeof(int64_t));
-    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) {
-      dep_class dc = classify(&P, d);
-      int32_t dS = P.depth[dc.S];
-      for (int64_t i = 0; i < L.n && rc == ORC_OK; ++i) {
-        if (L.x[i] != P.dc[d]) continue;
-        /* target t = v restricted to the common loops, minus k on S */
-        for (int32_t j = 0; j <= dS; ++j) t[j] = L.vec[L.voff[i] + j];
-        t[dS] -= P.dk[d];
-        int64_t c = 0;
-        if (t[dS] > 0) {
-          for (int64_t q = 0; q < L.n; ++q) {
-            if (L.x[q] != P.dp[d]) continue;
-            int cmp = 0;
-            for (int32_t j = 0; j <= dS && cmp == 0; ++j) {
-              int64_t a = L.vec[L.voff[q] + j];
-              cmp = a < t[j] ? -1 : a > t[j];
-            }
-            if (cmp <= 0) ++c;
-          }
-        }
-        rc = store(out, base + L.g[i], mode, c, &dc, ord ? ord + ioff[P.dp[d]] : NULL);
-      }
-      base += P.total[P.xl[P.dc[d]]];
-    }
-    free(ord); free(ioff);
-    free(t); free(L.x); free(L.g); free(L.voff); free(L.vec);
+    if (rc == ORC_OK) rc = per_consumer_view(&P, mode, out + base, prog_bruteforce);
+    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) base += cons_total(&P, d);
     prog_close(&P);
     if (rc) return rc;
   }
@@ -543,8 +648,8 @@ int orc_thresholds(const orc_batch *b, int mode, int32_t *out) {
   for (int32_t p = 0; p < b->n_programs; ++p) {
     prog_t P;
     int rc = prog_open(b, p, &P);
-    if (rc == ORC_OK) rc = prog_thresholds(&P, mode, out + base);
-    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) base += P.total[P.xl[P.dc[d]]];
+    if (rc == ORC_OK) rc = per_consumer_view(&P, mode, out + base, prog_thresholds);
+    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) base += cons_total(&P, d);
     prog_close(&P);
     if (rc) return rc;
   }
@@ -619,9 +724,10 @@ int orc_register_replay(const orc_batch *b, int mode, int32_t *out) {
       for (int32_t d = 0; d < P.nd; ++d) {
         R.cls[d] = classify(&P, d);
         R.pair_off[d] = off;
-        off += P.total[P.xl[P.dc[d]]];
+        off += cons_total(&P, d);
       }
       for (int32_t e = 0; e < P.ne; ++e) {
+        prog_view(&P, e);                   /* engine e walks its own trips */
         memset(R.r, 0, (size_t)P.nl * sizeof(int64_t));
         memset(R.rh, 0, (size_t)P.nl * sizeof(int64_t));
         R.e = e;
@@ -652,10 +758,10 @@ int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[
     prog_t P;
     int rc = prog_open(b, p, &P);
     int64_t np = 0;
-    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) np += P.total[P.xl[P.dc[d]]];
+    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) np += cons_total(&P, d);
     int32_t *want = (int32_t *)malloc(((size_t)np + 1) * sizeof(int32_t));
     if (rc == ORC_OK && !want) rc = ORC_ERR_OOM;
-    if (rc == ORC_OK) rc = prog_thresholds(&P, mode, want);
+    if (rc == ORC_OK) rc = per_consumer_view(&P, mode, want, prog_thresholds);
     for (int64_t i = 0; i < np && rc == ORC_OK; ++i) {
       int32_t got = thr[base + i];
       if (got == want[i]) continue;
@@ -742,7 +848,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
     E->bar_passed = 0;
     if (!X->barrier) E->t += X->stmt_cost;
     int32_t m = -it - 1;
-    int32_t trip = P->trips[P->tptr[m] + f->g];
+    int32_t trip = trip_on(P, m, e, f->g);
     f->item++;
     if (trip > 0) {
       frame *c = &E->st[E->sp++];
@@ -803,18 +909,19 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   int64_t stmt_cost = unrolled ? 0 : q->c_regop;
   /* the static time bound */
   u128 bound = 0;
-  int64_t stmts = 0, iters = 0;
-  for (int32_t l = 1; l < nl; ++l) { stmts += P->total[P->par[l]]; iters += P->total[l]; }
+  int64_t stmts = 0, iters = 0;      /* summed over the engines */
+  for (int32_t e = 0; e < ne; ++e)
+    for (int32_t l = 1; l < nl; ++l) { stmts += tot_on(P, P->par[l], e); iters += tot_on(P, l, e); }
   for (int32_t x = 0; x < nx; ++x) {
     int64_t per = (int64_t)P->xlat[x] + q->ii;
     if (!barrier) per += wcost[x];
-    bound += (u128)P->total[P->xl[x]] * (u128)per;
+    bound += (u128)inst_total(P, x) * (u128)per;
   }
-  if (barrier) {
-    bound += (u128)ne * (u128)iters * (u128)q->c_branch;
-    bound += (u128)(stmts + iters) * (u128)q->c_barrier;
+  if (barrier) {                     /* shared trips: every engine has the same counts */
+    bound += (u128)iters * (u128)q->c_branch;
+    bound += (u128)(stmts / ne + iters / ne) * (u128)q->c_barrier;
   } else {
-    bound += (u128)ne * ((u128)stmts * (u128)stmt_cost + (u128)iters * (u128)iter_cost);
+    bound += (u128)stmts * (u128)stmt_cost + (u128)iters * (u128)iter_cost;
   }
   if (bound > (u128)INT32_MAX) {
     free(wcost);
@@ -839,12 +946,12 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
             !incs || !E) ? ORC_ERR_OOM : ORC_OK;
   if (rc == ORC_OK) {
     int64_t off = 0;
-    for (int32_t d = 0; d < nd; ++d) { X.pair_off[d] = off; off += P->total[P->xl[P->dc[d]]]; }
+    for (int32_t d = 0; d < nd; ++d) { X.pair_off[d] = off; off += cons_total(P, d); }
     off = 0;
     for (int32_t x = 0; x < nx; ++x) {
-      X.inst_off[x] = off; off += P->total[P->xl[x]];
+      X.inst_off[x] = off; off += inst_total(P, x);
       X.own_sem[x] = mode == ORC_COUNT ? x : mode == ORC_PERLOOP ? P->xl[x] * ne + P->xe[x] : P->xe[x];
-      incs[X.own_sem[x]] += P->total[P->xl[x]];
+      incs[X.own_sem[x]] += inst_total(P, x);
     }
     for (int32_t d = 0; d < nd; ++d) {
       int32_t p = P->dp[d];
@@ -919,11 +1026,13 @@ int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim
   for (int32_t p = 0; p < b->n_programs; ++p) {
     prog_t P;
     int rc = prog_open(b, p, &P);
+    /* per-engine trips: no common barrier sequence, no per-engine positions */
+    if (rc == ORC_OK && P.div && (variant != ORC_BARRIER_FREE || mode == ORC_PERENGINE)) rc = ORC_ERR_ARG;
     if (rc == ORC_OK)
       rc = sim_program(&P, mode, thr + pbase, prm, variant, makespan + p, checksum + p,
                        status + p, issue ? issue + ibase : NULL, retire ? retire + ibase : NULL);
-    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) pbase += P.total[P.xl[P.dc[d]]];
-    for (int32_t x = 0; x < P.nx && rc == ORC_OK; ++x) ibase += P.total[P.xl[x]];
+    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) pbase += cons_total(&P, d);
+    for (int32_t x = 0; x < P.nx && rc == ORC_OK; ++x) ibase += inst_total(&P, x);
     prog_close(&P);
     if (rc) return rc;
   }

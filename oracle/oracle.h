@@ -30,6 +30,12 @@ typedef struct {
   const int32_t *dep_prod, *dep_cons, *dep_k;
   const int64_t *trip_ptr;
   const int32_t *trips;
+  /* optional per-engine trip counts (NULL: every engine runs `trips`): one
+   * row per (program, loop, engine), programs in order, then loops, then
+   * engines; a row holds the loop's trips on that engine during each global
+   * iteration of its parent on that engine.  When set, `trips` is unused. */
+  const int64_t *eng_trip_ptr;
+  const int32_t *eng_trips;
 } orc_batch;
 
 enum { ORC_OK = 0, ORC_ERR_ARG = 1, ORC_ERR_MALFORMED = 2, ORC_ERR_NOT_ALLOCATABLE = 3,
@@ -60,6 +66,17 @@ typedef struct {
   int32_t c_barrier;          /* all-engine barrier handshake + reset          */
   int32_t c_wait_ops_perengine_level; /* per-engine mode: per enclosing loop level */
 } orc_sim_params;
+
+/* Per-engine trip counts (control-flow divergence, Sec. 7.5): each engine
+ * walks the common loop tree with its own trips.  A dependency's pairs are
+ * its consumer's instances, and Eq. (1) is evaluated on the consumer
+ * engine's loop state (the loop-entry counts H_e of the consumer's engine:
+ * the registers an implementation reads); the producer's semaphore counts
+ * the producer engine's retirements, so a wait the producer engine never
+ * reaches leaves the program deadlocked.  Count and per-loop modes only,
+ * barrier-free simulation only (ORC_ERR_ARG otherwise).
+ * Global iteration indices, instance and pair layouts are per engine: an
+ * instruction has one instance per iteration of its loop on its engine. */
 
 /* Sizes: pairs and instances in the layouts above. */
 int orc_sizes(const orc_batch *b, int64_t *n_pairs, int64_t *n_instances);

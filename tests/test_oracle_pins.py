@@ -570,3 +570,164 @@ def test_program_ranges_are_independent():
     sub = workloads.concat([full], programs=[(0, p) for p in range(17, 27)])
     for k, v in sub.arrays().items():
         assert np.array_equal(v, getattr(part, k)), k
+
+
+# ------------------------------------------- per-engine trip counts (Sec. 7.5)
+
+def _divergent_batches(n=30, permille=300, **kw):
+    for seed in range(n):
+        b = workloads.random_trees(500 + seed, 1, workloads.tree_params(**kw))
+        yield seed, workloads.diverge(b, 900 + seed, permille)
+
+
+def test_divergent_rows_equal_to_shared_trips_change_nothing():
+    """Per-engine rows that repeat the shared trips give the shared batch's
+    thresholds, checks and timelines exactly."""
+    b = workloads.random_trees(31, 40, workloads.tree_params(engines_hi=4, loops_hi=5, trip_hi=4))
+    same = workloads.diverge(b, 3, permille=0)
+    assert same.divergent
+    assert oracle.sizes(same) == oracle.sizes(b)
+    for mode in (COUNT, PERLOOP):
+        t0, t1 = oracle.thresholds(b, mode), oracle.thresholds(same, mode)
+        assert np.array_equal(t0, t1)
+        assert np.array_equal(oracle.thresholds_bruteforce(same, mode), t1)
+        r0 = oracle.simulate(b, t0, mode, oracle.BARRIER_FREE, timeline=True)
+        r1 = oracle.simulate(same, t1, mode, oracle.BARRIER_FREE, timeline=True)
+        for f in ("status", "makespan", "checksum", "issue", "retire"):
+            assert np.array_equal(getattr(r0, f), getattr(r1, f)), (mode, f)
+
+
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def test_divergent_definition_counting_and_registers_agree(mode):
+    """Eq. (1) by enumeration on the consumer engine's walk, the counting
+    form and the consumer engine's register replay agree on divergent
+    programs; the checker accepts the result."""
+    n_div = 0
+    for seed, b in _divergent_batches(40, engines_hi=4, loops_hi=5, body_hi=5, trip_hi=4, max_depth=3):
+        t = oracle.thresholds(b, mode)
+        assert np.array_equal(oracle.thresholds_bruteforce(b, mode), t), seed
+        assert np.array_equal(oracle.register_replay(b, mode), t), seed
+        assert oracle.check(b, t, mode) == (0, 0, -1)
+        n_div += oracle.sizes(b) != oracle.sizes(workloads.random_trees(500 + seed, 1, workloads.tree_params(
+            engines_hi=4, loops_hi=5, body_hi=5, trip_hi=4, max_depth=3)))
+    assert n_div >= 10          # the rows really diverge
+
+
+def test_divergence_example_sec75():
+    """Sec. 7.5's case: offset 0 from a producer on one engine to a consumer
+    on another, both in a loop that runs zero times on the producer's engine
+    and once on the consumer's.  The consumer's threshold is 1 (its own
+    engine entered the loop once), the producer's count never reaches it, and
+    the program deadlocks."""
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [1], eng_trips=[[0], [1]])
+    p = b.instr(A, 0, 0)
+    c = b.instr(A, 1, 1)
+    b.dep(p, c, 0)
+    batch = b.batch()
+    assert oracle.sizes(batch) == (1, 1)     # one consumer instance; the producer never runs
+    for mode in (COUNT, PERLOOP):
+        t = oracle.thresholds(batch, mode)
+        assert t.tolist() == [1]
+        r = oracle.simulate(batch, t, mode, oracle.BARRIER_FREE)
+        assert (r.status[0], r.makespan[0], int(r.checksum[0])) == (7, -1, 0)
+
+
+@pytest.mark.parametrize("mp,mc,k", [(3, 3, 0), (2, 5, 1), (5, 2, 0), (4, 6, 2), (0, 3, 3), (2, 4, 1)])
+def test_divergent_single_loop_closed_form(mp, mc, k):
+    """One loop under the top level, producer on engine 0 (mp iterations) and
+    consumer on engine 1 (mc iterations), offset k: the consumer's g-th
+    instance (1-based) waits for max(0, g - k) producer instances, and the
+    program deadlocks exactly when the last of these exceeds mp; otherwise
+    every consumer issues after that producer instance retires."""
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [mp], eng_trips=[[mp], [mc]])
+    p = b.instr(A, 0, 0, latency=5)
+    c = b.instr(A, 1, 1, latency=2)
+    b.dep(p, c, k)
+    batch = b.batch()
+    want = [max(0, g - k) for g in range(1, mc + 1)]
+    assert oracle.thresholds(batch, COUNT).tolist() == want
+    assert oracle.thresholds(batch, PERLOOP).tolist() == want          # N = K = 1
+    r = oracle.simulate(batch, np.array(want, np.int32), COUNT, oracle.BARRIER_FREE, timeline=True)
+    if max(want, default=0) > mp:
+        assert r.status[0] == 7
+    else:
+        assert r.status[0] == 0
+        for g, c_ in enumerate(want):
+            if c_ > 0:
+                assert r.issue[mp + g] >= r.retire[c_ - 1]
+
+
+def test_divergent_unreachable_wait_deadlocks():
+    """A count threshold above the producer's instances on its own engine can
+    never be met: every such program ends in deadlock (status 7)."""
+    seen = 0
+    for seed, b in _divergent_batches(60, engines_hi=4, loops_hi=5, body_hi=5, trip_hi=4, max_depth=3):
+        t = oracle.thresholds(b, COUNT)
+        r = oracle.simulate(b, t, COUNT, oracle.BARRIER_FREE)
+        unreachable = False
+        off = 0
+        for d in range(b.n_deps):
+            px, cx = int(b.dep_prod[d]), int(b.dep_cons[d])
+            n_prod = _instances(b, px)
+            n_cons = _instances(b, cx)
+            if n_cons and int(t[off:off + n_cons].max()) > n_prod:
+                unreachable = True
+            off += n_cons
+        if unreachable:
+            seen += 1
+            assert r.status[0] == 7, seed
+    assert seen >= 3
+
+
+def _instances(b, x):
+    """Instances of instruction x of a one-program batch on its own engine."""
+    e = int(b.instr_engine[x])
+    tot = [0] * b.n_loops
+    tot[0] = 1
+    for l in range(1, b.n_loops):
+        tot[l] = int(b.engine_trips(0, l, e).sum())
+    return tot[int(b.instr_loop[x])]
+
+
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP])
+def test_divergent_timing_matches_recursive_statement(mode):
+    """Per-engine trips in the semaphore machine and in the recursive
+    statement (each engine's events follow its own trips; a wait for a
+    producer instance its engine never runs never ends): same makespans,
+    checksums, timelines and deadlocks."""
+    prm = oracle.sim_params(ii=2, c_branch=3, c_regop=1, c_barrier=7)
+    n_ok = n_dead = 0
+    for seed, b in _divergent_batches(80, permille=400, engines_hi=3, loops_hi=4, body_hi=4, trip_hi=3,
+                                      max_depth=3):
+        thr = oracle.thresholds(b, mode)
+        thr_c = oracle.thresholds(b, COUNT)
+        r = oracle.simulate(b, thr, mode, oracle.BARRIER_FREE, prm, timeline=True)
+        try:
+            ms, chk, tl = timing_model.simulate(b, thr_c, prm, False, wait_ops(b, mode, prm))
+        except timing_model.Deadlock:
+            assert r.status[0] == 7, seed
+            n_dead += 1
+            continue
+        assert r.status[0] == 0, seed
+        assert r.makespan[0] == ms and int(r.checksum[0]) == chk, seed
+        off = 0
+        for x in range(b.n_instrs):
+            n = _instances(b, x)
+            for g in range(n):
+                assert (r.issue[off + g], r.retire[off + g]) == tl[(x, g)], seed
+            off += n
+        n_ok += 1
+    assert n_ok >= 10 and n_dead >= 3
+
+
+def test_divergent_rejects_barrier_and_per_engine():
+    """The barrier scheme (no common barrier sequence) and per-engine values
+    are not defined with per-engine trips."""
+    _, b = next(_divergent_batches(1))
+    with pytest.raises(oracle.OracleError):
+        oracle.thresholds(b, PERENGINE)
+    t = oracle.thresholds(b, PERLOOP)
+    with pytest.raises(oracle.OracleError):
+        oracle.simulate(b, t, PERLOOP, oracle.BARRIER)

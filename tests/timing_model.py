@@ -13,7 +13,9 @@ engine's datapath instances.  Costs (barrier-free / barrier scheme):
 stmt c_regop / barrier; iter c_branch + 2*c_regop / c_branch; end - / barrier;
 datapath: t += the wait ops of its dependencies (barrier-free only), issue =
 max(t, producer retirements), retire = max(issue + lat, previous retire),
-t = issue + ii.  Barrier j: release = max over engines of max(t, last
+t = issue + ii.  With per-engine trip counts each engine's event list follows
+its own trips, and a wait for a producer instance its engine never runs
+never ends (deadlock).  Barrier j: release = max over engines of max(t, last
 retire) + c_barrier.  Unrolled (the straight-line program): as barrier-free
 without stmt, iter or wait-op costs.
 """
@@ -37,7 +39,7 @@ def _events(batch, e, barrier):
         body[int(par[l])].append((int(batch.loop_pos[l]), ("loop", l)))
     for l in body:
         body[l].sort()
-    trips = {l: batch.trips[batch.trip_ptr[l]:batch.trip_ptr[l + 1]] for l in range(nl)}
+    trips = {l: batch.engine_trips(0, l, e) for l in range(nl)}   # engine e's own trips
     nxt = [0] * nl
     ev = []
 

@@ -18,7 +18,13 @@ A batch is a structure of arrays (program-local ids, int32 unless noted):
   innermost common loop;
 * ``trip_ptr`` (int64, ``[n_loops+1]``) and ``trips``: the trips of loop ``l``
   during each global iteration of its parent, ``trips[trip_ptr[l]:trip_ptr[l+1]]``;
-  the top-level loop has the single trip 1.
+  the top-level loop has the single trip 1;
+* optional, for engines whose trip counts diverge: ``eng_trip_ptr`` (int64,
+  one entry per (program, loop, engine) row plus one) and ``eng_trips``: row
+  ``R_p + l*n_engines + e`` (``R_p`` = rows of the programs before ``p``)
+  holds the trips of loop ``l`` on engine ``e`` during each global iteration
+  of its parent on that engine.  When present they replace ``trips`` (which
+  then holds engine 0's trips).
 
 The named configurations follow the five workload families the engine is
 measured on (a small single-loop program, a depth-2 nest, a tiled GEMM, causal
@@ -130,6 +136,24 @@ class Batch:
     dep_k: np.ndarray
     trip_ptr: np.ndarray
     trips: np.ndarray
+    eng_trip_ptr: np.ndarray | None = None
+    eng_trips: np.ndarray | None = None
+
+    @property
+    def divergent(self) -> bool:
+        return self.eng_trip_ptr is not None
+
+    def engine_trips(self, p: int, l: int, e: int) -> np.ndarray:
+        """Trips of program p's loop l on engine e (program-local l)."""
+        if self.eng_trip_ptr is None:
+            g = int(self.prog_loop_ptr[p]) + l
+            return self.trips[self.trip_ptr[g]:self.trip_ptr[g + 1]]
+        r = self.row_base(p) + l * int(self.prog_n_engines[p]) + e
+        return self.eng_trips[self.eng_trip_ptr[r]:self.eng_trip_ptr[r + 1]]
+
+    def row_base(self, p: int) -> int:
+        nl = np.diff(self.prog_loop_ptr[:p + 1]).astype(np.int64)
+        return int((nl * self.prog_n_engines[:p].astype(np.int64)).sum())
 
     @property
     def n_loops(self) -> int:
@@ -144,7 +168,8 @@ class Batch:
         return int(self.dep_prod.shape[0])
 
     def arrays(self):
-        return {f.name: getattr(self, f.name) for f in fields(self) if f.name != "n_programs"}
+        return {f.name: getattr(self, f.name) for f in fields(self)
+                if f.name != "n_programs" and getattr(self, f.name) is not None}
 
     def copy(self) -> "Batch":
         return Batch(self.n_programs, **{k: v.copy() for k, v in self.arrays().items()})
@@ -244,8 +269,17 @@ def concat(batches, programs=None) -> Batch:
                              "trips")}
     lp, ip, dp, ne, tp = [0], [0], [0], [], []
     trip_base = 0
+    divergent = any(batches[bi].divergent for bi, _ in programs)
+    etp, etrips, ebase = [], [], 0
     for bi, p in programs:
         b = batches[bi]
+        if divergent:               # one row per (loop, engine), shared trips repeated
+            for l in range(int(b.prog_loop_ptr[p + 1] - b.prog_loop_ptr[p])):
+                for e in range(int(b.prog_n_engines[p])):
+                    t = b.engine_trips(p, l, e)
+                    etp.append(ebase)
+                    etrips.append(t)
+                    ebase += len(t)
         l0, l1 = int(b.prog_loop_ptr[p]), int(b.prog_loop_ptr[p + 1])
         x0, x1 = int(b.prog_instr_ptr[p]), int(b.prog_instr_ptr[p + 1])
         d0, d1 = int(b.prog_dep_ptr[p]), int(b.prog_dep_ptr[p + 1])
@@ -275,8 +309,60 @@ def concat(batches, programs=None) -> Batch:
         prog_dep_ptr=np.array(dp, dtype=np.int32),
         prog_n_engines=np.array(ne, dtype=np.int32),
         trip_ptr=cat(tp, np.int64),
+        eng_trip_ptr=np.array(etp + [ebase], dtype=np.int64) if divergent else None,
+        eng_trips=cat(etrips, np.int32) if divergent else None,
         **{k: cat(v, np.int32) for k, v in parts.items()},
     )
+
+
+def diverge(batch: Batch, seed: int, permille: int = 200, trip_hi: int | None = None) -> Batch:
+    """Per-engine trip counts from a shared-trip batch: every engine starts
+    from the shared trips, each (loop, engine) trip is moved by one (up or
+    down, not below 0) with probability permille/1000, and a parent iteration
+    that exists on one engine only gets a trip drawn uniformly in
+    [0, trip_hi] (default: the loop's largest shared trip).  Engine 0 keeps
+    the shared trips of loops whose parents did not diverge, so some
+    programs stay aligned.  A pure function of (batch, seed, program id)."""
+    etp, etrips, ebase = [], [], 0
+    trips0, tp0 = [], [0]
+    for p in range(batch.n_programs):
+        rng = np.random.default_rng([int(seed) & 0xFFFFFFFF, p])
+        l0, l1 = int(batch.prog_loop_ptr[p]), int(batch.prog_loop_ptr[p + 1])
+        ne = int(batch.prog_n_engines[p])
+        par = batch.loop_parent[l0:l1]
+        rows = [[None] * ne for _ in range(l1 - l0)]
+        for e in range(ne):
+            total = {}
+            for l in range(l1 - l0):
+                base = batch.trips[batch.trip_ptr[l0 + l]:batch.trip_ptr[l0 + l + 1]]
+                if l == 0:
+                    t = np.array([1], dtype=np.int64)
+                else:
+                    n = total[int(par[l])]
+                    hi = trip_hi if trip_hi is not None else (int(base.max()) if base.size else 2)
+                    t = np.empty(n, dtype=np.int64)
+                    m = min(n, base.size)
+                    t[:m] = base[:m]
+                    if n > m:
+                        t[m:] = rng.integers(0, hi + 1, size=n - m)
+                    move = rng.random(n) < permille / 1000.0
+                    step = np.where(rng.random(n) < 0.5, -1, 1)
+                    t = np.where(move, np.maximum(t + step, 0), t)
+                total[l] = int(t.sum())
+                rows[l][e] = t.astype(np.int32)
+        for l in range(l1 - l0):
+            for e in range(ne):
+                etp.append(ebase)
+                etrips.append(rows[l][e])
+                ebase += rows[l][e].size
+            trips0.append(rows[l][0])
+            tp0.append(tp0[-1] + rows[l][0].size)
+    b = batch.copy()
+    b.trips = np.concatenate(trips0).astype(np.int32) if trips0 else np.zeros(0, np.int32)
+    b.trip_ptr = np.array(tp0, dtype=np.int64)
+    b.eng_trip_ptr = np.array(etp + [ebase], dtype=np.int64)
+    b.eng_trips = np.concatenate(etrips).astype(np.int32) if etrips else np.zeros(0, np.int32)
+    return b
 
 
 class ProgramBuilder:
@@ -289,12 +375,17 @@ class ProgramBuilder:
 
     def __init__(self, n_engines: int):
         self.ne = n_engines
+        self.eng = {}
         self.loops = [(-1, 0, [1])]
         self.instrs = []
         self.deps = []
 
-    def loop(self, parent: int, pos: int, trips) -> int:
+    def loop(self, parent: int, pos: int, trips, eng_trips=None) -> int:
+        """``eng_trips``: optional list of per-engine trip lists (divergent
+        trip counts); without it every engine runs ``trips``."""
         self.loops.append((parent, pos, list(trips)))
+        if eng_trips is not None:
+            self.eng[len(self.loops) - 1] = [list(t) for t in eng_trips]
         return len(self.loops) - 1
 
     def instr(self, loop: int, pos: int, engine: int, latency: int = 1) -> int:
@@ -325,4 +416,19 @@ class ProgramBuilder:
             dep_cons=col(self.deps, 1) if self.deps else i32([]),
             dep_k=col(self.deps, 2) if self.deps else i32([]),
             trip_ptr=np.array(tp, dtype=np.int64), trips=i32(trips),
+            eng_trip_ptr=self._eng_ptr(), eng_trips=self._eng_trips(),
         )
+
+    def _eng_rows(self):
+        return [self.eng.get(l, [t] * self.ne)[e] for l, (_, _, t) in enumerate(self.loops)
+                for e in range(self.ne)]
+
+    def _eng_ptr(self):
+        if not self.eng:
+            return None
+        return np.concatenate([[0], np.cumsum([len(r) for r in self._eng_rows()])]).astype(np.int64)
+
+    def _eng_trips(self):
+        if not self.eng:
+            return None
+        return np.array([x for r in self._eng_rows() for x in r], dtype=np.int32)
