@@ -107,7 +107,28 @@ enum {
  *   trip_ptr [n_loops+1] (starting at 0) and trips [trip_ptr[n_loops]]: loop
  *     l has one trip count (>= 0) per global iteration of its parent, in
  *     trips[trip_ptr[l] .. trip_ptr[l+1]); the top-level loop has exactly one
- *     entry, equal to 1. */
+ *     entry, equal to 1;
+ *   eng_trip_ptr, eng_trips (optional, both NULL for trips shared by all
+ *     engines): per-engine trip counts (control-flow divergence, Sec. 7.5).
+ *     One row per (program, loop, engine) -- programs in order, then loops,
+ *     then engines, so program p's (loop l, engine e) is row R_p + l*ne + e
+ *     with R_p the rows of the programs before p; eng_trip_ptr [rows+1]
+ *     (starting at 0) and eng_trips [eng_trip_ptr[rows]]: a row holds the
+ *     loop's trips on that engine during each global iteration of its parent
+ *     on that engine (the top-level loop: one entry, 1).  When set, trip_ptr
+ *     and trips are not read.  Every engine then walks the loop tree with its
+ *     own trips; global iteration indices, instance and pair layouts are per
+ *     engine (an instruction has one instance per iteration of its loop on
+ *     its engine, a dependency one pair per instance of its consumer), and
+ *     Eq. (1) is evaluated on the consumer engine's loop state (the loop-entry
+ *     counts of the consumer's engine, the registers a consumer reads), while
+ *     the producer's semaphore counts the producer engine's retirements: a
+ *     wait that engine never reaches deadlocks the program.  Such handles
+ *     take COUNT and PERLOOP thresholds and the barrier-free simulation only
+ *     (SYNC_ERR_ARG otherwise): the barrier scheme needs every engine to meet
+ *     the same barriers, and a per-engine wait value is a position in the
+ *     producer engine's stream, which the consumer's loop state no longer
+ *     determines. */
 typedef struct {
   int32_t n_programs;
   const int32_t *prog_loop_ptr, *prog_instr_ptr, *prog_dep_ptr;
@@ -117,6 +138,8 @@ typedef struct {
   const int32_t *dep_prod, *dep_cons, *dep_k;
   const int64_t *trip_ptr;
   const int32_t *trips;
+  const int64_t *eng_trip_ptr;
+  const int32_t *eng_trips;
 } sync_batch_desc;
 
 typedef struct {

@@ -46,7 +46,8 @@ class BatchDesc(ctypes.Structure):
             "prog_loop_ptr", "prog_instr_ptr", "prog_dep_ptr", "prog_n_engines",
             "loop_parent", "loop_pos", "instr_loop", "instr_pos", "instr_engine",
             "instr_latency", "dep_prod", "dep_cons", "dep_k")
-    ] + [("trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("trips", ctypes.POINTER(ctypes.c_int32))]
+    ] + [("trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("trips", ctypes.POINTER(ctypes.c_int32)),
+         ("eng_trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("eng_trips", ctypes.POINTER(ctypes.c_int32))]
 
 
 class Sizes(ctypes.Structure):
@@ -133,8 +134,14 @@ def batch_desc(batch):
     desc = BatchDesc()
     desc.n_programs = int(get("n_programs"))
     for name, _ in BatchDesc._fields_[1:]:
-        is64 = name == "trip_ptr"
-        a = np.ascontiguousarray(get(name), dtype=np.int64 if is64 else np.int32)
+        is64 = name in ("trip_ptr", "eng_trip_ptr")
+        try:
+            v = get(name)
+        except (KeyError, AttributeError):
+            v = None
+        if v is None:                       # shared trips: per-engine rows stay NULL
+            continue
+        a = np.ascontiguousarray(v, dtype=np.int64 if is64 else np.int32)
         keep.append(a)
         setattr(desc, name, a.ctypes.data_as(ctypes.POINTER(ctypes.c_int64 if is64 else ctypes.c_int32)))
     return desc, keep

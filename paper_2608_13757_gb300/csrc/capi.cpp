@@ -91,7 +91,10 @@ struct ProgScratch {
   std::vector<int32_t> depth, body_ptr, body, rank, nloop_eng, x_ndeps, x_dep_begin;
   std::vector<int32_t> x_own[kModes], x_hstride[kModes], x_koff[kModes], x_levels;
   std::vector<int64_t> total, keys;
-  std::vector<int64_t> tstart_of;                 // derived trip-start array per loop, -1 if none
+  std::vector<int64_t> etot;                      // per-engine trips: iterations per (loop, engine)
+  std::vector<LoopInfo> el;                       // per-engine trips: loop table per (loop, engine)
+  std::vector<int32_t> xid;                       // per-engine trips: expansion-table entry per (loop, engine)
+  std::vector<int64_t> tstart_of;                 // derived trip-start array per loop (and engine), -1 if none
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
 };
 
@@ -135,13 +138,15 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   check_csr(d.prog_instr_ptr, P, "prog_instr_ptr");
   check_csr(d.prog_dep_ptr, P, "prog_dep_ptr");
   const int64_t NL = d.prog_loop_ptr[P], NX = d.prog_instr_ptr[P], ND = d.prog_dep_ptr[P];
-  if (NL > 0 && (!d.loop_parent || !d.loop_pos || !d.trip_ptr))
+  const bool div = d.eng_trip_ptr != nullptr;     // per-engine trip counts
+  if (NL > 0 && (!d.loop_parent || !d.loop_pos || (!div && !d.trip_ptr)))
     raise(SYNC_ERR_ARG, "loop arrays must not be NULL");
   if (NX > 0 && (!d.instr_loop || !d.instr_pos || !d.instr_engine || !d.instr_latency))
     raise(SYNC_ERR_ARG, "instruction arrays must not be NULL");
   if (ND > 0 && (!d.dep_prod || !d.dep_cons || !d.dep_k))
     raise(SYNC_ERR_ARG, "dependency arrays must not be NULL");
-  if (NL > 0) {
+  if (div && d.eng_trip_ptr[0] != 0) raise(SYNC_ERR_MALFORMED, "eng_trip_ptr[0] must be 0");
+  if (NL > 0 && !div) {
     if (d.trip_ptr[0] != 0) raise(SYNC_ERR_MALFORMED, "trip_ptr[0] must be 0");
     for (int64_t l = 0; l < NL; ++l)
       if (d.trip_ptr[l + 1] < d.trip_ptr[l]) raise(SYNC_ERR_MALFORMED, "trip_ptr is not nondecreasing");
@@ -169,7 +174,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
   std::vector<int64_t> hist_len(kModes, 0);
-  std::vector<uint8_t> reads_rowptr(NL, 0);
+  std::vector<LoopInfo> xloops;             // every (loop[, engine]) iteration space, in pidx order
+  std::vector<uint8_t> reads_rowptr;        // per xloops entry: read by a nested producer's count
+  int64_t erow = 0;                         // per-engine trips: first row of the program
   std::vector<DeriveJob> jobs;
   int64_t n_derived = 0;
   int64_t n_pairs = 0, n_pairs_padded = 0, n_inst = 0, n_iters = 0, rowptr_len = 0;
@@ -186,7 +193,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     const int32_t* lpos = d.loop_pos + l0;
     S.depth.assign(nl, 0);
     S.total.assign(nl, 0);
-    S.tstart_of.assign(nl, -1);
+    S.tstart_of.assign((size_t)nl * (div ? ne : 1), -1);
     S.anc_of.clear();
     if (par[0] != -1) raise(SYNC_ERR_MALFORMED, where(p, "loop 0 must have parent -1, loop", 0));
     int32_t depth_max = 0;
@@ -197,31 +204,69 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       if (S.depth[l] > SYNC_MAX_DEPTH) raise(SYNC_ERR_MALFORMED, where(p, "nesting deeper than SYNC_MAX_DEPTH, loop", l));
       depth_max = std::max(depth_max, S.depth[l]);
     }
-    // trips and iteration totals
-    for (int32_t l = 0; l < nl; ++l) {
-      const int64_t gl = l0 + l;
-      const int64_t t0 = d.trip_ptr[gl], t1 = d.trip_ptr[gl + 1];
-      const int64_t want = l == 0 ? 1 : S.total[par[l]];
-      if (t1 - t0 != want) raise(SYNC_ERR_MALFORMED, where(p, "trip count array length != parent's iterations, loop", l));
+    // trips and iteration totals: one iteration space per loop, or per
+    // (loop, engine) with per-engine trips; trip prefix sums (rowptr) appended
+    auto add_space = [&](int32_t l, const int32_t* trips, int64_t want) -> LoopInfo {
       int64_t tot = 0;
-      for (int64_t j = t0; j < t1; ++j) {
-        const int32_t t = d.trips[j];
-        if (t < 0) raise(SYNC_ERR_MALFORMED, where(p, "negative trip count, loop", l));
-        tot += t;
+      for (int64_t j = 0; j < want; ++j) {
+        if (trips[j] < 0) raise(SYNC_ERR_MALFORMED, where(p, "negative trip count, loop", l));
+        tot += trips[j];
       }
       if (l == 0 && tot != 1) raise(SYNC_ERR_MALFORMED, where(p, "top-level loop must run once, loop", 0));
       if (tot > kI32Max) raise(SYNC_ERR_OVERFLOW, where(p, "iterations exceed INT32_MAX, loop", l));
-      S.total[l] = tot;
-      LoopInfo& L = loop[gl];
+      LoopInfo L;
+      std::memset(&L, 0, sizeof L);
       L.parent = l == 0 ? -1 : l0 + par[l];
       L.total = (int32_t)tot;
       L.n_parent = (int32_t)want;
       L.depth = S.depth[l];
       L.rowptr_off = rowptr_len;
       L.pidx_off = n_iters;
+      rowptr_host.push_back(0);
+      for (int64_t j = 0; j < want; ++j) rowptr_host.push_back(rowptr_host.back() + trips[j]);
       rowptr_len += want + 1;
       n_iters += tot;
+      xloops.push_back(L);
+      reads_rowptr.push_back(0);
+      return L;
+    };
+    if (!div) {
+      for (int32_t l = 0; l < nl; ++l) {
+        const int64_t gl = l0 + l;
+        const int64_t t0 = d.trip_ptr[gl], t1 = d.trip_ptr[gl + 1];
+        const int64_t want = l == 0 ? 1 : S.total[par[l]];
+        if (t1 - t0 != want) raise(SYNC_ERR_MALFORMED, where(p, "trip count array length != parent's iterations, loop", l));
+        loop[gl] = add_space(l, d.trips + t0, want);
+        S.total[l] = loop[gl].total;
+      }
+      S.xid.assign((size_t)nl * ne, 0);
+      for (int32_t l = 0; l < nl; ++l)
+        for (int32_t e = 0; e < ne; ++e) S.xid[(size_t)l * ne + e] = (int32_t)xloops.size() - nl + l;
+    } else {
+      S.etot.assign((size_t)nl * ne, 0);
+      S.el.assign((size_t)nl * ne, LoopInfo{});
+      S.xid.assign((size_t)nl * ne, 0);
+      for (int32_t l = 0; l < nl; ++l)
+        for (int32_t e = 0; e < ne; ++e) {
+          const int64_t r = erow + (int64_t)l * ne + e;
+          const int64_t t0 = d.eng_trip_ptr[r], t1 = d.eng_trip_ptr[r + 1];
+          const int64_t want = l == 0 ? 1 : S.etot[(size_t)par[l] * ne + e];
+          if (t1 - t0 != want)
+            raise(SYNC_ERR_MALFORMED, where(p, "per-engine trip row length != parent's iterations on the engine, loop", l));
+          if (want > 0 && !d.eng_trips) raise(SYNC_ERR_ARG, "eng_trips must not be NULL");
+          S.xid[(size_t)l * ne + e] = (int32_t)xloops.size();
+          S.el[(size_t)l * ne + e] = add_space(l, d.eng_trips + t0, want);
+          S.etot[(size_t)l * ne + e] = S.el[(size_t)l * ne + e].total;
+        }
+      for (int32_t l = 0; l < nl; ++l) {            // engine 0's spaces stand for the loops
+        loop[l0 + l] = S.el[(size_t)l * ne];
+        S.total[l] = S.etot[(size_t)l * ne];
+      }
+      erow += (int64_t)nl * ne;
     }
+    // iterations of loop l on engine e, and that iteration space
+    auto tot = [&](int32_t l, int32_t e) -> int64_t { return div ? S.etot[(size_t)l * ne + e] : S.total[l]; };
+    auto space = [&](int32_t l, int32_t e) -> const LoopInfo& { return div ? S.el[(size_t)l * ne + e] : loop[l0 + l]; };
     // instructions
     for (int32_t x = 0; x < nx; ++x) {
       const int64_t gx = x0 + x;
@@ -269,19 +314,28 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     pi.le_base = (int32_t)op_ptr.size();
     __int128 agg = 0;
     for (int32_t x = 0; x < nx; ++x) {
-      const int64_t tot = S.total[d.instr_loop[x0 + x]];
-      agg += (__int128)tot * d.instr_latency[x0 + x];
+      const int64_t n = tot(d.instr_loop[x0 + x], d.instr_engine[x0 + x]);
+      agg += (__int128)n * d.instr_latency[x0 + x];
       inst_off[x0 + x] = n_inst;
-      n_inst += tot;
-      pi.n_inst += tot;
+      n_inst += n;
+      pi.n_inst += n;
     }
     pi.agg_lat = agg > (__int128)INT64_MAX ? INT64_MAX : (int64_t)agg;
     {
       std::vector<int64_t> per_engine(ne, 0);
-      for (int32_t x = 0; x < nx; ++x) per_engine[d.instr_engine[x0 + x]] += S.total[d.instr_loop[x0 + x]];
+      for (int32_t x = 0; x < nx; ++x)
+        per_engine[d.instr_engine[x0 + x]] += tot(d.instr_loop[x0 + x], d.instr_engine[x0 + x]);
       for (int64_t c : per_engine) if (c > kI32Max) ord_overflow = true;
     }
-    for (int32_t l = 1; l < nl; ++l) { pi.n_stmt += S.total[par[l]]; pi.n_iter += S.total[l]; }
+    for (int32_t e = 0; e < ne; ++e) {
+      int64_t st = 0, it = 0;
+      for (int32_t l = 1; l < nl; ++l) { st += tot(par[l], e); it += tot(l, e); }
+      pi.eng_stmt += st;
+      pi.eng_iter += it;
+      pi.n_stmt = std::max(pi.n_stmt, st);
+      pi.n_iter = std::max(pi.n_iter, it);
+    }
+    pi.divergent = div ? 1 : 0;
     S.x_ndeps.assign(nx, 0);
     S.x_dep_begin.assign(nx, d0);
     for (int m = 0; m < kModes; ++m) { S.x_own[m].assign(nx, -1); S.x_hstride[m].assign(nx, 0); S.x_koff[m].assign(nx, 0); }
@@ -319,61 +373,65 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         if (off != 1) raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested backward producer needs offset 1, dependency", k));
         kase = CASE_NEST_BWD;
       }
-      const int32_t N = S.nloop_eng[(size_t)Pl * ne + d.instr_engine[x0 + px]];
+      const int32_t ep = d.instr_engine[x0 + px], ec = d.instr_engine[x0 + cx];
+      const int32_t N = S.nloop_eng[(size_t)Pl * ne + ep];
       const int32_t K = S.rank[px];
-      if ((int64_t)N * S.total[Pl] > kI32Max)
+      if ((int64_t)N * tot(Pl, ep) > kI32Max)
         raise(SYNC_ERR_OVERFLOW, where(p, "per-loop semaphore value N*iterations exceeds INT32_MAX, dependency", k));
       DepInfo& D = dep[gd];
       std::memset(&D, 0, sizeof D);
-      D.total = (int32_t)S.total[Cl];
+      D.total = (int32_t)tot(Cl, ec);            // consumer instances, on its engine
       D.up = S.depth[Cl] - S.depth[Sl];
       D.clen = S.depth[Pl] - S.depth[Sl];
       D.kase = kase;
       D.k = off; D.N = N; D.K = K;
       D.path = (int64_t)path.size();
-      for (int32_t l = Cl; l != Sl; l = par[l]) path.push_back(loop[l0 + l].pidx_off);
-      for (int32_t l = Pl; l != Sl; l = par[l]) reads_rowptr[l0 + l] = 1;
+      // everything below is read on the consumer engine's iteration spaces
+      // (Eq. (1) with that engine's loop-entry counts)
+      for (int32_t l = Cl; l != Sl; l = par[l]) path.push_back(space(l, ec).pidx_off);
+      for (int32_t l = Pl; l != Sl; l = par[l]) reads_rowptr[S.xid[(size_t)l * ne + ec]] = 1;
       // derived arrays: trip starts of S, and the S-ancestors of the consumer loop
-      if (S.tstart_of[Sl] < 0) {
-        S.tstart_of[Sl] = n_derived;
+      const size_t skey = div ? (size_t)Sl * ne + ec : (size_t)Sl;
+      if (S.tstart_of[skey] < 0) {
+        S.tstart_of[skey] = n_derived;
         DeriveJob J{};
-        J.out = n_derived; J.a = loop[l0 + Sl].pidx_off; J.b = loop[l0 + Sl].rowptr_off;
-        J.n = (int32_t)S.total[Sl]; J.kind = DERIVE_TSTART;
+        J.out = n_derived; J.a = space(Sl, ec).pidx_off; J.b = space(Sl, ec).rowptr_off;
+        J.n = (int32_t)tot(Sl, ec); J.kind = DERIVE_TSTART;
         jobs.push_back(J);
-        n_derived += pad4(S.total[Sl]);
+        n_derived += pad4(tot(Sl, ec));
       }
-      D.tstart = S.tstart_of[Sl];
+      D.tstart = S.tstart_of[skey];
       if (ord_off[x0 + px] < 0) {
         ord_off[x0 + px] = n_ord;
-        n_ord += S.total[Pl];
+        n_ord += tot(Pl, ep);
       }
       D.ordp = ord_off[x0 + px];
       D.src = D.tstart;
       if (D.up > 0) {
-        const int64_t key = (int64_t)Cl * nl + Sl;
+        const int64_t key = ((int64_t)Cl * nl + Sl) * (div ? ne : 1) + (div ? ec : 0);
         auto f = S.anc_of.find(key);
         if (f == S.anc_of.end()) {
           DeriveJob J{};
           J.out = n_derived; J.a = D.path; J.b = 0;
-          J.n = (int32_t)S.total[Cl]; J.kind = DERIVE_ANC; J.up = D.up;
+          J.n = (int32_t)tot(Cl, ec); J.kind = DERIVE_ANC; J.up = D.up;
           jobs.push_back(J);
           f = S.anc_of.emplace(key, n_derived).first;
-          n_derived += pad4(S.total[Cl]);
+          n_derived += pad4(tot(Cl, ec));
         }
         D.src = f->second;
       }
-      path.push_back(loop[l0 + Sl].pidx_off);
-      path.push_back(loop[l0 + Sl].rowptr_off);
+      path.push_back(space(Sl, ec).pidx_off);
+      path.push_back(space(Sl, ec).rowptr_off);
       {
         const size_t at = path.size();
-        for (int32_t l = Pl; l != Sl; l = par[l]) path.push_back(loop[l0 + l].rowptr_off);
+        for (int32_t l = Pl; l != Sl; l = par[l]) path.push_back(space(l, ec).rowptr_off);
         std::reverse(path.begin() + at, path.end());
       }
       D.seg_off = n_pairs_padded;
       seg[gd] = n_pairs_padded;
-      n_pairs += S.total[Cl];
-      n_pairs_padded += pad4(S.total[Cl]);
-      pi.n_pairs += S.total[Cl];
+      n_pairs += tot(Cl, ec);
+      n_pairs_padded += pad4(tot(Cl, ec));
+      pi.n_pairs += tot(Cl, ec);
       dep_N[gd] = N;
       dep_K[gd] = K;
     }
@@ -383,7 +441,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     // iteration); mode 2 = one per engine (one increment per instance of the
     // engine, numbered by the instance's ordinal)
     std::vector<int64_t> inst_eng(ne, 0);
-    for (int32_t x = 0; x < nx; ++x) inst_eng[d.instr_engine[x0 + x]] += S.total[d.instr_loop[x0 + x]];
+    for (int32_t x = 0; x < nx; ++x)
+      inst_eng[d.instr_engine[x0 + x]] += tot(d.instr_loop[x0 + x], d.instr_engine[x0 + x]);
     auto sem_key = [&](int m, int32_t x) {
       const int32_t e = d.instr_engine[x0 + x];
       return m == 0 ? x : m == 1 ? d.instr_loop[x0 + x] * ne + e : e;
@@ -393,7 +452,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     for (int32_t k = 0; k < nd; ++k) {
       const int64_t gd = d0 + k;
       S.x_levels[d.dep_cons[gd]] += levels(d.dep_prod[gd]);
-      pi.pair_levels += (int64_t)levels(d.dep_prod[gd]) * S.total[d.instr_loop[x0 + d.dep_cons[gd]]];
+      pi.pair_levels += (int64_t)levels(d.dep_prod[gd]) *
+                        tot(d.instr_loop[x0 + d.dep_cons[gd]], d.instr_engine[x0 + d.dep_cons[gd]]);
     }
     std::vector<int32_t> sem_of(std::max(nx, nl * ne), -1);
     for (int m = 0; m < kModes; ++m) {
@@ -407,7 +467,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         if (sem_of[key] < 0) {
           sem_of[key] = (int32_t)sem_hist.size();
           sem_hist.push_back(hist_len[m]);
-          hist_len[m] += m == 0 ? S.total[Pl] : m == 1 ? dep_N[gd] * S.total[Pl] : inst_eng[d.instr_engine[x0 + px]];
+          const int32_t ep = d.instr_engine[x0 + px];
+          hist_len[m] += m == 0 ? tot(Pl, ep) : m == 1 ? dep_N[gd] * tot(Pl, ep) : inst_eng[ep];
         }
       }
       pi.nsem[m] = (int32_t)sem_hist.size();
@@ -445,7 +506,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
           const int32_t it = S.body[i];
           if (it < 0) {
             const int32_t m = -it - 1;
-            const int64_t rp = loop[l0 + m].rowptr_off;
+            const int64_t rp = space(m, e).rowptr_off;
             ops.push_back(make_int4(OP_LOOP, pi.le_base + m * ne, (int32_t)(uint32_t)(rp & 0xffffffffu),
                                     (int32_t)(rp >> 32)));
             for (int m = 0; m < kModes; ++m) opsem[m].push_back(make_int4(-1, 0, 0, 0));
@@ -520,14 +581,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   plan_ptr.push_back((int32_t)plan.size());
   seg[ND] = n_pairs_padded;
 
-  // trip prefix sums (rowptr) per loop: [0, t0, t0+t1, ...]
-  rowptr_host.resize(rowptr_len);
-  for (int64_t l = 0; l < NL; ++l) {
-    int32_t* rp = rowptr_host.data() + loop[l].rowptr_off;
-    const int64_t t0 = d.trip_ptr[l];
-    rp[0] = 0;
-    for (int32_t j = 0; j < loop[l].n_parent; ++j) rp[j + 1] = rp[j] + d.trips[t0 + j];
-  }
   // tile tables
   const int64_t n_tiles = (n_pairs_padded + kTilePairs - 1) / kTilePairs;
   std::vector<int32_t> tile_first(n_tiles + 1, ND > 0 ? (int32_t)(ND - 1) : 0);
@@ -549,13 +602,14 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       tile_job[t] = (int32_t)ji;
     }
   }
+  const int64_t NXL = (int64_t)xloops.size();
   const int64_t n_itiles = (n_iters + kTilePairs - 1) / kTilePairs;
-  std::vector<int32_t> tile_loop(n_itiles + 1, NL > 0 ? (int32_t)(NL - 1) : 0);
+  std::vector<int32_t> tile_loop(n_itiles + 1, NXL > 0 ? (int32_t)(NXL - 1) : 0);
   {
     int64_t li = 0;
     for (int64_t t = 0; t < n_itiles; ++t) {
       const int64_t q = t * kTilePairs;
-      while (li + 1 < NL && loop[li + 1].pidx_off <= q) ++li;
+      while (li + 1 < NXL && xloops[li + 1].pidx_off <= q) ++li;
       tile_loop[t] = (int32_t)li;
     }
   }
@@ -579,8 +633,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     int64_t sb = (int64_t)ND * (int64_t)sizeof(DepInfo) + 8 * (ND + 1) + 8 * (int64_t)path.size() +
                  4 * (int64_t)tile_first.size();
     sb += 4 * n_derived;
-    for (int64_t l = 0; l < NL; ++l)
-      if (reads_rowptr[l]) sb += 4 * ((int64_t)loop[l].n_parent + 1);
+    for (size_t l = 0; l < xloops.size(); ++l)
+      if (reads_rowptr[l]) sb += 4 * ((int64_t)xloops[l].n_parent + 1);
     h.sz.struct_bytes = sb;
   }
   h.seg_host = seg;
@@ -640,7 +694,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     h.lsem = h.upload(both, stream, "sweep lane semaphores");
   }
   h.n_lanes = (int64_t)lrec.size();
-  cuda_check(launch_expand(h.loop, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
+  LoopInfo* d_xloops = h.upload(xloops, stream, "iteration spaces");
+  h.divergent = div;
+  cuda_check(launch_expand(d_xloops, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
   cuda_check(launch_derive(d_jobs, d_tile_job, h.rowptr, h.pidx, h.path, h.derived, n_derived, h.num_sms, stream),
              "derive");
   cuda_check(cudaStreamSynchronize(stream), "load");
@@ -688,6 +744,17 @@ static ThrArgs thr_args(const sync_programs* h, sync_thr_mode mode) {
 }
 
 // thresholds and check: all three encodings
+// Per-engine trip counts: per-engine wait values are not defined (a position
+// in the producer engine's stream that the consumer's loop state no longer
+// determines), and the barrier scheme has no common barrier sequence.
+static void check_divergent(const sync_programs* h, sync_thr_mode mode, bool sim, sync_sim_variant variant) {
+  if (!h->divergent) return;
+  if (mode == SYNC_THR_PERENGINE)
+    raise(SYNC_ERR_ARG, "per-engine trip counts: per-engine thresholds are not defined");
+  if (sim && variant != SYNC_SIM_BARRIER_FREE)
+    raise(SYNC_ERR_ARG, "per-engine trip counts: only the barrier-free schedule is defined");
+}
+
 static void check_thr_mode(sync_thr_mode mode) {
   if (mode != SYNC_THR_COUNT && mode != SYNC_THR_PERLOOP && mode != SYNC_THR_PERENGINE)
     raise(SYNC_ERR_ARG, "unknown threshold mode");
@@ -715,6 +782,7 @@ sync_status sync_eval_thresholds(const sync_programs* h, sync_thr_mode mode, int
   try {
     if (!h) raise(SYNC_ERR_ARG, "handle must not be NULL");
     check_thr_mode(mode);
+    check_divergent(h, mode, false, SYNC_SIM_BARRIER_FREE);
     if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
     if (reinterpret_cast<uintptr_t>(d_thr) % 16) raise(SYNC_ERR_ARG, "d_thr must be 16-byte aligned");
     cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
@@ -732,6 +800,7 @@ sync_status sync_check_minimal(const sync_programs* h, sync_thr_mode mode, const
   try {
     if (!h || !d_counts || !d_first_bad) raise(SYNC_ERR_ARG, "handle and outputs must not be NULL");
     check_thr_mode(mode);
+    check_divergent(h, mode, false, SYNC_SIM_BARRIER_FREE);
     if (h->sz.n_pairs_padded > 0 && !d_thr) raise(SYNC_ERR_ARG, "d_thr must not be NULL");
     if (reinterpret_cast<uintptr_t>(d_thr) % 16) raise(SYNC_ERR_ARG, "d_thr must be 16-byte aligned");
     cuda_check(cudaSetDevice(h->device), "cudaSetDevice");
@@ -761,6 +830,7 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
     raise(SYNC_ERR_ARG, "unknown variant");
   if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
     raise(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
+  check_divergent(h, mode, true, variant);
   if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
     raise(SYNC_ERR_ARG, "per-program outputs must not be NULL");
   if ((d_issue == nullptr) != (d_retire == nullptr)) raise(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");

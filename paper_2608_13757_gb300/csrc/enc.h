@@ -60,8 +60,11 @@ struct alignas(16) ProgInfo {
   int64_t agg_lat;    // sum over instructions of instances * latency (saturated)
   int64_t n_inst;     // datapath instances
   int64_t n_pairs;    // (dependency, consumer instance) pairs
-  int64_t n_stmt;     // loop statements reached (sum over non-top loops of total(parent))
-  int64_t n_iter;     // loop iterations (sum over non-top loops of total)
+  int64_t n_stmt;     // loop statements one engine reaches (sum over non-top loops of
+                      // total(parent); per-engine trips: the largest over the engines)
+  int64_t n_iter;     // loop iterations of one engine (likewise)
+  int64_t eng_stmt;   // loop statements summed over the engines
+  int64_t eng_iter;   // loop iterations summed over the engines
   int64_t pair_levels;  // sum over pairs of the per-engine wait's extra levels
   int32_t ne;
   int32_t le_base;    // row of (top-level loop, engine 0); row of (program-local
@@ -69,7 +72,7 @@ struct alignas(16) ProgInfo {
   int32_t nsem[kModes];    // waited semaphores, per threshold mode
   int32_t semhb_off[kModes];  // first entry of the program's history bases, per mode
   int32_t loop_base;  // global id of the program's top-level loop
-  int32_t pad_;
+  int32_t divergent;  // 1: engines run their own trip counts (per-engine kernel only)
 };
 
 // Program-order sweep tables.  Per loop, a plan: its body cut at child loops

@@ -40,6 +40,7 @@ struct sync_programs {
   mutable std::mutex ord_mu;
   mutable int32_t* ord = nullptr;
   mutable bool ord_ready = false;
+  bool divergent = false;           // some program runs per-engine trip counts
   int64_t n_ord = 0;
   bool ord_overflow = false;        // an engine of a program has > INT32_MAX instances
   std::vector<int64_t> ord_off_host;  // per instruction: pool offset or -1

@@ -104,9 +104,9 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
     if (MODE == SYNC_THR_PERENGINE)
       b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
-    const u64 ctl = sat_add(sat_mul((u64)pi.n_stmt, (u64)q.c_regop),
-                            sat_mul((u64)pi.n_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop));
-    b = sat_add(b, sat_mul((u64)pi.ne, ctl));
+    // control operations of every engine (their own trips)
+    b = sat_add(b, sat_add(sat_mul((u64)pi.eng_stmt, (u64)q.c_regop),
+                           sat_mul((u64)pi.eng_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop)));
   }
   return b;
 }

@@ -2,7 +2,8 @@
 //
 // Under a common loop tree every engine meets the same loop statements and
 // iteration boundaries, so one walker per program can visit the tree once for
-// all engines.  The body of each loop is cut at its child loops into
+// all engines (programs whose engines run their own trip counts go straight
+// to the per-engine kernel).  The body of each loop is cut at its child loops into
 // straight-line segments; a segment is taken as one chunk of up to 32 datapath
 // records (more chunks if longer), or -- barrier-free, for a short innermost
 // body -- as several consecutive iterations at once.  The chunk's lanes are
@@ -83,9 +84,9 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
     if (MODE == SYNC_THR_PERENGINE)
       b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
-    const u64 ctl = sat_add(sat_mul((u64)pi.n_stmt, (u64)q.c_regop),
-                            sat_mul((u64)pi.n_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop));
-    b = sat_add(b, sat_mul((u64)pi.ne, ctl));
+    // control operations of every engine (their own trips)
+    b = sat_add(b, sat_add(sat_mul((u64)pi.eng_stmt, (u64)q.c_regop),
+                           sat_mul((u64)pi.eng_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop)));
   }
   return b;
 }
@@ -686,6 +687,13 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     if (slot >= a.n_programs) break;
     const int p = __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
+    if (pi.divergent) {               // engines on their own trips: no common walk
+      if (lane == 0) {
+        a.status[p] = SIM_FALLBACK;
+        a.fallback[1 + atomicAdd(a.fallback, 1)] = p;
+      }
+      continue;
+    }
     if (time_bound<MODE, BB>(pi, a.prm, cwait) > 2147483647ull) {
       if (lane == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
       continue;

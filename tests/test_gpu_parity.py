@@ -59,7 +59,7 @@ def compare_all(sg, batch, params=None, timeline=False, modes=MODES):
         assert np.array_equal(got, want), f"thresholds differ (mode {mode})"
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
-        for v in variants_for(mode):
+        for v in ((oracle.BARRIER_FREE,) if batch.divergent else variants_for(mode)):
             ref = oracle.simulate(batch, want, mode, v, prm, timeline=timeline)
             res = sg.sync_simulate(h, mode, thr, sim_params(prm), v, timeline=timeline)
             fused, fcounts, ffirst = sg.sync_simulate_fused(h, mode, sim_params(prm), v, timeline=timeline,
@@ -84,6 +84,62 @@ def _instances_per_program(batch):
     for p in range(batch.n_programs):
         out.append(oracle.sizes(batch.program(p))[1])
     return np.array(out, dtype=np.int64)
+
+
+# ------------------------------------------- per-engine trip counts (NEXT-2)
+
+@pytest.mark.parametrize("seed", range(4))
+def test_divergent_random_trees(sg, seed):
+    """Engines on their own trips (Sec. 7.5): thresholds on the consumer
+    engine's loop state, the checker, and the barrier-free simulation (array
+    and fused) with its deadlocks, equal to the oracle's."""
+    base = workloads.random_trees(6000 + seed, 150, workloads.tree_params(
+        engines_hi=5, loops_hi=5, body_hi=6, trip_hi=4, max_depth=4))
+    batch = workloads.diverge(base, 7000 + seed, permille=250)
+    compare_all(sg, batch, timeline=True, modes=MODES,
+                params=oracle.sim_params(ii=2, c_branch=3, c_regop=2))
+    st = oracle.simulate(batch, oracle.thresholds(batch, COUNT), COUNT).status
+    assert (st == 7).any() and (st == 0).any()          # both outcomes are exercised
+
+
+@pytest.mark.parametrize("name,n", [("depth2", 48), ("chain", 300), ("attention", 2)])
+def test_divergent_configs(sg, name, n):
+    batch = workloads.diverge(workloads.generate(name, n_programs=n), 11, permille=30)
+    compare_all(sg, batch, timeline=name == "depth2", modes=MODES)
+
+
+def test_divergent_mixed_with_shared_and_aligned(sg):
+    """A batch mixing aligned per-engine rows (identical to shared trips) and
+    divergent ones: the aligned programs give the shared batch's results."""
+    shared = workloads.random_trees(6100, 60)
+    aligned = workloads.diverge(shared, 1, permille=0)
+    mixed = workloads.concat([aligned, workloads.diverge(shared, 2, permille=400)])
+    compare_all(sg, mixed, timeline=True, modes=MODES)
+    h = sg.sync_load_programs(aligned)
+    h2 = sg.sync_load_programs(shared)
+    for mode in MODES:
+        t1, t2 = sg.sync_eval_thresholds(h, mode), sg.sync_eval_thresholds(h2, mode)
+        import torch
+        assert torch.equal(t1, t2)
+        r1 = sg.sync_simulate(h, mode, t1)
+        r2 = sg.sync_simulate(h2, mode, t2)
+        for f in ("status", "makespan", "checksum"):
+            assert torch.equal(getattr(r1, f), getattr(r2, f)), (mode, f)
+
+
+def test_divergent_rejects_barrier_and_per_engine(sg):
+    batch = workloads.diverge(workloads.random_trees(6200, 10), 3, permille=300)
+    h = sg.sync_load_programs(batch)
+    with pytest.raises(sg.SyncError) as err:
+        sg.sync_eval_thresholds(h, sg.THR_PERENGINE)
+    assert err.value.status == sg.ERR_ARG
+    thr = sg.sync_eval_thresholds(h, sg.THR_PERLOOP)
+    for v in (sg.SIM_BARRIER, sg.SIM_UNROLLED):
+        with pytest.raises(sg.SyncError) as err:
+            sg.sync_simulate(h, sg.THR_PERLOOP, thr, variant=v)
+        assert err.value.status == sg.ERR_ARG
+    with pytest.raises(sg.SyncError):
+        sg.sync_simulate_fused(h, sg.THR_PERLOOP, variant=sg.SIM_BARRIER)
 
 
 # ------------------------------------------------------------------ configs
