@@ -46,7 +46,7 @@ def _compile(src: str) -> str:
         cmd = [NVCC] + ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                                "-Xptxas", "-warn-spills", "-c", src, "-o", obj] + inc
     else:
-        cmd = ["g++", "-O2", "-std=c++17", "-fPIC", "-Wall", "-Wextra", "-c", src, "-o", obj,
+        cmd = ["g++", "-O2", "-std=c++17", "-fPIC", "-pthread", "-Wall", "-Wextra", "-c", src, "-o", obj,
                "-I", os.path.join(CUDA_HOME, "include")] + inc
     subprocess.check_call(cmd)
     return obj
@@ -63,7 +63,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
         objs = list(ex.map(_compile, _sources()))
     tmp = LIB + f".tmp{os.getpid()}"
     subprocess.check_call([NVCC] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs +
-                          ["-Xlinker", "-rpath=" + os.path.join(CUDA_HOME, "lib64")])
+                          ["-Xlinker", "-rpath=" + os.path.join(CUDA_HOME, "lib64"), "-Xcompiler", "-pthread"])
     os.replace(tmp, LIB)
     if verbose:
         print("built", LIB)

@@ -2,12 +2,16 @@
 // device encoding) and the launch wrappers.  Declarations and contracts are
 // in include/sync.h.
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
+#include <exception>
 #include <memory>
 #include <mutex>
 #include <new>
 #include <string>
+#include <thread>
 #include <unordered_map>
+#include <utility>
 #include <vector>
 
 #include "enc.h"
@@ -70,6 +74,19 @@ constexpr int64_t kI32Max = 2147483647;
 
 int64_t pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
+// Threads of the loader's per-program pass: one per hardware thread (at most
+// 32) while each gets at least 256 programs.  SYNCGB_LOAD_THREADS=n sets the
+// count (tests use it to run the block join on small batches).
+int load_threads(int32_t P) {
+  int n = 0;
+  if (const char* v = std::getenv("SYNCGB_LOAD_THREADS")) n = std::atoi(v);
+  if (n <= 0) {
+    n = std::min(32, (int)std::max(1u, std::thread::hardware_concurrency()));
+    n = (int)std::min<int64_t>(n, std::max<int64_t>(1, P / 256));
+  }
+  return std::max(1, std::min(n, std::max(1, (int)P)));
+}
+
 }  // namespace
 
 namespace {
@@ -96,6 +113,48 @@ struct ProgScratch {
   std::vector<int32_t> xid;                       // per-engine trips: expansion-table entry per (loop, engine)
   std::vector<int64_t> tstart_of;                 // derived trip-start array per loop (and engine), -1 if none
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
+};
+
+// Host arrays that are filled right after allocation: default-initialised,
+// so allocating one does not write it first.
+template <class T>
+struct NoInit : std::allocator<T> {
+  template <class U>
+  struct rebind { using other = NoInit<U>; };
+  NoInit() = default;
+  template <class U>
+  NoInit(const NoInit<U>&) {}
+  template <class U>
+  void construct(U* p) { ::new (static_cast<void*>(p)) U; }
+  template <class U, class... A>
+  void construct(U* p, A&&... a) { ::new (static_cast<void*>(p)) U(std::forward<A>(a)...); }
+};
+template <class T>
+using HostVec = std::vector<T, NoInit<T>>;
+
+// What the per-program pass appends, for one block of consecutive programs.
+// Offsets recorded in it (into the rowptr, parent-index, pair, derived,
+// path, op, plan, chunk, lane, semaphore-base, history and ordinal spaces)
+// are relative to the block's start; joining the blocks shifts them.
+struct Part {
+  std::vector<int32_t> rowptr_host;
+  std::vector<int64_t> path;
+  std::vector<uint8_t> path_kind;          // per path entry: 0 parent-index offset, 1 rowptr offset
+  std::vector<int32_t> op_ptr, opstop;
+  std::vector<int2> rowinfo;
+  std::vector<int4> ops, opsem[kModes];
+  std::vector<int64_t> semhb;
+  std::vector<uint8_t> semhb_mode;         // per semaphore base: its mode (history space)
+  std::vector<int32_t> plan_ptr;
+  std::vector<int4> plan, chunks, lrec, lmeta, lsem[kModes];
+  std::vector<LoopInfo> xloops;
+  std::vector<uint8_t> reads_rowptr;
+  std::vector<DeriveJob> jobs;
+  int64_t n_ord = 0, n_derived = 0, n_pairs = 0, n_pairs_padded = 0, n_inst = 0, n_iters = 0, rowptr_len = 0;
+  int64_t hist_len[kModes] = {0, 0, 0};
+  bool ord_overflow = false;
+  int32_t nsem_max[kModes] = {0, 0, 0}, ne_max = 0, depth_max = 0;
+  std::exception_ptr error;
 };
 
 // Appends one sweep chunk: lanes `recs` (program-local instructions, already
@@ -154,35 +213,52 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   }
 
   // ------------------------------------ per-program validation and tables
+  // Indexed by global loop / dependency / program / instruction id: written
+  // by the block that owns the id (offsets block-relative until the join).
   std::vector<LoopInfo> loop(NL);
-  std::vector<int32_t> rowptr_host;
   std::vector<DepInfo> dep(ND);
-  std::vector<int64_t> path;
   std::vector<ProgInfo> prog(P);
-  std::vector<int32_t> op_ptr, opstop;
-  std::vector<int2> rowinfo;
-  std::vector<int4> ops, opsem[kModes];
-  std::vector<int64_t> inst_off(NX), dseg(ND), semhb;
+  std::vector<int64_t> inst_off(NX), dseg(ND);
   std::vector<int32_t> ddep(ND);
   std::vector<int32_t> dsem[kModes] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
-  std::vector<int32_t> plan_ptr;
-  std::vector<int4> plan, chunks, lrec, lmeta, lsem[kModes];
   std::vector<int64_t> seg(ND + 1, 0);
   std::vector<int64_t> ord_off(NX, -1);   // per instruction: ordinal pool offset (waited producers)
-  int64_t n_ord = 0;
-  bool ord_overflow = false;
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
-  std::vector<int64_t> hist_len(kModes, 0);
-  std::vector<LoopInfo> xloops;             // every (loop[, engine]) iteration space, in pidx order
-  std::vector<uint8_t> reads_rowptr;        // per xloops entry: read by a nested producer's count
-  int64_t erow = 0;                         // per-engine trips: first row of the program
-  std::vector<DeriveJob> jobs;
-  int64_t n_derived = 0;
-  int64_t n_pairs = 0, n_pairs_padded = 0, n_inst = 0, n_iters = 0, rowptr_len = 0;
+
+  // Programs [p_begin, p_end) into `part`; erow0: their first per-engine row.
+  auto run_block = [&d, div, &loop, &dep, &prog, &inst_off, &dseg, &ddep, &dsem, &seg, &ord_off, &dep_N,
+                    &dep_K](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
+  auto& rowptr_host = part.rowptr_host;
+  auto& path = part.path;
+  auto& op_ptr = part.op_ptr;
+  auto& opstop = part.opstop;
+  auto& rowinfo = part.rowinfo;
+  auto& ops = part.ops;
+  auto& opsem = part.opsem;
+  auto& semhb = part.semhb;
+  auto& plan_ptr = part.plan_ptr;
+  auto& plan = part.plan;
+  auto& chunks = part.chunks;
+  auto& lrec = part.lrec;
+  auto& lmeta = part.lmeta;
+  auto& lsem = part.lsem;
+  auto& xloops = part.xloops;
+  auto& reads_rowptr = part.reads_rowptr;
+  auto& jobs = part.jobs;
+  auto& n_ord = part.n_ord;
+  auto& n_derived = part.n_derived;
+  auto& n_pairs = part.n_pairs;
+  auto& n_pairs_padded = part.n_pairs_padded;
+  auto& n_inst = part.n_inst;
+  auto& n_iters = part.n_iters;
+  auto& rowptr_len = part.rowptr_len;
+  auto& hist_len = part.hist_len;
+  auto push_path = [&](int64_t v, uint8_t kind) { path.push_back(v); part.path_kind.push_back(kind); };
+  int64_t erow = erow0;                     // per-engine trips: first row of the program
   ProgScratch S;
 
-  for (int32_t p = 0; p < P; ++p) {
+  for (int32_t p = p_begin; p < p_end; ++p) {
     const int32_t l0 = d.prog_loop_ptr[p], x0 = d.prog_instr_ptr[p], d0 = d.prog_dep_ptr[p];
     const int32_t nl = d.prog_loop_ptr[p + 1] - l0, nx = d.prog_instr_ptr[p + 1] - x0,
                   nd = d.prog_dep_ptr[p + 1] - d0;
@@ -325,7 +401,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       std::vector<int64_t> per_engine(ne, 0);
       for (int32_t x = 0; x < nx; ++x)
         per_engine[d.instr_engine[x0 + x]] += tot(d.instr_loop[x0 + x], d.instr_engine[x0 + x]);
-      for (int64_t c : per_engine) if (c > kI32Max) ord_overflow = true;
+      for (int64_t c : per_engine) if (c > kI32Max) part.ord_overflow = true;
     }
     for (int32_t e = 0; e < ne; ++e) {
       int64_t st = 0, it = 0;
@@ -388,7 +464,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       D.path = (int64_t)path.size();
       // everything below is read on the consumer engine's iteration spaces
       // (Eq. (1) with that engine's loop-entry counts)
-      for (int32_t l = Cl; l != Sl; l = par[l]) path.push_back(space(l, ec).pidx_off);
+      for (int32_t l = Cl; l != Sl; l = par[l]) push_path(space(l, ec).pidx_off, 0);
       for (int32_t l = Pl; l != Sl; l = par[l]) reads_rowptr[S.xid[(size_t)l * ne + ec]] = 1;
       // derived arrays: trip starts of S, and the S-ancestors of the consumer loop
       const size_t skey = div ? (size_t)Sl * ne + ec : (size_t)Sl;
@@ -420,11 +496,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         }
         D.src = f->second;
       }
-      path.push_back(space(Sl, ec).pidx_off);
-      path.push_back(space(Sl, ec).rowptr_off);
+      push_path(space(Sl, ec).pidx_off, 0);
+      push_path(space(Sl, ec).rowptr_off, 1);
       {
         const size_t at = path.size();
-        for (int32_t l = Pl; l != Sl; l = par[l]) path.push_back(space(l, ec).rowptr_off);
+        for (int32_t l = Pl; l != Sl; l = par[l]) push_path(space(l, ec).rowptr_off, 1);
         std::reverse(path.begin() + at, path.end());
       }
       D.seg_off = n_pairs_padded;
@@ -474,6 +550,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       pi.nsem[m] = (int32_t)sem_hist.size();
       pi.semhb_off[m] = (int32_t)semhb.size();
       semhb.insert(semhb.end(), sem_hist.begin(), sem_hist.end());
+      part.semhb_mode.insert(part.semhb_mode.end(), sem_hist.size(), (uint8_t)m);
       for (int32_t x = 0; x < nx; ++x) {
         const int32_t l = d.instr_loop[x0 + x];
         const int32_t s = sem_of[sem_key(m, x)];
@@ -572,10 +649,189 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         add_chunk(d, x0, S, recs, copies, k, chunks, lrec, lmeta, lsem);
       }
     }
-    for (int m = 0; m < kModes; ++m) h.nsem_max[m] = std::max(h.nsem_max[m], pi.nsem[m]);
-    h.ne_max = std::max(h.ne_max, ne);
-    h.depth_max = std::max(h.depth_max, depth_max);
+    for (int m = 0; m < kModes; ++m) part.nsem_max[m] = std::max(part.nsem_max[m], pi.nsem[m]);
+    part.ne_max = std::max(part.ne_max, ne);
+    part.depth_max = std::max(part.depth_max, depth_max);
     if ((int64_t)ops.size() > kI32Max) raise(SYNC_ERR_OVERFLOW, "op records exceed INT32_MAX entries");
+  }
+  };
+
+  // Blocks of consecutive programs of about equal work, one per thread.
+  std::vector<int64_t> work(P), erow_of(P + 1, 0);
+  for (int32_t p = 0; p < P; ++p) {
+    const int64_t nl = d.prog_loop_ptr[p + 1] - d.prog_loop_ptr[p];
+    const int64_t ne = std::max<int64_t>(1, std::min<int64_t>(32, d.prog_n_engines[p]));
+    const int64_t trips = div || nl == 0 ? nl * ne : d.trip_ptr[d.prog_loop_ptr[p + 1]] - d.trip_ptr[d.prog_loop_ptr[p]];
+    work[p] = 16 + (nl + d.prog_instr_ptr[p + 1] - d.prog_instr_ptr[p]) * ne + (d.prog_dep_ptr[p + 1] - d.prog_dep_ptr[p]) +
+              std::max<int64_t>(trips, 0);
+    erow_of[p + 1] = erow_of[p] + nl * d.prog_n_engines[p];
+  }
+  const int n_threads = load_threads(P);
+  std::vector<int32_t> cut(n_threads + 1, P);
+  {
+    int64_t total = 0;
+    for (int64_t w : work) total += w;
+    int64_t acc = 0;
+    int b = 1;
+    cut[0] = 0;
+    for (int32_t p = 0; p < P && b < n_threads; ++p) {
+      acc += work[p];
+      while (b < n_threads && acc * n_threads >= total * b) cut[b++] = p + 1;
+    }
+  }
+  std::vector<Part> parts(n_threads);
+  {
+    std::vector<std::thread> pool;
+    for (int t = 0; t < n_threads; ++t) {
+      auto job = [&, t] {
+        try {
+          run_block(parts[t], cut[t], cut[t + 1], erow_of[cut[t]]);
+        } catch (...) {
+          parts[t].error = std::current_exception();
+        }
+      };
+      if (t + 1 < n_threads) pool.emplace_back(job); else job();
+    }
+    for (auto& th : pool) th.join();
+    for (auto& pt : parts)
+      if (pt.error) std::rethrow_exception(pt.error);
+  }
+
+  // ------------------------------------------------- join the blocks
+  // Each block's bases in every space are the sizes of the blocks before it;
+  // every block then copies itself into place, shifting the offsets it holds.
+  struct Base {
+    int64_t rowptr, iters, pairs, derived, path, ord, inst, hist[kModes];
+    int64_t rowptr_host, ops, rows, plan, chunks, lanes, semhb, xloops, jobs, opstop, pairs_raw;
+  };
+  std::vector<Base> base(n_threads + 1);
+  std::memset(base.data(), 0, sizeof(Base) * base.size());
+  for (int t = 0; t < n_threads; ++t) {
+    const Part& pt = parts[t];
+    Base nb = base[t];
+    nb.rowptr += pt.rowptr_len; nb.iters += pt.n_iters; nb.pairs += pt.n_pairs_padded;
+    nb.derived += pt.n_derived; nb.path += (int64_t)pt.path.size(); nb.ord += pt.n_ord; nb.inst += pt.n_inst;
+    for (int m = 0; m < kModes; ++m) nb.hist[m] += pt.hist_len[m];
+    nb.rowptr_host += (int64_t)pt.rowptr_host.size(); nb.ops += (int64_t)pt.ops.size();
+    nb.rows += (int64_t)pt.op_ptr.size(); nb.plan += (int64_t)pt.plan.size(); nb.chunks += (int64_t)pt.chunks.size();
+    nb.lanes += (int64_t)pt.lrec.size(); nb.semhb += (int64_t)pt.semhb.size(); nb.xloops += (int64_t)pt.xloops.size();
+    nb.jobs += (int64_t)pt.jobs.size(); nb.opstop += (int64_t)pt.opstop.size(); nb.pairs_raw += pt.n_pairs;
+    base[t + 1] = nb;
+    for (int m = 0; m < kModes; ++m) h.nsem_max[m] = std::max(h.nsem_max[m], pt.nsem_max[m]);
+    h.ne_max = std::max(h.ne_max, pt.ne_max);
+    h.depth_max = std::max(h.depth_max, pt.depth_max);
+  }
+  const Base& all = base[n_threads];
+  if (all.ops > kI32Max) raise(SYNC_ERR_OVERFLOW, "op records exceed INT32_MAX entries");
+  HostVec<int32_t> rowptr_host(all.rowptr_host);
+  HostVec<int64_t> path(all.path);
+  HostVec<int32_t> op_ptr(all.rows), opstop(all.opstop);
+  HostVec<int2> rowinfo(all.rows);
+  HostVec<int4> ops(all.ops), opsem(kModes * all.ops);    // opsem: mode-major
+  HostVec<int64_t> semhb(all.semhb);
+  HostVec<int32_t> plan_ptr(NL);             // one entry per loop; the blocks own consecutive loops
+  HostVec<int4> plan(all.plan), chunks(all.chunks), lrec(all.lanes), lmeta(all.lanes);
+  HostVec<int4> lsem(kModes * all.lanes);                  // mode-major
+  HostVec<LoopInfo> xloops(all.xloops);
+  HostVec<uint8_t> reads_rowptr(all.xloops);
+  HostVec<DeriveJob> jobs(all.jobs);
+  const int64_t n_ord = all.ord, n_derived = all.derived, n_pairs = all.pairs_raw, n_pairs_padded = all.pairs;
+  const int64_t n_inst = all.inst, n_iters = all.iters;
+  std::vector<int64_t> hist_len(all.hist, all.hist + kModes);
+  bool ord_overflow = false;
+  for (const Part& pt : parts) ord_overflow = ord_overflow || pt.ord_overflow;
+  auto join_block = [&](int t) {
+    Part& pt = parts[t];
+    const Base& B = base[t];
+    const int32_t b_ops = (int32_t)B.ops, b_rows = (int32_t)B.rows, b_plan = (int32_t)B.plan;
+    const int32_t b_chunks = (int32_t)B.chunks, b_lanes = (int32_t)B.lanes, b_semhb = (int32_t)B.semhb;
+    // indexed by id: the block's programs, loops, instructions, dependencies
+    for (int32_t p = cut[t]; p < cut[t + 1]; ++p) {
+      ProgInfo& pi = prog[p];
+      pi.le_base += b_rows;
+      for (int m = 0; m < kModes; ++m) pi.semhb_off[m] += b_semhb;
+      for (int32_t l = d.prog_loop_ptr[p]; l < d.prog_loop_ptr[p + 1]; ++l) {
+        loop[l].rowptr_off += B.rowptr;
+        loop[l].pidx_off += B.iters;
+      }
+      for (int32_t x = d.prog_instr_ptr[p]; x < d.prog_instr_ptr[p + 1]; ++x) {
+        inst_off[x] += B.inst;
+        if (ord_off[x] >= 0) ord_off[x] += B.ord;
+      }
+      for (int32_t k = d.prog_dep_ptr[p]; k < d.prog_dep_ptr[p + 1]; ++k) {
+        DepInfo& D = dep[k];
+        D.seg_off += B.pairs;
+        D.src += B.derived;
+        D.tstart += B.derived;
+        D.path += B.path;
+        D.ordp += B.ord;
+        seg[k] += B.pairs;
+        dseg[k] += B.pairs;
+      }
+    }
+    // appended: into place, shifting the offsets they hold
+    std::copy(pt.rowptr_host.begin(), pt.rowptr_host.end(), rowptr_host.begin() + B.rowptr_host);
+    for (size_t i = 0; i < pt.path.size(); ++i)
+      path[B.path + i] = pt.path[i] + (pt.path_kind[i] ? B.rowptr : B.iters);
+    for (size_t i = 0; i < pt.op_ptr.size(); ++i) op_ptr[B.rows + i] = pt.op_ptr[i] + b_ops;
+    for (size_t i = 0; i < pt.rowinfo.size(); ++i)
+      rowinfo[B.rows + i] = make_int2(pt.rowinfo[i].x + b_ops, pt.rowinfo[i].y);
+    for (size_t i = 0; i < pt.opstop.size(); ++i) opstop[B.opstop + i] = pt.opstop[i] + b_ops;
+    for (size_t i = 0; i < pt.ops.size(); ++i) {
+      int4 v = pt.ops[i];
+      if (v.x == OP_LOOP) {
+        const int64_t rp = (int64_t)(((uint64_t)(uint32_t)v.w << 32) | (uint32_t)v.z) + B.rowptr;
+        v = make_int4(OP_LOOP, v.y + b_rows, (int32_t)(uint32_t)(rp & 0xffffffffu), (int32_t)(rp >> 32));
+      }
+      ops[B.ops + i] = v;
+    }
+    for (int m = 0; m < kModes; ++m) {
+      std::copy(pt.opsem[m].begin(), pt.opsem[m].end(), opsem.begin() + m * all.ops + B.ops);
+      std::copy(pt.lsem[m].begin(), pt.lsem[m].end(), lsem.begin() + m * all.lanes + B.lanes);
+    }
+    for (size_t i = 0; i < pt.semhb.size(); ++i) semhb[B.semhb + i] = pt.semhb[i] + B.hist[pt.semhb_mode[i]];
+    const int32_t l_first = d.prog_loop_ptr[cut[t]];
+    for (size_t i = 0; i < pt.plan_ptr.size(); ++i) plan_ptr[l_first + i] = pt.plan_ptr[i] + b_plan;
+    for (size_t i = 0; i < pt.plan.size(); ++i) {
+      int4 v = pt.plan[i];
+      if (v.x == ITEM_SEG) {
+        v.y += b_chunks;
+        if (v.w >= 0) v.w += b_chunks;
+      }
+      plan[B.plan + i] = v;
+    }
+    for (size_t i = 0; i < pt.chunks.size(); ++i) {
+      const int4 v = pt.chunks[i];
+      chunks[B.chunks + i] = make_int4(v.x + b_lanes, v.y, v.z, v.w);
+    }
+    std::copy(pt.lrec.begin(), pt.lrec.end(), lrec.begin() + B.lanes);
+    std::copy(pt.lmeta.begin(), pt.lmeta.end(), lmeta.begin() + B.lanes);
+    for (size_t i = 0; i < pt.xloops.size(); ++i) {
+      LoopInfo L = pt.xloops[i];
+      L.rowptr_off += B.rowptr;
+      L.pidx_off += B.iters;
+      xloops[B.xloops + i] = L;
+    }
+    std::copy(pt.reads_rowptr.begin(), pt.reads_rowptr.end(), reads_rowptr.begin() + B.xloops);
+    for (size_t i = 0; i < pt.jobs.size(); ++i) {
+      DeriveJob J = pt.jobs[i];
+      J.out += B.derived;
+      if (J.kind == DERIVE_TSTART) {
+        J.a += B.iters;
+        J.b += B.rowptr;
+      } else {
+        J.a += B.path;
+      }
+      jobs[B.jobs + i] = J;
+    }
+    Part released;
+    std::swap(pt, released);                     // the block's memory goes with it
+  };
+  {
+    std::vector<std::thread> pool;
+    for (int t = 0; t + 1 < n_threads; ++t) pool.emplace_back(join_block, t);
+    join_block(n_threads - 1);
+    for (auto& th : pool) th.join();
   }
   op_ptr.push_back((int32_t)ops.size());
   plan_ptr.push_back((int32_t)plan.size());
@@ -666,10 +922,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.rowinfo = h.upload(rowinfo, stream, "row info");
   h.ops = h.upload(ops, stream, "op records");
   h.opstop = h.upload(opstop, stream, "op stops");
+  h.opsem = h.upload(opsem, stream, "op semaphore records");
   {
-    std::vector<int4> both(opsem[0]);
-    for (int m = 1; m < kModes; ++m) both.insert(both.end(), opsem[m].begin(), opsem[m].end());
-    h.opsem = h.upload(both, stream, "op semaphore records");
     std::vector<int32_t> dboth(dsem[0]);
     for (int m = 1; m < kModes; ++m) dboth.insert(dboth.end(), dsem[m].begin(), dsem[m].end());
     h.dsem = h.upload(dboth, stream, "dependency semaphores");
@@ -688,11 +942,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.chunk = h.upload(chunks, stream, "sweep chunks");
   h.lrec = h.upload(lrec, stream, "sweep lanes");
   h.lmeta = h.upload(lmeta, stream, "sweep lane meta");
-  {
-    std::vector<int4> both(lsem[0]);
-    for (int m = 1; m < kModes; ++m) both.insert(both.end(), lsem[m].begin(), lsem[m].end());
-    h.lsem = h.upload(both, stream, "sweep lane semaphores");
-  }
+  h.lsem = h.upload(lsem, stream, "sweep lane semaphores");
   h.n_lanes = (int64_t)lrec.size();
   LoopInfo* d_xloops = h.upload(xloops, stream, "iteration spaces");
   h.divergent = div;

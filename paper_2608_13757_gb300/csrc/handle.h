@@ -84,8 +84,8 @@ struct sync_programs {
     cudaSetDevice(prev);
   }
 
-  template <class T>
-  T* upload(const std::vector<T>& v, cudaStream_t s, const char* what) {
+  template <class V, class T = typename V::value_type>
+  T* upload(const V& v, cudaStream_t s, const char* what) {
     const size_t bytes = std::max<size_t>(v.size(), 1) * sizeof(T);
     void* p = nullptr;
     syncgb::cuda_or_raise(cudaMalloc(&p, bytes), what);

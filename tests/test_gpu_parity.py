@@ -376,6 +376,35 @@ def test_repeated_calls_are_identical(sg):
     assert not np.array_equal(a.makespan.cpu().numpy(), b.makespan.cpu().numpy())
 
 
+# ------------------------------------------------------------------ loader
+
+def test_loader_blocks_join_identically(sg, monkeypatch):
+    """The loader's per-program pass runs in blocks of programs on several
+    threads and joins them: any block count gives the same device encoding,
+    so the same thresholds, checks and schedules."""
+    import torch
+    batch = workloads.concat([workloads.random_trees(8000, 97, workloads.tree_params(
+        engines_hi=5, loops_hi=5, body_hi=6, trip_hi=4, max_depth=4)), workloads.generate("depth2", n_programs=20),
+        workloads.diverge(workloads.random_trees(8001, 40), 5, permille=200)])
+    results = []
+    for n in ("1", "3", "7"):
+        monkeypatch.setenv("SYNCGB_LOAD_THREADS", n)
+        h = sg.sync_load_programs(batch)
+        out = []
+        for mode in MODES:
+            thr = sg.sync_eval_thresholds(h, mode)
+            counts, fb = sg.sync_check_minimal(h, mode, thr)
+            r = sg.sync_simulate(h, mode, thr, timeline=True)
+            out.append((thr.cpu(), counts.cpu(), fb.cpu(), r.makespan.cpu(), r.checksum.cpu(), r.status.cpu(),
+                        r.issue.cpu(), r.retire.cpu()))
+        results.append(out)
+        h.close()
+    for other in results[1:]:
+        for a, b in zip(results[0], other):
+            for x, y in zip(a, b):
+                assert torch.equal(x, y)
+
+
 # ------------------------------------------------- full sizes, sampled checks
 
 @pytest.mark.parametrize("name", ["chain", "depth2", "attention", "syncbound"])
