@@ -31,9 +31,19 @@ METRIC = "dynamic consumer instances/sec (threshold+check+sim), bit-exact; % HBM
 UNIT = "pairs/s"
 WORKLOADS = {
     # name -> description for config.workload
+    "small": "1 program, 2 engines, one loop of 16 iterations, 6-instruction body, 3 cross-engine "
+             "dependencies (one carried at distance 1)",
+    "depth2": "4096 programs, 4 engines, loop depth 2, trips U[1,64] with the inner trip redrawn per "
+              "outer iteration, 16-instruction bodies, 8 dependencies per body",
+    "gemm": "1 program shaped like a tiled 4096x4096x4096 GEMM: 5 engines, M/N/K nest 32x8x32, "
+            "double-buffered dependencies at distance 2",
+    "attention": "256 programs shaped like causal flash attention: head(32) > q-tile(64) > kv-tile "
+                 "(trip = q-tile index), 5 engines, 12-instruction body, running max/sum carried deps",
     "chain": "65536 random chain programs: 2-5 engines, up to 3 loops below the top level, "
              "trips U[0,32] redrawn per parent iteration, 1-32 instructions per body, "
              "dependency density 0.3",
+    "syncbound": "65536 sync-bound programs: single-instruction conditionals alternating engines, "
+                 "each depending on the previous, one distance-1 dependency per loop",
 }
 KERNELS = ("thresholds", "check", "sim_barrier_free", "sim_barrier")
 CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -417,6 +427,7 @@ def main():
     roof, kernels = roofline(res, hbm_peak, peak_kind, clk.get("sm_mhz"), args.config)
     line = {
         "metric": METRIC, "value": total_pairs / (ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "instances_per_s": (res["sizes"].n_instances * world) / (ms / 1e3),
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
         "config": {"workload": WORKLOADS.get(args.config, args.config), "programs_per_gpu": res["P"],
