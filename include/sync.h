@@ -10,8 +10,9 @@
  * loop of trip 0 or 1; the program itself is a top-level loop that runs
  * once).  Loops form a tree; a loop body is an ordered list of items --
  * datapath instructions, each bound to one engine, and child loops -- ordered
- * by a per-item position.  All engines walk this common tree with the same
- * trip counts.  A dependency (producer p, consumer c, offset k) is carried at
+ * by a per-item position.  All engines walk this common tree, with the same
+ * trip counts unless the batch gives per-engine trips (sync_batch_desc).  A
+ * dependency (producer p, consumer c, offset k) is carried at
  * the innermost common loop S of p and c: consumer iteration v waits for the
  * producer through target t = v - k on S (Sec. 5.1).
  *
@@ -37,6 +38,12 @@
  * Instance layout (optional timelines): instruction-major in batch
  * instruction order; instruction x owns one int32 per global iteration of its
  * loop, starting at the sum of the instance counts of earlier instructions.
+ *
+ * Environment (read at each call; both only change how the work is split):
+ *  - SYNCGB_LOAD_THREADS=n: host threads of sync_load_programs (default one
+ *    per hardware thread, at most 32, at least 256 programs each).
+ *  - SYNCGB_WIDE_INDEX=1: the threshold and check kernels index pairs with
+ *    64-bit integers even when 32 bits suffice.
  */
 #ifndef SYNC_H
 #define SYNC_H
