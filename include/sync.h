@@ -176,6 +176,12 @@ typedef struct {
                                  strictly between the top level and the
                                  producer's loop (3: the term N_l*(r_l - 1) of
                                  Sec. 6.1's path sum, O(D) in Table 1) */
+  int32_t trip_register_elision; /* 1: omit r-hat of every loop at which only
+                                 offset-0 dependencies are carried (Sec. 5.1:
+                                 its no-wait check r-hat <= 0 never holds when
+                                 a consumer issues), so its loop statement and
+                                 iteration starts lose one register op each;
+                                 0: every loop keeps r-hat (the default) */
 } sync_sim_params;
 
 typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
@@ -249,6 +255,9 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  * engine cursor t:
  *   loop statement: barrier-free t += c_regop (r-hat := 0); barrier: barrier
  *   iteration start: barrier-free t += c_branch + 2*c_regop; barrier: t += c_branch
+ *   (with trip_register_elision, a loop that carries only offset-0
+ *   dependencies, or none, costs 0 at its statement and c_branch + c_regop
+ *   at each iteration start, barrier-free)
  *   iteration end: barrier only: barrier
  *   datapath x: barrier-free t += sum over its dependencies of the wait
  *     ops: c_wait_ops_count (COUNT), c_wait_ops_perloop (PERLOOP), or

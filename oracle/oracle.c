@@ -44,11 +44,15 @@
  * oracle's own statement; its constants are parameters, and the model is
  * pinned by closed forms and invariants in the tests rather than by numbers
  * printed in the paper.  Integer cycles.  Each engine keeps a cursor t
- * (starting at 0) and walks the common loop tree with the shared trip counts:
+ * (starting at 0) and walks the common loop tree with the shared trip counts
+ * (or its own, with per-engine trips):
  *  - loop statement reached:   barrier-free: t += c_regop (r-hat := 0);
  *                              barrier scheme: an all-engine barrier;
  *  - iteration start:          barrier-free: t += c_branch + 2*c_regop
  *                              (branch, r++, r-hat++); barrier: t += c_branch;
+ *    with trip-register elision, a loop at which only offset-0 dependencies
+ *    are carried (or none) keeps no r-hat (Sec. 5.1): barrier-free, its
+ *    statement costs 0 and each iteration start c_branch + c_regop;
  *  - iteration end:            barrier scheme only: an all-engine barrier;
  *  - datapath instruction x with dependency set D(x):
  *      barrier-free: t += sum over D(x) of the wait-value ops (Table 1):
@@ -796,7 +800,7 @@ typedef struct {
   const orc_sim_params *prm;
   int mode, barrier;
   int64_t *wcost;              /* per instruction: wait-value ops before issue */
-  int64_t iter_cost, stmt_cost; /* per iteration start / loop statement */
+  int64_t *iter_cost, *stmt_cost; /* per loop: iteration start / loop statement */
   const int32_t *thr;          /* program's pairs */
   int64_t *pair_off;           /* per dep */
   int32_t *own_sem, *dep_sem;  /* semaphore incremented by x / waited by d */
@@ -830,7 +834,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
     }
     E->bar_passed = 0;
     if (++f->g < f->g_end) {                   /* next iteration starts */
-      E->t += X->iter_cost;
+      E->t += X->iter_cost[f->loop];
       E->next[f->loop]++;
       f->item = 0;
     } else {
@@ -846,8 +850,8 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
       return S_BARRIER;
     }
     E->bar_passed = 0;
-    if (!X->barrier) E->t += X->stmt_cost;
     int32_t m = -it - 1;
+    if (!X->barrier) E->t += X->stmt_cost[m];
     int32_t trip = trip_on(P, m, e, f->g);
     f->item++;
     if (trip > 0) {
@@ -855,7 +859,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
       c->loop = m; c->item = 0;
       c->g = E->next[m]; c->g_end = c->g + trip;
       E->next[m]++;
-      E->t += X->iter_cost;
+      E->t += X->iter_cost[m];
     }
     return S_PROGRESS;
   }
@@ -905,13 +909,34 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     }
     wcost[P->dc[d]] += c;
   }
-  int64_t iter_cost = unrolled ? 0 : barrier ? q->c_branch : q->c_branch + 2 * (int64_t)q->c_regop;
-  int64_t stmt_cost = unrolled ? 0 : q->c_regop;
+  /* per loop: the register ops of its statement (r-hat := 0) and of each
+   * iteration start (branch, r++, r-hat++); with trip-register elision a
+   * loop that carries only offset-0 dependencies (or none) has no r-hat
+   * (Sec. 5.1), barrier-free */
+  int64_t *iter_cost = (int64_t *)calloc((size_t)nl, sizeof(int64_t));
+  int64_t *stmt_cost = (int64_t *)calloc((size_t)nl, sizeof(int64_t));
+  int8_t *needs_rhat = (int8_t *)calloc((size_t)nl, sizeof(int8_t));
+  if (!iter_cost || !stmt_cost || !needs_rhat) {
+    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost);
+    return ORC_ERR_OOM;
+  }
+  for (int32_t d = 0; d < nd; ++d)
+    if (P->dk[d] > 0) needs_rhat[classify(P, d).S] = 1;
+  for (int32_t l = 0; l < nl; ++l) {
+    int elide = q->trip_register_elision && !needs_rhat[l];
+    iter_cost[l] = unrolled ? 0 : barrier ? q->c_branch : q->c_branch + (elide ? 1 : 2) * (int64_t)q->c_regop;
+    stmt_cost[l] = unrolled || elide ? 0 : q->c_regop;
+  }
+  free(needs_rhat);
   /* the static time bound */
-  u128 bound = 0;
+  u128 bound = 0, ctl = 0;
   int64_t stmts = 0, iters = 0;      /* summed over the engines */
   for (int32_t e = 0; e < ne; ++e)
-    for (int32_t l = 1; l < nl; ++l) { stmts += tot_on(P, P->par[l], e); iters += tot_on(P, l, e); }
+    for (int32_t l = 1; l < nl; ++l) {
+      stmts += tot_on(P, P->par[l], e);
+      iters += tot_on(P, l, e);
+      ctl += (u128)tot_on(P, P->par[l], e) * (u128)stmt_cost[l] + (u128)tot_on(P, l, e) * (u128)iter_cost[l];
+    }
   for (int32_t x = 0; x < nx; ++x) {
     int64_t per = (int64_t)P->xlat[x] + q->ii;
     if (!barrier) per += wcost[x];
@@ -921,10 +946,10 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     bound += (u128)iters * (u128)q->c_branch;
     bound += (u128)(stmts / ne + iters / ne) * (u128)q->c_barrier;
   } else {
-    bound += (u128)stmts * (u128)stmt_cost + (u128)iters * (u128)iter_cost;
+    bound += ctl;
   }
   if (bound > (u128)INT32_MAX) {
-    free(wcost);
+    free(wcost); free(iter_cost); free(stmt_cost);
     *makespan = -1; *checksum = 0; *status = ORC_SIM_OVERFLOW;
     return ORC_OK;
   }
@@ -1010,7 +1035,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   for (int32_t e = 0; E && e < ne; ++e) { free(E[e].st); free(E[e].next); }
   for (int32_t s = 0; X.times && s < nsem; ++s) free(X.times[s]);
   free(E); free(incs); free(X.pair_off); free(X.inst_off); free(X.own_sem); free(X.dep_sem);
-  free(X.value); free(X.times); free(wcost);
+  free(X.value); free(X.times); free(wcost); free(iter_cost); free(stmt_cost);
   return rc;
 }
 

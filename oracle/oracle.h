@@ -65,6 +65,7 @@ typedef struct {
   int32_t c_wait_ops_perloop; /* wait-value ops per dependency, per-loop mode  */
   int32_t c_barrier;          /* all-engine barrier handshake + reset          */
   int32_t c_wait_ops_perengine_level; /* per-engine mode: per enclosing loop level */
+  int32_t trip_register_elision; /* 1: no r-hat for loops carrying only offset-0 deps */
 } orc_sim_params;
 
 /* Per-engine trip counts (control-flow divergence, Sec. 7.5): each engine

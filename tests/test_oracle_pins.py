@@ -731,3 +731,78 @@ def test_divergent_rejects_barrier_and_per_engine():
     t = oracle.thresholds(b, PERLOOP)
     with pytest.raises(oracle.OracleError):
         oracle.simulate(b, t, PERLOOP, oracle.BARRIER)
+
+
+# ------------------------------------------------ trip-register elision (Sec. 5.1)
+
+def _no_rhat_loops(batch):
+    """Loops (program-local, not the top level) at which no dependency with
+    a nonzero offset is carried: their trip register can be omitted."""
+    cls = oracle.classify(batch)
+    needs = {int(cls.S[d]) for d in range(batch.n_deps) if int(batch.dep_k[d]) > 0}
+    return {l for l in range(1, batch.n_loops) if l not in needs}
+
+
+@pytest.mark.parametrize("T,lat", [(1, 1), (5, 3), (12, 1)])
+def test_elision_closed_form_one_engine(T, lat):
+    """One engine, one loop of T iterations with one instruction and no
+    dependency: without r-hat the loop statement and every iteration start
+    lose one register op, so the makespan drops by exactly c_regop * (1 + T)."""
+    b = workloads.ProgramBuilder(1)
+    L = b.loop(0, 0, [T])
+    b.instr(L, 0, 0, latency=lat)
+    batch = b.batch()
+    t = oracle.thresholds(batch, PERLOOP)
+    for c_regop in (1, 4):
+        prm0 = oracle.sim_params(c_regop=c_regop, c_branch=2)
+        prm1 = oracle.sim_params(c_regop=c_regop, c_branch=2, trip_register_elision=1)
+        m0 = oracle.simulate(batch, t, PERLOOP, oracle.BARRIER_FREE, prm0).makespan[0]
+        m1 = oracle.simulate(batch, t, PERLOOP, oracle.BARRIER_FREE, prm1).makespan[0]
+        assert m0 - m1 == c_regop * (1 + T)
+        # the barrier scheme has no registers to elide
+        b0 = oracle.simulate(batch, t, PERLOOP, oracle.BARRIER, prm0).makespan[0]
+        b1 = oracle.simulate(batch, t, PERLOOP, oracle.BARRIER, prm1).makespan[0]
+        assert b0 == b1
+
+
+def test_elision_keeps_rhat_for_carried_offsets():
+    """A loop carrying a dependency with offset 1 keeps its trip register:
+    the flag changes nothing for a program whose only loop carries one."""
+    b = workloads.ProgramBuilder(2)
+    L = b.loop(0, 0, [6])
+    x = b.instr(L, 0, 0, latency=2)
+    y = b.instr(L, 1, 1, latency=3)
+    b.dep(x, y, 1)
+    batch = b.batch()
+    assert _no_rhat_loops(batch) == set()
+    t = oracle.thresholds(batch, PERLOOP)
+    m0 = oracle.simulate(batch, t, PERLOOP, oracle.BARRIER_FREE).makespan[0]
+    m1 = oracle.simulate(batch, t, PERLOOP, oracle.BARRIER_FREE,
+                         oracle.sim_params(trip_register_elision=1)).makespan[0]
+    assert m0 == m1
+
+
+@pytest.mark.parametrize("mode", [COUNT, PERLOOP, PERENGINE])
+def test_elision_matches_recursive_statement(mode):
+    """With trip-register elision the semaphore machine and the recursive
+    statement (each elided loop's statement free, its iteration starts one
+    register op cheaper) agree on makespans, checksums and timelines."""
+    prm = oracle.sim_params(ii=2, c_branch=3, c_regop=2, c_wait_ops_perengine_level=2,
+                            trip_register_elision=1)
+    n = 0
+    for seed, batch in _random_batches(50):
+        thr = oracle.thresholds(batch, mode)
+        thr_c = oracle.thresholds(batch, COUNT)
+        r = oracle.simulate(batch, thr, mode, oracle.BARRIER_FREE, prm, timeline=True)
+        assert r.status[0] == 0
+        ms, chk, tl = timing_model.simulate(batch, thr_c, prm, False, wait_ops(batch, mode, prm),
+                                            no_rhat=_no_rhat_loops(batch))
+        assert r.makespan[0] == ms and int(r.checksum[0]) == chk, seed
+        off = 0
+        tot = loop_totals(batch)
+        for x in range(batch.n_instrs):
+            for g in range(int(tot[batch.instr_loop[x]])):
+                assert (r.issue[off + g], r.retire[off + g]) == tl[(x, g)]
+            off += int(tot[batch.instr_loop[x]])
+        n += 1
+    assert n == 50

@@ -50,11 +50,11 @@ def _events(batch, e, barrier):
                     ev.append(("x", i, g))
                 continue
             m = i
-            ev.append(("stmt",))
+            ev.append(("stmt", m))
             for _ in range(int(trips[m][g])):
                 gm = nxt[m]
                 nxt[m] += 1
-                ev.append(("iter",))
+                ev.append(("iter", m))
                 run(m, gm)
                 if barrier:
                     ev.append(("end",))
@@ -63,9 +63,11 @@ def _events(batch, e, barrier):
     return ev
 
 
-def simulate(batch, thr_count, params, barrier, cwait, unrolled=False):
+def simulate(batch, thr_count, params, barrier, cwait, unrolled=False, no_rhat=()):
     """(makespan, checksum, {(x, g): (issue, retire)}) or raises Deadlock.
-    cwait: wait ops per dependency, an int or a function of the dependency."""
+    cwait: wait ops per dependency, an int or a function of the dependency.
+    no_rhat: loops without a trip register (their statement costs nothing
+    and their iteration starts one register op less, barrier-free)."""
     wait_ops = cwait if callable(cwait) else (lambda d: cwait)
     ne = int(batch.prog_n_engines[0])
     ev = [_events(batch, e, barrier) for e in range(ne)]
@@ -137,11 +139,12 @@ def simulate(batch, thr_count, params, barrier, cwait, unrolled=False):
                 rel = max(rel, ft, flr)
             out = (rel + params.c_barrier, lr, None, None)
         elif v[0] == "stmt":
-            out = (t + (0 if unrolled else params.c_regop), lr, None, None)
+            out = (t + (0 if unrolled or v[1] in no_rhat else params.c_regop), lr, None, None)
         elif unrolled:  # iteration start of the unrolled program: nothing
             out = (t, lr, None, None)
-        else:  # iteration start
-            out = (t + params.c_branch + (0 if barrier else 2 * params.c_regop), lr, None, None)
+        else:  # iteration start: branch, r++ and (unless elided) r-hat++
+            regops = 0 if barrier else (1 if v[1] in no_rhat else 2)
+            out = (t + params.c_branch + regops * params.c_regop, lr, None, None)
         busy.discard(key)
         memo[key] = out
         return out
