@@ -112,6 +112,7 @@ struct ProgScratch {
   std::vector<LoopInfo> el;                       // per-engine trips: loop table per (loop, engine)
   std::vector<int32_t> xid;                       // per-engine trips: expansion-table entry per (loop, engine)
   std::vector<int64_t> tstart_of;                 // derived trip-start array per loop (and engine), -1 if none
+  std::vector<uint8_t> needs_rhat;                // per loop: carries a dependency with offset > 0
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
 };
 
@@ -225,10 +226,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<int64_t> ord_off(NX, -1);   // per instruction: ordinal pool offset (waited producers)
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
+  std::vector<int32_t> lflag(NL, 0);       // per loop: carries no offset > 0 (trip register elidable)
 
   // Programs [p_begin, p_end) into `part`; erow0: their first per-engine row.
   auto run_block = [&d, div, &loop, &dep, &prog, &inst_off, &dseg, &ddep, &dsem, &seg, &ord_off, &dep_N,
-                    &dep_K](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
+                    &dep_K, &lflag](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
   auto& rowptr_host = part.rowptr_host;
   auto& path = part.path;
   auto& op_ptr = part.op_ptr;
@@ -271,6 +273,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     S.total.assign(nl, 0);
     S.tstart_of.assign((size_t)nl * (div ? ne : 1), -1);
     S.anc_of.clear();
+    S.needs_rhat.assign(nl, 0);
     if (par[0] != -1) raise(SYNC_ERR_MALFORMED, where(p, "loop 0 must have parent -1, loop", 0));
     int32_t depth_max = 0;
     for (int32_t l = 1; l < nl; ++l) {
@@ -431,6 +434,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       while (S.depth[b] > S.depth[a]) { cb = b; b = par[b]; }
       while (a != b) { ca = a; a = par[a]; cb = b; b = par[b]; }
       const int32_t Sl = a;
+      if (off > 0) S.needs_rhat[Sl] = 1;           // r-hat_S's no-wait check matters
       const int32_t ppos = ca < 0 ? d.instr_pos[x0 + px] : lpos[ca];
       const int32_t cpos = cb < 0 ? d.instr_pos[x0 + cx] : lpos[cb];
       const bool forward = cpos > ppos;
@@ -510,6 +514,16 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       pi.n_pairs += tot(Cl, ec);
       dep_N[gd] = N;
       dep_K[gd] = K;
+    }
+    // loops whose trip register can be elided (Sec. 5.1: only offset-0
+    // dependencies carried there, or none), and their control counts
+    for (int32_t l = 1; l < nl; ++l) {
+      lflag[l0 + l] = S.needs_rhat[l] ? 0 : 1;
+      if (S.needs_rhat[l]) continue;
+      for (int32_t e = 0; e < ne; ++e) {
+        pi.el_stmt += tot(par[l], e);
+        pi.el_iter += tot(l, e);
+      }
     }
     // semaphores that some dependency waits on, per mode, with their history
     // slots: mode 0 = one per producer instruction (one increment per
@@ -598,7 +612,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         const int32_t end_idx = (int32_t)ops.size();
         ops.push_back(make_int4(OP_END, 0, 0, 0));
         for (int m = 0; m < kModes; ++m) opsem[m].push_back(make_int4(-1, 0, 0, 0));
-        rowinfo.push_back(make_int2(end_idx, has_loop ? 1 : 0));
+        rowinfo.push_back(make_int2(end_idx, (has_loop ? 1 : 0) | (lflag[l0 + l] ? 2 : 0)));
         // next LOOP or END record at or after each record of the row
         opstop.resize(ops.size());
         int32_t next = end_idx;
@@ -633,7 +647,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         }
         if (!at_end) {
           ++nloops;
-          plan.push_back(make_int4(ITEM_LOOP, l0 + (-it - 1), 0, 0));
+          plan.push_back(make_int4(ITEM_LOOP, l0 + (-it - 1), lflag[l0 + (-it - 1)], 0));
         }
       }
       // a short body with no child loop: a template of several iterations
@@ -938,6 +952,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.next_slot = h.alloc<int32_t>(1, "program-slot counter");
   h.fallback = h.alloc<int32_t>((int64_t)P + 1, "fallback list");
   h.plan_ptr = h.upload(plan_ptr, stream, "sweep plan offsets");
+  h.lflag = h.upload(lflag, stream, "loop flags");
   h.plan = h.upload(plan, stream, "sweep plan");
   h.chunk = h.upload(chunks, stream, "sweep chunks");
   h.lrec = h.upload(lrec, stream, "sweep lanes");
@@ -1129,7 +1144,7 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
   w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
   w.issue = d_issue; w.retire = d_retire;
   w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
-  w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring;
+  w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring; w.lflag = h->lflag;
   w.dep = a.dep; w.ddep = a.ddep; w.path = a.path; w.ord = a.ord;
   w.chk_counts = a.chk_counts; w.chk_first = a.chk_first;
   const bool barrier = variant == SYNC_SIM_BARRIER;

@@ -65,6 +65,8 @@ struct alignas(16) ProgInfo {
   int64_t n_iter;     // loop iterations of one engine (likewise)
   int64_t eng_stmt;   // loop statements summed over the engines
   int64_t eng_iter;   // loop iterations summed over the engines
+  int64_t el_stmt;    // of these, those of loops that carry no offset > 0 (whose trip
+  int64_t el_iter;    // register can be elided)
   int64_t pair_levels;  // sum over pairs of the per-engine wait's extra levels
   int32_t ne;
   int32_t le_base;    // row of (top-level loop, engine 0); row of (program-local
@@ -78,7 +80,7 @@ struct alignas(16) ProgInfo {
 // Program-order sweep tables.  Per loop, a plan: its body cut at child loops
 // into straight-line segments; items [plan_ptr[l], plan_ptr[l+1]):
 //   {ITEM_SEG, first chunk, chunks, multi-iteration chunk or -1}
-//   {ITEM_LOOP, child loop (global id), 0, 0}
+//   {ITEM_LOOP, child loop (global id), child's elidable-trip-register flag, 0}
 // A chunk holds up to 32 datapath records of one segment (all engines), in
 // lanes ordered engine-major (then iteration copy, then body position):
 //   chunk {first lane record, lanes, iteration copies, engine bitmask}
@@ -102,7 +104,8 @@ constexpr int32_t LANE_RUN_LAST = 2;
 //   end       {OP_END, 0, 0, 0}
 // Per record: opstop = index of the first LOOP or END record at or after it
 // in its row.  Per row: op_ptr = first record, rowinfo = {END record index,
-// 1 if the row holds a LOOP record}.
+// bit 0: the row holds a LOOP record, bit 1: the row's loop carries no
+// offset > 0 (its trip register can be elided)}.
 // Per-mode semaphore records parallel to the op records (mode 0 = one
 // semaphore per producer instruction, mode 1 = one per (loop, engine),
 // mode 2 = one per engine):
@@ -227,6 +230,7 @@ struct SweepArgs {
   int32_t sem_cap;
   int32_t frame_depth;
   int32_t ring;              // latest increments kept per semaphore (power of two)
+  const int32_t* lflag;      // per loop: 1 if it carries no offset > 0 (trip register elidable)
   // fused simulation (thresholds from the walk's loop state, no threshold
   // array): dep is set (NULL otherwise) and thr is unused
   const DepInfo* dep;

@@ -31,6 +31,7 @@ struct sync_programs {
   int32_t* pidx = nullptr;
   syncgb::DepInfo* dep = nullptr;
   int32_t* ddep = nullptr;          // per consumer-grouped dependency: dependency id
+  int32_t* lflag = nullptr;         // per loop: trip register elidable
   int64_t* seg = nullptr;
   int32_t* tile_first = nullptr;
   int64_t* path = nullptr;

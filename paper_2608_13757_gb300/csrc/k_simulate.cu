@@ -104,9 +104,15 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
     if (MODE == SYNC_THR_PERENGINE)
       b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
-    // control operations of every engine (their own trips)
-    b = sat_add(b, sat_add(sat_mul((u64)pi.eng_stmt, (u64)q.c_regop),
-                           sat_mul((u64)pi.eng_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop)));
+    // control operations of every engine (their own trips): r-hat := 0 at
+    // statements and the branch, r++ and r-hat++ at iteration starts, minus
+    // the r-hat ops of loops without a trip register when that is elided
+    const u64 el = q.trip_register_elision ? 1 : 0;
+    const u64 rhat_stmts = (u64)pi.eng_stmt - el * (u64)pi.el_stmt;
+    const u64 rhat_iters = (u64)pi.eng_iter - el * (u64)pi.el_iter;
+    b = sat_add(b, sat_mul(rhat_stmts, (u64)q.c_regop));
+    b = sat_add(b, sat_mul((u64)pi.eng_iter, (u64)q.c_branch + (u64)q.c_regop));
+    b = sat_add(b, sat_mul(rhat_iters, (u64)q.c_regop));
   }
   return b;
 }
@@ -128,6 +134,7 @@ struct Smem {
 struct Eng {
   int32_t row, pbeg, rend, ptr, g, g_end, sp;
   int32_t lo;              // start of the current trip
+  int32_t ic;              // iteration-start cost of the current row's loop
   bool loops;              // the current row holds a child loop
   int32_t t, lastret;
   int32_t bar_gen;         // barrier generation this engine waits to see pass
@@ -174,7 +181,11 @@ __device__ __forceinline__ void set_row(const SimArgs& a, Eng& E, int32_t row) {
   E.pbeg = __ldg(a.op_ptr + row);
   const int2 ri = __ldg(a.rowinfo + row);
   E.rend = ri.x;
-  E.loops = ri.y != 0;
+  E.loops = (ri.y & 1) != 0;
+  // barrier-free with trip-register elision, a loop carrying no offset > 0
+  // has no r-hat++ at its iteration starts
+  const int32_t ic = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+  E.ic = !BB && a.prm.trip_register_elision && (ri.y & 2) ? ic - a.prm.c_regop : ic;
 }
 
 // Fused simulation: the wait value of consumer-grouped dependency r for the
@@ -210,7 +221,6 @@ template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng& E, int w, int lane,
                                            int ne, unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
-  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int32_t ii = a.prm.ii;
   Frame* frames = S.frames + w * a.frame_depth;
   bool moved = false;
@@ -234,7 +244,10 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
     }
     if (r0.x == OP_LOOP) {                           // a loop statement
       E.bar_passed = false;
-      if (!BB) E.t += a.prm.c_regop;
+      if (!BB) {                                     // r-hat := 0, unless the child has none
+        const bool el = a.prm.trip_register_elision && (__ldg(a.rowinfo + r0.y + w).y & 2);
+        E.t += el ? 0 : a.prm.c_regop;
+      }
       const int64_t rp = lohi(r0.z, r0.w) + E.g;
       const int32_t lo = __ldg(a.rowptr + rp), hi = __ldg(a.rowptr + rp + 1);
       ++E.ptr;
@@ -247,7 +260,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
         E.g = lo;
         E.g_end = hi;
         E.lo = lo;
-        E.t += iter_cost;
+        E.t += E.ic;
       }
       moved = true;
       continue;
@@ -256,7 +269,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
       if (E.sp == 0) { E.state = ST_DONE; return true; }   // the top-level loop runs once
       E.bar_passed = false;
       if (++E.g < E.g_end) {
-        E.t += iter_cost;
+        E.t += E.ic;
         E.ptr = E.pbeg;
       } else {
         __syncwarp();
@@ -331,7 +344,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
     int32_t A = 0, B = kNeg;
     if (in) {
       if (dp) { A = wcost + ii; B = waited ? ready + ii : kNeg; }
-      else A = iter_cost;
+      else A = E.ic;
     }
     for (int o = 1; o < 32; o <<= 1) {
       const int32_t Ap = __shfl_up_sync(kFull, A, o), Bp = __shfl_up_sync(kFull, B, o);
@@ -438,7 +451,7 @@ __global__ void __launch_bounds__(1024) k_simulate(const SimArgs a) {
     E.t = 0; E.lastret = 0; E.bar_gen = 0; E.n = 0;
     E.state = live ? ST_RUN : ST_DONE;
     E.bar_passed = false;
-    E.row = 0; E.pbeg = 0; E.rend = 0; E.loops = false; E.ptr = 0;
+    E.row = 0; E.pbeg = 0; E.rend = 0; E.loops = false; E.ptr = 0; E.ic = 0;
     if (live) {
       set_row<MODE, BB, TL>(a, E, pi.le_base + w);
       E.ptr = E.pbeg;

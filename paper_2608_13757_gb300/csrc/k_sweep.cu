@@ -84,9 +84,15 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
     if (MODE == SYNC_THR_PERENGINE)
       b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
-    // control operations of every engine (their own trips)
-    b = sat_add(b, sat_add(sat_mul((u64)pi.eng_stmt, (u64)q.c_regop),
-                           sat_mul((u64)pi.eng_iter, (u64)q.c_branch + 2ull * (u64)q.c_regop)));
+    // control operations of every engine (their own trips): r-hat := 0 at
+    // statements and the branch, r++ and r-hat++ at iteration starts, minus
+    // the r-hat ops of loops without a trip register when that is elided
+    const u64 el = q.trip_register_elision ? 1 : 0;
+    const u64 rhat_stmts = (u64)pi.eng_stmt - el * (u64)pi.el_stmt;
+    const u64 rhat_iters = (u64)pi.eng_iter - el * (u64)pi.el_iter;
+    b = sat_add(b, sat_mul(rhat_stmts, (u64)q.c_regop));
+    b = sat_add(b, sat_mul((u64)pi.eng_iter, (u64)q.c_branch + (u64)q.c_regop));
+    b = sat_add(b, sat_mul(rhat_iters, (u64)q.c_regop));
   }
   return b;
 }
@@ -199,10 +205,9 @@ __device__ __forceinline__ void set_groups(const WarpSmem& S, const LaneRec& L, 
 template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, const LaneRec& L,
                                          const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
-                                         int32_t ctag, int lane, int lc, int32_t lo_c,
+                                         int32_t ctag, int lane, int lc, int32_t lo_c, int32_t iter_cost,
                                          unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
-  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int4 rec = L.rec, sr = L.sr;
   const bool have = lane < ch.y;
   const bool valid = have && L.meta.y < copies;
@@ -394,9 +399,9 @@ __device__ __forceinline__ int32_t fused_iter(const SweepArgs& a, const WarpSmem
 template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi,
                                              const int4 ch, const LaneRec& L, int32_t lo, int32_t hi,
-                                             int32_t ctag, int lane, int lc, unsigned long long& chk) {
+                                             int32_t ctag, int lane, int lc, int32_t iter_cost,
+                                             unsigned long long& chk) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
-  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
   const int32_t ii = a.prm.ii;
   const int32_t copies = ch.z;
   const bool have = lane < ch.y;
@@ -616,14 +621,13 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
 template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi, const int4 ch,
                                         int32_t lo, int32_t hi, int32_t ctag, int lane, int lc,
-                                        unsigned long long& chk) {
-  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+                                        int32_t iter_cost, unsigned long long& chk) {
   const int32_t copies = ch.z;
   const bool have = lane < ch.y;
   LaneRec L;
   load_lane(a, ch, lane, L);
   if (!__ballot_sync(kFull, have && L.rec.z > kMaxDeps))
-    return run_loop_regs<MODE, BB, TL, FUSED>(a, S, pi, ch, L, lo, hi, ctag, lane, lc, chk);
+    return run_loop_regs<MODE, BB, TL, FUSED>(a, S, pi, ch, L, lo, hi, ctag, lane, lc, iter_cost, chk);
   set_groups(S, L, lane, have, min(copies, hi - lo), ctag);
   int32_t Tn[kMaxDeps];
   load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - lo, lo + L.meta.y, lc, lo, Tn);
@@ -635,7 +639,7 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
     const int32_t gn = g + v;
     if (gn < hi) load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - gn, gn + L.meta.y, lc, lo, Tn);
     if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
-    const int verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, chk);
+    const int verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk);
     if (verdict) return verdict;
     g = gn;
     if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
@@ -678,7 +682,13 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     S.rmask = a.ring - 1;
   }
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
-  const int32_t iter_cost = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+  // iteration-start and statement costs of a loop; a loop flagged as
+  // carrying only offset-0 dependencies keeps no trip register when the
+  // elision is on (barrier-free: no r-hat := 0, no r-hat++)
+  const bool elide = !BB && a.prm.trip_register_elision != 0;
+  const int32_t ic_full = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
+  auto iter_cost_of = [&](int32_t flag) { return elide && flag ? ic_full - a.prm.c_regop : ic_full; };
+  auto stmt_cost_of = [&](int32_t flag) { return elide && flag ? 0 : a.prm.c_regop; };
 
   for (;;) {
     int slot = 0;
@@ -712,6 +722,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     __syncwarp();
     unsigned long long chk = 0;
     int32_t loop = pi.loop_base, item = 0, g = 0, g_end = 1, sp = 0, ctag = 0;
+    int32_t iter_cost = ic_full;                       // of the loop being walked
     int32_t pbeg = __ldg(a.plan_ptr + loop), pend = __ldg(a.plan_ptr + loop + 1);
     int verdict = SYNC_PROG_OK;
     for (;;) {
@@ -726,6 +737,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         } else {
           const Frame f = S.frames[--sp];
           loop = f.loop; item = f.item; g = f.g; g_end = f.g_end;
+          iter_cost = iter_cost_of(__ldg(a.lflag + loop));
           pbeg = __ldg(a.plan_ptr + loop);
           pend = __ldg(a.plan_ptr + loop + 1);
         }
@@ -736,15 +748,16 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         if (BB) {
           barrier_all(S, pi.ne, a.prm.c_barrier, lane);
         } else {
-          if (lane < pi.ne) S.t[lane] += a.prm.c_regop;
+          if (lane < pi.ne) S.t[lane] += stmt_cost_of(it.z);
         }
+        const int32_t child_ic = iter_cost_of(it.z);
         const LoopInfo L = a.loop[it.y];
         const int32_t lo = __ldg(a.rowptr + L.rowptr_off + g), hi = __ldg(a.rowptr + L.rowptr_off + g + 1);
         ++item;
         if (lo < hi) {
           const int32_t cb = __ldg(a.plan_ptr + it.y), ce = __ldg(a.plan_ptr + it.y + 1);
           __syncwarp();
-          if (lane < pi.ne) S.t[lane] += iter_cost;    // the first iteration starts
+          if (lane < pi.ne) S.t[lane] += child_ic;    // the first iteration starts
           __syncwarp();
           if (ce - cb == 1) {
             const int4 body = __ldg(a.plan + cb);
@@ -752,7 +765,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
             if (body.x == ITEM_SEG && (multi || body.z == 1)) {
               // a loop around one chunk: all its iterations in registers
               verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + (multi ? body.w : body.y)), lo,
-                                                      hi, ++ctag, lane, sp + 1, chk);
+                                                      hi, ++ctag, lane, sp + 1, child_ic, chk);
               if (verdict) break;
               continue;
             }
@@ -761,6 +774,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
           ++sp;
           if (FUSED && lane == 0) S.lvl[sp] = make_int2(lo, lo);
           loop = it.y; item = 0; g = lo; g_end = hi;
+          iter_cost = child_ic;
           pbeg = cb;
           pend = ce;
         }
@@ -777,7 +791,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
         load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y && Lr.meta.y < v, g + Lr.meta.y, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, v, ++ctag);
-        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, chk);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, iter_cost, chk);
         if (verdict) break;
         g += v - 1;
         item = pend - pbeg;                            // continue at the END of iteration g
@@ -791,7 +805,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
         load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y, g, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, 1, ++ctag);
-        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, chk);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, iter_cost, chk);
       }
       if (verdict) break;
       ++item;

@@ -376,6 +376,27 @@ def test_repeated_calls_are_identical(sg):
     assert not np.array_equal(a.makespan.cpu().numpy(), b.makespan.cpu().numpy())
 
 
+# ------------------------------------------------- trip-register elision
+
+@pytest.mark.parametrize("seed", range(3))
+def test_trip_register_elision(sg, seed):
+    """Loops that carry only offset-0 dependencies keep no trip register
+    (Sec. 5.1) when the switch is on: every mode and scheme, array and
+    fused, equal to the oracle; and a batch where no loop qualifies gives the
+    same schedules with the switch on and off."""
+    batch = workloads.concat([workloads.random_trees(9000 + seed, 120, workloads.tree_params(
+        engines_hi=5, loops_hi=6, body_hi=6, trip_hi=4, max_depth=4)), workloads.generate("depth2", n_programs=8),
+        workloads.generate("small")])
+    compare_all(sg, batch, timeline=True, modes=ALL_MODES,
+                params=oracle.sim_params(ii=2, c_branch=3, c_regop=4, trip_register_elision=1))
+
+
+def test_trip_register_elision_divergent(sg):
+    batch = workloads.diverge(workloads.random_trees(9100, 80), 3, permille=200)
+    compare_all(sg, batch, timeline=True, modes=MODES,
+                params=oracle.sim_params(c_regop=3, trip_register_elision=1))
+
+
 # ------------------------------------------------------------------ loader
 
 def test_loader_blocks_join_identically(sg, monkeypatch):
