@@ -148,7 +148,11 @@ template <int MODE, typename I>
 __global__ void __launch_bounds__(kThreads, 8) k_check(const CheckArgs a) {
   const I stride = (I)gridDim.x * kThreads, n_chunks = (I)a.t.n_chunks;
   const I end = (n_chunks + 31) & ~I(31);
-  for (I c = (I)blockIdx.x * kThreads + threadIdx.x; c < end; c += stride) {
+  for (I cf = (I)blockIdx.x * kThreads + threadIdx.x; cf < end; cf += stride) {
+    // 32-chunk groups from the last one down (lanes ascending inside a
+    // group): the thresholds written last by the threshold kernel, still
+    // in L2 when this kernel follows it, are read first
+    const I c = end - 32 - (cf & ~I(31)) + (cf & 31);
     const I q = c * kChunk;
     bool bad = false;
     int4 v = make_int4(0, 0, 0, 0), m = v;
