@@ -147,7 +147,7 @@ struct Part {
   std::vector<int64_t> semhb;
   std::vector<uint8_t> semhb_mode;         // per semaphore base: its mode (history space)
   std::vector<int32_t> plan_ptr;
-  std::vector<int4> plan, chunks, lrec, lmeta, lsem[kModes];
+  std::vector<int4> plan, paux, chunks, lrec, lmeta, lsem[kModes];
   std::vector<LoopInfo> xloops;
   std::vector<uint8_t> reads_rowptr;
   std::vector<DeriveJob> jobs;
@@ -241,6 +241,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   auto& semhb = part.semhb;
   auto& plan_ptr = part.plan_ptr;
   auto& plan = part.plan;
+  auto& paux = part.paux;
   auto& chunks = part.chunks;
   auto& lrec = part.lrec;
   auto& lmeta = part.lmeta;
@@ -623,6 +624,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       }
     // program-order sweep plan: per loop, its body cut at child loops into
     // straight-line segments, each segment in chunks of <= 32 engine-sorted lanes
+    const size_t plan_first_loop = plan_ptr.size(), plan_first_item = plan.size();
     for (int32_t l = 0; l < nl; ++l) {
       plan_ptr.push_back((int32_t)plan.size());
       std::vector<int32_t> seg;
@@ -662,6 +664,23 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         plan.back().w = (int32_t)chunks.size();
         add_chunk(d, x0, S, recs, copies, k, chunks, lrec, lmeta, lsem);
       }
+    }
+    // per loop statement, what the walker needs without further lookups:
+    // the child's rowptr offset, and the chunk that holds its whole body
+    // (barrier-free: the multi-iteration template if there is one), or -1
+    paux.resize(plan.size(), make_int4(0, 0, -1, -1));
+    for (size_t i = plan_first_item; i < plan.size(); ++i) {
+      if (plan[i].x != ITEM_LOOP) continue;
+      const int32_t m = plan[i].y - l0;
+      const size_t b = plan_ptr[plan_first_loop + m];
+      const size_t e = m + 1 < nl ? (size_t)plan_ptr[plan_first_loop + m + 1] : plan.size();
+      int32_t bf = -1, bb = -1;
+      if (e - b == 1 && plan[b].x == ITEM_SEG) {
+        if (plan[b].z == 1) bf = bb = plan[b].y;
+        if (plan[b].w >= 0) bf = plan[b].w;
+      }
+      const int64_t rp = loop[l0 + m].rowptr_off;
+      paux[i] = make_int4((int32_t)(uint32_t)(rp & 0xffffffffu), (int32_t)(rp >> 32), bf, bb);
     }
     for (int m = 0; m < kModes; ++m) part.nsem_max[m] = std::max(part.nsem_max[m], pi.nsem[m]);
     part.ne_max = std::max(part.ne_max, ne);
@@ -744,7 +763,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   HostVec<int4> ops(all.ops), opsem(kModes * all.ops);    // opsem: mode-major
   HostVec<int64_t> semhb(all.semhb);
   HostVec<int32_t> plan_ptr(NL);             // one entry per loop; the blocks own consecutive loops
-  HostVec<int4> plan(all.plan), chunks(all.chunks), lrec(all.lanes), lmeta(all.lanes);
+  HostVec<int4> plan(all.plan), paux(all.plan), chunks(all.chunks), lrec(all.lanes), lmeta(all.lanes);
   HostVec<int4> lsem(kModes * all.lanes);                  // mode-major
   HostVec<LoopInfo> xloops(all.xloops);
   HostVec<uint8_t> reads_rowptr(all.xloops);
@@ -813,6 +832,13 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         if (v.w >= 0) v.w += b_chunks;
       }
       plan[B.plan + i] = v;
+      int4 x = pt.paux[i];
+      if (v.x == ITEM_LOOP) {
+        const int64_t rp = (int64_t)(((uint64_t)(uint32_t)x.y << 32) | (uint32_t)x.x) + B.rowptr;
+        x = make_int4((int32_t)(uint32_t)(rp & 0xffffffffu), (int32_t)(rp >> 32), x.z >= 0 ? x.z + b_chunks : -1,
+                      x.w >= 0 ? x.w + b_chunks : -1);
+      }
+      paux[B.plan + i] = x;
     }
     for (size_t i = 0; i < pt.chunks.size(); ++i) {
       const int4 v = pt.chunks[i];
@@ -954,6 +980,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.plan_ptr = h.upload(plan_ptr, stream, "sweep plan offsets");
   h.lflag = h.upload(lflag, stream, "loop flags");
   h.plan = h.upload(plan, stream, "sweep plan");
+  h.paux = h.upload(paux, stream, "sweep loop statements");
   h.chunk = h.upload(chunks, stream, "sweep chunks");
   h.lrec = h.upload(lrec, stream, "sweep lanes");
   h.lmeta = h.upload(lmeta, stream, "sweep lane meta");
@@ -1144,7 +1171,7 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
   w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
   w.issue = d_issue; w.retire = d_retire;
   w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
-  w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring; w.lflag = h->lflag;
+  w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring; w.lflag = h->lflag; w.paux = h->paux;
   w.dep = a.dep; w.ddep = a.ddep; w.path = a.path; w.ord = a.ord;
   w.chk_counts = a.chk_counts; w.chk_first = a.chk_first;
   const bool barrier = variant == SYNC_SIM_BARRIER;

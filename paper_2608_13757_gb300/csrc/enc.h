@@ -231,6 +231,8 @@ struct SweepArgs {
   int32_t frame_depth;
   int32_t ring;              // latest increments kept per semaphore (power of two)
   const int32_t* lflag;      // per loop: 1 if it carries no offset > 0 (trip register elidable)
+  const int4* paux;          // per plan item (loop statements): {child rowptr offset lo, hi,
+                             // chunk of its whole body barrier-free, barrier} (-1: none)
   // fused simulation (thresholds from the walk's loop state, no threshold
   // array): dep is set (NULL otherwise) and thr is unused
   const DepInfo* dep;

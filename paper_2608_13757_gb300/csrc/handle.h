@@ -32,6 +32,7 @@ struct sync_programs {
   syncgb::DepInfo* dep = nullptr;
   int32_t* ddep = nullptr;          // per consumer-grouped dependency: dependency id
   int32_t* lflag = nullptr;         // per loop: trip register elidable
+  int4* paux = nullptr;             // per sweep plan item: loop-statement side record
   int64_t* seg = nullptr;
   int32_t* tile_first = nullptr;
   int64_t* path = nullptr;

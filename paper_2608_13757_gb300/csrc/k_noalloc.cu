@@ -103,7 +103,7 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
   w.makespan = d_makespan; w.checksum = d_checksum; w.status = d_status;
   w.issue = d_issue; w.retire = d_retire;
   w.prm = q; w.n_programs = h->sz.n_programs; w.mode = mode;
-  w.sem_cap = sem_cap; w.frame_depth = frame_depth; w.ring = ring; w.lflag = h->lflag;
+  w.sem_cap = sem_cap; w.frame_depth = frame_depth; w.ring = ring; w.lflag = h->lflag; w.paux = h->paux;
   st = cuda_error(launch_sweep(w, barrier, h->num_sms, s), "sweep simulator kernel");
   if (st != SYNC_OK) return st;
   SimArgs a;

@@ -751,25 +751,25 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
           if (lane < pi.ne) S.t[lane] += stmt_cost_of(it.z);
         }
         const int32_t child_ic = iter_cost_of(it.z);
-        const LoopInfo L = a.loop[it.y];
-        const int32_t lo = __ldg(a.rowptr + L.rowptr_off + g), hi = __ldg(a.rowptr + L.rowptr_off + g + 1);
+        // the statement's side record: the child's trip prefix sums, and the
+        // chunk holding its whole body (if one does), fetched together
+        const int4 ax = __ldg(a.paux + pbeg + item);
+        const int64_t rp = (int64_t)(((uint64_t)(uint32_t)ax.y << 32) | (uint32_t)ax.x);
+        const int32_t lo = __ldg(a.rowptr + rp + g), hi = __ldg(a.rowptr + rp + g + 1);
+        const int32_t body_chunk = BB ? ax.w : ax.z;
         ++item;
         if (lo < hi) {
-          const int32_t cb = __ldg(a.plan_ptr + it.y), ce = __ldg(a.plan_ptr + it.y + 1);
           __syncwarp();
           if (lane < pi.ne) S.t[lane] += child_ic;    // the first iteration starts
           __syncwarp();
-          if (ce - cb == 1) {
-            const int4 body = __ldg(a.plan + cb);
-            const bool multi = !BB && body.w >= 0;
-            if (body.x == ITEM_SEG && (multi || body.z == 1)) {
-              // a loop around one chunk: all its iterations in registers
-              verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + (multi ? body.w : body.y)), lo,
-                                                      hi, ++ctag, lane, sp + 1, child_ic, chk);
-              if (verdict) break;
-              continue;
-            }
+          if (body_chunk >= 0) {
+            // a loop around one chunk: all its iterations in registers
+            verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + body_chunk), lo, hi, ++ctag, lane,
+                                                    sp + 1, child_ic, chk);
+            if (verdict) break;
+            continue;
           }
+          const int32_t cb = __ldg(a.plan_ptr + it.y), ce = __ldg(a.plan_ptr + it.y + 1);
           if (lane == 0) S.frames[sp] = Frame{loop, item, g, g_end};
           ++sp;
           if (FUSED && lane == 0) S.lvl[sp] = make_int2(lo, lo);
