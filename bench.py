@@ -326,9 +326,16 @@ def cpu_baseline(config, sample, mode_name):
     with ThreadPoolExecutor(max_workers=cores) as ex:
         pairs = sum(ex.map(work, batches))
     dt = time.perf_counter() - t0
+    # one core on the first 1/64 of the sample (at least one program)
+    one = workloads.generate(config, n_programs=max(1, sample // 64))
+    t1 = time.perf_counter()
+    pairs1 = work(one)
+    dt1 = time.perf_counter() - t1
     return {"value": pairs / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "single_core_value": pairs1 / dt1,
             "sample": f"programs 0..{sample - 1} of the {config} workload ({pairs} pairs), "
-                      f"thresholds + check + barrier-free and barrier simulation, {dt:.2f} s wall"}
+                      f"thresholds + check + barrier-free and barrier simulation, {dt:.2f} s wall; "
+                      f"single core: programs 0..{max(1, sample // 64) - 1} ({pairs1} pairs), {dt1:.2f} s"}
 
 
 def run_reference(args, rank, world):
