@@ -228,9 +228,31 @@ def run_gpu(args, rank, world, local_rank):
     return out
 
 
-def run_e2e(args, sg, batch, mode, prm, dev, P):
-    """The same step through the public API from host arrays: load (host to
-    device copies), the four kernels, and the results read back to the host."""
+def launch_step(sg, h, mode, prm, fused, bufs=None):
+    """Enqueues one step's kernels on the current stream and the read-back of
+    its results into pinned host buffers; returns (buffers, device tensors
+    to keep alive until the stream has run them)."""
+    import torch
+    if fused:
+        thr = None
+        r1, counts, fb = sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER_FREE, check=True)
+        r2 = sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER)
+    else:
+        thr = sg.sync_eval_thresholds(h, mode)
+        counts, fb = sg.sync_check_minimal(h, mode, thr)
+        r1 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE)
+        r2 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER)
+    res = [counts, fb, r1.makespan, r1.checksum, r1.status, r2.makespan, r2.checksum, r2.status]
+    if bufs is None:
+        bufs = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in res]
+    for b, x in zip(bufs, res):
+        b.copy_(x, non_blocking=True)
+    return bufs, (thr, res)
+
+
+def e2e_serial(args, sg, batch, mode, prm, dev):
+    """One step at a time: load (host encoding + host-to-device copies), the
+    four kernels, the results read back, the device idle meanwhile."""
     import torch
     steps = max(1, min(args.steps, 3))
     times, h2d, d2h = [], 0, 0
@@ -238,17 +260,7 @@ def run_e2e(args, sg, batch, mode, prm, dev, P):
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         h = sg.sync_load_programs(batch, device=dev.index)
-        if args.pipeline == "fused":
-            thr = None
-            r1, counts, fb = sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER_FREE, check=True)
-            r2 = sg.sync_simulate_fused(h, mode, prm, sg.SIM_BARRIER)
-        else:
-            thr = sg.sync_eval_thresholds(h, mode)
-            counts, fb = sg.sync_check_minimal(h, mode, thr)
-            r1 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER_FREE)
-            r2 = sg.sync_simulate(h, mode, thr, prm, sg.SIM_BARRIER)
-        host = [t.cpu() for t in (counts, fb, r1.makespan, r1.checksum, r1.status,
-                                  r2.makespan, r2.checksum, r2.status)]
+        host, keep = launch_step(sg, h, mode, prm, args.pipeline == "fused")
         torch.cuda.synchronize()
         t1 = time.perf_counter()
         if i > 0:
@@ -256,8 +268,57 @@ def run_e2e(args, sg, batch, mode, prm, dev, P):
         h2d = h.sizes.h2d_bytes
         d2h = sum(x.numel() * x.element_size() for x in host)
         h.close()
-        del thr
+        del keep
     return {"s": statistics.median(times), "h2d": int(h2d), "d2h": int(d2h)}
+
+
+def e2e_pipelined(args, sg, batch, mode, prm, dev, steps, bufs):
+    """K steps as a stream of batches: the host builds and copies step i+1's
+    encoding on a second stream while the device runs step i's kernels and
+    read-back; the time runs from the first load to the last result on the
+    host (pipeline fill and drain included).  Handles are released after
+    the last step."""
+    import torch
+    load_stream = torch.cuda.Stream(device=dev)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    handles, keeps = [], []
+    h = sg.sync_load_programs(batch, device=dev.index, stream=load_stream)
+    for i in range(steps):
+        handles.append(h)
+        host, keep = launch_step(sg, h, mode, prm, args.pipeline == "fused", bufs[i])
+        keeps.append(keep)
+        if i + 1 < steps:
+            h = sg.sync_load_programs(batch, device=dev.index, stream=load_stream)
+    torch.cuda.synchronize()
+    t1 = time.perf_counter()
+    for x in handles:
+        x.close()
+    return (t1 - t0) / steps, handles[0].sizes.h2d_bytes
+
+
+def run_e2e(args, sg, batch, mode, prm, dev, P):
+    """The same step through the public API from host arrays: load (host to
+    device copies), the four kernels, and the results read back to the host;
+    steps pipelined (host build of the next batch beside the device's work
+    on this one), and one at a time for comparison."""
+    import torch
+    serial = e2e_serial(args, sg, batch, mode, prm, dev)
+    steps = max(4, args.steps)
+    # pinned result buffers per step, allocated before the timed region
+    h = sg.sync_load_programs(batch, device=dev.index)
+    bufs = []
+    for _ in range(steps):
+        b, keep = launch_step(sg, h, mode, prm, args.pipeline == "fused")
+        bufs.append(b)
+    torch.cuda.synchronize()
+    h.close()
+    del keep
+    e2e_pipelined(args, sg, batch, mode, prm, dev, steps, bufs)          # warm-up (allocator)
+    s, h2d = e2e_pipelined(args, sg, batch, mode, prm, dev, steps, bufs)
+    ok = bool(int(bufs[-1][4].max()) == 0 and int(bufs[-1][7].max()) == 0 and int(bufs[-1][0].sum()) == 0)
+    d2h = sum(x.numel() * x.element_size() for x in bufs[-1])
+    return {"s": s, "h2d": int(h2d), "d2h": int(d2h), "steps": steps, "results_ok": ok, "serial_s": serial["s"]}
 
 
 def shard(rank: int, programs_per_rank: int):
@@ -420,7 +481,9 @@ def main():
     ms = res["ms"]
     pairs = res["sizes"].n_pairs
     e2e_s = res["e2e"]["s"] if "e2e" in res else None
+    serial_s = res["e2e"]["serial_s"] if "e2e" in res else None
     if world > 1:
+        _, serial_s, _ = reduce_over_ranks(ms, serial_s, pairs, "cuda")
         ms, e2e_s, total_pairs = reduce_over_ranks(ms, e2e_s, pairs, "cuda")
     else:
         total_pairs = float(pairs)
@@ -454,7 +517,11 @@ def main():
     }
     if e2e_s:
         line["e2e"] = {"value": total_pairs / e2e_s, "unit": UNIT,
-                       "h2d_bytes_per_step": res["e2e"]["h2d"], "d2h_bytes_per_step": res["e2e"]["d2h"]}
+                       "h2d_bytes_per_step": res["e2e"]["h2d"], "d2h_bytes_per_step": res["e2e"]["d2h"],
+                       "steps": res["e2e"]["steps"], "results_ok": res["e2e"]["results_ok"],
+                       "pipelined": "host encoding and copies of step i+1 on a second stream beside "
+                                    "the kernels and read-back of step i; fill and drain timed",
+                       "serial_value": total_pairs / serial_s if serial_s else None}
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.config, min(args.cpu_sample, res["P"]), args.mode)
     print(json.dumps(line), flush=True)

@@ -910,12 +910,14 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     }
   }
   // programs in descending order of simulated work
+  // (key = -work, program id): distinct pairs, so the order is total and
+  // equal work keeps program order
+  std::vector<std::pair<int64_t, int32_t>> by_work(P);
+  for (int32_t p = 0; p < P; ++p)
+    by_work[p] = {-(prog[p].n_inst + prog[p].n_pairs + (prog[p].n_stmt + prog[p].n_iter) * prog[p].ne), p};
+  std::sort(by_work.begin(), by_work.end());
   std::vector<int32_t> order(P);
-  for (int32_t p = 0; p < P; ++p) order[p] = p;
-  std::stable_sort(order.begin(), order.end(), [&](int32_t u, int32_t v) {
-    auto w = [&](int32_t q) { return prog[q].n_inst + prog[q].n_pairs + (prog[q].n_stmt + prog[q].n_iter) * prog[q].ne; };
-    return w(u) > w(v);
-  });
+  for (int32_t p = 0; p < P; ++p) order[p] = by_work[p].second;
 
   h.sz.n_pairs = n_pairs;
   h.sz.n_pairs_padded = n_pairs_padded;
