@@ -143,11 +143,11 @@ struct Part {
   std::vector<uint8_t> path_kind;          // per path entry: 0 parent-index offset, 1 rowptr offset
   std::vector<int32_t> op_ptr, opstop;
   std::vector<int2> rowinfo;
-  std::vector<int4> ops, opsem[kModes];
+  std::vector<int4> ops;
   std::vector<int64_t> semhb;
   std::vector<uint8_t> semhb_mode;         // per semaphore base: its mode (history space)
   std::vector<int32_t> plan_ptr;
-  std::vector<int4> plan, paux, chunks, lrec, lmeta, lsem[kModes];
+  std::vector<int4> plan, paux, chunks, lrec, lmeta;
   std::vector<LoopInfo> xloops;
   std::vector<uint8_t> reads_rowptr;
   std::vector<DeriveJob> jobs;
@@ -158,26 +158,25 @@ struct Part {
   std::exception_ptr error;
 };
 
-// Appends one sweep chunk: lanes `recs` (program-local instructions, already
-// engine-major) with their iteration copies.
-void add_chunk(const sync_batch_desc& d, int32_t x0, const ProgScratch& S, const std::vector<int32_t>& recs,
-               const std::vector<int32_t>& copies, int32_t ncopies, std::vector<int4>& chunks,
-               std::vector<int4>& lrec, std::vector<int4>& lmeta, std::vector<int4> (&lsem)[kModes]) {
+// Appends one sweep chunk: n <= 32 lanes `recs` (program-local
+// instructions, already engine-major) with their iteration copies (nullptr:
+// all copy 0).
+void add_chunk(const sync_batch_desc& d, int32_t x0, const ProgScratch& S, const int32_t* recs,
+               const int32_t* copies, int32_t n, int32_t ncopies, std::vector<int4>& chunks,
+               std::vector<int4>& lrec, std::vector<int4>& lmeta) {
   const int32_t base = (int32_t)lrec.size();
-  const int32_t n = (int32_t)recs.size();
-  int32_t emask = 0;
+  int32_t eng[32];
+  for (int32_t i = 0; i < n; ++i) eng[i] = d.instr_engine[x0 + recs[i]];
+  int32_t emask = 0, head = 0;
   for (int32_t i = 0; i < n; ++i) {
-    const int32_t x = recs[i];
-    const int32_t e = d.instr_engine[x0 + x];
+    const int32_t x = recs[i], e = eng[i];
+    const int32_t c = copies ? copies[i] : 0;
     emask |= 1 << e;
-    int32_t head = i;
-    while (head > 0 && d.instr_engine[x0 + recs[head - 1]] == e) --head;
-    const bool last = i + 1 == n || d.instr_engine[x0 + recs[i + 1]] != e;
-    const bool first_in_copy = copies[i] > 0 && (i == head || copies[i - 1] != copies[i]);
+    if (i > 0 && eng[i - 1] != e) head = i;          // first lane of the engine's run
+    const bool last = i + 1 == n || eng[i + 1] != e;
+    const bool first_in_copy = c > 0 && (i == head || copies[i - 1] != c);
     lrec.push_back(make_int4(x0 + x, d.instr_latency[x0 + x], S.x_ndeps[x], S.x_dep_begin[x]));
-    lmeta.push_back(make_int4(e, copies[i], head, (first_in_copy ? LANE_ITER_START : 0) | (last ? LANE_RUN_LAST : 0)));
-    for (int m = 0; m < kModes; ++m)
-      lsem[m].push_back(make_int4(S.x_own[m][x], S.x_hstride[m][x], S.x_koff[m][x], m == 2 ? S.x_levels[x] : 0));
+    lmeta.push_back(make_int4(e, c, head, (first_in_copy ? LANE_ITER_START : 0) | (last ? LANE_RUN_LAST : 0)));
   }
   chunks.push_back(make_int4(base, n, ncopies, emask));
 }
@@ -227,17 +226,20 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   // per dependency, for the simulator's semaphore numbering
   std::vector<int32_t> dep_N(ND), dep_K(ND);
   std::vector<int32_t> lflag(NL, 0);       // per loop: carries no offset > 0 (trip register elidable)
+  // per mode and instruction: {own semaphore or -1, history stride, offset,
+  // per-engine wait levels}, gathered on the device into the op and lane
+  // records that name the instruction
+  HostVec<int4> xsem((size_t)kModes * NX);
 
   // Programs [p_begin, p_end) into `part`; erow0: their first per-engine row.
   auto run_block = [&d, div, &loop, &dep, &prog, &inst_off, &dseg, &ddep, &dsem, &seg, &ord_off, &dep_N,
-                    &dep_K, &lflag](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
+                    &dep_K, &lflag, &xsem, NX](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
   auto& rowptr_host = part.rowptr_host;
   auto& path = part.path;
   auto& op_ptr = part.op_ptr;
   auto& opstop = part.opstop;
   auto& rowinfo = part.rowinfo;
   auto& ops = part.ops;
-  auto& opsem = part.opsem;
   auto& semhb = part.semhb;
   auto& plan_ptr = part.plan_ptr;
   auto& plan = part.plan;
@@ -245,7 +247,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   auto& chunks = part.chunks;
   auto& lrec = part.lrec;
   auto& lmeta = part.lmeta;
-  auto& lsem = part.lsem;
   auto& xloops = part.xloops;
   auto& reads_rowptr = part.reads_rowptr;
   auto& jobs = part.jobs;
@@ -570,9 +571,12 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         const int32_t l = d.instr_loop[x0 + x];
         const int32_t s = sem_of[sem_key(m, x)];
         S.x_own[m][x] = s;
-        if (s < 0) continue;
-        S.x_hstride[m][x] = m == 0 ? 1 : m == 1 ? S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]] : -1;
-        S.x_koff[m][x] = m == 0 ? 1 : m == 1 ? S.rank[x] : 0;
+        if (s >= 0) {
+          S.x_hstride[m][x] = m == 0 ? 1 : m == 1 ? S.nloop_eng[(size_t)l * ne + d.instr_engine[x0 + x]] : -1;
+          S.x_koff[m][x] = m == 0 ? 1 : m == 1 ? S.rank[x] : 0;
+        }
+        xsem[(size_t)m * NX + x0 + x] =
+            make_int4(s, S.x_hstride[m][x], S.x_koff[m][x], m == 2 ? S.x_levels[x] : 0);
       }
       // dependencies grouped by consumer (stable by dependency id)
       if (m == 0)
@@ -601,18 +605,13 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
             const int64_t rp = space(m, e).rowptr_off;
             ops.push_back(make_int4(OP_LOOP, pi.le_base + m * ne, (int32_t)(uint32_t)(rp & 0xffffffffu),
                                     (int32_t)(rp >> 32)));
-            for (int m = 0; m < kModes; ++m) opsem[m].push_back(make_int4(-1, 0, 0, 0));
             has_loop = true;
           } else if (d.instr_engine[x0 + it] == e) {
             ops.push_back(make_int4(x0 + it, d.instr_latency[x0 + it], S.x_ndeps[it], S.x_dep_begin[it]));
-            for (int m = 0; m < kModes; ++m)
-              opsem[m].push_back(make_int4(S.x_own[m][it], S.x_hstride[m][it], S.x_koff[m][it],
-                                           m == 2 ? S.x_levels[it] : 0));
           }
         }
         const int32_t end_idx = (int32_t)ops.size();
         ops.push_back(make_int4(OP_END, 0, 0, 0));
-        for (int m = 0; m < kModes; ++m) opsem[m].push_back(make_int4(-1, 0, 0, 0));
         rowinfo.push_back(make_int2(end_idx, (has_loop ? 1 : 0) | (lflag[l0 + l] ? 2 : 0)));
         // next LOOP or END record at or after each record of the row
         opstop.resize(ops.size());
@@ -627,26 +626,27 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     const size_t plan_first_loop = plan_ptr.size(), plan_first_item = plan.size();
     for (int32_t l = 0; l < nl; ++l) {
       plan_ptr.push_back((int32_t)plan.size());
-      std::vector<int32_t> seg;
-      int32_t nseg = 0, nloops = 0;
+      int32_t seg0 = S.body_ptr[l], nseg = 0, nloops = 0;   // current segment: body[seg0 .. i)
       for (int32_t i = S.body_ptr[l]; i <= S.body_ptr[l + 1]; ++i) {
         const bool at_end = i == S.body_ptr[l + 1];
         const int32_t it = at_end ? -1 : S.body[i];
-        if (!at_end && it >= 0) { seg.push_back(it); continue; }
-        if (!seg.empty()) {
+        if (!at_end && it >= 0) continue;
+        if (i > seg0) {
           ++nseg;
           const int32_t first_chunk = (int32_t)chunks.size();
-          for (size_t b = 0; b < seg.size(); b += 32) {
-            std::vector<int32_t> piece(seg.begin() + b, seg.begin() + std::min(seg.size(), b + 32));
-            std::stable_sort(piece.begin(), piece.end(), [&](int32_t u, int32_t v) {
-              return d.instr_engine[x0 + u] < d.instr_engine[x0 + v];
-            });
-            std::vector<int32_t> copy0(piece.size(), 0);
-            add_chunk(d, x0, S, piece, copy0, 1, chunks, lrec, lmeta, lsem);
+          for (int32_t b = seg0; b < i; b += 32) {
+            // up to 32 records, engine-major and in body order within an
+            // engine (a counting sort by engine)
+            const int32_t n = std::min<int32_t>(32, i - b);
+            int32_t cnt[33] = {0}, piece[32];
+            for (int32_t j = 0; j < n; ++j) ++cnt[d.instr_engine[x0 + S.body[b + j]] + 1];
+            for (int32_t e = 0; e < ne; ++e) cnt[e + 1] += cnt[e];
+            for (int32_t j = 0; j < n; ++j) piece[cnt[d.instr_engine[x0 + S.body[b + j]]]++] = S.body[b + j];
+            add_chunk(d, x0, S, piece, nullptr, n, 1, chunks, lrec, lmeta);
           }
           plan.push_back(make_int4(ITEM_SEG, first_chunk, (int32_t)chunks.size() - first_chunk, -1));
-          seg.clear();
         }
+        seg0 = i + 1;
         if (!at_end) {
           ++nloops;
           plan.push_back(make_int4(ITEM_LOOP, l0 + (-it - 1), lflag[l0 + (-it - 1)], 0));
@@ -656,13 +656,13 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       const int32_t L = S.body_ptr[l + 1] - S.body_ptr[l];
       if (nloops == 0 && nseg == 1 && L >= 1 && L <= 16) {
         const int32_t k = 32 / L;
-        std::vector<int32_t> recs, copies;
+        int32_t recs[32], copies[32], n = 0;
         for (int32_t e = 0; e < ne; ++e)
           for (int32_t c = 0; c < k; ++c)
             for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i)
-              if (d.instr_engine[x0 + S.body[i]] == e) { recs.push_back(S.body[i]); copies.push_back(c); }
+              if (d.instr_engine[x0 + S.body[i]] == e) { recs[n] = S.body[i]; copies[n++] = c; }
         plan.back().w = (int32_t)chunks.size();
-        add_chunk(d, x0, S, recs, copies, k, chunks, lrec, lmeta, lsem);
+        add_chunk(d, x0, S, recs, copies, n, k, chunks, lrec, lmeta);
       }
     }
     // per loop statement, what the walker needs without further lookups:
@@ -760,11 +760,10 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   HostVec<int64_t> path(all.path);
   HostVec<int32_t> op_ptr(all.rows), opstop(all.opstop);
   HostVec<int2> rowinfo(all.rows);
-  HostVec<int4> ops(all.ops), opsem(kModes * all.ops);    // opsem: mode-major
+  HostVec<int4> ops(all.ops);
   HostVec<int64_t> semhb(all.semhb);
   HostVec<int32_t> plan_ptr(NL);             // one entry per loop; the blocks own consecutive loops
   HostVec<int4> plan(all.plan), paux(all.plan), chunks(all.chunks), lrec(all.lanes), lmeta(all.lanes);
-  HostVec<int4> lsem(kModes * all.lanes);                  // mode-major
   HostVec<LoopInfo> xloops(all.xloops);
   HostVec<uint8_t> reads_rowptr(all.xloops);
   HostVec<DeriveJob> jobs(all.jobs);
@@ -817,10 +816,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         v = make_int4(OP_LOOP, v.y + b_rows, (int32_t)(uint32_t)(rp & 0xffffffffu), (int32_t)(rp >> 32));
       }
       ops[B.ops + i] = v;
-    }
-    for (int m = 0; m < kModes; ++m) {
-      std::copy(pt.opsem[m].begin(), pt.opsem[m].end(), opsem.begin() + m * all.ops + B.ops);
-      std::copy(pt.lsem[m].begin(), pt.lsem[m].end(), lsem.begin() + m * all.lanes + B.lanes);
     }
     for (size_t i = 0; i < pt.semhb.size(); ++i) semhb[B.semhb + i] = pt.semhb[i] + B.hist[pt.semhb_mode[i]];
     const int32_t l_first = d.prog_loop_ptr[cut[t]];
@@ -964,7 +959,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.rowinfo = h.upload(rowinfo, stream, "row info");
   h.ops = h.upload(ops, stream, "op records");
   h.opstop = h.upload(opstop, stream, "op stops");
-  h.opsem = h.upload(opsem, stream, "op semaphore records");
+  h.opsem = h.alloc<int4>(kModes * (int64_t)ops.size(), "op semaphore records");
   {
     std::vector<int32_t> dboth(dsem[0]);
     for (int m = 1; m < kModes; ++m) dboth.insert(dboth.end(), dsem[m].begin(), dsem[m].end());
@@ -986,11 +981,14 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.chunk = h.upload(chunks, stream, "sweep chunks");
   h.lrec = h.upload(lrec, stream, "sweep lanes");
   h.lmeta = h.upload(lmeta, stream, "sweep lane meta");
-  h.lsem = h.upload(lsem, stream, "sweep lane semaphores");
+  h.lsem = h.alloc<int4>(kModes * (int64_t)lrec.size(), "sweep lane semaphores");
+  const int4* d_xsem = h.upload(xsem, stream, "instruction semaphore records");
   h.n_lanes = (int64_t)lrec.size();
   LoopInfo* d_xloops = h.upload(xloops, stream, "iteration spaces");
   h.divergent = div;
   cuda_check(launch_expand(d_xloops, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
+  cuda_check(launch_sem_records(d_xsem, NX, h.ops, h.n_ops, h.lrec, h.n_lanes, h.opsem, h.lsem, h.num_sms, stream),
+             "semaphore records");
   cuda_check(launch_derive(d_jobs, d_tile_job, h.rowptr, h.pidx, h.path, h.derived, n_derived, h.num_sms, stream),
              "derive");
   cuda_check(cudaStreamSynchronize(stream), "load");

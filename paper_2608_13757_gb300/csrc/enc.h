@@ -248,6 +248,13 @@ struct SweepArgs {
 // with pidx_off[l] <= t*kTilePairs), with one extra entry n_loops-1.
 cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const int32_t* rowptr,
                           int32_t* pidx, int64_t n_iters, int num_sms, cudaStream_t s);
+// Semaphore records of the op rows and sweep lanes, per threshold mode,
+// gathered from the per-instruction table xsem[m * n_instrs + x] by the
+// record's global instruction x (LOOP and END op records: {-1, 0, 0, 0}):
+// opsem[m * n_ops + r], lsem[m * n_lanes + i].
+cudaError_t launch_sem_records(const int4* xsem, int64_t n_instrs, const int4* ops, int64_t n_ops,
+                               const int4* lrec, int64_t n_lanes, int4* opsem, int4* lsem, int num_sms,
+                               cudaStream_t s);
 // tile_job[t] = job whose output holds pool entry t*kTilePairs.
 cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
                           const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,

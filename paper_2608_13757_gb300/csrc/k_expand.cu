@@ -36,6 +36,25 @@ k_expand(const LoopInfo* __restrict__ loop, const int32_t* __restrict__ tile_loo
   }
 }
 
+// One thread per (mode, op record or lane): the record's semaphore entry
+// copied from its instruction's.
+__global__ void __launch_bounds__(kThreads)
+k_sem_records(const int4* __restrict__ xsem, int64_t n_instrs, const int4* __restrict__ ops, int64_t n_ops,
+              const int4* __restrict__ lrec, int64_t n_lanes, int4* __restrict__ opsem, int4* __restrict__ lsem) {
+  const int64_t per = n_ops + n_lanes, n = kModes * per;
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < n; q += stride) {
+    const int64_t m = q / per, r = q - m * per;
+    if (r < n_ops) {
+      const int32_t x = ops[r].x;
+      opsem[m * n_ops + r] = x >= 0 ? xsem[m * n_instrs + x] : make_int4(-1, 0, 0, 0);
+    } else {
+      const int64_t i = r - n_ops;
+      lsem[m * n_lanes + i] = xsem[m * n_instrs + lrec[i].x];
+    }
+  }
+}
+
 // One thread per derived entry; the job is found inside the range the
 // host's tile table gives.
 __global__ void __launch_bounds__(kThreads)
@@ -136,6 +155,18 @@ cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const 
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
   k_derive<<<grid, kThreads, 0, s>>>(jobs, tile_job, rowptr, pidx, path, derived, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sem_records(const int4* xsem, int64_t n_instrs, const int4* ops, int64_t n_ops,
+                               const int4* lrec, int64_t n_lanes, int4* opsem, int4* lsem, int num_sms,
+                               cudaStream_t s) {
+  const int64_t n = kModes * (n_ops + n_lanes);
+  if (n == 0) return cudaSuccess;
+  const int64_t want = (n + kThreads - 1) / kThreads;
+  const int64_t cap = (int64_t)num_sms * 8;
+  const int grid = (int)(want < cap ? want : cap);
+  k_sem_records<<<grid, kThreads, 0, s>>>(xsem, n_instrs, ops, n_ops, lrec, n_lanes, opsem, lsem);
   return cudaGetLastError();
 }
 
