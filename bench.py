@@ -304,7 +304,7 @@ def run_e2e(args, sg, batch, mode, prm, dev, P):
     on this one), and one at a time for comparison."""
     import torch
     serial = e2e_serial(args, sg, batch, mode, prm, dev)
-    steps = max(4, args.steps)
+    steps = max(8, args.steps)
     # pinned result buffers per step, allocated before the timed region
     h = sg.sync_load_programs(batch, device=dev.index)
     bufs = []

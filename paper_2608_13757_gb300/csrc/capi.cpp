@@ -114,24 +114,10 @@ struct ProgScratch {
   std::vector<int64_t> tstart_of;                 // derived trip-start array per loop (and engine), -1 if none
   std::vector<uint8_t> needs_rhat;                // per loop: carries a dependency with offset > 0
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
+  std::vector<int32_t> by_cons, cons_next, sem_of;  // dependencies by consumer; semaphore per key
+  std::vector<int64_t> inst_eng, sem_hist;        // instances per engine; history bases of one mode
 };
 
-// Host arrays that are filled right after allocation: default-initialised,
-// so allocating one does not write it first.
-template <class T>
-struct NoInit : std::allocator<T> {
-  template <class U>
-  struct rebind { using other = NoInit<U>; };
-  NoInit() = default;
-  template <class U>
-  NoInit(const NoInit<U>&) {}
-  template <class U>
-  void construct(U* p) { ::new (static_cast<void*>(p)) U; }
-  template <class U, class... A>
-  void construct(U* p, A&&... a) { ::new (static_cast<void*>(p)) U(std::forward<A>(a)...); }
-};
-template <class T>
-using HostVec = std::vector<T, NoInit<T>>;
 
 // What the per-program pass appends, for one block of consecutive programs.
 // Offsets recorded in it (into the rowptr, parent-index, pair, derived,
@@ -215,17 +201,18 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   // ------------------------------------ per-program validation and tables
   // Indexed by global loop / dependency / program / instruction id: written
   // by the block that owns the id (offsets block-relative until the join).
-  std::vector<LoopInfo> loop(NL);
-  std::vector<DepInfo> dep(ND);
-  std::vector<ProgInfo> prog(P);
-  std::vector<int64_t> inst_off(NX), dseg(ND);
-  std::vector<int32_t> ddep(ND);
-  std::vector<int32_t> dsem[kModes] = {std::vector<int32_t>(ND), std::vector<int32_t>(ND), std::vector<int32_t>(ND)};
-  std::vector<int64_t> seg(ND + 1, 0);
-  std::vector<int64_t> ord_off(NX, -1);   // per instruction: ordinal pool offset (waited producers)
+  HostVec<LoopInfo> loop(NL);
+  HostVec<DepInfo> dep(ND);
+  HostVec<ProgInfo> prog(P);
+  HostVec<int64_t> inst_off(NX), dseg(ND);
+  HostVec<int32_t> ddep(ND);
+  HostVec<int32_t> dsem((size_t)kModes * ND);   // [kModes][n_deps]
+  HostVec<int64_t> seg(ND + 1);
+  HostVec<int64_t> ord_off(NX);   // per instruction: ordinal pool offset (waited producers) or -1
   // per dependency, for the simulator's semaphore numbering
-  std::vector<int32_t> dep_N(ND), dep_K(ND);
-  std::vector<int32_t> lflag(NL, 0);       // per loop: carries no offset > 0 (trip register elidable)
+  HostVec<int32_t> dep_N(ND), dep_K(ND);
+  HostVec<int32_t> dep_count(ND);          // consumer instances per dependency (host copy)
+  HostVec<int32_t> lflag(NL);              // per loop: carries no offset > 0 (trip register elidable)
   // per mode and instruction: {own semaphore or -1, history stride, offset,
   // per-engine wait levels}, gathered on the device into the op and lane
   // records that name the instruction
@@ -233,7 +220,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
 
   // Programs [p_begin, p_end) into `part`; erow0: their first per-engine row.
   auto run_block = [&d, div, &loop, &dep, &prog, &inst_off, &dseg, &ddep, &dsem, &seg, &ord_off, &dep_N,
-                    &dep_K, &lflag, &xsem, NX](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
+                    &dep_K, &lflag, &xsem, &dep_count, NX, ND](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
   auto& rowptr_host = part.rowptr_host;
   auto& path = part.path;
   auto& op_ptr = part.op_ptr;
@@ -267,6 +254,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     const int32_t nl = d.prog_loop_ptr[p + 1] - l0, nx = d.prog_instr_ptr[p + 1] - x0,
                   nd = d.prog_dep_ptr[p + 1] - d0;
     const int32_t ne = d.prog_n_engines[p];
+    std::fill(ord_off.begin() + x0, ord_off.begin() + x0 + nx, (int64_t)-1);
     if (nl < 1) raise(SYNC_ERR_MALFORMED, where(p, "has no top-level loop", 0));
     if (ne < 1 || ne > 32) raise(SYNC_ERR_MALFORMED, where(p, "n_engines", ne));
     const int32_t* par = d.loop_parent + l0;
@@ -363,7 +351,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     for (int32_t l = 0; l < nl; ++l) S.body_ptr[l + 1] += S.body_ptr[l];
     S.keys.resize(S.body_ptr[nl]);
     {
-      std::vector<int32_t> fill(S.body_ptr.begin(), S.body_ptr.end() - 1);
+      auto& fill = S.cons_next;                  // scratch: next free slot per body
+      fill.assign(S.body_ptr.begin(), S.body_ptr.end() - 1);
       for (int32_t x = 0; x < nx; ++x)
         S.keys[fill[d.instr_loop[x0 + x]]++] = ((int64_t)d.instr_pos[x0 + x] << 32) | (uint32_t)x;
       for (int32_t l = 1; l < nl; ++l)
@@ -403,7 +392,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     }
     pi.agg_lat = agg > (__int128)INT64_MAX ? INT64_MAX : (int64_t)agg;
     {
-      std::vector<int64_t> per_engine(ne, 0);
+      auto& per_engine = S.inst_eng;            // scratch: instances per engine
+      per_engine.assign(ne, 0);
       for (int32_t x = 0; x < nx; ++x)
         per_engine[d.instr_engine[x0 + x]] += tot(d.instr_loop[x0 + x], d.instr_engine[x0 + x]);
       for (int64_t c : per_engine) if (c > kI32Max) part.ord_overflow = true;
@@ -422,8 +412,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     for (int m = 0; m < kModes; ++m) { S.x_own[m].assign(nx, -1); S.x_hstride[m].assign(nx, 0); S.x_koff[m].assign(nx, 0); }
     S.x_levels.assign(nx, 0);
     // dependencies: innermost common loop S, cases of Sec. 5.2, N and K
-    std::vector<int32_t> by_cons(nd);
-    for (int32_t k = 0; k < nd; ++k) by_cons[k] = k;
     for (int32_t k = 0; k < nd; ++k) {
       const int64_t gd = d0 + k;
       const int32_t px = d.dep_prod[gd], cx = d.dep_cons[gd], off = d.dep_k[gd];
@@ -463,6 +451,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       DepInfo& D = dep[gd];
       std::memset(&D, 0, sizeof D);
       D.total = (int32_t)tot(Cl, ec);            // consumer instances, on its engine
+      dep_count[gd] = D.total;
       D.up = S.depth[Cl] - S.depth[Sl];
       D.clen = S.depth[Pl] - S.depth[Sl];
       D.kase = kase;
@@ -519,6 +508,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     }
     // loops whose trip register can be elided (Sec. 5.1: only offset-0
     // dependencies carried there, or none), and their control counts
+    lflag[l0] = 0;
     for (int32_t l = 1; l < nl; ++l) {
       lflag[l0 + l] = S.needs_rhat[l] ? 0 : 1;
       if (S.needs_rhat[l]) continue;
@@ -532,7 +522,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     // iteration); mode 1 = one per (loop, engine) (N increments per
     // iteration); mode 2 = one per engine (one increment per instance of the
     // engine, numbered by the instance's ordinal)
-    std::vector<int64_t> inst_eng(ne, 0);
+    auto& inst_eng = S.inst_eng;
+    inst_eng.assign(ne, 0);
     for (int32_t x = 0; x < nx; ++x)
       inst_eng[d.instr_engine[x0 + x]] += tot(d.instr_loop[x0 + x], d.instr_engine[x0 + x]);
     auto sem_key = [&](int m, int32_t x) {
@@ -547,10 +538,25 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       pi.pair_levels += (int64_t)levels(d.dep_prod[gd]) *
                         tot(d.instr_loop[x0 + d.dep_cons[gd]], d.instr_engine[x0 + d.dep_cons[gd]]);
     }
-    std::vector<int32_t> sem_of(std::max(nx, nl * ne), -1);
+    // dependencies grouped by consumer, stable by dependency id (a counting
+    // sort); a consumer's dependencies start at x_dep_begin (d0 if none)
+    auto& by_cons = S.by_cons;
+    by_cons.resize(nd);
+    auto& next = S.cons_next;
+    next.resize(nx);
+    for (int32_t k = 0; k < nd; ++k) S.x_ndeps[d.dep_cons[d0 + k]]++;
+    for (int32_t x = 0, at = 0; x < nx; ++x) {
+      if (S.x_ndeps[x] > 0) S.x_dep_begin[x] = d0 + at;
+      next[x] = at;
+      at += S.x_ndeps[x];
+    }
+    for (int32_t k = 0; k < nd; ++k) by_cons[next[d.dep_cons[d0 + k]]++] = k;
+    auto& sem_of = S.sem_of;
+    auto& sem_hist = S.sem_hist;
+    sem_of.resize(std::max(nx, nl * ne));
     for (int m = 0; m < kModes; ++m) {
       std::fill(sem_of.begin(), sem_of.end(), -1);
-      std::vector<int64_t> sem_hist;
+      sem_hist.clear();
       for (int32_t k = 0; k < nd; ++k) {
         const int64_t gd = d0 + k;
         const int32_t px = d.dep_prod[gd];
@@ -578,19 +584,12 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         xsem[(size_t)m * NX + x0 + x] =
             make_int4(s, S.x_hstride[m][x], S.x_koff[m][x], m == 2 ? S.x_levels[x] : 0);
       }
-      // dependencies grouped by consumer (stable by dependency id)
-      if (m == 0)
-        std::stable_sort(by_cons.begin(), by_cons.end(), [&](int32_t u, int32_t v) {
-          return d.dep_cons[d0 + u] < d.dep_cons[d0 + v];
-        });
       for (int32_t i = 0; i < nd; ++i) {
         const int64_t gd = d0 + by_cons[i];
-        dsem[m][d0 + i] = sem_of[sem_key(m, d.dep_prod[gd])];
+        dsem[(size_t)m * ND + d0 + i] = sem_of[sem_key(m, d.dep_prod[gd])];
         if (m == 0) { dseg[d0 + i] = seg[gd]; ddep[d0 + i] = (int32_t)gd; }
       }
     }
-    for (int32_t i = nd - 1; i >= 0; --i) S.x_dep_begin[d.dep_cons[d0 + by_cons[i]]] = d0 + i;
-    for (int32_t i = 0; i < nd; ++i) S.x_ndeps[d.dep_cons[d0 + by_cons[i]]]++;
     // per-(loop, engine) op records: own instructions and child loops in body
     // order, then an END record
     for (int32_t l = 0; l < nl; ++l)
@@ -872,47 +871,61 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   plan_ptr.push_back((int32_t)plan.size());
   seg[ND] = n_pairs_padded;
 
-  // tile tables
-  const int64_t n_tiles = (n_pairs_padded + kTilePairs - 1) / kTilePairs;
-  std::vector<int32_t> tile_first(n_tiles + 1, ND > 0 ? (int32_t)(ND - 1) : 0);
-  {
-    int64_t di = 0;
-    for (int64_t t = 0; t < n_tiles; ++t) {
-      const int64_t q = t * kTilePairs;
-      while (di + 1 < ND && seg[di + 1] <= q) ++di;
-      tile_first[t] = (int32_t)di;
-    }
-  }
-  const int64_t n_jtiles = (n_derived + kTilePairs - 1) / kTilePairs;
-  std::vector<int32_t> tile_job(n_jtiles + 1, jobs.empty() ? 0 : (int32_t)(jobs.size() - 1));
-  {
-    int64_t ji = 0;
-    for (int64_t t = 0; t < n_jtiles; ++t) {
-      const int64_t q = t * kTilePairs;
-      while (ji + 1 < (int64_t)jobs.size() && jobs[ji + 1].out <= q) ++ji;
-      tile_job[t] = (int32_t)ji;
-    }
-  }
-  const int64_t NXL = (int64_t)xloops.size();
-  const int64_t n_itiles = (n_iters + kTilePairs - 1) / kTilePairs;
-  std::vector<int32_t> tile_loop(n_itiles + 1, NXL > 0 ? (int32_t)(NXL - 1) : 0);
-  {
-    int64_t li = 0;
-    for (int64_t t = 0; t < n_itiles; ++t) {
-      const int64_t q = t * kTilePairs;
-      while (li + 1 < NXL && xloops[li + 1].pidx_off <= q) ++li;
-      tile_loop[t] = (int32_t)li;
-    }
-  }
-  // programs in descending order of simulated work
-  // (key = -work, program id): distinct pairs, so the order is total and
-  // equal work keeps program order
-  std::vector<std::pair<int64_t, int32_t>> by_work(P);
-  for (int32_t p = 0; p < P; ++p)
-    by_work[p] = {-(prog[p].n_inst + prog[p].n_pairs + (prog[p].n_stmt + prog[p].n_iter) * prog[p].ne), p};
-  std::sort(by_work.begin(), by_work.end());
+  // tile tables: table[t] = largest i < n with start(i) <= t * kTilePairs
+  // (start nondecreasing), one extra entry n-1; all three in one pool of
+  // threads, each table cut into slices of about 256k steps
+  std::vector<std::thread> tile_pool;
+  struct JoinAll {
+    std::vector<std::thread>& v;
+    ~JoinAll() { for (auto& th : v) if (th.joinable()) th.join(); }
+  } tile_join{tile_pool};                      // also when something below throws
+  auto tile_table = [&tile_pool, n_threads](std::vector<int32_t>& table, int64_t n_tiles, int64_t n, auto start) {
+    table.assign(n_tiles + 1, n > 0 ? (int32_t)(n - 1) : 0);
+    if (n == 0) return;
+    auto fill = [&table, n, start](int64_t t0, int64_t t1) {
+      int64_t lo = 0, hi = n - 1;                // largest i with start(i) <= t0 * kTilePairs
+      while (lo < hi) {
+        const int64_t mid = (lo + hi + 1) / 2;
+        if (start(mid) <= t0 * kTilePairs) lo = mid; else hi = mid - 1;
+      }
+      for (int64_t t = t0, i = lo; t < t1; ++t) {
+        while (i + 1 < n && start(i + 1) <= t * kTilePairs) ++i;
+        table[t] = (int32_t)i;
+      }
+    };
+    const int64_t nt = std::max<int64_t>(1, std::min<int64_t>(n_threads, (n_tiles + n) / (1 << 18)));
+    for (int64_t k = 0; k < nt; ++k) tile_pool.emplace_back(fill, n_tiles * k / nt, n_tiles * (k + 1) / nt);
+  };
+  std::vector<int32_t> tile_first, tile_job, tile_loop;
+  tile_table(tile_first, (n_pairs_padded + kTilePairs - 1) / kTilePairs, ND, [&seg](int64_t i) { return seg[i]; });
+  tile_table(tile_job, (n_derived + kTilePairs - 1) / kTilePairs, (int64_t)jobs.size(),
+             [&jobs](int64_t i) { return jobs[i].out; });
+  tile_table(tile_loop, (n_iters + kTilePairs - 1) / kTilePairs, (int64_t)xloops.size(),
+             [&xloops](int64_t i) { return xloops[i].pidx_off; });
+  // programs in descending order of simulated work, equal work in program
+  // order: a stable least-significant-digit radix sort (11-bit digits) of
+  // the works' complements
   std::vector<int32_t> order(P);
-  for (int32_t p = 0; p < P; ++p) order[p] = by_work[p].second;
+  {
+    std::vector<uint64_t> key(P);
+    uint64_t all_bits = 0;
+    for (int32_t p = 0; p < P; ++p) {
+      const int64_t w = prog[p].n_inst + prog[p].n_pairs + (prog[p].n_stmt + prog[p].n_iter) * prog[p].ne;
+      key[p] = ~(uint64_t)w;                     // w >= 0: larger work, smaller key
+      order[p] = p;
+    }
+    for (int32_t p = 0; p < P; ++p) all_bits |= key[p] ^ key[0];   // the digits that differ somewhere
+    std::vector<int32_t> tmp(P);
+    for (int shift = 0; shift < 64; shift += 11) {
+      if (((all_bits >> shift) & 0x7ff) == 0) continue;
+      int32_t cnt[2049] = {0};
+      for (int32_t i = 0; i < P; ++i) ++cnt[((key[order[i]] >> shift) & 0x7ff) + 1];
+      for (int b = 0; b < 2048; ++b) cnt[b + 1] += cnt[b];
+      for (int32_t i = 0; i < P; ++i) tmp[cnt[(key[order[i]] >> shift) & 0x7ff]++] = order[i];
+      order.swap(tmp);
+    }
+  }
+  for (auto& th : tile_pool) th.join();      // the tables are read from here on
 
   h.sz.n_pairs = n_pairs;
   h.sz.n_pairs_padded = n_pairs_padded;
@@ -930,12 +943,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       if (reads_rowptr[l]) sb += 4 * ((int64_t)xloops[l].n_parent + 1);
     h.sz.struct_bytes = sb;
   }
-  h.seg_host = seg;
+  h.seg_host = std::move(seg);
   h.ord_off_host = std::move(ord_off);
   h.n_ord = n_ord;
   h.ord_overflow = ord_overflow;
-  h.count_host.resize(ND);
-  for (int64_t i = 0; i < ND; ++i) h.count_host[i] = dep[i].total;
+  h.count_host = std::move(dep_count);
   h.n_chunks = n_pairs_padded / kChunk;
 
   // ---------------------------------------------------------------- device
@@ -946,7 +958,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.rowptr = h.upload(rowptr_host, stream, "rowptr");
   h.pidx = h.alloc<int32_t>(n_iters, "parent indices");
   h.dep = h.upload(dep, stream, "dependency table");
-  h.seg = h.upload(seg, stream, "segment offsets");
+  h.seg = h.upload(h.seg_host, stream, "segment offsets");
   h.tile_first = h.upload(tile_first, stream, "tile table");
   h.path = h.upload(path, stream, "path pool");
   h.derived = h.alloc<int32_t>(n_derived, "derived trip starts and ancestors");
@@ -961,9 +973,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.opstop = h.upload(opstop, stream, "op stops");
   h.opsem = h.alloc<int4>(kModes * (int64_t)ops.size(), "op semaphore records");
   {
-    std::vector<int32_t> dboth(dsem[0]);
-    for (int m = 1; m < kModes; ++m) dboth.insert(dboth.end(), dsem[m].begin(), dsem[m].end());
-    h.dsem = h.upload(dboth, stream, "dependency semaphores");
+    h.dsem = h.upload(dsem, stream, "dependency semaphores");
   }
   h.n_ops = (int64_t)ops.size();
   h.dseg = h.upload(dseg, stream, "dependency segments");

@@ -8,6 +8,23 @@
 #include "enc.h"
 
 namespace syncgb {
+// Host arrays that are filled right after allocation: default-initialised,
+// so allocating one does not write it first.
+template <class T>
+struct NoInit : std::allocator<T> {
+  template <class U>
+  struct rebind { using other = NoInit<U>; };
+  NoInit() = default;
+  template <class U>
+  NoInit(const NoInit<U>&) {}
+  template <class U>
+  void construct(U* p) { ::new (static_cast<void*>(p)) U; }
+  template <class U, class... A>
+  void construct(U* p, A&&... a) { ::new (static_cast<void*>(p)) U(std::forward<A>(a)...); }
+};
+template <class T>
+using HostVec = std::vector<T, NoInit<T>>;
+
 // Throws the loader's failure for a CUDA error (caught at the C ABI).
 void cuda_or_raise(cudaError_t e, const char* what);
 // Sets the message sync_last_error() returns on this thread; returns status.
@@ -22,8 +39,8 @@ struct sync_programs {
   int device = 0;
   int num_sms = 0;
   sync_sizes sz{};
-  std::vector<int64_t> seg_host;
-  std::vector<int32_t> count_host;
+  syncgb::HostVec<int64_t> seg_host;
+  syncgb::HostVec<int32_t> count_host;
   std::vector<void*> blocks;
   // threshold / checker encoding
   syncgb::LoopInfo* loop = nullptr;
@@ -45,7 +62,7 @@ struct sync_programs {
   bool divergent = false;           // some program runs per-engine trip counts
   int64_t n_ord = 0;
   bool ord_overflow = false;        // an engine of a program has > INT32_MAX instances
-  std::vector<int64_t> ord_off_host;  // per instruction: pool offset or -1
+  syncgb::HostVec<int64_t> ord_off_host;  // per instruction: pool offset or -1
   int64_t n_chunks = 0;
   // simulator encoding
   syncgb::ProgInfo* prog = nullptr;
