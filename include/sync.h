@@ -135,7 +135,23 @@ enum {
  *     (SYNC_ERR_ARG otherwise): the barrier scheme needs every engine to meet
  *     the same barriers, and a per-engine wait value is a position in the
  *     producer engine's stream, which the consumer's loop state no longer
- *     determines. */
+ *     determines;
+ *   nonalloc_policy: what the loader does with a dependency outside the
+ *     allocatable cases (see sync_load_programs): SYNC_NONALLOC_REJECT
+ *     (0, the default) fails the load; SYNC_NONALLOC_BARRIER takes the
+ *     paper's fallback to the barrier scheme for the ones a barrier can
+ *     enforce (Sec. 5.2: a producer nested below S with a forward offset
+ *     k >= 1 or a backward offset k >= 2, whose target lies in an earlier
+ *     iteration of S): such a dependency gets no semaphore wait (its wait
+ *     value is 0 in every threshold array and the checker skips its pairs)
+ *     and its carrying loop S, unless S is the top level, gets an all-engine
+ *     barrier at the end of every iteration (drain-and-release, as in the
+ *     barrier scheme) in the barrier-free simulation; the barrier scheme has
+ *     those barriers already.  Such a batch takes the barrier-free and
+ *     barrier simulations (SYNC_ERR_ARG for the unrolled variant) and shared
+ *     trips (SYNC_ERR_ARG with per-engine trips). */
+typedef enum { SYNC_NONALLOC_REJECT = 0, SYNC_NONALLOC_BARRIER = 1 } sync_nonalloc_policy;
+
 typedef struct {
   int32_t n_programs;
   const int32_t *prog_loop_ptr, *prog_instr_ptr, *prog_dep_ptr;
@@ -147,6 +163,7 @@ typedef struct {
   const int32_t *trips;
   const int64_t *eng_trip_ptr;
   const int32_t *eng_trips;
+  int32_t nonalloc_policy;    /* sync_nonalloc_policy */
 } sync_batch_desc;
 
 typedef struct {
@@ -196,7 +213,11 @@ typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
  * indices, dependency table, per-(loop, engine) instruction streams.
  * Returns SYNC_ERR_MALFORMED for structural errors (listed with sync.h's
  * batch description), SYNC_ERR_NOT_ALLOCATABLE for a dependency outside the
- * cases above, SYNC_ERR_OVERFLOW when a loop's iteration total, a per-loop
+ * cases above (with SYNC_NONALLOC_BARRIER: one that no barrier at the end
+ * of its carrying loop's iterations enforces either -- a nested backward
+ * offset 0, or offset 0 to a later producer on the same engine),
+ * SYNC_ERR_ARG for a policy value outside sync_nonalloc_policy or barrier
+ * fallbacks in a batch with per-engine trips, SYNC_ERR_OVERFLOW when a loop's iteration total, a per-loop
  * threshold N*total, a pair count or an instance count exceeds INT32_MAX
  * (int64 totals are supported for pairs and instances across programs).
  * On SYNC_OK, *out receives a handle to free with sync_free_programs.  The
@@ -220,7 +241,8 @@ sync_status sync_pair_offsets(const sync_programs *h, int64_t *offsets, int32_t 
  * counted through the current / previous S-iteration when forward /
  * backward), in `mode`'s encoding (Eq. 3, Eq. 5 or Sec. 6.1).
  * d_thr: [n_pairs_padded] int32, caller-owned device memory, fully written
- * (padding entries 0).
+ * (padding entries 0, and the pairs of a dependency taken by the barrier
+ * fallback of SYNC_NONALLOC_BARRIER: 0, no wait).
  * The first PERENGINE call (thresholds or check) on a handle derives the
  * engine-stream positions of the waited producers' instances on the GPU: it
  * allocates device memory held by the handle (sync_sizes.device_bytes grows)
@@ -239,7 +261,8 @@ sync_status sync_eval_thresholds(const sync_programs *h, sync_thr_mode mode, int
  * d_counts: [2] uint64 device -- unsafe, over-synchronised pair counts;
  * d_first_bad: [1] int64 device -- smallest offending index into d_thr, or
  * -1.  Both are overwritten (no accumulation across calls); padding entries
- * of d_thr are ignored. */
+ * of d_thr and the pairs of barrier-fallback dependencies (enforced by
+ * barriers, not by a wait value) are ignored. */
 sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const int32_t *d_thr,
                                unsigned long long *d_counts, long long *d_first_bad,
                                void *stream);
@@ -258,8 +281,11 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  *   (with trip_register_elision, a loop that carries only offset-0
  *   dependencies, or none, costs 0 at its statement and c_branch + c_regop
  *   at each iteration start, barrier-free)
- *   iteration end: barrier only: barrier
- *   datapath x: barrier-free t += sum over its dependencies of the wait
+ *   iteration end: barrier: barrier; barrier-free: a barrier at the end of
+ *     each iteration of a loop that carries a barrier-fallback dependency
+ *     (SYNC_NONALLOC_BARRIER), none otherwise
+ *   datapath x (barrier-fallback dependencies are not waited on and cost
+ *     nothing here): barrier-free t += sum over its dependencies of the wait
  *     ops: c_wait_ops_count (COUNT), c_wait_ops_perloop (PERLOOP), or
  *     c_wait_ops_perloop + c_wait_ops_perengine_level * (depth of the
  *     producer's loop - 1, at least 0; the top level has depth 0)
@@ -272,8 +298,8 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  *   the top-level loop costs nothing; makespan = max over engines of
  *   max(t, last retire).
  * UNROLLED: as barrier-free with c_branch, c_regop and every wait-op cost
- * taken as 0 (ii and latencies unchanged); it requires PERENGINE and returns
- * SYNC_ERR_ARG otherwise.
+ * taken as 0 (ii and latencies unchanged); it requires PERENGINE and a batch
+ * without barrier-fallback dependencies, and returns SYNC_ERR_ARG otherwise.
  * Outputs per program (device, [n_programs]): d_makespan (int32, -1 unless
  * status OK), d_checksum (uint64, 0 unless OK: the sum mod 2^64 over
  * datapath instances of (a << 32) | b in 32-bit arithmetic, a = (issue ^

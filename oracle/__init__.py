@@ -26,7 +26,7 @@ _HDR = [os.path.join(_HERE, "oracle.h")]
 
 COUNT, PERLOOP, PERENGINE = 0, 1, 2
 BARRIER_FREE, BARRIER, UNROLLED = 0, 1, 2
-CASE_PS, CASE_NEST_FWD, CASE_NEST_BWD, CASE_NONE = 0, 1, 2, 3
+CASE_PS, CASE_NEST_FWD, CASE_NEST_BWD, CASE_NONE, CASE_BARRIER = 0, 1, 2, 3, 4
 SIM_OK, SIM_OVERFLOW, SIM_DEADLOCK = 0, 4, 7
 
 
@@ -50,7 +50,8 @@ class _Batch(ctypes.Structure):
             "loop_parent", "loop_pos", "instr_loop", "instr_pos", "instr_engine",
             "instr_latency", "dep_prod", "dep_cons", "dep_k")
     ] + [("trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("trips", ctypes.POINTER(ctypes.c_int32)),
-         ("eng_trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("eng_trips", ctypes.POINTER(ctypes.c_int32))]
+         ("eng_trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("eng_trips", ctypes.POINTER(ctypes.c_int32)),
+         ("nonalloc_policy", ctypes.c_int32)]
 
 
 class SimParams(ctypes.Structure):
@@ -105,7 +106,8 @@ class _View:
         self.keep = {}
         cb = _Batch()
         cb.n_programs = int(batch.n_programs)
-        for name, _ in _Batch._fields_[1:]:
+        cb.nonalloc_policy = int(getattr(batch, "nonalloc_policy", 0))
+        for name, _ in _Batch._fields_[1:-1]:
             a = getattr(batch, name, None)
             if a is None:                 # shared trips: the per-engine rows stay NULL
                 continue

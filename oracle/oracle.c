@@ -53,8 +53,14 @@
  *    with trip-register elision, a loop at which only offset-0 dependencies
  *    are carried (or none) keeps no r-hat (Sec. 5.1): barrier-free, its
  *    statement costs 0 and each iteration start c_branch + c_regop;
- *  - iteration end:            barrier scheme only: an all-engine barrier;
- *  - datapath instruction x with dependency set D(x):
+ *  - iteration end:            barrier scheme: an all-engine barrier;
+ *                              barrier-free: the same barrier at the end
+ *                              of each iteration of a loop that carries a
+ *                              barrier-fallback dependency (Sec. 5.2's
+ *                              fallback to the barrier scheme, batch
+ *                              nonalloc_policy 1), none otherwise;
+ *  - datapath instruction x with dependency set D(x) (barrier-fallback
+ *    dependencies left out: they are not waited on):
  *      barrier-free: t += sum over D(x) of the wait-value ops (Table 1):
  *        c_wait_ops_count (count), c_wait_ops_perloop (per-loop), or
  *        c_wait_ops_perloop + c_wait_ops_perengine_level * max(0, depth(P)
@@ -82,6 +88,7 @@
  * where e is the engine and n the instance's 1-based ordinal among engine
  * e's datapath instances.  Status: 4 when the static time bound
  *   sum_x inst(x)*(lat(x)+ii+wait ops(x)) + E*(stmts*c_regop + iters*(c_branch+2*c_regop))
+ *   + (iterations of loops with fallback barriers)*c_barrier
  * (barrier-free; unrolled: without the control and wait terms), or
  *   sum_x inst(x)*(lat(x)+ii) + E*iters*c_branch + (stmts+iters)*c_barrier
  * (barrier scheme) exceeds INT32_MAX; 7 when no engine can make progress
@@ -112,6 +119,7 @@ typedef struct {
   int32_t *body_ptr, *body;          /* items by position: x >= 0, or -(loop+1) */
   int32_t *prod_ptr, *prod_dep;      /* dependencies grouped by producer */
   int32_t *cons_ptr, *cons_dep;      /* dependencies grouped by consumer */
+  int policy;                        /* the batch's nonalloc_policy */
 } prog_t;
 
 static void prog_close(prog_t *P) {
@@ -176,6 +184,7 @@ static int prog_open(const orc_batch *b, int32_t p, prog_t *P) {
   P->nx = b->prog_instr_ptr[p + 1] - x0;
   P->nd = b->prog_dep_ptr[p + 1] - d0;
   P->ne = b->prog_n_engines[p];
+  P->policy = b->nonalloc_policy;
   if (P->nl < 1 || P->nx < 0 || P->nd < 0 || P->ne < 1 || P->ne > 32) return ORC_ERR_MALFORMED;
   P->par = b->loop_parent + l0; P->lpos = b->loop_pos + l0;
   P->xl = b->instr_loop + x0; P->xp = b->instr_pos + x0;
@@ -355,9 +364,9 @@ static dep_class classify(const prog_t *P, int32_t d) {
   if (cp < 0) {
     c.kase = (k == 0 && !forward && P->xe[p] == P->xe[x]) ? ORC_CASE_NONE : ORC_CASE_PS;
   } else if (forward) {
-    c.kase = k == 0 ? ORC_CASE_NEST_FWD : ORC_CASE_NONE;
+    c.kase = k == 0 ? ORC_CASE_NEST_FWD : P->policy ? ORC_CASE_BARRIER : ORC_CASE_NONE;
   } else {
-    c.kase = k == 1 ? ORC_CASE_NEST_BWD : ORC_CASE_NONE;
+    c.kase = k == 1 ? ORC_CASE_NEST_BWD : (P->policy && k >= 2) ? ORC_CASE_BARRIER : ORC_CASE_NONE;
   }
   c.N = 0; c.K = 1;
   for (int32_t y = 0; y < P->nx; ++y) {
@@ -685,6 +694,7 @@ static void replay_body(replay_ctx *R, int32_t l) {
         const dep_class *c = &R->cls[d];
         int64_t slot = R->pair_off[d] + (R->r[P->xl[it]] - 1);
         if (c->kase == ORC_CASE_NONE) { R->out[slot] = -1; continue; }
+        if (c->kase == ORC_CASE_BARRIER) { R->out[slot] = 0; continue; }   /* no wait emitted */
         int64_t k = P->dk[d];
         int64_t mask = R->rh[c->S] > k ? 1 : 0;                              /* Eq. (2) */
         int64_t expr = c->kase == ORC_CASE_PS ? nat_sub(R->r[c->S], k) : R->r[c->P];
@@ -766,11 +776,16 @@ int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[
     int32_t *want = (int32_t *)malloc(((size_t)np + 1) * sizeof(int32_t));
     if (rc == ORC_OK && !want) rc = ORC_ERR_OOM;
     if (rc == ORC_OK) rc = per_consumer_view(&P, mode, want, prog_thresholds);
-    for (int64_t i = 0; i < np && rc == ORC_OK; ++i) {
-      int32_t got = thr[base + i];
-      if (got == want[i]) continue;
-      counts[got < want[i] ? 0 : 1]++;
-      if (*first_bad < 0) *first_bad = base + i;
+    int64_t i = 0;
+    for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) {
+      int64_t n = cons_total(&P, d);
+      if (classify(&P, d).kase == ORC_CASE_BARRIER) { i += n; continue; }   /* enforced by barriers */
+      for (int64_t j = 0; j < n; ++j, ++i) {
+        int32_t got = thr[base + i];
+        if (got == want[i]) continue;
+        counts[got < want[i] ? 0 : 1]++;
+        if (*first_bad < 0) *first_bad = base + i;
+      }
     }
     free(want);
     prog_close(&P);
@@ -808,6 +823,8 @@ typedef struct {
   int64_t **times;             /* per waited semaphore: retire time of each increment */
   int32_t *issue, *retire;     /* program's instances, or NULL */
   int64_t *inst_off;           /* per instruction, program-local */
+  int8_t *dep_bar;             /* per dep: barrier fallback (no wait) */
+  int8_t *loop_bar;            /* per loop: all-engine barrier at the end of each iteration */
 } sim_ctx;
 
 static uint64_t inst_term(int64_t issue, int64_t retire, int32_t e, int64_t n) {
@@ -827,7 +844,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
   int32_t blen = P->body_ptr[f->loop + 1] - P->body_ptr[f->loop];
   if (f->item == blen) {                       /* end of an iteration's body */
     if (f->loop == 0) { E->state = E_DONE; return S_DONE; }
-    if (X->barrier && !E->bar_passed) {
+    if ((X->barrier || X->loop_bar[f->loop]) && !E->bar_passed) {
       E->arrival = max64(E->t, E->lastret);
       E->state = E_BAR;
       return S_BARRIER;
@@ -869,6 +886,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
   int64_t ready = 0;
   for (int32_t j = P->cons_ptr[it]; j < P->cons_ptr[it + 1]; ++j) {
     int32_t d = P->cons_dep[j];
+    if (X->dep_bar[d]) continue;               /* enforced by a barrier, not waited on */
     int32_t T = X->thr[X->pair_off[d] + f->g];
     if (T <= 0) continue;
     int32_t s = X->dep_sem[d];
@@ -900,8 +918,22 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   int unrolled = variant == ORC_UNROLLED;       /* straight-line: no control or wait-value ops */
   /* wait-value ops of each dependency (Table 1; per-engine: O(D), Sec. 6.1) */
   int64_t *wcost = (int64_t *)calloc((size_t)nx + 1, sizeof(int64_t));
-  if (!wcost) return ORC_ERR_OOM;
+  int8_t *dep_bar = (int8_t *)calloc((size_t)nd + 1, sizeof(int8_t));
+  int8_t *loop_bar = (int8_t *)calloc((size_t)nl, sizeof(int8_t));
+  if (!wcost || !dep_bar || !loop_bar) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_OOM; }
+  /* barrier fallback (Sec. 5.2): no wait; a barrier ends every iteration of
+   * the carrying loop S (none at the top level, which runs once) */
+  int any_bar = 0;
+  for (int32_t d = 0; d < nd; ++d) {
+    dep_class c = classify(P, d);
+    if (c.kase != ORC_CASE_BARRIER) continue;
+    dep_bar[d] = 1;
+    any_bar = 1;
+    if (c.S != 0) loop_bar[c.S] = 1;
+  }
+  if (any_bar && unrolled) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_ARG; }
   for (int32_t d = 0; d < nd && !unrolled; ++d) {
+    if (dep_bar[d]) continue;
     int64_t c = mode == ORC_COUNT ? q->c_wait_ops_count : q->c_wait_ops_perloop;
     if (mode == ORC_PERENGINE) {
       int32_t lev = P->depth[P->xl[P->dp[d]]] - 1;
@@ -917,11 +949,11 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   int64_t *stmt_cost = (int64_t *)calloc((size_t)nl, sizeof(int64_t));
   int8_t *needs_rhat = (int8_t *)calloc((size_t)nl, sizeof(int8_t));
   if (!iter_cost || !stmt_cost || !needs_rhat) {
-    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost);
+    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(dep_bar); free(loop_bar);
     return ORC_ERR_OOM;
   }
-  for (int32_t d = 0; d < nd; ++d)
-    if (P->dk[d] > 0) needs_rhat[classify(P, d).S] = 1;
+  for (int32_t d = 0; d < nd; ++d)     /* a barrier-fallback dependency reads no register */
+    if (P->dk[d] > 0 && !dep_bar[d]) needs_rhat[classify(P, d).S] = 1;
   for (int32_t l = 0; l < nl; ++l) {
     int elide = q->trip_register_elision && !needs_rhat[l];
     iter_cost[l] = unrolled ? 0 : barrier ? q->c_branch : q->c_branch + (elide ? 1 : 2) * (int64_t)q->c_regop;
@@ -947,9 +979,11 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     bound += (u128)(stmts / ne + iters / ne) * (u128)q->c_barrier;
   } else {
     bound += ctl;
+    for (int32_t l = 1; l < nl; ++l)  /* the fallback barriers: one per iteration of a flagged loop */
+      if (loop_bar[l]) bound += (u128)P->total[l] * (u128)q->c_barrier;
   }
   if (bound > (u128)INT32_MAX) {
-    free(wcost); free(iter_cost); free(stmt_cost);
+    free(wcost); free(iter_cost); free(stmt_cost); free(dep_bar); free(loop_bar);
     *makespan = -1; *checksum = 0; *status = ORC_SIM_OVERFLOW;
     return ORC_OK;
   }
@@ -958,6 +992,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   X.P = P; X.prm = q; X.mode = mode; X.barrier = barrier; X.wcost = wcost; X.thr = thr;
   X.iter_cost = iter_cost; X.stmt_cost = stmt_cost;
   X.issue = issue; X.retire = retire;
+  X.dep_bar = dep_bar; X.loop_bar = loop_bar;
   int32_t nsem = mode == ORC_COUNT ? nx : mode == ORC_PERLOOP ? nl * ne : ne;
   X.pair_off = (int64_t *)malloc(((size_t)nd + 1) * sizeof(int64_t));
   X.inst_off = (int64_t *)malloc(((size_t)nx + 1) * sizeof(int64_t));
@@ -982,7 +1017,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
       int32_t p = P->dp[d];
       X.dep_sem[d] = mode == ORC_COUNT ? p : mode == ORC_PERLOOP ? P->xl[p] * ne + P->xe[p] : P->xe[p];
       int32_t s = X.dep_sem[d];
-      if (!X.times[s]) {
+      if (!dep_bar[d] && !X.times[s]) {
         X.times[s] = (int64_t *)malloc(((size_t)incs[s] + 1) * sizeof(int64_t));
         if (!X.times[s]) rc = ORC_ERR_OOM;
       }
@@ -1036,6 +1071,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   for (int32_t s = 0; X.times && s < nsem; ++s) free(X.times[s]);
   free(E); free(incs); free(X.pair_off); free(X.inst_off); free(X.own_sem); free(X.dep_sem);
   free(X.value); free(X.times); free(wcost); free(iter_cost); free(stmt_cost);
+  free(dep_bar); free(loop_bar);
   return rc;
 }
 
@@ -1053,6 +1089,8 @@ int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim
     int rc = prog_open(b, p, &P);
     /* per-engine trips: no common barrier sequence, no per-engine positions */
     if (rc == ORC_OK && P.div && (variant != ORC_BARRIER_FREE || mode == ORC_PERENGINE)) rc = ORC_ERR_ARG;
+    for (int32_t d = 0; d < P.nd && rc == ORC_OK && P.div; ++d)   /* no common barriers */
+      if (classify(&P, d).kase == ORC_CASE_BARRIER) rc = ORC_ERR_ARG;
     if (rc == ORC_OK)
       rc = sim_program(&P, mode, thr + pbase, prm, variant, makespan + p, checksum + p,
                        status + p, issue ? issue + ibase : NULL, retire ? retire + ibase : NULL);

@@ -36,6 +36,10 @@ typedef struct {
    * iteration of its parent on that engine.  When set, `trips` is unused. */
   const int64_t *eng_trip_ptr;
   const int32_t *eng_trips;
+  /* 0: every dependency is taken as a semaphore wait; 1: the fallback of
+   * Sec. 5.2 to the barrier scheme for the non-allocatable dependencies a
+   * barrier enforces (ORC_CASE_BARRIER below) */
+  int32_t nonalloc_policy;
 } orc_batch;
 
 enum { ORC_OK = 0, ORC_ERR_ARG = 1, ORC_ERR_MALFORMED = 2, ORC_ERR_NOT_ALLOCATABLE = 3,
@@ -48,8 +52,13 @@ enum { ORC_OK = 0, ORC_ERR_ARG = 1, ORC_ERR_MALFORMED = 2, ORC_ERR_NOT_ALLOCATAB
  * c-th instance in its engine's dynamic instruction stream, 0 when c = 0 */
 enum { ORC_COUNT = 0, ORC_PERLOOP = 1, ORC_PERENGINE = 2 };
 
-/* allocatable cases of Sec. 5.2 */
-enum { ORC_CASE_PS = 0, ORC_CASE_NEST_FWD = 1, ORC_CASE_NEST_BWD = 2, ORC_CASE_NONE = 3 };
+/* allocatable cases of Sec. 5.2; with nonalloc_policy 1, ORC_CASE_BARRIER is
+ * a producer nested below S with a forward offset >= 1 or a backward offset
+ * >= 2 (its target lies in an earlier iteration of S, so an all-engine
+ * barrier at the end of every iteration of S enforces it); ORC_CASE_NONE is
+ * what remains outside the cases */
+enum { ORC_CASE_PS = 0, ORC_CASE_NEST_FWD = 1, ORC_CASE_NEST_BWD = 2, ORC_CASE_NONE = 3,
+       ORC_CASE_BARRIER = 4 };
 
 /* simulator variants (UNROLLED: the straight-line program, per-engine
  * thresholds, no loop-control or wait-value operations) and per-program
@@ -98,13 +107,15 @@ int orc_thresholds(const orc_batch *b, int mode, int32_t *out);
 /* The paper's registers replayed literally per engine (Fig. 7/8): r-hat := 0
  * at each loop statement, r++ and r-hat++ at each iteration start, and the
  * masked wait value of Eq. (2)/(3)/(5) before each consumer.  Entries of
- * non-allocatable dependencies are set to -1.  Count and per-loop modes
+ * non-allocatable dependencies are set to -1, those of ORC_CASE_BARRIER
+ * dependencies to 0 (the barrier fallback emits no wait).  Count and per-loop modes
  * only. */
 int orc_register_replay(const orc_batch *b, int mode, int32_t *out);
 
 /* Minimality check of a threshold array against Eq. (1): counts[0] = pairs
  * whose threshold is below the minimum (unsafe), counts[1] = above it
- * (over-synchronised); first_bad = first such pair index or -1. */
+ * (over-synchronised); first_bad = first such pair index or -1.  The pairs
+ * of ORC_CASE_BARRIER dependencies are skipped (a barrier enforces them). */
 int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[2],
               int64_t *first_bad);
 
@@ -114,6 +125,12 @@ int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[
  * (per-loop) or the producer's engine semaphore, which every retirement on
  * that engine increments (per-engine), until its value reaches the
  * threshold.  The unrolled variant needs per-engine thresholds.
+ * ORC_CASE_BARRIER dependencies are not waited on and cost no wait ops; the
+ * loop that carries one (unless it is the top level) ends every iteration
+ * with an all-engine barrier, also barrier-free (the barrier scheme has
+ * those barriers anyway); the static time bound counts one c_barrier per
+ * such barrier.  Such programs take neither the unrolled variant nor
+ * per-engine trips (ORC_ERR_ARG).
  * issue/retire may be NULL. */
 int orc_simulate(const orc_batch *b, int mode, const int32_t *thr, const orc_sim_params *prm,
                  int variant, int32_t *makespan, uint64_t *checksum, int32_t *status,

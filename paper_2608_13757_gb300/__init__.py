@@ -47,7 +47,10 @@ class BatchDesc(ctypes.Structure):
             "loop_parent", "loop_pos", "instr_loop", "instr_pos", "instr_engine",
             "instr_latency", "dep_prod", "dep_cons", "dep_k")
     ] + [("trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("trips", ctypes.POINTER(ctypes.c_int32)),
-         ("eng_trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("eng_trips", ctypes.POINTER(ctypes.c_int32))]
+         ("eng_trip_ptr", ctypes.POINTER(ctypes.c_int64)), ("eng_trips", ctypes.POINTER(ctypes.c_int32)),
+         ("nonalloc_policy", ctypes.c_int32)]
+
+NONALLOC_REJECT, NONALLOC_BARRIER = 0, 1
 
 
 class Sizes(ctypes.Structure):
@@ -133,7 +136,11 @@ def batch_desc(batch):
     keep = []
     desc = BatchDesc()
     desc.n_programs = int(get("n_programs"))
-    for name, _ in BatchDesc._fields_[1:]:
+    try:
+        desc.nonalloc_policy = int(get("nonalloc_policy"))
+    except (KeyError, AttributeError):
+        desc.nonalloc_policy = NONALLOC_REJECT
+    for name, _ in BatchDesc._fields_[1:-1]:
         is64 = name in ("trip_ptr", "eng_trip_ptr")
         try:
             v = get(name)

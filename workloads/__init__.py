@@ -107,13 +107,13 @@ class TreeParams(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "engines_lo", "engines_hi", "max_depth", "loops_lo", "loops_hi", "body_lo", "body_hi",
         "trip_lo", "trip_hi", "cond_permille", "lat_lo", "lat_hi", "dep_permille",
-        "max_deps_per_cons", "k_max", "any_k")]
+        "max_deps_per_cons", "k_max", "any_k", "nest_far_permille")]
 
 
 def tree_params(**kw) -> TreeParams:
     d = dict(engines_lo=1, engines_hi=4, max_depth=3, loops_lo=0, loops_hi=4, body_lo=0,
              body_hi=4, trip_lo=0, trip_hi=3, cond_permille=150, lat_lo=1, lat_hi=8,
-             dep_permille=500, max_deps_per_cons=2, k_max=2, any_k=0)
+             dep_permille=500, max_deps_per_cons=2, k_max=2, any_k=0, nest_far_permille=0)
     d.update(kw)
     return TreeParams(**d)
 
@@ -138,6 +138,9 @@ class Batch:
     trips: np.ndarray
     eng_trip_ptr: np.ndarray | None = None
     eng_trips: np.ndarray | None = None
+    # what the loader does with non-allocatable dependencies: 0 rejects,
+    # 1 falls back to barriers at the end of the carrying loop's iterations
+    nonalloc_policy: int = 0
 
     @property
     def divergent(self) -> bool:
@@ -169,10 +172,11 @@ class Batch:
 
     def arrays(self):
         return {f.name: getattr(self, f.name) for f in fields(self)
-                if f.name != "n_programs" and getattr(self, f.name) is not None}
+                if f.name not in ("n_programs", "nonalloc_policy") and getattr(self, f.name) is not None}
 
     def copy(self) -> "Batch":
-        return Batch(self.n_programs, **{k: v.copy() for k, v in self.arrays().items()})
+        return Batch(self.n_programs, **{k: v.copy() for k, v in self.arrays().items()},
+                     nonalloc_policy=self.nonalloc_policy)
 
     def nbytes(self) -> int:
         return int(sum(v.nbytes for v in self.arrays().values()))
@@ -311,6 +315,7 @@ def concat(batches, programs=None) -> Batch:
         trip_ptr=cat(tp, np.int64),
         eng_trip_ptr=np.array(etp + [ebase], dtype=np.int64) if divergent else None,
         eng_trips=cat(etrips, np.int32) if divergent else None,
+        nonalloc_policy=max((batches[bi].nonalloc_policy for bi, _ in programs), default=0),
         **{k: cat(v, np.int32) for k, v in parts.items()},
     )
 

@@ -487,6 +487,8 @@ static void gen_tree(pbuild *b, rng_t *r, const synth_tree_params *p) {
            * only when the producer is earlier in that body */
           int32_t hi = p->k_max < 1 ? 1 : p->k_max;
           k = xpos > ppos ? rng_uni(r, 0, p->k_max) : rng_uni(r, 1, hi);
+        } else if (p->nest_far_permille > 0 && rng_uni(r, 0, 999) < p->nest_far_permille) {
+          k = xpos > ppos ? rng_uni(r, 1, p->k_max + 1) : rng_uni(r, 2, p->k_max + 2);
         } else {
           k = xpos > ppos ? 0 : 1;
         }

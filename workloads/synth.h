@@ -47,6 +47,9 @@ typedef struct {
   int32_t max_deps_per_cons;
   int32_t k_max;
   int32_t any_k;                /* 1: offsets drawn freely (may be non-allocatable) */
+  int32_t nest_far_permille;    /* chance that a nested producer gets an offset
+                                   beyond the allocatable one (forward 1..k_max+1,
+                                   backward 2..k_max+2): a barrier-fallback case */
 } synth_tree_params;
 
 /* Programs first_program .. first_program+n_programs-1 of a fixed config; a
