@@ -113,6 +113,8 @@ struct ProgScratch {
   std::vector<int32_t> xid;                       // per-engine trips: expansion-table entry per (loop, engine)
   std::vector<int64_t> tstart_of;                 // derived trip-start array per loop (and engine), -1 if none
   std::vector<uint8_t> needs_rhat;                // per loop: carries a dependency with offset > 0
+  std::vector<uint8_t> fbar;                      // per loop: ends its iterations with a fallback barrier
+  std::vector<uint8_t> dep_bar;                   // per dependency: barrier fallback (not waited on)
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
   std::vector<int32_t> by_cons, cons_next, sem_of;  // dependencies by consumer; semaphore per key
   std::vector<int64_t> inst_eng, sem_hist;        // instances per engine; history bases of one mode
@@ -141,6 +143,7 @@ struct Part {
   int64_t hist_len[kModes] = {0, 0, 0};
   bool ord_overflow = false;
   int32_t nsem_max[kModes] = {0, 0, 0}, ne_max = 0, depth_max = 0;
+  int64_t n_bar_deps = 0;                  // barrier-fallback dependencies
   std::exception_ptr error;
 };
 
@@ -176,6 +179,8 @@ std::string where(int32_t p, const char* what, int64_t i) {
 static void build(const sync_batch_desc& d, int device, cudaStream_t stream, sync_programs& h) {
   // ---------------------------------------------------------- shape checks
   if (d.n_programs < 0) raise(SYNC_ERR_ARG, "n_programs < 0");
+  if (d.nonalloc_policy != SYNC_NONALLOC_REJECT && d.nonalloc_policy != SYNC_NONALLOC_BARRIER)
+    raise(SYNC_ERR_ARG, "nonalloc_policy is not a sync_nonalloc_policy");
   const int32_t P = d.n_programs;
   if (!d.prog_loop_ptr || !d.prog_instr_ptr || !d.prog_dep_ptr || (P > 0 && !d.prog_n_engines))
     raise(SYNC_ERR_ARG, "program CSR arrays must not be NULL");
@@ -247,6 +252,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   auto& hist_len = part.hist_len;
   auto push_path = [&](int64_t v, uint8_t kind) { path.push_back(v); part.path_kind.push_back(kind); };
   int64_t erow = erow0;                     // per-engine trips: first row of the program
+  const bool fallback = d.nonalloc_policy == SYNC_NONALLOC_BARRIER;
   ProgScratch S;
 
   for (int32_t p = p_begin; p < p_end; ++p) {
@@ -264,6 +270,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     S.tstart_of.assign((size_t)nl * (div ? ne : 1), -1);
     S.anc_of.clear();
     S.needs_rhat.assign(nl, 0);
+    S.fbar.assign(nl, 0);
+    S.dep_bar.assign(nd, 0);
     if (par[0] != -1) raise(SYNC_ERR_MALFORMED, where(p, "loop 0 must have parent -1, loop", 0));
     int32_t depth_max = 0;
     for (int32_t l = 1; l < nl; ++l) {
@@ -424,7 +432,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       while (S.depth[b] > S.depth[a]) { cb = b; b = par[b]; }
       while (a != b) { ca = a; a = par[a]; cb = b; b = par[b]; }
       const int32_t Sl = a;
-      if (off > 0) S.needs_rhat[Sl] = 1;           // r-hat_S's no-wait check matters
       const int32_t ppos = ca < 0 ? d.instr_pos[x0 + px] : lpos[ca];
       const int32_t cpos = cb < 0 ? d.instr_pos[x0 + cx] : lpos[cb];
       const bool forward = cpos > ppos;
@@ -437,13 +444,39 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
           raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "offset 0 to a later producer on the same engine, dependency", k));
         kase = CASE_PS;
       } else if (forward) {
-        if (off != 0) raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested forward producer needs offset 0, dependency", k));
-        kase = CASE_NEST_FWD;
+        // a larger offset targets an earlier iteration of S: with the
+        // fallback, barriers at the ends of S's iterations enforce it
+        if (off != 0 && !fallback)
+          raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested forward producer needs offset 0, dependency", k));
+        kase = off == 0 ? CASE_NEST_FWD : CASE_BARRIER;
       } else {
-        if (off != 1) raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested backward producer needs offset 1, dependency", k));
-        kase = CASE_NEST_BWD;
+        if (off != 1 && (!fallback || off == 0))
+          raise(SYNC_ERR_NOT_ALLOCATABLE, where(p, "nested backward producer needs offset 1, dependency", k));
+        kase = off == 1 ? CASE_NEST_BWD : CASE_BARRIER;
       }
       const int32_t ep = d.instr_engine[x0 + px], ec = d.instr_engine[x0 + cx];
+      S.dep_bar[k] = kase == CASE_BARRIER;
+      if (kase == CASE_BARRIER) {
+        // no wait value, semaphore, register or derived array: its pairs stay
+        // in the threshold layout (wait value 0) and S ends its iterations
+        // with all-engine barriers (none at the top level, which runs once)
+        if (div) raise(SYNC_ERR_ARG, where(p, "barrier fallback with per-engine trip counts, dependency", k));
+        if (Sl != 0) S.fbar[Sl] = 1;
+        DepInfo& D = dep[gd];
+        std::memset(&D, 0, sizeof D);
+        D.total = (int32_t)tot(Cl, ec);
+        dep_count[gd] = D.total;
+        D.kase = kase;
+        D.k = off;
+        D.seg_off = n_pairs_padded;
+        seg[gd] = n_pairs_padded;
+        n_pairs += tot(Cl, ec);
+        n_pairs_padded += pad4(tot(Cl, ec));
+        dep_N[gd] = 0;
+        dep_K[gd] = 0;
+        continue;
+      }
+      if (off > 0) S.needs_rhat[Sl] = 1;           // r-hat_S's no-wait check matters
       const int32_t N = S.nloop_eng[(size_t)Pl * ne + ep];
       const int32_t K = S.rank[px];
       if ((int64_t)N * tot(Pl, ep) > kI32Max)
@@ -508,6 +541,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     }
     // loops whose trip register can be elided (Sec. 5.1: only offset-0
     // dependencies carried there, or none), and their control counts
+    for (int32_t l = 1; l < nl; ++l)              // the barrier fallback's barriers (shared trips)
+      if (S.fbar[l]) pi.fb_iters += tot(l, 0);
+    for (int32_t k = 0; k < nd; ++k) part.n_bar_deps += S.dep_bar[k];
     lflag[l0] = 0;
     for (int32_t l = 1; l < nl; ++l) {
       lflag[l0 + l] = S.needs_rhat[l] ? 0 : 1;
@@ -533,6 +569,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     // per-engine waits: loops strictly between the top level and the producer's loop
     auto levels = [&](int32_t px) { return std::max(0, S.depth[d.instr_loop[x0 + px]] - 1); };
     for (int32_t k = 0; k < nd; ++k) {
+      if (S.dep_bar[k]) continue;                  // not waited on
       const int64_t gd = d0 + k;
       S.x_levels[d.dep_cons[gd]] += levels(d.dep_prod[gd]);
       pi.pair_levels += (int64_t)levels(d.dep_prod[gd]) *
@@ -544,13 +581,16 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     by_cons.resize(nd);
     auto& next = S.cons_next;
     next.resize(nx);
-    for (int32_t k = 0; k < nd; ++k) S.x_ndeps[d.dep_cons[d0 + k]]++;
+    for (int32_t k = 0; k < nd; ++k)
+      if (!S.dep_bar[k]) S.x_ndeps[d.dep_cons[d0 + k]]++;
     for (int32_t x = 0, at = 0; x < nx; ++x) {
       if (S.x_ndeps[x] > 0) S.x_dep_begin[x] = d0 + at;
       next[x] = at;
       at += S.x_ndeps[x];
     }
-    for (int32_t k = 0; k < nd; ++k) by_cons[next[d.dep_cons[d0 + k]]++] = k;
+    int32_t nw = 0;                                // waited dependencies, grouped first
+    for (int32_t k = 0; k < nd; ++k)
+      if (!S.dep_bar[k]) { by_cons[next[d.dep_cons[d0 + k]]++] = k; ++nw; }
     auto& sem_of = S.sem_of;
     auto& sem_hist = S.sem_hist;
     sem_of.resize(std::max(nx, nl * ne));
@@ -558,6 +598,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       std::fill(sem_of.begin(), sem_of.end(), -1);
       sem_hist.clear();
       for (int32_t k = 0; k < nd; ++k) {
+        if (S.dep_bar[k]) continue;                // not waited on: no semaphore of its own
         const int64_t gd = d0 + k;
         const int32_t px = d.dep_prod[gd];
         const int32_t Pl = d.instr_loop[x0 + px];
@@ -584,10 +625,14 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         xsem[(size_t)m * NX + x0 + x] =
             make_int4(s, S.x_hstride[m][x], S.x_koff[m][x], m == 2 ? S.x_levels[x] : 0);
       }
-      for (int32_t i = 0; i < nd; ++i) {
+      for (int32_t i = 0; i < nw; ++i) {
         const int64_t gd = d0 + by_cons[i];
         dsem[(size_t)m * ND + d0 + i] = sem_of[sem_key(m, d.dep_prod[gd])];
         if (m == 0) { dseg[d0 + i] = seg[gd]; ddep[d0 + i] = (int32_t)gd; }
+      }
+      for (int32_t i = nw; i < nd; ++i) {          // slots of barrier-fallback dependencies: unused
+        dsem[(size_t)m * ND + d0 + i] = -1;
+        if (m == 0) { dseg[d0 + i] = 0; ddep[d0 + i] = (int32_t)(d0 + i); }
       }
     }
     // per-(loop, engine) op records: own instructions and child loops in body
@@ -611,7 +656,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         }
         const int32_t end_idx = (int32_t)ops.size();
         ops.push_back(make_int4(OP_END, 0, 0, 0));
-        rowinfo.push_back(make_int2(end_idx, (has_loop ? 1 : 0) | (lflag[l0 + l] ? 2 : 0)));
+        rowinfo.push_back(make_int2(end_idx, (has_loop ? 1 : 0) | (lflag[l0 + l] ? 2 : 0) | (S.fbar[l] ? 4 : 0)));
         // next LOOP or END record at or after each record of the row
         opstop.resize(ops.size());
         int32_t next = end_idx;
@@ -771,6 +816,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   std::vector<int64_t> hist_len(all.hist, all.hist + kModes);
   bool ord_overflow = false;
   for (const Part& pt : parts) ord_overflow = ord_overflow || pt.ord_overflow;
+  h.n_bar_deps = 0;
+  for (const Part& pt : parts) h.n_bar_deps += pt.n_bar_deps;
   auto join_block = [&](int t) {
     Part& pt = parts[t];
     const Base& B = base[t];
@@ -1132,6 +1179,8 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
     raise(SYNC_ERR_ARG, "unknown variant");
   if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
     raise(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
+  if (variant == SYNC_SIM_UNROLLED && h->n_bar_deps > 0)
+    raise(SYNC_ERR_ARG, "the unrolled variant takes no barrier-fallback dependencies");
   check_divergent(h, mode, true, variant);
   if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))
     raise(SYNC_ERR_ARG, "per-program outputs must not be NULL");

@@ -12,7 +12,7 @@
 
 namespace syncgb {
 
-enum : int32_t { CASE_PS = 0, CASE_NEST_FWD = 1, CASE_NEST_BWD = 2 };
+enum : int32_t { CASE_PS = 0, CASE_NEST_FWD = 1, CASE_NEST_BWD = 2, CASE_BARRIER = 3 };
 
 // Pairs are processed in chunks of 4 consecutive entries (one int4).  A tile
 // is the span one 256-thread CTA covers in one pass.
@@ -68,6 +68,8 @@ struct alignas(16) ProgInfo {
   int64_t el_stmt;    // of these, those of loops that carry no offset > 0 (whose trip
   int64_t el_iter;    // register can be elided)
   int64_t pair_levels;  // sum over pairs of the per-engine wait's extra levels
+  int64_t fb_iters;   // iterations ended by a barrier-fallback barrier (barrier-free);
+                      // > 0: simulated by the per-engine kernel
   int32_t ne;
   int32_t le_base;    // row of (top-level loop, engine 0); row of (program-local
                       // loop l, engine e) = le_base + l*ne + e
@@ -105,7 +107,8 @@ constexpr int32_t LANE_RUN_LAST = 2;
 // Per record: opstop = index of the first LOOP or END record at or after it
 // in its row.  Per row: op_ptr = first record, rowinfo = {END record index,
 // bit 0: the row holds a LOOP record, bit 1: the row's loop carries no
-// offset > 0 (its trip register can be elided)}.
+// offset > 0 (its trip register can be elided), bit 2: the row's loop ends
+// every iteration with a barrier-fallback barrier}.
 // Per-mode semaphore records parallel to the op records (mode 0 = one
 // semaphore per producer instruction, mode 1 = one per (loop, engine),
 // mode 2 = one per engine):

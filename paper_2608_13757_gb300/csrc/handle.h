@@ -60,6 +60,7 @@ struct sync_programs {
   mutable int32_t* ord = nullptr;
   mutable bool ord_ready = false;
   bool divergent = false;           // some program runs per-engine trip counts
+  int64_t n_bar_deps = 0;           // barrier-fallback dependencies (no unrolled variant)
   int64_t n_ord = 0;
   bool ord_overflow = false;        // an engine of a program has > INT32_MAX instances
   syncgb::HostVec<int64_t> ord_off_host;  // per instruction: pool offset or -1

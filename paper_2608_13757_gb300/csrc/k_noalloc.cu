@@ -62,6 +62,8 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
     return set_error(SYNC_ERR_ARG, "unknown variant");
   if (variant == SYNC_SIM_UNROLLED && mode != SYNC_THR_PERENGINE)
     return set_error(SYNC_ERR_ARG, "the unrolled variant takes per-engine thresholds");
+  if (variant == SYNC_SIM_UNROLLED && h->n_bar_deps > 0)
+    return set_error(SYNC_ERR_ARG, "the unrolled variant takes no barrier-fallback dependencies");
   if (h->divergent && (mode == SYNC_THR_PERENGINE || variant != SYNC_SIM_BARRIER_FREE))
     return set_error(SYNC_ERR_ARG, "per-engine trip counts: barrier-free count or per-loop simulation only");
   if (h->sz.n_programs > 0 && (!d_makespan || !d_checksum || !d_status))

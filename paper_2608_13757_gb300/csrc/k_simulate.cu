@@ -113,6 +113,7 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul(rhat_stmts, (u64)q.c_regop));
     b = sat_add(b, sat_mul((u64)pi.eng_iter, (u64)q.c_branch + (u64)q.c_regop));
     b = sat_add(b, sat_mul(rhat_iters, (u64)q.c_regop));
+    b = sat_add(b, sat_mul((u64)pi.fb_iters, (u64)q.c_barrier));   // barrier-fallback barriers
   }
   return b;
 }
@@ -136,6 +137,8 @@ struct Eng {
   int32_t lo;              // start of the current trip
   int32_t ic;              // iteration-start cost of the current row's loop
   bool loops;              // the current row holds a child loop
+  bool fbar;               // barrier-free: the current row's loop ends each iteration
+                           // with a barrier-fallback barrier
   int32_t t, lastret;
   int32_t bar_gen;         // barrier generation this engine waits to see pass
   uint32_t n;              // datapath instances issued so far
@@ -182,6 +185,7 @@ __device__ __forceinline__ void set_row(const SimArgs& a, Eng& E, int32_t row) {
   const int2 ri = __ldg(a.rowinfo + row);
   E.rend = ri.x;
   E.loops = (ri.y & 1) != 0;
+  E.fbar = !BB && (ri.y & 4) != 0;
   // barrier-free with trip-register elision, a loop carrying no offset > 0
   // has no r-hat++ at its iteration starts
   const int32_t ic = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
@@ -225,7 +229,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
   Frame* frames = S.frames + w * a.frame_depth;
   bool moved = false;
   int spins = kSpin;
-  if (BB && E.state == ST_BAR) {                     // waiting at a barrier
+  if (E.state == ST_BAR) {                           // waiting at a barrier
     if (!barrier_poll(S, E, spins)) return false;
     E.t = *(volatile int32_t*)(S.slot + 3);
     E.state = ST_RUN;
@@ -234,8 +238,10 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
   }
   for (int c = 0; c < kChunks; ++c) {
     const int4 r0 = __ldg(a.ops + E.ptr);
-    if (BB && (r0.x == OP_LOOP || (r0.x == OP_END && E.sp != 0)) && !E.bar_passed) {
+    const bool at_end = r0.x == OP_END && E.sp != 0;
+    if ((BB ? r0.x == OP_LOOP || at_end : E.fbar && at_end) && !E.bar_passed) {
       // an all-engine barrier before the loop statement / after the iteration
+      // (barrier-free: after each iteration of a loop with a fallback barrier)
       moved = true;
       if (!barrier_arrive<BB>(a, S, E, w, lane, ne) && !barrier_poll(S, E, spins)) return true;
       E.t = *(volatile int32_t*)(S.slot + 3);
@@ -281,7 +287,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
       continue;
     }
     // ---- a chunk of datapath events (and, run-on, iteration starts)
-    const bool periodic = !BB && !E.loops;
+    const bool periodic = !BB && !E.loops && !E.fbar;
     const int32_t period = E.rend - E.pbeg + 1;      // the body's records and its END
     int32_t idx, gj;
     bool valid, is_end;
@@ -451,7 +457,7 @@ __global__ void __launch_bounds__(1024) k_simulate(const SimArgs a) {
     E.t = 0; E.lastret = 0; E.bar_gen = 0; E.n = 0;
     E.state = live ? ST_RUN : ST_DONE;
     E.bar_passed = false;
-    E.row = 0; E.pbeg = 0; E.rend = 0; E.loops = false; E.ptr = 0; E.ic = 0;
+    E.row = 0; E.pbeg = 0; E.rend = 0; E.loops = false; E.fbar = false; E.ptr = 0; E.ic = 0;
     if (live) {
       set_row<MODE, BB, TL>(a, E, pi.le_base + w);
       E.ptr = E.pbeg;
@@ -478,7 +484,7 @@ __global__ void __launch_bounds__(1024) k_simulate(const SimArgs a) {
         n_live += S.w_state[i] != ST_DONE;
       }
       // a barrier released after its waiters stopped polling is progress too
-      const bool released = BB && S.slot[2] != E.bar_gen && E.state == ST_BAR;
+      const bool released = S.slot[2] != E.bar_gen && E.state == ST_BAR;
       const bool any_released = __syncthreads_or(released) != 0;
       // the watchdog reads thread 0's clock so that every thread agrees
       if (threadIdx.x == 0) S.w_ms[0] = clock64() - started > kWatchdogCycles;

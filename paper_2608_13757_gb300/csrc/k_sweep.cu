@@ -2,8 +2,9 @@
 //
 // Under a common loop tree every engine meets the same loop statements and
 // iteration boundaries, so one walker per program can visit the tree once for
-// all engines (programs whose engines run their own trip counts go straight
-// to the per-engine kernel).  The body of each loop is cut at its child loops into
+// all engines (programs whose engines run their own trip counts, and
+// barrier-free the programs with the barriers of the non-allocatable
+// fallback, go straight to the per-engine kernel).  The body of each loop is cut at its child loops into
 // straight-line segments; a segment is taken as one chunk of up to 32 datapath
 // records (more chunks if longer), or -- barrier-free, for a short innermost
 // body -- as several consecutive iterations at once.  The chunk's lanes are
@@ -93,6 +94,7 @@ __device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, con
     b = sat_add(b, sat_mul(rhat_stmts, (u64)q.c_regop));
     b = sat_add(b, sat_mul((u64)pi.eng_iter, (u64)q.c_branch + (u64)q.c_regop));
     b = sat_add(b, sat_mul(rhat_iters, (u64)q.c_regop));
+    b = sat_add(b, sat_mul((u64)pi.fb_iters, (u64)q.c_barrier));   // barrier-fallback barriers
   }
   return b;
 }
@@ -697,7 +699,9 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     if (slot >= a.n_programs) break;
     const int p = __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
-    if (pi.divergent) {               // engines on their own trips: no common walk
+    // engines on their own trips (no common walk), or barrier-free with the
+    // barriers of the non-allocatable fallback: the per-engine kernel
+    if (pi.divergent || (!BB && pi.fb_iters > 0)) {
       if (lane == 0) {
         a.status[p] = SIM_FALLBACK;
         a.fallback[1 + atomicAdd(a.fallback, 1)] = p;
