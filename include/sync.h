@@ -143,7 +143,8 @@ enum {
  *     enforce (Sec. 5.2: a producer nested below S with a forward offset
  *     k >= 1 or a backward offset k >= 2, whose target lies in an earlier
  *     iteration of S): such a dependency gets no semaphore wait (its wait
- *     value is 0 in every threshold array and the checker skips its pairs)
+ *     value is 0 in every threshold array, and the checker takes 0 as its
+ *     minimum)
  *     and its carrying loop S, unless S is the top level, gets an all-engine
  *     barrier at the end of every iteration (drain-and-release, as in the
  *     barrier scheme) in the barrier-free simulation; the barrier scheme has
@@ -261,8 +262,9 @@ sync_status sync_eval_thresholds(const sync_programs *h, sync_thr_mode mode, int
  * d_counts: [2] uint64 device -- unsafe, over-synchronised pair counts;
  * d_first_bad: [1] int64 device -- smallest offending index into d_thr, or
  * -1.  Both are overwritten (no accumulation across calls); padding entries
- * of d_thr and the pairs of barrier-fallback dependencies (enforced by
- * barriers, not by a wait value) are ignored. */
+ * of d_thr are ignored.  A barrier-fallback dependency (SYNC_NONALLOC_BARRIER)
+ * is enforced by barriers, not by its wait value: its minimum is 0, so a
+ * positive stored value counts as over-synchronised. */
 sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const int32_t *d_thr,
                                unsigned long long *d_counts, long long *d_first_bad,
                                void *stream);

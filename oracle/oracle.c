@@ -779,11 +779,12 @@ int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[
     int64_t i = 0;
     for (int32_t d = 0; d < P.nd && rc == ORC_OK; ++d) {
       int64_t n = cons_total(&P, d);
-      if (classify(&P, d).kase == ORC_CASE_BARRIER) { i += n; continue; }   /* enforced by barriers */
+      /* a barrier enforces a barrier-fallback dependency: its minimum is 0 */
+      int bar = classify(&P, d).kase == ORC_CASE_BARRIER;
       for (int64_t j = 0; j < n; ++j, ++i) {
-        int32_t got = thr[base + i];
-        if (got == want[i]) continue;
-        counts[got < want[i] ? 0 : 1]++;
+        int32_t got = thr[base + i], need = bar ? 0 : want[i];
+        if (got == need) continue;
+        counts[got < need ? 0 : 1]++;
         if (*first_bad < 0) *first_bad = base + i;
       }
     }

@@ -114,8 +114,9 @@ int orc_register_replay(const orc_batch *b, int mode, int32_t *out);
 
 /* Minimality check of a threshold array against Eq. (1): counts[0] = pairs
  * whose threshold is below the minimum (unsafe), counts[1] = above it
- * (over-synchronised); first_bad = first such pair index or -1.  The pairs
- * of ORC_CASE_BARRIER dependencies are skipped (a barrier enforces them). */
+ * (over-synchronised); first_bad = first such pair index or -1.  An
+ * ORC_CASE_BARRIER dependency is enforced by a barrier: its minimum is 0, so
+ * any positive value over-synchronises. */
 int orc_check(const orc_batch *b, int mode, const int32_t *thr, uint64_t counts[2],
               int64_t *first_bad);
 

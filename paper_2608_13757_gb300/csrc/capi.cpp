@@ -462,12 +462,22 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         // with all-engine barriers (none at the top level, which runs once)
         if (div) raise(SYNC_ERR_ARG, where(p, "barrier fallback with per-engine trip counts, dependency", k));
         if (Sl != 0) S.fbar[Sl] = 1;
+        // for the threshold and check kernels: a producer in S with an offset
+        // no trip reaches, over a zero trip-start array (a derive job of
+        // length 0 fills its region with zeros), so the masked wait value
+        // (Eq. 2) and the required minimum are 0 on every pair
         DepInfo& D = dep[gd];
         std::memset(&D, 0, sizeof D);
         D.total = (int32_t)tot(Cl, ec);
         dep_count[gd] = D.total;
-        D.kase = kase;
-        D.k = off;
+        D.kase = CASE_PS;
+        D.k = (int32_t)kI32Max;
+        DeriveJob J{};
+        J.out = n_derived; J.n = 0; J.kind = DERIVE_TSTART;
+        jobs.push_back(J);
+        D.tstart = D.src = n_derived;
+        n_derived += pad4(tot(Cl, ec));
+        D.path = (int64_t)path.size();
         D.seg_off = n_pairs_padded;
         seg[gd] = n_pairs_padded;
         n_pairs += tot(Cl, ec);

@@ -48,8 +48,6 @@ __device__ __forceinline__ int find_dep(const ThrArgs& a, I q) {
 // non-decreasing), all in parallel.
 template <bool CHECK>
 __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D, int32_t g0, int mode) {
-  // a barrier-fallback dependency emits no wait (and has no derived arrays)
-  if (D.kase == CASE_BARRIER) return make_int4(0, 0, 0, 0);
   const int32_t n = D.total - g0 < kChunk ? D.total - g0 : kChunk;   // >= 1
   const int32_t* ts = a.derived + D.tstart;
   const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.src + g0));
@@ -162,14 +160,12 @@ __global__ void __launch_bounds__(kThreads, 8) k_check(const CheckArgs a) {
     if (c < n_chunks) {
       prefetch_l2(a.thr + q);
       const DepInfo D = a.t.dep[find_dep(a.t, q)];
-      if (D.kase != CASE_BARRIER) {              // barrier-fallback pairs: enforced by barriers
-        const int32_t g0 = (int32_t)(q - D.seg_off);
-        m = chunk_values<true>(a.t, D, g0, MODE);
-        v = __ldcs(reinterpret_cast<const int4*>(a.thr + q));
-        // padding entries are not pairs: the checker reads only the first n
-        n = D.total - g0;
-        bad = v.x != m.x || (n > 1 && v.y != m.y) || (n > 2 && v.z != m.z) || (n > 3 && v.w != m.w);
-      }
+      const int32_t g0 = (int32_t)(q - D.seg_off);
+      m = chunk_values<true>(a.t, D, g0, MODE);
+      v = __ldcs(reinterpret_cast<const int4*>(a.thr + q));
+      // padding entries are not pairs: the checker reads only the first n
+      n = D.total - g0;
+      bad = v.x != m.x || (n > 1 && v.y != m.y) || (n > 2 && v.z != m.z) || (n > 3 && v.w != m.w);
     }
     if (__ballot_sync(0xffffffffu, bad)) report(a, v, m, n, q, bad);
   }

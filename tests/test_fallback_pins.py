@@ -9,7 +9,8 @@ The pins: the classification, a timeline worked out by hand, the paper's
 dependency-satisfaction condition Eq. (1) holding on every simulated
 instance (the fallback must enforce what the wait would have), the barrier
 scheme being unchanged by the fallback, the static bound's barrier term, and
-the combinations the fallback does not take.  No GPU.
+the checker's minimum of 0 on barrier-enforced pairs, and the combinations
+the fallback does not take.  No GPU.
 """
 import numpy as np
 import pytest
@@ -180,7 +181,7 @@ def test_barrier_scheme_is_unchanged_by_the_fallback():
         assert np.array_equal(r0.checksum, r1.checksum)
 
 
-def test_check_skips_barrier_pairs_and_replay_matches_eq1_elsewhere():
+def test_check_on_barrier_pairs_and_replay_matches_eq1_elsewhere():
     b = with_policy(workloads.random_trees(20262, 120, workloads.tree_params(**FAR)), 1)
     cls = oracle.classify(b).kase
     for mode in (COUNT, PERLOOP):
@@ -193,8 +194,11 @@ def test_check_skips_barrier_pairs_and_replay_matches_eq1_elsewhere():
         assert np.array_equal(rep[~bar], eq1[~bar])            # Thm. 1 on the allocatable pairs
         assert oracle.check(b, rep, mode)[:2] == (0, 0)
         junk = rep.copy()
-        junk[bar] = 12345                                      # not read: enforced by barriers
-        assert oracle.check(b, junk, mode)[:2] == (0, 0)
+        junk[bar] = 12345                  # a barrier enforces these: any wait is one too many
+        assert oracle.check(b, junk, mode)[:2] == (0, int(bar.sum()))
+        eq1_there = rep.copy()
+        eq1_there[bar] = eq1[bar]          # Eq. (1)'s count waited on as well: redundant
+        assert oracle.check(b, eq1_there, mode)[:2] == (0, int((eq1[bar] > 0).sum()))
 
 
 def test_bound_counts_the_fallback_barriers():

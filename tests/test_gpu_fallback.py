@@ -2,7 +2,7 @@
 
 A batch loaded with SYNC_NONALLOC_BARRIER: nested producers with a forward
 offset >= 1 or a backward offset >= 2 get no semaphore wait (wait value 0,
-skipped by the checker) and their carrying loop ends every iteration with an
+the checker's minimum) and their carrying loop ends every iteration with an
 all-engine barrier.  Thresholds, check, barrier-free and barrier
 simulations (array and fused, every mode, full timelines) must equal the
 oracle's; the rejected combinations must fail loudly.
@@ -109,19 +109,22 @@ def test_fallback_hand_timeline(sg):
     assert r.makespan.cpu().tolist()[:1] == [148]
 
 
-def test_fallback_check_ignores_barrier_pairs(sg):
+def test_fallback_check_minimum_zero_on_barrier_pairs(sg):
     b = with_policy(workloads.random_trees(31020, 80, workloads.tree_params(**FAR)), 1)
     h = sg.sync_load_programs(b)
     thr, got = gpu_thresholds(sg, h, PERLOOP)
     idx = h.unpadded_index()
     bar = barrier_pairs(b)
     assert bar.any()
+    import torch
     junk = thr.clone()
-    junk[idx[bar]] = 777                          # not read: barriers enforce these
+    sel = torch.from_numpy(idx[bar]).to(junk.device)
+    junk[sel] = 777                               # barriers enforce these: a wait over-synchronises
     counts, fb = sg.sync_check_minimal(h, PERLOOP, junk)
-    assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
-    i = int(np.flatnonzero(~bar & (got > 0))[0])  # a waited pair: still checked
-    junk[idx[i]] = 0
+    assert counts.cpu().tolist() == [0, int(bar.sum())] and fb.item() == int(idx[bar][0])
+    i = int(np.flatnonzero(~bar & (got > 0))[0])  # a waited pair below its minimum: unsafe
+    junk[sel] = 0
+    junk[int(idx[i])] = 0
     counts, fb = sg.sync_check_minimal(h, PERLOOP, junk)
     assert counts.cpu().tolist() == [1, 0] and fb.item() == int(idx[i])
 
