@@ -134,18 +134,25 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def traffic_for(kernel: str, workload: str):
-    """DRAM bytes per launch from a committed ncu summary, if it was taken on
-    the current kernel sources."""
+def profile_entry(kernel: str, workload: str):
+    """A kernel's record in the committed ncu summary (profiles/traffic.json),
+    if it was taken on the current kernel sources."""
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             d = json.load(f)
         e = d.get(workload, {}).get(kernel)
         if e and e.get("source_hash") == kernel_hash():
-            return e["dram_bytes_per_launch"]
+            return e
     except Exception:
         pass
     return None
+
+
+def traffic_for(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel sources."""
+    e = profile_entry(kernel, workload)
+    return e["dram_bytes_per_launch"] if e else None
 
 
 def run_gpu(args, rank, world, local_rank):
@@ -455,6 +462,17 @@ def roofline(res, hbm_peak, peak_kind, sm_mhz, workload):
         kernels[name] = {"bound": "alu", "ms": pk[name], "achieved": ach, "peak": lanes_peak,
                          "unit": "Tops/s", "frac": ach / lanes_peak, "alg_ops": ops,
                          "traffic": traffic_for(name, workload)}
+        # what bounds the sweep in practice: warp-instruction issue (one per
+        # SM sub-partition per cycle); instructions per instance from the
+        # committed capture of the same sources, times live CUDA-event time
+        e = profile_entry(name, workload)
+        if e and e.get("warp_inst_per_instance") and t > 0:
+            wi = e["warp_inst_per_instance"] * sz.n_instances
+            ipk = 152 * 4 * (sm_mhz or 2070.0) * 1e6 / 1e9
+            kernels[name]["issue"] = {"warp_inst_per_instance": e["warp_inst_per_instance"],
+                                      "achieved": wi / t / 1e9, "peak": ipk, "unit": "Ginst/s",
+                                      "frac": wi / t / 1e9 / ipk,
+                                      "source": "instructions per instance from the 8192-program ncu capture"}
     dom = max(pk, key=pk.get)
     d = dict(kernels[dom])
     d["kernel"] = dom
