@@ -100,3 +100,36 @@ def test_noalloc_refuses_batches_beyond_its_scratch(sg):
     assert err.value.status == sg.ERR_ARG
     assert "scratch" in str(err.value)
     h.close()
+
+
+def test_noalloc_with_the_barrier_fallback(sg):
+    """Programs with fallback barriers (handed to the per-engine kernel,
+    barrier-free) beside ordinary ones: the same results as sync_simulate,
+    and the unrolled variant refused here too."""
+    import torch
+    from tests.test_fallback_pins import FAR, nested_program
+    batch = workloads.concat([workloads.generate("depth2", n_programs=8),
+                              workloads.random_trees(43, 40, workloads.tree_params(**FAR)),
+                              nested_program(1), nested_program(3, backward=True)])
+    batch.nonalloc_policy = 1
+    h = sg.sync_load_programs(batch)
+    inst = _instances_per_program(batch)
+    for mode in (sg.THR_COUNT, sg.THR_PERLOOP, sg.THR_PERENGINE):
+        thr = sg.sync_eval_thresholds(h, mode)
+        for variant in (sg.SIM_BARRIER_FREE, sg.SIM_BARRIER):
+            ref = sg.sync_simulate(h, mode, thr, variant=variant, timeline=True)
+            torch.cuda.synchronize()
+            ok = ref.status.cpu().numpy() == sg.PROG_OK
+            defined = torch.from_numpy(np.repeat(ok, inst)).cuda()
+            out = _outputs(sg, h)
+            sg.sync_simulate_noalloc(h, mode, thr, variant=variant, out=out)
+            torch.cuda.synchronize()
+            for f in ("status", "makespan", "checksum"):
+                assert torch.equal(getattr(out, f), getattr(ref, f)), (mode, variant, f)
+            for f in ("issue", "retire"):
+                assert torch.equal(getattr(out, f)[defined], getattr(ref, f)[defined]), (mode, variant, f)
+    thr = sg.sync_eval_thresholds(h, sg.THR_PERENGINE)
+    with pytest.raises(sg.SyncError) as err:
+        sg.sync_simulate_noalloc(h, sg.THR_PERENGINE, thr, variant=sg.SIM_UNROLLED, out=_outputs(sg, h))
+    assert err.value.status == sg.ERR_ARG
+    h.close()
