@@ -200,15 +200,24 @@ __device__ __forceinline__ void set_groups(const WarpSmem& S, const LaneRec& L, 
   __syncwarp();
 }
 
+// Barrier scheme, iterations of one loop through run_chunk: the lane's
+// schedule of the last fully computed iteration relative to its start, and
+// the in-chunk increments its waits targeted.
+struct BbRep {
+  bool on = false;
+  int32_t sig = 0, issue = 0, retire = 0, t = 0;
+};
+
 // One chunk: `copies` iterations (g .. g+copies-1) of a segment's records,
 // given the lane's record, its first thresholds T and the semaphore groups
 // of this chunk (set_groups with the same copies and ctag).  Returns 0,
-// SYNC_PROG_DEADLOCK or SIM_FALLBACK.
-template <int MODE, bool BB, bool TL, bool FUSED>
+// SYNC_PROG_DEADLOCK or SIM_FALLBACK.  REP (barrier scheme, consecutive
+// iterations of one loop): see the replay below.
+template <int MODE, bool BB, bool TL, bool FUSED, bool REP = false>
 __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, const LaneRec& L,
                                          const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
                                          int32_t ctag, int lane, int lc, int32_t lo_c, int32_t iter_cost,
-                                         unsigned long long& chk) {
+                                         unsigned long long& chk, BbRep& rp) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int4 rec = L.rec, sr = L.sr;
   const bool have = lane < ch.y;
@@ -254,8 +263,28 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
   const int32_t wcost = BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * sr.w : 0);
   const int32_t apre = (L.meta.w & LANE_ITER_START) ? iter_cost : 0;
   const int32_t A = valid ? apre + wcost + a.prm.ii : 0;
-  int32_t r_intra = kNeg;                      // retire of in-chunk producers (lower bound)
   int32_t issue = 0, retire = 0, t_after = 0;
+  // REP: every engine starts the iteration at the same cursor t_in with all
+  // earlier work retired (the barriers before the loop statement and after
+  // each iteration), so only in-chunk waits can bind and the schedule
+  // relative to t_in depends only on which in-chunk increments the waits
+  // target (their source lanes, 5 bits each, and their count): the same
+  // targets as the last computed iteration give its schedule, shifted
+  int32_t sig = 0;
+  bool replay = false;
+  if (REP) {
+    sig = n_intra;
+#pragma unroll
+    for (int i = 0; i < kMaxIntra; ++i)
+      if (i < n_intra) sig |= intra[i] << (3 + 5 * i);
+    replay = rp.on && !__ballot_sync(kFull, valid && sig != rp.sig);
+  }
+  if (replay) {
+    issue = t_in + rp.issue;
+    retire = t_in + rp.retire;
+    t_after = t_in + rp.t;
+  } else {
+  int32_t r_intra = kNeg;                      // retire of in-chunk producers (lower bound)
   const bool any_intra = __ballot_sync(kFull, n_intra > 0) != 0;
   const int passes = any_intra ? ch.y + 2 : 1;
   bool settled = false;
@@ -293,6 +322,14 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
     r_intra = nr;
   }
   if (!settled) return SYNC_PROG_DEADLOCK;   // a cycle of waits inside the chunk
+  if (REP) {
+    rp.on = true;
+    rp.sig = sig;
+    rp.issue = issue - t_in;
+    rp.retire = retire - t_in;
+    rp.t = t_after - t_in;
+  }
+  }
 
   // publish increments, instance counts, checksum terms, engine state
   const unsigned vm = __ballot_sync(kFull, valid);
@@ -633,6 +670,7 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
   set_groups(S, L, lane, have, min(copies, hi - lo), ctag);
   int32_t Tn[kMaxDeps];
   load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - lo, lo + L.meta.y, lc, lo, Tn);
+  BbRep rp;                                     // barrier scheme: replayed iterations
   for (int32_t g = lo; g < hi;) {
     const int32_t v = min(copies, hi - g);
     int32_t T[kMaxDeps];
@@ -641,7 +679,7 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
     const int32_t gn = g + v;
     if (gn < hi) load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - gn, gn + L.meta.y, lc, lo, Tn);
     if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
-    const int verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk);
+    const int verdict = run_chunk<MODE, BB, TL, FUSED, BB>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk, rp);
     if (verdict) return verdict;
     g = gn;
     if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
@@ -699,6 +737,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     if (slot >= a.n_programs) break;
     const int p = __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
+    BbRep no_rep;                     // a segment's chunk is not replayed
     // engines on their own trips (no common walk), or barrier-free with the
     // barriers of the non-allocatable fallback: the per-engine kernel
     if (pi.divergent || (!BB && pi.fb_iters > 0)) {
@@ -795,7 +834,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
         load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y && Lr.meta.y < v, g + Lr.meta.y, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, v, ++ctag);
-        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, iter_cost, chk);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, iter_cost, chk, no_rep);
         if (verdict) break;
         g += v - 1;
         item = pend - pbeg;                            // continue at the END of iteration g
@@ -809,7 +848,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
         load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y, g, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, 1, ++ctag);
-        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, iter_cost, chk);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, iter_cost, chk, no_rep);
       }
       if (verdict) break;
       ++item;
