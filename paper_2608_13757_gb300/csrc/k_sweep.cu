@@ -208,16 +208,24 @@ struct BbRep {
   int32_t sig = 0, issue = 0, retire = 0, t = 0;
 };
 
+// Barrier-free, whole iterations of one loop through run_chunk: the lane's
+// issue and retire in the last computed iteration and their change since
+// the one before (n: iterations computed so far).
+struct BfPred {
+  int n = 0;
+  int32_t issue = 0, retire = 0, d_issue = 0, d_retire = 0;
+};
+
 // One chunk: `copies` iterations (g .. g+copies-1) of a segment's records,
 // given the lane's record, its first thresholds T and the semaphore groups
 // of this chunk (set_groups with the same copies and ctag).  Returns 0,
 // SYNC_PROG_DEADLOCK or SIM_FALLBACK.  REP (barrier scheme, consecutive
 // iterations of one loop): see the replay below.
-template <int MODE, bool BB, bool TL, bool FUSED, bool REP = false>
+template <int MODE, bool BB, bool TL, bool FUSED, bool REP = false, bool PRED = false>
 __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, const int4 ch, const LaneRec& L,
                                          const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
                                          int32_t ctag, int lane, int lc, int32_t lo_c, int32_t iter_cost,
-                                         unsigned long long& chk, BbRep& rp) {
+                                         unsigned long long& chk, BbRep& rp, BfPred& pd) {
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int4 rec = L.rec, sr = L.sr;
   const bool have = lane < ch.y;
@@ -279,11 +287,49 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
       if (i < n_intra) sig |= intra[i] << (3 + 5 * i);
     replay = rp.on && !__ballot_sync(kFull, valid && sig != rp.sig);
   }
+  // PRED (barrier-free, whole iterations): extrapolate each lane's issue and
+  // retire from the last two iterations and run one pass of the model on
+  // it; if the pass reproduces the prediction on every lane, the prediction
+  // is a fixed point of the chunk's equations -- and they have exactly one
+  // (a cycle of waits admits none: along it each issue would have to follow
+  // its own retirement), so it is the schedule the relaxation would reach
+  bool predicted = false;
+  if (PRED && pd.n >= 2) {
+    const int32_t pi_ = pd.issue + pd.d_issue, pr_ = pd.retire + pd.d_retire;
+    int32_t nr = kNeg;
+#pragma unroll
+    for (int i = 0; i < kMaxIntra; ++i) {
+      const int32_t src = i < n_intra ? intra[i] : lane;
+      const int32_t rv = __shfl_sync(kFull, pr_, src);
+      if (i < n_intra) nr = max(nr, rv);
+    }
+    const int32_t ready = max(known, nr);
+    int32_t Ai = A, Bi = (valid && ready >= 0) ? ready + a.prm.ii : kNeg;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t Ap = __shfl_up_sync(kFull, Ai, o), Bp = __shfl_up_sync(kFull, Bi, o);
+      if (lane - o >= head) { Bi = max(Bp + Ai, Bi); Ai = Ap + Ai; }
+    }
+    const int32_t ta = max(t_in + Ai, Bi);
+    int32_t vv = valid ? ta - a.prm.ii + rec.y : kNeg;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t vp = __shfl_up_sync(kFull, vv, o);
+      if (lane - o >= head) vv = max(vv, vp);
+    }
+    const int32_t rt = max(lr_in, vv);
+    predicted = !__ballot_sync(kFull, valid && (ta - a.prm.ii != pi_ || rt != pr_));
+    if (predicted) {
+      t_after = ta;
+      issue = ta - a.prm.ii;
+      retire = rt;
+    }
+  }
   if (replay) {
     issue = t_in + rp.issue;
     retire = t_in + rp.retire;
     t_after = t_in + rp.t;
-  } else {
+  } else if (!predicted) {
   int32_t r_intra = kNeg;                      // retire of in-chunk producers (lower bound)
   const bool any_intra = __ballot_sync(kFull, n_intra > 0) != 0;
   const int passes = any_intra ? ch.y + 2 : 1;
@@ -329,6 +375,13 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
     rp.retire = retire - t_in;
     rp.t = t_after - t_in;
   }
+  }
+  if (PRED) {
+    pd.d_issue = issue - pd.issue;
+    pd.d_retire = retire - pd.retire;
+    pd.issue = issue;
+    pd.retire = retire;
+    ++pd.n;
   }
 
   // publish increments, instance counts, checksum terms, engine state
@@ -671,6 +724,7 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
   int32_t Tn[kMaxDeps];
   load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - lo, lo + L.meta.y, lc, lo, Tn);
   BbRep rp;                                     // barrier scheme: replayed iterations
+  BfPred pd;                                    // barrier-free: predicted iterations
   for (int32_t g = lo; g < hi;) {
     const int32_t v = min(copies, hi - g);
     int32_t T[kMaxDeps];
@@ -679,7 +733,9 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
     const int32_t gn = g + v;
     if (gn < hi) load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - gn, gn + L.meta.y, lc, lo, Tn);
     if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
-    const int verdict = run_chunk<MODE, BB, TL, FUSED, BB>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk, rp);
+    if (!BB && v < copies) pd.n = 0;            // the last, partial chunk: not predicted
+    const int verdict =
+        run_chunk<MODE, BB, TL, FUSED, BB, !BB>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk, rp, pd);
     if (verdict) return verdict;
     g = gn;
     if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
@@ -737,7 +793,8 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     if (slot >= a.n_programs) break;
     const int p = __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
-    BbRep no_rep;                     // a segment's chunk is not replayed
+    BbRep no_rep;                     // a segment's chunk is neither replayed
+    BfPred no_pred;                   // nor predicted
     // engines on their own trips (no common walk), or barrier-free with the
     // barriers of the non-allocatable fallback: the per-engine kernel
     if (pi.divergent || (!BB && pi.fb_iters > 0)) {
@@ -834,7 +891,8 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
         load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y && Lr.meta.y < v, g + Lr.meta.y, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, v, ++ctag);
-        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, iter_cost, chk, no_rep);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, iter_cost, chk, no_rep,
+                                                  no_pred);
         if (verdict) break;
         g += v - 1;
         item = pend - pbeg;                            // continue at the END of iteration g
@@ -848,7 +906,8 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         const int32_t lo_c = FUSED ? S.lvl[sp].y : 0;
         load_thr<MODE, FUSED>(a, S, Lr, lane < ch.y, g, sp, lo_c, T);
         set_groups(S, Lr, lane, lane < ch.y, 1, ++ctag);
-        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, iter_cost, chk, no_rep);
+        verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, 1, ctag, lane, sp, lo_c, iter_cost, chk, no_rep,
+                                                  no_pred);
       }
       if (verdict) break;
       ++item;
