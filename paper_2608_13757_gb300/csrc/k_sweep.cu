@@ -747,6 +747,68 @@ __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, c
   return 0;
 }
 
+// A loop statement whose one iteration (global index g, walk level lc) runs
+// a one-record chunk -- a conditional around one instruction, the common
+// shape of synchronisation-bound code: the instance's cursor map applied
+// directly, without scans.  Lane 0 takes the wait decisions (so a fused
+// check counts each pair once); the verdicts are run_chunk's: a wait past
+// the published increments hands the program over, one on its own
+// increment is a cycle.
+template <int MODE, bool BB, bool TL, bool FUSED>
+__device__ __forceinline__ int run_single(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi,
+                                          const int4 ch, int32_t g, int lane, int lc,
+                                          unsigned long long& chk) {
+  const int4 rec = __ldg(a.lrec + ch.x), sr = __ldg(a.lsem + ch.x);
+  const int32_t e = __ldg(a.lmeta + ch.x).x;
+  int32_t ready = kNeg;
+  int flag = 0;                                 // 1: a cycle, 2: handed over
+  if (lane == 0) {
+    for (int j = 0; j < rec.z; ++j) {
+      const int32_t T = FUSED ? fused_wait<MODE>(a, S, rec.w + j, g, lc, g)
+                              : __ldg(a.thr + __ldg(a.dseg + rec.w + j) + g);
+      if (T <= 0) continue;
+      const int32_t s = __ldg(a.dsem + rec.w + j), pub = S.semv[s];
+      if (T <= pub) {
+        ready = max(ready, pub - T <= S.rmask ? S.ring[s * (S.rmask + 1) + ((T - 1) & S.rmask)]
+                                              : a.hist[S.semhb[s] + (T - 1)]);
+      } else {
+        flag = max(flag, s == sr.x && T - pub == 1 ? 1 : 2);
+      }
+    }
+  }
+  flag = __shfl_sync(kFull, flag, 0);
+  if (flag == 2) return SIM_FALLBACK;
+  if (flag == 1) return SYNC_PROG_DEADLOCK;
+  ready = __shfl_sync(kFull, ready, 0);
+  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
+  const int32_t wcost = BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * sr.w : 0);
+  const int32_t t_in = S.t[e], lr_in = S.lr[e];
+  const uint32_t nj = (uint32_t)S.nn[e] + 1;
+  const int32_t t_after = max(t_in + wcost + a.prm.ii, ready >= 0 ? ready + a.prm.ii : kNeg);
+  const int32_t issue = t_after - a.prm.ii, retire = max(lr_in, issue + rec.y);
+  __syncwarp();
+  if (lane == 0) {
+    if (sr.x >= 0) {
+      const int32_t n = sr.y < 0 ? (int32_t)nj : sr.y * g + sr.z;
+      S.ring[sr.x * (S.rmask + 1) + ((n - 1) & S.rmask)] = retire;
+      a.hist[S.semhb[sr.x] + (n - 1)] = retire;
+      S.semv[sr.x] += 1;
+    }
+    chk += inst_term(issue, retire, (uint32_t)e, nj);
+    if (TL) {
+      const int64_t o = __ldg(a.inst_off + rec.x) + g;
+      a.issue[o] = issue;
+      a.retire[o] = retire;
+    }
+    S.t[e] = t_after;
+    S.lr[e] = retire;
+    S.nn[e] = (int32_t)nj;
+  }
+  __syncwarp();
+  if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
+  return 0;
+}
+
 template <int MODE, bool BB, bool TL, bool FUSED>
 __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -863,9 +925,14 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
           if (lane < pi.ne) S.t[lane] += child_ic;    // the first iteration starts
           __syncwarp();
           if (body_chunk >= 0) {
-            // a loop around one chunk: all its iterations in registers
-            verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + body_chunk), lo, hi, ++ctag, lane,
-                                                    sp + 1, child_ic, chk);
+            // one iteration of one record: applied directly; otherwise a
+            // loop around one chunk: all its iterations in registers
+            const int4 one = hi - lo == 1 && ax.w >= 0 ? __ldg(a.chunk + ax.w) : make_int4(0, 0, 0, 0);
+            if (one.y == 1)
+              verdict = run_single<MODE, BB, TL, FUSED>(a, S, pi, one, lo, lane, sp + 1, chk);
+            else
+              verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + body_chunk), lo, hi, ++ctag, lane,
+                                                      sp + 1, child_ic, chk);
             if (verdict) break;
             continue;
           }
