@@ -706,47 +706,6 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
   return 0;
 }
 
-// Iterations lo .. hi-1 of a loop whose body is one straight-line segment of
-// one chunk (or, barrier-free, one multi-iteration chunk); the first
-// iteration start has been charged.  The lane's record and thresholds stay
-// in registers; the next chunk's thresholds load while this one runs.
-template <int MODE, bool BB, bool TL, bool FUSED>
-__device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi, const int4 ch,
-                                        int32_t lo, int32_t hi, int32_t ctag, int lane, int lc,
-                                        int32_t iter_cost, unsigned long long& chk) {
-  const int32_t copies = ch.z;
-  const bool have = lane < ch.y;
-  LaneRec L;
-  load_lane(a, ch, lane, L);
-  if (!__ballot_sync(kFull, have && L.rec.z > kMaxDeps))
-    return run_loop_regs<MODE, BB, TL, FUSED>(a, S, pi, ch, L, lo, hi, ctag, lane, lc, iter_cost, chk);
-  set_groups(S, L, lane, have, min(copies, hi - lo), ctag);
-  int32_t Tn[kMaxDeps];
-  load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - lo, lo + L.meta.y, lc, lo, Tn);
-  BbRep rp;                                     // barrier scheme: replayed iterations
-  BfPred pd;                                    // barrier-free: predicted iterations
-  for (int32_t g = lo; g < hi;) {
-    const int32_t v = min(copies, hi - g);
-    int32_t T[kMaxDeps];
-#pragma unroll
-    for (int j = 0; j < kMaxDeps; ++j) T[j] = Tn[j];
-    const int32_t gn = g + v;
-    if (gn < hi) load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - gn, gn + L.meta.y, lc, lo, Tn);
-    if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
-    if (!BB && v < copies) pd.n = 0;            // the last, partial chunk: not predicted
-    const int verdict =
-        run_chunk<MODE, BB, TL, FUSED, BB, !BB>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk, rp, pd);
-    if (verdict) return verdict;
-    g = gn;
-    if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
-    if (g < hi) {
-      if (lane < pi.ne) S.t[lane] += iter_cost;
-      __syncwarp();
-    }
-  }
-  return 0;
-}
-
 // A loop statement whose one iteration (global index g, walk level lc) runs
 // a one-record chunk -- a conditional around one instruction, the common
 // shape of synchronisation-bound code: the instance's cursor map applied
@@ -806,6 +765,51 @@ __device__ __forceinline__ int run_single(const SweepArgs& a, const WarpSmem& S,
   }
   __syncwarp();
   if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
+  return 0;
+}
+
+// Iterations lo .. hi-1 of a loop whose body is one straight-line segment of
+// one chunk (or, barrier-free, one multi-iteration chunk); the first
+// iteration start has been charged.  The lane's record and thresholds stay
+// in registers; the next chunk's thresholds load while this one runs.
+template <int MODE, bool BB, bool TL, bool FUSED>
+__device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi, const int4 ch,
+                                        int32_t single, int32_t lo, int32_t hi, int32_t ctag, int lane, int lc,
+                                        int32_t iter_cost, unsigned long long& chk) {
+  if (single >= 0) {                            // one iteration: of one record?
+    const int4 one = __ldg(a.chunk + single);
+    if (one.y == 1) return run_single<MODE, BB, TL, FUSED>(a, S, pi, one, lo, lane, lc, chk);
+  }
+  const int32_t copies = ch.z;
+  const bool have = lane < ch.y;
+  LaneRec L;
+  load_lane(a, ch, lane, L);
+  if (!__ballot_sync(kFull, have && L.rec.z > kMaxDeps))
+    return run_loop_regs<MODE, BB, TL, FUSED>(a, S, pi, ch, L, lo, hi, ctag, lane, lc, iter_cost, chk);
+  set_groups(S, L, lane, have, min(copies, hi - lo), ctag);
+  int32_t Tn[kMaxDeps];
+  load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - lo, lo + L.meta.y, lc, lo, Tn);
+  BbRep rp;                                     // barrier scheme: replayed iterations
+  BfPred pd;                                    // barrier-free: predicted iterations
+  for (int32_t g = lo; g < hi;) {
+    const int32_t v = min(copies, hi - g);
+    int32_t T[kMaxDeps];
+#pragma unroll
+    for (int j = 0; j < kMaxDeps; ++j) T[j] = Tn[j];
+    const int32_t gn = g + v;
+    if (gn < hi) load_thr<MODE, FUSED>(a, S, L, have && L.meta.y < hi - gn, gn + L.meta.y, lc, lo, Tn);
+    if (v < copies && g > lo) set_groups(S, L, lane, have, v, ctag);   // the last, partial chunk
+    if (!BB && v < copies) pd.n = 0;            // the last, partial chunk: not predicted
+    const int verdict =
+        run_chunk<MODE, BB, TL, FUSED, BB, !BB>(a, S, ch, L, T, g, v, ctag, lane, lc, lo, iter_cost, chk, rp, pd);
+    if (verdict) return verdict;
+    g = gn;
+    if (BB) barrier_all(S, pi.ne, a.prm.c_barrier, lane);
+    if (g < hi) {
+      if (lane < pi.ne) S.t[lane] += iter_cost;
+      __syncwarp();
+    }
+  }
   return 0;
 }
 
@@ -927,12 +931,9 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
           if (body_chunk >= 0) {
             // one iteration of one record: applied directly; otherwise a
             // loop around one chunk: all its iterations in registers
-            const int4 one = hi - lo == 1 && ax.w >= 0 ? __ldg(a.chunk + ax.w) : make_int4(0, 0, 0, 0);
-            if (one.y == 1)
-              verdict = run_single<MODE, BB, TL, FUSED>(a, S, pi, one, lo, lane, sp + 1, chk);
-            else
-              verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + body_chunk), lo, hi, ++ctag, lane,
-                                                      sp + 1, child_ic, chk);
+            verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + body_chunk),
+                                                    hi - lo == 1 ? ax.w : -1, lo, hi, ++ctag, lane,
+                                                    sp + 1, child_ic, chk);
             if (verdict) break;
             continue;
           }
