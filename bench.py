@@ -9,8 +9,10 @@ consumer instance) pairs -- per second, summed over all ranks.
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
 With N > 1 the script runs under torchrun, one rank per GPU; every rank
-processes its own programs (program ids rank*P .. rank*P+P-1, weak scaling)
-and no data crosses ranks.  Rank 0 prints one JSON line.
+processes its own programs (program ids rank*P .. rank*P+P-1, weak scaling),
+or with --split one batch cut into contiguous program ranges of about equal
+instance counts (strong scaling); no data crosses ranks.  Rank 0 prints one
+JSON line.
 """
 from __future__ import annotations
 
@@ -61,6 +63,9 @@ def parse():
     ap.add_argument("--programs", type=int, default=None, help="programs per rank")
     ap.add_argument("--first-program", type=int, default=0,
                     help="id of rank 0's first program (ranks follow contiguously)")
+    ap.add_argument("--split", action="store_true",
+                    help="strong scaling: one batch (--programs, default the config's) cut into contiguous "
+                         "program ranges of about equal instance counts, one per rank")
     ap.add_argument("--mode", choices=("perloop", "count"), default="perloop")
     ap.add_argument("--pipeline", choices=("arrays", "fused"), default="arrays",
                     help="arrays: threshold kernel, checker, two simulations over the stored thresholds; "
@@ -162,7 +167,13 @@ def run_gpu(args, rank, world, local_rank):
 
     torch.cuda.set_device(local_rank)
     mode = sg.THR_PERLOOP if args.mode == "perloop" else sg.THR_COUNT
-    first, P = shard(rank, args.programs or workloads.CONFIGS[args.config][1])
+    total = args.programs or workloads.CONFIGS[args.config][1]
+    if args.split:
+        whole = workloads.generate(args.config, n_programs=total, first_program=args.first_program)
+        first, P = split_balanced(instances_per_program(whole), world)[rank]
+        del whole
+    else:
+        first, P = shard(rank, total)
     first += args.first_program
     batch = workloads.generate(args.config, n_programs=P, first_program=first)
     t0 = time.perf_counter()
@@ -228,7 +239,8 @@ def run_gpu(args, rank, world, local_rank):
     if fused:                             # no threshold kernel or checker launched
         per_kernel["thresholds"] = per_kernel["check"] = 0.0
     out = dict(ms=total_ms / args.steps, per_kernel=per_kernel, sizes=sz, clocks=clk, ok=ok,
-               load_s=load_s, P=P)
+               load_s=load_s, P=P, first=first,
+               num_sms=torch.cuda.get_device_properties(dev).multi_processor_count)
     if not args.no_e2e:
         out["e2e"] = run_e2e(args, sg, batch, mode, prm, dev, P)
     h.close()
@@ -331,6 +343,41 @@ def run_e2e(args, sg, batch, mode, prm, dev, P):
 def shard(rank: int, programs_per_rank: int):
     """Program ids of a rank: rank*P .. rank*P+P-1 (weak scaling, no overlap)."""
     return rank * programs_per_rank, programs_per_rank
+
+
+def instances_per_program(batch):
+    """Dynamic datapath instances of every program of a batch (shared trips):
+    a loop's iterations are the sum of its trips, an instruction has one
+    instance per iteration of its loop."""
+    import numpy as np
+    tp = np.asarray(batch.trip_ptr, dtype=np.int64)
+    trips = np.asarray(batch.trips, dtype=np.int64)
+    csum = np.concatenate([[0], np.cumsum(trips)])
+    loop_total = csum[tp[1:]] - csum[tp[:-1]]
+    inst = loop_total[np.asarray(batch.instr_loop, dtype=np.int64) +
+                      np.repeat(np.asarray(batch.prog_loop_ptr[:-1], dtype=np.int64),
+                                np.diff(batch.prog_instr_ptr))]
+    isum = np.concatenate([[0], np.cumsum(inst)])
+    ip = np.asarray(batch.prog_instr_ptr, dtype=np.int64)
+    return isum[ip[1:]] - isum[ip[:-1]]
+
+
+def split_balanced(work, world: int):
+    """Contiguous program ranges [(first, count)] for `world` ranks over
+    per-program `work`: rank r's range ends at the first program whose
+    cumulative work reaches r+1 world-ths of the total (strong scaling: the
+    ranks process one batch, each about the same number of instances)."""
+    import numpy as np
+    work = np.asarray(work, dtype=np.int64)
+    cum = np.cumsum(work)
+    total = int(cum[-1]) if cum.size else 0
+    cuts = [0]
+    for r in range(1, world):
+        target = total * r // world
+        cuts.append(max(cuts[-1], int(np.searchsorted(cum, target, side="left")) + 1 if total else 0))
+    cuts.append(int(work.size))
+    cuts = [min(c, int(work.size)) for c in cuts]
+    return [(cuts[r], cuts[r + 1] - cuts[r]) for r in range(world)]
 
 
 def reduce_over_ranks(ms: float, e2e_s, pairs: int, device):
@@ -438,6 +485,7 @@ def run_reference(args, rank, world):
 
 def roofline(res, hbm_peak, peak_kind, sm_mhz, workload):
     sz, pk = res["sizes"], res["per_kernel"]
+    sms = res.get("num_sms") or 152
     # algorithmic bytes per launch: thresholds written / read once (padded
     # array) plus the loop-structure arrays and tables, each once
     alg = {"thresholds": 4 * sz.n_pairs_padded + sz.struct_bytes,
@@ -450,11 +498,19 @@ def roofline(res, hbm_peak, peak_kind, sm_mhz, workload):
         ach = alg[name] / t / 1e9 if t > 0 else 0.0
         kernels[name] = {"bound": "hbm", "ms": pk[name], "achieved": ach, "peak": hbm_peak,
                          "unit": "GB/s", "frac": ach / hbm_peak, "alg_bytes": alg[name],
+                         "out_bytes": 4 * sz.n_pairs_padded,
+                         "frac_out_only": 4 * sz.n_pairs_padded / t / 1e9 / hbm_peak if t > 0 else 0.0,
                          "traffic": traffic_for(name, workload)}
+        # the same time against the DRAM bytes ncu measured for this kernel
+        # (a full-size capture of the current sources), when there is one
+        if kernels[name]["traffic"] and t > 0:
+            kernels[name]["dram_achieved"] = kernels[name]["traffic"] / t / 1e9
+            kernels[name]["dram_frac"] = kernels[name]["dram_achieved"] / hbm_peak
     # simulator: integer ops of the max-plus recurrence (per instance: wait
     # cost, one max per dependency, issue, retire max, cursor, checksum terms)
-    # against the SM integer lanes: 152 SMs x 128 lanes x clock
-    lanes_peak = 152 * 128 * (sm_mhz or 2070.0) * 1e6 / 1e12
+    # against the SM integer lanes: SMs x 128 int32 lanes x clock (nominal
+    # unit counts, not a measured peak)
+    lanes_peak = sms * 128 * (sm_mhz or 2070.0) * 1e6 / 1e12
     for name in ("sim_barrier_free", "sim_barrier"):
         ops = 12 * sz.n_instances + 2 * sz.n_pairs
         t = pk[name] / 1e3
@@ -468,15 +524,17 @@ def roofline(res, hbm_peak, peak_kind, sm_mhz, workload):
         e = profile_entry(name, workload)
         if e and e.get("warp_inst_per_instance") and t > 0:
             wi = e["warp_inst_per_instance"] * sz.n_instances
-            ipk = 152 * 4 * (sm_mhz or 2070.0) * 1e6 / 1e9
+            ipk = sms * 4 * (sm_mhz or 2070.0) * 1e6 / 1e9
             kernels[name]["issue"] = {"warp_inst_per_instance": e["warp_inst_per_instance"],
                                       "achieved": wi / t / 1e9, "peak": ipk, "unit": "Ginst/s",
                                       "frac": wi / t / 1e9 / ipk,
-                                      "source": "instructions per instance from the 8192-program ncu capture"}
+                                      "source": e.get("issue_source", "instructions per instance from an "
+                                                                      "ncu capture of the current sources")}
     dom = max(pk, key=pk.get)
     d = dict(kernels[dom])
     d["kernel"] = dom
-    d["peak_source"] = peak_kind if d["bound"] == "hbm" else "derived: 152 SMs x 128 int32 lanes x SM clock"
+    d["peak_source"] = (peak_kind if d["bound"] == "hbm" else
+                        f"nominal, derived: {sms} SMs x 128 int32 lanes x median SM clock (no measured integer peak)")
     return d, kernels
 
 
@@ -517,13 +575,21 @@ def main():
         "metric": METRIC, "value": total_pairs / (ms / 1e3), "unit": UNIT, "n_gpus": world,
         "instances_per_s": (res["sizes"].n_instances * world) / (ms / 1e3),
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "scaling": "strong" if args.split else "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
         "config": {"workload": WORKLOADS.get(args.config, args.config), "programs_per_gpu": res["P"],
                    "pairs_per_gpu": int(pairs), "instances_per_gpu": int(res["sizes"].n_instances),
                    "threshold_mode": args.mode, "pipeline": args.pipeline,
                    "l2": "inputs larger than L2 (thresholds "
                    f"{4 * res['sizes'].n_pairs_padded / 1e9:.2f} GB per pass)",
-                   "parallelism": f"programs sharded over {world} GPU(s)"},
+                   "parallelism": (f"one batch of {args.programs or res['P'] * world} programs split over "
+                                   f"{world} GPU(s) by instance count" if args.split else
+                                   f"programs sharded over {world} GPU(s)"),
+                   # code-size proxy (RQ2) of rank 0's programs: looped barrier-free vs unrolled
+                   "code_bytes": {"looped": int(res["sizes"].code_bytes_looped),
+                                  "unrolled": int(res["sizes"].code_bytes_unrolled),
+                                  "unrolled_over_looped": (res["sizes"].code_bytes_unrolled /
+                                                           max(res["sizes"].code_bytes_looped, 1)),
+                                  "bytes_per_instruction": 16}},
         "roofline": roof,
         "kernels": kernels,
         # per step: thresholds, check, and per schedule the sweep plus the

@@ -75,9 +75,6 @@ typedef enum {
  * (program order), or 0 when c = 0. */
 typedef enum { SYNC_THR_COUNT = 0, SYNC_THR_PERLOOP = 1, SYNC_THR_PERENGINE = 2 } sync_thr_mode;
 
-/* Schedules simulated: barrier-free waits only, or the barrier-based scheme
- * of Sec. 3.4 (an all-engine barrier at every loop statement and at the end
- * of every iteration). */
 /* Simulation variants.  BARRIER_FREE: the thresholds as semaphore waits
  * (Sec. 5).  BARRIER: all-engine barriers at loop statements and iteration
  * ends (Sec. 3.4).  UNROLLED: the straight-line program the loops would
@@ -92,7 +89,11 @@ enum {
   SYNC_PROG_OK = 0,
   SYNC_PROG_OVERFLOW = 4,        /* static time bound exceeds INT32_MAX        */
   SYNC_PROG_DEADLOCK = 7,        /* no engine can progress before the end      */
-  SYNC_PROG_ROUND_GUARD = 8      /* internal round limit hit (a defect)        */
+  SYNC_PROG_ROUND_GUARD = 8,     /* internal round limit hit (a defect)        */
+  SYNC_PROG_TIMEOUT = 10         /* the per-engine kernel gave up on a program
+                                    after about 2 s of GPU time (a bound on a
+                                    shared GPU, not a verdict on the program:
+                                    rerun it); the sweep never reports it      */
 };
 
 /* Deepest supported nesting below the top-level loop. */
@@ -176,11 +177,29 @@ typedef struct {
   int64_t device_bytes;     /* device memory held by the handle               */
   int64_t h2d_bytes;        /* bytes sync_load_programs copied host -> device */
   int64_t struct_bytes;     /* encoding bytes the threshold and check kernels
-                               read besides the thresholds, each array once:
-                               per-iteration trip starts and ancestors derived
-                               at load time, trip prefix sums of nested
-                               producers' loops, dependency tables            */
+                               read besides the thresholds (COUNT and PERLOOP),
+                               each array once: per-iteration trip starts and
+                               ancestors derived at load time, trip prefix
+                               sums of nested producers' loops and their
+                               offsets, dependency, segment and tile tables
+                               (PERENGINE reads the engine-stream positions of
+                               the waited producers' instances besides)       */
+  int64_t code_bytes_looped;   /* code-size proxy of the barrier-free program
+                                  (the code-size comparison of Sec. 7, RQ2), at
+                                  SYNC_CODE_BYTES_PER_INSTR per instruction:
+                                  every datapath instruction once; per waited
+                                  dependency 5 wait-value ops (per-loop, Table
+                                  1) and the wait; per loop below the top level
+                                  and engine 4 control ops (r-hat := 0 at the
+                                  statement, branch, r++, r-hat++); per engine
+                                  one barrier per loop with fallback barriers */
+  int64_t code_bytes_unrolled; /* the same for the unrolled program: one
+                                  instruction per datapath instance and one
+                                  static wait per waited pair                 */
 } sync_sizes;
+
+/* Instruction size of the code-size proxy (a 128-bit instruction word). */
+#define SYNC_CODE_BYTES_PER_INSTR 16
 
 /* Timing-model constants in cycles, all >= 0 (see sync_simulate). */
 typedef struct {
@@ -355,8 +374,14 @@ sync_status sync_simulate_fused(const sync_programs *h, sync_thr_mode mode, cons
  * sync_last_error(), before anything is launched.  The call zeroes the
  * counters it needs on `stream`; the history is written before it is read.
  *
- * The first call on a device looks up the array's device address (with that
- * device current); make that first call before any stream capture.  All
+ * Every call looks up the array's device address with the handle's device
+ * current.  With CUDA's lazy module loading (the default) the array is only
+ * reserved when the library's module is first loaded on a device, which is
+ * this lookup in the first call there: that call needs
+ * SYNC_NOALLOC_SCRATCH_BYTES of free device memory and fails with
+ * SYNC_ERR_CUDA without it.  A caller whose allocator reserves device memory
+ * up front should therefore make one warm-up call (on a small batch) at
+ * set-up, before the reservation and before any stream capture.  All
  * calls share the one array and it keeps the last call's contents, so calls
  * whose work overlaps on the GPU (other streams, other threads) race with
  * each other: serialise them, e.g. on one stream. */

@@ -82,13 +82,14 @@ def _load():
         bp = P(_Batch)
         lib.orc_sizes.argtypes = [bp, i64p, i64p]
         lib.orc_classify.argtypes = [bp, i32p, i32p, i32p, i32p, i32p]
+        lib.orc_code_size.argtypes = [bp, i64p, i64p]
         lib.orc_thresholds_bruteforce.argtypes = [bp, ctypes.c_int, i32p]
         lib.orc_thresholds.argtypes = [bp, ctypes.c_int, i32p]
         lib.orc_register_replay.argtypes = [bp, ctypes.c_int, i32p]
         lib.orc_check.argtypes = [bp, ctypes.c_int, i32p, u64p, i64p]
         lib.orc_simulate.argtypes = [bp, ctypes.c_int, i32p, P(SimParams), ctypes.c_int, i32p,
                                      u64p, i32p, i32p, i32p]
-        for f in ("orc_sizes", "orc_classify", "orc_thresholds_bruteforce", "orc_thresholds",
+        for f in ("orc_sizes", "orc_code_size", "orc_classify", "orc_thresholds_bruteforce", "orc_thresholds",
                   "orc_register_replay", "orc_check", "orc_simulate"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
@@ -133,6 +134,17 @@ def sizes(batch):
     npairs, ninst = ctypes.c_int64(), ctypes.c_int64()
     _check(lib.orc_sizes(ctypes.byref(v.cb), ctypes.byref(npairs), ctypes.byref(ninst)), "sizes")
     return npairs.value, ninst.value
+
+
+CODE_BYTES_PER_INSTR = 16
+
+
+def code_size(batch):
+    """(looped, unrolled) code-size proxy in instructions (see oracle.h)."""
+    lib, v = _load(), _View(batch)
+    lp, un = ctypes.c_int64(), ctypes.c_int64()
+    _check(lib.orc_code_size(ctypes.byref(v.cb), ctypes.byref(lp), ctypes.byref(un)), "code_size")
+    return lp.value, un.value
 
 
 @dataclass

@@ -452,6 +452,35 @@ int orc_sizes(const orc_batch *b, int64_t *n_pairs, int64_t *n_instances) {
   return ORC_OK;
 }
 
+int orc_code_size(const orc_batch *b, int64_t *looped, int64_t *unrolled) {
+  if (!b || !looped || !unrolled || b->n_programs < 0) return ORC_ERR_ARG;
+  int64_t lp = 0, un = 0;
+  for (int32_t p = 0; p < b->n_programs; ++p) {
+    prog_t P;
+    int rc = prog_open(b, p, &P);
+    if (rc) { prog_close(&P); return rc; }
+    int8_t *bar_loop = (int8_t *)calloc((size_t)P.nl, 1);
+    if (!bar_loop) { prog_close(&P); return ORC_ERR_OOM; }
+    lp += P.nx;
+    for (int32_t x = 0; x < P.nx; ++x) un += inst_total(&P, x);
+    for (int32_t d = 0; d < P.nd; ++d) {
+      dep_class c = classify(&P, d);
+      if (c.kase == ORC_CASE_BARRIER) {            /* no wait: a barrier ends S's iterations */
+        if (c.S != 0) bar_loop[c.S] = 1;
+        continue;
+      }
+      lp += 5 + 1;                                  /* wait-value ops and the wait */
+      un += cons_total(&P, d);                      /* one static wait per pair */
+    }
+    for (int32_t l = 1; l < P.nl; ++l) lp += (int64_t)P.ne * (4 + bar_loop[l]);
+    free(bar_loop);
+    prog_close(&P);
+  }
+  *looped = lp;
+  *unrolled = un;
+  return ORC_OK;
+}
+
 int orc_classify(const orc_batch *b, int32_t *S, int32_t *Pl, int32_t *kase, int32_t *N,
                  int32_t *K) {
   if (!b || b->n_programs < 0) return ORC_ERR_ARG;

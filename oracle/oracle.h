@@ -91,6 +91,17 @@ typedef struct {
 /* Sizes: pairs and instances in the layouts above. */
 int orc_sizes(const orc_batch *b, int64_t *n_pairs, int64_t *n_instances);
 
+/* Code-size proxy of the code-size comparison (Sec. 7, RQ2), in
+ * instructions, summed over the programs.  The looped barrier-free program
+ * (per-loop semaphores): every datapath instruction once; per dependency that
+ * is waited on (not a barrier fallback) the 5 wait-value ops of Table 1 and
+ * the wait instruction; per engine, every loop below the top level costs 4
+ * control instructions (r-hat := 0, the branch, r++, r-hat++) and every loop
+ * that ends its iterations with fallback barriers one barrier.  The unrolled
+ * program: one instruction per datapath instance and one static wait per
+ * (waited dependency, consumer instance) pair. */
+int orc_code_size(const orc_batch *b, int64_t *looped, int64_t *unrolled);
+
 /* Per dependency: innermost common loop S, producer parent loop P (program-
  * local ids), allocatable case (ORC_CASE_*), N and K of the per-loop
  * allocation.  Any output pointer may be NULL. */

@@ -25,13 +25,14 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libsyncgb.so")
 OK, ERR_ARG, ERR_MALFORMED, ERR_NOT_ALLOCATABLE, ERR_OVERFLOW, ERR_CUDA, ERR_OOM = range(7)
 THR_COUNT, THR_PERLOOP, THR_PERENGINE = 0, 1, 2
 SIM_BARRIER_FREE, SIM_BARRIER, SIM_UNROLLED = 0, 1, 2
-PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD = 0, 4, 7, 8
+PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD, PROG_TIMEOUT = 0, 4, 7, 8, 10
 
 # every symbol include/sync.h declares
 EXPORTS = ("sync_load_programs", "sync_query", "sync_pair_offsets", "sync_eval_thresholds",
            "sync_check_minimal", "sync_simulate", "sync_simulate_fused", "sync_simulate_noalloc",
            "sync_free_programs", "sync_last_error")
 NOALLOC_SCRATCH_BYTES = 64 << 20
+CODE_BYTES_PER_INSTR = 16
 
 
 class SyncError(RuntimeError):
@@ -59,7 +60,8 @@ class Sizes(ctypes.Structure):
                 ("n_programs", ctypes.c_int32), ("n_loops", ctypes.c_int32),
                 ("n_instrs", ctypes.c_int32), ("n_deps", ctypes.c_int32),
                 ("device_bytes", ctypes.c_int64), ("h2d_bytes", ctypes.c_int64),
-                ("struct_bytes", ctypes.c_int64)]
+                ("struct_bytes", ctypes.c_int64), ("code_bytes_looped", ctypes.c_int64),
+                ("code_bytes_unrolled", ctypes.c_int64)]
 
 
 class SimParams(ctypes.Structure):

@@ -74,6 +74,11 @@ constexpr int64_t kI32Max = 2147483647;
 
 int64_t pad4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
+// Code-size proxy: wait-value ops of a per-loop wait (Table 1) and control
+// ops of a loop on one engine (r-hat := 0, branch, r++, r-hat++).
+constexpr int64_t kCodeWaitOps = 5;
+constexpr int64_t kCodeLoopOps = 4;
+
 // Threads of the loader's per-program pass: one per hardware thread (at most
 // 32) while each gets at least 256 programs.  SYNCGB_LOAD_THREADS=n sets the
 // count (tests use it to run the block join on small batches).
@@ -144,6 +149,7 @@ struct Part {
   bool ord_overflow = false;
   int32_t nsem_max[kModes] = {0, 0, 0}, ne_max = 0, depth_max = 0;
   int64_t n_bar_deps = 0;                  // barrier-fallback dependencies
+  int64_t code_looped = 0, code_unrolled = 0;   // static instructions (code-size proxy)
   std::exception_ptr error;
 };
 
@@ -554,6 +560,20 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     for (int32_t l = 1; l < nl; ++l)              // the barrier fallback's barriers (shared trips)
       if (S.fbar[l]) pi.fb_iters += tot(l, 0);
     for (int32_t k = 0; k < nd; ++k) part.n_bar_deps += S.dep_bar[k];
+    // code-size proxy (the code-size comparison of Sec. 7, RQ2): the looped
+    // program holds each datapath instruction once, per waited dependency
+    // the per-loop wait-value ops of Table 1 and the wait, per loop and
+    // engine its control (r-hat := 0 at the statement, branch, r++, r-hat++),
+    // and per engine one barrier per loop that ends its iterations with a
+    // fallback barrier; the unrolled program holds one instruction per
+    // instance and one static wait per waited pair
+    {
+      int64_t waited = 0, fb_loops = 0;
+      for (int32_t k = 0; k < nd; ++k) waited += S.dep_bar[k] ? 0 : 1;
+      for (int32_t l = 1; l < nl; ++l) fb_loops += S.fbar[l] ? 1 : 0;
+      part.code_looped += nx + (kCodeWaitOps + 1) * waited + (int64_t)ne * (kCodeLoopOps * (nl - 1) + fb_loops);
+      part.code_unrolled += pi.n_inst + pi.n_pairs;
+    }
     lflag[l0] = 0;
     for (int32_t l = 1; l < nl; ++l) {
       lflag[l0 + l] = S.needs_rhat[l] ? 0 : 1;
@@ -827,7 +847,11 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   bool ord_overflow = false;
   for (const Part& pt : parts) ord_overflow = ord_overflow || pt.ord_overflow;
   h.n_bar_deps = 0;
-  for (const Part& pt : parts) h.n_bar_deps += pt.n_bar_deps;
+  for (const Part& pt : parts) {
+    h.n_bar_deps += pt.n_bar_deps;
+    h.sz.code_bytes_looped += SYNC_CODE_BYTES_PER_INSTR * pt.code_looped;
+    h.sz.code_bytes_unrolled += SYNC_CODE_BYTES_PER_INSTR * pt.code_unrolled;
+  }
   auto join_block = [&](int t) {
     Part& pt = parts[t];
     const Base& B = base[t];
@@ -993,7 +1017,12 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.sz.n_instrs = (int32_t)NX;
   h.sz.n_deps = (int32_t)ND;
   {
-    int64_t sb = (int64_t)ND * (int64_t)sizeof(DepInfo) + 8 * (ND + 1) + 8 * (int64_t)path.size() +
+    // of the path pool the kernels read only the rowptr offsets from S's
+    // child down to a nested producer's loop (clen per dependency); the
+    // pidx offsets are read at load time only
+    int64_t path_read = 0;
+    for (int64_t d = 0; d < ND; ++d) path_read += dep[d].clen;
+    int64_t sb = (int64_t)ND * (int64_t)sizeof(DepInfo) + 8 * (ND + 1) + 8 * path_read +
                  4 * (int64_t)tile_first.size();
     sb += 4 * n_derived;
     for (size_t l = 0; l < xloops.size(); ++l)

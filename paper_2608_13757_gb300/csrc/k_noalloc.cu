@@ -3,16 +3,18 @@
 // For callers that cannot call cudaMalloc / cudaFree around a simulation,
 // the scratch the simulator needs (semaphore history, program-slot counter,
 // fallback list) comes from one array declared statically in device memory
-// here instead of from the handle.  Every GPU that loads the library holds the
-// array until the process exits.  Its device address is looked up once per
-// device, with that device current, on the first call on that device.  All
-// calls share the array and it keeps the last call's contents: the counters
-// the kernels start from are zeroed on the caller's stream by every call, the
-// history is written before it is read, and calls whose work overlaps on the
-// GPU race with each other.
+// here instead of from the handle.  A GPU holds the array from the moment the
+// library's module is loaded on it until the process exits; with CUDA's lazy
+// module loading that is the first call on that device (the address lookup
+// below loads it).  The array's device address is looked up on every call,
+// with the call's device current, so a re-created context (after
+// cudaDeviceReset) never sees a stale address.  All calls share the array
+// and it keeps the last call's contents: the counters the kernels start from
+// are zeroed on the caller's stream by every call, the history is written
+// before it is read, and calls whose work overlaps on the GPU race with each
+// other.
 #include <algorithm>
 #include <cstring>
-#include <mutex>
 #include <string>
 
 #include "handle.h"
@@ -25,20 +27,13 @@ constexpr size_t kScratchInts = SYNC_NOALLOC_SCRATCH_BYTES / sizeof(int32_t);
 // then (at a 256-byte boundary) the semaphore history.
 static __device__ __align__(256) int32_t g_scratch[kScratchInts];
 
-constexpr int kMaxDevices = 256;
-std::mutex g_mutex;
-int32_t* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of g_scratch on `device` (which must be current).
-cudaError_t scratch_on(int device, int32_t** out) {
-  std::lock_guard<std::mutex> lock(g_mutex);
-  if (!g_scratch_ptr[device]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[device] = static_cast<int32_t*>(p);
-  }
-  *out = g_scratch_ptr[device];
+// Device address of g_scratch in the current context (looked up each call:
+// cheap once the module is loaded, and never stale after a context reset).
+cudaError_t scratch_address(int32_t** out) {
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
+  if (e != cudaSuccess) return e;
+  *out = static_cast<int32_t*>(p);
   return cudaSuccess;
 }
 
@@ -73,7 +68,6 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
     return set_error(SYNC_ERR_ARG, "d_issue and d_retire: both or neither");
   sync_sim_params q;
   if (!sim_params_for(*params, variant, q)) return set_error(SYNC_ERR_ARG, "timing constants must be >= 0");
-  if (h->device < 0 || h->device >= kMaxDevices) return set_error(SYNC_ERR_ARG, "device id out of range");
   // the scratch must hold two counters, the fallback list and the history
   const int64_t list_ints = ((2 + (int64_t)h->sz.n_programs) + 63) & ~int64_t(63);
   const int64_t need = list_ints + h->hist_len[mode];
@@ -89,7 +83,7 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
   sync_status st = cuda_error(cudaSetDevice(h->device), "cudaSetDevice");
   if (st != SYNC_OK) return st;
   int32_t* base = nullptr;
-  st = cuda_error(scratch_on(h->device, &base), "cudaGetSymbolAddress");
+  st = cuda_error(scratch_address(&base), "cudaGetSymbolAddress");
   if (st != SYNC_OK) return st;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -42,7 +42,8 @@ namespace {
 constexpr int kChunks = 16;                 // chunks per warp per round
 constexpr int kSpin = 64;                   // polls of a semaphore or barrier per round
 // A program still running after this many SM clock cycles (about 2 s) stops at
-// the next round boundary with status 8, so a launch always ends.
+// the next round boundary with SYNC_PROG_TIMEOUT, so a launch always ends;
+// the deterministic round guard (status 8) stays the only defect verdict.
 constexpr long long kWatchdogCycles = 4000000000ll;
 constexpr unsigned kFull = 0xffffffffu;
 // "-infinity" of the max-plus maps t' = max(t + A, B): cursors are >= 0 and
@@ -489,7 +490,8 @@ __global__ void __launch_bounds__(1024) k_simulate(const SimArgs a) {
       // the watchdog reads thread 0's clock so that every thread agrees
       if (threadIdx.x == 0) S.w_ms[0] = clock64() - started > kWatchdogCycles;
       __syncthreads();
-      if (++rounds > guard || S.w_ms[0]) verdict = SYNC_PROG_ROUND_GUARD;
+      if (++rounds > guard) verdict = SYNC_PROG_ROUND_GUARD;
+      else if (S.w_ms[0]) verdict = SYNC_PROG_TIMEOUT;
       else if (n_live == 0) verdict = SYNC_PROG_OK;
       else if (!any_moved && !any_released) verdict = SYNC_PROG_DEADLOCK;
       __syncthreads();

@@ -426,44 +426,75 @@ def test_loader_blocks_join_identically(sg, monkeypatch):
                 assert torch.equal(x, y)
 
 
-# ------------------------------------------------- full sizes, sampled checks
+# ------------------------------------------------- full sizes, every program
 
 @pytest.mark.parametrize("name", ["chain", "depth2", "attention", "syncbound"])
-def test_full_size_sampled(sg, name):
-    """The full configuration in one launch; a sample of its programs is
-    recomputed by the oracle program by program."""
+def test_full_size_every_program(sg, name):
+    """The full configuration in one launch per kernel, every program
+    recomputed by the oracle (spread over the host cores): every threshold
+    in all three encodings, and every program's status, makespan and
+    checksum under each scheme -- from the threshold array and fused."""
     import torch
+    from tests import oracle_pool
     batch = workloads.generate(name)
     P = batch.n_programs
     h = sg.sync_load_programs(batch)
-    rng = np.random.default_rng(5)
-    sample = np.unique(np.concatenate([[0, P - 1], rng.choice(P, size=min(P, 12), replace=False)]))
+    mask = oracle_pool.unpadded_mask(h.pair_offsets, h.pair_counts)
     for mode in ALL_MODES:
+        variants = variants_for(mode)
+        want_thr, want = oracle_pool.run_config(name, mode, variants)
         thr = sg.sync_eval_thresholds(h, mode)
-        host = thr.cpu().numpy()
+        host = thr.cpu().numpy()[:mask.size]
+        assert (host[~mask] == 0).all(), (name, mode, "padding")
+        got = host[mask]
+        assert got.size == want_thr.size
+        bad = np.flatnonzero(got != want_thr)
+        assert bad.size == 0, (name, mode, bad[:8], got[bad[:8]], want_thr[bad[:8]])
+        del host, got
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
-        sims = {v: sg.sync_simulate(h, mode, thr, variant=v) for v in variants_for(mode)}
-        for v in variants_for(mode):      # fused: identical results on every program
+        for v in variants:
+            res = sg.sync_simulate(h, mode, thr, variant=v)
             f, fc, ff = sg.sync_simulate_fused(h, mode, variant=v, check=True)
             assert fc.cpu().tolist() == [0, 0] and ff.item() == -1, (name, mode, v)
-            for k in ("status", "makespan", "checksum"):
-                assert torch.equal(getattr(f, k), getattr(sims[v], k)), (name, mode, v, k)
-        for p in sample.tolist():
-            one = workloads.generate(name, n_programs=1, first_program=p)
-            want = oracle.thresholds(one, mode)
-            d0, d1 = int(batch.prog_dep_ptr[p]), int(batch.prog_dep_ptr[p + 1])
-            got = np.concatenate([host[h.pair_offsets[d]:h.pair_offsets[d] + h.pair_counts[d]]
-                                  for d in range(d0, d1)] or [np.zeros(0, np.int32)])
-            assert np.array_equal(got, want), (name, mode, p)
-            for v in variants_for(mode):
-                ref = oracle.simulate(one, want, mode, v)
-                assert sims[v].status[p].item() == ref.status[0]
-                assert sims[v].makespan[p].item() == ref.makespan[0], (name, mode, v, p)
-                assert np.uint64(sims[v].checksum[p].item() & (2 ** 64 - 1)) == ref.checksum[0]
+            ref = want[v]
+            for label, r in (("array", res), ("fused", f)):
+                st = r.status.cpu().numpy()[:P]
+                assert np.array_equal(st, ref.status), (name, mode, v, label, "status")
+                ms = r.makespan.cpu().numpy()[:P]
+                bad = np.flatnonzero(ms != ref.makespan)
+                assert bad.size == 0, (name, mode, v, label, bad[:8])
+                ck = r.checksum.cpu().numpy()[:P].view(np.uint64)
+                assert np.array_equal(ck, ref.checksum), (name, mode, v, label, "checksum")
+        del thr
+        torch.cuda.empty_cache()
+    h.close()
 
 
 def test_full_size_gemm_timeline(sg):
     """The single 1.25M-instance GEMM program, complete timeline."""
     batch = workloads.generate("gemm")
     compare_all(sg, batch, timeline=True, modes=(PERLOOP,))
+
+
+# ------------------------------------------------------ code-size proxy (RQ2)
+
+def test_code_size_proxy_matches_oracle(sg):
+    """sync_sizes' code-size proxy of the looped and unrolled programs equals
+    the oracle's instruction counts times the stated instruction size, on
+    every config shape, random trees, per-engine trips and the barrier
+    fallback."""
+    from tests.test_fallback_pins import FAR
+    fb = workloads.random_trees(44, 40, workloads.tree_params(**FAR))
+    fb.nonalloc_policy = 1
+    batches = [workloads.generate(n, n_programs=k) for n, k in
+               (("small", None), ("depth2", 16), ("gemm", None), ("attention", 1), ("chain", 300),
+                ("syncbound", 300))]
+    batches += [workloads.random_trees(45, 100),
+                workloads.diverge(workloads.random_trees(46, 50), 1, permille=200), fb]
+    for b in batches:
+        h = sg.sync_load_programs(b)
+        lo, un = oracle.code_size(b)
+        assert h.sizes.code_bytes_looped == sg.CODE_BYTES_PER_INSTR * lo
+        assert h.sizes.code_bytes_unrolled == sg.CODE_BYTES_PER_INSTR * un
+        h.close()

@@ -806,3 +806,45 @@ def test_elision_matches_recursive_statement(mode):
             off += int(tot[batch.instr_loop[x]])
         n += 1
     assert n == 50
+
+
+# ------------------------------------------------------ code-size proxy (RQ2)
+
+def test_code_size_small_by_hand():
+    """The small config: 6 instructions on 2 engines in one loop of 16
+    iterations, 3 dependencies.  Looped: 6 instructions + 3 x (5 wait-value
+    ops + 1 wait) + 2 engines x 4 control ops = 32; unrolled: 96 instances +
+    48 pairs = 144."""
+    b = workloads.generate("small")
+    assert oracle.sizes(b) == (48, 96)
+    assert oracle.code_size(b) == (32, 144)
+
+
+def test_code_size_counts_fallback_barriers_not_waits():
+    """A nested producer at forward offset 1 taken by the barrier fallback:
+    no wait instructions for it, one barrier per engine for its loop; the
+    unrolled count leaves its pairs out."""
+    b = workloads.ProgramBuilder(2)
+    A = b.loop(0, 0, [3])
+    B = b.loop(A, 0, [2, 2, 2])
+    p = b.instr(B, 0, 0)
+    c = b.instr(A, 1, 1)
+    q = b.instr(A, 2, 0)
+    b.dep(p, c, 1)                       # nested forward, offset 1: barrier fallback
+    b.dep(c, q, 0)                       # producer in S, offset 0: a wait
+    batch = b.batch()
+    batch.nonalloc_policy = 1
+    # 3 instructions + 1 waited dependency x 6 + 2 engines x (2 loops x 4 + 1 barrier loop)
+    assert oracle.code_size(batch) == (3 + 6 + 2 * (8 + 1), 6 + 3 + 3 + 3)
+
+
+def test_code_size_looped_is_independent_of_trips():
+    """The looped program does not grow with the trip counts; the unrolled
+    one grows with the instances and pairs."""
+    small = workloads.generate("small")
+    big = small.copy()
+    big.trips = big.trips * np.array([1] + [10] * (big.trips.size - 1), dtype=np.int32)
+    lo, un = oracle.code_size(small)
+    lo2, un2 = oracle.code_size(big)
+    npairs, ninst = oracle.sizes(big)
+    assert lo2 == lo and un2 == ninst + npairs == 10 * un

@@ -67,16 +67,24 @@ def _outputs(sg, h):
 
 
 def test_noalloc_matches_simulate_on_consecutive_calls(sg):
+    """Two calls in a row per mode and scheme equal sync_simulate's results
+    and, independently of that path, the oracle's (statuses, makespans,
+    checksums and the timelines of the programs that complete)."""
     import torch
+    import oracle
     batch = _batch()
     h = sg.sync_load_programs(batch)
     P = h.sizes.n_programs
     inst = _instances_per_program(batch)
+    idx = h.unpadded_index()
     for mode in (sg.THR_COUNT, sg.THR_PERLOOP, sg.THR_PERENGINE):
         thr = sg.sync_eval_thresholds(h, mode)
+        want_thr = oracle.thresholds(batch, mode)
+        assert np.array_equal(thr.cpu().numpy()[idx], want_thr)
         unrolled = (sg.SIM_UNROLLED,) if mode == sg.THR_PERENGINE else ()
         for variant in (sg.SIM_BARRIER_FREE, sg.SIM_BARRIER) + unrolled:
             ref = sg.sync_simulate(h, mode, thr, variant=variant, timeline=True)
+            orc = oracle.simulate(batch, want_thr, mode, variant, timeline=True)
             torch.cuda.synchronize()
             ok = ref.status.cpu().numpy() == sg.PROG_OK
             assert ok.sum() >= P - 2 and (~ok).any()
@@ -89,6 +97,13 @@ def test_noalloc_matches_simulate_on_consecutive_calls(sg):
                     assert torch.equal(getattr(out, f), getattr(ref, f)), (mode, variant, f)
                 for f in ("issue", "retire"):
                     assert torch.equal(getattr(out, f)[defined], getattr(ref, f)[defined]), (mode, variant, f)
+                assert np.array_equal(out.status.cpu().numpy(), orc.status), (mode, variant)
+                assert np.array_equal(out.makespan.cpu().numpy(), orc.makespan), (mode, variant)
+                assert np.array_equal(out.checksum.cpu().numpy().view(np.uint64), orc.checksum), (mode, variant)
+                mask = np.repeat(orc.status == 0, inst)
+                for f in ("issue", "retire"):
+                    got = getattr(out, f).cpu().numpy()[:mask.size]
+                    assert np.array_equal(got[mask], getattr(orc, f)[mask]), (mode, variant, f)
     h.close()
 
 
