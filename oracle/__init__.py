@@ -57,15 +57,16 @@ class _Batch(ctypes.Structure):
 class SimParams(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "ii", "c_branch", "c_regop", "c_wait_ops_count", "c_wait_ops_perloop", "c_barrier",
-        "c_wait_ops_perengine_level", "trip_register_elision")]
+        "c_wait_ops_perengine_level", "trip_register_elision", "licm", "cse")]
 
 
 def sim_params(**kw) -> SimParams:
     """Timing-model constants; defaults ii=1, c_branch=1, c_regop=1, 3 / 5 wait
     ops per dependency (count / per-loop, Table 1), c_barrier=32, and 3 more
-    ops per enclosing loop level for a per-engine wait (Sec. 6.1)."""
+    ops per enclosing loop level for a per-engine wait (Sec. 6.1); the ALU
+    reductions of Sec. 6.2 (licm, cse) off."""
     d = dict(ii=1, c_branch=1, c_regop=1, c_wait_ops_count=3, c_wait_ops_perloop=5, c_barrier=32,
-             c_wait_ops_perengine_level=3, trip_register_elision=0)
+             c_wait_ops_perengine_level=3, trip_register_elision=0, licm=0, cse=0)
     d.update(kw)
     return SimParams(**d)
 

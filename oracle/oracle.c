@@ -76,11 +76,34 @@
  *  - unrolled variant (the straight-line program of Sec. 3.3 the loops would
  *    unroll to): as barrier-free with no loop statement, iteration start or
  *    wait-value costs; per-engine semaphores with static waits.
+ *  - ALU reductions of Sec. 6.2 (barrier-free; both off by default):
+ *    licm (per-engine waits only): the term of every loop l strictly between
+ *      the top level and the producer's loop P in the per-engine path sum
+ *      changes only when l starts an iteration, so it is kept in a cached
+ *      partial sum updated there: at each iteration start of l, engine e pays
+ *      c_wait_ops_perengine_level once per producer engine e' such that some
+ *      per-engine wait on e (a consumer on e) has its producer on e' and P
+ *      strictly below l; such a wait then costs c_wait_ops_perloop plus
+ *      c_regop (the read of the cached sum) instead of c_wait_ops_perloop +
+ *      c_wait_ops_perengine_level * levels (no read without levels);
+ *    cse: on one engine, within one visit of a straight-line segment of a
+ *      loop body (the items between two child loops, in one iteration), the
+ *      waits are taken in program order (an instruction's dependencies in
+ *      dependency order); a wait on the same producer with the same offset as
+ *      an earlier one reuses its value and costs 0; otherwise the mask
+ *      isGT(r-hat_S, k) of an earlier wait with the same S and k is reused
+ *      (min(c_regop, wait-value ops) less), and, per-engine, the outer
+ *      partial sum of an earlier wait with the same producer loop and
+ *      producer engine (its levels term, or with licm its read) is reused.
  * A semaphore's value reaches v at the retire time of its v-th increment
  * (increments of one semaphore all come from one engine, in retire order;
  * a per-engine semaphore is incremented by every retirement on its engine).
  * Under the barrier scheme the waits stay in place; after a barrier they can
  * only be already satisfied or concern the current barrier interval.
+ * With licm (per-engine, barrier-free) the bound adds c_wait_ops_perengine_level
+ * for every cached-sum update (per iteration of l on e, per producer engine
+ * counted above) and c_regop for every pair of a per-engine wait with
+ * levels.  CSE only removes costs and changes no bound.
  * Checksum: the sum (mod 2^64) over datapath instances of
  *   (a << 32) | b, with 32-bit arithmetic mod 2^32,
  *   a = (issue ^ (n*0x9E3779B9 + e)) * 0x85EBCA6B, a ^= a >> 13,
@@ -845,7 +868,8 @@ typedef struct {
   const orc_sim_params *prm;
   int mode, barrier;
   int64_t *wcost;              /* per instruction: wait-value ops before issue */
-  int64_t *iter_cost, *stmt_cost; /* per loop: iteration start / loop statement */
+  int64_t *iter_cost;          /* per (loop l, engine e), at l*ne + e: iteration start */
+  int64_t *stmt_cost;          /* per loop: loop statement */
   const int32_t *thr;          /* program's pairs */
   int64_t *pair_off;           /* per dep */
   int32_t *own_sem, *dep_sem;  /* semaphore incremented by x / waited by d */
@@ -881,7 +905,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
     }
     E->bar_passed = 0;
     if (++f->g < f->g_end) {                   /* next iteration starts */
-      E->t += X->iter_cost[f->loop];
+      E->t += X->iter_cost[(int64_t)f->loop * P->ne + e];
       E->next[f->loop]++;
       f->item = 0;
     } else {
@@ -906,7 +930,7 @@ static int step(sim_ctx *X, engine *E, int32_t e) {
       c->loop = m; c->item = 0;
       c->g = E->next[m]; c->g_end = c->g + trip;
       E->next[m]++;
-      E->t += X->iter_cost[m];
+      E->t += X->iter_cost[(int64_t)m * P->ne + e];
     }
     return S_PROGRESS;
   }
@@ -962,15 +986,48 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     if (c.S != 0) loop_bar[c.S] = 1;
   }
   if (any_bar && unrolled) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_ARG; }
-  for (int32_t d = 0; d < nd && !unrolled; ++d) {
-    if (dep_bar[d]) continue;
-    int64_t c = mode == ORC_COUNT ? q->c_wait_ops_count : q->c_wait_ops_perloop;
-    if (mode == ORC_PERENGINE) {
-      int32_t lev = P->depth[P->xl[P->dp[d]]] - 1;
-      c += (int64_t)q->c_wait_ops_perengine_level * (lev > 0 ? lev : 0);
+  /* Each loop body is walked in item order; a child loop ends a straight-
+   * line segment.  Every waited dependency of a consumer costs its wait-value
+   * ops, reduced by the CSE rules (see the header) against the earlier waits
+   * of the same engine in the same segment. */
+  typedef struct { int32_t e, p, k, S, Pl, pe; } wait_key;
+  wait_key *seen = (wait_key *)malloc(((size_t)nd + 1) * sizeof(wait_key));
+  if (!seen) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_OOM; }
+  const int64_t cw = mode == ORC_COUNT ? q->c_wait_ops_count : q->c_wait_ops_perloop;
+  for (int32_t l = 0; l < nl && !unrolled; ++l) {
+    int32_t nseen = 0;
+    for (int32_t i = P->body_ptr[l]; i < P->body_ptr[l + 1]; ++i) {
+      int32_t x = P->body[i];
+      if (x < 0) { nseen = 0; continue; }        /* a child loop ends the segment */
+      for (int32_t j = P->cons_ptr[x]; j < P->cons_ptr[x + 1]; ++j) {
+        int32_t d = P->cons_dep[j];
+        if (dep_bar[d]) continue;
+        dep_class dc = classify(P, d);
+        wait_key w = { P->xe[x], P->dp[d], P->dk[d], dc.S, dc.P, P->xe[P->dp[d]] };
+        int32_t lev = mode == ORC_PERENGINE ? P->depth[dc.P] - 1 : 0;
+        if (lev < 0) lev = 0;
+        /* the outer part of a per-engine wait: its levels, or the cached read */
+        int64_t outer = mode != ORC_PERENGINE ? 0
+                        : q->licm ? (lev > 0 ? q->c_regop : 0)
+                                  : (int64_t)q->c_wait_ops_perengine_level * lev;
+        int64_t c = cw + outer;
+        if (q->cse) {
+          int same = 0, mask = 0, part = 0;
+          for (int32_t s2 = 0; s2 < nseen; ++s2) {
+            if (seen[s2].e != w.e) continue;
+            if (seen[s2].p == w.p && seen[s2].k == w.k) same = 1;
+            if (seen[s2].S == w.S && seen[s2].k == w.k) mask = 1;
+            if (seen[s2].Pl == w.Pl && seen[s2].pe == w.pe) part = 1;
+          }
+          int64_t m = q->c_regop < cw ? q->c_regop : cw;
+          c = same ? 0 : cw - (mask ? m : 0) + (part ? 0 : outer);
+          seen[nseen++] = w;
+        }
+        wcost[x] += c;
+      }
     }
-    wcost[P->dc[d]] += c;
   }
+  free(seen);
   /* per loop: the register ops of its statement (r-hat := 0) and of each
    * iteration start (branch, r++, r-hat++); with trip-register elision a
    * loop that carries only offset-0 dependencies (or none) has no r-hat
@@ -984,11 +1041,40 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   }
   for (int32_t d = 0; d < nd; ++d)     /* a barrier-fallback dependency reads no register */
     if (P->dk[d] > 0 && !dep_bar[d]) needs_rhat[classify(P, d).S] = 1;
+  /* LICM (per-engine, barrier-free): cached path sums kept per (loop l,
+   * engine e), one per producer engine e' (bit e' of pe_of[l*ne + e]) */
+  uint32_t *pe_of = (uint32_t *)calloc((size_t)nl * ne, sizeof(uint32_t));
+  int64_t licm_updates = 0, lv_pairs = 0;        /* for the static bound */
+  if (!pe_of) {
+    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(dep_bar); free(loop_bar);
+    return ORC_ERR_OOM;
+  }
+  int licm = q->licm && mode == ORC_PERENGINE && !barrier && !unrolled;
+  for (int32_t d = 0; d < nd && licm; ++d) {
+    if (dep_bar[d]) continue;
+    int32_t Pl = P->xl[P->dp[d]];
+    if (P->depth[Pl] > 1) lv_pairs += cons_total(P, d);
+    for (int32_t l = P->par[Pl]; l > 0; l = P->par[l])
+      pe_of[(int64_t)l * ne + P->xe[P->dc[d]]] |= 1u << P->xe[P->dp[d]];
+  }
   for (int32_t l = 0; l < nl; ++l) {
     int elide = q->trip_register_elision && !needs_rhat[l];
     iter_cost[l] = unrolled ? 0 : barrier ? q->c_branch : q->c_branch + (elide ? 1 : 2) * (int64_t)q->c_regop;
     stmt_cost[l] = unrolled || elide ? 0 : q->c_regop;
   }
+  /* per (loop, engine): the iteration start, plus the cached-sum updates */
+  int64_t *iter_cost_e = (int64_t *)calloc((size_t)nl * ne + 1, sizeof(int64_t));
+  if (!iter_cost_e) {
+    free(pe_of); free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(dep_bar); free(loop_bar);
+    return ORC_ERR_OOM;
+  }
+  for (int32_t l = 0; l < nl; ++l)
+    for (int32_t e = 0; e < ne; ++e) {
+      int32_t n = __builtin_popcount(pe_of[(int64_t)l * ne + e]);
+      iter_cost_e[(int64_t)l * ne + e] = iter_cost[l] + (int64_t)q->c_wait_ops_perengine_level * n;
+      licm_updates += (int64_t)n * tot_on(P, l, e);
+    }
+  free(pe_of);
   free(needs_rhat);
   /* the static time bound */
   u128 bound = 0, ctl = 0;
@@ -1011,8 +1097,11 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     bound += ctl;
     for (int32_t l = 1; l < nl; ++l)  /* the fallback barriers: one per iteration of a flagged loop */
       if (loop_bar[l]) bound += (u128)P->total[l] * (u128)q->c_barrier;
+    if (licm)                         /* cached-sum updates and reads */
+      bound += (u128)licm_updates * (u128)q->c_wait_ops_perengine_level + (u128)lv_pairs * (u128)q->c_regop;
   }
   if (bound > (u128)INT32_MAX) {
+    free(iter_cost_e);
     free(wcost); free(iter_cost); free(stmt_cost); free(dep_bar); free(loop_bar);
     *makespan = -1; *checksum = 0; *status = ORC_SIM_OVERFLOW;
     return ORC_OK;
@@ -1020,7 +1109,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   sim_ctx X;
   memset(&X, 0, sizeof X);
   X.P = P; X.prm = q; X.mode = mode; X.barrier = barrier; X.wcost = wcost; X.thr = thr;
-  X.iter_cost = iter_cost; X.stmt_cost = stmt_cost;
+  X.iter_cost = iter_cost_e; X.stmt_cost = stmt_cost;
   X.issue = issue; X.retire = retire;
   X.dep_bar = dep_bar; X.loop_bar = loop_bar;
   int32_t nsem = mode == ORC_COUNT ? nx : mode == ORC_PERLOOP ? nl * ne : ne;
@@ -1101,7 +1190,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   for (int32_t s = 0; X.times && s < nsem; ++s) free(X.times[s]);
   free(E); free(incs); free(X.pair_off); free(X.inst_off); free(X.own_sem); free(X.dep_sem);
   free(X.value); free(X.times); free(wcost); free(iter_cost); free(stmt_cost);
-  free(dep_bar); free(loop_bar);
+  free(iter_cost_e); free(dep_bar); free(loop_bar);
   return rc;
 }
 

@@ -75,6 +75,10 @@ typedef struct {
   int32_t c_barrier;          /* all-engine barrier handshake + reset          */
   int32_t c_wait_ops_perengine_level; /* per-engine mode: per enclosing loop level */
   int32_t trip_register_elision; /* 1: no r-hat for loops carrying only offset-0 deps */
+  int32_t licm;               /* 1: loop-invariant code motion of the per-engine
+                                 path sums (Sec. 6.2), see oracle.c */
+  int32_t cse;                /* 1: common-subexpression elimination of wait
+                                 values within a straight-line segment (Sec. 6.2) */
 } orc_sim_params;
 
 /* Per-engine trip counts (control-flow divergence, Sec. 7.5): each engine

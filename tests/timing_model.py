@@ -63,11 +63,16 @@ def _events(batch, e, barrier):
     return ev
 
 
-def simulate(batch, thr_count, params, barrier, cwait, unrolled=False, no_rhat=()):
+def simulate(batch, thr_count, params, barrier, cwait, unrolled=False, no_rhat=(), inst_wait=None,
+             iter_extra=None):
     """(makespan, checksum, {(x, g): (issue, retire)}) or raises Deadlock.
     cwait: wait ops per dependency, an int or a function of the dependency.
     no_rhat: loops without a trip register (their statement costs nothing
-    and their iteration starts one register op less, barrier-free)."""
+    and their iteration starts one register op less, barrier-free).
+    inst_wait: optional function of an instruction giving its total wait ops
+    (replaces the sum of cwait over its dependencies); iter_extra: optional
+    function (loop, engine) -> extra cycles at each iteration start of the
+    loop on the engine (barrier-free)."""
     wait_ops = cwait if callable(cwait) else (lambda d: cwait)
     ne = int(batch.prog_n_engines[0])
     ev = [_events(batch, e, barrier) for e in range(ne)]
@@ -116,7 +121,8 @@ def simulate(batch, thr_count, params, barrier, cwait, unrolled=False, no_rhat=(
         if v[0] == "x":
             x, g = v[1], v[2]
             ds = deps_of.get(x, [])
-            tw = t + (0 if barrier or unrolled else sum(wait_ops(d) for d in ds))
+            own = inst_wait(x) if inst_wait is not None else sum(wait_ops(d) for d in ds)
+            tw = t + (0 if barrier or unrolled else own)
             ready = 0
             for d in ds:
                 c = int(thr_count[pair_off[d] + g])
@@ -144,7 +150,8 @@ def simulate(batch, thr_count, params, barrier, cwait, unrolled=False, no_rhat=(
             out = (t, lr, None, None)
         else:  # iteration start: branch, r++ and (unless elided) r-hat++
             regops = 0 if barrier else (1 if v[1] in no_rhat else 2)
-            out = (t + params.c_branch + regops * params.c_regop, lr, None, None)
+            extra = iter_extra(v[1], e) if iter_extra is not None and not barrier else 0
+            out = (t + params.c_branch + regops * params.c_regop + extra, lr, None, None)
         busy.discard(key)
         memo[key] = out
         return out
