@@ -100,10 +100,11 @@
  * a per-engine semaphore is incremented by every retirement on its engine).
  * Under the barrier scheme the waits stay in place; after a barrier they can
  * only be already satisfied or concern the current barrier interval.
- * With licm (per-engine, barrier-free) the bound adds c_wait_ops_perengine_level
- * for every cached-sum update (per iteration of l on e, per producer engine
- * counted above) and c_regop for every pair of a per-engine wait with
- * levels.  CSE only removes costs and changes no bound.
+ * The bound counts the wait ops before the reductions of Sec. 6.2; with licm
+ * (per-engine, barrier-free) it adds c_wait_ops_perengine_level for every
+ * cached-sum update (per iteration of l on e, per producer engine counted
+ * above) and c_regop for every pair of a per-engine wait with levels.  CSE
+ * only removes costs and changes no bound.
  * Checksum: the sum (mod 2^64) over datapath instances of
  *   (a << 32) | b, with 32-bit arithmetic mod 2^32,
  *   a = (issue ^ (n*0x9E3779B9 + e)) * 0x85EBCA6B, a ^= a >> 13,
@@ -972,9 +973,12 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   int unrolled = variant == ORC_UNROLLED;       /* straight-line: no control or wait-value ops */
   /* wait-value ops of each dependency (Table 1; per-engine: O(D), Sec. 6.1) */
   int64_t *wcost = (int64_t *)calloc((size_t)nx + 1, sizeof(int64_t));
+  /* the same without the reductions of Sec. 6.2: the static bound's term */
+  int64_t *wfull = (int64_t *)calloc((size_t)nx + 1, sizeof(int64_t));
+  if (!wfull) { free(wcost); return ORC_ERR_OOM; }
   int8_t *dep_bar = (int8_t *)calloc((size_t)nd + 1, sizeof(int8_t));
   int8_t *loop_bar = (int8_t *)calloc((size_t)nl, sizeof(int8_t));
-  if (!wcost || !dep_bar || !loop_bar) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_OOM; }
+  if (!wcost || !dep_bar || !loop_bar) { free(wcost); free(wfull); free(dep_bar); free(loop_bar); return ORC_ERR_OOM; }
   /* barrier fallback (Sec. 5.2): no wait; a barrier ends every iteration of
    * the carrying loop S (none at the top level, which runs once) */
   int any_bar = 0;
@@ -985,14 +989,14 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
     any_bar = 1;
     if (c.S != 0) loop_bar[c.S] = 1;
   }
-  if (any_bar && unrolled) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_ARG; }
+  if (any_bar && unrolled) { free(wcost); free(wfull); free(dep_bar); free(loop_bar); return ORC_ERR_ARG; }
   /* Each loop body is walked in item order; a child loop ends a straight-
    * line segment.  Every waited dependency of a consumer costs its wait-value
    * ops, reduced by the CSE rules (see the header) against the earlier waits
    * of the same engine in the same segment. */
   typedef struct { int32_t e, p, k, S, Pl, pe; } wait_key;
   wait_key *seen = (wait_key *)malloc(((size_t)nd + 1) * sizeof(wait_key));
-  if (!seen) { free(wcost); free(dep_bar); free(loop_bar); return ORC_ERR_OOM; }
+  if (!seen) { free(wcost); free(wfull); free(dep_bar); free(loop_bar); return ORC_ERR_OOM; }
   const int64_t cw = mode == ORC_COUNT ? q->c_wait_ops_count : q->c_wait_ops_perloop;
   for (int32_t l = 0; l < nl && !unrolled; ++l) {
     int32_t nseen = 0;
@@ -1011,6 +1015,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
                         : q->licm ? (lev > 0 ? q->c_regop : 0)
                                   : (int64_t)q->c_wait_ops_perengine_level * lev;
         int64_t c = cw + outer;
+        wfull[x] += cw + (mode == ORC_PERENGINE ? (int64_t)q->c_wait_ops_perengine_level * lev : 0);
         if (q->cse) {
           int same = 0, mask = 0, part = 0;
           for (int32_t s2 = 0; s2 < nseen; ++s2) {
@@ -1036,7 +1041,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   int64_t *stmt_cost = (int64_t *)calloc((size_t)nl, sizeof(int64_t));
   int8_t *needs_rhat = (int8_t *)calloc((size_t)nl, sizeof(int8_t));
   if (!iter_cost || !stmt_cost || !needs_rhat) {
-    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(dep_bar); free(loop_bar);
+    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(wfull); free(dep_bar); free(loop_bar);
     return ORC_ERR_OOM;
   }
   for (int32_t d = 0; d < nd; ++d)     /* a barrier-fallback dependency reads no register */
@@ -1046,7 +1051,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   uint32_t *pe_of = (uint32_t *)calloc((size_t)nl * ne, sizeof(uint32_t));
   int64_t licm_updates = 0, lv_pairs = 0;        /* for the static bound */
   if (!pe_of) {
-    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(dep_bar); free(loop_bar);
+    free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(wfull); free(dep_bar); free(loop_bar);
     return ORC_ERR_OOM;
   }
   int licm = q->licm && mode == ORC_PERENGINE && !barrier && !unrolled;
@@ -1065,7 +1070,7 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
   /* per (loop, engine): the iteration start, plus the cached-sum updates */
   int64_t *iter_cost_e = (int64_t *)calloc((size_t)nl * ne + 1, sizeof(int64_t));
   if (!iter_cost_e) {
-    free(pe_of); free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(dep_bar); free(loop_bar);
+    free(pe_of); free(iter_cost); free(stmt_cost); free(needs_rhat); free(wcost); free(wfull); free(dep_bar); free(loop_bar);
     return ORC_ERR_OOM;
   }
   for (int32_t l = 0; l < nl; ++l)
@@ -1085,11 +1090,13 @@ static int sim_program(prog_t *P, int mode, const int32_t *thr, const orc_sim_pa
       iters += tot_on(P, l, e);
       ctl += (u128)tot_on(P, P->par[l], e) * (u128)stmt_cost[l] + (u128)tot_on(P, l, e) * (u128)iter_cost[l];
     }
-  for (int32_t x = 0; x < nx; ++x) {
+  for (int32_t x = 0; x < nx; ++x) {        /* wait ops before the reductions of Sec. 6.2 */
     int64_t per = (int64_t)P->xlat[x] + q->ii;
-    if (!barrier) per += wcost[x];
+    if (!barrier) per += wfull[x];
     bound += (u128)inst_total(P, x) * (u128)per;
   }
+  free(wfull);
+  wfull = NULL;
   if (barrier) {                     /* shared trips: every engine has the same counts */
     bound += (u128)iters * (u128)q->c_branch;
     bound += (u128)(stmts / ne + iters / ne) * (u128)q->c_barrier;

@@ -268,3 +268,17 @@ def test_reductions_match_recursive_statement(mode, licm, cse):
             off += tot[int(batch.instr_loop[x])]
         n += 1
     assert n >= 25
+
+
+def test_bound_counts_wait_ops_before_the_reductions():
+    """The static bound takes the wait ops before CSE: 100 iterations of 8
+    consumers of one producer at 2^22 ops per wait exceed INT32_MAX before
+    CSE (status 4 with and without it), although with CSE only one wait per
+    iteration pays (100 * 2^22 < INT32_MAX)."""
+    b, T = _chain(1, [100], m_consumers=8)
+    thr = oracle.thresholds(b, COUNT)
+    for cse in (0, 1):
+        r = oracle.simulate(b, thr, COUNT, BF, oracle.sim_params(c_wait_ops_count=2 ** 22, cse=cse))
+        assert r.status[0] == 4 and r.makespan[0] == -1
+    r = oracle.simulate(b, thr, COUNT, BF, oracle.sim_params(c_wait_ops_count=2 ** 18, cse=1))
+    assert r.status[0] == 0 and r.makespan[0] > 100 * 2 ** 18
