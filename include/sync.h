@@ -219,6 +219,30 @@ typedef struct {
                                  a consumer issues), so its loop statement and
                                  iteration starts lose one register op each;
                                  0: every loop keeps r-hat (the default) */
+  int32_t licm;               /* 1: loop-invariant code motion of the per-engine
+                                 path sums (Sec. 6.2), barrier-free PERENGINE:
+                                 the term of each loop l strictly between the
+                                 top level and a producer's loop is kept in a
+                                 cached partial sum that engine e updates at
+                                 every iteration start of l (cost
+                                 c_wait_ops_perengine_level, once per producer
+                                 engine whose waits on e pass below l); a wait
+                                 then costs c_wait_ops_perloop plus c_regop
+                                 (the read of the cached sum; nothing when the
+                                 producer's loop has depth <= 1).  0: off */
+  int32_t cse;                /* 1: common-subexpression elimination of wait
+                                 values (Sec. 6.2), barrier-free: on one engine,
+                                 within one visit of a straight-line segment of
+                                 a loop body (the items between two child loops,
+                                 in one iteration), the waits in program order
+                                 (an instruction's dependencies in dependency
+                                 order) reuse an earlier wait's value when it
+                                 has the same producer and offset (no cost),
+                                 else its mask when it has the same carrying
+                                 loop S and offset (min(c_regop, wait ops) less)
+                                 and, PERENGINE, its outer partial sum when it
+                                 has the same producer loop and producer engine
+                                 (no levels term, or with licm no read).  0: off */
 } sync_sim_params;
 
 typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
@@ -318,6 +342,10 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  *     every engine continues at release
  *   the top-level loop costs nothing; makespan = max over engines of
  *   max(t, last retire).
+ * The ALU reductions licm and cse (sync_sim_params) change the wait-op and
+ * iteration-start costs above as described there; with licm the static time
+ * bound (SYNC_PROG_OVERFLOW) adds c_wait_ops_perengine_level per cached-sum
+ * update and c_regop per pair of a wait with a cached-sum read.
  * UNROLLED: as barrier-free with c_branch, c_regop and every wait-op cost
  * taken as 0 (ii and latencies unchanged); it requires PERENGINE and a batch
  * without barrier-fallback dependencies, and returns SYNC_ERR_ARG otherwise.

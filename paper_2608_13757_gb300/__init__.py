@@ -68,12 +68,12 @@ class SimParams(ctypes.Structure):
     """Timing-model constants (cycles); defaults as in the library's docs."""
     _fields_ = [(n, ctypes.c_int32) for n in (
         "ii", "c_branch", "c_regop", "c_wait_ops_count", "c_wait_ops_perloop", "c_barrier",
-        "c_wait_ops_perengine_level", "trip_register_elision")]
+        "c_wait_ops_perengine_level", "trip_register_elision", "licm", "cse")]
 
     def __init__(self, ii=1, c_branch=1, c_regop=1, c_wait_ops_count=3, c_wait_ops_perloop=5,
-                 c_barrier=32, c_wait_ops_perengine_level=3, trip_register_elision=0):
+                 c_barrier=32, c_wait_ops_perengine_level=3, trip_register_elision=0, licm=0, cse=0):
         super().__init__(ii, c_branch, c_regop, c_wait_ops_count, c_wait_ops_perloop, c_barrier,
-                         c_wait_ops_perengine_level, trip_register_elision)
+                         c_wait_ops_perengine_level, trip_register_elision, licm, cse)
 
 
 def load_library(path: str = LIB_PATH) -> ctypes.CDLL:

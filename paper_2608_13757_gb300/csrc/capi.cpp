@@ -2,6 +2,7 @@
 // device encoding) and the launch wrappers.  Declarations and contracts are
 // in include/sync.h.
 #include <algorithm>
+#include <array>
 #include <cstdlib>
 #include <cstring>
 #include <exception>
@@ -63,6 +64,7 @@ bool sim_params_for(const sync_sim_params& p, sync_sim_variant variant, sync_sim
   if (variant == SYNC_SIM_UNROLLED) {
     q.c_branch = q.c_regop = 0;
     q.c_wait_ops_count = q.c_wait_ops_perloop = q.c_wait_ops_perengine_level = 0;
+    q.licm = q.cse = 0;
   }
   return true;
 }
@@ -120,6 +122,9 @@ struct ProgScratch {
   std::vector<uint8_t> needs_rhat;                // per loop: carries a dependency with offset > 0
   std::vector<uint8_t> fbar;                      // per loop: ends its iterations with a fallback barrier
   std::vector<uint8_t> dep_bar;                   // per dependency: barrier fallback (not waited on)
+  std::vector<int32_t> dep_S;                     // per dependency: innermost common loop
+  std::vector<std::array<int32_t, 6>> cse_seen;   // waits of the current straight-line segment
+  std::vector<uint32_t> pe_of;                    // per (loop, engine): producer engines of cached sums
   std::unordered_map<int64_t, int64_t> anc_of;    // derived ancestor array per (consumer loop, S)
   std::vector<int32_t> by_cons, cons_next, sem_of;  // dependencies by consumer; semaphore per key
   std::vector<int64_t> inst_eng, sem_hist;        // instances per engine; history bases of one mode
@@ -150,6 +155,7 @@ struct Part {
   int32_t nsem_max[kModes] = {0, 0, 0}, ne_max = 0, depth_max = 0;
   int64_t n_bar_deps = 0;                  // barrier-fallback dependencies
   int64_t code_looped = 0, code_unrolled = 0;   // static instructions (code-size proxy)
+  std::vector<int32_t> hoist;              // per (loop, engine) row: LICM's cached sums
   std::exception_ptr error;
 };
 
@@ -228,10 +234,13 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   // per-engine wait levels}, gathered on the device into the op and lane
   // records that name the instruction
   HostVec<int4> xsem((size_t)kModes * NX);
+  HostVec<int4> xcse(NX);                  // Sec. 6.2 reductions: per-instruction wait counts
+  HostVec<int32_t> xlvr(NX);
 
   // Programs [p_begin, p_end) into `part`; erow0: their first per-engine row.
   auto run_block = [&d, div, &loop, &dep, &prog, &inst_off, &dseg, &ddep, &dsem, &seg, &ord_off, &dep_N,
-                    &dep_K, &lflag, &xsem, &dep_count, NX, ND](Part& part, int32_t p_begin, int32_t p_end, int64_t erow0) {
+                    &dep_K, &lflag, &xsem, &xcse, &xlvr, &dep_count, NX, ND](Part& part, int32_t p_begin,
+                                                                            int32_t p_end, int64_t erow0) {
   auto& rowptr_host = part.rowptr_host;
   auto& path = part.path;
   auto& op_ptr = part.op_ptr;
@@ -278,6 +287,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     S.needs_rhat.assign(nl, 0);
     S.fbar.assign(nl, 0);
     S.dep_bar.assign(nd, 0);
+    S.dep_S.assign(nd, 0);
     if (par[0] != -1) raise(SYNC_ERR_MALFORMED, where(p, "loop 0 must have parent -1, loop", 0));
     int32_t depth_max = 0;
     for (int32_t l = 1; l < nl; ++l) {
@@ -438,6 +448,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
       while (S.depth[b] > S.depth[a]) { cb = b; b = par[b]; }
       while (a != b) { ca = a; a = par[a]; cb = b; b = par[b]; }
       const int32_t Sl = a;
+      S.dep_S[k] = Sl;
       const int32_t ppos = ca < 0 ? d.instr_pos[x0 + px] : lpos[ca];
       const int32_t cpos = cb < 0 ? d.instr_pos[x0 + cx] : lpos[cb];
       const bool forward = cpos > ppos;
@@ -621,6 +632,56 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     int32_t nw = 0;                                // waited dependencies, grouped first
     for (int32_t k = 0; k < nd; ++k)
       if (!S.dep_bar[k]) { by_cons[next[d.dep_cons[d0 + k]]++] = k; ++nw; }
+    // Sec. 6.2's reductions.  CSE: per instruction, the counts its wait ops
+    // are made of when the waits of one engine in one visit of a straight-
+    // line segment are taken in program order (CostTables in enc.h).  LICM:
+    // per (loop, engine), the producer engines whose cached path sums the
+    // engine updates at the loop's iteration starts; the bound's terms.
+    {
+      auto& seen = S.cse_seen;
+      for (int32_t l = 0; l < nl; ++l) {
+        seen.clear();
+        for (int32_t i = S.body_ptr[l]; i < S.body_ptr[l + 1]; ++i) {
+          const int32_t x = S.body[i];
+          if (x < 0) { seen.clear(); continue; }      // a child loop ends the segment
+          const int32_t ex = d.instr_engine[x0 + x];
+          int4 c = make_int4(0, 0, 0, 0);
+          int32_t lvr = 0;
+          for (int32_t j = 0; j < S.x_ndeps[x]; ++j) {
+            const int32_t k = by_cons[S.x_dep_begin[x] - d0 + j];
+            const int64_t gd = d0 + k;
+            const int32_t px = d.dep_prod[gd], lev = levels(px);
+            const std::array<int32_t, 6> w = {ex, px, d.dep_k[gd], S.dep_S[k], d.instr_loop[x0 + px],
+                                              d.instr_engine[x0 + px]};
+            bool same = false, mask = false, outer = false;
+            for (const auto& o : seen) {
+              if (o[0] != ex) continue;
+              same = same || (o[1] == w[1] && o[2] == w[2]);     // the same value
+              mask = mask || (o[3] == w[3] && o[2] == w[2]);     // the same isGT(r-hat_S, k)
+              outer = outer || (o[4] == w[4] && o[5] == w[5]);   // the same outer path sum
+            }
+            lvr += lev > 0 ? 1 : 0;
+            if (!same) {
+              ++c.x;
+              if (mask) ++c.y;
+              if (!outer) { c.z += lev > 0 ? 1 : 0; c.w += lev; }
+            }
+            seen.push_back(w);
+          }
+          xcse[x0 + x] = c;
+          xlvr[x0 + x] = lvr;
+        }
+      }
+      S.pe_of.assign((size_t)nl * ne, 0u);
+      for (int32_t k = 0; k < nd; ++k) {
+        if (S.dep_bar[k]) continue;
+        const int64_t gd = d0 + k;
+        const int32_t px = d.dep_prod[gd], cx = d.dep_cons[gd];
+        const int32_t Pl = d.instr_loop[x0 + px], ec = d.instr_engine[x0 + cx];
+        if (S.depth[Pl] > 1) pi.lv_pairs += tot(d.instr_loop[x0 + cx], ec);
+        for (int32_t l = par[Pl]; l > 0; l = par[l]) S.pe_of[(size_t)l * ne + ec] |= 1u << d.instr_engine[x0 + px];
+      }
+    }
     auto& sem_of = S.sem_of;
     auto& sem_hist = S.sem_hist;
     sem_of.resize(std::max(nx, nl * ne));
@@ -687,6 +748,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
         const int32_t end_idx = (int32_t)ops.size();
         ops.push_back(make_int4(OP_END, 0, 0, 0));
         rowinfo.push_back(make_int2(end_idx, (has_loop ? 1 : 0) | (lflag[l0 + l] ? 2 : 0) | (S.fbar[l] ? 4 : 0)));
+        const int32_t nh = __builtin_popcount(S.pe_of[(size_t)l * ne + e]);
+        part.hoist.push_back(nh);
+        pi.licm_upd += (int64_t)nh * tot(l, e);
         // next LOOP or END record at or after each record of the row
         opstop.resize(ops.size());
         int32_t next = end_idx;
@@ -834,6 +898,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   HostVec<int64_t> path(all.path);
   HostVec<int32_t> op_ptr(all.rows), opstop(all.opstop);
   HostVec<int2> rowinfo(all.rows);
+  HostVec<int32_t> hoist(all.rows);
   HostVec<int4> ops(all.ops);
   HostVec<int64_t> semhb(all.semhb);
   HostVec<int32_t> plan_ptr(NL);             // one entry per loop; the blocks own consecutive loops
@@ -886,8 +951,10 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
     for (size_t i = 0; i < pt.path.size(); ++i)
       path[B.path + i] = pt.path[i] + (pt.path_kind[i] ? B.rowptr : B.iters);
     for (size_t i = 0; i < pt.op_ptr.size(); ++i) op_ptr[B.rows + i] = pt.op_ptr[i] + b_ops;
-    for (size_t i = 0; i < pt.rowinfo.size(); ++i)
+    for (size_t i = 0; i < pt.rowinfo.size(); ++i) {
       rowinfo[B.rows + i] = make_int2(pt.rowinfo[i].x + b_ops, pt.rowinfo[i].y);
+      hoist[B.rows + i] = pt.hoist[i];
+    }
     for (size_t i = 0; i < pt.opstop.size(); ++i) opstop[B.opstop + i] = pt.opstop[i] + b_ops;
     for (size_t i = 0; i < pt.ops.size(); ++i) {
       int4 v = pt.ops[i];
@@ -1055,6 +1122,9 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.order = h.upload(order, stream, "program order");
   h.op_ptr = h.upload(op_ptr, stream, "op record offsets");
   h.rowinfo = h.upload(rowinfo, stream, "row info");
+  h.cost.hoist = h.upload(hoist, stream, "cached-sum counts");
+  h.cost.xcse = h.upload(xcse, stream, "wait counts with CSE");
+  h.cost.xlvr = h.upload(xlvr, stream, "cached-sum reads");
   h.ops = h.upload(ops, stream, "op records");
   h.opstop = h.upload(opstop, stream, "op stops");
   h.opsem = h.alloc<int4>(kModes * (int64_t)ops.size(), "op semaphore records");
@@ -1252,6 +1322,7 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
   a.sem_cap = std::max(4, (h->nsem_max[mode] + 3) & ~3);
   a.frame_depth = std::max(1, h->depth_max);
   a.warps = h->ne_max;
+  a.cost = h->cost;
   if (fused) {
     a.dep = h->dep; a.ddep = h->ddep; a.path = h->path; a.ord = h->ord;
     a.chk_counts = d_counts; a.chk_first = reinterpret_cast<unsigned long long*>(d_first_bad);
@@ -1270,6 +1341,7 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
   w.issue = d_issue; w.retire = d_retire;
   w.prm = q; w.n_programs = a.n_programs; w.mode = mode;
   w.sem_cap = a.sem_cap; w.frame_depth = a.frame_depth; w.ring = ring; w.lflag = h->lflag; w.paux = h->paux;
+  w.cost = h->cost;
   w.dep = a.dep; w.ddep = a.ddep; w.path = a.path; w.ord = a.ord;
   w.chk_counts = a.chk_counts; w.chk_first = a.chk_first;
   const bool barrier = variant == SYNC_SIM_BARRIER;

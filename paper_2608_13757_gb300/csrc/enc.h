@@ -70,6 +70,9 @@ struct alignas(16) ProgInfo {
   int64_t pair_levels;  // sum over pairs of the per-engine wait's extra levels
   int64_t fb_iters;   // iterations ended by a barrier-fallback barrier (barrier-free);
                       // > 0: simulated by the per-engine kernel
+  int64_t licm_upd;   // LICM (per-engine waits): cached-sum updates, summed over the
+                      // (loop, engine) rows of their counts times the loop's iterations
+  int64_t lv_pairs;   // pairs of per-engine waits whose producer loop has depth > 1
   int32_t ne;
   int32_t le_base;    // row of (top-level loop, engine 0); row of (program-local
                       // loop l, engine e) = le_base + l*ne + e
@@ -165,6 +168,20 @@ struct CheckArgs {
   unsigned long long* first_bad;
 };
 
+// Sec. 6.2's ALU reductions (sync_sim_params.licm / cse), per instruction x:
+//   xcse[x] = {waits computed, of those with a reused mask, of those with a
+//              cached-sum read (producer loop depth > 1, outer sum not
+//              reused), their levels} with CSE;
+//   xlvr[x] = waits whose producer loop has depth > 1 (cached-sum reads
+//             without CSE);
+// per (loop, engine) row: hoist[row] = producer engines whose cached path
+// sums the engine updates at each iteration start of the loop (LICM).
+struct CostTables {
+  const int4* xcse;
+  const int32_t* xlvr;
+  const int32_t* hoist;
+};
+
 struct SimArgs {
   const ProgInfo* prog;
   const int32_t* order;      // program ids in descending-work order
@@ -201,6 +218,7 @@ struct SimArgs {
   const int32_t* ord;        // per-engine mode: engine-stream positions
   unsigned long long* chk_counts;  // optional: [2] unsafe / over-synchronised wait values
   unsigned long long* chk_first;   // optional: [1] smallest offending pair index
+  CostTables cost;
 };
 
 struct SweepArgs {
@@ -244,6 +262,7 @@ struct SweepArgs {
   const int32_t* ord;        // per-engine mode: engine-stream positions
   unsigned long long* chk_counts;  // optional: [2] unsafe / over-synchronised wait values
   unsigned long long* chk_first;   // optional: [1] smallest offending pair index
+  CostTables cost;
 };
 
 // Launchers (return the launch error, if any).

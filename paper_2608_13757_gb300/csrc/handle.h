@@ -70,6 +70,7 @@ struct sync_programs {
   int32_t* order = nullptr;
   int32_t* op_ptr = nullptr;
   int2* rowinfo = nullptr;
+  syncgb::CostTables cost{};        // Sec. 6.2 reductions: per-instruction and per-row counts
   int4* ops = nullptr;
   int32_t* opstop = nullptr;
   int4* opsem = nullptr;            // [kModes][n_ops]

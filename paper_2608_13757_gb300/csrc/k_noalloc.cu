@@ -100,6 +100,7 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
   w.issue = d_issue; w.retire = d_retire;
   w.prm = q; w.n_programs = h->sz.n_programs; w.mode = mode;
   w.sem_cap = sem_cap; w.frame_depth = frame_depth; w.ring = ring; w.lflag = h->lflag; w.paux = h->paux;
+  w.cost = h->cost;
   st = cuda_error(launch_sweep(w, barrier, h->num_sms, s), "sweep simulator kernel");
   if (st != SYNC_OK) return st;
   SimArgs a;
@@ -114,5 +115,6 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
   a.issue = d_issue; a.retire = d_retire;
   a.prm = q; a.n_programs = h->sz.n_programs; a.mode = mode;
   a.sem_cap = sem_cap; a.frame_depth = frame_depth; a.warps = h->ne_max;
+  a.cost = h->cost;
   return cuda_error(launch_simulate(a, barrier, h->num_sms, s), "per-engine simulator kernel");
 }

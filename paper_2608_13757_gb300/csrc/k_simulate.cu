@@ -34,6 +34,7 @@
 // CTAs are persistent and fetch program ids from a counter in descending-work
 // order.  Times are int32: a program whose static time bound exceeds
 // INT32_MAX gets status 4 without being simulated, so no time can overflow.
+#include "cost.cuh"
 #include "waitval.cuh"
 
 namespace syncgb {
@@ -71,13 +72,6 @@ __device__ __forceinline__ unsigned lanemask_le() {
   return m;
 }
 
-__device__ __forceinline__ unsigned long long sat_add(unsigned long long a, unsigned long long b) {
-  const unsigned long long r = a + b;
-  return r < a ? ~0ull : r;
-}
-__device__ __forceinline__ unsigned long long sat_mul(unsigned long long a, unsigned long long b) {
-  return __umul64hi(a, b) ? ~0ull : a * b;
-}
 __device__ __forceinline__ int64_t lohi(int32_t lo, int32_t hi) {
   return (int64_t)(((uint64_t)(uint32_t)hi << 32) | (uint32_t)lo);
 }
@@ -92,32 +86,6 @@ __device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t r
   return ((unsigned long long)x << 32) | y;
 }
 
-// Static time bound of a program under the given costs (saturating).
-template <int MODE, bool BB>
-__device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, const sync_sim_params& q,
-                                                         int32_t cwait) {
-  typedef unsigned long long u64;
-  u64 b = sat_add((u64)pi.agg_lat, sat_mul((u64)q.ii, (u64)pi.n_inst));
-  if (BB) {
-    b = sat_add(b, sat_mul(sat_mul((u64)pi.ne, (u64)pi.n_iter), (u64)q.c_branch));
-    b = sat_add(b, sat_mul((u64)(pi.n_stmt + pi.n_iter), (u64)q.c_barrier));
-  } else {
-    b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
-    if (MODE == SYNC_THR_PERENGINE)
-      b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
-    // control operations of every engine (their own trips): r-hat := 0 at
-    // statements and the branch, r++ and r-hat++ at iteration starts, minus
-    // the r-hat ops of loops without a trip register when that is elided
-    const u64 el = q.trip_register_elision ? 1 : 0;
-    const u64 rhat_stmts = (u64)pi.eng_stmt - el * (u64)pi.el_stmt;
-    const u64 rhat_iters = (u64)pi.eng_iter - el * (u64)pi.el_iter;
-    b = sat_add(b, sat_mul(rhat_stmts, (u64)q.c_regop));
-    b = sat_add(b, sat_mul((u64)pi.eng_iter, (u64)q.c_branch + (u64)q.c_regop));
-    b = sat_add(b, sat_mul(rhat_iters, (u64)q.c_regop));
-    b = sat_add(b, sat_mul((u64)pi.fb_iters, (u64)q.c_barrier));   // barrier-fallback barriers
-  }
-  return b;
-}
 
 struct Smem {
   int64_t* semhb;          // [sem_cap]
@@ -190,7 +158,7 @@ __device__ __forceinline__ void set_row(const SimArgs& a, Eng& E, int32_t row) {
   // barrier-free with trip-register elision, a loop carrying no offset > 0
   // has no r-hat++ at its iteration starts
   const int32_t ic = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
-  E.ic = !BB && a.prm.trip_register_elision && (ri.y & 2) ? ic - a.prm.c_regop : ic;
+  E.ic = (!BB && a.prm.trip_register_elision && (ri.y & 2) ? ic - a.prm.c_regop : ic) + hoist_ops<MODE, BB>(a, row);
 }
 
 // Fused simulation: the wait value of consumer-grouped dependency r for the
@@ -225,7 +193,6 @@ __device__ __forceinline__ int32_t fused_value(const SimArgs& a, const Frame* fr
 template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng& E, int w, int lane,
                                            int ne, unsigned long long& chk) {
-  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t ii = a.prm.ii;
   Frame* frames = S.frames + w * a.frame_depth;
   bool moved = false;
@@ -346,8 +313,7 @@ __device__ __forceinline__ bool run_engine(const SimArgs& a, const Smem& S, Eng&
       atomicMin(S.tally + 2, first);
     }
     // cursor maps t' = max(t + A, B), inclusive scan over the lanes
-    const int32_t wcost =
-        BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * srec.w : 0);
+    const int32_t wcost = BB ? 0 : wait_ops<MODE>(a, rec, srec.w);
     int32_t A = 0, B = kNeg;
     if (in) {
       if (dp) { A = wcost + ii; B = waited ? ready + ii : kNeg; }

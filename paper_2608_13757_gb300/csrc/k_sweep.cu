@@ -30,6 +30,7 @@
 // drained times.  Per-engine cursor, last retire and instance count live in
 // shared memory, read by the engine's lanes and written back by the last
 // lane of its run.
+#include "cost.cuh"
 #include "waitval.cuh"
 
 namespace syncgb {
@@ -52,13 +53,6 @@ __host__ __device__ __forceinline__ size_t warp_bytes(int sem_cap, int frame_dep
   return (per + 15) & ~(size_t)15;
 }
 
-__device__ __forceinline__ unsigned long long sat_add(unsigned long long a, unsigned long long b) {
-  const unsigned long long r = a + b;
-  return r < a ? ~0ull : r;
-}
-__device__ __forceinline__ unsigned long long sat_mul(unsigned long long a, unsigned long long b) {
-  return __umul64hi(a, b) ? ~0ull : a * b;
-}
 __device__ __forceinline__ unsigned lanemask_le() {
   unsigned m;
   asm("mov.u32 %0, %%lanemask_le;" : "=r"(m));
@@ -73,30 +67,12 @@ __device__ __forceinline__ unsigned long long inst_term(int32_t issue, int32_t r
   return ((unsigned long long)x << 32) | y;
 }
 
+
+// Engines pay different iteration-start costs only with LICM's cached-sum
+// updates (per-engine waits, barrier-free).
 template <int MODE, bool BB>
-__device__ __forceinline__ unsigned long long time_bound(const ProgInfo& pi, const sync_sim_params& q,
-                                                         int32_t cwait) {
-  typedef unsigned long long u64;
-  u64 b = sat_add((u64)pi.agg_lat, sat_mul((u64)q.ii, (u64)pi.n_inst));
-  if (BB) {
-    b = sat_add(b, sat_mul(sat_mul((u64)pi.ne, (u64)pi.n_iter), (u64)q.c_branch));
-    b = sat_add(b, sat_mul((u64)(pi.n_stmt + pi.n_iter), (u64)q.c_barrier));
-  } else {
-    b = sat_add(b, sat_mul((u64)cwait, (u64)pi.n_pairs));
-    if (MODE == SYNC_THR_PERENGINE)
-      b = sat_add(b, sat_mul((u64)q.c_wait_ops_perengine_level, (u64)pi.pair_levels));
-    // control operations of every engine (their own trips): r-hat := 0 at
-    // statements and the branch, r++ and r-hat++ at iteration starts, minus
-    // the r-hat ops of loops without a trip register when that is elided
-    const u64 el = q.trip_register_elision ? 1 : 0;
-    const u64 rhat_stmts = (u64)pi.eng_stmt - el * (u64)pi.el_stmt;
-    const u64 rhat_iters = (u64)pi.eng_iter - el * (u64)pi.el_iter;
-    b = sat_add(b, sat_mul(rhat_stmts, (u64)q.c_regop));
-    b = sat_add(b, sat_mul((u64)pi.eng_iter, (u64)q.c_branch + (u64)q.c_regop));
-    b = sat_add(b, sat_mul(rhat_iters, (u64)q.c_regop));
-    b = sat_add(b, sat_mul((u64)pi.fb_iters, (u64)q.c_barrier));   // barrier-fallback barriers
-  }
-  return b;
+__device__ __forceinline__ bool hoists(const SweepArgs& a) {
+  return !BB && MODE == SYNC_THR_PERENGINE && a.prm.licm != 0;
 }
 
 struct WarpSmem {
@@ -226,7 +202,6 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
                                          const int32_t (&T)[kMaxDeps], int32_t g, int32_t copies,
                                          int32_t ctag, int lane, int lc, int32_t lo_c, int32_t iter_cost,
                                          unsigned long long& chk, BbRep& rp, BfPred& pd) {
-  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int4 rec = L.rec, sr = L.sr;
   const bool have = lane < ch.y;
   const bool valid = have && L.meta.y < copies;
@@ -268,8 +243,11 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
             __ldg(a.dsem + rec.w + j));
   if (__ballot_sync(kFull, fallback)) return SIM_FALLBACK;
 
-  const int32_t wcost = BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * sr.w : 0);
-  const int32_t apre = (L.meta.w & LANE_ITER_START) ? iter_cost : 0;
+  const int32_t wcost = BB ? 0 : wait_ops<MODE>(a, rec, sr.w);
+  // iter_cost is the iteration-start cost of lane `lane`'s engine (engines
+  // differ only by LICM's cached-sum updates); a record takes its engine's
+  const int32_t ic_e = hoists<MODE, BB>(a) ? __shfl_sync(kFull, iter_cost, e) : iter_cost;
+  const int32_t apre = (L.meta.w & LANE_ITER_START) ? ic_e : 0;
   const int32_t A = valid ? apre + wcost + a.prm.ii : 0;
   int32_t issue = 0, retire = 0, t_after = 0;
   // REP: every engine starts the iteration at the same cursor t_in with all
@@ -493,7 +471,6 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
                                              const int4 ch, const LaneRec& L, int32_t lo, int32_t hi,
                                              int32_t ctag, int lane, int lc, int32_t iter_cost,
                                              unsigned long long& chk) {
-  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
   const int32_t ii = a.prm.ii;
   const int32_t copies = ch.z;
   const bool have = lane < ch.y;
@@ -545,8 +522,11 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
   bool rep = false;
   int32_t rd_issue = 0, rd_retire = 0, rd_t = 0, rd_r = 0, rk0 = 0, rk1 = 0;
 
-  const int32_t wcost = L.rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * L.sr.w : 0);
-  const int32_t P = (BB ? 0 : wcost) + ((L.meta.w & LANE_ITER_START) ? iter_cost : 0);
+  const int32_t wcost = BB ? 0 : wait_ops<MODE>(a, L.rec, L.sr.w);
+  // iter_cost: the iteration-start cost of lane `lane`'s engine (state
+  // lanes); a record lane takes its engine's
+  const int32_t ic_e = hoists<MODE, BB>(a) ? __shfl_sync(kFull, iter_cost, e) : iter_cost;
+  const int32_t P = wcost + ((L.meta.w & LANE_ITER_START) ? ic_e : 0);
   const int32_t A = P + ii;                           // cursor advance of a valid lane with no wait
   int32_t T0n = 0, T1n = 0;
   int32_t fk0 = -1, fc0 = 0, fn0 = 0, fk1 = -1, fc1 = 0, fn1 = 0;   // fused: see fused_setup
@@ -739,8 +719,7 @@ __device__ __forceinline__ int run_single(const SweepArgs& a, const WarpSmem& S,
   if (flag == 2) return SIM_FALLBACK;
   if (flag == 1) return SYNC_PROG_DEADLOCK;
   ready = __shfl_sync(kFull, ready, 0);
-  const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
-  const int32_t wcost = BB ? 0 : rec.z * cwait + (MODE == SYNC_THR_PERENGINE ? a.prm.c_wait_ops_perengine_level * sr.w : 0);
+  const int32_t wcost = BB ? 0 : wait_ops<MODE>(a, rec, sr.w);
   const int32_t t_in = S.t[e], lr_in = S.lr[e];
   const uint32_t nj = (uint32_t)S.nn[e] + 1;
   const int32_t t_after = max(t_in + wcost + a.prm.ii, ready >= 0 ? ready + a.prm.ii : kNeg);
@@ -849,7 +828,6 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
   // elision is on (barrier-free: no r-hat := 0, no r-hat++)
   const bool elide = !BB && a.prm.trip_register_elision != 0;
   const int32_t ic_full = BB ? a.prm.c_branch : a.prm.c_branch + 2 * a.prm.c_regop;
-  auto iter_cost_of = [&](int32_t flag) { return elide && flag ? ic_full - a.prm.c_regop : ic_full; };
   auto stmt_cost_of = [&](int32_t flag) { return elide && flag ? 0 : a.prm.c_regop; };
 
   for (;;) {
@@ -859,6 +837,13 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     if (slot >= a.n_programs) break;
     const int p = __ldg(a.order + slot);
     const ProgInfo pi = a.prog[p];
+    // the iteration-start cost of global loop `loop` on lane `lane`'s engine
+    // (lanes past the engines: any value); flag: its trip register is elidable
+    auto iter_cost_of = [&](int32_t flag, int32_t loop) {
+      int32_t c = elide && flag ? ic_full - a.prm.c_regop : ic_full;
+      if (hoists<MODE, BB>(a) && lane < pi.ne) c += hoist_ops<MODE, BB>(a, pi.le_base + (loop - pi.loop_base) * pi.ne + lane);
+      return c;
+    };
     BbRep no_rep;                     // a segment's chunk is neither replayed
     BfPred no_pred;                   // nor predicted
     // engines on their own trips (no common walk), or barrier-free with the
@@ -903,7 +888,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         } else {
           const Frame f = S.frames[--sp];
           loop = f.loop; item = f.item; g = f.g; g_end = f.g_end;
-          iter_cost = iter_cost_of(__ldg(a.lflag + loop));
+          iter_cost = iter_cost_of(__ldg(a.lflag + loop), loop);
           pbeg = __ldg(a.plan_ptr + loop);
           pend = __ldg(a.plan_ptr + loop + 1);
         }
@@ -916,7 +901,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         } else {
           if (lane < pi.ne) S.t[lane] += stmt_cost_of(it.z);
         }
-        const int32_t child_ic = iter_cost_of(it.z);
+        const int32_t child_ic = iter_cost_of(it.z, it.y);
         // the statement's side record: the child's trip prefix sums, and the
         // chunk holding its whole body (if one does), fetched together
         const int4 ax = __ldg(a.paux + pbeg + item);

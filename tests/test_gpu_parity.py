@@ -59,7 +59,10 @@ def compare_all(sg, batch, params=None, timeline=False, modes=MODES):
         assert np.array_equal(got, want), f"thresholds differ (mode {mode})"
         counts, fb = sg.sync_check_minimal(h, mode, thr)
         assert counts.cpu().tolist() == [0, 0] and fb.item() == -1
-        for v in ((oracle.BARRIER_FREE,) if batch.divergent else variants_for(mode)):
+        vs = (oracle.BARRIER_FREE,) if batch.divergent else variants_for(mode)
+        if getattr(batch, "nonalloc_policy", 0):     # barrier fallbacks: no unrolled variant
+            vs = tuple(v for v in vs if v != oracle.UNROLLED)
+        for v in vs:
             ref = oracle.simulate(batch, want, mode, v, prm, timeline=timeline)
             res = sg.sync_simulate(h, mode, thr, sim_params(prm), v, timeline=timeline)
             fused, fcounts, ffirst = sg.sync_simulate_fused(h, mode, sim_params(prm), v, timeline=timeline,
@@ -498,3 +501,81 @@ def test_code_size_proxy_matches_oracle(sg):
         assert h.sizes.code_bytes_looped == sg.CODE_BYTES_PER_INSTR * lo
         assert h.sizes.code_bytes_unrolled == sg.CODE_BYTES_PER_INSTR * un
         h.close()
+
+
+# ---------------------------------------- Sec. 6.2's ALU reductions (NEXT-3)
+
+REDUCTIONS = [dict(licm=1), dict(cse=1), dict(licm=1, cse=1)]
+
+
+@pytest.mark.parametrize("red", REDUCTIONS, ids=["licm", "cse", "licm+cse"])
+@pytest.mark.parametrize("seed", range(3))
+def test_alu_reductions_random_trees(sg, red, seed):
+    """LICM / CSE in every mode and scheme, array and fused, timelines
+    included, equal to the oracle on random trees with several waits per
+    consumer and deep producer loops."""
+    batch = workloads.random_trees(9300 + seed, 150, workloads.tree_params(
+        engines_hi=5, loops_hi=6, body_hi=6, trip_hi=4, max_depth=4, max_deps_per_cons=3))
+    compare_all(sg, batch, timeline=True, modes=ALL_MODES,
+                params=oracle.sim_params(ii=2, c_branch=3, c_regop=2, c_wait_ops_count=4, c_wait_ops_perloop=6,
+                                         c_wait_ops_perengine_level=3, **red))
+
+
+@pytest.mark.parametrize("name,n", [("depth2", 24), ("gemm", None), ("attention", 1), ("chain", 300),
+                                    ("syncbound", 300)])
+def test_alu_reductions_configs(sg, name, n):
+    batch = workloads.generate(name, n_programs=n)
+    for red in REDUCTIONS:
+        compare_all(sg, batch, timeline=name == "depth2", modes=ALL_MODES, params=oracle.sim_params(**red))
+
+
+def test_alu_reductions_in_the_per_engine_kernel(sg):
+    """Programs the sweep hands to the per-engine kernel -- barrier
+    fallbacks (barrier-free), waits on later producers, per-engine trips --
+    with the reductions on."""
+    from tests.test_fallback_pins import FAR
+    fb = workloads.random_trees(9400, 60, workloads.tree_params(**FAR))
+    fb.nonalloc_policy = 1
+    b = workloads.ProgramBuilder(2)          # a consumer ahead of its producer on another engine
+    A = b.loop(0, 0, [3])
+    B = b.loop(A, 1, [2, 2, 2])
+    c = b.instr(A, 0, 1)
+    p = b.instr(B, 0, 0)
+    q = b.instr(A, 2, 0)
+    b.dep(q, c, 0)
+    b.dep(p, c, 1)
+    b.dep(p, q, 0)
+    fwd = b.batch()
+    fwd.nonalloc_policy = 1
+    mixed = workloads.concat([fb, fwd, workloads.generate("depth2", n_programs=6)])
+    for red in REDUCTIONS:
+        compare_all(sg, mixed, timeline=True, modes=ALL_MODES,
+                    params=oracle.sim_params(c_regop=2, c_wait_ops_perengine_level=4, **red))
+    div = workloads.diverge(workloads.random_trees(9401, 60, workloads.tree_params(max_deps_per_cons=3)), 4,
+                            permille=200)
+    compare_all(sg, div, timeline=True, modes=MODES, params=oracle.sim_params(cse=1))
+
+
+def test_alu_reductions_overflow_bound(sg):
+    """The static bound with LICM's cached-sum updates (the oracle's pinned
+    overflow case) and with wait ops counted before CSE."""
+    b = workloads.ProgramBuilder(1)
+    A = b.loop(0, 0, [1100])
+    B = b.loop(A, 0, [1] * 1100)
+    p = b.instr(B, 0, 0)
+    C = b.loop(A, 1, [0] * 1100)
+    x = b.instr(C, 0, 0)
+    b.dep(p, x, 0)
+    c = workloads.ProgramBuilder(1)
+    L = c.loop(0, 0, [100])
+    pc = c.instr(L, 0, 0)
+    for i in range(8):
+        c.dep(pc, c.instr(L, 10 + i, 0), 0)
+    batch = workloads.concat([b.batch(), c.batch()])
+    for kw in (dict(c_wait_ops_perengine_level=2 ** 21, licm=1), dict(c_wait_ops_perengine_level=2 ** 20, licm=1),
+               dict(c_wait_ops_count=2 ** 22, c_wait_ops_perloop=2 ** 22, cse=1)):
+        compare_all(sg, batch, modes=ALL_MODES, params=oracle.sim_params(**kw))
+    thr = oracle.thresholds(batch, PERENGINE)
+    st = oracle.simulate(batch, thr, PERENGINE, oracle.BARRIER_FREE,
+                         oracle.sim_params(c_wait_ops_perengine_level=2 ** 21, licm=1)).status
+    assert st[0] == 4
