@@ -534,6 +534,7 @@ def test_alu_reductions_in_the_per_engine_kernel(sg):
     fallbacks (barrier-free), waits on later producers, per-engine trips --
     with the reductions on."""
     from tests.test_fallback_pins import FAR
+    from tests.test_gpu_fallback import compare_fallback
     fb = workloads.random_trees(9400, 60, workloads.tree_params(**FAR))
     fb.nonalloc_policy = 1
     b = workloads.ProgramBuilder(2)          # a consumer ahead of its producer on another engine
@@ -545,12 +546,12 @@ def test_alu_reductions_in_the_per_engine_kernel(sg):
     b.dep(q, c, 0)
     b.dep(p, c, 1)
     b.dep(p, q, 0)
-    fwd = b.batch()
-    fwd.nonalloc_policy = 1
-    mixed = workloads.concat([fb, fwd, workloads.generate("depth2", n_programs=6)])
+    fwd = workloads.concat([b.batch(), workloads.generate("depth2", n_programs=6)])
+    mixed = workloads.concat([fb, workloads.generate("depth2", n_programs=6)])
     for red in REDUCTIONS:
-        compare_all(sg, mixed, timeline=True, modes=ALL_MODES,
-                    params=oracle.sim_params(c_regop=2, c_wait_ops_perengine_level=4, **red))
+        prm = oracle.sim_params(c_regop=2, c_wait_ops_perengine_level=4, **red)
+        compare_fallback(sg, mixed, prm=prm)           # fallback barriers: wait values 0 on their pairs
+        compare_all(sg, fwd, timeline=True, modes=ALL_MODES, params=prm)
     div = workloads.diverge(workloads.random_trees(9401, 60, workloads.tree_params(max_deps_per_cons=3)), 4,
                             permille=200)
     compare_all(sg, div, timeline=True, modes=MODES, params=oracle.sim_params(cse=1))
