@@ -131,9 +131,23 @@ class ClockSampler:
 
 # ------------------------------------------------------------- GPU side
 
-def kernel_hash() -> str:
+# the sources each kernel's code is compiled from (enc.h: the shared tables)
+KERNEL_SOURCES = {
+    "thresholds": ("k_thresholds.cu", "waitval.cuh", "enc.h"),
+    "check": ("k_thresholds.cu", "waitval.cuh", "enc.h"),
+    "sim_barrier_free": ("k_sweep.cu", "k_simulate.cu", "cost.cuh", "waitval.cuh", "enc.h"),
+    "sim_barrier": ("k_sweep.cu", "k_simulate.cu", "cost.cuh", "waitval.cuh", "enc.h"),
+}
+
+
+def kernel_hash(kernel: str = "sim_barrier_free", read=None) -> str:
+    """Hash of the sources a kernel is built from (read(name) -> bytes
+    overrides reading them from the tree)."""
     h = hashlib.sha256()
-    for f in ("k_thresholds.cu", "k_simulate.cu", "k_sweep.cu", "enc.h", "waitval.cuh"):
+    for f in KERNEL_SOURCES[kernel]:
+        if read is not None:
+            h.update(read(f))
+            continue
         with open(os.path.join(ROOT, "paper_2608_13757_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -141,12 +155,12 @@ def kernel_hash() -> str:
 
 def profile_entry(kernel: str, workload: str):
     """A kernel's record in the committed ncu summary (profiles/traffic.json),
-    if it was taken on the current kernel sources."""
+    if it was taken on the current sources of that kernel."""
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             d = json.load(f)
         e = d.get(workload, {}).get(kernel)
-        if e and e.get("source_hash") == kernel_hash():
+        if e and e.get("source_hash") == kernel_hash(kernel):
             return e
     except Exception:
         pass

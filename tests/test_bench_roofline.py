@@ -46,6 +46,6 @@ def test_roofline_takes_profile_records(monkeypatch):
 
 
 def test_profile_records_need_the_current_sources(monkeypatch):
-    monkeypatch.setattr(bench, "kernel_hash", lambda: "not-the-captured-hash")
+    monkeypatch.setattr(bench, "kernel_hash", lambda *a, **k: "not-the-captured-hash")
     assert bench.traffic_for("thresholds", "chain") is None
     assert bench.profile_entry("sim_barrier_free", "chain") is None
