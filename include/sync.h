@@ -44,6 +44,9 @@
  *    per hardware thread, at most 32, at least 256 programs each).
  *  - SYNCGB_WIDE_INDEX=1: the threshold and check kernels index pairs with
  *    64-bit integers even when 32 bits suffice.
+ *  - SYNCGB_SPLIT_MIN=n (read by sync_load_programs): the fewest instances a
+ *    program needs to be simulated in pieces on several warps (default
+ *    65536; see sync_simulate).
  */
 #ifndef SYNC_H
 #define SYNC_H
@@ -196,6 +199,9 @@ typedef struct {
   int64_t code_bytes_unrolled; /* the same for the unrolled program: one
                                   instruction per datapath instance and one
                                   static wait per waited pair                 */
+  int32_t n_split_programs;    /* programs sync_simulate may simulate in pieces
+                                  on several warps (see sync_simulate)        */
+  int32_t n_pieces;            /* their pieces                                */
 } sync_sizes;
 
 /* Instruction size of the code-size proxy (a 128-bit instruction word). */
@@ -346,6 +352,14 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  * iteration-start costs above as described there; with licm the static time
  * bound (SYNC_PROG_OVERFLOW) adds c_wait_ops_perengine_level per cached-sum
  * update and c_regop per pair of a wait with a cached-sum read.
+ * Large programs (sync_sizes.n_split_programs) whose top-level body is one
+ * loop L are simulated in pieces -- runs of L's iterations -- on separate
+ * warps when every wait of a piece targets an increment of the same piece
+ * (checked on the thresholds of each call; otherwise, and whenever a piece
+ * deadlocks or waits forward, the program is simulated whole): the barrier
+ * scheme from the barrier before each piece, the barrier-free scheme by
+ * composing the pieces' max-plus maps of the engines' cursors and last
+ * retires.  The results are identical either way.
  * UNROLLED: as barrier-free with c_branch, c_regop and every wait-op cost
  * taken as 0 (ii and latencies unchanged); it requires PERENGINE and a batch
  * without barrier-fallback dependencies, and returns SYNC_ERR_ARG otherwise.

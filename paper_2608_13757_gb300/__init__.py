@@ -61,7 +61,8 @@ class Sizes(ctypes.Structure):
                 ("n_instrs", ctypes.c_int32), ("n_deps", ctypes.c_int32),
                 ("device_bytes", ctypes.c_int64), ("h2d_bytes", ctypes.c_int64),
                 ("struct_bytes", ctypes.c_int64), ("code_bytes_looped", ctypes.c_int64),
-                ("code_bytes_unrolled", ctypes.c_int64)]
+                ("code_bytes_unrolled", ctypes.c_int64), ("n_split_programs", ctypes.c_int32),
+                ("n_pieces", ctypes.c_int32)]
 
 
 class SimParams(ctypes.Structure):

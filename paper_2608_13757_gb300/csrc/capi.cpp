@@ -188,6 +188,146 @@ std::string where(int32_t p, const char* what, int64_t i) {
 
 }  // namespace
 
+// Piece-parallel simulation (PieceArgs in enc.h): which programs are split,
+// into which pieces, and what each piece starts from.  A program qualifies
+// when its top-level body is one loop L (no instruction of its own), its
+// engines share their trips and it has no fallback barriers, L runs at least
+// twice, and it is large against the batch: at least 65536 instances (the
+// environment variable SYNCGB_SPLIT_MIN sets another floor) and
+// more than 8 times the instances per resident sweep warp (152 SMs x 24
+// warps on a GB300) of the whole batch, so that its serial walk, not the
+// batch's throughput, bounds the simulation (the barrier scheme runs each
+// piece twice).  The barrier-free scheme runs 2*ne + 1 passes per piece, so
+// it splits only programs above 4 * (2*ne + 1) times that share.
+static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop, const HostVec<int32_t>& rowptr,
+                         const HostVec<int4>& xsem, const HostVec<DepInfo>& dep, const HostVec<int64_t>& seg,
+                         const HostVec<int64_t>& semhb, const HostVec<ProgInfo>& prog, int64_t n_inst,
+                         cudaStream_t stream, sync_programs& h) {
+  const int32_t P = d.n_programs;
+  const int64_t NX = d.prog_instr_ptr[P];
+  const double share = (double)n_inst / ((double)h.num_sms * 24.0);
+  int64_t min_inst = 65536;                       // SYNCGB_SPLIT_MIN=n lowers it (tests)
+  if (const char* e = std::getenv("SYNCGB_SPLIT_MIN")) min_inst = std::max<int64_t>(1, std::atoll(e));
+  std::vector<int32_t> split_of(P, -1);
+  std::vector<SplitProg> splits;
+  std::vector<PieceInfo> pieces;
+  std::vector<VDep> vdep;
+  std::vector<int32_t> pub, cnt, bf_init;
+  int64_t hist_split[kModes] = {0, 0, 0};
+  int32_t ne_max = 0;
+  std::vector<int32_t> path, row;
+  for (int32_t p = 0; p < P; ++p) {
+    const ProgInfo& pi = prog[p];
+    if (pi.divergent || pi.fb_iters > 0 || pi.n_inst < min_inst || (double)pi.n_inst <= 8.0 * share) continue;
+    const int32_t l0 = d.prog_loop_ptr[p], nl = d.prog_loop_ptr[p + 1] - l0;
+    const int32_t x0 = d.prog_instr_ptr[p], nx = d.prog_instr_ptr[p + 1] - x0;
+    int32_t L = -1, children = 0;
+    bool own = false;
+    for (int32_t l = 1; l < nl; ++l)
+      if (d.loop_parent[l0 + l] == 0) { ++children; L = l; }
+    for (int32_t x = 0; x < nx; ++x) own = own || d.instr_loop[x0 + x] == 0;
+    if (children != 1 || own) continue;
+    const int32_t T = loop[l0 + L].total;
+    if (T < 2) continue;
+    // instances of instruction x before iteration g of L: L's iterations
+    // 0..g-1 hold, for a loop m below L, the iterations of m that start
+    // before them -- the trip prefix sums composed from L's child down to m
+    auto count = [&](int32_t x, int32_t g) {
+      int32_t m = d.instr_loop[x0 + x];
+      path.clear();
+      for (; m != L; m = d.loop_parent[l0 + m]) path.push_back(m);
+      int64_t c = g;
+      for (size_t i = path.size(); i-- > 0;) c = rowptr[loop[l0 + path[i]].rowptr_off + c];
+      return (int32_t)c;
+    };
+    // pieces: at most 64 runs of L's iterations, of about equal instances
+    const int32_t np = std::min<int32_t>(T, 64);
+    std::vector<int32_t> bnd(np + 1, 0);
+    bnd[np] = T;
+    if ((int64_t)T * nx <= (4 << 20)) {
+      std::vector<int64_t> before(T + 1, 0);         // instances before each iteration of L
+      for (int32_t g = 0; g <= T; ++g)
+        for (int32_t x = 0; x < nx; ++x) before[g] += count(x, g);
+      for (int32_t j = 1; j < np; ++j) {
+        const int64_t target = before[T] * j / np;
+        int32_t g = (int32_t)(std::lower_bound(before.begin(), before.end(), target) - before.begin());
+        bnd[j] = std::min(std::max(g, bnd[j - 1] + 1), T - (np - j));
+      }
+    } else {
+      for (int32_t j = 1; j < np; ++j) bnd[j] = (int32_t)((int64_t)T * j / np);
+    }
+    SplitProg S{};
+    S.prog = p; S.first_piece = (int32_t)pieces.size(); S.n_pieces = np; S.nx = nx;
+    S.ne = pi.ne; S.loop = l0 + L;
+    S.cnt_base = (int64_t)cnt.size();
+    for (int32_t j = 0; j <= np; ++j)
+      for (int32_t x = 0; x < nx; ++x) cnt.push_back(count(x, bnd[j]));
+    S.vdep0 = (int32_t)vdep.size();
+    for (int32_t k = d.prog_dep_ptr[p]; k < d.prog_dep_ptr[p + 1]; ++k) {
+      if (dep[k].kase == CASE_BARRIER) continue;
+      VDep v{};
+      v.seg = seg[k];
+      v.cons = d.dep_cons[k];
+      for (int m = 0; m < kModes; ++m) v.sem[m] = xsem[(size_t)m * NX + x0 + d.dep_prod[k]].x;
+      vdep.push_back(v);
+    }
+    S.vdep1 = (int32_t)vdep.size();
+    // a semaphore's increments before a point: the instances before it of the
+    // instructions that increment it (each instance increments once)
+    int64_t span[kModes] = {0, 0, 0};
+    for (int32_t j = 0; j < np; ++j) {
+      PieceInfo pc{};
+      pc.prog = p; pc.split = (int32_t)splits.size(); pc.loop = l0 + L; pc.g0 = bnd[j]; pc.g1 = bnd[j + 1];
+      const int32_t* c = cnt.data() + S.cnt_base + (int64_t)j * nx;
+      for (int m = 0; m < kModes; ++m) {
+        pc.pub_off[m] = (int32_t)pub.size();
+        pub.resize(pub.size() + pi.nsem[m], 0);
+        for (int32_t x = 0; x < nx; ++x) {
+          const int32_t sm = xsem[(size_t)m * NX + x0 + x].x;
+          if (sm >= 0) pub[pc.pub_off[m] + sm] += c[x];
+        }
+      }
+      pc.nbase_off = (int32_t)pub.size();
+      pub.resize(pub.size() + pi.ne, 0);
+      for (int32_t x = 0; x < nx; ++x) pub[pc.nbase_off + d.instr_engine[x0 + x]] += c[x];
+      pieces.push_back(pc);
+    }
+    // probe histories: the program's history entries, per probe, at the
+    // split programs' running offset (its entries are contiguous per mode)
+    const int32_t* tot = cnt.data() + S.cnt_base + (int64_t)np * nx;
+    for (int m = 0; m < kModes; ++m) {
+      for (int32_t x = 0; x < nx; ++x)
+        if (xsem[(size_t)m * NX + x0 + x].x >= 0) span[m] += tot[x];
+      const int64_t first = pi.nsem[m] > 0 ? semhb[pi.semhb_off[m]] : 0;
+      for (int32_t j = 0; j < np; ++j) pieces[S.first_piece + j].hdelta[m] = hist_split[m] - first;
+      hist_split[m] += span[m];
+    }
+    const bool bf = (double)pi.n_inst > 4.0 * (2.0 * pi.ne + 1.0) * share;
+    bf_init.push_back(bf ? 0 : 1);
+    if (bf) ne_max = std::max(ne_max, pi.ne);
+    split_of[p] = (int32_t)splits.size();
+    splits.push_back(S);
+  }
+  if (splits.empty()) return;
+  h.n_split = (int32_t)splits.size();
+  h.n_pieces = (int32_t)pieces.size();
+  h.sz.n_split_programs = h.n_split;
+  h.sz.n_pieces = h.n_pieces;
+  h.probes_bf = std::max(1, 2 * ne_max);
+  h.any_bf = ne_max > 0;
+  for (int m = 0; m < kModes; ++m) h.phist_len[m] = hist_split[m];
+  h.pieces = h.upload(pieces, stream, "pieces");
+  h.splits = h.upload(splits, stream, "split programs");
+  h.prog_split = h.upload(split_of, stream, "program split index");
+  h.piece_pub = h.upload(pub, stream, "piece start counts");
+  h.piece_cnt = h.upload(cnt, stream, "piece instance counts");
+  h.vdep = h.upload(vdep, stream, "split programs' dependencies");
+  h.piece_bf_init = h.upload(bf_init, stream, "barrier-free split flags");
+  h.piece_fail = h.alloc<int32_t>(h.n_split, "piece validation flags");
+  h.piece_out = h.alloc<int32_t>((int64_t)h.n_pieces * h.probes_bf * 64, "piece probe states");
+  h.piece_x = h.alloc<int32_t>((int64_t)h.n_pieces * 64, "piece start states");
+}
+
 static void build(const sync_batch_desc& d, int device, cudaStream_t stream, sync_programs& h) {
   // ---------------------------------------------------------- shape checks
   if (d.n_programs < 0) raise(SYNC_ERR_ARG, "n_programs < 0");
@@ -1152,6 +1292,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.n_lanes = (int64_t)lrec.size();
   LoopInfo* d_xloops = h.upload(xloops, stream, "iteration spaces");
   h.divergent = div;
+  build_pieces(d, loop, rowptr_host, xsem, dep, h.seg_host, semhb, prog, n_inst, stream, h);
   cuda_check(launch_expand(d_xloops, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
   cuda_check(launch_sem_records(d_xsem, NX, h.ops, h.n_ops, h.lrec, h.n_lanes, h.opsem, h.lsem, h.num_sms, stream),
              "semaphore records");
@@ -1275,6 +1416,16 @@ sync_status sync_check_minimal(const sync_programs* h, sync_thr_mode mode, const
   }
 }
 
+// The probe runs' private semaphore histories of a mode (barrier-free piece
+// simulation), allocated on first use and kept by the handle.
+static int32_t* probe_history(const sync_programs* h, sync_thr_mode mode) {
+  std::lock_guard<std::mutex> lock(h->phist_mu);
+  if (!h->phist[mode])
+    h->phist[mode] = h->alloc_lazy<int32_t>((int64_t)h->probes_bf * std::max<int64_t>(h->phist_len[mode], 1),
+                                            "probe histories");
+  return h->phist[mode];
+}
+
 // Both simulation entry points: thresholds from d_thr, or (fused) from the
 // simulators' loop state, optionally checked.
 static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, const int32_t* d_thr,
@@ -1345,6 +1496,24 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
   w.dep = a.dep; w.ddep = a.ddep; w.path = a.path; w.ord = a.ord;
   w.chk_counts = a.chk_counts; w.chk_first = a.chk_first;
   const bool barrier = variant == SYNC_SIM_BARRIER;
+  // split programs (array thresholds): simulated piece by piece on many warps
+  // first; the sweep skips the ones the pieces completed
+  if (!fused && h->n_split > 0 && (barrier || h->any_bf)) {
+    const size_t flags = sizeof(int32_t) * (size_t)h->n_split;
+    if (barrier) {
+      cuda_check(cudaMemsetAsync(h->piece_fail, 0, flags, st), "cudaMemsetAsync");
+    } else {
+      w.pcs.phist = probe_history(h, mode);
+      w.pcs.phist_len = h->phist_len[mode];
+      cuda_check(cudaMemcpyAsync(h->piece_fail, h->piece_bf_init, flags, cudaMemcpyDeviceToDevice, st),
+                 "cudaMemcpyAsync");
+    }
+    w.pcs.piece = h->pieces; w.pcs.split = h->splits; w.pcs.prog_split = h->prog_split;
+    w.pcs.pub = h->piece_pub; w.pcs.fail = h->piece_fail; w.pcs.out = h->piece_out; w.pcs.x = h->piece_x;
+    w.pcs.n_pieces = h->n_pieces;
+    w.pcs.probes = barrier ? 1 : h->probes_bf;
+    cuda_check(launch_pieces(w, barrier, h->vdep, h->piece_cnt, h->n_split, h->num_sms, st), "piece simulation");
+  }
   cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");
   a.only = h->fallback;
   cuda_check(launch_simulate(a, barrier, h->num_sms, st), "per-engine simulator kernel");

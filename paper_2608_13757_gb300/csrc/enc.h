@@ -182,6 +182,62 @@ struct CostTables {
   const int32_t* hoist;
 };
 
+// Piece-parallel simulation of a large program whose top-level body is one
+// loop L: the program is cut into pieces of consecutive iterations of L,
+// simulated on separate warps.  Per piece (built at load time): the
+// instances of every instruction before it, and from those the engines'
+// instance counts and each waited semaphore's published increments at its
+// start.  Per call: a validation that every wait of a piece targets an
+// increment the piece itself produces (else the program is simulated whole),
+// then barrier scheme: one pass per piece from a barrier release at 0 and a
+// prefix sum of the piece durations; barrier-free: the piece's end state
+// (engine cursors and last retires) is a max-plus linear map of its start
+// state, read off by one probe run per state variable (the variable raised
+// by kProbe, the others 0), composed piece by piece.  A final pass runs
+// every piece from its true start state.
+constexpr int32_t kProbe = 1 << 30;         // probe offset; split programs' time bound < kProbe
+
+struct alignas(16) PieceInfo {
+  int64_t hdelta[kModes];   // probe runs: history entry = semhb + hdelta + probe * probe_hist_len[mode]
+  int32_t prog, split;      // program id, its index among the split programs
+  int32_t loop, g0, g1;     // iterations [g0, g1) of L (global loop id and iteration indices)
+  int32_t pub_off[kModes];  // published increments at the start, per waited semaphore (pool pub)
+  int32_t nbase_off;        // engines' instances before the piece (pool pub)
+  int32_t pad_;
+};
+
+struct alignas(16) SplitProg {
+  int64_t cnt_base;         // instances of instruction x before piece j: cnt[cnt_base + j*nx + x]
+                            // (j = n_pieces: all of them)
+  int32_t prog, first_piece, n_pieces, nx;
+  int32_t vdep0, vdep1;     // its waited dependencies in vdep
+  int32_t ne, loop;         // engines, L (global id)
+};
+
+// A waited dependency of a split program, for the validation.
+struct alignas(16) VDep {
+  int64_t seg;              // its segment in the threshold layout
+  int32_t cons;             // consumer (program-local instruction)
+  int32_t sem[kModes];      // waited semaphore (program-local), per mode
+  int32_t pad_[2];
+};
+
+// What the piece kernels (and the ordinary sweep, to skip the programs they
+// simulated) read.
+struct PieceArgs {
+  const PieceInfo* piece;   // [n_pieces]
+  const SplitProg* split;   // [n_split]
+  const int32_t* prog_split;  // [n_programs]: index among the split programs, -1 if none (NULL: none)
+  const int32_t* pub;       // published increments / engine instance counts at piece starts
+  int32_t* fail;            // [n_split]: 0 = simulated by pieces in this call
+  int32_t* out;             // [n_pieces * probes * 64]: end states of the probe runs
+  int32_t* x;               // [n_pieces * 64]: true start states (cursors, then last retires)
+  int32_t* phist;           // probe runs' private semaphore history
+  int64_t phist_len;        // entries per probe
+  int32_t n_pieces, probes; // this launch: items = n_pieces * probes
+  int32_t final_pass;       // 0: probe / relative pass, 1: from the true start states
+};
+
 struct SimArgs {
   const ProgInfo* prog;
   const int32_t* order;      // program ids in descending-work order
@@ -263,6 +319,7 @@ struct SweepArgs {
   unsigned long long* chk_counts;  // optional: [2] unsafe / over-synchronised wait values
   unsigned long long* chk_first;   // optional: [1] smallest offending pair index
   CostTables cost;
+  PieceArgs pcs;             // piece-parallel simulation (prog_split NULL: none)
 };
 
 // Launchers (return the launch error, if any).
@@ -296,6 +353,12 @@ cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStr
 // the per-engine kernel (launch_simulate with SimArgs::only set).
 cudaError_t launch_sweep(const SweepArgs& a, bool barrier, int num_sms, cudaStream_t s);
 size_t sweep_smem_bytes(int sem_cap, int frame_depth, int ring);
+// Piece-parallel simulation of the split programs (a.pcs): validation, the
+// probe (barrier-free) or relative (barrier) pass, the composition of the
+// pieces, and the final pass; the programs it completes are marked in
+// a.pcs.fail (0) for launch_sweep to skip.  thr: the threshold array.
+cudaError_t launch_pieces(const SweepArgs& a, bool barrier, const VDep* vdep, const int32_t* cnt, int n_split,
+                          int num_sms, cudaStream_t s);
 // Largest ring (32, 16, ..., 1) whose sweep shared memory fits in `limit`
 // bytes, or 0 if none does.
 int sweep_ring_for(int sem_cap, int frame_depth, size_t limit);

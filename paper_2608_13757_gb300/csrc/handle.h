@@ -91,6 +91,22 @@ struct sync_programs {
   int4* lsem = nullptr;             // [kModes][n_lanes]
   int64_t n_lanes = 0;
   int64_t hist_len[syncgb::kModes] = {0, 0, 0};  // history entries needed per threshold mode
+  // piece-parallel simulation of large programs (PieceArgs in enc.h)
+  int32_t n_split = 0, n_pieces = 0, probes_bf = 0;
+  bool any_bf = false;                  // some split program is also split barrier-free
+  syncgb::PieceInfo* pieces = nullptr;
+  syncgb::SplitProg* splits = nullptr;
+  int32_t* prog_split = nullptr;        // per program: its index among the split programs, or -1
+  int32_t* piece_pub = nullptr;         // published increments / engine instance counts at piece starts
+  int32_t* piece_cnt = nullptr;         // instances of each instruction before each piece
+  syncgb::VDep* vdep = nullptr;
+  int32_t* piece_fail = nullptr;        // scratch [n_split]
+  int32_t* piece_bf_init = nullptr;     // [n_split]: 1 = simulated whole barrier-free (too few programs gain)
+  int32_t* piece_out = nullptr;         // scratch: probe end states
+  int32_t* piece_x = nullptr;           // scratch: start states
+  int64_t phist_len[syncgb::kModes] = {0, 0, 0};   // probe history entries per probe, per mode
+  mutable std::mutex phist_mu;
+  mutable int32_t* phist[syncgb::kModes] = {nullptr, nullptr, nullptr};   // allocated on first use
   int32_t nsem_max[syncgb::kModes] = {0, 0, 0};
   int32_t ne_max = 1;
   int32_t depth_max = 0;
