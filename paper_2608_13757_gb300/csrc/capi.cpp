@@ -201,8 +201,8 @@ std::string where(int32_t p, const char* what, int64_t i) {
 // it splits only programs above 4 * (2*ne + 1) times that share.
 static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop, const HostVec<int32_t>& rowptr,
                          const HostVec<int4>& xsem, const HostVec<DepInfo>& dep, const HostVec<int64_t>& seg,
-                         const HostVec<int64_t>& semhb, const HostVec<ProgInfo>& prog, int64_t n_inst,
-                         cudaStream_t stream, sync_programs& h) {
+                         const HostVec<int64_t>& semhb, const HostVec<ProgInfo>& prog, const HostVec<int64_t>& inst_off,
+                         int64_t n_inst, cudaStream_t stream, sync_programs& h) {
   const int32_t P = d.n_programs;
   const int64_t NX = d.prog_instr_ptr[P];
   const double share = (double)n_inst / ((double)h.num_sms * 24.0);
@@ -214,6 +214,7 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
   std::vector<VDep> vdep;
   std::vector<int32_t> pub, cnt, bf_init;
   int64_t hist_split[kModes] = {0, 0, 0};
+  int64_t inst_bb = 0, inst_bf = 0;               // compact instance spaces (barrier scheme, barrier-free)
   int32_t ne_max = 0;
   std::vector<int32_t> path, row;
   for (int32_t p = 0; p < P; ++p) {
@@ -258,7 +259,7 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
     }
     SplitProg S{};
     S.prog = p; S.first_piece = (int32_t)pieces.size(); S.n_pieces = np; S.nx = nx;
-    S.ne = pi.ne; S.loop = l0 + L;
+    S.ne = pi.ne; S.loop = l0 + L; S.x0 = x0;
     S.cnt_base = (int64_t)cnt.size();
     for (int32_t j = 0; j <= np; ++j)
       for (int32_t x = 0; x < nx; ++x) cnt.push_back(count(x, bnd[j]));
@@ -305,6 +306,14 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
     const bool bf = (double)pi.n_inst > 4.0 * (2.0 * pi.ne + 1.0) * share;
     bf_init.push_back(bf ? 0 : 1);
     if (bf) ne_max = std::max(ne_max, pi.ne);
+    // the program's instances in the compact scratch of the stored times
+    const int64_t first = nx > 0 ? inst_off[x0] : 0;
+    for (int32_t j = 0; j < np; ++j) {
+      pieces[S.first_piece + j].tl[0] = inst_bb - first;
+      pieces[S.first_piece + j].tl[1] = bf ? inst_bf - first : 0;
+    }
+    inst_bb += pi.n_inst;
+    if (bf) inst_bf += pi.n_inst;
     split_of[p] = (int32_t)splits.size();
     splits.push_back(S);
   }
@@ -316,6 +325,13 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
   h.probes_bf = std::max(1, 2 * ne_max);
   h.any_bf = ne_max > 0;
   for (int m = 0; m < kModes; ++m) h.phist_len[m] = hist_split[m];
+  for (const SplitProg& S : splits) h.nx_max_split = std::max(h.nx_max_split, S.nx);
+  h.pinst[0] = inst_bb;
+  h.pinst[1] = inst_bf;
+  {
+    std::vector<int32_t> xe(d.instr_engine, d.instr_engine + NX);
+    h.xeng = h.upload(xe, stream, "instruction engines");
+  }
   h.pieces = h.upload(pieces, stream, "pieces");
   h.splits = h.upload(splits, stream, "split programs");
   h.prog_split = h.upload(split_of, stream, "program split index");
@@ -1292,7 +1308,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.n_lanes = (int64_t)lrec.size();
   LoopInfo* d_xloops = h.upload(xloops, stream, "iteration spaces");
   h.divergent = div;
-  build_pieces(d, loop, rowptr_host, xsem, dep, h.seg_host, semhb, prog, n_inst, stream, h);
+  build_pieces(d, loop, rowptr_host, xsem, dep, h.seg_host, semhb, prog, inst_off, n_inst, stream, h);
   cuda_check(launch_expand(d_xloops, d_tile_loop, h.rowptr, h.pidx, n_iters, h.num_sms, stream), "expand");
   cuda_check(launch_sem_records(d_xsem, NX, h.ops, h.n_ops, h.lrec, h.n_lanes, h.opsem, h.lsem, h.num_sms, stream),
              "semaphore records");
@@ -1426,6 +1442,19 @@ static int32_t* probe_history(const sync_programs* h, sync_thr_mode mode) {
   return h->phist[mode];
 }
 
+// The stored times of the piece runs: per instance of the split programs
+// (barrier-free: of the ones split barrier-free) issue and retire per run
+// and the position in its engine's stream; allocated on first use.
+static int32_t* stored_times(const sync_programs* h, bool barrier) {
+  std::lock_guard<std::mutex> lock(h->phist_mu);
+  const int k = barrier ? 0 : 1;
+  if (!h->ptimes[k]) {
+    const int64_t runs = barrier ? 1 : h->probes_bf;
+    h->ptimes[k] = h->alloc_lazy<int32_t>((2 * runs + 1) * std::max<int64_t>(h->pinst[k], 1), "piece times");
+  }
+  return h->ptimes[k];
+}
+
 // Both simulation entry points: thresholds from d_thr, or (fused) from the
 // simulators' loop state, optionally checked.
 static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, const int32_t* d_thr,
@@ -1512,7 +1541,12 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
     w.pcs.pub = h->piece_pub; w.pcs.fail = h->piece_fail; w.pcs.out = h->piece_out; w.pcs.x = h->piece_x;
     w.pcs.n_pieces = h->n_pieces;
     w.pcs.probes = barrier ? 1 : h->probes_bf;
-    cuda_check(launch_pieces(w, barrier, h->vdep, h->piece_cnt, h->n_split, h->num_sms, st), "piece simulation");
+    w.pcs.xeng = h->xeng;
+    w.pcs.nx_max = h->nx_max_split;
+    w.pcs.plen = h->pinst[barrier ? 0 : 1];
+    SweepArgs wp = w;
+    wp.pcs.ptimes = stored_times(h, barrier);      // the piece runs store their times
+    cuda_check(launch_pieces(wp, barrier, h->vdep, h->piece_cnt, h->n_split, h->num_sms, st), "piece simulation");
   }
   cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");
   a.only = h->fallback;

@@ -189,16 +189,18 @@ struct CostTables {
 // instance counts and each waited semaphore's published increments at its
 // start.  Per call: a validation that every wait of a piece targets an
 // increment the piece itself produces (else the program is simulated whole),
-// then barrier scheme: one pass per piece from a barrier release at 0 and a
+// then barrier scheme: one run per piece from a barrier release at 0 and a
 // prefix sum of the piece durations; barrier-free: the piece's end state
 // (engine cursors and last retires) is a max-plus linear map of its start
 // state, read off by one probe run per state variable (the variable raised
-// by kProbe, the others 0), composed piece by piece.  A final pass runs
-// every piece from its true start state.
+// by kProbe, the others 0), composed piece by piece.  The runs store every
+// instance's times, from which a last pass forms the true ones.
 constexpr int32_t kProbe = 1 << 30;         // probe offset; split programs' time bound < kProbe
 
 struct alignas(16) PieceInfo {
   int64_t hdelta[kModes];   // probe runs: history entry = semhb + hdelta + probe * probe_hist_len[mode]
+  int64_t tl[2];            // compact scratch index of instance o = o + tl[0] (barrier scheme: every
+                            // split program) or o + tl[1] (barrier-free: the ones split barrier-free)
   int32_t prog, split;      // program id, its index among the split programs
   int32_t loop, g0, g1;     // iterations [g0, g1) of L (global loop id and iteration indices)
   int32_t pub_off[kModes];  // published increments at the start, per waited semaphore (pool pub)
@@ -212,6 +214,7 @@ struct alignas(16) SplitProg {
   int32_t prog, first_piece, n_pieces, nx;
   int32_t vdep0, vdep1;     // its waited dependencies in vdep
   int32_t ne, loop;         // engines, L (global id)
+  int32_t x0, pad_[3];      // its first instruction (global id)
 };
 
 // A waited dependency of a split program, for the validation.
@@ -234,8 +237,12 @@ struct PieceArgs {
   int32_t* x;               // [n_pieces * 64]: true start states (cursors, then last retires)
   int32_t* phist;           // probe runs' private semaphore history
   int64_t phist_len;        // entries per probe
+  int32_t* ptimes;          // stored times of the piece runs (tl_write in sweep.cuh)
+  int64_t plen;             // instances of the compact scratch
+  const int32_t* xeng;      // engine of every instruction (global id)
   int32_t n_pieces, probes; // this launch: items = n_pieces * probes
-  int32_t final_pass;       // 0: probe / relative pass, 1: from the true start states
+  int32_t nx_max;           // most instructions of a split program
+  int32_t pad_;
 };
 
 struct SimArgs {
@@ -354,9 +361,10 @@ cudaError_t launch_simulate(const SimArgs& a, bool barrier, int num_sms, cudaStr
 cudaError_t launch_sweep(const SweepArgs& a, bool barrier, int num_sms, cudaStream_t s);
 size_t sweep_smem_bytes(int sem_cap, int frame_depth, int ring);
 // Piece-parallel simulation of the split programs (a.pcs): validation, the
-// probe (barrier-free) or relative (barrier) pass, the composition of the
-// pieces, and the final pass; the programs it completes are marked in
-// a.pcs.fail (0) for launch_sweep to skip.  thr: the threshold array.
+// probe (barrier-free) or relative (barrier) runs, the composition of the
+// pieces, and the pass that forms the instances' true times (checksums,
+// timelines); the programs it completes are marked in a.pcs.fail (0) for
+// launch_sweep to skip.
 cudaError_t launch_pieces(const SweepArgs& a, bool barrier, const VDep* vdep, const int32_t* cnt, int n_split,
                           int num_sms, cudaStream_t s);
 // Largest ring (32, 16, ..., 1) whose sweep shared memory fits in `limit`

@@ -107,6 +107,10 @@ struct sync_programs {
   int64_t phist_len[syncgb::kModes] = {0, 0, 0};   // probe history entries per probe, per mode
   mutable std::mutex phist_mu;
   mutable int32_t* phist[syncgb::kModes] = {nullptr, nullptr, nullptr};   // allocated on first use
+  int64_t pinst[2] = {0, 0};            // instances of the split programs (barrier scheme, barrier-free)
+  mutable int32_t* ptimes[2] = {nullptr, nullptr};   // their stored times, allocated on first use
+  int32_t* xeng = nullptr;              // engine per instruction (split batches)
+  int32_t nx_max_split = 1;             // most instructions of a split program
   int32_t nsem_max[syncgb::kModes] = {0, 0, 0};
   int32_t ne_max = 1;
   int32_t depth_max = 0;

@@ -19,9 +19,15 @@
 //     and the others at 0; since no path weight reaches kProbe (the time
 //     bound of a split program is below it), output o of probe q is
 //     kProbe + M[o][q] when o depends on q and below kProbe otherwise.
-// The pieces of a program are then composed in order (x_{j+1} = M_j x_j), and
-// the final pass runs every piece from its true start state x_j, writing the
-// timelines, the history and the checksum.
+// The pieces of a program are then composed in order (x_{j+1} = M_j x_j).  The
+// same linearity holds for every instance's issue and retire times, which
+// the piece runs store (per probe, with the instance's position in its
+// engine's stream): a memory-bound pass then forms the true times from the
+// start states -- shifted by the piece's start (barrier scheme), or the
+// maximum over the probes of stored time - kProbe + start value (barrier-
+// free) -- for the checksum and the timelines.
+#include <algorithm>
+
 #include "sweep.cuh"
 
 namespace syncgb {
@@ -62,7 +68,7 @@ __global__ void __launch_bounds__(kValThreads) k_piece_validate(const SweepArgs 
 }
 
 // One warp per split program: the pieces' start states in order, the
-// program's makespan and status; the checksum is zeroed for the final pass
+// program's makespan and status; the checksum is zeroed for the fix-up pass
 // to accumulate.  State variable v < ne is engine v's cursor, ne + v its
 // last retire (stored at x[64 * piece + v] and x[64 * piece + 32 + v]).
 template <bool BB>
@@ -130,6 +136,65 @@ __global__ void k_piece_resolve(const SweepArgs a, int n_split) {
   }
 }
 
+// Blocks (piece, y): instructions y, y + gridDim.y, ... of the piece's
+// program; every instance of the piece gets its true issue and retire times
+// from the stored ones (see the top of this file) and adds its checksum
+// term; the timelines, if requested, are written here.
+template <bool BB>
+__global__ void __launch_bounds__(kValThreads) k_piece_fixup(const SweepArgs a, const int32_t* __restrict__ cnt) {
+  __shared__ int32_t xs[64];
+  __shared__ unsigned long long part[kValThreads / 32];
+  const int piece = blockIdx.x;
+  const PieceInfo pc = a.pcs.piece[piece];
+  if (*(volatile int32_t*)(a.pcs.fail + pc.split)) return;
+  const SplitProg sp = a.pcs.split[pc.split];
+  const int j = piece - sp.first_piece, ne = sp.ne, nv = BB ? 1 : 2 * ne;
+  if (threadIdx.x < 64) xs[threadIdx.x] = a.pcs.x[(int64_t)piece * 64 + threadIdx.x];
+  __syncthreads();
+  const int32_t* __restrict__ pt = a.pcs.ptimes;
+  const int64_t N = a.pcs.plen, tl = pc.tl[BB ? 0 : 1];
+  const int64_t ordv = 2 * (int64_t)a.pcs.probes * N;
+  unsigned long long chk = 0;
+  for (int x = blockIdx.y; x < sp.nx; x += gridDim.y) {
+    const int32_t lo = __ldg(cnt + sp.cnt_base + (int64_t)j * sp.nx + x);
+    const int32_t hi = __ldg(cnt + sp.cnt_base + (int64_t)(j + 1) * sp.nx + x);
+    if (lo >= hi) continue;
+    const int64_t o0 = __ldg(a.inst_off + sp.x0 + x);
+    const uint32_t e = (uint32_t)__ldg(a.pcs.xeng + sp.x0 + x);
+    for (int32_t g = lo + (int32_t)threadIdx.x; g < hi; g += kValThreads) {
+      const int64_t o = o0 + g, i = o + tl;
+      int32_t issue, retire;
+      if (BB) {
+        issue = __ldg(pt + i) + xs[0];
+        retire = __ldg(pt + N + i) + xs[0];
+      } else {
+        int64_t bi = -1, br = -1;
+        for (int q = 0; q < nv; ++q) {
+          const int32_t xq = xs[q < ne ? q : 32 + q - ne];
+          const int32_t ti = __ldg(pt + 2 * q * N + i), tr = __ldg(pt + (2 * q + 1) * N + i);
+          if (ti >= kProbe) bi = max(bi, (int64_t)(ti - kProbe) + xq);
+          if (tr >= kProbe) br = max(br, (int64_t)(tr - kProbe) + xq);
+        }
+        issue = (int32_t)bi;
+        retire = (int32_t)br;
+      }
+      chk += inst_term(issue, retire, e, (uint32_t)__ldg(pt + ordv + i));
+      if (a.issue) {
+        a.issue[o] = issue;
+        a.retire[o] = retire;
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) chk += __shfl_xor_sync(0xffffffffu, chk, o);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = chk;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long t = 0;
+    for (int w = 0; w < kValThreads / 32; ++w) t += part[w];
+    atomicAdd(a.checksum + sp.prog, t);
+  }
+}
+
 template <class K>
 cudaError_t launch_items(K kern, const SweepArgs& a, int64_t items, size_t smem, int num_sms, cudaStream_t s) {
   if (items <= 0) return cudaSuccess;
@@ -155,20 +220,16 @@ cudaError_t pieces(const SweepArgs& a, const VDep* vdep, const int32_t* cnt, int
   k_piece_validate<MODE, BB><<<a.pcs.n_pieces, kValThreads, 0, s>>>(a, vdep, cnt);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  // probe / relative pass: no timelines
-  SweepArgs p1 = a;
-  p1.pcs.final_pass = 0;
-  p1.issue = p1.retire = nullptr;
-  e = launch_items(k_sweep<MODE, BB, false, false, true>, p1, (int64_t)a.pcs.n_pieces * a.pcs.probes, smem,
+  // the probe / relative runs, storing every instance's times
+  e = launch_items(k_sweep<MODE, BB, true, false, true>, a, (int64_t)a.pcs.n_pieces * a.pcs.probes, smem,
                    num_sms, s);
   if (e != cudaSuccess) return e;
   k_piece_resolve<BB><<<(n_split * 32 + 255) / 256, 256, 0, s>>>(a, n_split);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  SweepArgs p2 = a;
-  p2.pcs.final_pass = 1;
-  p2.pcs.probes = 1;
-  return a.issue ? launch_items(k_sweep<MODE, BB, true, false, true>, p2, a.pcs.n_pieces, smem, num_sms, s)
-                 : launch_items(k_sweep<MODE, BB, false, false, true>, p2, a.pcs.n_pieces, smem, num_sms, s);
+  // (piece, instruction slice) blocks: about 2048 or more in all
+  const int ys = std::max(1, std::min(a.pcs.nx_max, (2048 + a.pcs.n_pieces - 1) / a.pcs.n_pieces));
+  k_piece_fixup<BB><<<dim3(a.pcs.n_pieces, ys), kValThreads, 0, s>>>(a, cnt);
+  return cudaGetLastError();
 }
 
 }  // namespace

@@ -51,7 +51,7 @@ struct Frame { int32_t loop, item, g, g_end; };
 // Shared memory of one warp (program), 16-byte aligned.
 __host__ __device__ __forceinline__ size_t warp_bytes(int sem_cap, int frame_depth, int ring) {
   const size_t per = (size_t)(20 + 4 * ring + 32) * sem_cap + sizeof(Frame) * (size_t)frame_depth +
-                     8 * (size_t)(frame_depth + 1) + 3 * 8 + 8 + 3 * 4 * 32;
+                     8 * (size_t)(frame_depth + 1) + 3 * 8 + 8 + 3 * 4 * 32 + 16 + 8;
   return (per + 15) & ~(size_t)15;
 }
 
@@ -91,7 +91,26 @@ struct WarpSmem {
   Frame* frames;       // [depth]
   int2* lvl;           // [depth + 1] per level of the walk: {current iteration, start of its trip}
   unsigned long long* tally;  // [3] fused check: unsafe, over-synchronised, first offending pair
+  int64_t* tlx;        // [2] piece runs: compact instance offset, probe (see tl_write)
 };
+
+// The timeline entry of instance o (instance layout).  Piece runs (stored
+// times, PieceArgs.ptimes set) write the compact scratch instead: probe q's
+// issue and retire at ptimes[2q * N + i] and ptimes[(2q + 1) * N + i], and
+// (probe 0) the instance's position in its engine's stream at
+// ptimes[2 * probes * N + i], i = o + the piece's compact offset.
+__device__ __forceinline__ void tl_write(const SweepArgs& a, const WarpSmem& S, int64_t o, int32_t issue,
+                                         int32_t retire, uint32_t nj) {
+  if (a.pcs.ptimes) {
+    const int64_t N = a.pcs.plen, i = o + S.tlx[0], q = S.tlx[1];
+    a.pcs.ptimes[2 * q * N + i] = issue;
+    a.pcs.ptimes[(2 * q + 1) * N + i] = retire;
+    if (q == 0) a.pcs.ptimes[2 * (int64_t)a.pcs.probes * N + i] = (int32_t)nj;
+  } else {
+    a.issue[o] = issue;
+    a.retire[o] = retire;
+  }
+}
 
 // Fused simulation: the wait value of consumer-grouped dependency r for the
 // consumer instance at global iteration gl of the loop at walk level lc
@@ -377,11 +396,7 @@ __device__ __forceinline__ int run_chunk(const SweepArgs& a, const WarpSmem& S, 
   }
   if (valid) {
     chk += inst_term(issue, retire, (uint32_t)e, nj);
-    if (TL) {
-      const int64_t o = __ldg(a.inst_off + rec.x) + gl;
-      a.issue[o] = issue;
-      a.retire[o] = retire;
-    }
+    if (TL) tl_write(a, S, __ldg(a.inst_off + rec.x) + gl, issue, retire, nj);
   }
   __syncwarp();
   if (prod) {
@@ -659,10 +674,7 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     }
     if (valid) {
       chk += inst_term(issue, retire, (uint32_t)e, nj);
-      if (TL) {
-        a.issue[tl_off + gl] = issue;
-        a.retire[tl_off + gl] = retire;
-      }
+      if (TL) tl_write(a, S, tl_off + gl, issue, retire, nj);
     }
     pub0 += __popc(wg0 & vm);
     pub1 += __popc(wg1 & vm);
@@ -735,11 +747,7 @@ __device__ __forceinline__ int run_single(const SweepArgs& a, const WarpSmem& S,
       S.semv[sr.x] += 1;
     }
     chk += inst_term(issue, retire, (uint32_t)e, nj);
-    if (TL) {
-      const int64_t o = __ldg(a.inst_off + rec.x) + g;
-      a.issue[o] = issue;
-      a.retire[o] = retire;
-    }
+    if (TL) tl_write(a, S, __ldg(a.inst_off + rec.x) + g, issue, retire, nj);
     S.t[e] = t_after;
     S.lr[e] = retire;
     S.nn[e] = (int32_t)nj;
@@ -821,11 +829,12 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     S.tag = reinterpret_cast<int32_t*>(p); p += 4 * a.sem_cap;
     S.ring = reinterpret_cast<int32_t*>(p); p += 4 * (size_t)a.ring * a.sem_cap;
     S.rank_lane = reinterpret_cast<uint8_t*>(p); p += 32 * (size_t)a.sem_cap;
+    p = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 7) & ~uintptr_t(7));
     if (!BB) {
-      p = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 7) & ~uintptr_t(7));
       S.tally = reinterpret_cast<unsigned long long*>(p); p += 3 * 8;
-      S.lvl = reinterpret_cast<int2*>(p);
+      S.lvl = reinterpret_cast<int2*>(p); p += 8 * (a.frame_depth + 1);
     }
+    S.tlx = reinterpret_cast<int64_t*>(p);
     S.rmask = a.ring - 1;
   }
   const int32_t cwait = MODE == SYNC_THR_COUNT ? a.prm.c_wait_ops_count : a.prm.c_wait_ops_perloop;
@@ -860,8 +869,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     const ProgInfo pi = a.prog[p];
     if (PIECE) {
       // a failed validation, or a probe past this program's state variables
-      if (*(volatile int32_t*)(a.pcs.fail + pc.split) || probe >= (BB || a.pcs.final_pass ? 1 : 2 * pi.ne))
-        continue;
+      if (*(volatile int32_t*)(a.pcs.fail + pc.split) || probe >= (BB ? 1 : 2 * pi.ne)) continue;
     }
     // the iteration-start cost of global loop `loop` on lane `lane`'s engine
     // (lanes past the engines: any value); flag: its trip register is elidable
@@ -887,7 +895,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       continue;
     }
     // probe runs write a private history (each probe its own)
-    const bool probe_hist = PIECE && !BB && !a.pcs.final_pass;
+    const bool probe_hist = PIECE && !BB;
     for (int i = lane; i < pi.nsem[MODE]; i += 32) {
       S.semv[i] = PIECE ? __ldg(a.pcs.pub + pc.pub_off[MODE] + i) : 0;
       S.semhb[i] = __ldg(a.semhb + pi.semhb_off[MODE] + i);
@@ -896,17 +904,12 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     }
     if (PIECE) {
       // the start state: probe `probe` raises state variable `probe` (cursors
-      // 0..ne-1, then last retires) by kProbe; the final pass starts from
-      // the composed state; the barrier scheme's relative pass from 0
-      int32_t t0 = 0, l0 = 0;
-      if (a.pcs.final_pass) {
-        if (lane < pi.ne) { t0 = a.pcs.x[piece * 64 + lane]; l0 = a.pcs.x[piece * 64 + 32 + lane]; }
-      } else if (!BB) {
-        t0 = lane == probe ? kProbe : 0;
-        l0 = lane + pi.ne == probe ? kProbe : 0;
-      }
+      // 0..ne-1, then last retires) by kProbe; the barrier scheme runs from
+      // a release at 0.  The instances' times go to the compact scratch.
+      const int32_t t0 = !BB && lane == probe ? kProbe : 0, l0 = !BB && lane + pi.ne == probe ? kProbe : 0;
       S.t[lane] = t0; S.lr[lane] = l0;
       S.nn[lane] = lane < pi.ne ? __ldg(a.pcs.pub + pc.nbase_off + lane) : 0;
+      if (lane == 0) { S.tlx[0] = pc.tl[BB ? 0 : 1]; S.tlx[1] = probe; }
     } else {
       S.t[lane] = 0; S.lr[lane] = 0; S.nn[lane] = 0;
     }
@@ -1029,10 +1032,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       // any verdict but OK (a deadlock, a wait reaching forward): the
       // program is simulated whole by the sweep, which reports it
       if (verdict != SYNC_PROG_OK && lane == 0) atomicExch(a.pcs.fail + pc.split, 1);
-      if (a.pcs.final_pass) {
-        for (int o = 16; o > 0; o >>= 1) chk += __shfl_xor_sync(kFull, chk, o);
-        if (lane == 0) atomicAdd(a.checksum + p, chk);
-      } else if (lane < pi.ne) {
+      if (lane < pi.ne) {
         int32_t* o = a.pcs.out + ((int64_t)piece * a.pcs.probes + probe) * 64;
         o[lane] = S.t[lane];
         o[32 + lane] = S.lr[lane];
