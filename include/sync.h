@@ -46,7 +46,8 @@
  *    64-bit integers even when 32 bits suffice.
  *  - SYNCGB_SPLIT_MIN=n (read by sync_load_programs): the fewest instances a
  *    program needs to be simulated in pieces on several warps (default
- *    65536; see sync_simulate).
+ *    65536; see sync_simulate); SYNCGB_SPLIT_SPEC=1: such programs are
+ *    always speculated, never probed, barrier-free.
  */
 #ifndef SYNC_H
 #define SYNC_H
@@ -359,7 +360,11 @@ sync_status sync_check_minimal(const sync_programs *h, sync_thr_mode mode, const
  * deadlocks or waits forward, the program is simulated whole): the barrier
  * scheme from the barrier before each piece, the barrier-free scheme by
  * composing the pieces' max-plus maps of the engines' cursors and last
- * retires.  The results are identical either way.
+ * retires (read off by one probe run per cursor and last retire), or, for
+ * a batch of many such programs, by speculation: a piece runs from a guessed
+ * start and is accepted when its true start differs from the guess by one
+ * constant in every cursor and last retire (a few rounds of guesses at
+ * most).  The results are identical either way.
  * UNROLLED: as barrier-free with c_branch, c_regop and every wait-op cost
  * taken as 0 (ii and latencies unchanged); it requires PERENGINE and a batch
  * without barrier-fallback dependencies, and returns SYNC_ERR_ARG otherwise.

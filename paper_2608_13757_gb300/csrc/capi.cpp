@@ -197,8 +197,9 @@ std::string where(int32_t p, const char* what, int64_t i) {
 // more than 8 times the instances per resident sweep warp (152 SMs x 24
 // warps on a GB300) of the whole batch, so that its serial walk, not the
 // batch's throughput, bounds the simulation (the barrier scheme runs each
-// piece twice).  The barrier-free scheme runs 2*ne + 1 passes per piece, so
-// it splits only programs above 4 * (2*ne + 1) times that share.
+// piece twice).  Barrier-free, a program is probed (2*ne runs per piece)
+// when it stays above 4 * (2*ne + 1) times that share, and speculated
+// otherwise (SYNCGB_SPLIT_SPEC=1 speculates always).
 static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop, const HostVec<int32_t>& rowptr,
                          const HostVec<int4>& xsem, const HostVec<DepInfo>& dep, const HostVec<int64_t>& seg,
                          const HostVec<int64_t>& semhb, const HostVec<ProgInfo>& prog, const HostVec<int64_t>& inst_off,
@@ -208,6 +209,8 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
   const double share = (double)n_inst / ((double)h.num_sms * 24.0);
   int64_t min_inst = 65536;                       // SYNCGB_SPLIT_MIN=n lowers it (tests)
   if (const char* e = std::getenv("SYNCGB_SPLIT_MIN")) min_inst = std::max<int64_t>(1, std::atoll(e));
+  const char* spec_env = std::getenv("SYNCGB_SPLIT_SPEC");   // 1: speculate, never probe (tests)
+  const bool force_spec = spec_env && spec_env[0] == '1';
   std::vector<int32_t> split_of(P, -1);
   std::vector<SplitProg> splits;
   std::vector<PieceInfo> pieces;
@@ -303,7 +306,9 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
       for (int32_t j = 0; j < np; ++j) pieces[S.first_piece + j].hdelta[m] = hist_split[m] - first;
       hist_split[m] += span[m];
     }
-    const bool bf = (double)pi.n_inst > 4.0 * (2.0 * pi.ne + 1.0) * share;
+    // barrier-free: probed when the 2*ne runs per piece still leave the
+    // program far above the batch's share per warp, speculated otherwise
+    const bool bf = !force_spec && (double)pi.n_inst > 4.0 * (2.0 * pi.ne + 1.0) * share;
     bf_init.push_back(bf ? 0 : 1);
     if (bf) ne_max = std::max(ne_max, pi.ne);
     // the program's instances in the compact scratch of the stored times
@@ -320,10 +325,10 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
   if (splits.empty()) return;
   h.n_split = (int32_t)splits.size();
   h.n_pieces = (int32_t)pieces.size();
+  for (int32_t c : bf_init) (c ? h.n_spec : h.n_probed) += 1;
   h.sz.n_split_programs = h.n_split;
   h.sz.n_pieces = h.n_pieces;
   h.probes_bf = std::max(1, 2 * ne_max);
-  h.any_bf = ne_max > 0;
   for (int m = 0; m < kModes; ++m) h.phist_len[m] = hist_split[m];
   for (const SplitProg& S : splits) h.nx_max_split = std::max(h.nx_max_split, S.nx);
   h.pinst[0] = inst_bb;
@@ -338,7 +343,12 @@ static void build_pieces(const sync_batch_desc& d, const HostVec<LoopInfo>& loop
   h.piece_pub = h.upload(pub, stream, "piece start counts");
   h.piece_cnt = h.upload(cnt, stream, "piece instance counts");
   h.vdep = h.upload(vdep, stream, "split programs' dependencies");
-  h.piece_bf_init = h.upload(bf_init, stream, "barrier-free split flags");
+  h.piece_cls = h.upload(bf_init, stream, "barrier-free split classes");
+  h.spec_need = h.alloc<int32_t>(h.n_pieces, "speculation: runs due");
+  h.spec_has = h.alloc<int32_t>(h.n_pieces, "speculation: runs done");
+  h.spec_xhat = h.alloc<int32_t>((int64_t)h.n_pieces * 64, "speculation: guessed starts");
+  h.piece_shift = h.alloc<int32_t>(h.n_pieces, "piece shifts");
+  h.spec_vp = h.alloc<int32_t>(h.n_split, "speculation: accepted pieces");
   h.piece_fail = h.alloc<int32_t>(h.n_split, "piece validation flags");
   h.piece_out = h.alloc<int32_t>((int64_t)h.n_pieces * h.probes_bf * 64, "piece probe states");
   h.piece_x = h.alloc<int32_t>((int64_t)h.n_pieces * 64, "piece start states");
@@ -1527,26 +1537,32 @@ static void simulate(const sync_programs* h, sync_thr_mode mode, bool fused, con
   const bool barrier = variant == SYNC_SIM_BARRIER;
   // split programs (array thresholds): simulated piece by piece on many warps
   // first; the sweep skips the ones the pieces completed
-  if (!fused && h->n_split > 0 && (barrier || h->any_bf)) {
-    const size_t flags = sizeof(int32_t) * (size_t)h->n_split;
-    if (barrier) {
-      cuda_check(cudaMemsetAsync(h->piece_fail, 0, flags, st), "cudaMemsetAsync");
-    } else {
-      w.pcs.phist = probe_history(h, mode);
-      w.pcs.phist_len = h->phist_len[mode];
-      cuda_check(cudaMemcpyAsync(h->piece_fail, h->piece_bf_init, flags, cudaMemcpyDeviceToDevice, st),
-                 "cudaMemcpyAsync");
-    }
+  if (!fused && h->n_split > 0) {
+    cuda_check(cudaMemsetAsync(h->piece_fail, 0, sizeof(int32_t) * (size_t)h->n_split, st), "cudaMemsetAsync");
     w.pcs.piece = h->pieces; w.pcs.split = h->splits; w.pcs.prog_split = h->prog_split;
     w.pcs.pub = h->piece_pub; w.pcs.fail = h->piece_fail; w.pcs.out = h->piece_out; w.pcs.x = h->piece_x;
     w.pcs.n_pieces = h->n_pieces;
-    w.pcs.probes = barrier ? 1 : h->probes_bf;
+    w.pcs.out_probes = h->probes_bf;
     w.pcs.xeng = h->xeng;
     w.pcs.nx_max = h->nx_max_split;
-    w.pcs.plen = h->pinst[barrier ? 0 : 1];
+    w.pcs.cls = h->piece_cls; w.pcs.need = h->spec_need; w.pcs.has = h->spec_has; w.pcs.xhat = h->spec_xhat;
+    w.pcs.shift = h->piece_shift; w.pcs.vp = h->spec_vp;
     SweepArgs wp = w;
-    wp.pcs.ptimes = stored_times(h, barrier);      // the piece runs store their times
-    cuda_check(launch_pieces(wp, barrier, h->vdep, h->piece_cnt, h->n_split, h->num_sms, st), "piece simulation");
+    PieceLaunch L{h->vdep, h->piece_cnt, stored_times(h, true), h->pinst[0], h->n_split, 0, 0};
+    if (barrier) {
+      wp.pcs.probes = 1;
+    } else {
+      L.n_probed = h->n_probed;
+      L.n_spec = h->n_spec;
+      wp.pcs.probes = h->probes_bf;
+      if (h->n_probed > 0) {                       // the probes' histories and stored times
+        wp.pcs.phist = probe_history(h, mode);
+        wp.pcs.phist_len = h->phist_len[mode];
+        wp.pcs.ptimes = stored_times(h, false);
+        wp.pcs.plen = h->pinst[1];
+      }
+    }
+    cuda_check(launch_pieces(wp, barrier, L, h->num_sms, st), "piece simulation");
   }
   cuda_check(launch_sweep(w, barrier, h->num_sms, st), "sweep simulator kernel");
   a.only = h->fallback;

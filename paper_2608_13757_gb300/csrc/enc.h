@@ -233,7 +233,8 @@ struct PieceArgs {
   const int32_t* prog_split;  // [n_programs]: index among the split programs, -1 if none (NULL: none)
   const int32_t* pub;       // published increments / engine instance counts at piece starts
   int32_t* fail;            // [n_split]: 0 = simulated by pieces in this call
-  int32_t* out;             // [n_pieces * probes * 64]: end states of the probe runs
+  int32_t* out;             // [n_pieces * out_probes * 64]: end states of the runs (run q of a piece
+                            // at 64 * (out_probes * piece + q))
   int32_t* x;               // [n_pieces * 64]: true start states (cursors, then last retires)
   int32_t* phist;           // probe runs' private semaphore history
   int64_t phist_len;        // entries per probe
@@ -242,7 +243,19 @@ struct PieceArgs {
   const int32_t* xeng;      // engine of every instruction (global id)
   int32_t n_pieces, probes; // this launch: items = n_pieces * probes
   int32_t nx_max;           // most instructions of a split program
-  int32_t pad_;
+  int32_t out_probes;       // end states per piece in out (its stride: 64 * out_probes per piece)
+  // barrier-free speculation (split programs with cls 1, too many to probe):
+  // a piece runs from a guessed start state xhat; it is accepted when its
+  // true start equals xhat plus one shift for every state variable (the
+  // times are then the stored ones plus that shift); a rejected piece runs
+  // again from its true start, the later ones from guesses of the last round
+  int32_t spec;             // 1: this launch runs the speculative pieces
+  const int32_t* cls;       // [n_split]: 0 = probed, 1 = speculated (barrier-free)
+  int32_t* need;            // [n_pieces]: run in the next round
+  int32_t* has;             // [n_pieces]: has run at least once
+  int32_t* xhat;            // [n_pieces * 64]: start state of its last run
+  int32_t* shift;           // [n_pieces]: accepted pieces: true times - stored times
+  int32_t* vp;              // [n_split]: pieces accepted so far
 };
 
 struct SimArgs {
@@ -365,8 +378,14 @@ size_t sweep_smem_bytes(int sem_cap, int frame_depth, int ring);
 // pieces, and the pass that forms the instances' true times (checksums,
 // timelines); the programs it completes are marked in a.pcs.fail (0) for
 // launch_sweep to skip.
-cudaError_t launch_pieces(const SweepArgs& a, bool barrier, const VDep* vdep, const int32_t* cnt, int n_split,
-                          int num_sms, cudaStream_t s);
+struct PieceLaunch {
+  const VDep* vdep;
+  const int32_t* cnt;
+  int32_t* one;              // stored times of single runs (barrier scheme, speculation)
+  int64_t one_len;           // instances of all split programs
+  int32_t n_split, n_probed, n_spec;   // split programs; of these barrier-free probed / speculated
+};
+cudaError_t launch_pieces(const SweepArgs& a, bool barrier, const PieceLaunch& L, int num_sms, cudaStream_t s);
 // Largest ring (32, 16, ..., 1) whose sweep shared memory fits in `limit`
 // bytes, or 0 if none does.
 int sweep_ring_for(int sem_cap, int frame_depth, size_t limit);

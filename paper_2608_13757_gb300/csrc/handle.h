@@ -93,7 +93,6 @@ struct sync_programs {
   int64_t hist_len[syncgb::kModes] = {0, 0, 0};  // history entries needed per threshold mode
   // piece-parallel simulation of large programs (PieceArgs in enc.h)
   int32_t n_split = 0, n_pieces = 0, probes_bf = 0;
-  bool any_bf = false;                  // some split program is also split barrier-free
   syncgb::PieceInfo* pieces = nullptr;
   syncgb::SplitProg* splits = nullptr;
   int32_t* prog_split = nullptr;        // per program: its index among the split programs, or -1
@@ -101,7 +100,13 @@ struct sync_programs {
   int32_t* piece_cnt = nullptr;         // instances of each instruction before each piece
   syncgb::VDep* vdep = nullptr;
   int32_t* piece_fail = nullptr;        // scratch [n_split]
-  int32_t* piece_bf_init = nullptr;     // [n_split]: 1 = simulated whole barrier-free (too few programs gain)
+  int32_t* piece_cls = nullptr;         // [n_split]: barrier-free, 0 = probed, 1 = speculated
+  int32_t n_probed = 0, n_spec = 0;     // split programs of each class
+  int32_t* spec_need = nullptr;         // speculation scratch (PieceArgs)
+  int32_t* spec_has = nullptr;
+  int32_t* spec_xhat = nullptr;
+  int32_t* spec_vp = nullptr;
+  int32_t* piece_shift = nullptr;
   int32_t* piece_out = nullptr;         // scratch: probe end states
   int32_t* piece_x = nullptr;           // scratch: start states
   int64_t phist_len[syncgb::kModes] = {0, 0, 0};   // probe history entries per probe, per mode

@@ -868,8 +868,12 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
     }
     const ProgInfo pi = a.prog[p];
     if (PIECE) {
-      // a failed validation, or a probe past this program's state variables
-      if (*(volatile int32_t*)(a.pcs.fail + pc.split) || probe >= (BB ? 1 : 2 * pi.ne)) continue;
+      // a failed validation, a probe past this program's state variables, a
+      // program of the other barrier-free class, a speculative piece with no
+      // run due
+      if (*(volatile int32_t*)(a.pcs.fail + pc.split) || probe >= (BB || a.pcs.spec ? 1 : 2 * pi.ne)) continue;
+      if (!BB && (__ldg(a.pcs.cls + pc.split) != 0) != (a.pcs.spec != 0)) continue;
+      if (a.pcs.spec && !*(volatile int32_t*)(a.pcs.need + piece)) continue;
     }
     // the iteration-start cost of global loop `loop` on lane `lane`'s engine
     // (lanes past the engines: any value); flag: its trip register is elidable
@@ -894,8 +898,9 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       if (lane == 0) { a.makespan[p] = -1; a.checksum[p] = 0; a.status[p] = SYNC_PROG_OVERFLOW; }
       continue;
     }
-    // probe runs write a private history (each probe its own)
-    const bool probe_hist = PIECE && !BB;
+    // probe runs write a private history (each probe its own); the barrier
+    // scheme's and the speculated pieces' single runs write the real one
+    const bool probe_hist = PIECE && !BB && !a.pcs.spec;
     for (int i = lane; i < pi.nsem[MODE]; i += 32) {
       S.semv[i] = PIECE ? __ldg(a.pcs.pub + pc.pub_off[MODE] + i) : 0;
       S.semhb[i] = __ldg(a.semhb + pi.semhb_off[MODE] + i);
@@ -906,10 +911,14 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       // the start state: probe `probe` raises state variable `probe` (cursors
       // 0..ne-1, then last retires) by kProbe; the barrier scheme runs from
       // a release at 0.  The instances' times go to the compact scratch.
-      const int32_t t0 = !BB && lane == probe ? kProbe : 0, l0 = !BB && lane + pi.ne == probe ? kProbe : 0;
+      int32_t t0 = !BB && lane == probe ? kProbe : 0, l0 = !BB && lane + pi.ne == probe ? kProbe : 0;
+      if (a.pcs.spec && lane < pi.ne) {              // a speculative piece: its guessed start
+        t0 = a.pcs.xhat[(int64_t)piece * 64 + lane];
+        l0 = a.pcs.xhat[(int64_t)piece * 64 + 32 + lane];
+      }
       S.t[lane] = t0; S.lr[lane] = l0;
       S.nn[lane] = lane < pi.ne ? __ldg(a.pcs.pub + pc.nbase_off + lane) : 0;
-      if (lane == 0) { S.tlx[0] = pc.tl[BB ? 0 : 1]; S.tlx[1] = probe; }
+      if (lane == 0) { S.tlx[0] = pc.tl[BB || a.pcs.spec ? 0 : 1]; S.tlx[1] = probe; }
     } else {
       S.t[lane] = 0; S.lr[lane] = 0; S.nn[lane] = 0;
     }
@@ -1033,10 +1042,11 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
       // program is simulated whole by the sweep, which reports it
       if (verdict != SYNC_PROG_OK && lane == 0) atomicExch(a.pcs.fail + pc.split, 1);
       if (lane < pi.ne) {
-        int32_t* o = a.pcs.out + ((int64_t)piece * a.pcs.probes + probe) * 64;
+        int32_t* o = a.pcs.out + ((int64_t)piece * a.pcs.out_probes + probe) * 64;
         o[lane] = S.t[lane];
         o[32 + lane] = S.lr[lane];
       }
+      if (a.pcs.spec && lane == 0) { a.pcs.need[piece] = 0; a.pcs.has[piece] = 1; }
       __syncwarp();
       continue;
     }

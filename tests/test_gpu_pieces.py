@@ -64,9 +64,12 @@ def wrap_in_loop(batch, reps, seed):
     return workloads.concat(parts)
 
 
+@pytest.mark.parametrize("spec", ["0", "1"], ids=["probes", "speculation"])
 @pytest.mark.parametrize("seed", range(3))
-def test_pieces_random_trees(sg, seed, monkeypatch):
+def test_pieces_random_trees(sg, seed, spec, monkeypatch):
+    """Barrier-free pieces probed, or speculated (SYNCGB_SPLIT_SPEC=1)."""
     monkeypatch.setenv("SYNCGB_SPLIT_MIN", "1")
+    monkeypatch.setenv("SYNCGB_SPLIT_SPEC", spec)
     base = workloads.random_trees(9500 + seed, 60, workloads.tree_params(
         engines_hi=5, loops_hi=5, body_hi=6, trip_hi=4, max_depth=3, max_deps_per_cons=2))
     batch = wrap_in_loop(base, 3 + seed, seed)
@@ -77,17 +80,22 @@ def test_pieces_random_trees(sg, seed, monkeypatch):
                 params=oracle.sim_params(ii=2, c_branch=3, c_regop=2, c_barrier=9))
 
 
+@pytest.mark.parametrize("spec", ["0", "1"], ids=["probes", "speculation"])
 @pytest.mark.parametrize("red", [dict(licm=1, cse=1), dict(trip_register_elision=1)])
-def test_pieces_with_cost_switches(sg, red, monkeypatch):
+def test_pieces_with_cost_switches(sg, red, spec, monkeypatch):
     monkeypatch.setenv("SYNCGB_SPLIT_MIN", "1")
+    monkeypatch.setenv("SYNCGB_SPLIT_SPEC", spec)
     batch = wrap_in_loop(workloads.random_trees(9600, 60, workloads.tree_params(
         engines_hi=4, loops_hi=5, body_hi=6, trip_hi=4, max_depth=3)), 4, 7)
     compare_all(sg, batch, timeline=True, modes=ALL_MODES, params=oracle.sim_params(c_regop=2, **red))
 
 
-def test_pieces_configs(sg):
+@pytest.mark.parametrize("spec", ["0", "1"], ids=["probes", "speculation"])
+def test_pieces_configs(sg, spec, monkeypatch):
     """The GEMM program and two attention programs split at the default
-    floor; their pieces' results equal the oracle's."""
+    floor (their 32 outer iterations are identical in shape, so speculation
+    accepts most guesses); their results equal the oracle's."""
+    monkeypatch.setenv("SYNCGB_SPLIT_SPEC", spec)
     for name, n in (("gemm", None), ("attention", 2)):
         batch = workloads.generate(name, n_programs=n)
         h = sg.sync_load_programs(batch)
