@@ -29,9 +29,9 @@ template <int MODE, class A>
 __device__ __forceinline__ int32_t wait_ops(const A& a, const int4 rec, int32_t levels) {
   const sync_sim_params& q = a.prm;
   const int32_t cw = MODE == SYNC_THR_COUNT ? q.c_wait_ops_count : q.c_wait_ops_perloop;
-  if (rec.z == 0) return 0;
   if (!(q.licm | q.cse))
     return rec.z * cw + (MODE == SYNC_THR_PERENGINE ? q.c_wait_ops_perengine_level * levels : 0);
+  if (rec.z == 0) return 0;
   const int4 c = q.cse ? __ldg(a.cost.xcse + rec.x)
                        : make_int4(rec.z, 0, MODE == SYNC_THR_PERENGINE ? __ldg(a.cost.xlvr + rec.x) : 0, levels);
   int32_t w = c.x * cw - c.y * min(q.c_regop, cw);
