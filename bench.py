@@ -135,8 +135,8 @@ class ClockSampler:
 KERNEL_SOURCES = {
     "thresholds": ("k_thresholds.cu", "waitval.cuh", "enc.h"),
     "check": ("k_thresholds.cu", "waitval.cuh", "enc.h"),
-    "sim_barrier_free": ("k_sweep.cu", "k_simulate.cu", "cost.cuh", "waitval.cuh", "enc.h"),
-    "sim_barrier": ("k_sweep.cu", "k_simulate.cu", "cost.cuh", "waitval.cuh", "enc.h"),
+    "sim_barrier_free": ("k_sweep.cu", "sweep.cuh", "k_simulate.cu", "cost.cuh", "waitval.cuh", "enc.h"),
+    "sim_barrier": ("k_sweep.cu", "sweep.cuh", "k_simulate.cu", "cost.cuh", "waitval.cuh", "enc.h"),
 }
 
 
@@ -237,10 +237,12 @@ def run_gpu(args, rank, world, local_rank):
     # keep the GPU busy (about 5 ms) while the host queues the timed steps, so
     # host-side launch latency never shows up as GPU time between the events
     torch.cuda._sleep(10_000_000)
+    launches0 = sg.kernel_launches()
     start.record(stream)
     for k in range(args.steps):
         step(evs[k])
     end.record(stream)
+    launches = sg.kernel_launches() - launches0
     torch.cuda.synchronize()
     clk = clocks.stop()
     dist_barrier(world)
@@ -252,7 +254,7 @@ def run_gpu(args, rank, world, local_rank):
     per_kernel = {k: v / args.steps for k, v in per_kernel.items()}
     if fused:                             # no threshold kernel or checker launched
         per_kernel["thresholds"] = per_kernel["check"] = 0.0
-    out = dict(ms=total_ms / args.steps, per_kernel=per_kernel, sizes=sz, clocks=clk, ok=ok,
+    out = dict(ms=total_ms / args.steps, per_kernel=per_kernel, sizes=sz, clocks=clk, ok=ok, launches=launches,
                load_s=load_s, P=P, first=first,
                num_sms=torch.cuda.get_device_properties(dev).multi_processor_count)
     if not args.no_e2e:
@@ -606,9 +608,11 @@ def main():
                                   "bytes_per_instruction": 16}},
         "roofline": roof,
         "kernels": kernels,
-        # per step: thresholds, check, and per schedule the sweep plus the
-        # per-engine kernel for programs it hands over
-        "gpu_launches": (4 if args.pipeline == "fused" else 6) * args.steps,
+        # the library's own count of the kernels it launched in the timed
+        # region: per step thresholds, check, and per schedule the sweep, the
+        # per-engine kernel for programs it hands over and, where programs are
+        # cut into pieces, the piece kernels
+        "gpu_launches": res["launches"],
         "results_minimal_and_deadlock_free": res["ok"],
         "load_s": res["load_s"],
         "clocks": clk or None,

@@ -445,6 +445,14 @@ void sync_free_programs(sync_programs *h);
 /* Message for the last non-OK status returned on this thread ("" if none). */
 const char *sync_last_error(void);
 
+/* Number of kernels this library has launched in this process, over every
+ * handle, stream and thread: the loader's kernels, and per call of the
+ * entry points above the kernels it enqueued (sync_simulate: one sweep and
+ * one per-engine launch per call, plus the piece-parallel kernels when
+ * programs are cut into pieces).  A launch counts once the CUDA runtime has
+ * accepted it.  Monotonic; reading it has no other effect and cannot fail. */
+int64_t sync_kernel_launches(void);
+
 #ifdef __cplusplus
 }
 #endif

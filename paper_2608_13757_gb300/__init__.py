@@ -30,7 +30,7 @@ PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD, PROG_TIMEOUT = 0, 4, 7,
 # every symbol include/sync.h declares
 EXPORTS = ("sync_load_programs", "sync_query", "sync_pair_offsets", "sync_eval_thresholds",
            "sync_check_minimal", "sync_simulate", "sync_simulate_fused", "sync_simulate_noalloc",
-           "sync_free_programs", "sync_last_error")
+           "sync_free_programs", "sync_last_error", "sync_kernel_launches")
 NOALLOC_SCRATCH_BYTES = 64 << 20
 CODE_BYTES_PER_INSTR = 16
 
@@ -98,8 +98,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sync_free_programs.restype = None
     lib.sync_last_error.argtypes = []
     lib.sync_last_error.restype = ctypes.c_char_p
+    lib.sync_kernel_launches.argtypes = []
+    lib.sync_kernel_launches.restype = ctypes.c_int64
     for f in EXPORTS:
-        if f not in ("sync_free_programs", "sync_last_error"):
+        if f not in ("sync_free_programs", "sync_last_error", "sync_kernel_launches"):
             getattr(lib, f).restype = ctypes.c_int
     return lib
 
@@ -113,6 +115,11 @@ def lib() -> ctypes.CDLL:
     if _lib is None:
         _lib = load_library()
     return _lib
+
+
+def kernel_launches() -> int:
+    """Kernels the library has launched in this process so far."""
+    return int(lib().sync_kernel_launches())
 
 
 def _check(status: int):

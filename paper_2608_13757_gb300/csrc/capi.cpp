@@ -3,6 +3,7 @@
 // in include/sync.h.
 #include <algorithm>
 #include <array>
+#include <atomic>
 #include <cstdlib>
 #include <cstring>
 #include <exception>
@@ -53,6 +54,9 @@ sync_status set_error(sync_status status, const std::string& msg) {
   return status;
 }
 void cuda_or_raise(cudaError_t e, const char* what) { cuda_check(e, what); }
+
+std::atomic<int64_t> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 // Timing constants a variant runs with: the unrolled variant has no loop
 // control and static waits, so it costs neither.
@@ -1599,5 +1603,7 @@ sync_status sync_simulate_fused(const sync_programs* h, sync_thr_mode mode, cons
 void sync_free_programs(sync_programs* h) { delete h; }
 
 const char* sync_last_error(void) { return g_err.c_str(); }
+
+int64_t sync_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"

@@ -391,4 +391,13 @@ cudaError_t launch_pieces(const SweepArgs& a, bool barrier, const PieceLaunch& L
 int sweep_ring_for(int sem_cap, int frame_depth, size_t limit);
 size_t simulate_smem_bytes(int warps, int sem_cap, int frame_depth);
 
+// Kernels this library has launched in this process (every handle and
+// stream), counted by launched() after each launch the runtime accepted.
+void count_launch();
+inline cudaError_t launched() {
+  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) count_launch();
+  return e;
+}
+
 }  // namespace syncgb

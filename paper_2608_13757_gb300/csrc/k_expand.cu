@@ -144,7 +144,7 @@ cudaError_t launch_ordinals(const ProgInfo* prog, const int32_t* order, int32_t 
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
   k_ordinals<<<grid, kThreads, 0, s>>>(prog, order, n_programs, ne_max, op_ptr, ops, rowptr, ord_off, ord);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
@@ -155,7 +155,7 @@ cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const 
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
   k_derive<<<grid, kThreads, 0, s>>>(jobs, tile_job, rowptr, pidx, path, derived, n);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_sem_records(const int4* xsem, int64_t n_instrs, const int4* ops, int64_t n_ops,
@@ -167,7 +167,7 @@ cudaError_t launch_sem_records(const int4* xsem, int64_t n_instrs, const int4* o
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
   k_sem_records<<<grid, kThreads, 0, s>>>(xsem, n_instrs, ops, n_ops, lrec, n_lanes, opsem, lsem);
-  return cudaGetLastError();
+  return launched();
 }
 
 cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const int32_t* rowptr,
@@ -177,7 +177,7 @@ cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const 
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
   k_expand<<<grid, kThreads, 0, s>>>(loop, tile_loop, rowptr, pidx, n_iters);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace syncgb

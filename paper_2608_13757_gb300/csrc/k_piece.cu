@@ -330,7 +330,7 @@ cudaError_t launch_items(K kern, const SweepArgs& a, int64_t items, size_t smem,
   e = cudaMemsetAsync(a.next_slot, 0, sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
   kern<<<grid, kWarps * 32, smem, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 template <int MODE, bool BB>
@@ -338,7 +338,7 @@ cudaError_t pieces(const SweepArgs& a, const PieceLaunch& L, int num_sms, cudaSt
   const size_t smem = sweep_smem_bytes(a.sem_cap, a.frame_depth, a.ring);
   const int warp_blocks = (L.n_split * 32 + 255) / 256;
   k_piece_validate<MODE, BB><<<a.pcs.n_pieces, kValThreads, 0, s>>>(a, L.vdep, L.cnt);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launched();
   if (e != cudaSuccess) return e;
   // barrier scheme, or barrier-free probes: one launch of runs storing
   // every instance's times, then the composition
@@ -350,7 +350,7 @@ cudaError_t pieces(const SweepArgs& a, const PieceLaunch& L, int num_sms, cudaSt
                      num_sms, s);
     if (e != cudaSuccess) return e;
     k_piece_resolve<BB><<<warp_blocks, 256, 0, s>>>(p, L.n_split);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launched()) != cudaSuccess) return e;
   }
   // barrier-free speculation: rounds of runs and acceptance checks
   if (!BB && L.n_spec > 0) {
@@ -360,18 +360,18 @@ cudaError_t pieces(const SweepArgs& a, const PieceLaunch& L, int num_sms, cudaSt
     p.pcs.ptimes = L.one;
     p.pcs.plen = L.one_len;
     k_spec_init<<<warp_blocks, 256, 0, s>>>(p, L.n_split);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launched()) != cudaSuccess) return e;
     for (int r = 0; r < kSpecRounds; ++r) {
       e = launch_items(k_sweep<MODE, BB, true, false, true>, p, p.pcs.n_pieces, smem, num_sms, s);
       if (e != cudaSuccess) return e;
       k_spec_resolve<<<warp_blocks, 256, 0, s>>>(p, L.n_split, r == kSpecRounds - 1);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      if ((e = launched()) != cudaSuccess) return e;
     }
   }
   // (piece, instruction slice) blocks: about 2048 or more in all
   const int ys = std::max(1, std::min(a.pcs.nx_max, (2048 + a.pcs.n_pieces - 1) / a.pcs.n_pieces));
   k_piece_fixup<BB><<<dim3(a.pcs.n_pieces, ys), kValThreads, 0, s>>>(a, L.cnt, L.one, L.one_len);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace

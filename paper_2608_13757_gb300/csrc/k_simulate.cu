@@ -501,7 +501,7 @@ cudaError_t launch3(const SimArgs& a, size_t smem, int num_sms, cudaStream_t s) 
     e = cudaMemsetAsync(a.next_slot, 0, sizeof(int32_t), s);
     if (e != cudaSuccess) return e;
     kern<<<grid, threads, smem, s>>>(a);
-    return cudaGetLastError();
+    return launched();
   };
   if (a.dep) return a.issue ? run(k_simulate<MODE, BB, true, true>) : run(k_simulate<MODE, BB, false, true>);
   return a.issue ? run(k_simulate<MODE, BB, true, false>) : run(k_simulate<MODE, BB, false, false>);

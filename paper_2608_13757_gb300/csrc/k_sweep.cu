@@ -21,7 +21,7 @@ cudaError_t launch3(const SweepArgs& a, size_t smem, int num_sms, cudaStream_t s
     if (e == cudaSuccess) e = cudaMemsetAsync(a.fallback, 0, sizeof(int32_t), s);
     if (e != cudaSuccess) return e;
     kern<<<grid, kWarps * 32, smem, s>>>(a);
-    return cudaGetLastError();
+    return launched();
   };
   if (a.dep) return a.issue ? run(k_sweep<MODE, BB, true, true>) : run(k_sweep<MODE, BB, false, true>);
   return a.issue ? run(k_sweep<MODE, BB, true, false>) : run(k_sweep<MODE, BB, false, false>);

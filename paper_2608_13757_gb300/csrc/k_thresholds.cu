@@ -202,7 +202,7 @@ cudaError_t launch_thr_mode(const ThrArgs& a, int32_t* thr, int num_sms, cudaStr
   if (e != cudaSuccess) return e;
   if (wide_index(a.n_chunks, grid)) k_thresholds<MODE, int64_t><<<grid, kThreads, 0, s>>>(a, thr);
   else k_thresholds<MODE, int32_t><<<grid, kThreads, 0, s>>>(a, thr);
-  return cudaGetLastError();
+  return launched();
 }
 
 template <int MODE>
@@ -212,7 +212,7 @@ cudaError_t launch_check_mode(const CheckArgs& a, int num_sms, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   if (wide_index(a.t.n_chunks, grid)) k_check<MODE, int64_t><<<grid, kThreads, 0, s>>>(a);
   else k_check<MODE, int32_t><<<grid, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  return launched();
 }
 
 }  // namespace

@@ -40,6 +40,16 @@ def test_no_gpu_dependency_at_import(sg):
     assert sg.lib().sync_last_error() is not None
 
 
+def test_launch_counter_reads_without_a_gpu(sg):
+    """The launch counter is readable with no device and counts only
+    launches the runtime accepted: without a device, none."""
+    import torch
+    n = sg.kernel_launches()
+    assert isinstance(n, int) and n >= 0 and sg.kernel_launches() == n
+    if not torch.cuda.is_available():
+        assert n == 0
+
+
 def _status(sg, batch):
     desc, keep = sg.batch_desc(batch)
     h = ctypes.c_void_p()

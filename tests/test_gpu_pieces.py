@@ -126,3 +126,37 @@ def test_pieces_refuse_waits_into_earlier_pieces(sg, monkeypatch):
             assert np.array_equal(r.makespan.cpu().numpy()[:1], ref.makespan)
             assert np.array_equal(r.checksum.cpu().numpy()[:1].view(np.uint64), ref.checksum)
     h.close()
+
+
+@pytest.mark.parametrize("spec", ["0", "1"], ids=["probes", "speculation"])
+def test_kernel_launch_count(sg, spec, monkeypatch):
+    """The library's launch counter: one kernel per threshold and check
+    call, two per simulation of unsplit programs (the sweep and the
+    per-engine kernel), and the piece kernels on top where programs are
+    split: barrier scheme validation, runs, composition and fixup;
+    barrier-free validation, then probes (runs, composition) and/or
+    speculation (start, four rounds of runs and acceptance), then fixup."""
+    monkeypatch.setenv("SYNCGB_SPLIT_SPEC", spec)
+    mode = oracle.PERLOOP
+    for name, split in (("depth2", False), ("gemm", True)):
+        batch = workloads.generate(name, n_programs=64 if name == "depth2" else None)
+        h = sg.sync_load_programs(batch)
+        assert (h.sizes.n_split_programs > 0) == split
+        n0 = sg.kernel_launches()
+        thr = sg.sync_eval_thresholds(h, mode)
+        assert sg.kernel_launches() - n0 == 1
+        sg.sync_check_minimal(h, mode, thr)
+        assert sg.kernel_launches() - n0 == 2
+        n0 = sg.kernel_launches()
+        sg.sync_simulate(h, mode, thr, variant=oracle.BARRIER)
+        assert sg.kernel_launches() - n0 == (2 + 4 if split else 2)
+        n0 = sg.kernel_launches()
+        sg.sync_simulate(h, mode, thr, variant=oracle.BARRIER_FREE)
+        bf = sg.kernel_launches() - n0
+        if not split:
+            assert bf == 2
+        elif spec == "1":
+            assert bf == 2 + 1 + 1 + 4 * 2 + 1
+        else:
+            assert bf in (2 + 1 + 2 + 1, 2 + 1 + 2 + 9 + 1, 2 + 1 + 9 + 1)
+        h.close()
