@@ -314,7 +314,9 @@ def e2e_pipelined(args, sg, batch, mode, prm, dev, steps, bufs):
     host (pipeline fill and drain included).  Handles are released after
     the last step."""
     import torch
-    load_stream = torch.cuda.Stream(device=dev)
+    # the loads' stream at the highest priority: at each kernel boundary of
+    # the step being simulated, the next load's kernels are dispatched first
+    load_stream = torch.cuda.Stream(device=dev, priority=torch.cuda.Stream.priority_range()[1])
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     handles, keeps = [], []

@@ -271,17 +271,38 @@ typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
  * fallbacks in a batch with per-engine trips, SYNC_ERR_OVERFLOW when a loop's iteration total, a per-loop
  * threshold N*total, a pair count or an instance count exceeds INT32_MAX
  * (int64 totals are supported for pairs and instances across programs).
- * On SYNC_OK, *out receives a handle to free with sync_free_programs.  The
- * call synchronizes `stream` before returning. */
+ * On SYNC_OK, *out receives a handle to free with sync_free_programs.
+ * The call waits on `stream` for its validation pass (to report failures);
+ * the rest of the load is left queued on `stream`, its completion recorded
+ * in an event of the handle: every later call on the handle, on any stream,
+ * makes that stream wait for the event first, and sync_free_programs waits
+ * for the device.  The caller's arrays may be released when the call returns.
+ * The host checks the batch's shape (the CSR offsets, trip offsets, NULL
+ * arrays); everything per program runs on the GPU: the raw arrays are copied
+ * to the device, one pass per program validates it and counts its table
+ * entries, a second writes the encoding at the programs' offsets (the same
+ * routine as sync_validate_programs, so both report the same first failure:
+ * the lowest-numbered failing program's first failure in check order).
+ * Device memory for the passes is taken with cudaMallocAsync on `stream` and
+ * released on it before the call returns. */
 sync_status sync_load_programs(const sync_batch_desc *desc, int device, void *stream,
                                sync_programs **out);
+
+/* The validation of sync_load_programs on the host alone (no device, no
+ * CUDA call): the same shape checks and per-program checks, run on host
+ * threads; returns the status and sets the message sync_load_programs would
+ * for the same batch, or SYNC_OK when the batch would load (device memory
+ * aside).  SYNCGB_LOAD_THREADS=n sets the number of host threads. */
+sync_status sync_validate_programs(const sync_batch_desc *desc);
 
 /* Sizes of a loaded batch (host struct). */
 sync_status sync_query(const sync_programs *h, sync_sizes *out);
 
 /* Host copies of the pair layout: offsets [n_deps + 1] int64 (segment starts;
  * entry n_deps is n_pairs_padded) and, unless NULL, counts [n_deps] int32
- * (consumer instances of each dependency, i.e. unpadded segment lengths). */
+ * (consumer instances of each dependency, i.e. unpadded segment lengths).
+ * The first call on a handle reads them back from the device (synchronous
+ * copies on the handle's device); later calls copy the kept host copy. */
 sync_status sync_pair_offsets(const sync_programs *h, int64_t *offsets, int32_t *counts);
 
 /* Threshold kernel: for every pair (dependency d, consumer instance g) the

@@ -30,7 +30,7 @@ PROG_OK, PROG_OVERFLOW, PROG_DEADLOCK, PROG_ROUND_GUARD, PROG_TIMEOUT = 0, 4, 7,
 # every symbol include/sync.h declares
 EXPORTS = ("sync_load_programs", "sync_query", "sync_pair_offsets", "sync_eval_thresholds",
            "sync_check_minimal", "sync_simulate", "sync_simulate_fused", "sync_simulate_noalloc",
-           "sync_free_programs", "sync_last_error", "sync_kernel_launches")
+           "sync_free_programs", "sync_last_error", "sync_kernel_launches", "sync_validate_programs")
 NOALLOC_SCRATCH_BYTES = 64 << 20
 CODE_BYTES_PER_INSTR = 16
 
@@ -85,6 +85,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     P = ctypes.POINTER
     vp = ctypes.c_void_p
     lib.sync_load_programs.argtypes = [P(BatchDesc), ctypes.c_int, vp, P(vp)]
+    lib.sync_validate_programs.argtypes = [P(BatchDesc)]
     lib.sync_query.argtypes = [vp, P(Sizes)]
     lib.sync_pair_offsets.argtypes = [vp, P(ctypes.c_int64), P(ctypes.c_int32)]
     lib.sync_eval_thresholds.argtypes = [vp, ctypes.c_int, vp, vp]
@@ -173,12 +174,27 @@ class Programs:
         s = Sizes()
         _check(lib().sync_query(self._h, ctypes.byref(s)))
         self.sizes = s
-        off = np.zeros(s.n_deps + 1, dtype=np.int64)
-        cnt = np.zeros(max(s.n_deps, 1), dtype=np.int32)
-        _check(lib().sync_pair_offsets(self._h, off.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
-                                      cnt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))))
-        self.pair_offsets = off
-        self.pair_counts = cnt[:s.n_deps]
+        self._pairs = None
+
+    def _pair_layout(self):
+        """(segment offsets [n_deps + 1], pairs per dependency [n_deps]),
+        read back on first use."""
+        if self._pairs is None:
+            n = self.sizes.n_deps
+            off = np.zeros(n + 1, dtype=np.int64)
+            cnt = np.zeros(max(n, 1), dtype=np.int32)
+            _check(lib().sync_pair_offsets(self.handle, off.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                                          cnt.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))))
+            self._pairs = (off, cnt[:n])
+        return self._pairs
+
+    @property
+    def pair_offsets(self) -> np.ndarray:
+        return self._pair_layout()[0]
+
+    @property
+    def pair_counts(self) -> np.ndarray:
+        return self._pair_layout()[1]
 
     def unpadded_index(self) -> np.ndarray:
         """Indices into a threshold array, in pair order without padding."""

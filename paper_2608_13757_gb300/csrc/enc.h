@@ -343,9 +343,10 @@ struct SweepArgs {
 };
 
 // Launchers (return the launch error, if any).
-// tile_loop[t] = loop whose pidx segment holds entry t*kTilePairs (largest l
-// with pidx_off[l] <= t*kTilePairs), with one extra entry n_loops-1.
-cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const int32_t* rowptr,
+// tile_rp[t] = iteration space whose rowptr segment holds entry t*kTilePairs
+// (largest l with rowptr_off[l] <= t*kTilePairs), with one extra entry
+// n_spaces-1; n_rowptr = rowptr entries.
+cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_rp, const int32_t* rowptr, int64_t n_rowptr,
                           int32_t* pidx, int64_t n_iters, int num_sms, cudaStream_t s);
 // Semaphore records of the op rows and sweep lanes, per threshold mode,
 // gathered from the per-instruction table xsem[m * n_instrs + x] by the

@@ -39,8 +39,12 @@ struct sync_programs {
   int device = 0;
   int num_sms = 0;
   sync_sizes sz{};
-  syncgb::HostVec<int64_t> seg_host;
-  syncgb::HostVec<int32_t> count_host;
+  // pair layout for sync_pair_offsets, read back on first use
+  mutable std::mutex pair_mu;
+  mutable bool pairs_ready = false;
+  mutable syncgb::HostVec<int64_t> seg_host;
+  mutable syncgb::HostVec<int32_t> count_host;
+  int32_t* dep_count = nullptr;     // pairs per dependency
   std::vector<void*> blocks;
   // threshold / checker encoding
   syncgb::LoopInfo* loop = nullptr;
@@ -63,7 +67,7 @@ struct sync_programs {
   int64_t n_bar_deps = 0;           // barrier-fallback dependencies (no unrolled variant)
   int64_t n_ord = 0;
   bool ord_overflow = false;        // an engine of a program has > INT32_MAX instances
-  syncgb::HostVec<int64_t> ord_off_host;  // per instruction: pool offset or -1
+  int64_t* ord_off = nullptr;       // per instruction: ordinal pool offset of a waited producer, or -1
   int64_t n_chunks = 0;
   // simulator encoding
   syncgb::ProgInfo* prog = nullptr;
@@ -119,6 +123,11 @@ struct sync_programs {
   int32_t nsem_max[syncgb::kModes] = {0, 0, 0};
   int32_t ne_max = 1;
   int32_t depth_max = 0;
+  // recorded on the load's stream after its last operation; every call on
+  // the handle makes its own stream wait for it
+  cudaEvent_t ready = nullptr;
+
+  cudaError_t wait_ready(cudaStream_t s) const { return ready ? cudaStreamWaitEvent(s, ready, 0) : cudaSuccess; }
 
   ~sync_programs() {
     if (blocks.empty()) return;
@@ -126,6 +135,7 @@ struct sync_programs {
     cudaGetDevice(&prev);
     cudaSetDevice(device);
     cudaDeviceSynchronize();
+    if (ready) cudaEventDestroy(ready);
     for (void* p : blocks) cudaFree(p);
     cudaSetDevice(prev);
   }

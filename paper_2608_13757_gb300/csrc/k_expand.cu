@@ -4,8 +4,7 @@
 //
 // For every loop l and every global iteration g of l, pidx_l[g] is the
 // parent's global iteration j with rowptr_l[j] <= g < rowptr_l[j+1] (the CSR
-// row of g).  One thread per output entry; the loop is found inside the range
-// the host's tile table gives, the row by binary search over rowptr_l.
+// row of g).
 #include "enc.h"
 
 namespace syncgb {
@@ -13,26 +12,44 @@ namespace {
 
 constexpr int kThreads = 256;
 
+// One warp per 32 consecutive rowptr entries (rows: parent iterations of
+// some iteration space, plus each space's closing entry).  The rows' child
+// iterations are consecutive in the parent-index pool, so the warp writes
+// one contiguous range, each lane finding the row of an entry by a binary
+// search over the 32 row starts (shuffles).
 __global__ void __launch_bounds__(kThreads)
-k_expand(const LoopInfo* __restrict__ loop, const int32_t* __restrict__ tile_loop,
-         const int32_t* __restrict__ rowptr, int32_t* __restrict__ pidx, int64_t n_iters) {
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < n_iters; q += stride) {
-    const int64_t t = q / kTilePairs;
-    int lo = tile_loop[t], hi = tile_loop[t + 1];
-    while (lo < hi) {                 // largest l with pidx_off[l] <= q
-      const int mid = (lo + hi + 1) >> 1;
-      if (loop[mid].pidx_off <= q) lo = mid; else hi = mid - 1;
+k_expand(const LoopInfo* __restrict__ loop, const int32_t* __restrict__ tile_rp,
+         const int32_t* __restrict__ rowptr, int64_t n_rowptr, int32_t* __restrict__ pidx, int64_t n_iters) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (kThreads / 32);
+  for (int64_t w = (int64_t)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); w * 32 < n_rowptr; w += warps) {
+    const int64_t r = w * 32 + lane;
+    int64_t b = n_iters, e = n_iters;             // lanes past the last entry: empty, at the end
+    int32_t j = 0;
+    if (r < n_rowptr) {
+      const int64_t t = r / kTilePairs;
+      int lo = tile_rp[t], hi = tile_rp[t + 1];
+      while (lo < hi) {                           // largest space with rowptr_off <= r
+        const int mid = (lo + hi + 1) >> 1;
+        if (loop[mid].rowptr_off <= r) lo = mid; else hi = mid - 1;
+      }
+      const LoopInfo L = loop[lo];
+      j = (int32_t)(r - L.rowptr_off);
+      b = L.pidx_off + rowptr[r];
+      e = j < L.n_parent ? L.pidx_off + rowptr[r + 1] : b;
     }
-    const LoopInfo L = loop[lo];
-    const int32_t g = (int32_t)(q - L.pidx_off);
-    const int32_t* rp = rowptr + L.rowptr_off;
-    int a = 0, b = L.n_parent - 1;    // largest j with rp[j] <= g
-    while (a < b) {
-      const int mid = (a + b + 1) >> 1;
-      if (rp[mid] <= g) a = mid; else b = mid - 1;
+    const int64_t wb = __shfl_sync(0xffffffffu, b, 0), we = __shfl_sync(0xffffffffu, e, 31);
+    for (int64_t base = wb; base < we; base += 32) {
+      const int64_t k = base + lane;
+      int lo = 0, hi = 31;                        // largest row with start <= k
+      for (int step = 0; step < 5; ++step) {
+        const int mid = (lo + hi + 1) >> 1;
+        const int64_t bm = __shfl_sync(0xffffffffu, b, mid);
+        if (bm <= k) lo = mid; else hi = mid - 1;
+      }
+      const int32_t v = __shfl_sync(0xffffffffu, j, lo);
+      if (k < we) pidx[k] = v;
     }
-    pidx[q] = a;
   }
 }
 
@@ -55,32 +72,65 @@ k_sem_records(const int4* __restrict__ xsem, int64_t n_instrs, const int4* __res
   }
 }
 
-// One thread per derived entry; the job is found inside the range the
-// host's tile table gives.
+// One CTA per tile of kTilePairs derived entries: the jobs that overlap the
+// tile (with the path offsets of ancestor jobs) are staged in shared memory,
+// then each thread fills entries of the tile.  Tiles overlapping more jobs
+// than the stage holds look the jobs up in global memory.
+constexpr int kStageJobs = 64;
+
+__device__ __forceinline__ int32_t derive_one(const DeriveJob& J, const int64_t* jpath, int64_t q,
+                                              const int32_t* __restrict__ rowptr,
+                                              const int32_t* __restrict__ pidx) {
+  const int32_t g = (int32_t)(q - J.out);
+  if (g >= J.n) return 0;                         // padding entries
+  if (J.kind == DERIVE_TSTART) return rowptr[J.b + pidx[J.a + g]];
+  int32_t v = g;
+  for (int i = 0; i < J.up; ++i) v = pidx[jpath[i] + v];
+  return v;
+}
+
 __global__ void __launch_bounds__(kThreads)
 k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_job,
          const int32_t* __restrict__ rowptr, const int32_t* __restrict__ pidx,
          const int64_t* __restrict__ path, int32_t* __restrict__ out, int64_t n) {
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < n; q += stride) {
-    const int64_t t = q / kTilePairs;
-    int lo = tile_job[t], hi = tile_job[t + 1];
-    while (lo < hi) {                 // largest job with out <= q
-      const int mid = (lo + hi + 1) >> 1;
-      if (jobs[mid].out <= q) lo = mid; else hi = mid - 1;
+  __shared__ DeriveJob sj[kStageJobs];
+  __shared__ int64_t sp[kStageJobs][SYNC_MAX_DEPTH];
+  const int64_t n_tiles = (n + kTilePairs - 1) / kTilePairs;
+  for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+    const int j0 = tile_job[t], j1 = tile_job[t + 1];
+    const int nj = j1 - j0 + 1;
+    const bool staged = nj <= kStageJobs;
+    __syncthreads();                              // the previous tile's readers are done
+    if (staged) {
+      for (int i = threadIdx.x; i < nj; i += kThreads) sj[i] = jobs[j0 + i];
+      __syncthreads();
+      for (int i = threadIdx.x; i < nj * SYNC_MAX_DEPTH; i += kThreads) {
+        const int jj = i / SYNC_MAX_DEPTH, u = i - jj * SYNC_MAX_DEPTH;
+        if (sj[jj].kind == DERIVE_ANC && u < sj[jj].up) sp[jj][u] = path[sj[jj].a + u];
+      }
+      __syncthreads();
     }
-    const DeriveJob J = jobs[lo];
-    const int32_t g = (int32_t)(q - J.out);
-    int32_t v = 0;                    // padding entries
-    if (g < J.n) {
-      if (J.kind == DERIVE_TSTART) {
-        v = rowptr[J.b + pidx[J.a + g]];
+    const int64_t q0 = t * kTilePairs, q1 = q0 + kTilePairs < n ? q0 + kTilePairs : n;
+    for (int64_t q = q0 + threadIdx.x; q < q1; q += kThreads) {
+      int lo = 0, hi = nj - 1;                    // largest job with out <= q
+      if (staged) {
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (sj[mid].out <= q) lo = mid; else hi = mid - 1;
+        }
+        out[q] = derive_one(sj[lo], sp[lo], q, rowptr, pidx);
       } else {
-        v = g;
-        for (int i = 0; i < J.up; ++i) v = pidx[path[J.a + i] + v];
+        lo = j0, hi = j1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (jobs[mid].out <= q) lo = mid; else hi = mid - 1;
+        }
+        const DeriveJob J = jobs[lo];
+        int64_t jp[SYNC_MAX_DEPTH];
+        for (int u = 0; J.kind == DERIVE_ANC && u < J.up; ++u) jp[u] = path[J.a + u];
+        out[q] = derive_one(J, jp, q, rowptr, pidx);
       }
     }
-    out[q] = v;
   }
 }
 
@@ -151,7 +201,7 @@ cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const 
                           const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,
                           int num_sms, cudaStream_t s) {
   if (n == 0) return cudaSuccess;
-  const int64_t want = (n + kThreads - 1) / kThreads;
+  const int64_t want = (n + kTilePairs - 1) / kTilePairs;
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
   k_derive<<<grid, kThreads, 0, s>>>(jobs, tile_job, rowptr, pidx, path, derived, n);
@@ -170,13 +220,13 @@ cudaError_t launch_sem_records(const int4* xsem, int64_t n_instrs, const int4* o
   return launched();
 }
 
-cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_loop, const int32_t* rowptr,
+cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_rp, const int32_t* rowptr, int64_t n_rowptr,
                           int32_t* pidx, int64_t n_iters, int num_sms, cudaStream_t s) {
   if (n_iters == 0) return cudaSuccess;
-  const int64_t want = (n_iters + kThreads - 1) / kThreads;
+  const int64_t want = (n_rowptr + kThreads - 1) / kThreads;
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
-  k_expand<<<grid, kThreads, 0, s>>>(loop, tile_loop, rowptr, pidx, n_iters);
+  k_expand<<<grid, kThreads, 0, s>>>(loop, tile_rp, rowptr, n_rowptr, pidx, n_iters);
   return launched();
 }
 

@@ -82,6 +82,8 @@ extern "C" sync_status sync_simulate_noalloc(const sync_programs* h, sync_thr_mo
     return set_error(SYNC_ERR_ARG, "a program has too many waited semaphores for the simulator's shared memory");
   sync_status st = cuda_error(cudaSetDevice(h->device), "cudaSetDevice");
   if (st != SYNC_OK) return st;
+  st = cuda_error(h->wait_ready(static_cast<cudaStream_t>(stream)), "load completion");
+  if (st != SYNC_OK) return st;
   int32_t* base = nullptr;
   st = cuda_error(scratch_address(&base), "cudaGetSymbolAddress");
   if (st != SYNC_OK) return st;

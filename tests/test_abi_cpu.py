@@ -51,18 +51,17 @@ def test_launch_counter_reads_without_a_gpu(sg):
 
 
 def _status(sg, batch):
+    """The loader's validation on the host (sync_validate_programs runs the
+    loader's per-program pass on host threads; no device needed)."""
     desc, keep = sg.batch_desc(batch)
-    h = ctypes.c_void_p()
-    st = sg.lib().sync_load_programs(ctypes.byref(desc), 0, None, ctypes.byref(h))
-    if st == sg.OK:
-        sg.lib().sync_free_programs(h)
+    st = sg.lib().sync_validate_programs(ctypes.byref(desc))
     return st, sg.lib().sync_last_error().decode()
 
 
 
 
 def _validated(sg):
-    return {sg.OK, sg.ERR_CUDA}
+    return {sg.OK}
 
 
 def test_valid_batch_passes_validation(sg):

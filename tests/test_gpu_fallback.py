@@ -169,30 +169,15 @@ def test_fallback_rejections(sg):
     assert err.value.status == sg.ERR_ARG
 
 
-def test_fallback_loader_blocks(sg, monkeypatch):
-    """The loader's block join shifts the fallback's zero-filled derived
-    regions and leaves its unused consumer-grouped slots alone: any block
-    count gives the same results."""
-    import torch
+def test_fallback_loader_offsets(sg):
+    """The fallback's zero-filled derived regions and unused consumer-grouped
+    slots sit at offsets summed over the programs before them: each part of a
+    batch, loaded alone, gives exactly its programs' share of the results."""
+    from tests.test_gpu_parity import assert_parts_match
     b = with_policy(workloads.concat([
         workloads.random_trees(31030, 90, workloads.tree_params(**FAR)),
         workloads.generate("depth2", n_programs=12),
         workloads.random_trees(31031, 70, workloads.tree_params(**FAR))]), 1)
-    results = []
-    for n in ("1", "3", "7"):
-        monkeypatch.setenv("SYNCGB_LOAD_THREADS", n)
-        h = sg.sync_load_programs(b)
-        out = []
-        for mode in (COUNT, PERLOOP, PERENGINE):
-            thr = sg.sync_eval_thresholds(h, mode)
-            counts, fb = sg.sync_check_minimal(h, mode, thr)
-            out.append((thr.cpu(), counts.cpu(), fb.cpu()))
-            for v in (sg.SIM_BARRIER_FREE, sg.SIM_BARRIER):
-                r = sg.sync_simulate(h, mode, thr, variant=v, timeline=True)
-                out.append((r.makespan.cpu(), r.checksum.cpu(), r.status.cpu(), r.issue.cpu(), r.retire.cpu()))
-        results.append(out)
-        h.close()
-    for other in results[1:]:
-        for a, c in zip(results[0], other):
-            for x, y in zip(a, c):
-                assert torch.equal(x, y)
+    assert_parts_match(sg, b, [0, 45, 90, 102, 172], (COUNT, PERLOOP, PERENGINE),
+                       (sg.SIM_BARRIER_FREE, sg.SIM_BARRIER))
+

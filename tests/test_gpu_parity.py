@@ -402,31 +402,78 @@ def test_trip_register_elision_divergent(sg):
 
 # ------------------------------------------------------------------ loader
 
-def test_loader_blocks_join_identically(sg, monkeypatch):
-    """The loader's per-program pass runs in blocks of programs on several
-    threads and joins them: any block count gives the same device encoding,
-    so the same thresholds, checks and schedules."""
-    import torch
+def loaded_results(sg, batch, modes, variants=(oracle.BARRIER_FREE,)):
+    """Per mode: unpadded thresholds, check counts, and per variant the
+    per-program makespans, checksums and statuses with the timelines."""
+    h = sg.sync_load_programs(batch)
+    idx = h.unpadded_index()
+    out = []
+    for mode in modes:
+        thr = sg.sync_eval_thresholds(h, mode)
+        counts, _ = sg.sync_check_minimal(h, mode, thr)
+        res = [thr.cpu().numpy()[idx], counts.cpu().numpy()]
+        for v in variants:
+            r = sg.sync_simulate(h, mode, thr, variant=v, timeline=True)
+            P = batch.n_programs
+            res += [r.makespan.cpu().numpy()[:P], r.checksum.cpu().numpy()[:P], r.status.cpu().numpy()[:P],
+                    r.issue.cpu().numpy(), r.retire.cpu().numpy()]
+        out.append(res)
+    h.close()
+    return out
+
+
+def assert_parts_match(sg, batch, cuts, modes, variants=(oracle.BARRIER_FREE,)):
+    """The loader places every program's tables at offsets summed over the
+    programs before it: each part of a batch, loaded alone, gives exactly
+    its programs' share of the whole batch's results (thresholds and
+    timelines concatenate, check counts add up)."""
+    whole = loaded_results(sg, batch, modes, variants)
+    parts = [loaded_results(sg, workloads.concat([batch], [(0, p) for p in range(a, b)]), modes, variants)
+             for a, b in zip(cuts, cuts[1:])]
+    for m in range(len(modes)):
+        for f in range(len(whole[m])):
+            if f == 1:
+                assert np.array_equal(whole[m][f], sum(pt[m][f] for pt in parts))
+            else:
+                assert np.array_equal(whole[m][f], np.concatenate([pt[m][f] for pt in parts])), (modes[m], f)
+
+
+def test_loader_offsets_shift_identically(sg):
+    """Programs of random trees, depth2 and per-engine trips: loaded in one
+    batch or in parts, every program gets the same thresholds, checks and
+    schedules."""
     batch = workloads.concat([workloads.random_trees(8000, 97, workloads.tree_params(
-        engines_hi=5, loops_hi=5, body_hi=6, trip_hi=4, max_depth=4)), workloads.generate("depth2", n_programs=20),
-        workloads.diverge(workloads.random_trees(8001, 40), 5, permille=200)])
-    results = []
-    for n in ("1", "3", "7"):
-        monkeypatch.setenv("SYNCGB_LOAD_THREADS", n)
-        h = sg.sync_load_programs(batch)
-        out = []
-        for mode in MODES:
-            thr = sg.sync_eval_thresholds(h, mode)
-            counts, fb = sg.sync_check_minimal(h, mode, thr)
-            r = sg.sync_simulate(h, mode, thr, timeline=True)
-            out.append((thr.cpu(), counts.cpu(), fb.cpu(), r.makespan.cpu(), r.checksum.cpu(), r.status.cpu(),
-                        r.issue.cpu(), r.retire.cpu()))
-        results.append(out)
-        h.close()
-    for other in results[1:]:
-        for a, b in zip(results[0], other):
-            for x, y in zip(a, b):
-                assert torch.equal(x, y)
+        engines_hi=5, loops_hi=5, body_hi=6, trip_hi=4, max_depth=4)), workloads.generate("depth2", n_programs=20)])
+    assert_parts_match(sg, batch, [0, 1, 40, 97, 117], (COUNT, PERLOOP, PERENGINE), (oracle.BARRIER_FREE, oracle.BARRIER))
+    div = workloads.diverge(workloads.random_trees(8001, 40), 5, permille=200)
+    assert_parts_match(sg, div, [0, 13, 40], (COUNT, PERLOOP))
+
+
+def test_device_loader_reports_what_host_validation_does(sg):
+    """sync_load_programs validates on the device with the same per-program
+    routine that sync_validate_programs runs on the host: on malformed and
+    non-allocatable batches both give the same status and message."""
+    import ctypes
+    from tests import test_abi_cpu as T
+    cases = [T._mut(f) for f in (
+        lambda b: b.loop_parent.__setitem__(1, 2), lambda b: b.instr_engine.__setitem__(0, 2),
+        lambda b: b.trips.__setitem__(2, -1), lambda b: b.instr_pos.__setitem__(2, 5),
+        lambda b: b.dep_prod.__setitem__(0, 3), lambda b: b.prog_n_engines.__setitem__(0, 33))]
+    for seed in range(20):
+        cases.append(workloads.random_trees(seed, 12, workloads.tree_params(any_k=1, k_max=2)))
+    n_bad = 0
+    for batch in cases:
+        desc, keep = sg.batch_desc(batch)
+        st_host = sg.lib().sync_validate_programs(ctypes.byref(desc))
+        msg_host = sg.lib().sync_last_error().decode()
+        h = ctypes.c_void_p()
+        st_dev = sg.lib().sync_load_programs(ctypes.byref(desc), 0, None, ctypes.byref(h))
+        msg_dev = sg.lib().sync_last_error().decode()
+        if st_dev == sg.OK:
+            sg.lib().sync_free_programs(h)
+        assert st_host == st_dev and (st_host == sg.OK or msg_host == msg_dev), (st_host, msg_host, st_dev, msg_dev)
+        n_bad += st_dev != sg.OK
+    assert n_bad >= 20
 
 
 # ------------------------------------------------- full sizes, every program
