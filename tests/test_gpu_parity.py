@@ -449,6 +449,60 @@ def test_loader_offsets_shift_identically(sg):
     assert_parts_match(sg, div, [0, 13, 40], (COUNT, PERLOOP))
 
 
+def test_concurrent_loads_share_the_host_pools(sg):
+    """Loads on several host threads at once (each takes its own scratch and
+    pinned arena from the loader's pools, or a new one): every handle gives
+    the results of the same batch loaded alone."""
+    import threading
+    batches = [workloads.random_trees(8100 + i, 60, workloads.tree_params(
+        engines_hi=5, loops_hi=5, body_hi=6, trip_hi=4, max_depth=4)) for i in range(3)]
+    batches.append(workloads.generate("chain", n_programs=3000))
+    want = [loaded_results(sg, b, (PERLOOP,)) for b in batches]
+    got = [None] * len(batches)
+    errors = []
+
+    def run(i):
+        try:
+            for _ in range(2):
+                got[i] = loaded_results(sg, batches[i], (PERLOOP,))
+        except Exception as e:          # reported below, on the test's thread
+            errors.append(e)
+
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(len(batches))]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors
+    for w, g in zip(want, got):
+        for a, b in zip(w[0], g[0]):
+            assert np.array_equal(a, b)
+
+
+def test_handle_is_ready_on_any_stream(sg):
+    """sync_load_programs returns with its device work queued on its stream;
+    a call on another stream right away waits for it (the handle's event)."""
+    import torch
+    batch = workloads.generate("chain", n_programs=1000)
+    want_thr = oracle.thresholds(batch, PERLOOP)
+    ref = oracle.simulate(batch, want_thr, PERLOOP, oracle.BARRIER_FREE)
+    load_stream = torch.cuda.Stream()
+    other = torch.cuda.Stream()
+    for _ in range(3):
+        torch.cuda.synchronize()
+        torch.cuda._sleep(20_000_000)            # keep the device busy so the load's work queues up
+        h = sg.sync_load_programs(batch, stream=load_stream)
+        with torch.cuda.stream(other):
+            thr = sg.sync_eval_thresholds(h, PERLOOP, stream=other)
+            r = sg.sync_simulate(h, PERLOOP, thr, stream=other)
+        other.synchronize()
+        idx = h.unpadded_index()
+        assert np.array_equal(thr.cpu().numpy()[idx], want_thr)
+        assert np.array_equal(r.makespan.cpu().numpy()[:batch.n_programs], ref.makespan)
+        assert np.array_equal(r.checksum.cpu().numpy()[:batch.n_programs].view(np.uint64), ref.checksum)
+        h.close()
+
+
 def test_device_loader_reports_what_host_validation_does(sg):
     """sync_load_programs validates on the device with the same per-program
     routine that sync_validate_programs runs on the host: on malformed and
