@@ -278,13 +278,19 @@ typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
  * makes that stream wait for the event first, and sync_free_programs waits
  * for the device.  The caller's arrays may be released when the call returns.
  * The host checks the batch's shape (the CSR offsets, trip offsets, NULL
- * arrays); everything per program runs on the GPU: the raw arrays are copied
- * to the device, one pass per program validates it and counts its table
- * entries, a second writes the encoding at the programs' offsets (the same
- * routine as sync_validate_programs, so both report the same first failure:
- * the lowest-numbered failing program's first failure in check order).
- * Device memory for the passes is taken with cudaMallocAsync on `stream` and
- * released on it before the call returns. */
+ * arrays), then runs one routine per program in two passes on host threads
+ * (SYNCGB_LOAD_THREADS=n sets their number): the first validates the
+ * program and counts the entries it adds to each table, the second writes
+ * the encoding at the programs' offsets (the prefix sums of the counts)
+ * into pinned host memory, copied to the device in one transfer; the
+ * per-iteration tables (parent indices, derived arrays, per-mode semaphore
+ * records, tile tables) are then built on the device.  The first failure
+ * reported is the lowest-numbered failing program's first failure in check
+ * order, the same as sync_validate_programs reports.  The device encoding
+ * is one allocation owned by the handle.  The library keeps the passes'
+ * host scratch and the pinned staging memory for reuse by later loads (one
+ * set per load running at the same time, each grown to the largest batch
+ * it has held) until the process ends. */
 sync_status sync_load_programs(const sync_batch_desc *desc, int device, void *stream,
                                sync_programs **out);
 
