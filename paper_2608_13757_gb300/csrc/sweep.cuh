@@ -761,14 +761,13 @@ __device__ __forceinline__ int run_single(const SweepArgs& a, const WarpSmem& S,
 // one chunk (or, barrier-free, one multi-iteration chunk); the first
 // iteration start has been charged.  The lane's record and thresholds stay
 // in registers; the next chunk's thresholds load while this one runs.
+// `one`: with a single iteration, the chunk holding its whole body
+// (zeros otherwise); a chunk of one record is applied directly.
 template <int MODE, bool BB, bool TL, bool FUSED>
 __device__ __forceinline__ int run_loop(const SweepArgs& a, const WarpSmem& S, const ProgInfo& pi, const int4 ch,
-                                        int32_t single, int32_t lo, int32_t hi, int32_t ctag, int lane, int lc,
+                                        const int4 one, int32_t lo, int32_t hi, int32_t ctag, int lane, int lc,
                                         int32_t iter_cost, unsigned long long& chk) {
-  if (single >= 0) {                            // one iteration: of one record?
-    const int4 one = __ldg(a.chunk + single);
-    if (one.y == 1) return run_single<MODE, BB, TL, FUSED>(a, S, pi, one, lo, lane, lc, chk);
-  }
+  if (one.y == 1) return run_single<MODE, BB, TL, FUSED>(a, S, pi, one, lo, lane, lc, chk);
   const int32_t copies = ch.z;
   const bool have = lane < ch.y;
   LaneRec L;
@@ -966,20 +965,23 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         }
         continue;
       }
+      // the item and, for a loop statement, its side record (the child's
+      // trip prefix sums and the chunks holding its whole body), read
+      // together; then the trip bounds and those chunks, together
       const int4 it = __ldg(a.plan + pbeg + item);
+      const int4 ax = __ldg(a.paux + pbeg + item);
       if (it.x == ITEM_LOOP) {                         // a loop statement
+        const int64_t rp = (int64_t)(((uint64_t)(uint32_t)ax.y << 32) | (uint32_t)ax.x);
+        const int32_t lo = __ldg(a.rowptr + rp + g), hi = __ldg(a.rowptr + rp + g + 1);
+        const int32_t body_chunk = BB ? ax.w : ax.z;
+        const int4 chb = body_chunk >= 0 ? __ldg(a.chunk + body_chunk) : make_int4(0, 0, 0, 0);
+        const int4 one = ax.w < 0 ? make_int4(0, 0, 0, 0) : BB ? chb : __ldg(a.chunk + ax.w);
         if (BB) {
           barrier_all(S, pi.ne, a.prm.c_barrier, lane);
         } else {
           if (lane < pi.ne) S.t[lane] += stmt_cost_of(it.z);
         }
         const int32_t child_ic = iter_cost_of(it.z, it.y);
-        // the statement's side record: the child's trip prefix sums, and the
-        // chunk holding its whole body (if one does), fetched together
-        const int4 ax = __ldg(a.paux + pbeg + item);
-        const int64_t rp = (int64_t)(((uint64_t)(uint32_t)ax.y << 32) | (uint32_t)ax.x);
-        const int32_t lo = __ldg(a.rowptr + rp + g), hi = __ldg(a.rowptr + rp + g + 1);
-        const int32_t body_chunk = BB ? ax.w : ax.z;
         ++item;
         if (lo < hi) {
           __syncwarp();
@@ -988,9 +990,8 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
           if (body_chunk >= 0) {
             // one iteration of one record: applied directly; otherwise a
             // loop around one chunk: all its iterations in registers
-            verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, __ldg(a.chunk + body_chunk),
-                                                    hi - lo == 1 ? ax.w : -1, lo, hi, ++ctag, lane,
-                                                    sp + 1, child_ic, chk);
+            verdict = run_loop<MODE, BB, TL, FUSED>(a, S, pi, chb, hi - lo == 1 ? one : make_int4(0, 0, 0, 0), lo,
+                                                    hi, ++ctag, lane, sp + 1, child_ic, chk);
             if (verdict) break;
             continue;
           }
