@@ -328,8 +328,9 @@ struct SweepArgs {
   int32_t frame_depth;
   int32_t ring;              // latest increments kept per semaphore (power of two)
   const int32_t* lflag;      // per loop: 1 if it carries no offset > 0 (trip register elidable)
-  const int4* paux;          // per plan item (loop statements): {child rowptr offset lo, hi,
-                             // chunk of its whole body barrier-free, barrier} (-1: none)
+  const int4* paux;          // per plan item: loop statement {child rowptr offset lo, hi,
+                             // chunk of its whole body barrier-free, barrier} (-1: none);
+                             // segment: its first chunk's record
   // fused simulation (thresholds from the walk's loop state, no threshold
   // array): dep is set (NULL otherwise) and thr is unused
   const DepInfo* dep;

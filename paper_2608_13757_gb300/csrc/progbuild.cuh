@@ -875,15 +875,16 @@ struct ProgBuilder {
     }
   }
 
-  // per loop statement, what the walker needs without further lookups: the
-  // child's rowptr offset, and the chunk that holds its whole body
-  // (barrier-free: the multi-iteration template if there is one), or -1
+  // per plan item, what the walker reads beside it: for a loop statement
+  // the child's rowptr offset and the chunk that holds its whole body
+  // (barrier-free: the multi-iteration template if there is one), or -1;
+  // for a segment the record of its first chunk
   PB_HD void loop_statements(int64_t plan_first) {
     if constexpr (FILL) {
       for (int64_t i = plan_first; i < c[BC_PLAN]; ++i) {
         const int4 v = O.plan[i];
-        if (v.x != ITEM_LOOP) {
-          O.paux[i] = make_int4(0, 0, -1, -1);
+        if (v.x != ITEM_LOOP) {                   // a segment: its first chunk's record
+          O.paux[i] = O.chunks[v.y];
           continue;
         }
         const int32_t m = v.y - l0;

@@ -965,9 +965,10 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         }
         continue;
       }
-      // the item and, for a loop statement, its side record (the child's
-      // trip prefix sums and the chunks holding its whole body), read
-      // together; then the trip bounds and those chunks, together
+      // the item and its side record (a loop statement: the child's trip
+      // prefix sums and the chunks holding its whole body; a segment: its
+      // first chunk), read together; then a statement's trip bounds and
+      // chunks, together
       const int4 it = __ldg(a.plan + pbeg + item);
       const int4 ax = __ldg(a.paux + pbeg + item);
       if (it.x == ITEM_LOOP) {                         // a loop statement
@@ -1025,7 +1026,7 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         continue;
       }
       for (int c = 0; c < it.z && !verdict; ++c) {
-        const int4 ch = __ldg(a.chunk + it.y + c);
+        const int4 ch = c == 0 ? ax : __ldg(a.chunk + it.y + c);   // the first: read with the item
         LaneRec Lr;
         load_lane(a, ch, lane, Lr);
         int32_t T[kMaxDeps];
