@@ -249,8 +249,13 @@ struct ProgBuilder {
   PB_HD int32_t depth(int32_t l) const { return S.depth[l0 + l]; }
 
   // ------------------------------------------------------------ loops
+  // FILL runs after COUNT has passed every program: the scratch COUNT left
+  // for this program (depths, sorted bodies, ranks, consumer grouping) is
+  // still in place, indexed by the program's own ids, so FILL skips the
+  // stages that only rebuild it
   PB_HD bool loops() {
     for (int32_t x = 0; x < nx; ++x) O.ord_off[x0 + x] = -1;
+    if (FILL) return true;
     if (nl < 1) return fail(BE_NO_TOP, 0);
     if (ne < 1 || ne > 32) return fail(BE_ENGINES, ne);
     if (par[0] != -1) return fail(BE_ROOT, 0);
@@ -333,6 +338,7 @@ struct ProgBuilder {
   }
 
   PB_HD bool instrs() {
+    if (FILL) return true;
     for (int32_t x = 0; x < nx; ++x) {
       const int64_t gx = x0 + x;
       if (d.instr_loop[gx] < 0 || d.instr_loop[gx] >= nl) return fail(BE_X_LOOP, x);
@@ -348,6 +354,7 @@ struct ProgBuilder {
   PB_HD int32_t* bptr() const { return S.body_ptr + l0 + p; }
   PB_HD int32_t* body() const { return S.body + x0 + l0; }
   PB_HD bool bodies() {
+    if (FILL) return true;
     int32_t* bp = bptr();
     int64_t* keys = S.keys + x0 + l0;
     int32_t* bd = body();
@@ -374,6 +381,7 @@ struct ProgBuilder {
 
   // N (instructions directly in a loop body on one engine) and K (rank)
   PB_HD void ranks() {
+    if (FILL) return;
     for (int64_t i = 0; i < (int64_t)nl * ne; ++i) S.nloop_eng[row0 + i] = 0;
     const int32_t* bp = bptr();
     const int32_t* bd = body();
@@ -432,11 +440,6 @@ struct ProgBuilder {
   // dependencies: innermost common loop S, the cases of Sec. 5.2, N and K,
   // and everything the threshold kernels read for them
   PB_HD bool deps() {
-    for (int32_t x = 0; x < nx; ++x) {
-      S.x_ndeps[x0 + x] = 0;
-      S.x_dep_begin[x0 + x] = d0;
-      S.x_levels[x0 + x] = 0;
-    }
     for (int64_t i = 0; i < (int64_t)nl * ne; ++i) {
       S.tstart[row0 + i] = -1;
       S.pe_of[row0 + i] = 0;
@@ -611,6 +614,22 @@ struct ProgBuilder {
   // counting sort; a consumer's dependencies start at x_dep_begin, d0 if
   // none); returns the number of waited dependencies
   PB_HD int32_t group() {
+    if (FILL) {                                    // COUNT's grouping stands; the aggregate only
+      int32_t nw = 0;
+      for (int32_t k = 0; k < nd; ++k) {
+        const int64_t gd = d0 + k;
+        if (S.dep_bar[gd]) continue;
+        const int32_t cx = d.dep_cons[gd];
+        pi.pair_levels += (int64_t)levels(d.dep_prod[gd]) * tot(IL(cx), IE(cx));
+        ++nw;
+      }
+      return nw;
+    }
+    for (int32_t x = 0; x < nx; ++x) {
+      S.x_ndeps[x0 + x] = 0;
+      S.x_dep_begin[x0 + x] = d0;
+      S.x_levels[x0 + x] = 0;
+    }
     for (int32_t k = 0; k < nd; ++k) {
       const int64_t gd = d0 + k;
       if (S.dep_bar[gd]) continue;                 // not waited on
