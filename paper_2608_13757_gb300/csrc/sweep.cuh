@@ -557,6 +557,74 @@ __device__ __forceinline__ int run_loop_regs(const SweepArgs& a, const WarpSmem&
     if (vn && ndep > 1) T1n = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + lo + copy);
   }
   for (int32_t g = lo; g < hi;) {
+    // barrier scheme, array pipeline: a run of iterations that all replay the
+    // reference (their waits target the same in-chunk increments, none past
+    // the chunk's) in one pass.  Each starts at a barrier with every engine
+    // at the same cursor and everything earlier retired, so iteration j of
+    // the run starts at base + j*D, D = the reference's largest end (cursor
+    // or last retire) past its base, plus the barrier and the iteration
+    // start; its times are the reference's shifted by its start.
+    if (BB && !FUSED && rep && copies == 1) {
+      const unsigned vm = __ballot_sync(kFull, have);
+      const int32_t inc0 = __popc(wg0 & vm), inc1 = __popc(wg1 & vm);
+      const int32_t B = min(hi - g, 32);
+      int jm = B;                                     // this lane: first iteration that does not replay
+      if (have) {
+        for (int j = 0; j < jm; ++j) {
+          int k0 = 0, k1 = 0;
+          if (ndep > 0) {
+            const int32_t T = __ldg(L.tp[0] + g + j), pb = pub0 + j * inc0;
+            if (T > pb) k0 = T - pb <= inc0 ? T - pb : -1;   // -1: past the chunk's increments
+          }
+          if (ndep > 1) {
+            const int32_t T = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + g + j), pb = pub1 + j * inc1;
+            if (T > pb) k1 = T - pb <= inc1 ? T - pb : -1;
+          }
+          if (k0 != rk0 || k1 != rk1) jm = j;
+        }
+      }
+      const int32_t J = (int32_t)__reduce_min_sync(kFull, (unsigned)jm);
+      if (J > 0) {
+        const int32_t base = __shfl_sync(kFull, ts, 0);
+        const int32_t M = max(0, __reduce_max_sync(kFull, lane < pi.ne && present ? max(rd_t, rd_r) : 0));
+        const int32_t D = M + a.prm.c_barrier + __shfl_sync(kFull, iter_cost, 0);
+        const int32_t cnt = present ? __popc(vm & my_run) : 0;   // engine `lane`'s instances per iteration
+        const int32_t cnt_e = __shfl_sync(kFull, cnt, e), n_e = __shfl_sync(kFull, ns, e);
+        const int32_t rank = __popc(vm & lanemask_le() & run_from_head);
+        if (have) {
+          for (int32_t j = 0; j < J; ++j) {
+            const int32_t bj = base + j * D, issue = bj + rd_issue, retire = bj + rd_retire;
+            const int32_t gl = g + j;
+            const uint32_t nj = (uint32_t)(n_e + j * cnt_e + rank);
+            if (prod_lane) {
+              const int32_t n = own_stride < 0 ? (int32_t)nj : own_stride * gl + own_koff;
+              S.ring[own_ring + ((n - 1) & S.rmask)] = retire;
+              a.hist[own_hist + n] = retire;
+            }
+            chk += inst_term(issue, retire, (uint32_t)e, nj);
+            if (TL) tl_write(a, S, tl_off + gl, issue, retire, nj);
+          }
+        }
+        pub0 += J * inc0;
+        pub1 += J * inc1;
+        own_pub += J * __popc(own_grp & vm);
+        const int32_t blast = base + (J - 1) * D;     // the run's last iteration
+        if (lane < pi.ne) {
+          if (present) {
+            lrs = blast + rd_r;
+            ns += J * cnt;
+          }
+          ts = blast + M + a.prm.c_barrier + (g + J < hi ? iter_cost : 0);
+        }
+        __syncwarp();                                 // ring entries visible to the next iteration
+        g += J;
+        if (g < hi) {
+          if (have && ndep > 0) T0n = __ldg(L.tp[0] + g);
+          if (have && ndep > 1) T1n = __ldg(L.tp[kMaxDeps > 1 ? 1 : 0] + g);
+        }
+        continue;
+      }
+    }
     const int32_t v = min(copies, hi - g);
     int32_t T0, T1;
     if (FUSED) {
