@@ -154,6 +154,19 @@ def test_configs_bit_exact(sg, name, n):
     compare_all(sg, batch, timeline=name in ("small", "depth2"))
 
 
+@pytest.mark.parametrize("seed", range(4))
+def test_long_loops_bit_exact(sg, seed):
+    """Inner loops of up to 40 iterations with offsets up to 2: the barrier
+    sweep writes runs of replayed iterations in one pass, cut where a wait
+    first targets other in-chunk increments or reaches past the chunk's;
+    thresholds, schedules and full timelines equal the oracle's in both
+    schemes."""
+    batch = workloads.random_trees(9700 + seed, 60, workloads.tree_params(
+        engines_hi=5, loops_hi=4, body_hi=8, trip_lo=2, trip_hi=40, max_depth=3, k_max=2, dep_permille=700))
+    compare_all(sg, batch, timeline=True, modes=(COUNT, PERLOOP, PERENGINE),
+                params=oracle.sim_params(ii=2, c_branch=3, c_regop=2, c_barrier=7))
+
+
 @pytest.mark.parametrize("seed", range(6))
 def test_random_trees_bit_exact(sg, seed):
     batch = workloads.random_trees(1000 + seed, 150, workloads.tree_params(
