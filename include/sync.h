@@ -260,8 +260,9 @@ typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
  * never issue; producer nested below S and forward with offset 0; nested and
  * backward with offset 1), computes N and K of the per-loop allocation
  * (Sec. 5.5), and builds the device-resident encoding on `device`: loop
- * table, per-loop trip prefix sums (rowptr) and expanded parent-iteration
- * indices, dependency table, per-(loop, engine) instruction streams.
+ * table, per-loop trip prefix sums (rowptr), dependency table, the derived
+ * per-iteration arrays of the threshold kernels, per-(loop, engine)
+ * instruction streams.
  * Returns SYNC_ERR_MALFORMED for structural errors (listed with sync.h's
  * batch description), SYNC_ERR_NOT_ALLOCATABLE for a dependency outside the
  * cases above (with SYNC_NONALLOC_BARRIER: one that no barrier at the end
@@ -283,8 +284,8 @@ typedef struct sync_programs sync_programs;   /* opaque; owns device memory */
  * program and counts the entries it adds to each table, the second writes
  * the encoding at the programs' offsets (the prefix sums of the counts)
  * into pinned host memory, copied to the device in one transfer; the
- * per-iteration tables (parent indices, derived arrays, per-mode semaphore
- * records, tile tables) are then built on the device.  The first failure
+ * per-iteration tables (derived arrays, per-mode semaphore records, tile
+ * tables) are then built on the device.  The first failure
  * reported is the lowest-numbered failing program's first failure in check
  * order, the same as sync_validate_programs reports.  The device encoding
  * is one allocation owned by the handle.  The library keeps the passes'

@@ -23,7 +23,7 @@ LIB = os.path.join(LIBDIR, "libsyncgb.so")
 CUDA_HOME = os.environ.get("CUDA_HOME", "/usr/local/cuda")
 NVCC = os.path.join(CUDA_HOME, "bin", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-CU = ["k_tiles.cu", "k_expand.cu", "k_thresholds.cu", "k_simulate.cu", "k_sweep.cu", "k_piece.cu", "k_noalloc.cu"]
+CU = ["k_tiles.cu", "k_load.cu", "k_thresholds.cu", "k_simulate.cu", "k_sweep.cu", "k_piece.cu", "k_noalloc.cu"]
 CPP = ["capi.cpp"]
 HEADERS = [os.path.join(CSRC, "enc.h"), os.path.join(CSRC, "progbuild.cuh"), os.path.join(CSRC, "cost.cuh"), os.path.join(CSRC, "sweep.cuh"), os.path.join(CSRC, "handle.h"), os.path.join(CSRC, "waitval.cuh"), os.path.join(ROOT, "include", "sync.h")]
 

@@ -396,7 +396,7 @@ namespace {
 struct HostScratch {
   HostVec<int32_t> i32_nl[2], body_ptr, body, i32_nx[6], i32_rows[2], anc, i32_nd[3];
   HostVec<uint8_t> u8_nl[2], rpflag, dep_bar;
-  HostVec<int64_t> keys, i64_rows[4], ord_off, count, base;
+  HostVec<int64_t> keys, i64_rows[3], ord_off, count, base;
   HostVec<uint32_t> pe_of;
   HostVec<Seen> seen;
   HostVec<ProgSummary> sum;
@@ -525,8 +525,8 @@ void count_pass(const sync_batch_desc& d, const Shape& sh, HostScratch& H, Build
   for (int i = 0; i < 6; ++i) *nx_arrays[i] = sized(H.i32_nx[i], NX);
   S.nloop_eng = sized(H.i32_rows[0], rows);
   S.sem_row = sized(H.i32_rows[1], rows);
-  int64_t** row_arrays[4] = {&S.stot, &S.srp, &S.spi, &S.tstart};
-  for (int i = 0; i < 4; ++i) *row_arrays[i] = sized(H.i64_rows[i], rows);
+  int64_t** row_arrays[3] = {&S.stot, &S.srp, &S.tstart};
+  for (int i = 0; i < 3; ++i) *row_arrays[i] = sized(H.i64_rows[i], rows);
   S.pe_of = sized(H.pe_of, rows);
   S.rpflag = sized(H.rpflag, rows);
   S.anc = sized(H.anc, rows * SYNC_MAX_DEPTH);
@@ -547,6 +547,8 @@ void count_pass(const sync_batch_desc& d, const Shape& sh, HostScratch& H, Build
   check_uncovered(d, sh);
   int64_t* base = sized(H.base, (int64_t)Pq * kBuildCounts);
   for (int i = 0; i < kBuildCounts; ++i) tot[i] = 0;
+  // the derived pool opens with the all-zero ancestor array the programs share
+  for (int32_t p = 0; p < Pq; ++p) tot[BC_DERIVED] = std::max(tot[BC_DERIVED], a.sum[p].zero_len);
   for (int32_t p = 0; p < Pq; ++p)
     for (int i = 0; i < kBuildCounts; ++i) {
       base[(int64_t)p * kBuildCounts + i] = tot[i];
@@ -595,8 +597,8 @@ void work_order(const ProgSummary* sum, int32_t P, int32_t* order) {
 // per-program counts) and FILL (every table at the program's offsets) of
 // progbuild.cuh, one program at a time on host threads, FILL writing into a
 // pinned arena; the tables go to the device in one copy.  On the device,
-// from those tables: the tile tables, the parent-index expansion, the
-// per-mode semaphore records and the derived per-iteration arrays.  The
+// from those tables: the tile tables, the per-mode semaphore records and
+// the derived per-iteration arrays.  The
 // per-program passes are scalar, branchy code over small tables (a few
 // hundred entries per program); the per-iteration and per-pair arrays are
 // built by the GPU.
@@ -621,8 +623,8 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   int64_t hist_max = 0;
   for (int m = 0; m < kModes; ++m) hist_max = std::max(hist_max, h.hist_len[m] = cnt[BC_HIST + m]);
   const int64_t n_first_tiles = (n_pairs_padded + kTilePairs - 1) / kTilePairs;
-  const int64_t n_job_tiles = (n_derived + kTilePairs - 1) / kTilePairs;
-  const int64_t n_rp_tiles = (cnt[BC_ROWPTR] + kTilePairs - 1) / kTilePairs;
+  const int64_t n_drows = cnt[BC_DROWS];
+  const int64_t n_job_tiles = (n_drows + kJobTileRows - 1) / kJobTileRows;
   Layout L;   // the tables the host writes, then the device's own
   const size_t o_loop = L.add<LoopInfo>(NL), o_dep = L.add<DepInfo>(ND), o_prog = L.add<ProgInfo>(P);
   const size_t o_inst = L.add<int64_t>(NX), o_ord = L.add<int64_t>(NX), o_xsem = L.add<int4>(kModes * NX);
@@ -638,11 +640,10 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   const size_t o_chunks = L.add<int4>(cnt[BC_CHUNKS]), o_lrec = L.add<int4>(n_lanes), o_lmeta = L.add<int4>(n_lanes);
   const size_t o_order = L.add<int32_t>(P);
   const size_t host_bytes = L.bytes;
-  const size_t o_pidx = L.add<int32_t>(n_iters), o_derived = L.add<int32_t>(n_derived);
+  const size_t o_derived = L.add<int32_t>(n_derived);
   const size_t o_opsem = L.add<int4>(kModes * n_ops), o_lsem = L.add<int4>(kModes * n_lanes);
   const size_t o_hist = L.add<int32_t>(hist_max), o_slot = L.add<int32_t>(1), o_fallback = L.add<int32_t>((int64_t)P + 1);
   const size_t o_tile_first = L.add<int32_t>(n_first_tiles + 1), o_tile_job = L.add<int32_t>(n_job_tiles + 1);
-  const size_t o_tile_rp = L.add<int32_t>(n_rp_tiles + 1);
   char* dev = h.alloc<char>((int64_t)L.bytes, "encoding");
 
   // ------------------------------------------------------------- FILL
@@ -724,7 +725,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.lrec = reinterpret_cast<int4*>(D(o_lrec));
   h.lmeta = reinterpret_cast<int4*>(D(o_lmeta));
   h.order = reinterpret_cast<int32_t*>(D(o_order));
-  h.pidx = reinterpret_cast<int32_t*>(D(o_pidx));
   h.derived = reinterpret_cast<int32_t*>(D(o_derived));
   h.opsem = reinterpret_cast<int4*>(D(o_opsem));
   h.lsem = reinterpret_cast<int4*>(D(o_lsem));
@@ -732,16 +732,15 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.next_slot = reinterpret_cast<int32_t*>(D(o_slot));
   h.fallback = reinterpret_cast<int32_t*>(D(o_fallback));
   h.tile_first = reinterpret_cast<int32_t*>(D(o_tile_first));
-  const LoopInfo* d_xloops = reinterpret_cast<const LoopInfo*>(D(o_xloops));
   const DeriveJob* d_jobs = reinterpret_cast<const DeriveJob*>(D(o_jobs));
   int32_t* tile_job = reinterpret_cast<int32_t*>(D(o_tile_job));
-  int32_t* tile_rp = reinterpret_cast<int32_t*>(D(o_tile_rp));
 
   // ------------------------------------------------------------ sizes
-  int64_t struct_extra = 0, code_looped = 0, code_unrolled = 0, n_bar_deps = 0;
+  int64_t struct_extra = 0, code_looped = 0, code_unrolled = 0, n_bar_deps = 0, zero_len = 0;
   int32_t ne_max = 1, depth_max = 0, ord_overflow = 0;
   for (int32_t p = 0; p < P; ++p) {
     const ProgSummary& s = a.sum[p];
+    zero_len = std::max(zero_len, s.zero_len);
     struct_extra += s.struct_bytes;
     code_looped += s.code_looped;
     code_unrolled += s.code_unrolled;
@@ -760,7 +759,7 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   h.sz.n_instrs = (int32_t)NX;
   h.sz.n_deps = (int32_t)ND;
   // of the path pool the kernels read only the rowptr offsets from S's
-  // child down to a nested producer's loop; the pidx offsets are read at
+  // child down to a nested producer's loop; the consumer side's are read at
   // load time only
   h.sz.struct_bytes = ND * (int64_t)sizeof(DepInfo) + 8 * (ND + 1) + struct_extra + 4 * (n_first_tiles + 1) +
                       4 * n_derived;
@@ -791,14 +790,14 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
 
   // ----------------------------------------------------------- device
   cuda_check(launch_tile_tables(h.seg, ND, h.tile_first, n_first_tiles, d_jobs, n_jobs, tile_job, n_job_tiles,
-                                d_xloops, n_xloops, tile_rp, n_rp_tiles, h.num_sms, stream),
+                                h.num_sms, stream),
              "tile tables");
-  cuda_check(launch_expand(d_xloops, tile_rp, h.rowptr, cnt[BC_ROWPTR], h.pidx, n_iters, h.num_sms, stream),
-             "expand");
   cuda_check(launch_sem_records(reinterpret_cast<const int4*>(D(o_xsem)), NX, h.ops, n_ops, h.lrec, n_lanes, h.opsem,
                                 h.lsem, h.num_sms, stream),
              "semaphore records");
-  cuda_check(launch_derive(d_jobs, tile_job, h.rowptr, h.pidx, h.path, h.derived, n_derived, h.num_sms, stream),
+  if (zero_len > 0)
+    cuda_check(cudaMemsetAsync(h.derived, 0, (size_t)zero_len * sizeof(int32_t), stream), "derive");
+  cuda_check(launch_derive(d_jobs, tile_job, n_drows, h.rowptr, h.path, h.derived, n_derived, h.num_sms, stream),
              "derive");
   cuda_check(cudaEventCreateWithFlags(&h.ready, cudaEventDisableTiming), "load event");
   cuda_check(cudaEventRecord(h.ready, stream), "load event");
@@ -875,7 +874,7 @@ sync_status sync_pair_offsets(const sync_programs* h, int64_t* offsets, int32_t*
 static ThrArgs thr_args(const sync_programs* h, sync_thr_mode mode) {
   ThrArgs a;
   a.dep = h->dep; a.derived = h->derived; a.ord = h->ord; a.seg = h->seg; a.tile_first = h->tile_first;
-  a.path = h->path; a.rowptr = h->rowptr; a.pidx = h->pidx; a.n_chunks = h->n_chunks; a.mode = mode;
+  a.path = h->path; a.rowptr = h->rowptr; a.n_chunks = h->n_chunks; a.mode = mode;
   return a;
 }
 

@@ -21,11 +21,9 @@ constexpr int kTilePairs = 1024;
 
 // Per loop.  rowptr_l[j], j in [0, total(parent)], is the number of l's
 // iterations that start before the parent's global iteration j (exclusive
-// prefix sum of the trips); pidx_l[g] is the parent's global iteration during
-// l's global iteration g.  The top-level loop has rowptr [0, 1], pidx [0].
+// prefix sum of the trips).  The top-level loop has rowptr [0, 1].
 struct alignas(16) LoopInfo {
   int64_t rowptr_off;
-  int64_t pidx_off;
   int32_t parent;     // -1 for a top-level loop
   int32_t total;      // global iterations
   int32_t n_parent;   // total(parent), 1 for a top-level loop
@@ -33,10 +31,10 @@ struct alignas(16) LoopInfo {
 };
 
 // Per dependency.  `path` points into the int64 path pool:
-//   [0, up)            pidx offsets of the loops from the consumer's loop up
-//                      to (excluding) S, innermost first;
-//   up, up+1           pidx offset and rowptr offset of S;
-//   [up+2, up+2+clen)  rowptr offsets of the loops from S's child down to P
+//   [0, up)            rowptr offsets of the loops from the consumer's loop
+//                      up to (excluding) S, innermost first (read at load
+//                      time, for the consumer iterations' S-ancestors);
+//   [up, up+clen)      rowptr offsets of the loops from S's child down to P
 //                      (nested cases; clen = 0 when P = S).
 struct alignas(16) DepInfo {
   // read for every chunk: the first 48 bytes (three 16-byte loads)
@@ -131,21 +129,34 @@ constexpr int32_t OP_LOOP = -1;
 constexpr int32_t OP_END = -2;
 
 // Derived per-iteration arrays of the threshold and check kernels, built at
-// load time from the trip prefix sums and parent indices (one job each):
-//   DERIVE_TSTART  out[gs] = rowptr_S[pidx_S[gs]]   (a = pidx offset of S,
-//                  b = rowptr offset of S)
-//   DERIVE_ANC     out[g]  = g walked `up` levels up the parent indices
-//                  (a = path pool offset of the pidx offsets, innermost first)
-// Every array starts at a multiple of 4 entries, so a 4-pair chunk reads its
-// four entries with one int4 load.
+// load time from the trip prefix sums alone (one job each).  Both are
+// constant on runs of consecutive entries, one run per row:
+//   DERIVE_TSTART  per iteration gs of S, the first iteration of its trip.
+//                  Rows: S's parent iterations j; row j covers
+//                  [rowptr_S[j], rowptr_S[j+1]) with the value rowptr_S[j]
+//                  (path = rowptr offset of S).
+//   DERIVE_ANC     per iteration g of a loop `up` levels below S, its
+//                  enclosing S-iteration.  Rows: S's iterations j; row j
+//                  covers the first iterations below j, [R(j), R(j+1)), R
+//                  the trip prefix sums composed from S's child down to the
+//                  consumer's loop (path = path pool offset of their rowptr
+//                  offsets, innermost first), with the value j.
+// After its nrows rows a job has one more, [n, len) with the value 0: the
+// padding to a multiple of 4 entries (or, for a barrier-fallback
+// dependency, its whole zero-filled array).  Every array starts at a
+// multiple of 4 entries, so a 4-pair chunk reads its four entries with one
+// int4 load.
 enum : int32_t { DERIVE_TSTART = 0, DERIVE_ANC = 1 };
+constexpr int kJobTileRows = 32;   // rows per derive tile (one warp's rows)
 struct alignas(16) DeriveJob {
-  int64_t out;
-  int64_t a, b;
-  int32_t n;
+  int64_t out;        // derived pool offset of the array
+  int64_t row0;       // the job's first row among the rows of all jobs
+  int64_t path;
+  int64_t len;        // entries reserved (n padded)
+  int32_t nrows;
+  int32_t n;          // entries of the array proper
   int32_t kind;
   int32_t up;
-  int32_t pad_;
 };
 
 struct ThrArgs {
@@ -156,7 +167,6 @@ struct ThrArgs {
   const int32_t* tile_first; // [n_tiles + 1]
   const int64_t* path;
   const int32_t* rowptr;
-  const int32_t* pidx;
   int64_t n_chunks;
   int32_t mode;
 };
@@ -344,11 +354,6 @@ struct SweepArgs {
 };
 
 // Launchers (return the launch error, if any).
-// tile_rp[t] = iteration space whose rowptr segment holds entry t*kTilePairs
-// (largest l with rowptr_off[l] <= t*kTilePairs), with one extra entry
-// n_spaces-1; n_rowptr = rowptr entries.
-cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_rp, const int32_t* rowptr, int64_t n_rowptr,
-                          int32_t* pidx, int64_t n_iters, int num_sms, cudaStream_t s);
 // Semaphore records of the op rows and sweep lanes, per threshold mode,
 // gathered from the per-instruction table xsem[m * n_instrs + x] by the
 // record's global instruction x (LOOP and END op records: {-1, 0, 0, 0}):
@@ -356,10 +361,11 @@ cudaError_t launch_expand(const LoopInfo* loop, const int32_t* tile_rp, const in
 cudaError_t launch_sem_records(const int4* xsem, int64_t n_instrs, const int4* ops, int64_t n_ops,
                                const int4* lrec, int64_t n_lanes, int4* opsem, int4* lsem, int num_sms,
                                cudaStream_t s);
-// tile_job[t] = job whose output holds pool entry t*kTilePairs.
-cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, const int32_t* rowptr,
-                          const int32_t* pidx, const int64_t* path, int32_t* derived, int64_t n,
-                          int num_sms, cudaStream_t s);
+// tile_job[t] = job holding row t*kJobTileRows (largest i with jobs[i].row0
+// <= t*kJobTileRows), with one extra entry n_jobs-1; n_rows = rows of all
+// jobs, n = derived pool entries.
+cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, int64_t n_rows, const int32_t* rowptr,
+                          const int64_t* path, int32_t* derived, int64_t n, int num_sms, cudaStream_t s);
 // Per-engine allocation (Sec. 6.1): ord[ord_off[x] + g] = 1-based position of
 // instruction x's instance at global iteration g of its loop in its engine's
 // dynamic stream, for every x with ord_off[x] >= 0; one thread per (program,

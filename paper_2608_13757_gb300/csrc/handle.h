@@ -49,7 +49,6 @@ struct sync_programs {
   // threshold / checker encoding
   syncgb::LoopInfo* loop = nullptr;
   int32_t* rowptr = nullptr;
-  int32_t* pidx = nullptr;
   syncgb::DepInfo* dep = nullptr;
   int32_t* ddep = nullptr;          // per consumer-grouped dependency: dependency id
   int32_t* lflag = nullptr;         // per loop: trip register elidable

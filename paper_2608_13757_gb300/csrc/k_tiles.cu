@@ -1,14 +1,14 @@
-// Tile tables of the threshold, derive and expand kernels, built by the
-// loader on the device from the tables it copied there.
+// Tile tables of the threshold and derive kernels, built by the loader on
+// the device from the tables it copied there.
 #include "progbuild.cuh"
 
 namespace syncgb {
 namespace {
 
-// table[t] = largest i < n with start(i) <= t * kTilePairs (start
-// nondecreasing, start(0) = 0), for t < n_tiles; table[n_tiles] = n - 1.
+// table[t] = largest i < n with start(i) <= t * tile (start nondecreasing,
+// start(0) = 0), for t < n_tiles; table[n_tiles] = n - 1.
 template <class F>
-__global__ void k_tile_table(int32_t* table, int64_t n_tiles, int64_t n, F start) {
+__global__ void k_tile_table(int32_t* table, int64_t n_tiles, int64_t n, int64_t tile, F start) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t <= n_tiles; t += stride) {
     if (n == 0) { table[t] = 0; continue; }
@@ -16,7 +16,7 @@ __global__ void k_tile_table(int32_t* table, int64_t n_tiles, int64_t n, F start
     int64_t lo = 0, hi = n - 1;
     while (lo < hi) {
       const int64_t mid = (lo + hi + 1) / 2;
-      if (start(mid) <= t * kTilePairs) lo = mid; else hi = mid - 1;
+      if (start(mid) <= t * tile) lo = mid; else hi = mid - 1;
     }
     table[t] = (int32_t)lo;
   }
@@ -26,13 +26,9 @@ struct SegStart {
   const int64_t* seg;
   __device__ int64_t operator()(int64_t i) const { return seg[i]; }
 };
-struct JobStart {
+struct JobRowStart {
   const DeriveJob* jobs;
-  __device__ int64_t operator()(int64_t i) const { return jobs[i].out; }
-};
-struct RowptrStart {
-  const LoopInfo* xloops;
-  __device__ int64_t operator()(int64_t i) const { return xloops[i].rowptr_off; }
+  __device__ int64_t operator()(int64_t i) const { return jobs[i].row0; }
 };
 
 int grid_for(int64_t n, int threads, int num_sms) {
@@ -42,8 +38,9 @@ int grid_for(int64_t n, int threads, int num_sms) {
 }
 
 template <class F>
-cudaError_t tile_table(int32_t* table, int64_t n_tiles, int64_t n, F start, int num_sms, cudaStream_t s) {
-  k_tile_table<<<grid_for(n_tiles + 1, 256, num_sms), 256, 0, s>>>(table, n_tiles, n, start);
+cudaError_t tile_table(int32_t* table, int64_t n_tiles, int64_t n, int64_t tile, F start, int num_sms,
+                       cudaStream_t s) {
+  k_tile_table<<<grid_for(n_tiles + 1, 256, num_sms), 256, 0, s>>>(table, n_tiles, n, tile, start);
   return launched();
 }
 
@@ -51,11 +48,9 @@ cudaError_t tile_table(int32_t* table, int64_t n_tiles, int64_t n, F start, int 
 
 cudaError_t launch_tile_tables(const int64_t* seg, int64_t n_deps, int32_t* tile_first, int64_t n_first_tiles,
                                const DeriveJob* jobs, int64_t n_jobs, int32_t* tile_job, int64_t n_job_tiles,
-                               const LoopInfo* xloops, int64_t n_xloops, int32_t* tile_rp,
-                               int64_t n_rp_tiles, int num_sms, cudaStream_t s) {
-  cudaError_t e = tile_table(tile_first, n_first_tiles, n_deps, SegStart{seg}, num_sms, s);
-  if (e == cudaSuccess) e = tile_table(tile_job, n_job_tiles, n_jobs, JobStart{jobs}, num_sms, s);
-  if (e == cudaSuccess) e = tile_table(tile_rp, n_rp_tiles, n_xloops, RowptrStart{xloops}, num_sms, s);
+                               int num_sms, cudaStream_t s) {
+  cudaError_t e = tile_table(tile_first, n_first_tiles, n_deps, kTilePairs, SegStart{seg}, num_sms, s);
+  if (e == cudaSuccess) e = tile_table(tile_job, n_job_tiles, n_jobs, kJobTileRows, JobRowStart{jobs}, num_sms, s);
   return e;
 }
 

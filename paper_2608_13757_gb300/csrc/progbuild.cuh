@@ -41,7 +41,7 @@ constexpr int64_t kCodeLoopOps = 4;
 // Appended tables: entries each program appends, counted by COUNT.
 enum : int32_t {
   BC_ROWPTR = 0,   // trip prefix sums (n_parent + 1 per iteration space)
-  BC_ITERS,        // global loop iterations (parent-index pool)
+  BC_ITERS,        // global loop iterations
   BC_INST,         // datapath instances
   BC_PAIRS,        // (dependency, consumer instance) pairs
   BC_PADDED,       // pairs with every dependency's segment padded to 4
@@ -55,6 +55,7 @@ enum : int32_t {
   BC_LANES,        // sweep lanes
   BC_SEMHB,        // semaphore history bases
   BC_JOBS,         // derive jobs
+  BC_DROWS,        // rows of the derive jobs
   kBuildCounts
 };
 
@@ -100,7 +101,7 @@ struct BuildScratch {
   int32_t* body;                             // [NX + NL]
   int32_t *rank, *x_ndeps, *x_dep_begin, *x_levels, *cons_next, *sem_x;   // [NX]
   int32_t *nloop_eng, *sem_row;              // [rows]
-  int64_t *stot, *srp, *spi, *tstart;        // [rows] per iteration space
+  int64_t *stot, *srp, *tstart;              // [rows] per iteration space
   uint32_t* pe_of;                           // [rows]
   uint8_t* rpflag;                           // [rows]
   int32_t* anc;                              // [rows * SYNC_MAX_DEPTH]
@@ -147,6 +148,7 @@ struct alignas(16) ProgSummary {
   int64_t code_looped, code_unrolled;   // static instructions (code-size proxy)
   int64_t n_bar_deps;      // barrier-fallback dependencies
   int64_t struct_bytes;    // path entries and rowptr spaces the threshold kernels read
+  int64_t zero_len;        // entries of the longest all-zero ancestor array (shared)
   int64_t err_index;
   int32_t nsem[kModes];
   int32_t ne, depth_max, ord_overflow, err, splittable;
@@ -288,7 +290,6 @@ struct ProgBuilder {
     const int64_t r = row0 + (int64_t)l * ne + e;
     S.stot[r] = t;
     S.srp[r] = c[BC_ROWPTR];
-    S.spi[r] = c[BC_ITERS];
     S.rpflag[r] = 0;
     if (FILL) {
       LoopInfo L{};
@@ -297,7 +298,6 @@ struct ProgBuilder {
       L.n_parent = (int32_t)want;
       L.depth = depth(l);
       L.rowptr_off = c[BC_ROWPTR];
-      L.pidx_off = c[BC_ITERS];
       const int64_t xi = xbase + xid(l, e);
       O.xloops[xi] = L;
       int32_t* rp = O.rowptr + c[BC_ROWPTR];
@@ -424,14 +424,21 @@ struct ProgBuilder {
     pi.divergent = d.div ? 1 : 0;
   }
 
-  PB_HD void job(int64_t out, int64_t a, int64_t b, int64_t n, int32_t kind, int32_t up) {
+  // a derive job (enc.h) at the pool's end: nrows rows, n entries, len
+  // reserved, and the padding row
+  PB_HD void job(int64_t path, int64_t nrows, int64_t n, int64_t len, int32_t kind, int32_t up) {
     if (FILL) {
       DeriveJob J{};
-      J.out = out; J.a = a; J.b = b; J.n = (int32_t)n; J.kind = kind; J.up = up;
+      J.out = c[BC_DERIVED]; J.row0 = c[BC_DROWS]; J.path = path; J.len = len;
+      J.nrows = (int32_t)nrows; J.n = (int32_t)n; J.kind = kind; J.up = up;
       O.jobs[c[BC_JOBS]] = J;
     }
     c[BC_JOBS]++;
+    c[BC_DROWS] += nrows + 1;
+    c[BC_DERIVED] += len;
   }
+  // iterations of the parent of iteration space (l, e): the rows of its trips
+  PB_HD int64_t n_parent(int32_t l, int32_t e) const { return l == 0 ? 1 : tot(par[l], e); }
   PB_HD void push_path(int64_t v) {
     if (FILL) O.path[c[BC_PATH]] = v;
     c[BC_PATH]++;
@@ -502,8 +509,7 @@ struct ProgBuilder {
           O.dep_count[gd] = (int32_t)n;
           O.seg[gd] = c[BC_PADDED];
         }
-        job(c[BC_DERIVED], 0, 0, 0, DERIVE_TSTART, 0);
-        c[BC_DERIVED] += pad4(n);
+        job(0, 0, 0, pad4(n), DERIVE_TSTART, 0);
         c[BC_PAIRS] += n;
         c[BC_PADDED] += pad4(n);
         S.dep_N[gd] = 0;
@@ -523,14 +529,13 @@ struct ProgBuilder {
       D.path = c[BC_PATH];
       // everything below is read on the consumer engine's iteration spaces
       // (Eq. (1) with that engine's loop-entry counts)
-      for (int32_t l = Cl; l != Sl; l = par[l]) push_path(S.spi[sr(l, ec)]);
+      for (int32_t l = Cl; l != Sl; l = par[l]) push_path(S.srp[sr(l, ec)]);
       for (int32_t l = Pl; l != Sl; l = par[l]) S.rpflag[sr(l, ec)] = 1;
       // derived arrays: trip starts of S, and the S-ancestors of the consumer loop
       const int64_t skey = sr(Sl, ec);
       if (S.tstart[skey] < 0) {
         S.tstart[skey] = c[BC_DERIVED];
-        job(c[BC_DERIVED], S.spi[skey], S.srp[skey], tot(Sl, ec), DERIVE_TSTART, 0);
-        c[BC_DERIVED] += pad4(tot(Sl, ec));
+        job(S.srp[skey], n_parent(Sl, ec), tot(Sl, ec), pad4(tot(Sl, ec)), DERIVE_TSTART, 1);
       }
       D.tstart = S.tstart[skey];
       if (O.ord_off[x0 + px] < 0) {
@@ -539,19 +544,21 @@ struct ProgBuilder {
       }
       D.ordp = O.ord_off[x0 + px];
       D.src = D.tstart;
-      if (D.up > 0) {
+      if (D.up > 0 && tot(Sl, ec) == 1) {
+        // S runs once: every consumer iteration's S-ancestor is 0, an array
+        // all programs share (the derived pool's zero-filled head)
+        D.src = 0;
+        sm.zero_len = pb_max(sm.zero_len, pad4(n));
+      } else if (D.up > 0) {
         int32_t& first = S.anc[sr(Cl, ec) * SYNC_MAX_DEPTH + (D.up - 1)];
         if (first < 0) {
           first = k;
-          job(c[BC_DERIVED], D.path, 0, n, DERIVE_ANC, D.up);
           D.src = c[BC_DERIVED];
-          c[BC_DERIVED] += pad4(n);
+          job(D.path, tot(Sl, ec), n, pad4(n), DERIVE_ANC, D.up);
         } else {
           D.src = FILL ? O.dep[d0 + first].src : 0;
         }
       }
-      push_path(S.spi[skey]);
-      push_path(S.srp[skey]);
       // rowptr offsets from S's child down to the producer's loop
       for (int32_t l = Pl, i = D.clen - 1; l != Sl; l = par[l], --i)
         if (FILL) O.path[c[BC_PATH] + i] = S.srp[sr(l, ec)];
@@ -658,6 +665,7 @@ struct ProgBuilder {
   // per (loop, engine), the producer engines whose cached path sums the
   // engine updates at the loop's iteration starts; the bound's terms.
   PB_HD void reductions() {
+    if (!FILL) return;                             // nothing COUNT reports depends on them
     const int32_t* bp = bptr();
     const int32_t* bd = body();
     Seen* seen = S.seen + d0;
@@ -775,6 +783,16 @@ struct ProgBuilder {
   PB_HD void op_rows() {
     const int32_t* bp = bptr();
     const int32_t* bd = body();
+    if constexpr (!FILL) {
+      // every instruction on its engine's row, every child loop and an END
+      // record on each engine's row
+      for (int32_t l = 0; l < nl; ++l) {
+        int32_t nloops = 0;
+        for (int32_t i = bp[l]; i < bp[l + 1]; ++i) nloops += bd[i] < 0 ? 1 : 0;
+        c[BC_OPS] += (bp[l + 1] - bp[l] - nloops) + (int64_t)ne * (nloops + 1);
+      }
+      return;
+    }
     for (int32_t l = 0; l < nl; ++l)
       for (int32_t e = 0; e < ne; ++e) {
         const int64_t row = row0 + (int64_t)l * ne + e;
@@ -863,6 +881,11 @@ struct ProgBuilder {
             // up to 32 records, engine-major and in body order within an
             // engine (a counting sort by engine)
             const int32_t n = (int32_t)pb_min(32, i - b);
+            if constexpr (!FILL) {                // COUNT: the chunk's size only
+              c[BC_LANES] += n;
+              c[BC_CHUNKS]++;
+              continue;
+            }
             int32_t cnt[33], piece[32];
             for (int32_t e = 0; e <= 32; ++e) cnt[e] = 0;
             for (int32_t j = 0; j < n; ++j) ++cnt[IE(bd[b + j]) + 1];
@@ -883,6 +906,11 @@ struct ProgBuilder {
       const int32_t L = bp[l + 1] - bp[l];
       if (nloops == 0 && nseg == 1 && L >= 1 && L <= 16) {
         const int32_t k = 32 / L;
+        if constexpr (!FILL) {                    // COUNT: every record in each of k copies
+          c[BC_LANES] += (int64_t)k * L;
+          c[BC_CHUNKS]++;
+          continue;
+        }
         int32_t recs[32], copies[32], n = 0;
         for (int32_t e = 0; e < ne; ++e)
           for (int32_t cp = 0; cp < k; ++cp)
@@ -966,12 +994,10 @@ struct ProgBuilder {
   }
 };
 
-// Tile tables (k_tiles.cu) of the threshold kernels (segment starts), the
-// derive kernel (job outputs) and the expand kernel (iteration spaces'
-// rowptr offsets).
+// Tile tables (k_tiles.cu) of the threshold kernels (segment starts) and
+// the derive kernel (job rows).
 cudaError_t launch_tile_tables(const int64_t* seg, int64_t n_deps, int32_t* tile_first, int64_t n_first_tiles,
                                const DeriveJob* jobs, int64_t n_jobs, int32_t* tile_job, int64_t n_job_tiles,
-                               const LoopInfo* xloops, int64_t n_xloops, int32_t* tile_rp,
-                               int64_t n_rp_tiles, int num_sms, cudaStream_t s);
+                               int num_sms, cudaStream_t s);
 
 }  // namespace syncgb

@@ -14,7 +14,7 @@ namespace syncgb {
 // total(S)): compose the trip prefix sums from S's child down to P.
 template <class A>
 __device__ __forceinline__ int32_t count_down(const A& a, const DepInfo& D, int32_t x) {
-  for (int i = 0; i < D.clen; ++i) x = __ldg(a.rowptr + __ldg(a.path + D.path + D.up + 2 + i) + x);
+  for (int i = 0; i < D.clen; ++i) x = __ldg(a.rowptr + __ldg(a.path + D.path + D.up + i) + x);
   return x;
 }
 
