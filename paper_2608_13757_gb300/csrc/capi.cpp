@@ -547,8 +547,6 @@ void count_pass(const sync_batch_desc& d, const Shape& sh, HostScratch& H, Build
   check_uncovered(d, sh);
   int64_t* base = sized(H.base, (int64_t)Pq * kBuildCounts);
   for (int i = 0; i < kBuildCounts; ++i) tot[i] = 0;
-  // the derived pool opens with the all-zero ancestor array the programs share
-  for (int32_t p = 0; p < Pq; ++p) tot[BC_DERIVED] = std::max(tot[BC_DERIVED], a.sum[p].zero_len);
   for (int32_t p = 0; p < Pq; ++p)
     for (int i = 0; i < kBuildCounts; ++i) {
       base[(int64_t)p * kBuildCounts + i] = tot[i];
@@ -736,11 +734,10 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   int32_t* tile_job = reinterpret_cast<int32_t*>(D(o_tile_job));
 
   // ------------------------------------------------------------ sizes
-  int64_t struct_extra = 0, code_looped = 0, code_unrolled = 0, n_bar_deps = 0, zero_len = 0;
+  int64_t struct_extra = 0, code_looped = 0, code_unrolled = 0, n_bar_deps = 0;
   int32_t ne_max = 1, depth_max = 0, ord_overflow = 0;
   for (int32_t p = 0; p < P; ++p) {
     const ProgSummary& s = a.sum[p];
-    zero_len = std::max(zero_len, s.zero_len);
     struct_extra += s.struct_bytes;
     code_looped += s.code_looped;
     code_unrolled += s.code_unrolled;
@@ -795,8 +792,6 @@ static void build(const sync_batch_desc& d, int device, cudaStream_t stream, syn
   cuda_check(launch_sem_records(reinterpret_cast<const int4*>(D(o_xsem)), NX, h.ops, n_ops, h.lrec, n_lanes, h.opsem,
                                 h.lsem, h.num_sms, stream),
              "semaphore records");
-  if (zero_len > 0)
-    cuda_check(cudaMemsetAsync(h.derived, 0, (size_t)zero_len * sizeof(int32_t), stream), "derive");
   cuda_check(launch_derive(d_jobs, tile_job, n_drows, h.rowptr, h.path, h.derived, n_derived, h.num_sms, stream),
              "derive");
   cuda_check(cudaEventCreateWithFlags(&h.ready, cudaEventDisableTiming), "load event");

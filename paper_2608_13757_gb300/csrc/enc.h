@@ -40,7 +40,8 @@ struct alignas(16) DepInfo {
   // read for every chunk: the first 48 bytes (three 16-byte loads)
   int64_t seg_off;    // pair-layout offset of this dependency's segment
   int64_t src;        // derived pool, per consumer iteration: its trip start of S
-                      // (consumer directly in S) or its enclosing S-iteration (below S)
+                      // (consumer directly in S) or its enclosing S-iteration (below
+                      // S); -1 when S runs once (S-iteration 0, trip start 0)
   int64_t tstart;     // derived pool: first iteration of the trip, per iteration of S
   int32_t total;      // consumer instances (= total of the consumer's loop)
   int32_t k, N, K;

@@ -50,13 +50,18 @@ template <bool CHECK>
 __device__ __forceinline__ int4 chunk_values(const ThrArgs& a, const DepInfo& D, int32_t g0, int mode) {
   const int32_t n = D.total - g0 < kChunk ? D.total - g0 : kChunk;   // >= 1
   const int32_t* ts = a.derived + D.tstart;
-  const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.src + g0));
   int32_t gs[kChunk], st[kChunk];
-  if (D.up == 0) {
+  if (D.src < 0) {
+    // S runs once: every consumer iteration is in S-iteration 0, trip start 0
+#pragma unroll
+    for (int i = 0; i < kChunk; ++i) gs[i] = st[i] = 0;
+  } else if (D.up == 0) {
+    const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.src + g0));
     // consumer directly in S: g_S = g
     gs[0] = g0; gs[1] = g0 + 1; gs[2] = g0 + 2; gs[3] = g0 + 3;
     st[0] = x.x; st[1] = x.y; st[2] = x.z; st[3] = x.w;
   } else {
+    const int4 x = __ldg(reinterpret_cast<const int4*>(a.derived + D.src + g0));
     gs[0] = x.x; gs[1] = x.y; gs[2] = x.z; gs[3] = x.w;
     st[0] = __ldg(ts + gs[0]);
     st[3] = n > 3 && gs[3] != gs[0] ? __ldg(ts + gs[3]) : st[0];

@@ -148,7 +148,6 @@ struct alignas(16) ProgSummary {
   int64_t code_looped, code_unrolled;   // static instructions (code-size proxy)
   int64_t n_bar_deps;      // barrier-fallback dependencies
   int64_t struct_bytes;    // path entries and rowptr spaces the threshold kernels read
-  int64_t zero_len;        // entries of the longest all-zero ancestor array (shared)
   int64_t err_index;
   int32_t nsem[kModes];
   int32_t ne, depth_max, ord_overflow, err, splittable;
@@ -544,11 +543,10 @@ struct ProgBuilder {
       }
       D.ordp = O.ord_off[x0 + px];
       D.src = D.tstart;
-      if (D.up > 0 && tot(Sl, ec) == 1) {
-        // S runs once: every consumer iteration's S-ancestor is 0, an array
-        // all programs share (the derived pool's zero-filled head)
-        D.src = 0;
-        sm.zero_len = pb_max(sm.zero_len, pad4(n));
+      if (tot(Sl, ec) == 1) {
+        // S runs once: every consumer iteration lies in S-iteration 0, whose
+        // trip starts at 0; the kernels take both without reading an array
+        D.src = -1;
       } else if (D.up > 0) {
         int32_t& first = S.anc[sr(Cl, ec) * SYNC_MAX_DEPTH + (D.up - 1)];
         if (first < 0) {
