@@ -743,36 +743,36 @@ struct ProgBuilder {
       }
       pi.nsem[m] = nsem;
       sm.nsem[m] = nsem;
-      if constexpr (FILL) fill_semaphores(m, nw, sem);
     }
+    if constexpr (FILL) fill_semaphores(nw, sem_e);
   }
 
-  template <class F>
-  // the semaphore records of mode m (instructions, consumer-grouped dependencies)
-  PB_HD void fill_semaphores(int m, int32_t nw, F& sem) {
+  // the semaphore records of the three modes (instructions, consumer-grouped
+  // dependencies): per mode the semaphore and its history stride and offset
+  // (one increment per iteration; N per iteration at rank K; one per
+  // instance of the engine, numbered by its ordinal)
+  PB_HD void fill_semaphores(int32_t nw, const int32_t* sem_e) {
     for (int32_t x = 0; x < nx; ++x) {
-      const int32_t s = sem(x);
-      int32_t hstride = 0, koff = 0;
-      if (s >= 0) {
-        hstride = m == 0 ? 1 : m == 1 ? S.nloop_eng[row0 + (int64_t)IL(x) * ne + IE(x)] : -1;
-        koff = m == 0 ? 1 : m == 1 ? S.rank[x0 + x] : 0;
-      }
-      O.xsem[(int64_t)m * d.NX + x0 + x] = make_int4(s, hstride, koff, m == 2 ? S.x_levels[x0 + x] : 0);
+      const int32_t e = IE(x);
+      const int64_t row = row0 + (int64_t)IL(x) * ne + e;
+      const int32_t s0 = S.sem_x[x0 + x], s1 = S.sem_row[row], s2 = sem_e[e];
+      O.xsem[x0 + x] = make_int4(s0, s0 >= 0 ? 1 : 0, s0 >= 0 ? 1 : 0, 0);
+      O.xsem[d.NX + x0 + x] = make_int4(s1, s1 >= 0 ? S.nloop_eng[row] : 0, s1 >= 0 ? S.rank[x0 + x] : 0, 0);
+      O.xsem[2 * d.NX + x0 + x] = make_int4(s2, s2 >= 0 ? -1 : 0, 0, S.x_levels[x0 + x]);
     }
     for (int32_t i = 0; i < nw; ++i) {
       const int64_t gd = d0 + S.by_cons[d0 + i];
-      O.dsem[(int64_t)m * d.ND + d0 + i] = sem(d.dep_prod[gd]);
-      if (m == 0) {
-        O.dseg[d0 + i] = O.seg[gd];
-        O.ddep[d0 + i] = (int32_t)gd;
-      }
+      const int32_t px = d.dep_prod[gd], e = IE(px);
+      O.dsem[d0 + i] = S.sem_x[x0 + px];
+      O.dsem[d.ND + d0 + i] = S.sem_row[row0 + (int64_t)IL(px) * ne + e];
+      O.dsem[2 * d.ND + d0 + i] = sem_e[e];
+      O.dseg[d0 + i] = O.seg[gd];
+      O.ddep[d0 + i] = (int32_t)gd;
     }
     for (int32_t i = nw; i < nd; ++i) {          // slots of barrier-fallback dependencies: unused
-      O.dsem[(int64_t)m * d.ND + d0 + i] = -1;
-      if (m == 0) {
-        O.dseg[d0 + i] = 0;
-        O.ddep[d0 + i] = d0 + i;
-      }
+      for (int m = 0; m < kModes; ++m) O.dsem[(int64_t)m * d.ND + d0 + i] = -1;
+      O.dseg[d0 + i] = 0;
+      O.ddep[d0 + i] = d0 + i;
     }
   }
 
@@ -791,58 +791,71 @@ struct ProgBuilder {
       }
       return;
     }
-    for (int32_t l = 0; l < nl; ++l)
+    // one pass over each body: an engine's rows follow each other, so each
+    // item goes to its engine's write position (a child loop to every
+    // engine's); a LOOP or END record closes the instructions before it
+    // (their op stop is that record)
+    int64_t pos[32], pend[32];
+    int32_t cnt[32];
+    for (int32_t l = 0; l < nl; ++l) {
+      int32_t nloops = 0;
+      for (int32_t e = 0; e < ne; ++e) cnt[e] = 0;
+      for (int32_t i = bp[l]; i < bp[l + 1]; ++i) {
+        const int32_t it = bd[i];
+        if (it < 0) ++nloops; else ++cnt[IE(it)];
+      }
+      int64_t at = c[BC_OPS];
       for (int32_t e = 0; e < ne; ++e) {
-        const int64_t row = row0 + (int64_t)l * ne + e;
-        const int64_t first = c[BC_OPS];
-        if (FILL) O.op_ptr[row] = (int32_t)first;
-        bool has_loop = false;
-        for (int32_t i = bp[l]; i < bp[l + 1]; ++i) {
-          const int32_t it = bd[i];
-          if (it < 0) {
-            const int32_t m = -it - 1;
-            const int64_t rp = S.srp[sr(m, e)];
-            if (FILL)
-              O.ops[c[BC_OPS]] = make_int4(OP_LOOP, (int32_t)(row0 + (int64_t)m * ne),
-                                           (int32_t)(uint32_t)(rp & 0xffffffffu), (int32_t)(rp >> 32));
-            c[BC_OPS]++;
-            has_loop = true;
-          } else if (IE(it) == e) {
-            if (FILL)
-              O.ops[c[BC_OPS]] = make_int4(x0 + it, d.instr_latency[x0 + it], S.x_ndeps[x0 + it],
+        O.op_ptr[row0 + (int64_t)l * ne + e] = (int32_t)at;
+        pos[e] = pend[e] = at;
+        at += cnt[e] + nloops + 1;
+      }
+      auto close = [&](int32_t e, int64_t q) {
+        for (int64_t r = pend[e]; r <= q; ++r) O.opstop[r] = (int32_t)q;
+        pend[e] = q + 1;
+      };
+      for (int32_t i = bp[l]; i < bp[l + 1]; ++i) {
+        const int32_t it = bd[i];
+        if (it < 0) {
+          const int32_t m = -it - 1;
+          for (int32_t e = 0; e < ne; ++e) {
+            const int64_t rp = S.srp[sr(m, e)], q = pos[e]++;
+            O.ops[q] = make_int4(OP_LOOP, (int32_t)(row0 + (int64_t)m * ne), (int32_t)(uint32_t)(rp & 0xffffffffu),
+                                 (int32_t)(rp >> 32));
+            close(e, q);
+          }
+        } else {
+          O.ops[pos[IE(it)]++] = make_int4(x0 + it, d.instr_latency[x0 + it], S.x_ndeps[x0 + it],
                                            S.x_dep_begin[x0 + it]);
-            c[BC_OPS]++;
-          }
-        }
-        const int64_t end_idx = c[BC_OPS];
-        if (FILL) O.ops[end_idx] = make_int4(OP_END, 0, 0, 0);
-        c[BC_OPS]++;
-        const int32_t nh = pb_popc(S.pe_of[row]);
-        pi.licm_upd += (int64_t)nh * tot(l, e);
-        if constexpr (FILL) {
-          O.rowinfo[row] = make_int2((int32_t)end_idx, (has_loop ? 1 : 0) | (O.lflag[l0 + l] ? 2 : 0) |
-                                                           (S.fbar[l0 + l] ? 4 : 0));
-          O.hoist[row] = nh;
-          int32_t next = (int32_t)end_idx;
-          for (int64_t r = end_idx; r >= first; --r) {
-            if (O.ops[r].x < 0) next = (int32_t)r;
-            O.opstop[r] = next;
-          }
         }
       }
+      const int32_t flags = (nloops > 0 ? 1 : 0) | (O.lflag[l0 + l] ? 2 : 0) | (S.fbar[l0 + l] ? 4 : 0);
+      for (int32_t e = 0; e < ne; ++e) {
+        const int64_t row = row0 + (int64_t)l * ne + e, q = pos[e];
+        O.ops[q] = make_int4(OP_END, 0, 0, 0);
+        close(e, q);
+        const int32_t nh = pb_popc(S.pe_of[row]);
+        pi.licm_upd += (int64_t)nh * tot(l, e);
+        O.rowinfo[row] = make_int2((int32_t)q, flags);
+        O.hoist[row] = nh;
+      }
+      c[BC_OPS] = at;
+    }
   }
 
   // one sweep chunk: n <= 32 lanes `recs` (program-local instructions,
-  // already engine-major) with their iteration copies (nullptr: all copy 0)
-  PB_HD void add_chunk(const int32_t* recs, const int32_t* copies, int32_t n, int32_t ncopies) {
+  // already engine-major, their engines `engs`) with their iteration copies
+  // (nullptr: all copy 0)
+  PB_HD void add_chunk(const int32_t* recs, const int32_t* engs, const int32_t* copies, int32_t n,
+                       int32_t ncopies) {
     const int64_t base = c[BC_LANES];
     int32_t emask = 0, head = 0;
     for (int32_t i = 0; i < n; ++i) {
-      const int32_t x = recs[i], e = IE(x);
+      const int32_t x = recs[i], e = engs[i];
       const int32_t cp = copies ? copies[i] : 0;
       emask |= (int32_t)(1u << e);
-      if (i > 0 && IE(recs[i - 1]) != e) head = i;     // first lane of the engine's run
-      const bool last = i + 1 == n || IE(recs[i + 1]) != e;
+      if (i > 0 && engs[i - 1] != e) head = i;         // first lane of the engine's run
+      const bool last = i + 1 == n || engs[i + 1] != e;
       const bool first_in_copy = cp > 0 && (i == head || copies[i - 1] != cp);
       if (FILL) {
         O.lrec[c[BC_LANES]] = make_int4(x0 + x, d.instr_latency[x0 + x], S.x_ndeps[x0 + x], S.x_dep_begin[x0 + x]);
@@ -884,12 +897,16 @@ struct ProgBuilder {
               c[BC_CHUNKS]++;
               continue;
             }
-            int32_t cnt[33], piece[32];
-            for (int32_t e = 0; e <= 32; ++e) cnt[e] = 0;
-            for (int32_t j = 0; j < n; ++j) ++cnt[IE(bd[b + j]) + 1];
+            int32_t cnt[33], piece[32], peng[32], eng[32];
+            for (int32_t e = 0; e <= ne; ++e) cnt[e] = 0;
+            for (int32_t j = 0; j < n; ++j) ++cnt[(eng[j] = IE(bd[b + j])) + 1];
             for (int32_t e = 0; e < ne; ++e) cnt[e + 1] += cnt[e];
-            for (int32_t j = 0; j < n; ++j) piece[cnt[IE(bd[b + j])]++] = bd[b + j];
-            add_chunk(piece, nullptr, n, 1);
+            for (int32_t j = 0; j < n; ++j) {
+              const int32_t q = cnt[eng[j]]++;
+              piece[q] = bd[b + j];
+              peng[q] = eng[j];
+            }
+            add_chunk(piece, peng, nullptr, n, 1);
           }
           add_item(make_int4(ITEM_SEG, (int32_t)first_chunk, (int32_t)(c[BC_CHUNKS] - first_chunk), -1));
         }
@@ -909,13 +926,14 @@ struct ProgBuilder {
           c[BC_CHUNKS]++;
           continue;
         }
-        int32_t recs[32], copies[32], n = 0;
+        int32_t recs[32], engs[32], copies[32], n = 0, be[16];
+        for (int32_t i = 0; i < L; ++i) be[i] = IE(bd[bp[l] + i]);
         for (int32_t e = 0; e < ne; ++e)
           for (int32_t cp = 0; cp < k; ++cp)
-            for (int32_t i = bp[l]; i < bp[l + 1]; ++i)
-              if (IE(bd[i]) == e) { recs[n] = bd[i]; copies[n++] = cp; }
+            for (int32_t i = 0; i < L; ++i)
+              if (be[i] == e) { recs[n] = bd[bp[l] + i]; engs[n] = e; copies[n++] = cp; }
         if (FILL) O.plan[c[BC_PLAN] - 1].w = (int32_t)c[BC_CHUNKS];
-        add_chunk(recs, copies, n, k);
+        add_chunk(recs, engs, copies, n, k);
       }
     }
   }
