@@ -82,9 +82,46 @@ k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_jo
       }
     }
     const int64_t wb = __shfl_sync(kFull, b, 0), we = __shfl_sync(kFull, e, 31);
+    if (we - wb <= INT32_MAX - 64) {
+      // offsets from the warp's first entry fit 32 bits (a job of 2^31
+      // entries would not): 32-bit shuffles and compares
+      const int32_t rb = (int32_t)(b - wb), re = (int32_t)(e - wb), rend = (int32_t)(we - wb);
+      int32_t* o = out + wb;
+      for (int32_t base = 0; base < rend;) {
+        // the row holding entry `base`: the last lane whose range starts at
+        // or before it (ranges ascend; an empty one shares its start with
+        // the next)
+        const int own = 31 - __clz(__ballot_sync(kFull, rb <= base));
+        const int32_t oe = __shfl_sync(kFull, re, own);
+        if (oe - base >= 32) {
+          const int32_t ov = __shfl_sync(kFull, v, own);
+          const int32_t stop = base + ((oe - base) & ~31);
+          for (int32_t k = base + lane; k < stop; k += 32) o[k] = ov;
+          base = stop;
+          continue;
+        }
+        // the nonempty rows that meet the window, `own` first; an entry's row
+        // is the last of them starting at or before it
+        const unsigned rows = __ballot_sync(kFull, rb < re && rb < base + 32 && re > base);
+        const int32_t k = base + lane;
+        int jl = own;
+        if (__popc(rows) <= 4) {
+          for (unsigned rest = rows & (rows - 1); rest; rest &= rest - 1) {
+            const int L = __ffs(rest) - 1;
+            if (__shfl_sync(kFull, rb, L) <= k) jl = L;
+          }
+        } else {
+          jl = 0;
+          for (int step = 16; step > 0; step >>= 1)
+            if (__shfl_sync(kFull, rb, jl + step) <= k) jl += step;
+        }
+        const int32_t val = __shfl_sync(kFull, v, jl);
+        if (k < rend) o[k] = val;
+        base += 32;
+      }
+      continue;
+    }
     for (int64_t base = wb; base < we;) {
-      // the row holding entry `base`: the last lane whose range starts at or
-      // before it (ranges ascend; an empty one shares its start with the next)
       const int own = 31 - __clz(__ballot_sync(kFull, b <= base));
       const int64_t oe = __shfl_sync(kFull, e, own);
       if (oe - base >= 32) {
@@ -95,12 +132,10 @@ k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_jo
         continue;
       }
       const int64_t k = base + lane;
-      int lo = 0, hi = 31;                        // the last lane whose range starts at or before k
-      for (int step = 0; step < 5; ++step) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (__shfl_sync(kFull, b, mid) <= k) lo = mid; else hi = mid - 1;
-      }
-      const int32_t val = __shfl_sync(kFull, v, lo);
+      int jl = 0;                                 // the last lane whose range starts at or before k
+      for (int step = 16; step > 0; step >>= 1)
+        if (__shfl_sync(kFull, b, jl + step) <= k) jl += step;
+      const int32_t val = __shfl_sync(kFull, v, jl);
       if (k < we) out[k] = val;
       base += 32;
     }

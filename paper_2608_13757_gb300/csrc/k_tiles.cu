@@ -6,19 +6,24 @@ namespace syncgb {
 namespace {
 
 // table[t] = largest i < n with start(i) <= t * tile (start nondecreasing,
-// start(0) = 0), for t < n_tiles; table[n_tiles] = n - 1.
+// start(0) = 0), for t < n_tiles; table[n_tiles] = n - 1.  One thread per
+// item i writes the tiles whose first entry lies in [start(i), start(i+1))
+// (the last item's range is open): the ranges partition the entries, so
+// every tile is written once, by the last item starting at or before it
+// (items with empty ranges write none).
 template <class F>
 __global__ void k_tile_table(int32_t* table, int64_t n_tiles, int64_t n, int64_t tile, F start) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t <= n_tiles; t += stride) {
-    if (n == 0) { table[t] = 0; continue; }
-    if (t == n_tiles) { table[t] = (int32_t)(n - 1); continue; }
-    int64_t lo = 0, hi = n - 1;
-    while (lo < hi) {
-      const int64_t mid = (lo + hi + 1) / 2;
-      if (start(mid) <= t * tile) lo = mid; else hi = mid - 1;
-    }
-    table[t] = (int32_t)lo;
+  const int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i0 == 0) table[n_tiles] = n > 0 ? (int32_t)(n - 1) : 0;
+  if (n == 0) {
+    for (int64_t t = i0; t < n_tiles; t += stride) table[t] = 0;
+    return;
+  }
+  for (int64_t i = i0; i < n; i += stride) {
+    const int64_t s0 = start(i);
+    const int64_t t_end = i + 1 < n ? (start(i + 1) + tile - 1) / tile : n_tiles;   // first tile past the range
+    for (int64_t t = (s0 + tile - 1) / tile; t < t_end && t < n_tiles; ++t) table[t] = (int32_t)i;
   }
 }
 
@@ -40,7 +45,7 @@ int grid_for(int64_t n, int threads, int num_sms) {
 template <class F>
 cudaError_t tile_table(int32_t* table, int64_t n_tiles, int64_t n, int64_t tile, F start, int num_sms,
                        cudaStream_t s) {
-  k_tile_table<<<grid_for(n_tiles + 1, 256, num_sms), 256, 0, s>>>(table, n_tiles, n, tile, start);
+  k_tile_table<<<grid_for((n > n_tiles ? n : n_tiles) + 1, 256, num_sms), 256, 0, s>>>(table, n_tiles, n, tile, start);
   return launched();
 }
 
