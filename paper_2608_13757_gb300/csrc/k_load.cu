@@ -1,6 +1,8 @@
 // Load-time kernels: the derived per-iteration arrays of the threshold
 // kernels, the per-mode semaphore records of the simulators, and (on first
 // per-engine use) the engine-stream positions of producer instances.
+#include <cstdlib>
+
 #include "enc.h"
 
 namespace syncgb {
@@ -44,7 +46,7 @@ k_sem_records(const int4* __restrict__ xsem, int64_t n_instrs, const int4* __res
 __global__ void __launch_bounds__(kThreads)
 k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_job, int64_t n_rows,
          const int32_t* __restrict__ rowptr, const int64_t* __restrict__ path, int32_t* __restrict__ out,
-         int64_t n) {
+         int64_t n, int wide) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kThreads / 32);
   for (int64_t w = (int64_t)blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5); w * 32 < n_rows; w += warps) {
@@ -82,7 +84,7 @@ k_derive(const DeriveJob* __restrict__ jobs, const int32_t* __restrict__ tile_jo
       }
     }
     const int64_t wb = __shfl_sync(kFull, b, 0), we = __shfl_sync(kFull, e, 31);
-    if (we - wb <= INT32_MAX - 64) {
+    if (!wide && we - wb <= INT32_MAX - 64) {
       // offsets from the warp's first entry fit 32 bits (a job of 2^31
       // entries would not): 32-bit shuffles and compares
       const int32_t rb = (int32_t)(b - wb), re = (int32_t)(e - wb), rend = (int32_t)(we - wb);
@@ -211,7 +213,11 @@ cudaError_t launch_derive(const DeriveJob* jobs, const int32_t* tile_job, int64_
   const int64_t want = (n_rows + kThreads - 1) / kThreads;
   const int64_t cap = (int64_t)num_sms * 8;
   const int grid = (int)(want < cap ? want : cap);
-  k_derive<<<grid, kThreads, 0, s>>>(jobs, tile_job, n_rows, rowptr, path, derived, n);
+  // SYNCGB_WIDE_INDEX=1 takes the 64-bit write path everywhere (tests use
+  // it on small batches; otherwise only a warp's range past 2^31 entries does)
+  const char* f = std::getenv("SYNCGB_WIDE_INDEX");
+  const int wide = f && f[0] == '1' ? 1 : 0;
+  k_derive<<<grid, kThreads, 0, s>>>(jobs, tile_job, n_rows, rowptr, path, derived, n, wide);
   return launched();
 }
 

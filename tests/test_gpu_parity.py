@@ -289,6 +289,23 @@ def test_wide_index_kernels(sg, mode, monkeypatch):
     test_checker_planted_errors(sg, mode)
 
 
+@pytest.mark.parametrize("cfg", ["random", "gemm"])
+def test_wide_derive_path(sg, cfg, monkeypatch):
+    """The derive kernel's 64-bit write path (taken where a warp's rows span
+    past 2^31 derived entries) builds the same arrays: loaded with the
+    switch set, the thresholds equal the oracle's and the 32-bit path's."""
+    batch = (workloads.random_trees(4100, 150, workloads.tree_params(engines_hi=5, loops_hi=5, body_hi=6,
+                                                                       trip_hi=9, max_depth=4))
+             if cfg == "random" else workloads.generate("gemm"))
+    _, narrow = gpu_thresholds(sg, sg.sync_load_programs(batch), PERLOOP)
+    monkeypatch.setenv("SYNCGB_WIDE_INDEX", "1")
+    h = sg.sync_load_programs(batch)
+    monkeypatch.delenv("SYNCGB_WIDE_INDEX")
+    _, wide = gpu_thresholds(sg, h, PERLOOP)
+    assert np.array_equal(wide, narrow)
+    assert np.array_equal(wide, oracle.thresholds(batch, PERLOOP))
+
+
 def test_checker_detects_swapped_encoding(sg):
     """Count-mode values read as per-loop values are below the minimum wherever
     N > 1 and c > 0."""
