@@ -86,13 +86,19 @@ struct alignas(16) ProgInfo {
 
 // Program-order sweep tables.  Per loop, a plan: its body cut at child loops
 // into straight-line segments; items [plan_ptr[l], plan_ptr[l+1]):
-//   {ITEM_SEG, first chunk, chunks, multi-iteration chunk or -1}
+//   {ITEM_SEG, first chunk, chunks, w}
 //   {ITEM_LOOP, child loop (global id), child's elidable-trip-register flag, 0}
-// A chunk holds up to 32 datapath records of one segment (all engines), in
-// lanes ordered engine-major (then iteration copy, then body position):
-//   chunk {first lane record, lanes, iteration copies, engine bitmask}
+// with w >= 0 a multi-iteration chunk, w <= -2 (the body's last segment) a
+// chunk of that segment and the next iteration's first (chunk -2 - w), -1
+// neither.  A chunk holds up to 32 datapath records of one segment (all
+// engines), in lanes ordered engine-major (then iteration copy, then body
+// position):
+//   chunk {first lane record, lanes, iteration copies, engines with lanes in
+//          the last copy}
 // A multi-iteration chunk repeats a short innermost segment for `copies`
-// consecutive iterations (barrier-free sweep only).  Per lane:
+// consecutive iterations; a joined chunk holds a body's closing segment
+// (copy 0) and its opening one (copy 1) -- both for the barrier-free sweep
+// only, whose iteration start between the copies is inside the chunk.  Per lane:
 //   lrec {x (global instruction), latency, dependencies, first dependency}
 //   lmeta {engine, copy, first lane of the engine's run, flags}
 //     flags bit 0: first record of its engine in a copy >= 1 (an iteration

@@ -853,7 +853,7 @@ struct ProgBuilder {
     for (int32_t i = 0; i < n; ++i) {
       const int32_t x = recs[i], e = engs[i];
       const int32_t cp = copies ? copies[i] : 0;
-      emask |= (int32_t)(1u << e);
+      if (cp == ncopies - 1) emask |= (int32_t)(1u << e);   // engines in the last copy
       if (i > 0 && engs[i - 1] != e) head = i;         // first lane of the engine's run
       const bool last = i + 1 == n || engs[i + 1] != e;
       const bool first_in_copy = cp > 0 && (i == head || copies[i - 1] != cp);
@@ -935,6 +935,37 @@ struct ProgBuilder {
         if (FILL) O.plan[c[BC_PLAN] - 1].w = (int32_t)c[BC_CHUNKS];
         add_chunk(recs, engs, copies, n, k);
       }
+    }
+    // a body that opens with instructions (A) before its first child loop
+    // and closes with instructions (B) after its last: one more chunk, B
+    // (copy 0) with the next iteration's A (copy 1), for the barrier-free
+    // walk of every iteration but a trip's last; the B item, the body's
+    // last, names it (w = -2 - chunk).  These chunks follow all the
+    // program's others, which the barrier sweep keeps contiguous.
+    const int64_t plan_end = c[BC_PLAN];
+    for (int32_t l = 1; l < nl; ++l) {
+      int32_t fa = bp[l], lb = bp[l + 1], nloops = 0;
+      for (int32_t i = bp[l]; i < bp[l + 1]; ++i) nloops += bd[i] < 0 ? 1 : 0;
+      if (nloops == 0) continue;
+      while (fa < bp[l + 1] && bd[fa] >= 0) ++fa;     // the first child loop
+      while (lb > bp[l] && bd[lb - 1] >= 0) --lb;     // just past the last one
+      const int32_t na = fa - bp[l], nb = bp[l + 1] - lb;
+      if (na < 1 || nb < 1 || na + nb > 32) continue;
+      if constexpr (!FILL) {
+        c[BC_LANES] += na + nb;
+        c[BC_CHUNKS]++;
+        continue;
+      }
+      int32_t recs[32], engs[32], copies[32], n = 0;
+      for (int32_t e = 0; e < ne; ++e) {
+        for (int32_t i = lb; i < bp[l + 1]; ++i)
+          if (IE(bd[i]) == e) { recs[n] = bd[i]; engs[n] = e; copies[n++] = 0; }
+        for (int32_t i = bp[l]; i < fa; ++i)
+          if (IE(bd[i]) == e) { recs[n] = bd[i]; engs[n] = e; copies[n++] = 1; }
+      }
+      const int64_t last_item = (l + 1 < nl ? (int64_t)O.plan_ptr[l0 + l + 1] : plan_end) - 1;
+      O.plan[last_item].w = -2 - (int32_t)c[BC_CHUNKS];
+      add_chunk(recs, engs, copies, n, 2);
     }
   }
 

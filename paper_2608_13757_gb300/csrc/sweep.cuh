@@ -1077,8 +1077,14 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         continue;
       }
       // a straight-line segment
-      if (!BB && it.w >= 0) {                          // several iterations at once
-        const int4 ch = __ldg(a.chunk + it.w);
+      if (!BB && it.w != -1) {
+        // several iterations of a short innermost body at once (w >= 0), or
+        // the body's closing segment joined with the next iteration's
+        // opening one, whose iteration start is inside the chunk (w <= -2):
+        // unless this is the trip's last iteration the walk then goes on in
+        // iteration g+1 past its opening segment
+        const bool joined = it.w <= -2;
+        const int4 ch = __ldg(a.chunk + (joined ? -2 - it.w : it.w));
         const int32_t v = min(ch.z, g_end - g);
         LaneRec Lr;
         load_lane(a, ch, lane, Lr);
@@ -1089,6 +1095,13 @@ __global__ void __launch_bounds__(kWarps * 32, 3) k_sweep(const SweepArgs a) {
         verdict = run_chunk<MODE, BB, TL, FUSED>(a, S, ch, Lr, T, g, v, ctag, lane, sp, lo_c, iter_cost, chk, no_rep,
                                                   no_pred);
         if (verdict) break;
+        if (joined && v == 2) {
+          ++g;
+          if (FUSED && lane == 0) S.lvl[sp].x = g;
+          __syncwarp();
+          item = 1;
+          continue;
+        }
         g += v - 1;
         item = pend - pbeg;                            // continue at the END of iteration g
         continue;
