@@ -944,24 +944,32 @@ struct ProgBuilder {
     // program's others, which the barrier sweep keeps contiguous.
     const int64_t plan_end = c[BC_PLAN];
     for (int32_t l = 1; l < nl; ++l) {
-      int32_t fa = bp[l], lb = bp[l + 1], nloops = 0;
-      for (int32_t i = bp[l]; i < bp[l + 1]; ++i) nloops += bd[i] < 0 ? 1 : 0;
-      if (nloops == 0) continue;
-      while (fa < bp[l + 1] && bd[fa] >= 0) ++fa;     // the first child loop
-      while (lb > bp[l] && bd[lb - 1] >= 0) --lb;     // just past the last one
-      const int32_t na = fa - bp[l], nb = bp[l + 1] - lb;
+      const int32_t b0 = bp[l], b1 = bp[l + 1];
+      int32_t fa = b0;
+      while (fa < b1 && bd[fa] >= 0) ++fa;            // the first child loop
+      if (fa == b1) continue;                         // none
+      int32_t lb = b1;
+      while (bd[lb - 1] >= 0) --lb;                   // just past the last one
+      const int32_t na = fa - b0, nb = b1 - lb;
       if (na < 1 || nb < 1 || na + nb > 32) continue;
       if constexpr (!FILL) {
         c[BC_LANES] += na + nb;
         c[BC_CHUNKS]++;
         continue;
       }
-      int32_t recs[32], engs[32], copies[32], n = 0;
-      for (int32_t e = 0; e < ne; ++e) {
-        for (int32_t i = lb; i < bp[l + 1]; ++i)
-          if (IE(bd[i]) == e) { recs[n] = bd[i]; engs[n] = e; copies[n++] = 0; }
-        for (int32_t i = bp[l]; i < fa; ++i)
-          if (IE(bd[i]) == e) { recs[n] = bd[i]; engs[n] = e; copies[n++] = 1; }
+      // B's records (copy 0), then A's (copy 1), sorted stably by engine
+      int32_t rec[32], eng[32], cnt[33], recs[32], engs[32], copies[32];
+      int32_t n = 0;
+      for (int32_t i = lb; i < b1; ++i) { rec[n] = bd[i]; eng[n++] = IE(bd[i]); }
+      for (int32_t i = b0; i < fa; ++i) { rec[n] = bd[i]; eng[n++] = IE(bd[i]); }
+      for (int32_t e = 0; e <= ne; ++e) cnt[e] = 0;
+      for (int32_t j = 0; j < n; ++j) ++cnt[eng[j] + 1];
+      for (int32_t e = 0; e < ne; ++e) cnt[e + 1] += cnt[e];
+      for (int32_t j = 0; j < n; ++j) {
+        const int32_t q = cnt[eng[j]]++;
+        recs[q] = rec[j];
+        engs[q] = eng[j];
+        copies[q] = j < nb ? 0 : 1;
       }
       const int64_t last_item = (l + 1 < nl ? (int64_t)O.plan_ptr[l0 + l + 1] : plan_end) - 1;
       O.plan[last_item].w = -2 - (int32_t)c[BC_CHUNKS];
